@@ -1,0 +1,325 @@
+"""Pins of the CPU oracle to things other than itself (library routines, brute force, closed
+forms, the paper's worked example, invariants of the method). CPU only."""
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as tF
+
+import oracle
+import synth
+
+F64 = torch.float64
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def rnd(*shape, seed=0, scale=1.0):
+    g = torch.Generator().manual_seed(seed)
+    return torch.randn(*shape, generator=g, dtype=F64) * scale
+
+
+# ---------------------------------------------------------------- elementary operators
+def test_rms_norm_matches_library_and_closed_form():
+    x, g = rnd(7, 33, seed=1), rnd(33, seed=2)
+    ref = tF.rms_norm(x, (33,), weight=g, eps=1e-6)
+    assert torch.allclose(oracle.rms_norm(x, g, 1e-6), ref, rtol=1e-12, atol=1e-12)
+    # [3, 4]: mean square 12.5
+    y = oracle.rms_norm(torch.tensor([3.0, 4.0], dtype=F64), torch.ones(2, dtype=F64), 0.0)
+    assert torch.allclose(y, torch.tensor([3.0, 4.0], dtype=F64) / math.sqrt(12.5))
+
+
+def test_gelu_matches_library_and_identities():
+    x = torch.linspace(-8, 8, 1001, dtype=F64)
+    assert torch.allclose(oracle.gelu(x), tF.gelu(x, approximate="none"), atol=1e-14)
+    assert torch.allclose(oracle.gelu(x) - oracle.gelu(-x), x, atol=1e-12)  # Phi(x)+Phi(-x)=1
+    assert oracle.gelu(torch.tensor(1.0, dtype=F64)).item() == pytest.approx(
+        0.5 * (1 + math.erf(1 / math.sqrt(2))), rel=1e-15)
+
+
+def test_linear_is_x_wt_plus_b():
+    x, w, b = rnd(5, 7, seed=3), rnd(4, 7, seed=4), rnd(4, seed=5)
+    brute = torch.tensor([[sum(x[i, k] * w[j, k] for k in range(7)) + b[j] for j in range(4)]
+                          for i in range(5)], dtype=F64)
+    assert torch.allclose(oracle.linear(x, w, b), brute, atol=1e-12)
+
+
+def test_pixel_unshuffle_matches_library_and_index_formula():
+    C, H, W, p = 3, 6, 8, 2
+    z = rnd(C, H, W, seed=6)
+    tok = oracle.pixel_unshuffle(z, p)                       # [L][C p^2]
+    lib = tF.pixel_unshuffle(z[None], p)[0]                   # [C p^2][H/p][W/p]
+    assert torch.equal(tok, lib.reshape(C * p * p, -1).T)
+    for l in range((H // p) * (W // p)):
+        h, w_ = divmod(l, W // p)
+        for c in range(C):
+            for i in range(p):
+                for j in range(p):
+                    assert tok[l, c * p * p + i * p + j] == z[c, h * p + i, w_ * p + j]
+
+
+def test_pixel_shuffle_matches_library_and_inverts_unshuffle():
+    frames, gh, gw, C, rs = 2, 3, 4, 3, 4
+    L = gh * gw
+    F = rnd(frames * L, C * rs * rs, seed=7)
+    pix = oracle.pixel_shuffle(F, frames, gh, gw, C, rs)
+    assert pix.shape == (C, frames, gh * rs, gw * rs)
+    for tau in range(frames):
+        lib = tF.pixel_shuffle(F[tau * L:(tau + 1) * L].T.reshape(1, C * rs * rs, gh, gw), rs)[0]
+        assert torch.equal(pix[:, tau], lib)
+        # PixelShuffle o PixelUnshuffle = identity on one frame
+        assert torch.equal(oracle.pixel_unshuffle(pix[:, tau], rs), F[tau * L:(tau + 1) * L])
+    # one element by the index formula
+    c, tau, h, i, w_, j = 2, 1, 2, 3, 1, 0
+    assert pix[c, tau, h * rs + i, w_ * rs + j] == F[tau * L + h * gw + w_, c * rs * rs + i * rs + j]
+
+
+# ---------------------------------------------------------------- 3D-RoPE
+def test_rope_bands_at_head_dim_64():
+    assert oracle.rope_bands(64) == [(0, 24), (24, 20), (44, 20)]
+
+
+def test_rope_matches_complex_rotation_and_is_relative():
+    dh, L, base = 64, 9, 10000.0
+    x = rnd(2, L, dh, seed=8)
+    f = torch.arange(L, dtype=F64) * 3
+    y = torch.arange(L, dtype=F64) % 4
+    xx = torch.arange(L, dtype=F64) // 2
+    r = oracle.rope(x, f, y, xx, base)
+    # complex form: (x_2i + i x_2i+1) * exp(i pos theta_i), band by band
+    for (off, d), pos in zip(oracle.rope_bands(dh), (f, y, xx)):
+        th = torch.tensor([base ** (-2.0 * k / d) for k in range(d // 2)], dtype=F64)
+        zc = torch.complex(x[..., off:off + d:2], x[..., off + 1:off + d:2])
+        rot = zc * torch.exp(1j * pos[:, None] * th[None, :])
+        assert torch.allclose(r[..., off:off + d:2], rot.real, atol=1e-12)
+        assert torch.allclose(r[..., off + 1:off + d:2], rot.imag, atol=1e-12)
+    # rotations keep norms; zero position is the identity
+    assert torch.allclose(r.norm(dim=-1), x.norm(dim=-1), atol=1e-12)
+    z0 = torch.zeros(L, dtype=F64)
+    assert torch.allclose(oracle.rope(x, z0, z0, z0, base), x)
+    # <R_a q, R_b k> depends on a - b only, on every axis
+    q, k = rnd(1, 1, dh, seed=9), rnd(1, 1, dh, seed=10)
+    def dot(a, b):
+        pa = [torch.tensor([v], dtype=F64) for v in a]
+        pb = [torch.tensor([v], dtype=F64) for v in b]
+        return (oracle.rope(q, *pa, base) * oracle.rope(k, *pb, base)).sum().item()
+    assert dot((5, 2, 7), (3, 1, 4)) == pytest.approx(dot((12, 4, 9), (10, 3, 6)), abs=1e-10)
+    assert dot((5, 2, 7), (3, 1, 4)) != pytest.approx(dot((5, 2, 7), (4, 1, 4)), abs=1e-6)
+
+
+# ---------------------------------------------------------------- attention
+def test_attention_brute_force_gqa():
+    """Naive softmax attention with explicit exp / sum loops, tiny Lq x Lk, 4 heads on 2
+    KV groups."""
+    N, G, Lq, Lk, dh = 4, 2, 5, 13, 8
+    q, k, v = rnd(N, Lq, dh, seed=11), rnd(G, Lk, dh, seed=12), rnd(G, Lk, dh, seed=13)
+    out = oracle.attention(q, k, v)
+    for n in range(N):
+        g = n // (N // G)
+        for i in range(Lq):
+            s = [sum(q[n, i, d].item() * k[g, j, d].item() for d in range(dh)) / math.sqrt(dh)
+                 for j in range(Lk)]
+            e = [math.exp(x) for x in s]
+            tot = sum(e)
+            for d in range(dh):
+                o = sum(e[j] * v[g, j, d].item() for j in range(Lk)) / tot
+                assert out[n, i, d].item() == pytest.approx(o, rel=1e-10, abs=1e-12)
+
+
+def test_attention_matches_library_sdpa_and_gqa_special_cases():
+    N, G, Lq, Lk, dh = 6, 3, 17, 40, 16
+    q, k, v = rnd(N, Lq, dh, seed=14), rnd(G, Lk, dh, seed=15), rnd(G, Lk, dh, seed=16)
+    ref = tF.scaled_dot_product_attention(q, k.repeat_interleave(N // G, 0),
+                                          v.repeat_interleave(N // G, 0))
+    assert torch.allclose(oracle.attention(q, k, v), ref, atol=1e-12)
+    # G = N is MHA: duplicating each KV head N/G times and using G' = N changes nothing
+    kd, vd = k.repeat_interleave(N // G, 0), v.repeat_interleave(N // G, 0)
+    assert torch.allclose(oracle.attention(q, kd, vd), oracle.attention(q, k, v), atol=1e-12)
+    # G = 1 is MQA: every head reads the single group
+    o1 = oracle.attention(q, k[:1], v[:1])
+    for n in range(N):
+        assert torch.allclose(o1[n], oracle.attention(q[n:n + 1], k[:1], v[:1])[0], atol=1e-12)
+    # row blocking does not change the result
+    assert torch.allclose(oracle.attention(q, k, v, rows=3), oracle.attention(q, k, v), atol=1e-13)
+    # a mask equals dropping the masked keys
+    allowed = torch.zeros(Lq, Lk, dtype=torch.bool)
+    allowed[:, 10:30] = True
+    assert torch.allclose(oracle.attention(q, k, v, allowed),
+                          oracle.attention(q, k[:, 10:30], v[:, 10:30]), atol=1e-12)
+
+
+# ---------------------------------------------------------------- pixel quantisation
+def test_quantize_u8_special_values():
+    x = np.array([-1.0, 1.0, 0.0, -2.0, 3.0, np.nan, np.inf, -np.inf,
+                  -1.0 + 1 / 255, 0.5 / 127.5 - 1.0, 1.5 / 127.5 - 1.0], dtype=np.float32)
+    q = oracle.quantize_u8(x)
+    # (x+1)*127.5: -1 -> 0, 1 -> 255, 0 -> 127.5 -> 128 (ties to even), NaN -> 0
+    assert list(q[:8]) == [0, 255, 128, 0, 255, 0, 255, 0]
+    assert q[8] == 0 or q[8] == 1
+    # exact .5 ties go to even codes (the fp32 products land on 0.5 / 1.5 or next to them)
+    a = (np.float32(x[9]) + np.float32(1)).astype(np.float32) * np.float32(127.5)
+    assert q[9] == np.rint(np.float32(a))
+    every = np.arange(256, dtype=np.float32) / np.float32(127.5) - np.float32(1)
+    assert np.all(np.abs(oracle.quantize_u8(every).astype(int) - np.arange(256)) <= 1)
+
+
+# ---------------------------------------------------------------- streaming decode invariants
+def _setup(name, **kw):
+    cfg = synth.PRESETS[name].replace(**kw)
+    return cfg, synth.make_weights(cfg), synth.make_latents(cfg)
+
+
+def test_fig2_visibility_golden():
+    """Fig. 2(a): at W=2, z0 alone, z1 sees [z0, z1], z2 sees [z1, z2]."""
+    rows = {}
+    with open(os.path.join(GOLDEN, "fig2_visibility.txt")) as fh:
+        for line in fh:
+            line = line.split("#")[0].strip()
+            if line.startswith("window"):
+                W = int(line.split()[1])
+            elif line:
+                a, b = line.split(":")
+                rows[int(a)] = [int(x) for x in b.split()]
+    m = oracle.chunk_mask(torch.arange(3), W)
+    for i, seen in rows.items():
+        assert [j for j in range(3) if m[i, j]] == seen
+    # the streaming cache holds exactly those chunks after each step
+    cfg, w, z = _setup("tiny", window=W, chunks=3, n_blocks=1)
+    dec = oracle.StreamingDecoder(cfg, w)
+    keys_of_chunk = []
+    for t in range(3):
+        dec.decode_chunk(z[t])
+        K = dec.kB[0]
+        keys_of_chunk.append(K[:, -cfg.tokens:].clone())
+        want = rows[t]
+        assert K.shape[1] == len(want) * cfg.tokens
+        for slot, c in enumerate(want):
+            assert torch.equal(K[:, slot * cfg.tokens:(slot + 1) * cfg.tokens], keys_of_chunk[c])
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8"])
+def test_streaming_equals_masked_full_sequence(name):
+    """Sec. 3.3: sequential decoding with the rolling cache equals one pass under the block
+    sliding-window mask (the paper's training-inference consistency)."""
+    cfg, w, z = _setup(name)
+    a = oracle.decode_stream(cfg, w, z)
+    b = oracle.decode_full_masked(cfg, w, z)
+    for x, y in zip(a, b):
+        assert torch.allclose(x, y, atol=1e-12)
+
+
+def test_causality_later_chunks_do_not_matter():
+    cfg, w, z = _setup("small")
+    base = oracle.decode_stream(cfg, w, z)
+    z2 = z.copy()
+    z2[3:] = synth.make_latents(cfg, seed=77)[3:]
+    pert = oracle.decode_stream(cfg, w, z2)
+    for t in range(3):
+        assert torch.equal(base[t], pert[t])
+    assert not torch.allclose(base[3], pert[3])
+    # same for the masked full-sequence pass
+    fb = oracle.decode_full_masked(cfg, w, z2)
+    for t in range(3):
+        assert torch.allclose(fb[t], base[t], atol=1e-12)
+
+
+def test_eviction_one_block():
+    """One block, no refinement: chunk t's output ignores chunks <= t - W (evicted, Fig. 2a);
+    with two blocks the receptive field grows and it does change."""
+    W = 2
+    cfg, w, z = _setup("tiny", window=W, chunks=4, n_blocks=1)
+    z2 = z.copy()
+    z2[0] = -z[0] + 0.5
+    a, b = oracle.decode_stream(cfg, w, z), oracle.decode_stream(cfg, w, z2)
+    assert torch.allclose(a[2], b[2], atol=1e-13) and torch.allclose(a[3], b[3], atol=1e-13)
+    assert not torch.allclose(a[1], b[1])
+    cfg2 = cfg.replace(n_blocks=2)
+    w2 = synth.make_weights(cfg2)
+    a, b = oracle.decode_stream(cfg2, w2, z), oracle.decode_stream(cfg2, w2, z2)
+    assert not torch.allclose(a[2], b[2])       # reaches chunk 0 through block 1's cache
+    assert torch.allclose(a[3], b[3], atol=1e-13)
+
+
+@pytest.mark.parametrize("name", ["tiny_rt", "small"])
+def test_window_relative_rope_equals_absolute(name):
+    """Sec. 4.3: RoPE positions relative to the window give the same scores."""
+    cfg, w, z = _setup(name)
+    a = oracle.decode_stream(cfg, w, z, rope_mode="abs")
+    b = oracle.decode_stream(cfg, w, z, rope_mode="window")
+    for x, y in zip(a, b):
+        assert torch.allclose(x, y, atol=1e-10)
+
+
+def test_identity_blocks_reduce_to_closed_form():
+    """With zero out-projections and zero second MLP layers every block is the identity, and
+    the decoder reduces to head(upsample(RMS(embed(z)))) written with plain numpy."""
+    cfg, w, z = _setup("small", chunks=2)
+    for k in list(w):
+        if k.endswith(("out.w", "out.b", "mlp2.w", "mlp2.b")):
+            w[k] = np.zeros_like(w[k])
+    got = oracle.decode_stream(cfg, w, z)
+    L, D, rt, rs, p = cfg.tokens, cfg.hidden, cfg.r_t, cfg.r_s, cfg.patch
+    ww = {k: v.astype(np.float64) for k, v in w.items()}
+    erf = np.vectorize(math.erf)
+    for t in range(2):
+        x0 = np.zeros((L, cfg.c_in))
+        for c in range(cfg.latent_channels):
+            for yy in range(cfg.latent_h):
+                for xx in range(cfg.latent_w):
+                    l = (yy // p) * cfg.grid_w + xx // p
+                    x0[l, c * p * p + (yy % p) * p + xx % p] = z[t, c, yy, xx]
+        h = x0 @ ww["embed.w"].T + ww["embed.b"]
+        def rms(a, g):
+            return a / np.sqrt((a ** 2).mean(-1, keepdims=True) + cfg.norm_eps) * g
+        e = rms(h, ww["normf.g"]) @ ww["tup.w"].T + ww["tup.b"]
+        hf = np.concatenate([e[:, tau * D:(tau + 1) * D] for tau in range(rt)])
+        y = rms(hf, ww["normh.g"])
+        a1 = y @ ww["head1.w"].T + ww["head1.b"]
+        F = (0.5 * a1 * (1 + erf(a1 / math.sqrt(2)))) @ ww["head2.w"].T + ww["head2.b"]
+        pix = np.zeros((3, rt, cfg.out_h, cfg.out_w))
+        for tau in range(rt):
+            for l in range(L):
+                hh, w_ = divmod(l, cfg.grid_w)
+                blk = F[tau * L + l].reshape(3, rs, rs)
+                pix[:, tau, hh * rs:(hh + 1) * rs, w_ * rs:(w_ + 1) * rs] = blk
+        assert np.allclose(got[t].numpy(), np.clip(pix, -1, 1), atol=1e-12)
+
+
+def test_output_shapes_follow_compression_factors():
+    """8x spatial per latent cell, r_t frames per chunk: 480p -> 480x832, 720p -> 720x1280."""
+    for name, hw in [("480p", (480, 832)), ("720p", (720, 1280)), ("720p_wide", (720, 1280))]:
+        cfg = synth.PRESETS[name]
+        assert (cfg.out_h, cfg.out_w) == hw and cfg.r_s == 16 and cfg.head_out == 768
+        F = torch.zeros(cfg.r_t * cfg.tokens, cfg.head_out, dtype=F64)
+        pix = oracle.pixel_shuffle(F, cfg.r_t, cfg.grid_h, cfg.grid_w, 3, cfg.r_s)
+        assert tuple(pix.shape) == (3, 4) + hw
+    assert synth.PRESETS["480p"].tokens == 1560 and synth.PRESETS["720p"].tokens == 3600
+    cfg, w, z = _setup("tiny")
+    assert tuple(oracle.decode_stream(cfg, w, z)[0].shape) == (3, 1, 64, 64)
+
+
+def test_kv_cache_size_formula():
+    """Eq. kv_cache: G x (W L) x D_h per layer for K and V; refinement r_t W L (Sec. 3.3)."""
+    cfg = synth.PRESETS["480p"]
+    e = oracle.kv_cache_elems(cfg)
+    assert e["backbone_per_layer"] == 2 * 4 * 4 * 1560 * 64
+    assert e["refine_per_layer"] == 4 * e["backbone_per_layer"]
+    cfg, w, z = _setup("small")
+    dec = oracle.StreamingDecoder(cfg, w)
+    for t in range(cfg.chunks):
+        dec.decode_chunk(z[t])
+    assert dec.kB[0].numel() + dec.vB[0].numel() == oracle.kv_cache_elems(cfg)["backbone_per_layer"]
+    assert dec.kR[0].numel() + dec.vR[0].numel() == oracle.kv_cache_elems(cfg)["refine_per_layer"]
+
+
+def test_weights_and_latents_are_seeded_and_bf16_exact():
+    cfg = synth.PRESETS["tiny"]
+    a, b = synth.make_weights(cfg), synth.make_weights(cfg)
+    for k in a:
+        assert np.array_equal(a[k], b[k])
+        bf = torch.from_numpy(a[k]).to(torch.bfloat16).float().numpy()
+        assert np.array_equal(bf, a[k])       # exactly representable in bf16
+    z = synth.make_latents(synth.PRESETS["720p_wide"].replace(latent_h=4, latent_w=4), chunks=400)
+    c = np.corrcoef(z[:-1].ravel(), z[1:].ravel())[0, 1]
+    assert abs(c - 0.9) < 0.02                  # AR(1), rho = 0.9
