@@ -1,0 +1,166 @@
+/*
+ * flashdec.h - C ABI of the GB300 (sm_103a) FlashDecoder streaming decoder.
+ *
+ * The decoder turns one latent frame ("chunk") at a time into r_t pixel frames, keeping a
+ * rolling key/value cache of the last W_frm chunks per attention layer (Sec. 3.3 "Streaming
+ * with Rolling KV Cache", Eq. kv_cache, Algorithm 1). Per chunk t it runs:
+ *   PixelUnshuffle(p) + Linear_{C' p^2 -> D}              (Eq. projection, Sec. 4.3)
+ *   n_blocks x [RMSNorm, QKV + KV-norm + 3D-RoPE, attention over the cache, out-proj +
+ *               residual, RMSNorm, MLP 4x (GELU) + residual]          (Sec. 3.2)
+ *   RMSNorm, Linear_{D -> r_t D}, channel -> time reshape    (Eq. temporal_upsample)
+ *   n_refine x the same block on r_t L tokens, window r_t W  (Sec. 3.4 "Step 2")
+ *   RMSNorm, Linear_{D->D} + GELU, Linear_{D -> C r_s^2}, PixelShuffle(r_s), clamp
+ *                                                             (Sec. 3.4 "Step 3")
+ * Every step runs in the library's own CUDA kernels on the caller's stream.
+ *
+ * Conventions
+ *   - All calls return fd_status; none throws, exits or traps.
+ *   - Device pointers are CUDA device addresses on the current device; a stream argument is a
+ *     cudaStream_t passed as void* (NULL = the legacy default stream).
+ *   - A handle is not thread-safe; distinct handles may be used from distinct threads.
+ *   - Asynchronous device errors (a kernel's bounded wait giving up, a CUDA launch error)
+ *     put the handle in the FD_ERR_STATE state: later decode calls fail until fd_reset.
+ */
+#ifndef FLASHDEC_H
+#define FLASHDEC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  FD_OK = 0,
+  FD_ERR_INVALID_ARG = 1,     /* null / misaligned pointer, wrong size, bad enum          */
+  FD_ERR_CONFIG = 2,          /* configuration outside what the kernels support           */
+  FD_ERR_OOM = 3,             /* device allocation failed                                 */
+  FD_ERR_CUDA = 4,            /* a CUDA runtime call or kernel launch failed              */
+  FD_ERR_STATE = 5,           /* handle is in an error state: fd_reset it                 */
+  FD_ERR_DEVICE_TIMEOUT = 6,  /* a kernel's bounded wait gave up (see fd_sync_status)     */
+  FD_ERR_UNSUPPORTED = 7      /* device is not sm_103 / sm_100 class                      */
+} fd_status;
+
+typedef enum { FD_DTYPE_F32 = 0, FD_DTYPE_BF16 = 1, FD_DTYPE_U8 = 2 } fd_dtype;
+
+/*
+ * Decoder shape (names follow the paper: Sec. 3, Algorithm 1, Table "Model scaling").
+ * Supported: hidden / heads == 64 (D_h), heads % kv_groups == 0, hidden % 128 == 0,
+ * latent_h and latent_w divisible by patch, window >= 1, r_t >= 1, n_blocks >= 1,
+ * out_channels * (vae_spatial * patch)^2 % 64 == 0.
+ */
+typedef struct {
+  int32_t latent_channels; /* C'                                                  */
+  int32_t latent_h;        /* H' (latent rows per frame)                          */
+  int32_t latent_w;        /* W'                                                  */
+  int32_t patch;           /* PixelUnshuffle factor p on the latent (Sec. 4.3)    */
+  int32_t hidden;          /* D                                                   */
+  int32_t heads;           /* N query heads                                       */
+  int32_t kv_groups;       /* G key/value groups (GQA)                            */
+  int32_t mlp_ratio;       /* MLP hidden = mlp_ratio * D                          */
+  int32_t n_blocks;        /* backbone blocks                                     */
+  int32_t n_refine;        /* temporal-refinement blocks                          */
+  int32_t window;          /* W_frm, cached chunks including the current one      */
+  int32_t r_t;             /* temporal upsampling factor (frames per chunk)       */
+  int32_t vae_spatial;     /* pixels per latent cell side (8 for Wan2.1)          */
+  int32_t out_channels;    /* C (3)                                               */
+  int32_t out_dtype;       /* FD_DTYPE_F32 or FD_DTYPE_U8                         */
+  int32_t reserved;        /* must be 0                                           */
+  float norm_eps;          /* RMSNorm epsilon (1e-6)                              */
+  float rope_base;         /* RoPE base (10000)                                   */
+} fd_config;
+
+typedef struct fd_weights_s* fd_weights;
+typedef struct fd_handle_s* fd_handle;
+
+/* ------------------------------------------------------------------ sizes */
+
+/* Number of elements of the weight blob for cfg (0 if cfg is invalid). Blob order, each
+ * linear weight stored [out][in] row-major (nn.Linear layout):
+ *   embed.w [D][C' p^2], embed.b [D]
+ *   per backbone block b = 0 .. n_blocks-1:
+ *     norm1.g [D], qkv.w [(N+2G)*64][D], qkv.b [(N+2G)*64], knorm.g [64], vnorm.g [64],
+ *     out.w [D][N*64], out.b [D], norm2.g [D], mlp1.w [M*D][D], mlp1.b [M*D],
+ *     mlp2.w [D][M*D], mlp2.b [D]
+ *     (qkv rows: N query heads, then G key groups, then G value groups, 64 rows each)
+ *   normf.g [D], tup.w [r_t*D][D], tup.b [r_t*D]
+ *   per refinement block: the same twelve tensors
+ *   normh.g [D], head1.w [D][D], head1.b [D], head2.w [C r_s^2][D], head2.b [C r_s^2]
+ * with r_s = vae_spatial * patch and M = mlp_ratio. */
+size_t fd_weights_blob_elems(const fd_config* cfg);
+
+/* Bytes of one latent chunk: C' * H' * W' fp32, layout [C'][H'][W'] row-major. */
+size_t fd_latent_bytes(const fd_config* cfg);
+
+/* Bytes of one chunk of pixels: C * r_t * (H' 8) * (W' 8) elements of out_dtype, layout
+ * [C][r_t][H][W] row-major (planar channels, then frames; Sec. 3.4 Step 3). */
+size_t fd_pixels_bytes(const fd_config* cfg);
+
+/* Device bytes a handle allocates (rings, scratch), excluding the shared weights. */
+size_t fd_handle_device_bytes(const fd_config* cfg);
+
+/* ------------------------------------------------------------------ weights */
+
+/* Copy a host weight blob (order above) to the device, converting to bf16 (round to nearest
+ * even) for the linear weights and keeping biases and gains in fp32.
+ * blob_dtype: FD_DTYPE_F32 or FD_DTYPE_BF16. blob_bytes must equal
+ * fd_weights_blob_elems(cfg) * sizeof(element). Synchronous. The caller keeps ownership of
+ * host_blob; the library owns the device copy until fd_weights_destroy. A weights object may
+ * be shared by several handles (it must outlive them). */
+fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t blob_bytes,
+                            int blob_dtype, fd_weights* out);
+fd_status fd_weights_destroy(fd_weights w);
+
+/* ------------------------------------------------------------------ streams */
+
+/* Create a decoder stream state for cfg (must equal the weights' cfg): KV rings for every
+ * layer (backbone G x W L x 64 per K and V; refinement G x r_t W L x 64), activation scratch
+ * and a device chunk counter t = 0. Zero-fills the rings. Synchronous. */
+fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out);
+
+/* Decode chunk t (Algorithm 1, one loop iteration) and advance t.
+ * latent_dev: device fp32 [C'][H'][W'] (fd_latent_bytes), 16-byte aligned.
+ * pixels_dev: device buffer of fd_pixels_bytes, 16-byte aligned, written with clamped
+ *             pixels in [-1, 1] (fp32) or their uint8 codes
+ *             q = round_half_even((clamp(x,-1,1) + 1) * 127.5) (uint8; NaN -> 0).
+ * Both are used stream-ordered on `stream`; the call returns after enqueueing (no host
+ * synchronisation). Attention at chunk t covers the min(t+1, W) most recent chunks. */
+fd_status fd_decode_chunk(fd_handle h, const float* latent_dev, void* pixels_dev, void* stream);
+
+/* Decode one chunk for each of n handles (independent streams sharing one weights object),
+ * in order, on one CUDA stream. */
+fd_status fd_decode_chunks(fd_handle* hs, int n, const float* const* latents_dev,
+                           void* const* pixels_dev, void* stream);
+
+/* Restart the stream: t = 0 and the caches logically empty (their memory is not cleared;
+ * stale entries are never read because attention at chunk t reads only chunks <= t).
+ * Clears the error state. Synchronous with respect to the handle's previous work. */
+fd_status fd_reset(fd_handle h);
+
+/* Free everything the handle owns (after synchronising its last stream). */
+fd_status fd_destroy(fd_handle h);
+
+/* Host-side chunk counter (chunks decoded since create / reset). */
+int64_t fd_chunk_index(fd_handle h);
+
+/* Synchronise with the handle's last stream and read its device status word:
+ * FD_OK, FD_ERR_DEVICE_TIMEOUT (a bounded wait gave up) or FD_ERR_CUDA. */
+fd_status fd_sync_status(fd_handle h);
+
+/* Static description of a status code. */
+const char* fd_status_str(fd_status s);
+
+/* Copy layer `layer` of the backbone (which = 0) or refinement (which = 1) ring into host
+ * memory: K as [G][W * rows][64] bf16 bits, then V as [G][W * rows][64] bf16 bits (rows =
+ * L backbone, r_t L refinement; row slot*rows + r holds token r of the chunk in ring slot
+ * `slot` = chunk index mod W). dst_bytes must be >= 2 * G * W * rows * 64 * 2. Synchronous.
+ * For tests of the cache indexing. */
+fd_status fd_debug_read_ring(fd_handle h, int which, int layer, void* dst_host,
+                             size_t dst_bytes);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FLASHDEC_H */

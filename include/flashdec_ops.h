@@ -1,0 +1,85 @@
+/*
+ * flashdec_ops.h - kernel-level entry points of the FlashDecoder library.
+ *
+ * Each call enqueues one of the decoder's kernels on caller-owned device buffers and returns
+ * after enqueueing (stream-ordered, no host synchronisation). They exist so each step of the
+ * decode path (Algorithm 1) can be checked and timed on its own; fd_decode_chunk runs the
+ * same kernels. All pointers are device pointers unless stated; `stream` is a cudaStream_t
+ * as void*. `err_dev` is a device int32 the kernel ORs error bits into when one of its
+ * bounded waits gives up (1 TMA load, 2 MMA commit, 4 accumulator release, 8 shared-memory
+ * alignment); the caller zeroes it and reads it after synchronising. Argument errors are
+ * reported synchronously as FD_ERR_INVALID_ARG; nothing is launched then.
+ */
+#ifndef FLASHDEC_OPS_H
+#define FLASHDEC_OPS_H
+
+#include "flashdec.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  FD_EPI_F32 = 0,   /* out fp32 [M][N]  = A W^T + b                                   */
+  FD_EPI_RESID = 1, /* out fp32 [M][N] += A W^T + b          (residual, Sec. 3.2)      */
+  FD_EPI_GELU = 2,  /* out bf16 [M][N]  = GELU_erf(A W^T + b) (MLP, R7; head, Sec. 3.4) */
+  FD_EPI_TUP = 3    /* out fp32 [(N / tup_hidden) M][tup_hidden]: column tau*D + d of row
+                       l goes to row tau*M + l, column d (Eq. temporal_upsample)          */
+} fd_epilogue;
+
+/* Linear layer on the tensor cores (tcgen05, bf16 in, fp32 accumulate).
+ * A bf16 [M][K] row-major; W bf16 [N][K] row-major (nn.Linear); bias fp32 [N].
+ * Requires N % 32 == 0, K % 8 == 0, 16-byte aligned A / W / out. bn = output tile width
+ * (64, 128 or 256; 0 = library choice). */
+fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const void* W,
+                       const float* bias, void* out, int tup_hidden, int bn, int* err_dev,
+                       void* stream);
+
+/* Fused QKV projection of one attention block (Sec. 3.2, Sec. 3.3 step (2)):
+ *   [Q | K | V] = A Wqkv^T + b   (Wqkv rows: heads*64 query, groups*64 key, groups*64 value)
+ *   K, V <- RMSNorm over the 64 head dims with gains knorm_g / vnorm_g (KV-norm)
+ *   Q, K <- 3D-RoPE at temporal index t*frames_per_chunk + row / tokens, row and column of
+ *           token (row % tokens) in a grid of width grid_w (rope_base; bands 24/20/20 dims)
+ *   q_out bf16 [M][heads*64];  K -> k_ring bf16 [groups][ring_pitch][64] rows
+ *   (t mod window)*M + row;  V -> vt_ring bf16 [groups][64][ring_pitch] (transposed), same
+ *   key index.  M = frames_per_chunk * tokens; ring_pitch % 128 == 0, >= window * M. */
+fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* bqkv,
+                    const float* knorm_g, const float* vnorm_g, int heads, int groups,
+                    int tokens, int grid_w, int frames_per_chunk, int window, int t, float eps,
+                    float rope_base, void* q_out, void* k_ring, void* vt_ring, int ring_pitch,
+                    int bn, int* err_dev, void* stream);
+
+/* Attention of Lq queries over the first n_keys keys of a ring (Sec. 3.3, Eq. kv_cache):
+ *   out[r][n*64 + d] = sum_j softmax_j(q_n . k_j / 8) v_j[d],  KV group g = n / (heads/groups)
+ * q bf16 [Lq][heads*64]; k_ring bf16 [groups][ring_pitch][64]; vt_ring bf16
+ * [groups][64][ring_pitch]; out bf16 [Lq][heads*64]. 1 <= n_keys <= ring_pitch,
+ * ring_pitch % 128 == 0. Ring entries past n_keys must hold finite values. */
+fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const void* k_ring,
+                          const void* vt_ring, int ring_pitch, int n_keys, void* out,
+                          int* err_dev, void* stream);
+
+/* Rolling-cache append (Algorithm 1, cache update): fp32 k, v [groups][rows][64] rounded to
+ * bf16 (nearest even) into ring slot s = t mod window: k_ring[g][s*rows + r][d] and
+ * vt_ring[g][d][s*rows + r]. The oldest chunk's slot is overwritten (eviction). */
+fd_status fd_op_kv_append(const float* k, const float* v, int groups, int rows, int window,
+                          int t, int ring_pitch, void* k_ring, void* vt_ring, void* stream);
+
+/* u bf16 [M][D] = h / sqrt(mean(h^2) + eps) * g   (RMSNorm, Sec. 3.2); D % 128 == 0. */
+fd_status fd_op_rmsnorm(const float* h, const float* g, int M, int D, float eps, void* u,
+                        void* stream);
+
+/* PixelUnshuffle(p) of a latent frame z fp32 [C][H][W] into tokens x0 bf16 [(H/p)(W/p)][C p^2]
+ * (Sec. 4.3; raster token order of Eq. projection). */
+fd_status fd_op_unshuffle(const float* z, int C, int H, int W, int p, void* x0, void* stream);
+
+/* Pixel head (Sec. 3.4 Step 3): F fp32 [frames * gh * gw][C rs^2] -> pixels
+ * [C][frames][gh rs][gw rs], pix = clamp(F[tau*L + y/rs*gw + x/rs][c rs^2 + (y%rs) rs + x%rs],
+ * -1, 1), as fp32 or uint8 code round_half_even((pix + 1) * 127.5) (NaN -> 0). rs % 4 == 0. */
+fd_status fd_op_pixel_head(const float* F, int frames, int grid_h, int grid_w, int channels,
+                           int rs, int out_dtype, void* pixels, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FLASHDEC_OPS_H */

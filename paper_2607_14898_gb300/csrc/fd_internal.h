@@ -1,0 +1,89 @@
+// Internal launch interface between the host runtime (flashdec.cu) and the kernels
+// (fd_gemm.cu, fd_attn.cu, fd_small.cu). Not part of the public C ABI.
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+namespace fd {
+
+constexpr int kHeadDim = 64;     // D_h: every model size of the paper uses D / N = 64
+constexpr int kRopePairs = 32;   // D_h / 2 rotation pairs: 12 temporal, 10 row, 10 column
+constexpr int kBM = 128;         // GEMM / attention tile rows (one TMEM lane per row)
+constexpr int kBK = 64;          // K elements per stage (one 128-byte swizzle atom)
+
+enum EpiKind : int {
+  EPI_F32 = 0,    // out_f32[r][c] = acc + bias
+  EPI_RESID = 1,  // out_f32[r][c] += acc + bias (residual stream, in place)
+  EPI_GELU = 2,   // out_bf16[r][c] = bf16(GELU(acc + bias))
+  EPI_TUP = 3,    // temporal upsampling: column tau*D + d of row l -> out_f32[tau*L + l][d]
+  EPI_QKV = 4,    // bias, KV-norm, 3D-RoPE; Q to q_out, K/V into the cache ring slot
+};
+
+// Rotary / cache parameters of the fused QKV epilogue.
+struct QkvEpi {
+  int heads, groups;
+  const float* knorm_g;      // [64] KV-norm gain for K
+  const float* vnorm_g;      // [64] KV-norm gain for V
+  __nv_bfloat16* q_out;      // [M][heads * 64]
+  __nv_bfloat16* k_ring;     // [groups][ring_pitch][64]
+  __nv_bfloat16* vt_ring;    // [groups][64][ring_pitch]   (V stored transposed)
+  int ring_pitch;            // key rows per group (>= window * rows_per_chunk, multiple of 128)
+  int tokens;                // L_frm
+  int grid_w;                // token-grid width W'/p
+  int frames_per_chunk;      // 1 (backbone) or r_t (refinement)
+  int window;                // W_frm in chunks
+  const int* step_dev;       // chunk index t on the device, or null to use step_host
+  int step_host;
+  float eps;
+  int band_t, band_s;        // pairs in the temporal band and in each spatial band
+  double inv_freq[kRopePairs];  // base^(-2i/d_band), temporal pairs first, then row, column
+};
+
+struct GemmParams {
+  int M, N, K;
+  int epi;
+  const float* bias;         // [N]
+  float* out_f32;            // EPI_F32 / EPI_RESID / EPI_TUP
+  int ld_out;                // row pitch of out_f32 / out_bf16 (elements)
+  __nv_bfloat16* out_bf16;   // EPI_GELU
+  int tup_tokens, tup_hidden;
+  QkvEpi qkv;
+  int* err;
+};
+
+struct AttnParams {
+  int Lq;                    // query rows
+  int heads, groups;
+  int ring_pitch;            // key rows per group in the ring
+  int rows_per_chunk;        // keys appended per chunk
+  int window;
+  const int* step_dev;       // t on the device (keys = min(t+1, W) * rows_per_chunk) or null
+  int n_keys_host;           // used when step_dev is null
+  __nv_bfloat16* out;        // [Lq][heads * 64]
+  int ld_out;
+  float scale_log2;          // log2(e) / sqrt(D_h)
+  int* err;
+};
+
+// launch wrappers; return cudaGetLastError() of the launch
+cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p,
+                        int bn, int num_sms, cudaStream_t s);
+cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmK,
+                             const CUtensorMap& tmVt, const AttnParams& p, cudaStream_t s);
+cudaError_t launch_unshuffle(const float* z, int C, int H, int W, int p, __nv_bfloat16* x0,
+                             cudaStream_t s);
+cudaError_t launch_rmsnorm(const float* h, const float* g, int M, int D, float eps,
+                           __nv_bfloat16* u, cudaStream_t s);
+cudaError_t launch_pixel_head(const float* F, int frames, int gh, int gw, int C, int rs,
+                              int out_u8, void* pix, cudaStream_t s);
+cudaError_t launch_kv_append(const float* k, const float* v, int groups, int rows, int slot,
+                             int ring_pitch, __nv_bfloat16* k_ring, __nv_bfloat16* vt_ring,
+                             cudaStream_t s);
+cudaError_t launch_advance(int* step_dev, cudaStream_t s);
+
+// GEMM tile widths compiled in
+inline bool gemm_bn_supported(int bn) { return bn == 64 || bn == 128 || bn == 256; }
+
+}  // namespace fd

@@ -1,0 +1,162 @@
+// Bandwidth-bound kernels of the decode path.
+//   unshuffle    latent [C'][H'][W'] fp32 -> tokens [L][C' p^2] bf16 (PixelUnshuffle, Sec. 4.3;
+//                raster token order of Eq. projection)
+//   rmsnorm      h fp32 [M][D] -> bf16(h / sqrt(mean(h^2) + eps) * g)  (pre-norm, Sec. 3.2)
+//   pixel_head   F fp32 [frames*L][C r_s^2] -> PixelShuffle(r_s) + clamp to [-1, 1], fp32 or
+//                uint8 (Sec. 3.4 "Step 3"); one thread per 4 consecutive output pixels
+//   kv_append    fp32 K, V of one chunk -> bf16 ring slot (K rows, V transposed) (Sec. 3.3)
+//   advance      chunk counter t += 1 (device-resident, so a captured graph can be replayed)
+#include "fd_internal.h"
+#include "fd_ptx.cuh"
+
+namespace fd {
+
+__global__ void unshuffle_kernel(const float* __restrict__ z, int C, int H, int W, int p,
+                                 __nv_bfloat16* __restrict__ x0) {
+  const int gw = W / p;
+  const int cin = C * p * p;
+  const int total = (H / p) * gw * cin;
+  for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += gridDim.x * blockDim.x) {
+    const int l = idx / cin, ch = idx - l * cin;
+    const int c = ch / (p * p), ij = ch - c * p * p;
+    const int i = ij / p, j = ij - i * p;
+    const int h = l / gw, w = l - h * gw;
+    x0[idx] = __float2bfloat16_rn(z[(static_cast<size_t>(c) * H + h * p + i) * W + w * p + j]);
+  }
+}
+
+// one warp per row; D % 128 == 0
+__global__ void rmsnorm_kernel(const float* __restrict__ h, const float* __restrict__ g, int M,
+                               int D, float eps, __nv_bfloat16* __restrict__ u) {
+  const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= M) return;
+  const float4* hr = reinterpret_cast<const float4*>(h + static_cast<size_t>(row) * D);
+  const float4* g4 = reinterpret_cast<const float4*>(g);
+  float ss = 0.f;
+  for (int c = lane; c < D / 4; c += 32) {
+    const float4 v = hr[c];
+    ss = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, ss))));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  const float r = rsqrtf(ss / static_cast<float>(D) + eps);
+  uint2* ur = reinterpret_cast<uint2*>(u + static_cast<size_t>(row) * D);
+  for (int c = lane; c < D / 4; c += 32) {
+    const float4 v = hr[c];
+    const float4 gg = g4[c];
+    ur[c] = make_uint2(pack_bf16x2(v.x * r * gg.x, v.y * r * gg.y),
+                       pack_bf16x2(v.z * r * gg.z, v.w * r * gg.w));
+  }
+}
+
+__device__ __forceinline__ uint32_t quant_u8(float x) {
+  // NaN -> -1 through fmaxf, then the clamp; code = rint_even(fl(fl(x + 1) * 127.5))
+  x = fminf(fmaxf(x, -1.0f), 1.0f);
+  return static_cast<uint32_t>(__float2int_rn(__fmul_rn(__fadd_rn(x, 1.0f), 127.5f)));
+}
+
+// pix[c][tau][y][x] = clamp(F[tau*L + (y/rs)*gw + x/rs][c*rs*rs + (y%rs)*rs + x%rs]); rs % 4 == 0
+__global__ void pixel_head_kernel(const float* __restrict__ F, int frames, int gh, int gw, int C,
+                                  int rs, int out_u8, void* __restrict__ pix) {
+  const int Wo = gw * rs, Ho = gh * rs;
+  const int L = gh * gw;
+  const int ld = C * rs * rs;
+  const int q_per_row = Wo / 4;
+  const long long total = static_cast<long long>(C) * frames * Ho * q_per_row;
+  for (long long idx = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;
+       idx < total; idx += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int xq = static_cast<int>(idx % q_per_row);
+    long long r = idx / q_per_row;
+    const int y = static_cast<int>(r % Ho);
+    r /= Ho;
+    const int tau = static_cast<int>(r % frames);
+    const int c = static_cast<int>(r / frames);
+    const int x = 4 * xq;
+    const int tok = tau * L + (y / rs) * gw + x / rs;
+    const int ch = c * rs * rs + (y % rs) * rs + (x % rs);
+    const float4 v = *reinterpret_cast<const float4*>(F + static_cast<size_t>(tok) * ld + ch);
+    const size_t o = ((static_cast<size_t>(c) * frames + tau) * Ho + y) * Wo + x;
+    if (out_u8) {
+      const uint32_t packed = quant_u8(v.x) | (quant_u8(v.y) << 8) | (quant_u8(v.z) << 16) |
+                              (quant_u8(v.w) << 24);
+      *reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(pix) + o) = packed;
+    } else {
+      *reinterpret_cast<float4*>(static_cast<float*>(pix) + o) =
+          make_float4(fminf(fmaxf(v.x, -1.f), 1.f), fminf(fmaxf(v.y, -1.f), 1.f),
+                      fminf(fmaxf(v.z, -1.f), 1.f), fminf(fmaxf(v.w, -1.f), 1.f));
+    }
+  }
+}
+
+// K, V fp32 [groups][rows][64] -> k_ring[g][slot*rows + r][d], vt_ring[g][d][slot*rows + r]
+// (bf16, round to nearest even). Block: 32 x 8 threads over a 32-row x 64-dim tile; V goes
+// through shared memory so both the read and the transposed write are coalesced.
+__global__ void kv_append_kernel(const float* __restrict__ k, const float* __restrict__ v,
+                                 int rows, int slot, int pitch, __nv_bfloat16* __restrict__ k_ring,
+                                 __nv_bfloat16* __restrict__ vt_ring) {
+  __shared__ float tile[64][33];
+  const int g = blockIdx.y;
+  const int r0 = blockIdx.x * 32;
+  const size_t src = static_cast<size_t>(g) * rows * kHeadDim;
+  const size_t dst_row0 = static_cast<size_t>(g) * pitch + static_cast<size_t>(slot) * rows;
+  for (int rr = threadIdx.y; rr < 32; rr += blockDim.y) {
+    const int r = r0 + rr;
+    if (r >= rows) break;
+    for (int d = threadIdx.x; d < kHeadDim; d += 32) {
+      k_ring[(dst_row0 + r) * kHeadDim + d] = __float2bfloat16_rn(k[src + r * kHeadDim + d]);
+      tile[d][rr] = v[src + static_cast<size_t>(r) * kHeadDim + d];
+    }
+  }
+  __syncthreads();
+  for (int d = threadIdx.y; d < kHeadDim; d += blockDim.y) {
+    const int r = r0 + threadIdx.x;
+    if (r < rows)
+      vt_ring[(static_cast<size_t>(g) * kHeadDim + d) * pitch + slot * static_cast<size_t>(rows) +
+              r] = __float2bfloat16_rn(tile[d][threadIdx.x]);
+  }
+}
+
+__global__ void advance_kernel(int* step) { *step += 1; }
+
+static int grid_for(long long work, int threads) {
+  long long b = (work + threads - 1) / threads;
+  if (b > 152LL * 16) b = 152LL * 16;
+  return static_cast<int>(b < 1 ? 1 : b);
+}
+
+cudaError_t launch_unshuffle(const float* z, int C, int H, int W, int p, __nv_bfloat16* x0,
+                             cudaStream_t s) {
+  const long long total = static_cast<long long>(H / p) * (W / p) * C * p * p;
+  unshuffle_kernel<<<grid_for(total, 256), 256, 0, s>>>(z, C, H, W, p, x0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm(const float* h, const float* g, int M, int D, float eps,
+                           __nv_bfloat16* u, cudaStream_t s) {
+  rmsnorm_kernel<<<(M + 7) / 8, 256, 0, s>>>(h, g, M, D, eps, u);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pixel_head(const float* F, int frames, int gh, int gw, int C, int rs,
+                              int out_u8, void* pix, cudaStream_t s) {
+  const long long total = static_cast<long long>(C) * frames * gh * rs * gw * rs / 4;
+  pixel_head_kernel<<<grid_for(total, 256), 256, 0, s>>>(F, frames, gh, gw, C, rs, out_u8, pix);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_kv_append(const float* k, const float* v, int groups, int rows, int slot,
+                             int ring_pitch, __nv_bfloat16* k_ring, __nv_bfloat16* vt_ring,
+                             cudaStream_t s) {
+  dim3 grid((rows + 31) / 32, groups);
+  kv_append_kernel<<<grid, dim3(32, 8), 0, s>>>(k, v, rows, slot, ring_pitch, k_ring, vt_ring);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_advance(int* step_dev, cudaStream_t s) {
+  advance_kernel<<<1, 1, 0, s>>>(step_dev);
+  return cudaGetLastError();
+}
+
+}  // namespace fd

@@ -1,0 +1,835 @@
+// Host runtime of the C ABI (include/flashdec.h, include/flashdec_ops.h): configuration
+// checks, device weights, per-stream state (KV rings, scratch, chunk counter), TMA
+// descriptors, and the per-chunk kernel sequence of Algorithm 1.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+#include "fd_internal.h"
+#include "flashdec.h"
+#include "flashdec_ops.h"
+
+using fd::kHeadDim;
+
+namespace {
+
+// ---------------------------------------------------------------- driver entry points
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+bool load_encode() {
+  std::call_once(g_encode_once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  return g_encode != nullptr;
+}
+
+// 2D bf16 tensor [outer][inner] with row pitch row_bytes, 128-byte swizzled box
+// {box_inner (<= 64), box_outer}.
+bool tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+               uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  if (!load_encode()) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                  box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int g_num_sms = 0;
+int num_sms() {
+  if (g_num_sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (g_num_sms <= 0) g_num_sms = 1;
+  }
+  return g_num_sms;
+}
+
+fd_status check_device() {
+  int dev = 0, major = 0, minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return FD_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+    return FD_ERR_CUDA;
+  if (major != 10 || minor != 3) return FD_ERR_UNSUPPORTED;  // built for sm_103a only
+  return FD_OK;
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// ---------------------------------------------------------------- configuration
+struct Dims {
+  int C, H, W, p, D, N, G, Dh, Mr, nb, nr, Wn, rt, rs, Cout, cin, gh, gw, L, head_out, qkv_out;
+  bool u8;
+};
+
+bool valid_cfg(const fd_config* c) {
+  if (c == nullptr) return false;
+  if (c->latent_channels < 1 || c->latent_h < 1 || c->latent_w < 1 || c->patch < 1) return false;
+  if (c->latent_h % c->patch || c->latent_w % c->patch) return false;
+  if (c->heads < 1 || c->kv_groups < 1 || c->heads % c->kv_groups) return false;
+  if (c->hidden != c->heads * kHeadDim || c->hidden % 128) return false;
+  if (c->mlp_ratio < 1 || c->n_blocks < 1 || c->n_refine < 0 || c->window < 1 || c->r_t < 1)
+    return false;
+  if (c->vae_spatial < 1 || c->out_channels < 1) return false;
+  const int rs = c->vae_spatial * c->patch;
+  if (rs % 4) return false;
+  if ((c->out_channels * rs * rs) % 64) return false;
+  if ((c->latent_channels * c->patch * c->patch) % 8) return false;  // TMA row pitch
+  if (c->out_dtype != FD_DTYPE_F32 && c->out_dtype != FD_DTYPE_U8) return false;
+  if (c->reserved != 0) return false;
+  if (!(c->norm_eps >= 0.f) || !(c->rope_base > 1.f)) return false;
+  const long long L = static_cast<long long>(c->latent_h / c->patch) * (c->latent_w / c->patch);
+  if (L * c->r_t * c->window > (1LL << 26)) return false;
+  return true;
+}
+
+Dims dims_of(const fd_config* c) {
+  Dims d;
+  d.C = c->latent_channels; d.H = c->latent_h; d.W = c->latent_w; d.p = c->patch;
+  d.D = c->hidden; d.N = c->heads; d.G = c->kv_groups; d.Dh = kHeadDim; d.Mr = c->mlp_ratio;
+  d.nb = c->n_blocks; d.nr = c->n_refine; d.Wn = c->window; d.rt = c->r_t;
+  d.rs = c->vae_spatial * c->patch; d.Cout = c->out_channels;
+  d.cin = d.C * d.p * d.p; d.gh = d.H / d.p; d.gw = d.W / d.p; d.L = d.gh * d.gw;
+  d.head_out = d.Cout * d.rs * d.rs; d.qkv_out = (d.N + 2 * d.G) * kHeadDim;
+  d.u8 = c->out_dtype == FD_DTYPE_U8;
+  return d;
+}
+
+bool same_cfg(const fd_config* a, const fd_config* b) {
+  return std::memcmp(a, b, sizeof(fd_config)) == 0;
+}
+
+// blob element counts, in blob order
+struct BlobEntry { size_t elems; int kind; };  // kind: 0 weight (bf16 on device), 1 fp32
+void blob_layout(const Dims& d, std::vector<BlobEntry>& out) {
+  auto W = [&](size_t n) { out.push_back({n, 0}); };
+  auto F = [&](size_t n) { out.push_back({n, 1}); };
+  const size_t D = d.D, Dm = static_cast<size_t>(d.Mr) * d.D;
+  W(D * d.cin); F(D);
+  auto block = [&] {
+    F(D); W(static_cast<size_t>(d.qkv_out) * D); F(d.qkv_out); F(kHeadDim); F(kHeadDim);
+    W(D * d.N * kHeadDim); F(D); F(D); W(Dm * D); F(Dm); W(D * Dm); F(D);
+  };
+  for (int b = 0; b < d.nb; ++b) block();
+  F(D); W(static_cast<size_t>(d.rt) * D * D); F(static_cast<size_t>(d.rt) * D);
+  for (int b = 0; b < d.nr; ++b) block();
+  F(D); W(D * D); F(D); W(static_cast<size_t>(d.head_out) * D); F(d.head_out);
+}
+
+uint16_t f32_to_bf16_rne(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  if ((u & 0x7F800000u) == 0x7F800000u && (u & 0x007FFFFFu)) return 0x7FC0;  // NaN
+  const uint32_t lsb = (u >> 16) & 1u;
+  return static_cast<uint16_t>((u + 0x7FFFu + lsb) >> 16);
+}
+float bf16_to_f32(uint16_t b) {
+  const uint32_t u = static_cast<uint32_t>(b) << 16;
+  float f;
+  std::memcpy(&f, &u, 4);
+  return f;
+}
+
+// GEMM tile width for an M x N problem: fewest "waves x width" on the SM count
+int pick_bn(int M, int N) {
+  const int sms = num_sms();
+  int best = 128;
+  long long best_cost = -1;
+  for (int bn : {128, 256}) {
+    if (N % bn && bn != 128) continue;
+    const long long tiles = static_cast<long long>((M + 127) / 128) * ((N + bn - 1) / bn);
+    const long long waves = (tiles + sms - 1) / sms;
+    const long long cost = waves * bn * 100 + bn;  // prefer the narrower tile on ties
+    if (best_cost < 0 || cost < best_cost) { best_cost = cost; best = bn; }
+  }
+  return best;
+}
+
+struct Linear {
+  __nv_bfloat16* w = nullptr;  // [N][K]
+  float* b = nullptr;          // [N]
+  int N = 0, K = 0, bn = 128;
+  CUtensorMap tm;
+};
+
+struct LayerW {
+  float *g1 = nullptr, *g2 = nullptr, *kg = nullptr, *vg = nullptr;
+  Linear qkv, out, mlp1, mlp2;
+};
+
+}  // namespace
+
+struct fd_weights_s {
+  fd_config cfg;
+  Dims d;
+  void* arena = nullptr;
+  Linear embed, tup, head1, head2;
+  float *g_f = nullptr, *g_h = nullptr;
+  std::vector<LayerW> blocks, refine;
+  int live_handles = 0;
+};
+
+namespace {
+
+struct Ring {
+  __nv_bfloat16* k = nullptr;   // [G][pitch][64]
+  __nv_bfloat16* vt = nullptr;  // [G][64][pitch]
+  CUtensorMap tm_k, tm_vt;
+};
+
+}  // namespace
+
+struct fd_handle_s {
+  fd_config cfg;
+  Dims d;
+  fd_weights w = nullptr;
+  void* arena = nullptr;
+  size_t arena_bytes = 0;
+  int* state = nullptr;  // [0] chunk index t, [1] error bits
+  int64_t t_host = 0;
+  bool error = false;
+  cudaStream_t last_stream = nullptr;
+  // activations (rows: L for the backbone, r_t L for refinement / head)
+  __nv_bfloat16 *x0 = nullptr, *u = nullptr, *q = nullptr, *o = nullptr, *hid = nullptr;
+  float *h = nullptr, *hf = nullptr, *F = nullptr;
+  int pitchB = 0, pitchR = 0;
+  std::vector<Ring> ringB, ringR;
+  // A-operand / Q descriptors
+  CUtensorMap tm_x0, tm_uB, tm_uR, tm_oB, tm_oR, tm_hidB, tm_hidR, tm_hidH, tm_qB, tm_qR;
+};
+
+namespace {
+
+double rope_inv_freq(int i, int band_t, int band_s, double base) {
+  // pair i: temporal band (2*band_t dims) first, then row and column bands (2*band_s each)
+  int j, d;
+  if (i < band_t) { j = i; d = 2 * band_t; }
+  else if (i < band_t + band_s) { j = i - band_t; d = 2 * band_s; }
+  else { j = i - band_t - band_s; d = 2 * band_s; }
+  return std::pow(base, -2.0 * j / d);
+}
+
+void fill_rope(fd::QkvEpi& q, float base) {
+  q.band_s = kHeadDim / 6;                 // pairs per spatial band (10 at D_h = 64)
+  q.band_t = kHeadDim / 2 - 2 * q.band_s;  // temporal pairs (12)
+  for (int i = 0; i < fd::kRopePairs; ++i)
+    q.inv_freq[i] = rope_inv_freq(i, q.band_t, q.band_s, static_cast<double>(base));
+}
+
+fd_status launch_ok(cudaError_t e) { return e == cudaSuccess ? FD_OK : FD_ERR_CUDA; }
+
+fd_status run_linear(const CUtensorMap& tmA, const Linear& lin, int M, fd::GemmParams p,
+                     cudaStream_t s) {
+  p.M = M;
+  p.N = lin.N;
+  p.K = lin.K;
+  p.bias = lin.b;
+  return launch_ok(fd::launch_gemm(tmA, lin.tm, p, lin.bn, num_sms(), s));
+}
+
+// one Transformer block (Sec. 3.2) on `rows` tokens of residual stream hbuf, with ring r
+fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int rows, int fpc,
+                    int pitch, const CUtensorMap& tm_u, const CUtensorMap& tm_q,
+                    const CUtensorMap& tm_o, const CUtensorMap& tm_hid, cudaStream_t s) {
+  const Dims& d = h->d;
+  fd_status st;
+  if ((st = launch_ok(fd::launch_rmsnorm(hbuf, lw.g1, rows, d.D, h->cfg.norm_eps, h->u, s))))
+    return st;
+  fd::GemmParams p{};
+  p.err = h->state + 1;
+  p.epi = fd::EPI_QKV;
+  fd::QkvEpi& q = p.qkv;
+  q.heads = d.N; q.groups = d.G; q.knorm_g = lw.kg; q.vnorm_g = lw.vg; q.q_out = h->q;
+  q.k_ring = r.k; q.vt_ring = r.vt; q.ring_pitch = pitch; q.tokens = d.L; q.grid_w = d.gw;
+  q.frames_per_chunk = fpc; q.window = d.Wn; q.step_dev = h->state; q.step_host = 0;
+  q.eps = h->cfg.norm_eps;
+  fill_rope(q, h->cfg.rope_base);
+  if ((st = run_linear(tm_u, lw.qkv, rows, p, s))) return st;
+
+  fd::AttnParams a{};
+  a.Lq = rows; a.heads = d.N; a.groups = d.G; a.ring_pitch = pitch; a.rows_per_chunk = rows;
+  a.window = d.Wn; a.step_dev = h->state; a.n_keys_host = 0; a.out = h->o;
+  a.ld_out = d.N * kHeadDim; a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
+  a.err = h->state + 1;
+  if ((st = launch_ok(fd::launch_attention(tm_q, r.tm_k, r.tm_vt, a, s)))) return st;
+
+  fd::GemmParams po{};
+  po.err = h->state + 1;
+  po.epi = fd::EPI_RESID;
+  po.out_f32 = hbuf;
+  po.ld_out = d.D;
+  if ((st = run_linear(tm_o, lw.out, rows, po, s))) return st;
+  if ((st = launch_ok(fd::launch_rmsnorm(hbuf, lw.g2, rows, d.D, h->cfg.norm_eps, h->u, s))))
+    return st;
+  fd::GemmParams p1{};
+  p1.err = h->state + 1;
+  p1.epi = fd::EPI_GELU;
+  p1.out_bf16 = h->hid;
+  p1.ld_out = d.Mr * d.D;
+  if ((st = run_linear(tm_u, lw.mlp1, rows, p1, s))) return st;
+  return run_linear(tm_hid, lw.mlp2, rows, po, s);
+}
+
+fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_t s) {
+  const Dims& d = h->d;
+  const fd_weights w = h->w;
+  fd_status st;
+  if ((st = launch_ok(fd::launch_unshuffle(latent, d.C, d.H, d.W, d.p, h->x0, s)))) return st;
+  fd::GemmParams pe{};
+  pe.err = h->state + 1;
+  pe.epi = fd::EPI_F32;
+  pe.out_f32 = h->h;
+  pe.ld_out = d.D;
+  if ((st = run_linear(h->tm_x0, w->embed, d.L, pe, s))) return st;
+  for (int b = 0; b < d.nb; ++b)
+    if ((st = run_block(h, w->blocks[b], h->ringB[b], h->h, d.L, 1, h->pitchB, h->tm_uB, h->tm_qB,
+                        h->tm_oB, h->tm_hidB, s)))
+      return st;
+  // temporal upsampling: RMSNorm, Linear D -> r_t D, channel block tau -> refined frame tau
+  if ((st = launch_ok(fd::launch_rmsnorm(h->h, w->g_f, d.L, d.D, h->cfg.norm_eps, h->u, s))))
+    return st;
+  fd::GemmParams pt{};
+  pt.err = h->state + 1;
+  pt.epi = fd::EPI_TUP;
+  pt.out_f32 = h->hf;
+  pt.tup_tokens = d.L;
+  pt.tup_hidden = d.D;
+  if ((st = run_linear(h->tm_uB, w->tup, d.L, pt, s))) return st;
+  const int R = d.rt * d.L;
+  for (int b = 0; b < d.nr; ++b)
+    if ((st = run_block(h, w->refine[b], h->ringR[b], h->hf, R, d.rt, h->pitchR, h->tm_uR,
+                        h->tm_qR, h->tm_oR, h->tm_hidR, s)))
+      return st;
+  // spatial upsampling head: RMSNorm, Linear D->D + GELU, Linear D -> C r_s^2, PixelShuffle
+  if ((st = launch_ok(fd::launch_rmsnorm(h->hf, w->g_h, R, d.D, h->cfg.norm_eps, h->u, s))))
+    return st;
+  fd::GemmParams ph{};
+  ph.err = h->state + 1;
+  ph.epi = fd::EPI_GELU;
+  ph.out_bf16 = h->hid;
+  ph.ld_out = d.D;
+  if ((st = run_linear(h->tm_uR, w->head1, R, ph, s))) return st;
+  fd::GemmParams pf{};
+  pf.err = h->state + 1;
+  pf.epi = fd::EPI_F32;
+  pf.out_f32 = h->F;
+  pf.ld_out = d.head_out;
+  if ((st = run_linear(h->tm_hidH, w->head2, R, pf, s))) return st;
+  if ((st = launch_ok(fd::launch_pixel_head(h->F, d.rt, d.gh, d.gw, d.Cout, d.rs, d.u8 ? 1 : 0,
+                                            pixels, s))))
+    return st;
+  return launch_ok(fd::launch_advance(h->state, s));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" {
+
+const char* fd_status_str(fd_status s) {
+  switch (s) {
+    case FD_OK: return "ok";
+    case FD_ERR_INVALID_ARG: return "invalid argument";
+    case FD_ERR_CONFIG: return "unsupported configuration";
+    case FD_ERR_OOM: return "device out of memory";
+    case FD_ERR_CUDA: return "CUDA error";
+    case FD_ERR_STATE: return "handle in error state (fd_reset it)";
+    case FD_ERR_DEVICE_TIMEOUT: return "device wait timed out";
+    case FD_ERR_UNSUPPORTED: return "device is not sm_103";
+  }
+  return "unknown status";
+}
+
+size_t fd_weights_blob_elems(const fd_config* cfg) {
+  if (!valid_cfg(cfg)) return 0;
+  std::vector<BlobEntry> e;
+  blob_layout(dims_of(cfg), e);
+  size_t n = 0;
+  for (auto& x : e) n += x.elems;
+  return n;
+}
+
+size_t fd_latent_bytes(const fd_config* cfg) {
+  if (!valid_cfg(cfg)) return 0;
+  return static_cast<size_t>(cfg->latent_channels) * cfg->latent_h * cfg->latent_w * 4;
+}
+
+size_t fd_pixels_bytes(const fd_config* cfg) {
+  if (!valid_cfg(cfg)) return 0;
+  const Dims d = dims_of(cfg);
+  return static_cast<size_t>(d.Cout) * d.rt * d.gh * d.rs * d.gw * d.rs * (d.u8 ? 1 : 4);
+}
+
+static size_t handle_layout(const Dims& d, size_t* off /* 12 offsets */, int* pitchB,
+                            int* pitchR) {
+  const size_t R = static_cast<size_t>(d.rt) * d.L;
+  *pitchB = static_cast<int>(align_up(static_cast<size_t>(d.Wn) * d.L, 128));
+  *pitchR = static_cast<int>(align_up(static_cast<size_t>(d.Wn) * R, 128));
+  size_t sizes[11] = {
+      16,                                              // state
+      static_cast<size_t>(d.L) * d.cin * 2,            // x0
+      R * d.D * 2,                                     // u
+      R * d.N * kHeadDim * 2,                          // q
+      R * d.N * kHeadDim * 2,                          // o
+      R * static_cast<size_t>(d.Mr) * d.D * 2,         // hid
+      static_cast<size_t>(d.L) * d.D * 4,              // h
+      R * d.D * 4,                                     // hf
+      R * d.head_out * 4,                              // F
+      static_cast<size_t>(d.nb) * 2 * d.G * *pitchB * kHeadDim * 2,  // backbone rings
+      static_cast<size_t>(d.nr) * 2 * d.G * *pitchR * kHeadDim * 2,  // refinement rings
+  };
+  size_t cur = 0;
+  for (int i = 0; i < 11; ++i) {
+    off[i] = cur;
+    cur = align_up(cur + sizes[i], 1024);
+  }
+  off[11] = cur;
+  return cur;
+}
+
+size_t fd_handle_device_bytes(const fd_config* cfg) {
+  if (!valid_cfg(cfg)) return 0;
+  size_t off[12];
+  int a, b;
+  return handle_layout(dims_of(cfg), off, &a, &b);
+}
+
+fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t blob_bytes,
+                            int blob_dtype, fd_weights* out) {
+  if (out == nullptr) return FD_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!valid_cfg(cfg)) return FD_ERR_CONFIG;
+  if (host_blob == nullptr) return FD_ERR_INVALID_ARG;
+  if (blob_dtype != FD_DTYPE_F32 && blob_dtype != FD_DTYPE_BF16) return FD_ERR_INVALID_ARG;
+  const size_t esz = blob_dtype == FD_DTYPE_F32 ? 4 : 2;
+  if (blob_bytes != fd_weights_blob_elems(cfg) * esz) return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  if (!load_encode()) return FD_ERR_CUDA;
+
+  const Dims d = dims_of(cfg);
+  std::vector<BlobEntry> layout;
+  blob_layout(d, layout);
+  // device arena: bf16 weights then fp32 vectors, each 256-byte aligned
+  std::vector<size_t> doff(layout.size());
+  size_t cur = 0;
+  for (size_t i = 0; i < layout.size(); ++i) {
+    doff[i] = cur;
+    cur = align_up(cur + layout[i].elems * (layout[i].kind == 0 ? 2 : 4), 256);
+  }
+  std::vector<uint8_t> stage;
+  try {
+    stage.assign(cur, 0);
+  } catch (...) {
+    return FD_ERR_OOM;
+  }
+  size_t src = 0;
+  for (size_t i = 0; i < layout.size(); ++i) {
+    for (size_t k = 0; k < layout[i].elems; ++k, ++src) {
+      float f;
+      if (blob_dtype == FD_DTYPE_F32) {
+        std::memcpy(&f, static_cast<const uint8_t*>(host_blob) + 4 * src, 4);
+      } else {
+        uint16_t b;
+        std::memcpy(&b, static_cast<const uint8_t*>(host_blob) + 2 * src, 2);
+        f = bf16_to_f32(b);
+      }
+      if (layout[i].kind == 0) {
+        const uint16_t b = f32_to_bf16_rne(f);
+        std::memcpy(&stage[doff[i] + 2 * k], &b, 2);
+      } else {
+        std::memcpy(&stage[doff[i] + 4 * k], &f, 4);
+      }
+    }
+  }
+  fd_weights w = new (std::nothrow) fd_weights_s;
+  if (w == nullptr) return FD_ERR_OOM;
+  w->cfg = *cfg;
+  w->d = d;
+  if (cudaMalloc(&w->arena, cur) != cudaSuccess) {
+    delete w;
+    return FD_ERR_OOM;
+  }
+  if (cudaMemcpy(w->arena, stage.data(), cur, cudaMemcpyHostToDevice) != cudaSuccess) {
+    cudaFree(w->arena);
+    delete w;
+    return FD_ERR_CUDA;
+  }
+  uint8_t* base = static_cast<uint8_t*>(w->arena);
+  size_t idx = 0;
+  auto next = [&]() { return base + doff[idx++]; };
+  auto linear = [&](Linear& lin, int N, int K, int M) -> bool {
+    lin.w = reinterpret_cast<__nv_bfloat16*>(next());
+    lin.b = reinterpret_cast<float*>(next());
+    lin.N = N;
+    lin.K = K;
+    lin.bn = pick_bn(M, N);
+    return tmap_bf16(&lin.tm, lin.w, K, N, static_cast<uint64_t>(K) * 2, fd::kBK, lin.bn);
+  };
+  bool ok = linear(w->embed, d.D, d.cin, d.L);
+  auto block = [&](LayerW& lw, int M) {
+    lw.g1 = reinterpret_cast<float*>(next());
+    ok = ok && linear(lw.qkv, d.qkv_out, d.D, M);
+    lw.kg = reinterpret_cast<float*>(next());
+    lw.vg = reinterpret_cast<float*>(next());
+    ok = ok && linear(lw.out, d.D, d.N * kHeadDim, M);
+    lw.g2 = reinterpret_cast<float*>(next());
+    ok = ok && linear(lw.mlp1, d.Mr * d.D, d.D, M);
+    ok = ok && linear(lw.mlp2, d.D, d.Mr * d.D, M);
+  };
+  w->blocks.resize(d.nb);
+  for (auto& lw : w->blocks) block(lw, d.L);
+  w->g_f = reinterpret_cast<float*>(next());
+  ok = ok && linear(w->tup, d.rt * d.D, d.D, d.L);
+  w->refine.resize(d.nr);
+  for (auto& lw : w->refine) block(lw, d.rt * d.L);
+  w->g_h = reinterpret_cast<float*>(next());
+  ok = ok && linear(w->head1, d.D, d.D, d.rt * d.L);
+  ok = ok && linear(w->head2, d.head_out, d.D, d.rt * d.L);
+  if (!ok || idx != layout.size()) {
+    cudaFree(w->arena);
+    delete w;
+    return FD_ERR_CUDA;
+  }
+  *out = w;
+  return FD_OK;
+}
+
+fd_status fd_weights_destroy(fd_weights w) {
+  if (w == nullptr) return FD_ERR_INVALID_ARG;
+  if (w->live_handles > 0) return FD_ERR_STATE;
+  cudaFree(w->arena);
+  delete w;
+  return FD_OK;
+}
+
+fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
+  if (out == nullptr || w == nullptr) return FD_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!valid_cfg(cfg)) return FD_ERR_CONFIG;
+  if (!same_cfg(cfg, &w->cfg)) return FD_ERR_CONFIG;
+  fd_status st = check_device();
+  if (st) return st;
+  fd_handle h = new (std::nothrow) fd_handle_s;
+  if (h == nullptr) return FD_ERR_OOM;
+  h->cfg = *cfg;
+  h->d = dims_of(cfg);
+  h->w = w;
+  const Dims& d = h->d;
+  size_t off[12];
+  h->arena_bytes = handle_layout(d, off, &h->pitchB, &h->pitchR);
+  if (cudaMalloc(&h->arena, h->arena_bytes) != cudaSuccess) {
+    delete h;
+    return FD_ERR_OOM;
+  }
+  uint8_t* b = static_cast<uint8_t*>(h->arena);
+  h->state = reinterpret_cast<int*>(b + off[0]);
+  h->x0 = reinterpret_cast<__nv_bfloat16*>(b + off[1]);
+  h->u = reinterpret_cast<__nv_bfloat16*>(b + off[2]);
+  h->q = reinterpret_cast<__nv_bfloat16*>(b + off[3]);
+  h->o = reinterpret_cast<__nv_bfloat16*>(b + off[4]);
+  h->hid = reinterpret_cast<__nv_bfloat16*>(b + off[5]);
+  h->h = reinterpret_cast<float*>(b + off[6]);
+  h->hf = reinterpret_cast<float*>(b + off[7]);
+  h->F = reinterpret_cast<float*>(b + off[8]);
+  const size_t ringB_elems = static_cast<size_t>(d.G) * h->pitchB * kHeadDim;
+  const size_t ringR_elems = static_cast<size_t>(d.G) * h->pitchR * kHeadDim;
+  h->ringB.resize(d.nb);
+  h->ringR.resize(d.nr);
+  bool ok = true;
+  for (int i = 0; i < d.nb; ++i) {
+    Ring& r = h->ringB[i];
+    r.k = reinterpret_cast<__nv_bfloat16*>(b + off[9]) + 2 * i * ringB_elems;
+    r.vt = r.k + ringB_elems;
+    ok = ok && tmap_bf16(&r.tm_k, r.k, kHeadDim, static_cast<uint64_t>(d.G) * h->pitchB,
+                         kHeadDim * 2, 64, 128);
+    ok = ok && tmap_bf16(&r.tm_vt, r.vt, h->pitchB, static_cast<uint64_t>(d.G) * kHeadDim,
+                         static_cast<uint64_t>(h->pitchB) * 2, 64, 64);
+  }
+  for (int i = 0; i < d.nr; ++i) {
+    Ring& r = h->ringR[i];
+    r.k = reinterpret_cast<__nv_bfloat16*>(b + off[10]) + 2 * i * ringR_elems;
+    r.vt = r.k + ringR_elems;
+    ok = ok && tmap_bf16(&r.tm_k, r.k, kHeadDim, static_cast<uint64_t>(d.G) * h->pitchR,
+                         kHeadDim * 2, 64, 128);
+    ok = ok && tmap_bf16(&r.tm_vt, r.vt, h->pitchR, static_cast<uint64_t>(d.G) * kHeadDim,
+                         static_cast<uint64_t>(h->pitchR) * 2, 64, 64);
+  }
+  const uint64_t R = static_cast<uint64_t>(d.rt) * d.L;
+  const uint64_t NQ = static_cast<uint64_t>(d.N) * kHeadDim;
+  const uint64_t Dm = static_cast<uint64_t>(d.Mr) * d.D;
+  ok = ok && tmap_bf16(&h->tm_x0, h->x0, d.cin, d.L, d.cin * 2, 64, 128);
+  ok = ok && tmap_bf16(&h->tm_uB, h->u, d.D, d.L, d.D * 2, 64, 128);
+  ok = ok && tmap_bf16(&h->tm_uR, h->u, d.D, R, d.D * 2, 64, 128);
+  ok = ok && tmap_bf16(&h->tm_oB, h->o, NQ, d.L, NQ * 2, 64, 128);
+  ok = ok && tmap_bf16(&h->tm_oR, h->o, NQ, R, NQ * 2, 64, 128);
+  ok = ok && tmap_bf16(&h->tm_qB, h->q, NQ, d.L, NQ * 2, 64, 128);
+  ok = ok && tmap_bf16(&h->tm_qR, h->q, NQ, R, NQ * 2, 64, 128);
+  ok = ok && tmap_bf16(&h->tm_hidB, h->hid, Dm, d.L, Dm * 2, 64, 128);
+  ok = ok && tmap_bf16(&h->tm_hidR, h->hid, Dm, R, Dm * 2, 64, 128);
+  ok = ok && tmap_bf16(&h->tm_hidH, h->hid, d.D, R, static_cast<uint64_t>(d.D) * 2, 64, 128);
+  if (!ok || cudaMemset(h->arena, 0, h->arena_bytes) != cudaSuccess ||
+      cudaDeviceSynchronize() != cudaSuccess) {
+    cudaFree(h->arena);
+    delete h;
+    return FD_ERR_CUDA;
+  }
+  w->live_handles++;
+  *out = h;
+  return FD_OK;
+}
+
+fd_status fd_decode_chunk(fd_handle h, const float* latent_dev, void* pixels_dev, void* stream) {
+  if (h == nullptr || latent_dev == nullptr || pixels_dev == nullptr) return FD_ERR_INVALID_ARG;
+  if (!aligned16(latent_dev) || !aligned16(pixels_dev)) return FD_ERR_INVALID_ARG;
+  if (h->error) return FD_ERR_STATE;
+  if (h->t_host >= (1LL << 30)) return FD_ERR_STATE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  h->last_stream = s;
+  fd_status st = decode_one(h, latent_dev, pixels_dev, s);
+  if (st != FD_OK) {
+    h->error = true;
+    return st;
+  }
+  h->t_host++;
+  return FD_OK;
+}
+
+fd_status fd_decode_chunks(fd_handle* hs, int n, const float* const* latents_dev,
+                           void* const* pixels_dev, void* stream) {
+  if (hs == nullptr || n < 0 || (n > 0 && (latents_dev == nullptr || pixels_dev == nullptr)))
+    return FD_ERR_INVALID_ARG;
+  for (int i = 0; i < n; ++i) {
+    fd_status st = fd_decode_chunk(hs[i], latents_dev[i], pixels_dev[i], stream);
+    if (st != FD_OK) return st;
+  }
+  return FD_OK;
+}
+
+fd_status fd_reset(fd_handle h) {
+  if (h == nullptr) return FD_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) cudaGetLastError();
+  if (cudaMemset(h->state, 0, 2 * sizeof(int)) != cudaSuccess) return FD_ERR_CUDA;
+  if (cudaDeviceSynchronize() != cudaSuccess) return FD_ERR_CUDA;
+  h->t_host = 0;
+  h->error = false;
+  return FD_OK;
+}
+
+fd_status fd_destroy(fd_handle h) {
+  if (h == nullptr) return FD_ERR_INVALID_ARG;
+  cudaStreamSynchronize(h->last_stream);
+  cudaFree(h->arena);
+  if (h->w) h->w->live_handles--;
+  delete h;
+  return FD_OK;
+}
+
+int64_t fd_chunk_index(fd_handle h) { return h ? h->t_host : -1; }
+
+fd_status fd_sync_status(fd_handle h) {
+  if (h == nullptr) return FD_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) {
+    h->error = true;
+    return FD_ERR_CUDA;
+  }
+  int st[2] = {0, 0};
+  if (cudaMemcpy(st, h->state, sizeof(st), cudaMemcpyDeviceToHost) != cudaSuccess) {
+    h->error = true;
+    return FD_ERR_CUDA;
+  }
+  if (st[1] != 0) {
+    h->error = true;
+    return FD_ERR_DEVICE_TIMEOUT;
+  }
+  return h->error ? FD_ERR_STATE : FD_OK;
+}
+
+fd_status fd_debug_read_ring(fd_handle h, int which, int layer, void* dst_host,
+                             size_t dst_bytes) {
+  if (h == nullptr || dst_host == nullptr) return FD_ERR_INVALID_ARG;
+  const Dims& d = h->d;
+  const std::vector<Ring>& rings = which == 0 ? h->ringB : h->ringR;
+  if ((which != 0 && which != 1) || layer < 0 || layer >= static_cast<int>(rings.size()))
+    return FD_ERR_INVALID_ARG;
+  const int rows = which == 0 ? d.L : d.rt * d.L;
+  const int pitch = which == 0 ? h->pitchB : h->pitchR;
+  const size_t n = static_cast<size_t>(d.G) * d.Wn * rows * kHeadDim;
+  if (dst_bytes < 2 * n * 2) return FD_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) return FD_ERR_CUDA;
+  std::vector<uint16_t> kbuf(static_cast<size_t>(d.G) * pitch * kHeadDim);
+  std::vector<uint16_t> vbuf(kbuf.size());
+  if (cudaMemcpy(kbuf.data(), rings[layer].k, kbuf.size() * 2, cudaMemcpyDeviceToHost) ||
+      cudaMemcpy(vbuf.data(), rings[layer].vt, vbuf.size() * 2, cudaMemcpyDeviceToHost))
+    return FD_ERR_CUDA;
+  uint16_t* out = static_cast<uint16_t*>(dst_host);
+  const size_t span = static_cast<size_t>(d.Wn) * rows;
+  for (int g = 0; g < d.G; ++g)
+    for (size_t r = 0; r < span; ++r)
+      for (int c = 0; c < kHeadDim; ++c) {
+        out[(g * span + r) * kHeadDim + c] = kbuf[(static_cast<size_t>(g) * pitch + r) * kHeadDim + c];
+        out[n + (g * span + r) * kHeadDim + c] =
+            vbuf[(static_cast<size_t>(g) * kHeadDim + c) * pitch + r];
+      }
+  return FD_OK;
+}
+
+// ---------------------------------------------------------------- kernel-level entry points
+
+fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const void* W,
+                       const float* bias, void* out, int tup_hidden, int bn, int* err_dev,
+                       void* stream) {
+  if (M < 1 || N < 1 || K < 1 || A == nullptr || W == nullptr || bias == nullptr ||
+      out == nullptr || err_dev == nullptr)
+    return FD_ERR_INVALID_ARG;
+  if (N % 32 || K % 8 || !aligned16(A) || !aligned16(W) || !aligned16(out))
+    return FD_ERR_INVALID_ARG;
+  if (bn == 0) bn = pick_bn(M, N);
+  if (!fd::gemm_bn_supported(bn)) return FD_ERR_INVALID_ARG;
+  if (epilogue < FD_EPI_F32 || epilogue > FD_EPI_TUP) return FD_ERR_INVALID_ARG;
+  if (epilogue == FD_EPI_TUP && (tup_hidden < 32 || tup_hidden % 32 || N % tup_hidden))
+    return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  CUtensorMap ta, tb;
+  if (!tmap_bf16(&ta, A, K, M, static_cast<uint64_t>(K) * 2, 64, 128) ||
+      !tmap_bf16(&tb, W, K, N, static_cast<uint64_t>(K) * 2, 64, bn))
+    return FD_ERR_CUDA;
+  fd::GemmParams p{};
+  p.M = M; p.N = N; p.K = K; p.epi = epilogue; p.bias = bias; p.err = err_dev;
+  if (epilogue == FD_EPI_GELU) {
+    p.out_bf16 = static_cast<__nv_bfloat16*>(out);
+  } else {
+    p.out_f32 = static_cast<float*>(out);
+  }
+  p.ld_out = N;
+  p.tup_tokens = M;
+  p.tup_hidden = tup_hidden;
+  return launch_ok(fd::launch_gemm(ta, tb, p, bn, num_sms(), static_cast<cudaStream_t>(stream)));
+}
+
+fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* bqkv,
+                    const float* knorm_g, const float* vnorm_g, int heads, int groups,
+                    int tokens, int grid_w, int frames_per_chunk, int window, int t, float eps,
+                    float rope_base, void* q_out, void* k_ring, void* vt_ring, int ring_pitch,
+                    int bn, int* err_dev, void* stream) {
+  if (!A || !Wqkv || !bqkv || !knorm_g || !vnorm_g || !q_out || !k_ring || !vt_ring || !err_dev)
+    return FD_ERR_INVALID_ARG;
+  if (heads < 1 || groups < 1 || heads % groups || tokens < 1 || grid_w < 1 ||
+      tokens % grid_w || frames_per_chunk < 1 || window < 1 || t < 0 || K < 8 || K % 8)
+    return FD_ERR_INVALID_ARG;
+  if (M != frames_per_chunk * tokens) return FD_ERR_INVALID_ARG;
+  if (ring_pitch < window * M || ring_pitch % 128) return FD_ERR_INVALID_ARG;
+  if (bn == 0) bn = 128;
+  if (!fd::gemm_bn_supported(bn)) return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  const int N = (heads + 2 * groups) * kHeadDim;
+  CUtensorMap ta, tb;
+  if (!tmap_bf16(&ta, A, K, M, static_cast<uint64_t>(K) * 2, 64, 128) ||
+      !tmap_bf16(&tb, Wqkv, K, N, static_cast<uint64_t>(K) * 2, 64, bn))
+    return FD_ERR_CUDA;
+  fd::GemmParams p{};
+  p.M = M; p.N = N; p.K = K; p.epi = fd::EPI_QKV; p.bias = bqkv; p.err = err_dev;
+  fd::QkvEpi& q = p.qkv;
+  q.heads = heads; q.groups = groups; q.knorm_g = knorm_g; q.vnorm_g = vnorm_g;
+  q.q_out = static_cast<__nv_bfloat16*>(q_out);
+  q.k_ring = static_cast<__nv_bfloat16*>(k_ring);
+  q.vt_ring = static_cast<__nv_bfloat16*>(vt_ring);
+  q.ring_pitch = ring_pitch; q.tokens = tokens; q.grid_w = grid_w;
+  q.frames_per_chunk = frames_per_chunk; q.window = window; q.step_dev = nullptr;
+  q.step_host = t; q.eps = eps;
+  fill_rope(q, rope_base);
+  return launch_ok(fd::launch_gemm(ta, tb, p, bn, num_sms(), static_cast<cudaStream_t>(stream)));
+}
+
+fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const void* k_ring,
+                          const void* vt_ring, int ring_pitch, int n_keys, void* out,
+                          int* err_dev, void* stream) {
+  if (!q || !k_ring || !vt_ring || !out || !err_dev) return FD_ERR_INVALID_ARG;
+  if (Lq < 1 || heads < 1 || groups < 1 || heads % groups || n_keys < 1 ||
+      n_keys > ring_pitch || ring_pitch % 128)
+    return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  const uint64_t NQ = static_cast<uint64_t>(heads) * kHeadDim;
+  CUtensorMap tq, tk, tv;
+  if (!tmap_bf16(&tq, q, NQ, Lq, NQ * 2, 64, 128) ||
+      !tmap_bf16(&tk, k_ring, kHeadDim, static_cast<uint64_t>(groups) * ring_pitch, kHeadDim * 2,
+                 64, 128) ||
+      !tmap_bf16(&tv, vt_ring, ring_pitch, static_cast<uint64_t>(groups) * kHeadDim,
+                 static_cast<uint64_t>(ring_pitch) * 2, 64, 64))
+    return FD_ERR_CUDA;
+  fd::AttnParams a{};
+  a.Lq = Lq; a.heads = heads; a.groups = groups; a.ring_pitch = ring_pitch;
+  a.rows_per_chunk = n_keys; a.window = 1; a.step_dev = nullptr; a.n_keys_host = n_keys;
+  a.out = static_cast<__nv_bfloat16*>(out); a.ld_out = static_cast<int>(NQ);
+  a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
+  a.err = err_dev;
+  return launch_ok(fd::launch_attention(tq, tk, tv, a, static_cast<cudaStream_t>(stream)));
+}
+
+fd_status fd_op_kv_append(const float* k, const float* v, int groups, int rows, int window,
+                          int t, int ring_pitch, void* k_ring, void* vt_ring, void* stream) {
+  if (!k || !v || !k_ring || !vt_ring || groups < 1 || rows < 1 || window < 1 || t < 0)
+    return FD_ERR_INVALID_ARG;
+  if (ring_pitch < window * rows) return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  return launch_ok(fd::launch_kv_append(k, v, groups, rows, t % window, ring_pitch,
+                                        static_cast<__nv_bfloat16*>(k_ring),
+                                        static_cast<__nv_bfloat16*>(vt_ring),
+                                        static_cast<cudaStream_t>(stream)));
+}
+
+fd_status fd_op_rmsnorm(const float* h, const float* g, int M, int D, float eps, void* u,
+                        void* stream) {
+  if (!h || !g || !u || M < 1 || D < 128 || D % 128 || !aligned16(h) || !aligned16(g))
+    return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  return launch_ok(fd::launch_rmsnorm(h, g, M, D, eps, static_cast<__nv_bfloat16*>(u),
+                                      static_cast<cudaStream_t>(stream)));
+}
+
+fd_status fd_op_unshuffle(const float* z, int C, int H, int W, int p, void* x0, void* stream) {
+  if (!z || !x0 || C < 1 || p < 1 || H < p || W < p || H % p || W % p) return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  return launch_ok(fd::launch_unshuffle(z, C, H, W, p, static_cast<__nv_bfloat16*>(x0),
+                                        static_cast<cudaStream_t>(stream)));
+}
+
+fd_status fd_op_pixel_head(const float* F, int frames, int grid_h, int grid_w, int channels,
+                           int rs, int out_dtype, void* pixels, void* stream) {
+  if (!F || !pixels || frames < 1 || grid_h < 1 || grid_w < 1 || channels < 1 || rs < 4 ||
+      rs % 4 || !aligned16(F) || !aligned16(pixels))
+    return FD_ERR_INVALID_ARG;
+  if (out_dtype != FD_DTYPE_F32 && out_dtype != FD_DTYPE_U8) return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  return launch_ok(fd::launch_pixel_head(F, frames, grid_h, grid_w, channels, rs,
+                                         out_dtype == FD_DTYPE_U8 ? 1 : 0, pixels,
+                                         static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,275 @@
+"""Python binding of libflashdec.so (ctypes): argument marshalling only.
+
+Every step of the decode path runs in the library's CUDA kernels; this module only converts
+Python / torch arguments into the C ABI of include/flashdec.h and include/flashdec_ops.h.
+There is no fallback: if the library is missing or the device is not an sm_103 GPU, calls
+raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+_LIB = None
+
+FD_OK = 0
+STATUS = {0: "FD_OK", 1: "FD_ERR_INVALID_ARG", 2: "FD_ERR_CONFIG", 3: "FD_ERR_OOM",
+          4: "FD_ERR_CUDA", 5: "FD_ERR_STATE", 6: "FD_ERR_DEVICE_TIMEOUT",
+          7: "FD_ERR_UNSUPPORTED"}
+DTYPE_F32, DTYPE_BF16, DTYPE_U8 = 0, 1, 2
+EPI_F32, EPI_RESID, EPI_GELU, EPI_TUP = 0, 1, 2, 3
+
+
+class FdError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        super().__init__(f"{what}: {STATUS.get(code, code)}")
+        self.code = code
+
+
+class fd_config(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "latent_channels", "latent_h", "latent_w", "patch", "hidden", "heads", "kv_groups",
+        "mlp_ratio", "n_blocks", "n_refine", "window", "r_t", "vae_spatial", "out_channels",
+        "out_dtype", "reserved")] + [("norm_eps", ctypes.c_float), ("rope_base", ctypes.c_float)]
+
+
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_F = ctypes.c_float
+_SIGS = {
+    "fd_status_str": (ctypes.c_char_p, [_I]),
+    "fd_weights_blob_elems": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
+    "fd_latent_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
+    "fd_pixels_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
+    "fd_handle_device_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
+    "fd_weights_create": (_I, [ctypes.POINTER(fd_config), _P, ctypes.c_size_t, _I,
+                               ctypes.POINTER(_P)]),
+    "fd_weights_destroy": (_I, [_P]),
+    "fd_create": (_I, [ctypes.POINTER(fd_config), _P, ctypes.POINTER(_P)]),
+    "fd_decode_chunk": (_I, [_P, _P, _P, _P]),
+    "fd_decode_chunks": (_I, [ctypes.POINTER(_P), _I, ctypes.POINTER(_P), ctypes.POINTER(_P),
+                              _P]),
+    "fd_reset": (_I, [_P]),
+    "fd_destroy": (_I, [_P]),
+    "fd_chunk_index": (ctypes.c_int64, [_P]),
+    "fd_sync_status": (_I, [_P]),
+    "fd_debug_read_ring": (_I, [_P, _I, _I, _P, ctypes.c_size_t]),
+    "fd_op_linear": (_I, [_I, _I, _I, _I, _P, _P, _P, _P, _I, _I, _P, _P]),
+    "fd_op_qkv": (_I, [_I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _F, _F,
+                       _P, _P, _P, _I, _I, _P, _P]),
+    "fd_op_attention": (_I, [_I, _I, _I, _P, _P, _P, _I, _I, _P, _P, _P]),
+    "fd_op_kv_append": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _P, _P]),
+    "fd_op_rmsnorm": (_I, [_P, _P, _I, _I, _F, _P, _P]),
+    "fd_op_unshuffle": (_I, [_P, _I, _I, _I, _I, _P, _P]),
+    "fd_op_pixel_head": (_I, [_P, _I, _I, _I, _I, _I, _I, _P, _P]),
+}
+
+
+def lib(build_if_missing: bool = True) -> ctypes.CDLL:
+    """Load libflashdec.so (building it in-tree first if needed)."""
+    global _LIB
+    if _LIB is None:
+        path = _build.LIB
+        if build_if_missing:
+            path = _build.build()
+        if not os.path.exists(path):
+            raise RuntimeError(f"libflashdec.so not built ({path}); run __graft_entry__.build()")
+        L = ctypes.CDLL(path)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _LIB = L
+    return _LIB
+
+
+def _check(code: int, what: str) -> None:
+    if code != FD_OK:
+        raise FdError(code, what)
+
+
+def make_config(cfg) -> fd_config:
+    """fd_config from any object with the decoder's shape attributes (e.g. synth.FDConfig)."""
+    c = fd_config()
+    for n in ("latent_channels", "latent_h", "latent_w", "patch", "hidden", "heads",
+              "kv_groups", "mlp_ratio", "n_blocks", "n_refine", "window", "r_t", "vae_spatial",
+              "out_channels"):
+        setattr(c, n, int(getattr(cfg, n)))
+    c.out_dtype = DTYPE_U8 if getattr(cfg, "out_u8", False) else DTYPE_F32
+    c.reserved = 0
+    c.norm_eps = float(cfg.norm_eps)
+    c.rope_base = float(cfg.rope_base)
+    return c
+
+
+def weight_names(cfg) -> list[str]:
+    """Tensor names in weight-blob order (the order documented in include/flashdec.h)."""
+    blk = ["norm1.g", "qkv.w", "qkv.b", "knorm.g", "vnorm.g", "out.w", "out.b", "norm2.g",
+           "mlp1.w", "mlp1.b", "mlp2.w", "mlp2.b"]
+    names = ["embed.w", "embed.b"]
+    names += [f"blocks.{b}.{n}" for b in range(cfg.n_blocks) for n in blk]
+    names += ["normf.g", "tup.w", "tup.b"]
+    names += [f"refine.{b}.{n}" for b in range(cfg.n_refine) for n in blk]
+    names += ["normh.g", "head1.w", "head1.b", "head2.w", "head2.b"]
+    return names
+
+
+def pack_blob(cfg, weights: dict) -> np.ndarray:
+    """Concatenate a name -> array dict into one fp32 blob in blob order."""
+    return np.concatenate([np.asarray(weights[n], dtype=np.float32).ravel()
+                           for n in weight_names(cfg)])
+
+
+def _stream_ptr(stream) -> int:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return int(getattr(stream, "cuda_stream", stream))
+
+
+def _ptr(x) -> int:
+    if x is None:
+        return 0
+    return int(x.data_ptr()) if hasattr(x, "data_ptr") else int(x)
+
+
+class Weights:
+    """Device copy of the decoder weights (fd_weights_create); shareable by several Decoders."""
+
+    def __init__(self, cfg, blob: np.ndarray):
+        L = lib()
+        self.cfg = make_config(cfg)
+        blob = np.ascontiguousarray(blob)
+        dt = DTYPE_F32 if blob.dtype == np.float32 else DTYPE_BF16
+        if blob.dtype not in (np.float32, np.uint16):
+            raise TypeError("blob must be fp32, or bf16 bits as uint16")
+        out = _P()
+        _check(L.fd_weights_create(ctypes.byref(self.cfg), blob.ctypes.data, blob.nbytes, dt,
+                                   ctypes.byref(out)), "fd_weights_create")
+        self.handle = out
+
+    def close(self) -> None:
+        if getattr(self, "handle", None):
+            _check(lib().fd_weights_destroy(self.handle), "fd_weights_destroy")
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class Decoder:
+    """One decoder stream (fd_create): rolling caches + chunk counter."""
+
+    def __init__(self, cfg, weights: Weights):
+        L = lib()
+        self.cfg = make_config(cfg)
+        self.weights = weights
+        out = _P()
+        _check(L.fd_create(ctypes.byref(self.cfg), weights.handle, ctypes.byref(out)),
+               "fd_create")
+        self.handle = out
+
+    @property
+    def pixels_bytes(self) -> int:
+        return lib().fd_pixels_bytes(ctypes.byref(self.cfg))
+
+    @property
+    def latent_bytes(self) -> int:
+        return lib().fd_latent_bytes(ctypes.byref(self.cfg))
+
+    def decode_chunk(self, latent, pixels, stream=None) -> None:
+        _check(lib().fd_decode_chunk(self.handle, _ptr(latent), _ptr(pixels),
+                                     _stream_ptr(stream)), "fd_decode_chunk")
+
+    def reset(self) -> None:
+        _check(lib().fd_reset(self.handle), "fd_reset")
+
+    def sync_status(self) -> int:
+        return lib().fd_sync_status(self.handle)
+
+    @property
+    def chunk_index(self) -> int:
+        return lib().fd_chunk_index(self.handle)
+
+    def read_ring(self, which: int, layer: int, groups: int, window: int, rows: int):
+        """(K, V) of one layer's ring as bf16 bit arrays [G][W*rows][64]."""
+        n = groups * window * rows * 64
+        buf = np.zeros(2 * n, dtype=np.uint16)
+        _check(lib().fd_debug_read_ring(self.handle, which, layer, buf.ctypes.data, buf.nbytes),
+               "fd_debug_read_ring")
+        return (buf[:n].reshape(groups, window * rows, 64), buf[n:].reshape(groups, window * rows, 64))
+
+    def close(self) -> None:
+        if getattr(self, "handle", None):
+            _check(lib().fd_destroy(self.handle), "fd_destroy")
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def decode_chunks(decoders, latents, pixels, stream=None) -> None:
+    n = len(decoders)
+    hs = (_P * n)(*[d.handle for d in decoders])
+    ls = (_P * n)(*[_ptr(x) for x in latents])
+    ps = (_P * n)(*[_ptr(x) for x in pixels])
+    _check(lib().fd_decode_chunks(hs, n, ls, ps, _stream_ptr(stream)), "fd_decode_chunks")
+
+
+# ------------------------------------------------------------------ kernel-level entry points
+def op_linear(epi, A, W, bias, out, tup_hidden=0, bn=0, err=None, stream=None) -> None:
+    M, K = A.shape
+    N = W.shape[0]
+    _check(lib().fd_op_linear(epi, M, N, K, _ptr(A), _ptr(W), _ptr(bias), _ptr(out),
+                              tup_hidden, bn, _ptr(err), _stream_ptr(stream)), "fd_op_linear")
+
+
+def op_qkv(A, Wqkv, bqkv, knorm_g, vnorm_g, heads, groups, tokens, grid_w, frames_per_chunk,
+           window, t, eps, rope_base, q_out, k_ring, vt_ring, ring_pitch, bn=0, err=None,
+           stream=None) -> None:
+    M, K = A.shape
+    _check(lib().fd_op_qkv(M, K, _ptr(A), _ptr(Wqkv), _ptr(bqkv), _ptr(knorm_g), _ptr(vnorm_g),
+                           heads, groups, tokens, grid_w, frames_per_chunk, window, t, eps,
+                           rope_base, _ptr(q_out), _ptr(k_ring), _ptr(vt_ring), ring_pitch, bn,
+                           _ptr(err), _stream_ptr(stream)), "fd_op_qkv")
+
+
+def op_attention(q, k_ring, vt_ring, heads, groups, ring_pitch, n_keys, out, err=None,
+                 stream=None) -> None:
+    Lq = q.shape[0]
+    _check(lib().fd_op_attention(Lq, heads, groups, _ptr(q), _ptr(k_ring), _ptr(vt_ring),
+                                 ring_pitch, n_keys, _ptr(out), _ptr(err), _stream_ptr(stream)),
+           "fd_op_attention")
+
+
+def op_kv_append(k, v, window, t, ring_pitch, k_ring, vt_ring, stream=None) -> None:
+    G, rows, _ = k.shape
+    _check(lib().fd_op_kv_append(_ptr(k), _ptr(v), G, rows, window, t, ring_pitch, _ptr(k_ring),
+                                 _ptr(vt_ring), _stream_ptr(stream)), "fd_op_kv_append")
+
+
+def op_rmsnorm(h, g, eps, u, stream=None) -> None:
+    M, D = h.shape
+    _check(lib().fd_op_rmsnorm(_ptr(h), _ptr(g), M, D, eps, _ptr(u), _stream_ptr(stream)),
+           "fd_op_rmsnorm")
+
+
+def op_unshuffle(z, p, x0, stream=None) -> None:
+    C, H, W = z.shape
+    _check(lib().fd_op_unshuffle(_ptr(z), C, H, W, p, _ptr(x0), _stream_ptr(stream)),
+           "fd_op_unshuffle")
+
+
+def op_pixel_head(F, frames, grid_h, grid_w, channels, rs, out_dtype, pixels, stream=None) -> None:
+    _check(lib().fd_op_pixel_head(_ptr(F), frames, grid_h, grid_w, channels, rs, out_dtype,
+                                  _ptr(pixels), _stream_ptr(stream)), "fd_op_pixel_head")

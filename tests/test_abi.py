@@ -1,0 +1,70 @@
+"""The C-ABI library builds, loads, and exports every symbol its headers declare; host-only
+calls (sizes, validation, status strings) work without a GPU."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+fdp = pytest.importorskip("paper_2607_14898_gb300.flashdec")
+
+
+def declared_functions():
+    names = []
+    for h in ("flashdec.h", "flashdec_ops.h"):
+        src = open(os.path.join(ROOT, "include", h)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names += re.findall(r"\b(fd_\w+)\s*\(", src)
+    return sorted(set(names))
+
+
+def test_library_exports_every_declared_symbol():
+    L = fdp.lib()
+    names = declared_functions()
+    assert len(names) >= 20
+    for n in names:
+        assert hasattr(L, n), n
+    assert set(names) == set(fdp._SIGS), "binding signatures cover the header exactly"
+
+
+def test_blob_layout_matches_seeded_layout_and_binding_order():
+    L = fdp.lib()
+    for name, cfg in synth.PRESETS.items():
+        c = fdp.make_config(cfg)
+        want = sum(int(np.prod(s)) for _, s, _ in synth.weight_layout(cfg))
+        assert L.fd_weights_blob_elems(ctypes.byref(c)) == want, name
+        assert [n for n, _, _ in synth.weight_layout(cfg)] == fdp.weight_names(cfg)
+
+
+def test_sizes_follow_the_compression_factors():
+    L = fdp.lib()
+    c = fdp.make_config(synth.PRESETS["480p"])
+    assert L.fd_pixels_bytes(ctypes.byref(c)) == 3 * 4 * 480 * 832 * 4
+    assert L.fd_latent_bytes(ctypes.byref(c)) == 16 * 60 * 104 * 4
+    c = fdp.make_config(synth.PRESETS["720p"])
+    assert L.fd_pixels_bytes(ctypes.byref(c)) == 3 * 4 * 720 * 1280
+
+
+@pytest.mark.parametrize("field,value", [("hidden", 320), ("heads", 3), ("kv_groups", 3),
+                                         ("patch", 3), ("window", 0), ("r_t", 0),
+                                         ("n_blocks", 0), ("latent_channels", 1)])
+def test_invalid_configs_rejected(field, value):
+    L = fdp.lib()
+    cfg = synth.PRESETS["small"].replace(**{field: value})
+    assert L.fd_weights_blob_elems(ctypes.byref(fdp.make_config(cfg))) == 0
+
+
+def test_status_strings_and_null_arguments():
+    L = fdp.lib()
+    for code in range(8):
+        assert L.fd_status_str(code)
+    assert L.fd_weights_blob_elems(None) == 0
+    assert L.fd_decode_chunk(None, None, None, None) == 1
+    assert L.fd_reset(None) == 1 and L.fd_destroy(None) == 1
+    out = ctypes.c_void_p()
+    c = fdp.make_config(synth.PRESETS["tiny"])
+    assert L.fd_weights_create(ctypes.byref(c), None, 0, 0, ctypes.byref(out)) == 1

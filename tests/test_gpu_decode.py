@@ -1,0 +1,157 @@
+"""End-to-end parity of fd_decode_chunk (C ABI) with the CPU oracle, chunk by chunk, plus
+properties that hold at any size (determinism, causality, cache indexing)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from helpers import dev, f64, pixel_errors
+
+pytestmark = pytest.mark.gpu
+
+fdp = pytest.importorskip("paper_2607_14898_gb300.flashdec")
+
+# Tolerance on pixels in [-1, 1]: bf16 compute with fp32 accumulation against the fp64 oracle.
+MAX_ABS, MEAN_ABS = 2e-2, 2e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _setup(torch_threads):
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    fdp.lib()
+
+
+def gpu_stream(cfg, w, z, chunks=None, reset_and_repeat=False):
+    chunks = cfg.chunks if chunks is None else chunks
+    W = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    dec = fdp.Decoder(cfg, W)
+    shape = (cfg.out_channels, cfg.r_t, cfg.out_h, cfg.out_w)
+    dt = torch.uint8 if cfg.out_u8 else torch.float32
+    runs = []
+    for _ in range(2 if reset_and_repeat else 1):
+        outs = []
+        for t in range(chunks):
+            pix = torch.empty(shape, dtype=dt, device="cuda")
+            dec.decode_chunk(dev(z[t]), pix)
+            outs.append(pix)
+        torch.cuda.synchronize()
+        assert dec.sync_status() == fdp.FD_OK
+        runs.append([p.cpu() for p in outs])
+        dec.reset()
+    dec.close()
+    W.close()
+    return runs if reset_and_repeat else runs[0]
+
+
+def compare(cfg, got, want, what):
+    for t, (g, o) in enumerate(zip(got, want)):
+        if cfg.out_u8:
+            wc = oracle.quantize_u8(o.float().numpy()).astype(np.int32)
+            gc = g.numpy().astype(np.int32)
+            d = np.abs(gc - wc)
+            assert d.max() <= 3, f"{what} chunk {t}: max code diff {d.max()}"
+            assert d.mean() / 127.5 <= MEAN_ABS, f"{what} chunk {t}: mean {d.mean() / 127.5:.2e}"
+        else:
+            mx, mean = pixel_errors(g, o)
+            assert mx <= MAX_ABS and mean <= MEAN_ABS, \
+                f"{what} chunk {t}: max-abs {mx:.3e} mean-abs {mean:.3e}"
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8"])
+def test_decode_matches_oracle(name):
+    cfg = synth.PRESETS[name]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    want = oracle.decode_stream(cfg, w, z)
+    got = gpu_stream(cfg, w, z)
+    compare(cfg, got, want, name)
+
+
+def test_decode_deterministic_after_reset():
+    cfg = synth.PRESETS["small"]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    a, b = gpu_stream(cfg, w, z, reset_and_repeat=True)
+    for x, y in zip(a, b):
+        assert torch.equal(x, y)
+
+
+def test_decode_causality_on_gpu():
+    """Outputs of chunks < 3 are bit-identical when chunks >= 3 change."""
+    cfg = synth.PRESETS["small"]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    z2 = z.copy()
+    z2[3:] = synth.make_latents(cfg, seed=5)[3:]
+    a, b = gpu_stream(cfg, w, z), gpu_stream(cfg, w, z2)
+    for t in range(3):
+        assert torch.equal(a[t], b[t])
+    assert not torch.equal(a[3], b[3])
+
+
+def test_ring_slots_hold_the_window():
+    """After chunk t, ring slot s of the first backbone layer holds chunk j = s mod W of the
+    last W chunks: the same keys as the oracle's concat(tail) cache, slot by slot."""
+    cfg = synth.PRESETS["small"]  # W = 3, 5 chunks: slots wrap around
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    ref = oracle.StreamingDecoder(cfg, w)
+    Wt = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    dec = fdp.Decoder(cfg, Wt)
+    L, G, Wn = cfg.tokens, cfg.kv_groups, cfg.window
+    for t in range(cfg.chunks):
+        ref.decode_chunk(z[t])
+        pix = torch.empty(3, cfg.r_t, cfg.out_h, cfg.out_w, device="cuda")
+        dec.decode_chunk(dev(z[t]), pix)
+        kbits, vbits = dec.read_ring(0, 0, G, Wn, L)
+        kr = torch.from_numpy(kbits.view(np.int16)).view(torch.bfloat16).double()
+        oracle_k = ref.kB[0]                                   # [G][c L][64], oldest first
+        c = oracle_k.shape[1] // L
+        for i in range(c):
+            j = t - c + 1 + i
+            s = j % Wn
+            got = kr[:, s * L:(s + 1) * L]
+            want = oracle_k[:, i * L:(i + 1) * L]
+            err = float((got - want).abs().max())
+            assert err <= 2e-2 * float(want.abs().max()), (t, j, s, err)
+            # and it is not any other chunk's keys
+            for i2 in range(c):
+                if i2 != i:
+                    other = oracle_k[:, i2 * L:(i2 + 1) * L]
+                    assert float((got - other).abs().max()) > 10 * err
+    dec.close()
+    Wt.close()
+
+
+def test_api_errors():
+    cfg = synth.PRESETS["tiny"]
+    w = synth.make_weights(cfg)
+    Wt = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    dec = fdp.Decoder(cfg, Wt)
+    L = fdp.lib()
+    lat = torch.zeros(16, 8, 8, device="cuda")
+    pix = torch.zeros(3, 1, 64, 64, device="cuda")
+    assert L.fd_decode_chunk(dec.handle, 0, pix.data_ptr(), 0) == 1
+    assert L.fd_decode_chunk(dec.handle, lat.data_ptr() + 4, pix.data_ptr(), 0) == 1
+    bad = fdp.make_config(cfg.replace(hidden=320, heads=5))
+    assert L.fd_weights_blob_elems(bad) == 0
+    other = cfg.replace(window=3)
+    with pytest.raises(fdp.FdError) as e:
+        fdp.Decoder(other, Wt)
+    assert e.value.code == 2
+    # a weights object with live handles cannot be destroyed
+    assert L.fd_weights_destroy(Wt.handle) == 5
+    dec.decode_chunk(lat, pix)
+    assert dec.sync_status() == 0 and dec.chunk_index == 1
+    dec.close()
+    Wt.close()
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name,chunks", [("480p", 5), ("720p", 2)])
+def test_decode_full_size(name, chunks):
+    """The benchmark's own configurations at full size, first chunks (warm-up and, at 480p,
+    the full W = 4 window plus the first eviction)."""
+    cfg = synth.PRESETS[name]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg, chunks=chunks)
+    ref = oracle.StreamingDecoder(cfg, w)
+    want = [ref.decode_chunk(z[t]) for t in range(chunks)]
+    got = gpu_stream(cfg, w, z, chunks=chunks)
+    compare(cfg, got, want, name)

@@ -1,0 +1,261 @@
+"""Per-kernel parity of the CUDA path against the oracle's functions (through the C ABI's
+kernel-level entry points), on identical bf16-exact inputs."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import assert_close_scaled, bf16_values, dev, f64, randn
+
+pytestmark = pytest.mark.gpu
+
+fdp = pytest.importorskip("paper_2607_14898_gb300.flashdec")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    fdp.lib()
+
+
+def err_word():
+    return torch.zeros(1, dtype=torch.int32, device="cuda")
+
+
+def check_err(err):
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0, f"kernel reported error bits {int(err.item())}"
+
+
+def linear_case(M, N, K, seed):
+    A = bf16_values(randn((M, K), seed, 1.0))
+    W = bf16_values(randn((N, K), seed + 1, 1.0 / math.sqrt(K)))
+    b = randn((N,), seed + 2, 0.1)
+    return A, W, b
+
+
+# ------------------------------------------------------------------ tcgen05 GEMM
+@pytest.mark.parametrize("M,N,K,bn", [
+    (130, 256, 256, 128),     # ragged M (2 tiles), one K tile of 4 x 64
+    (64, 192, 16, 64),        # K < 64 (tiny patch-embed), zero-filled K tail
+    (520, 1024, 256, 256),    # 256-wide tiles
+    (1560, 1536, 1024, 128),  # 480p QKV shape: 13 x 12 tiles, persistent (> 1 tile per CTA)
+    (1560, 1024, 4096, 0),    # 480p MLP-down shape, library tile choice
+    (6240, 768, 1024, 0),     # 480p head layer 2 on r_t L tokens
+])
+def test_linear_f32(M, N, K, bn):
+    A, W, b = linear_case(M, N, K, seed=M + N + K)
+    out = torch.zeros(M, N, device="cuda")
+    err = err_word()
+    fdp.op_linear(fdp.EPI_F32, dev(A, torch.bfloat16), dev(W, torch.bfloat16), dev(b), out,
+                  bn=bn, err=err)
+    check_err(err)
+    want = oracle.linear(f64(A), f64(W), f64(b))
+    assert_close_scaled(out, want, 2e-5, "linear f32")
+
+
+def test_linear_resid_gelu_tup():
+    M, N, K, D = 520, 1024, 256, 256
+    A, W, b = linear_case(M, N, K, seed=11)
+    Ad, Wd, bd = dev(A, torch.bfloat16), dev(W, torch.bfloat16), dev(b)
+    want = oracle.linear(f64(A), f64(W), f64(b))
+    err = err_word()
+    # residual: h += A W^T + b
+    h0 = randn((M, N), 99)
+    h = dev(h0)
+    fdp.op_linear(fdp.EPI_RESID, Ad, Wd, bd, h, err=err)
+    check_err(err)
+    assert_close_scaled(h, f64(h0) + want, 2e-5, "residual")
+    # GELU -> bf16
+    g = torch.zeros(M, N, dtype=torch.bfloat16, device="cuda")
+    fdp.op_linear(fdp.EPI_GELU, Ad, Wd, bd, g, err=err)
+    check_err(err)
+    assert_close_scaled(g.float(), oracle.gelu(want), 8e-3, "gelu")
+    # temporal upsampling reshape: column tau*D + d of row l -> row tau*M + l
+    o = torch.zeros(N // D * M, D, device="cuda")
+    fdp.op_linear(fdp.EPI_TUP, Ad, Wd, bd, o, tup_hidden=D, err=err)
+    check_err(err)
+    rt = N // D
+    want_t = want.reshape(M, rt, D).transpose(0, 1).reshape(rt * M, D)
+    assert_close_scaled(o, want_t, 2e-5, "tup")
+
+
+# ------------------------------------------------------------------ fused QKV epilogue
+class Cfg:
+    def __init__(self, **kw):
+        self.__dict__.update(kw)
+
+
+@pytest.mark.parametrize("heads,groups,grid_h,grid_w,fpc,window,t,K", [
+    (4, 2, 10, 13, 4, 3, 5, 256),       # refinement-like: 4 frames per chunk, ragged rows
+    (16, 4, 30, 52, 1, 4, 7, 1024),     # 480p backbone block
+    (24, 3, 3, 5, 1, 8, 130, 1536),     # wide model, long stream (large temporal index)
+])
+def test_qkv_fused(heads, groups, grid_h, grid_w, fpc, window, t, K):
+    dh, eps, base = 64, 1e-6, 10000.0
+    tokens = grid_h * grid_w
+    M = fpc * tokens
+    N = (heads + 2 * groups) * dh
+    A, W, b = linear_case(M, N, K, seed=heads * 7 + t)
+    kg = bf16_values(1 + randn((dh,), 5, 0.1))
+    vg = bf16_values(1 + randn((dh,), 6, 0.1))
+    pitch = -(-window * M // 128) * 128
+    q_out = torch.zeros(M, heads * dh, dtype=torch.bfloat16, device="cuda")
+    k_ring = torch.zeros(groups, pitch, dh, dtype=torch.bfloat16, device="cuda")
+    vt_ring = torch.zeros(groups, dh, pitch, dtype=torch.bfloat16, device="cuda")
+    err = err_word()
+    fdp.op_qkv(dev(A, torch.bfloat16), dev(W, torch.bfloat16), dev(b), dev(kg), dev(vg), heads,
+               groups, tokens, grid_w, fpc, window, t, eps, base, q_out, k_ring, vt_ring, pitch,
+               err=err)
+    check_err(err)
+    # oracle: Linear, KV-norm, 3D-RoPE at (t*fpc + row // tokens, y, x)
+    qkv = oracle.linear(f64(A), f64(W), f64(b))
+    q = qkv[:, :heads * dh].reshape(M, heads, dh).transpose(0, 1)
+    k = qkv[:, heads * dh:(heads + groups) * dh].reshape(M, groups, dh).transpose(0, 1)
+    v = qkv[:, (heads + groups) * dh:].reshape(M, groups, dh).transpose(0, 1)
+    k = oracle.rms_norm(k, f64(kg), eps)
+    v = oracle.rms_norm(v, f64(vg), eps)
+    r = torch.arange(M)
+    pos = ((t * fpc + r // tokens).double(), ((r % tokens) // grid_w).double(),
+           ((r % tokens) % grid_w).double())
+    q = oracle.rope(q, *pos, base)
+    k = oracle.rope(k, *pos, base)
+    assert_close_scaled(q_out.float().reshape(M, heads, dh).transpose(0, 1), q, 1e-2, "Q")
+    slot = t % window
+    kr = k_ring.float()[:, slot * M:(slot + 1) * M]
+    vr = vt_ring.float()[:, :, slot * M:(slot + 1) * M].transpose(1, 2)
+    assert_close_scaled(kr, k, 1e-2, "K ring slot")
+    assert_close_scaled(vr, v, 1e-2, "V ring slot")
+    # nothing outside the slot was written
+    mask = torch.ones(pitch, dtype=torch.bool)
+    mask[slot * M:(slot + 1) * M] = False
+    assert float(k_ring.float()[:, mask].abs().max()) == 0.0
+    assert float(vt_ring.float()[:, :, mask].abs().max()) == 0.0
+
+
+# ------------------------------------------------------------------ attention
+def attention_case(Lq, heads, groups, pitch, n_keys, seed, qscale=1.5):
+    dh = 64
+    q = bf16_values(randn((Lq, heads * dh), seed, qscale))
+    k = bf16_values(randn((groups, pitch, dh), seed + 1))
+    v = bf16_values(randn((groups, pitch, dh), seed + 2))
+    # entries past n_keys hold large stale values: they must not leak in
+    k[:, n_keys:] *= 50
+    v[:, n_keys:] *= 50
+    return q, k, v
+
+
+def run_attention(q, k, v, heads, groups, pitch, n_keys):
+    Lq = q.shape[0]
+    out = torch.zeros(Lq, heads * 64, dtype=torch.bfloat16, device="cuda")
+    vt = np.ascontiguousarray(np.transpose(v, (0, 2, 1)))
+    err = err_word()
+    fdp.op_attention(dev(q, torch.bfloat16), dev(k, torch.bfloat16), dev(vt, torch.bfloat16),
+                     heads, groups, pitch, n_keys, out, err=err)
+    check_err(err)
+    return out.float().cpu()
+
+
+@pytest.mark.parametrize("Lq,heads,groups,n_keys", [
+    (520, 4, 2, 520),       # one chunk, ragged query tail
+    (520, 4, 2, 1300),      # ragged last key block
+    (130, 4, 1, 390),       # multi-query (G = 1)
+    (128, 4, 4, 128),       # MHA (G = N), exactly one block
+    (64, 2, 1, 1),          # a single key
+])
+def test_attention_small(Lq, heads, groups, n_keys):
+    pitch = max(128, -(-n_keys // 128) * 128 + 128)
+    q, k, v = attention_case(Lq, heads, groups, pitch, n_keys, seed=Lq + n_keys)
+    got = run_attention(q, k, v, heads, groups, pitch, n_keys)
+    qh = f64(q).reshape(Lq, heads, 64).transpose(0, 1)
+    want = oracle.attention(qh, f64(k)[:, :n_keys], f64(v)[:, :n_keys])
+    assert_close_scaled(got.reshape(Lq, heads, 64).transpose(0, 1), want, 1.5e-2, "attention")
+
+
+@pytest.mark.parametrize("Lq,heads,groups,n_keys", [
+    (6240, 16, 4, 24960),   # 480p refinement, steady state (4 chunks x 4 frames x 1560)
+    (3600, 16, 4, 14400),   # 720p backbone, steady state
+])
+def test_attention_full_size_sampled(Lq, heads, groups, n_keys):
+    pitch = -(-n_keys // 128) * 128
+    q, k, v = attention_case(Lq, heads, groups, pitch, n_keys, seed=7, qscale=1.0)
+    got = run_attention(q, k, v, heads, groups, pitch, n_keys)
+    rows = np.random.default_rng(0).choice(Lq, 48, replace=False)
+    rows = np.concatenate([rows, [0, Lq - 1]])
+    qh = f64(q[rows]).reshape(len(rows), heads, 64).transpose(0, 1)
+    want = oracle.attention(qh, f64(k)[:, :n_keys], f64(v)[:, :n_keys])
+    assert_close_scaled(got[rows].reshape(len(rows), heads, 64).transpose(0, 1), want, 1.5e-2,
+                        "attention sampled rows")
+
+
+# ------------------------------------------------------------------ cache append (bit-exact)
+def test_kv_append_ring_indexing_bit_exact():
+    """After appending chunk t, ring slot s holds chunk j with j = s mod W, t-W < j <= t, bit
+    for bit equal to the bf16 (nearest-even) rounding of its fp32 K / V."""
+    G, rows, W, dh = 3, 200, 3, 64
+    pitch = -(-W * rows // 128) * 128
+    k_ring = torch.zeros(G, pitch, dh, dtype=torch.bfloat16, device="cuda")
+    vt_ring = torch.zeros(G, dh, pitch, dtype=torch.bfloat16, device="cuda")
+    chunks = []
+    for t in range(7):
+        k = randn((G, rows, dh), 100 + t)
+        v = randn((G, rows, dh), 200 + t)
+        chunks.append((k, v))
+        fdp.op_kv_append(dev(k), dev(v), W, t, pitch, k_ring, vt_ring)
+        torch.cuda.synchronize()
+        kr = k_ring.view(torch.int16).cpu().numpy()
+        vr = vt_ring.view(torch.int16).cpu().numpy()
+        for j in range(max(0, t - W + 1), t + 1):
+            s = j % W
+            kb = torch.from_numpy(chunks[j][0]).to(torch.bfloat16).view(torch.int16).numpy()
+            vb = torch.from_numpy(chunks[j][1]).to(torch.bfloat16).view(torch.int16).numpy()
+            assert np.array_equal(kr[:, s * rows:(s + 1) * rows], kb), (t, j)
+            assert np.array_equal(vr[:, :, s * rows:(s + 1) * rows], vb.transpose(0, 2, 1)), (t, j)
+        assert not kr[:, W * rows:].any()   # padding rows never written
+
+
+# ------------------------------------------------------------------ RMSNorm, unshuffle, head
+def test_rmsnorm():
+    M, D = 1560, 1024
+    h = randn((M, D), 3, 2.0)
+    g = bf16_values(1 + randn((D,), 4, 0.02))
+    u = torch.zeros(M, D, dtype=torch.bfloat16, device="cuda")
+    fdp.op_rmsnorm(dev(h), dev(g), 1e-6, u)
+    torch.cuda.synchronize()
+    assert_close_scaled(u.float(), oracle.rms_norm(f64(h), f64(g), 1e-6), 8e-3, "rmsnorm")
+
+
+@pytest.mark.parametrize("C,H,W,p", [(16, 60, 104, 2), (16, 8, 8, 1)])
+def test_unshuffle_bit_exact(C, H, W, p):
+    z = randn((C, H, W), 8)
+    x0 = torch.zeros((H // p) * (W // p), C * p * p, dtype=torch.bfloat16, device="cuda")
+    fdp.op_unshuffle(dev(z), p, x0)
+    torch.cuda.synchronize()
+    want = oracle.pixel_unshuffle(torch.from_numpy(z), p).to(torch.bfloat16)
+    assert torch.equal(x0.cpu().view(torch.int16), want.view(torch.int16))
+
+
+@pytest.mark.parametrize("frames,gh,gw,rs,u8", [(4, 30, 52, 16, False), (4, 45, 80, 16, True),
+                                                (1, 8, 8, 8, False), (2, 3, 5, 8, True)])
+def test_pixel_head_bit_exact(frames, gh, gw, rs, u8):
+    C = 3
+    L = gh * gw
+    F = randn((frames * L, C * rs * rs), 9, 0.7)
+    # exact quantisation ties, the clamp limits, out-of-range values and NaN
+    special = np.array([-1.0, 1.0, 0.0, 2.5, -7.0, np.nan, 1 / 255.0 - 1.0,
+                        np.float32(0.5) / np.float32(127.5) - 1.0], dtype=np.float32)
+    F.reshape(-1)[:special.size] = special
+    out = torch.zeros(C, frames, gh * rs, gw * rs, dtype=torch.uint8 if u8 else torch.float32,
+                      device="cuda")
+    fdp.op_pixel_head(dev(F), frames, gh, gw, C, rs, fdp.DTYPE_U8 if u8 else fdp.DTYPE_F32, out)
+    torch.cuda.synchronize()
+    pix = oracle.pixel_shuffle(torch.from_numpy(F).double(), frames, gh, gw, C, rs)
+    if u8:
+        want = oracle.quantize_u8(pix.float().numpy())
+        assert np.array_equal(out.cpu().numpy(), want)
+    else:
+        pf = pix.float().numpy()
+        want = np.clip(np.where(np.isnan(pf), -1.0, pf), -1, 1).astype(np.float32)
+        assert np.array_equal(out.cpu().numpy(), want)
