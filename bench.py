@@ -1,0 +1,469 @@
+#!/usr/bin/env python
+"""Streaming-decode benchmark of the GB300 FlashDecoder library.
+
+One step = one 480p stream of 16 latent chunks decoded through the C ABI (fd_reset, then 16 x
+fd_decode_chunk), i.e. 64 output frames (r_t = 4 per chunk), the paper's FPS definition: total
+decoded frames / total decode time (Sec. 4.1 "Evaluation Metrics"). Inputs are synthetic,
+seeded latents shaped like Wan2.1 480p latents (16 x 60 x 104, PixelUnshuffle 2 -> 1560 tokens)
+and random-init bf16 weights of the 24-block, D = 1024 decoder; they are resident in HBM
+before the timed region. The weights alone (585 MB) exceed L2 (129 MB) and are re-read every
+chunk, so no L2 flush is needed between steps.
+
+Prints one JSON line (rank 0). --impl reference times the CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decoded frames/s and p50 per-chunk latency at 480p/720p; % bf16 TC peak"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="480p")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-secondary", action="store_true", help="skip the 720p line")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
+            p = json.load(fh)
+        return p["bf16_tflops"], p["bf16_tflops_sustained"], p["hbm_gbs"], "measured"
+    except Exception:
+        return 1900.0, 1700.0, 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu = gpu_id
+        self.proc = None
+        self.file = None
+
+    def __enter__(self):
+        try:
+            self.file = tempfile.TemporaryFile(mode="w+")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None:
+            return None
+        self.file.seek(0)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.file:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def source_hash(*names: str) -> str:
+    h = hashlib.sha256()
+    for n in names:
+        with open(os.path.join(ROOT, "paper_2607_14898_gb300", "csrc", n), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(kernel_file: str, workload: str):
+    """DRAM bytes per launch of a kernel from the committed ncu summary, if the kernel source
+    has not changed since the counters were taken (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    cur = source_hash(kernel_file)
+    with open(path) as fh:
+        for line in fh:
+            f = line.split()
+            if len(f) >= 4 and f[0] == kernel_file and f[1] == workload and f[2] == cur:
+                return float(f[3])
+    return None
+
+
+# ---------------------------------------------------------------------------------- GPU arm
+def run_ours(args, rank: int, world: int):
+    import numpy as np
+    import torch
+
+    import synth
+    from paper_2607_14898_gb300 import costs
+    from paper_2607_14898_gb300 import flashdec as fdp
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    def max_over_ranks(x: float) -> float:
+        if dist is None:
+            return x
+        t = torch.tensor([x], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def sum_over_ranks(x: float) -> float:
+        if dist is None:
+            return x
+        t = torch.tensor([x], device="cuda", dtype=torch.float64)
+        dist.all_reduce(t)
+        return float(t.item())
+
+    cfg = synth.PRESETS[args.workload]
+    chunks = cfg.chunks
+    frames_per_step = chunks * cfg.r_t
+    w = synth.make_weights(cfg)
+    blob = fdp.pack_blob(cfg, w)
+    weights = fdp.Weights(cfg, blob)
+    dec = fdp.Decoder(cfg, weights)
+    # replicas: rank r decodes its own stream (latent seed r)
+    z = torch.from_numpy(synth.make_latents(cfg, seed=cfg.latent_seed + rank)).cuda()
+    out_dtype = torch.uint8 if cfg.out_u8 else torch.float32
+    pix = [torch.empty(cfg.out_channels, cfg.r_t, cfg.out_h, cfg.out_w, dtype=out_dtype,
+                       device="cuda") for _ in range(chunks)]
+    stream = torch.cuda.Stream()
+
+    def step(events=None):
+        dec.reset()
+        for t in range(chunks):
+            if events is not None:
+                events[t][0].record(stream)
+            dec.decode_chunk(z[t], pix[t], stream)
+            if events is not None:
+                events[t][1].record(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    torch.cuda.synchronize()
+    if dec.sync_status() != fdp.FD_OK:
+        raise RuntimeError("device error during warm-up")
+
+    # ---------------------------------------------------------------- timed region
+    ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(chunks)]
+          for _ in range(args.steps)]
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    launches0 = dec.launch_count
+    barrier()
+    torch.cuda.synchronize()
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(local).uuid)
+    except Exception:
+        gpu_id = str(local)
+    with ClockSampler(gpu_id) as clocks:
+        with torch.cuda.stream(stream):
+            t0.record(stream)
+            for k in range(args.steps):
+                step(ev[k])
+            t1.record(stream)
+        torch.cuda.synchronize()
+    barrier()
+    gpu_launches = dec.launch_count - launches0
+    ms_total = t0.elapsed_time(t1)
+    ms_max = max_over_ranks(ms_total)
+    frames_all = sum_over_ranks(frames_per_step * args.steps)
+    lat = [ev[k][t][0].elapsed_time(ev[k][t][1]) for k in range(args.steps) for t in range(chunks)]
+    lat_steady = [ev[k][t][0].elapsed_time(ev[k][t][1]) for k in range(args.steps)
+                  for t in range(cfg.window - 1, chunks)]
+    if dec.sync_status() != fdp.FD_OK:
+        raise RuntimeError("device error in the timed region")
+    flops_step = costs.stream_flops(cfg, chunks)
+
+    # ---------------------------------------------------------------- per-kernel profile
+    dec.profile(True)
+    with torch.cuda.stream(stream):
+        for _ in range(args.steps):
+            step()
+    torch.cuda.synchronize()
+    prof = dec.profile_collect()
+    dec.profile(False)
+    kflops = {}
+    for t in range(chunks):
+        for k, v in costs.chunk_flops(cfg, t).items():
+            kflops[k] = kflops.get(k, 0) + v * args.steps
+    kbytes = {}
+    for t in range(chunks):
+        for k, v in costs.chunk_bytes(cfg, t).items():
+            kbytes[k] = kbytes.get(k, 0) + v * args.steps
+    burst, sustained, hbm, peak_src = peaks()
+    kernels = {}
+    for k, (n, ms) in prof.items():
+        if n == 0:
+            continue
+        e = {"launches": n, "ms_total": round(ms, 3), "us_per_launch": round(1e3 * ms / n, 2)}
+        if k in kflops:
+            e["tflops"] = round(kflops[k] / (ms * 1e-3) / 1e12, 1)
+        if k in kbytes:
+            e["gbs"] = round(kbytes[k] / (ms * 1e-3) / 1e9, 1)
+        kernels[k] = e
+    att_ms = prof["attn_backbone"][1] + prof["attn_refine"][1]
+    att_n = prof["attn_backbone"][0] + prof["attn_refine"][0]
+    att_flops = kflops["attn_backbone"] + kflops["attn_refine"]
+    att_tflops = att_flops / (att_ms * 1e-3) / 1e12
+    gemm_kinds = ["embed", "qkv", "out", "mlp1", "mlp2", "tup", "head1", "head2"]
+    gemm_ms = sum(prof[k][1] for k in gemm_kinds)
+    gemm_tflops = sum(kflops[k] for k in gemm_kinds) / (gemm_ms * 1e-3) / 1e12
+    prof_ms_step = sum(ms for _, ms in prof.values()) / args.steps
+
+    # ---------------------------------------------------------------- end to end (host buffers)
+    lat_host = torch.from_numpy(synth.make_latents(cfg, seed=cfg.latent_seed + rank)).pin_memory()
+    pix_host = [torch.empty(pix[0].shape, dtype=out_dtype).pin_memory() for _ in range(chunks)]
+
+    def step_host():
+        dec.reset()
+        for t in range(chunks):
+            dec.decode_chunk_host(lat_host[t], pix_host[t], stream)
+
+    with torch.cuda.stream(stream):
+        step_host()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(args.steps):
+            step_host()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1))
+    latent_bytes = cfg.latent_channels * cfg.latent_h * cfg.latent_w * 4
+    pixel_bytes = pix[0].numel() * pix[0].element_size()
+
+    value = frames_all / (ms_max * 1e-3)
+    line = {
+        "metric": METRIC,
+        "value": round(value, 2),
+        "unit": "frames/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_max / args.steps, 3),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) latents, random-init N(0,0.02) bf16 weights)",
+        "config": {
+            "workload": f"{cfg.name} single stream per GPU: latent 16x{cfg.latent_h}x"
+                        f"{cfg.latent_w}, patch 2 ({cfg.tokens} tokens/chunk), {chunks} chunks "
+                        f"per step, {cfg.n_blocks}+{cfg.n_refine} blocks, D={cfg.hidden}, "
+                        f"{cfg.heads} heads / {cfg.kv_groups} KV groups, W={cfg.window}, r_t="
+                        f"{cfg.r_t}, output {cfg.out_h}x{cfg.out_w} "
+                        f"{'uint8' if cfg.out_u8 else 'fp32'}",
+            "frames_per_step": frames_per_step,
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+            "l2": "no flush: per-chunk working set (585 MB bf16 weights) > 129 MB L2",
+        },
+        "latency_ms": {"p50": round(statistics.median(lat), 3),
+                       "p99": round(sorted(lat)[max(0, int(0.99 * len(lat)) - 1)], 3),
+                       "steady_p50": round(statistics.median(lat_steady), 3),
+                       "steady_frames_per_s": round(cfg.r_t / (statistics.median(lat_steady)
+                                                               * 1e-3), 2)},
+        "tensor_tflops_step": round(flops_step * args.steps / (ms_total * 1e-3) / 1e12, 1),
+        "tensor_frac_step": round(flops_step * args.steps / (ms_total * 1e-3) / 1e12
+                                  / sustained, 3),
+        "clocks": clocks.summary(),
+        "e2e": {"value": round(frames_all / (e2e_ms * 1e-3), 2), "unit": "frames/s",
+                "h2d_bytes_per_step": chunks * latent_bytes,
+                "d2h_bytes_per_step": chunks * pixel_bytes,
+                "call": "fd_decode_chunk_host (pinned host latents / pixels)"},
+        "gpu_launches": int(gpu_launches),
+        "roofline": {"kernel": "attention (attn_kernel, backbone + refinement launches)",
+                     "bound": "tensor", "achieved": round(att_tflops, 1),
+                     "peak": sustained, "unit": "TFLOP/s",
+                     "frac": round(att_tflops / sustained, 3),
+                     "peak_source": f"bf16_tflops_sustained ({peak_src}); kernel timed inside "
+                                    "a long step",
+                     "traffic": ncu_traffic("fd_attn.cu", cfg.name),
+                     "flops_per_launch": round(att_flops / att_n),
+                     "us_per_launch": round(1e3 * att_ms / att_n, 2),
+                     "measured_over": f"{args.steps} profiled steps of the same workload "
+                                      "(CUDA events around each launch on its stream)",
+                     "gemm_tflops": round(gemm_tflops, 1),
+                     "gemm_frac": round(gemm_tflops / sustained, 3),
+                     "profiled_ms_per_step": round(prof_ms_step, 3)},
+        "kernels": kernels,
+    }
+    if rank == 0 and world == 1 and not args.no_secondary and cfg.name == "480p":
+        line["secondary"] = secondary_720p(args, stream, blob)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(cfg, w)
+    dec.close()
+    weights.close()
+    if dist is not None:
+        dist.destroy_process_group()
+    return line
+
+
+def secondary_720p(args, stream, blob):
+    """720p stream (uint8 pixels): frames/s and per-chunk latency, same procedure. The model
+    (and so the weight blob) is the 480p one; only the latent grid differs."""
+    import statistics as st
+
+    import torch
+
+    import synth
+    from paper_2607_14898_gb300 import flashdec as fdp
+
+    cfg = synth.PRESETS["720p"]
+    chunks = 16
+    weights = fdp.Weights(cfg, blob)
+    dec = fdp.Decoder(cfg, weights)
+    z = torch.from_numpy(synth.make_latents(cfg, chunks=chunks)).cuda()
+    pix = [torch.empty(3, cfg.r_t, cfg.out_h, cfg.out_w, dtype=torch.uint8, device="cuda")
+           for _ in range(chunks)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(chunks)]
+
+    def step(record):
+        dec.reset()
+        for t in range(chunks):
+            if record:
+                ev[t][0].record(stream)
+            dec.decode_chunk(z[t], pix[t], stream)
+            if record:
+                ev[t][1].record(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(1, args.warmup)):
+            step(False)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        step(True)
+        b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b)
+    lat = [ev[t][0].elapsed_time(ev[t][1]) for t in range(chunks)]
+    steady = lat[cfg.window - 1:]
+    ok = dec.sync_status() == fdp.FD_OK
+    dec.close()
+    weights.close()
+    return {"workload": f"720p single stream, {chunks} chunks, uint8 pixels",
+            "frames_per_s": round(chunks * cfg.r_t / (ms * 1e-3), 2),
+            "p50_ms": round(st.median(lat), 3), "steady_p50_ms": round(st.median(steady), 3),
+            "p99_ms": round(max(lat), 3), "device_ok": ok}
+
+
+def oracle_chunk_seconds(cfg, w, threads: int) -> float:
+    """Time the CPU oracle decoding chunk 0 of the stream (full model)."""
+    import torch
+
+    import oracle
+    import synth
+    torch.set_num_threads(threads)
+    z = synth.make_latents(cfg, chunks=1)
+    dec = oracle.StreamingDecoder(cfg, w)
+    t = time.perf_counter()
+    dec.decode_chunk(z[0])
+    return time.perf_counter() - t
+
+
+def cpu_baseline(cfg, w):
+    threads = os.cpu_count() or 1
+    sec = oracle_chunk_seconds(cfg, w, threads)
+    return {"value": round(cfg.r_t / sec, 4), "unit": "frames/s", "cores": threads,
+            "kind": "oracle",
+            "sample": f"chunk 0 of the {cfg.name} stream (cache holds 1 chunk), full "
+                      f"{cfg.n_blocks}+{cfg.n_refine}-block model, fp64 PyTorch CPU, "
+                      f"{sec:.1f} s for {cfg.r_t} frames"}
+
+
+# ---------------------------------------------------------------------------- reference arm
+def run_reference(args):
+    import synth
+    cfg = synth.PRESETS[args.workload]
+    w = synth.make_weights(cfg)
+    threads = os.cpu_count() or 1
+    for _ in range(args.warmup):
+        oracle_chunk_seconds(cfg, w, threads)
+    secs = [oracle_chunk_seconds(cfg, w, threads) for _ in range(args.steps)]
+    total = sum(secs)
+    value = cfg.r_t * args.steps / total
+    sample = (f"per step: chunk 0 of the {cfg.name} stream (decoder reset), full "
+              f"{cfg.n_blocks}+{cfg.n_refine}-block model, fp64 PyTorch CPU oracle")
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "frames/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(1e3 * total / args.steps, 1), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{cfg.name} single stream (oracle sample)", "sample": sample},
+        "cpu_baseline": {"value": round(value, 4), "unit": "frames/s", "cores": threads,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "frames/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        print(json.dumps(run_reference(args)), flush=True)
+        return
+    line = run_ours(args, rank, world)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -122,7 +122,7 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out);
 /* Decode chunk t (Algorithm 1, one loop iteration) and advance t.
  * latent_dev: device fp32 [C'][H'][W'] (fd_latent_bytes), 16-byte aligned.
  * pixels_dev: device buffer of fd_pixels_bytes, 16-byte aligned, written with clamped
- *             pixels in [-1, 1] (fp32) or their uint8 codes
+ *             pixels in [-1, 1] (fp32; NaN -> -1) or their uint8 codes
  *             q = round_half_even((clamp(x,-1,1) + 1) * 127.5) (uint8; NaN -> 0).
  * Both are used stream-ordered on `stream`; the call returns after enqueueing (no host
  * synchronisation). Attention at chunk t covers the min(t+1, W) most recent chunks. */
@@ -133,9 +133,17 @@ fd_status fd_decode_chunk(fd_handle h, const float* latent_dev, void* pixels_dev
 fd_status fd_decode_chunks(fd_handle* hs, int n, const float* const* latents_dev,
                            void* const* pixels_dev, void* stream);
 
+/* Like fd_decode_chunk, with the latent and the pixels in HOST memory (pinned for
+ * asynchronous copies): the latent is copied into a library-owned device buffer, decoded, and
+ * the pixels copied back, all stream-ordered on `stream`. The host buffers must stay valid
+ * until the stream reaches the end of the copy-back. */
+fd_status fd_decode_chunk_host(fd_handle h, const float* latent_host, void* pixels_host,
+                               void* stream);
+
 /* Restart the stream: t = 0 and the caches logically empty (their memory is not cleared;
  * stale entries are never read because attention at chunk t reads only chunks <= t).
- * Clears the error state. Synchronous with respect to the handle's previous work. */
+ * Clears the error state. Stream-ordered: enqueued on the stream of the handle's last decode
+ * call, so the next decode on that stream starts from chunk 0 without a host wait. */
 fd_status fd_reset(fd_handle h);
 
 /* Free everything the handle owns (after synchronising its last stream). */
@@ -150,6 +158,24 @@ fd_status fd_sync_status(fd_handle h);
 
 /* Static description of a status code. */
 const char* fd_status_str(fd_status s);
+
+/* Kernel kinds of the decode path, for the per-kernel profile. */
+typedef enum {
+  FD_K_UNSHUFFLE = 0, FD_K_EMBED = 1, FD_K_RMSNORM = 2, FD_K_QKV = 3, FD_K_ATTN_B = 4,
+  FD_K_ATTN_R = 5, FD_K_OUT = 6, FD_K_MLP1 = 7, FD_K_MLP2 = 8, FD_K_TUP = 9, FD_K_HEAD1 = 10,
+  FD_K_HEAD2 = 11, FD_K_PIXEL = 12, FD_K_ADVANCE = 13, FD_K_COUNT = 14
+} fd_kernel_kind;
+
+/* Per-kernel profile (tracing): while enabled, every kernel the handle launches is bracketed
+ * by CUDA events on its stream. fd_profile_collect synchronises, adds each kind's launch count
+ * and device milliseconds into launches[FD_K_COUNT] / ms[FD_K_COUNT] (caller zeroes them) and
+ * clears the recorded events. Attention is split into backbone (FD_K_ATTN_B) and refinement
+ * (FD_K_ATTN_R) launches. */
+fd_status fd_profile_enable(fd_handle h, int enable);
+fd_status fd_profile_collect(fd_handle h, int64_t* launches, double* ms);
+
+/* Number of kernels this handle has launched since fd_create. */
+int64_t fd_launch_count(fd_handle h);
 
 /* Copy layer `layer` of the backbone (which = 0) or refinement (which = 1) ring into host
  * memory: K as [G][W * rows][64] bf16 bits, then V as [G][W * rows][64] bf16 bits (rows =

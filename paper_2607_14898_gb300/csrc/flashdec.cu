@@ -214,6 +214,15 @@ struct fd_handle_s {
   std::vector<Ring> ringB, ringR;
   // A-operand / Q descriptors
   CUtensorMap tm_x0, tm_uB, tm_uR, tm_oB, tm_oR, tm_hidB, tm_hidR, tm_hidH, tm_qB, tm_qR;
+  // host-buffer decode: library-owned device copies of the latent and the pixels
+  float* latent_buf = nullptr;
+  void* pixel_buf = nullptr;
+  // tracing: launch count and, while profiling, one event pair per launch
+  int64_t launches = 0;
+  bool profiling = false;
+  std::vector<cudaEvent_t> ev_start, ev_stop;
+  std::vector<int> ev_kind;
+  size_t ev_used = 0;
 };
 
 namespace {
@@ -236,25 +245,60 @@ void fill_rope(fd::QkvEpi& q, float base) {
 
 fd_status launch_ok(cudaError_t e) { return e == cudaSuccess ? FD_OK : FD_ERR_CUDA; }
 
-fd_status run_linear(const CUtensorMap& tmA, const Linear& lin, int M, fd::GemmParams p,
-                     cudaStream_t s) {
+// Launch one kernel of the decode path: counts it and, while profiling, brackets it with a
+// pair of CUDA events on its stream.
+template <class Fn>
+fd_status traced(fd_handle h, int kind, cudaStream_t s, Fn&& fn) {
+  size_t slot = 0;
+  if (h->profiling) {
+    slot = h->ev_used++;
+    if (slot == h->ev_start.size()) {
+      cudaEvent_t a, b;
+      if (cudaEventCreate(&a) != cudaSuccess) return FD_ERR_CUDA;
+      if (cudaEventCreate(&b) != cudaSuccess) {
+        cudaEventDestroy(a);
+        return FD_ERR_CUDA;
+      }
+      h->ev_start.push_back(a);
+      h->ev_stop.push_back(b);
+      h->ev_kind.push_back(kind);
+    }
+    h->ev_kind[slot] = kind;
+    if (cudaEventRecord(h->ev_start[slot], s) != cudaSuccess) return FD_ERR_CUDA;
+  }
+  const fd_status st = launch_ok(fn());
+  if (st != FD_OK) return st;
+  h->launches++;
+  if (h->profiling && cudaEventRecord(h->ev_stop[slot], s) != cudaSuccess) return FD_ERR_CUDA;
+  return FD_OK;
+}
+
+fd_status run_linear(fd_handle h, int kind, const CUtensorMap& tmA, const Linear& lin, int M,
+                     fd::GemmParams p, cudaStream_t s) {
   p.M = M;
   p.N = lin.N;
   p.K = lin.K;
   p.bias = lin.b;
-  return launch_ok(fd::launch_gemm(tmA, lin.tm, p, lin.bn, num_sms(), s));
+  p.err = h->state + 1;
+  return traced(h, kind, s, [&] { return fd::launch_gemm(tmA, lin.tm, p, lin.bn, num_sms(), s); });
+}
+
+fd_status run_norm(fd_handle h, const float* x, const float* g, int rows, cudaStream_t s) {
+  const int D = h->d.D;
+  const float eps = h->cfg.norm_eps;
+  __nv_bfloat16* u = h->u;
+  return traced(h, FD_K_RMSNORM, s, [&] { return fd::launch_rmsnorm(x, g, rows, D, eps, u, s); });
 }
 
 // one Transformer block (Sec. 3.2) on `rows` tokens of residual stream hbuf, with ring r
 fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int rows, int fpc,
                     int pitch, const CUtensorMap& tm_u, const CUtensorMap& tm_q,
-                    const CUtensorMap& tm_o, const CUtensorMap& tm_hid, cudaStream_t s) {
+                    const CUtensorMap& tm_o, const CUtensorMap& tm_hid, bool refine,
+                    cudaStream_t s) {
   const Dims& d = h->d;
   fd_status st;
-  if ((st = launch_ok(fd::launch_rmsnorm(hbuf, lw.g1, rows, d.D, h->cfg.norm_eps, h->u, s))))
-    return st;
+  if ((st = run_norm(h, hbuf, lw.g1, rows, s))) return st;
   fd::GemmParams p{};
-  p.err = h->state + 1;
   p.epi = fd::EPI_QKV;
   fd::QkvEpi& q = p.qkv;
   q.heads = d.N; q.groups = d.G; q.knorm_g = lw.kg; q.vnorm_g = lw.vg; q.q_out = h->q;
@@ -262,81 +306,80 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
   q.frames_per_chunk = fpc; q.window = d.Wn; q.step_dev = h->state; q.step_host = 0;
   q.eps = h->cfg.norm_eps;
   fill_rope(q, h->cfg.rope_base);
-  if ((st = run_linear(tm_u, lw.qkv, rows, p, s))) return st;
+  if ((st = run_linear(h, FD_K_QKV, tm_u, lw.qkv, rows, p, s))) return st;
 
   fd::AttnParams a{};
   a.Lq = rows; a.heads = d.N; a.groups = d.G; a.ring_pitch = pitch; a.rows_per_chunk = rows;
   a.window = d.Wn; a.step_dev = h->state; a.n_keys_host = 0; a.out = h->o;
   a.ld_out = d.N * kHeadDim; a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
   a.err = h->state + 1;
-  if ((st = launch_ok(fd::launch_attention(tm_q, r.tm_k, r.tm_vt, a, s)))) return st;
+  if ((st = traced(h, refine ? FD_K_ATTN_R : FD_K_ATTN_B, s,
+                   [&] { return fd::launch_attention(tm_q, r.tm_k, r.tm_vt, a, s); })))
+    return st;
 
   fd::GemmParams po{};
-  po.err = h->state + 1;
   po.epi = fd::EPI_RESID;
   po.out_f32 = hbuf;
   po.ld_out = d.D;
-  if ((st = run_linear(tm_o, lw.out, rows, po, s))) return st;
-  if ((st = launch_ok(fd::launch_rmsnorm(hbuf, lw.g2, rows, d.D, h->cfg.norm_eps, h->u, s))))
-    return st;
+  if ((st = run_linear(h, FD_K_OUT, tm_o, lw.out, rows, po, s))) return st;
+  if ((st = run_norm(h, hbuf, lw.g2, rows, s))) return st;
   fd::GemmParams p1{};
-  p1.err = h->state + 1;
   p1.epi = fd::EPI_GELU;
   p1.out_bf16 = h->hid;
   p1.ld_out = d.Mr * d.D;
-  if ((st = run_linear(tm_u, lw.mlp1, rows, p1, s))) return st;
-  return run_linear(tm_hid, lw.mlp2, rows, po, s);
+  if ((st = run_linear(h, FD_K_MLP1, tm_u, lw.mlp1, rows, p1, s))) return st;
+  return run_linear(h, FD_K_MLP2, tm_hid, lw.mlp2, rows, po, s);
 }
 
 fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_t s) {
   const Dims& d = h->d;
   const fd_weights w = h->w;
   fd_status st;
-  if ((st = launch_ok(fd::launch_unshuffle(latent, d.C, d.H, d.W, d.p, h->x0, s)))) return st;
+  __nv_bfloat16* x0 = h->x0;
+  if ((st = traced(h, FD_K_UNSHUFFLE, s,
+                   [&] { return fd::launch_unshuffle(latent, d.C, d.H, d.W, d.p, x0, s); })))
+    return st;
   fd::GemmParams pe{};
-  pe.err = h->state + 1;
   pe.epi = fd::EPI_F32;
   pe.out_f32 = h->h;
   pe.ld_out = d.D;
-  if ((st = run_linear(h->tm_x0, w->embed, d.L, pe, s))) return st;
+  if ((st = run_linear(h, FD_K_EMBED, h->tm_x0, w->embed, d.L, pe, s))) return st;
   for (int b = 0; b < d.nb; ++b)
     if ((st = run_block(h, w->blocks[b], h->ringB[b], h->h, d.L, 1, h->pitchB, h->tm_uB, h->tm_qB,
-                        h->tm_oB, h->tm_hidB, s)))
+                        h->tm_oB, h->tm_hidB, false, s)))
       return st;
   // temporal upsampling: RMSNorm, Linear D -> r_t D, channel block tau -> refined frame tau
-  if ((st = launch_ok(fd::launch_rmsnorm(h->h, w->g_f, d.L, d.D, h->cfg.norm_eps, h->u, s))))
-    return st;
+  if ((st = run_norm(h, h->h, w->g_f, d.L, s))) return st;
   fd::GemmParams pt{};
-  pt.err = h->state + 1;
   pt.epi = fd::EPI_TUP;
   pt.out_f32 = h->hf;
   pt.tup_tokens = d.L;
   pt.tup_hidden = d.D;
-  if ((st = run_linear(h->tm_uB, w->tup, d.L, pt, s))) return st;
+  if ((st = run_linear(h, FD_K_TUP, h->tm_uB, w->tup, d.L, pt, s))) return st;
   const int R = d.rt * d.L;
   for (int b = 0; b < d.nr; ++b)
     if ((st = run_block(h, w->refine[b], h->ringR[b], h->hf, R, d.rt, h->pitchR, h->tm_uR,
-                        h->tm_qR, h->tm_oR, h->tm_hidR, s)))
+                        h->tm_qR, h->tm_oR, h->tm_hidR, true, s)))
       return st;
   // spatial upsampling head: RMSNorm, Linear D->D + GELU, Linear D -> C r_s^2, PixelShuffle
-  if ((st = launch_ok(fd::launch_rmsnorm(h->hf, w->g_h, R, d.D, h->cfg.norm_eps, h->u, s))))
-    return st;
+  if ((st = run_norm(h, h->hf, w->g_h, R, s))) return st;
   fd::GemmParams ph{};
-  ph.err = h->state + 1;
   ph.epi = fd::EPI_GELU;
   ph.out_bf16 = h->hid;
   ph.ld_out = d.D;
-  if ((st = run_linear(h->tm_uR, w->head1, R, ph, s))) return st;
+  if ((st = run_linear(h, FD_K_HEAD1, h->tm_uR, w->head1, R, ph, s))) return st;
   fd::GemmParams pf{};
-  pf.err = h->state + 1;
   pf.epi = fd::EPI_F32;
   pf.out_f32 = h->F;
   pf.ld_out = d.head_out;
-  if ((st = run_linear(h->tm_hidH, w->head2, R, pf, s))) return st;
-  if ((st = launch_ok(fd::launch_pixel_head(h->F, d.rt, d.gh, d.gw, d.Cout, d.rs, d.u8 ? 1 : 0,
-                                            pixels, s))))
+  if ((st = run_linear(h, FD_K_HEAD2, h->tm_hidH, w->head2, R, pf, s))) return st;
+  const float* F = h->F;
+  if ((st = traced(h, FD_K_PIXEL, s, [&] {
+         return fd::launch_pixel_head(F, d.rt, d.gh, d.gw, d.Cout, d.rs, d.u8 ? 1 : 0, pixels, s);
+       })))
     return st;
-  return launch_ok(fd::launch_advance(h->state, s));
+  int* state = h->state;
+  return traced(h, FD_K_ADVANCE, s, [&] { return fd::launch_advance(state, s); });
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -379,12 +422,12 @@ size_t fd_pixels_bytes(const fd_config* cfg) {
   return static_cast<size_t>(d.Cout) * d.rt * d.gh * d.rs * d.gw * d.rs * (d.u8 ? 1 : 4);
 }
 
-static size_t handle_layout(const Dims& d, size_t* off /* 12 offsets */, int* pitchB,
+static size_t handle_layout(const Dims& d, size_t* off /* 14 offsets */, int* pitchB,
                             int* pitchR) {
   const size_t R = static_cast<size_t>(d.rt) * d.L;
   *pitchB = static_cast<int>(align_up(static_cast<size_t>(d.Wn) * d.L, 128));
   *pitchR = static_cast<int>(align_up(static_cast<size_t>(d.Wn) * R, 128));
-  size_t sizes[11] = {
+  size_t sizes[13] = {
       16,                                              // state
       static_cast<size_t>(d.L) * d.cin * 2,            // x0
       R * d.D * 2,                                     // u
@@ -396,19 +439,21 @@ static size_t handle_layout(const Dims& d, size_t* off /* 12 offsets */, int* pi
       R * d.head_out * 4,                              // F
       static_cast<size_t>(d.nb) * 2 * d.G * *pitchB * kHeadDim * 2,  // backbone rings
       static_cast<size_t>(d.nr) * 2 * d.G * *pitchR * kHeadDim * 2,  // refinement rings
+      static_cast<size_t>(d.C) * d.H * d.W * 4,                      // latent (host decode)
+      static_cast<size_t>(d.Cout) * d.rt * d.gh * d.rs * d.gw * d.rs * (d.u8 ? 1 : 4),  // pixels
   };
   size_t cur = 0;
-  for (int i = 0; i < 11; ++i) {
+  for (int i = 0; i < 13; ++i) {
     off[i] = cur;
     cur = align_up(cur + sizes[i], 1024);
   }
-  off[11] = cur;
+  off[13] = cur;
   return cur;
 }
 
 size_t fd_handle_device_bytes(const fd_config* cfg) {
   if (!valid_cfg(cfg)) return 0;
-  size_t off[12];
+  size_t off[14];
   int a, b;
   return handle_layout(dims_of(cfg), off, &a, &b);
 }
@@ -535,7 +580,7 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   h->d = dims_of(cfg);
   h->w = w;
   const Dims& d = h->d;
-  size_t off[12];
+  size_t off[14];
   h->arena_bytes = handle_layout(d, off, &h->pitchB, &h->pitchR);
   if (cudaMalloc(&h->arena, h->arena_bytes) != cudaSuccess) {
     delete h;
@@ -551,6 +596,8 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   h->h = reinterpret_cast<float*>(b + off[6]);
   h->hf = reinterpret_cast<float*>(b + off[7]);
   h->F = reinterpret_cast<float*>(b + off[8]);
+  h->latent_buf = reinterpret_cast<float*>(b + off[11]);
+  h->pixel_buf = b + off[12];
   const size_t ringB_elems = static_cast<size_t>(d.G) * h->pitchB * kHeadDim;
   const size_t ringR_elems = static_cast<size_t>(d.G) * h->pitchR * kHeadDim;
   h->ringB.resize(d.nb);
@@ -625,11 +672,29 @@ fd_status fd_decode_chunks(fd_handle* hs, int n, const float* const* latents_dev
   return FD_OK;
 }
 
+fd_status fd_decode_chunk_host(fd_handle h, const float* latent_host, void* pixels_host,
+                               void* stream) {
+  if (h == nullptr || latent_host == nullptr || pixels_host == nullptr) return FD_ERR_INVALID_ARG;
+  if (h->error) return FD_ERR_STATE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t lb = fd_latent_bytes(&h->cfg), pb = fd_pixels_bytes(&h->cfg);
+  if (cudaMemcpyAsync(h->latent_buf, latent_host, lb, cudaMemcpyHostToDevice, s) != cudaSuccess) {
+    h->error = true;
+    return FD_ERR_CUDA;
+  }
+  fd_status st = fd_decode_chunk(h, h->latent_buf, h->pixel_buf, stream);
+  if (st != FD_OK) return st;
+  if (cudaMemcpyAsync(pixels_host, h->pixel_buf, pb, cudaMemcpyDeviceToHost, s) != cudaSuccess) {
+    h->error = true;
+    return FD_ERR_CUDA;
+  }
+  return FD_OK;
+}
+
 fd_status fd_reset(fd_handle h) {
   if (h == nullptr) return FD_ERR_INVALID_ARG;
-  if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) cudaGetLastError();
-  if (cudaMemset(h->state, 0, 2 * sizeof(int)) != cudaSuccess) return FD_ERR_CUDA;
-  if (cudaDeviceSynchronize() != cudaSuccess) return FD_ERR_CUDA;
+  if (cudaMemsetAsync(h->state, 0, 2 * sizeof(int), h->last_stream) != cudaSuccess)
+    return FD_ERR_CUDA;
   h->t_host = 0;
   h->error = false;
   return FD_OK;
@@ -638,11 +703,39 @@ fd_status fd_reset(fd_handle h) {
 fd_status fd_destroy(fd_handle h) {
   if (h == nullptr) return FD_ERR_INVALID_ARG;
   cudaStreamSynchronize(h->last_stream);
+  for (size_t i = 0; i < h->ev_start.size(); ++i) {
+    cudaEventDestroy(h->ev_start[i]);
+    cudaEventDestroy(h->ev_stop[i]);
+  }
   cudaFree(h->arena);
   if (h->w) h->w->live_handles--;
   delete h;
   return FD_OK;
 }
+
+fd_status fd_profile_enable(fd_handle h, int enable) {
+  if (h == nullptr) return FD_ERR_INVALID_ARG;
+  h->profiling = enable != 0;
+  return FD_OK;
+}
+
+fd_status fd_profile_collect(fd_handle h, int64_t* launches, double* ms) {
+  if (h == nullptr || launches == nullptr || ms == nullptr) return FD_ERR_INVALID_ARG;
+  for (size_t i = 0; i < h->ev_used; ++i) {
+    if (cudaEventSynchronize(h->ev_stop[i]) != cudaSuccess) return FD_ERR_CUDA;
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, h->ev_start[i], h->ev_stop[i]) != cudaSuccess) return FD_ERR_CUDA;
+    const int k = h->ev_kind[i];
+    if (k >= 0 && k < FD_K_COUNT) {
+      launches[k] += 1;
+      ms[k] += t;
+    }
+  }
+  h->ev_used = 0;
+  return FD_OK;
+}
+
+int64_t fd_launch_count(fd_handle h) { return h ? h->launches : -1; }
 
 int64_t fd_chunk_index(fd_handle h) { return h ? h->t_host : -1; }
 

@@ -22,6 +22,9 @@ STATUS = {0: "FD_OK", 1: "FD_ERR_INVALID_ARG", 2: "FD_ERR_CONFIG", 3: "FD_ERR_OO
           7: "FD_ERR_UNSUPPORTED"}
 DTYPE_F32, DTYPE_BF16, DTYPE_U8 = 0, 1, 2
 EPI_F32, EPI_RESID, EPI_GELU, EPI_TUP = 0, 1, 2, 3
+# fd_kernel_kind order
+KERNEL_KINDS = ["unshuffle", "embed", "rmsnorm", "qkv", "attn_backbone", "attn_refine", "out",
+                "mlp1", "mlp2", "tup", "head1", "head2", "pixel", "advance"]
 
 
 class FdError(RuntimeError):
@@ -53,7 +56,12 @@ _SIGS = {
     "fd_decode_chunk": (_I, [_P, _P, _P, _P]),
     "fd_decode_chunks": (_I, [ctypes.POINTER(_P), _I, ctypes.POINTER(_P), ctypes.POINTER(_P),
                               _P]),
+    "fd_decode_chunk_host": (_I, [_P, _P, _P, _P]),
     "fd_reset": (_I, [_P]),
+    "fd_profile_enable": (_I, [_P, _I]),
+    "fd_profile_collect": (_I, [_P, ctypes.POINTER(ctypes.c_int64),
+                                ctypes.POINTER(ctypes.c_double)]),
+    "fd_launch_count": (ctypes.c_int64, [_P]),
     "fd_destroy": (_I, [_P]),
     "fd_chunk_index": (ctypes.c_int64, [_P]),
     "fd_sync_status": (_I, [_P]),
@@ -188,8 +196,30 @@ class Decoder:
         _check(lib().fd_decode_chunk(self.handle, _ptr(latent), _ptr(pixels),
                                      _stream_ptr(stream)), "fd_decode_chunk")
 
+    def decode_chunk_host(self, latent_host, pixels_host, stream=None) -> None:
+        """Decode from / to host buffers (numpy arrays or pinned torch tensors)."""
+        lp = latent_host.ctypes.data if isinstance(latent_host, np.ndarray) else _ptr(latent_host)
+        pp = pixels_host.ctypes.data if isinstance(pixels_host, np.ndarray) else _ptr(pixels_host)
+        _check(lib().fd_decode_chunk_host(self.handle, lp, pp, _stream_ptr(stream)),
+               "fd_decode_chunk_host")
+
     def reset(self) -> None:
         _check(lib().fd_reset(self.handle), "fd_reset")
+
+    def profile(self, enable: bool) -> None:
+        _check(lib().fd_profile_enable(self.handle, 1 if enable else 0), "fd_profile_enable")
+
+    def profile_collect(self) -> dict:
+        """{kind name: (launches, device ms)} since the last collect."""
+        n = len(KERNEL_KINDS)
+        launches = (ctypes.c_int64 * n)()
+        ms = (ctypes.c_double * n)()
+        _check(lib().fd_profile_collect(self.handle, launches, ms), "fd_profile_collect")
+        return {k: (int(launches[i]), float(ms[i])) for i, k in enumerate(KERNEL_KINDS)}
+
+    @property
+    def launch_count(self) -> int:
+        return lib().fd_launch_count(self.handle)
 
     def sync_status(self) -> int:
         return lib().fd_sync_status(self.handle)
