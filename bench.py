@@ -332,6 +332,8 @@ def run_ours(args, rank: int, world: int):
                      "peak_source": f"bf16_tflops_sustained ({peak_src}); kernel timed inside "
                                     "a long step",
                      "traffic": ncu_traffic("fd_attn.cu", cfg.name),
+                     "traffic_launch": "ncu DRAM read+write bytes of one steady-state "
+                                       "refinement launch (profiles/traffic.txt)",
                      "flops_per_launch": round(att_flops / att_n),
                      "us_per_launch": round(1e3 * att_ms / att_n, 2),
                      "measured_over": f"{args.steps} profiled steps of the same workload "
