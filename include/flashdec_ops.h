@@ -53,10 +53,15 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
  *   out[r][n*64 + d] = sum_j softmax_j(q_n . k_j / 8) v_j[d],  KV group g = n / (heads/groups)
  * q bf16 [Lq][heads*64]; k_ring bf16 [groups][ring_pitch][64]; vt_ring bf16
  * [groups][64][ring_pitch]; out bf16 [Lq][heads*64]. 1 <= n_keys <= ring_pitch,
- * ring_pitch % 128 == 0. Ring entries past n_keys must hold finite values. */
+ * ring_pitch % 128 == 0. Ring entries past n_keys must hold finite values.
+ * splits: the key range is divided over `splits` CTAs per (query tile, head) whose partial
+ * results a second kernel combines (0 = library choice, 1..16). With more than one split,
+ * `workspace` is a caller-owned device buffer of fd_attention_workspace_bytes(...) bytes
+ * (16-byte aligned) that the call overwrites; calls sharing it must not overlap. */
+size_t fd_attention_workspace_bytes(int Lq, int heads, int groups, int n_keys, int splits);
 fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const void* k_ring,
                           const void* vt_ring, int ring_pitch, int n_keys, void* out,
-                          int* err_dev, void* stream);
+                          int splits, void* workspace, int* err_dev, void* stream);
 
 /* Rolling-cache append (Algorithm 1, cache update): fp32 k, v [groups][rows][64] rounded to
  * bf16 (nearest even) into ring slot s = t mod window: k_ring[g][s*rows + r][d] and

@@ -1,77 +1,115 @@
 // Chunk-window flash attention on tcgen05 (Sec. 3.3 "Attention Pattern", Eq. kv_cache).
 //
-// Query tile of 128 rows x one head per CTA; keys are the first n_keys rows of the layer's
-// ring (the min(t+1, W) cached chunks: ring slots 0..c-1 always hold exactly those chunks,
-// and softmax does not depend on key order). No mask tensor: only the ragged last key block
-// is cut at n_keys. GQA: head n reads KV group n / (N / G).
+// Keys are the first n_keys rows of the layer's ring: ring slots 0..c-1 always hold exactly
+// the c = min(t+1, W) cached chunks, keys carry their RoPE rotation from the append, and
+// softmax does not depend on key order, so no mask tensor is needed; only the ragged last key
+// block is cut at n_keys. GQA: head n reads KV group n / (N / G).
 //
-// Per key block of 128 (warps 0-3 = 128 threads, one query row / TMEM lane per thread):
-//   S  = Q K^T          tcgen05.mma M=128 N=128 K=64, fp32 in TMEM columns [0, 128)
-//   softmax             each thread loads its S row, online max / sum in fp32 (log2 domain),
-//                       writes P = exp2(s - m) as bf16 into a 128-byte-swizzled smem tile
-//   O_blk = P V         tcgen05.mma M=128 N=64 K=128 with B = V^T from the transposed V ring,
-//                       fp32 in TMEM columns [128, 192); the thread folds it into its
-//                       register accumulator o = o * alpha + O_blk
-// K / V^T blocks are double-buffered TMA loads; S for block j+1 is issued right after P V for
-// block j, so it overlaps the O_blk read-back. Two CTAs per SM overlap one CTA's MMAs with the
-// other's softmax.
+// One CTA = two 128-row tiles X = 0, 1 that share one KV group (two heads of the group on one
+// query tile, or two query tiles of one head), so each K / V block is loaded once for both.
+// Optionally the key range is split over `splits` CTAs whose partial results a second kernel
+// combines (balances the grid over the SMs).
+//
+// Warp roles (320 threads):
+//   warp 8        TMA: Q tiles once, then K and V^T blocks of 128 keys into a 3-stage ring
+//   warp 9        one thread issues the MMAs, ping-ponging the two tiles:
+//                   S_X  = Q_X K^T       M=128 N=128 K=64, fp32 in TMEM columns [128X, 128X+128)
+//                   O_X += P_X [V^T;1]   M=128 N=80  K=128, A = P_X read from TMEM, B = V^T
+//                                         with a ones row appended, so column 64 of O_X
+//                                         accumulates the row sums of P
+//   warps 0-3 / 4-7  softmax of tile 0 / 1, one query row (TMEM lane) per thread: load S,
+//                 running max in the log2 domain, P = exp2(s - m) written back as bf16 into
+//                 the first 64 columns of S_X (P aliases S). O_X lives in TMEM; it is rescaled
+//                 (load, multiply, store) only when a row's max grows by more than 2^8, so
+//                 P stays <= 256 and the rescale is rare.
+// The tensor core executes tcgen05.mma in issue order, so S_X(j+1), issued after the P V MMA
+// of block j, never overwrites P_X(j) before it has been read.
 #include "fd_internal.h"
 #include "fd_ptx.cuh"
 
 namespace fd {
 
 namespace attn {
-constexpr int kQBytes = 128 * 128;       // Q tile [128][64] bf16
-constexpr int kKBytes = 128 * 128;       // K block [128 keys][64] bf16
-constexpr int kVBytes = 2 * 64 * 128;    // V^T block: 2 sub-tiles [64 dh][64 keys] bf16
-constexpr int kPBytes = 2 * 128 * 128;   // P: 2 sub-tiles [128 rows][64 keys] bf16
+constexpr int kStages = 3;
+constexpr int kQBytes = 128 * 128;           // Q tile [128 rows][64] bf16
+constexpr int kKBytes = 128 * 128;           // K block [128 keys][64] bf16
+constexpr int kVRows = 80;                   // 64 rows of V^T, a ones row, 15 zero rows
+constexpr int kVSub = kVRows * 128;          // one 64-key sub-tile, 10 KB
+constexpr int kVBytes = 2 * kVSub;           // V^T block of 128 keys
+constexpr int kVLoadBytes = 2 * 64 * 128;    // bytes TMA writes into a V^T block
 constexpr int kOffQ = 0;
-constexpr int kOffK = kOffQ + kQBytes;               // 2 stages
-constexpr int kOffV = kOffK + 2 * kKBytes;           // 2 stages
-constexpr int kOffP = kOffV + 2 * kVBytes;
-constexpr int kOffBar = kOffP + kPBytes;
-constexpr int kSmem = kOffBar + 128;
-constexpr int kTmemCols = 256;
-constexpr uint32_t kColO = 128;
+constexpr int kOffK = 2 * kQBytes;
+constexpr int kOffV = kOffK + kStages * kKBytes;
+constexpr int kOffBar = kOffV + kStages * kVBytes;
+constexpr int kSmem = kOffBar + 256;
+constexpr int kThreads = 320;
+constexpr int kTmemCols = 512;
+constexpr uint32_t kColO = 256;              // O_X at columns 256 + 80 X
+constexpr uint32_t kColOStride = 80;
+constexpr float kRescaleLog2 = 8.0f;
+// barrier indices
+constexpr int kBarQ = 0, kBarKvFull = 1, kBarKvEmpty = 1 + kStages, kBarS = 1 + 2 * kStages,
+              kBarP = kBarS + 2, kBarODone = kBarP + 2, kBarDone = kBarODone + 2,
+              kNumBars = kBarDone + 1;
+static_assert(kNumBars * 8 + 4 <= 256, "barrier area");
+static_assert(kSmem <= 227 * 1024, "shared memory");
 }  // namespace attn
 
-__global__ void __launch_bounds__(128, 2)
+__global__ void __launch_bounds__(attn::kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
   using namespace attn;
   extern __shared__ __align__(1024) uint8_t smem[];
-  const int tid = threadIdx.x;
-  const int warp = tid >> 5;
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
   const uint32_t base = smem_u32(smem);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
-  const uint32_t bar_q = smem_u32(bars + 0);
-  const uint32_t bar_kv = smem_u32(bars + 1);  // [2]
-  const uint32_t bar_s = smem_u32(bars + 3);
-  const uint32_t bar_o = smem_u32(bars + 4);
-  const uint32_t bar_done = smem_u32(bars + 5);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 6);
   const bool aligned = (base & 1023u) == 0;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
+  const uint32_t bar0 = smem_u32(bars);
+  auto bar = [&](int i) { return bar0 + 8u * static_cast<uint32_t>(i); };
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kNumBars);
 
-  const int q0 = blockIdx.x * kBM;
-  const int head = blockIdx.y;
-  const int g = head / (p.heads / p.groups);
+  // the two tiles of this CTA: (query tile qt0, head hd0) and (qt1, hd1)
+  const int qt0 = p.pair_heads ? blockIdx.x : 2 * blockIdx.x;
+  const int qt1 = p.pair_heads ? blockIdx.x : 2 * blockIdx.x + 1;
+  const int hd0 = p.pair_heads ? 2 * blockIdx.y : blockIdx.y;
+  const int hd1 = p.pair_heads ? 2 * blockIdx.y + 1 : blockIdx.y;
+  const int g = hd0 / (p.heads / p.groups);
   int n_keys = p.n_keys_host;
   if (p.step_dev != nullptr) {
     const int t = *p.step_dev;
     n_keys = (t + 1 < p.window ? t + 1 : p.window) * p.rows_per_chunk;
   }
-  const int nblk = (n_keys + 127) / 128;
-  const int key_row0 = g * p.ring_pitch;
+  const int nblk_all = (n_keys + 127) / 128;
+  const int per = (nblk_all + p.splits - 1) / p.splits;
+  const int kb0 = blockIdx.z * per;
+  const int kb_end = kb0 + per < nblk_all ? kb0 + per : nblk_all;
+  const int nblk = kb_end > kb0 ? kb_end - kb0 : 0;
 
-  if (tid == 0) {
+  if (threadIdx.x == 0) {
     if (!aligned) atomicOr(p.err, ERR_SMEM_ALIGN);
-    mbar_init(bar_q, 1);
-    mbar_init(bar_kv, 1);
-    mbar_init(bar_kv + 8, 1);
-    mbar_init(bar_s, 1);
-    mbar_init(bar_o, 1);
-    mbar_init(bar_done, 1);
+    mbar_init(bar(kBarQ), 1);
+    for (int st = 0; st < kStages; ++st) {
+      mbar_init(bar(kBarKvFull + st), 1);
+      mbar_init(bar(kBarKvEmpty + st), 1);
+    }
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(bar(kBarS + x), 1);
+      mbar_init(bar(kBarP + x), 128);
+      mbar_init(bar(kBarODone + x), 1);
+    }
+    mbar_init(bar(kBarDone), 1);
     fence_barrier_init();
+  }
+  if (warp == 8 && aligned) {
+    // rows 64..79 of every V^T sub-tile: row 64 = 1.0 (row sums of P), rows 65..79 = 0
+    for (int i = lane; i < kStages * 2 * 16 * 8; i += 32) {
+      const int chunk = i & 7, row = 64 + ((i >> 3) & 15), sub = i >> 7;
+      const uint32_t v = row == 64 ? 0x3F803F80u : 0u;
+      *reinterpret_cast<uint4*>(smem + kOffV + sub * kVSub + row * 128 + chunk * 16) =
+          make_uint4(v, v, v, v);
+    }
+    fence_proxy_async_smem();
   }
   if (warp == 0) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
@@ -81,162 +119,259 @@ __global__ void __launch_bounds__(128, 2)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tlane = static_cast<uint32_t>(warp * 32) << 16;
-  const uint32_t idesc_s = idesc_bf16_f32(128, 128);
-  const uint32_t idesc_o = idesc_bf16_f32(128, 64);
 
-  int last_loaded[2] = {-1, -1};  // block index last loaded into each K/V stage (thread 0)
-  int last_waited[2] = {-1, -1};
-  auto load_kv = [&](int j, int st) {
-    const uint32_t b = bar_kv + 8 * st;
-    mbar_expect_tx(b, kKBytes + kVBytes);
-    tma_load_2d(base + kOffK + st * kKBytes, &tmK, b, 0, key_row0 + j * 128);
-    tma_load_2d(base + kOffV + st * kVBytes, &tmV, b, j * 128, g * kHeadDim);
-    tma_load_2d(base + kOffV + st * kVBytes + kVBytes / 2, &tmV, b, j * 128 + 64, g * kHeadDim);
-    last_loaded[st] = j;
-  };
-  auto issue_s = [&](int j) {  // S = Q K_j^T  (thread 0 only); always commits bar_s
-    const int st = j & 1;
-    const bool got = mbar_wait(bar_kv + 8 * st, (j >> 1) & 1, p.err, ERR_WAIT_TMA);
-    if (got) last_waited[st] = j;
-    tc_fence_after();
-    if (got) {
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        mma_bf16_ss(tmem, sdesc_k_sw128(base + kOffQ + 32 * k),
-                    sdesc_k_sw128(base + kOffK + st * kKBytes + 32 * k), idesc_s, k != 0);
-    }
-    mma_commit(bar_s);
-  };
-
-  bool issued_any = false;
-  if (aligned && nblk > 0 && tid == 0) {
-    prefetch_tmap(&tmQ);
-    prefetch_tmap(&tmK);
-    prefetch_tmap(&tmV);
-    mbar_expect_tx(bar_q, kQBytes);
-    tma_load_2d(base + kOffQ, &tmQ, bar_q, head * kHeadDim, q0);
-    load_kv(0, 0);
-    if (nblk > 1) load_kv(1, 1);
-    mbar_wait(bar_q, 0, p.err, ERR_WAIT_TMA);
-    issue_s(0);
-    issued_any = true;
-  }
-
-  const float sl2 = p.scale_log2;
-  float m_run = -INFINITY, l_run = 0.f;
-  float o[64];
-#pragma unroll
-  for (int d = 0; d < 64; ++d) o[d] = 0.f;
-
-  const int my_row = tid;  // row within the tile == TMEM lane
-  uint8_t* sP = smem + kOffP;
-  bool fail = !aligned;     // block-uniform when the loop is left
-  for (int j = 0; j < nblk && aligned; ++j) {
-    fail |= !mbar_wait(bar_s, j & 1, p.err, ERR_WAIT_MMA);
-    tc_fence_after();
-    uint32_t sr[4][32];
-    __syncwarp();
-#pragma unroll
-    for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(tmem + tlane + 32 * c, sr[c]);
-    tmem_ld_wait();
-    const int valid = n_keys - j * 128;  // >= 1
-    float mx = -INFINITY;
-#pragma unroll
-    for (int c = 0; c < 4; ++c)
-#pragma unroll
-      for (int e = 0; e < 32; ++e) {
-        float s = __uint_as_float(sr[c][e]);
-        if (32 * c + e >= valid) s = -INFINITY;
-        sr[c][e] = __float_as_uint(s);
-        mx = fmaxf(mx, s);
+  if (warp == 8) {
+    // ------------------------------------------------------------ TMA loads
+    if (lane == 0 && aligned && nblk > 0) {
+      prefetch_tmap(&tmQ);
+      prefetch_tmap(&tmK);
+      prefetch_tmap(&tmV);
+      mbar_expect_tx(bar(kBarQ), 2 * kQBytes);
+      tma_load_2d(base + kOffQ, &tmQ, bar(kBarQ), hd0 * kHeadDim, qt0 * kBM);
+      tma_load_2d(base + kOffQ + kQBytes, &tmQ, bar(kBarQ), hd1 * kHeadDim, qt1 * kBM);
+      int j = 0;
+      for (; j < nblk; ++j) {
+        const int st = j % kStages;
+        if (!mbar_wait(bar(kBarKvEmpty + st), ((j / kStages) & 1) ^ 1, p.err, ERR_WAIT_MMA))
+          break;
+        const uint32_t b = bar(kBarKvFull + st);
+        const int kb = kb0 + j;
+        mbar_expect_tx(b, kKBytes + kVLoadBytes);
+        tma_load_2d(base + kOffK + st * kKBytes, &tmK, b, 0, g * p.ring_pitch + kb * 128);
+        tma_load_2d(base + kOffV + st * kVBytes, &tmV, b, kb * 128, g * kHeadDim);
+        tma_load_2d(base + kOffV + st * kVBytes + kVSub, &tmV, b, kb * 128 + 64, g * kHeadDim);
       }
-    const float m_new = fmaxf(m_run, mx * sl2);
-    const float alpha = ex2_approx(m_run - m_new);
-    float lsum = 0.f;
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-#pragma unroll
-      for (int e8 = 0; e8 < 4; ++e8) {
-        float pv[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          pv[e] = ex2_approx(fmaf(__uint_as_float(sr[c][8 * e8 + e]), sl2, -m_new));
-          lsum += pv[e];
-        }
-        const uint32_t key = 32 * c + 8 * e8;  // first key of this 16-byte chunk
-        const uint32_t off = (key >> 6) * (128 * 128) + sw128_offset(my_row, key & 63);
-        *reinterpret_cast<uint4*>(sP + off) =
-            make_uint4(pack_bf16x2(pv[0], pv[1]), pack_bf16x2(pv[2], pv[3]),
-                       pack_bf16x2(pv[4], pv[5]), pack_bf16x2(pv[6], pv[7]));
-      }
+      // nothing may be in flight when the CTA exits
+      mbar_wait(bar(kBarQ), 0, p.err, ERR_WAIT_TMA);
+      for (int i = j - 1; i >= 0 && i >= j - kStages; --i)
+        mbar_wait(bar(kBarKvFull + i % kStages), (i / kStages) & 1, p.err, ERR_WAIT_TMA);
     }
-    l_run = l_run * alpha + lsum;
-    m_run = m_new;
-    fence_proxy_async_smem();  // P (generic-proxy stores) visible to the tensor core
-    tc_fence_before();
-    if (__syncthreads_or(fail)) {  // also orders every S / O_blk TMEM read before the MMAs
-      fail = true;
-      break;
-    }
-    if (tid == 0) {
+  } else if (warp == 9) {
+    // ------------------------------------------------------------ MMA issue
+    if (lane == 0 && aligned && nblk > 0) {
+      const uint32_t idesc_s = idesc_bf16_f32(128, 128);
+      const uint32_t idesc_o = idesc_bf16_f32(128, kVRows);
+      bool ok = mbar_wait(bar(kBarQ), 0, p.err, ERR_WAIT_TMA) &&
+                mbar_wait(bar(kBarKvFull), 0, p.err, ERR_WAIT_TMA);
       tc_fence_after();
-      const uint32_t vst = base + kOffV + (j & 1) * kVBytes;
+      auto issue_s = [&](int x, int st) {
 #pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint32_t sub = kk >> 2, within = (kk & 3) * 32;
-        mma_bf16_ss(tmem + kColO, sdesc_k_sw128(base + kOffP + sub * (128 * 128) + within),
-                    sdesc_k_sw128(vst + sub * (64 * 128) + within), idesc_o, kk != 0);
+        for (int k = 0; k < 4; ++k)
+          mma_bf16_ss(tmem + 128u * x, sdesc_k_sw128(base + kOffQ + x * kQBytes + 32 * k),
+                      sdesc_k_sw128(base + kOffK + st * kKBytes + 32 * k), idesc_s, k != 0);
+        mma_commit(bar(kBarS + x));
+      };
+      if (ok) {
+        issue_s(0, 0);
+        issue_s(1, 0);
       }
-      mma_commit(bar_o);
-      if (j + 1 < nblk) issue_s(j + 1);
-    }
-    const bool o_ok = mbar_wait(bar_o, j & 1, p.err, ERR_WAIT_MMA);
-    fail |= !o_ok;
-    tc_fence_after();
-    uint32_t orr[2][32];
-    __syncwarp();
-    tmem_ld_32x32b_x32(tmem + tlane + kColO, orr[0]);
-    tmem_ld_32x32b_x32(tmem + tlane + kColO + 32, orr[1]);
-    tmem_ld_wait();
+      for (int j = 0; j < nblk && ok; ++j) {
+        const int st = j % kStages;
+        for (int x = 0; x < 2 && ok; ++x) {
+          if (!mbar_wait(bar(kBarP + x), j & 1, p.err, ERR_WAIT_EPI)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t o_tmem = tmem + kColO + kColOStride * x;
 #pragma unroll
-    for (int d = 0; d < 32; ++d) {
-      o[d] = fmaf(o[d], alpha, __uint_as_float(orr[0][d]));
-      o[32 + d] = fmaf(o[32 + d], alpha, __uint_as_float(orr[1][d]));
+          for (int kk = 0; kk < 8; ++kk)
+            mma_bf16_ts(o_tmem, tmem + 128u * x + 8u * kk,
+                        sdesc_k_sw128(base + kOffV + st * kVBytes + (kk >> 2) * kVSub +
+                                      (kk & 3) * 32),
+                        idesc_o, (j | kk) != 0);
+          if (x == 1) mma_commit(bar(kBarKvEmpty + st));  // K_j, V_j no longer read
+          if (j + 1 < nblk) {
+            const int st1 = (j + 1) % kStages;
+            if (x == 0) {
+              ok = mbar_wait(bar(kBarKvFull + st1), ((j + 1) / kStages) & 1, p.err,
+                             ERR_WAIT_TMA);
+              tc_fence_after();
+            }
+            if (ok) issue_s(x, st1);
+          } else {
+            mma_commit(bar(kBarODone + x));
+          }
+        }
+      }
+      mma_commit(bar(kBarDone));
+      mbar_wait(bar(kBarDone), 0, p.err, ERR_WAIT_MMA);
     }
-    tc_fence_before();
-    if (tid == 0 && o_ok && j + 2 < nblk) load_kv(j + 2, j & 1);  // stage free: P V_j done
-  }
-  const bool ok = !fail;
-
-  // output row: O / l as bf16
-  const int row = q0 + my_row;
-  if (ok && row < p.Lq) {
-    const float inv = 1.0f / l_run;
-    uint4* dst = reinterpret_cast<uint4*>(p.out + static_cast<size_t>(row) * p.ld_out +
-                                          head * kHeadDim);
+  } else {
+    // ------------------------------------------------------------ softmax, tile x
+    const int x = warp >> 2;
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    const uint32_t s_col = tmem + lane_off + 128u * x;
+    const uint32_t o_col = tmem + lane_off + kColO + kColOStride * x;
+    const float sl2 = p.scale_log2;
+    float m_used = -INFINITY;
+    bool ok = aligned;
+    for (int j = 0; j < nblk && ok; ++j) {
+      const bool got = mbar_wait(bar(kBarS + x), j & 1, p.err, ERR_WAIT_MMA);
+      if (!__all_sync(0xffffffffu, got)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      uint32_t sr[4][32];
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
-      dst[j] = make_uint4(pack_bf16x2(o[8 * j] * inv, o[8 * j + 1] * inv),
-                          pack_bf16x2(o[8 * j + 2] * inv, o[8 * j + 3] * inv),
-                          pack_bf16x2(o[8 * j + 4] * inv, o[8 * j + 5] * inv),
-                          pack_bf16x2(o[8 * j + 6] * inv, o[8 * j + 7] * inv));
+      for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(s_col + 32 * c, sr[c]);
+      tmem_ld_wait();
+      const int valid = n_keys - (kb0 + j) * 128;
+      if (valid < 128) {  // ragged last key block (block-uniform branch)
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (32 * c + e >= valid) sr[c][e] = 0xff800000u;  // -inf
+      }
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+#pragma unroll
+        for (int e = 0; e < 32; e += 2)
+          mx = fmax3(mx, __uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1]));
+      const float mb = mx * sl2;
+      const bool grow = mb > m_used + kRescaleLog2;
+      const float m_new = grow ? mb : m_used;
+      if (__any_sync(0xffffffffu, grow && j > 0)) {
+        // rescale this warp's O rows (the P V MMA of block j-1 has completed: its commit
+        // preceded the one that released S_X(j))
+        // (32 columns at a time: S stays live in registers meanwhile)
+        const float f = (grow && j > 0) ? ex2_approx(m_used - m_new) : 1.0f;
+#pragma unroll 1
+        for (int c = 0; c < 64; c += 32) {
+          uint32_t o0[32];
+          tmem_ld_32x32b_x32(o_col + c, o0);
+          tmem_ld_wait();
+#pragma unroll
+          for (int d = 0; d < 32; ++d) o0[d] = __float_as_uint(__uint_as_float(o0[d]) * f);
+          tmem_st_32x32b_x32(o_col + c, o0);
+        }
+        uint32_t o2[16];
+        tmem_ld_32x32b_x16(o_col + 64, o2);
+        tmem_ld_wait();
+#pragma unroll
+        for (int d = 0; d < 16; ++d) o2[d] = __float_as_uint(__uint_as_float(o2[d]) * f);
+        tmem_st_32x32b_x16(o_col + 64, o2);
+      }
+      m_used = m_new;
+      const float neg = -m_used;
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        uint32_t pk[32];
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc)
+#pragma unroll
+          for (int e = 0; e < 32; e += 2) {
+            const int c = 2 * half + cc;
+            const float a = ex2_approx(fmaf(__uint_as_float(sr[c][e]), sl2, neg));
+            const float b = ex2_approx(fmaf(__uint_as_float(sr[c][e + 1]), sl2, neg));
+            pk[cc * 16 + (e >> 1)] = pack_bf16x2(a, b);
+          }
+        tmem_st_32x32b_x32(s_col + 32 * half, pk);
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(bar(kBarP + x));
+    }
+    // ------------------------------------------------------------ output of tile x
+    float o[64];
+    float l = 0.f;
+#pragma unroll
+    for (int d = 0; d < 64; ++d) o[d] = 0.f;
+    if (ok && nblk > 0) {
+      const bool got = mbar_wait(bar(kBarODone + x), 0, p.err, ERR_WAIT_MMA);
+      ok = __all_sync(0xffffffffu, got);
+      if (ok) {
+        tc_fence_after();
+        uint32_t o0[32], o1[32], o2[16];
+        tmem_ld_32x32b_x32(o_col, o0);
+        tmem_ld_32x32b_x32(o_col + 32, o1);
+        tmem_ld_32x32b_x16(o_col + 64, o2);
+        tmem_ld_wait();
+#pragma unroll
+        for (int d = 0; d < 32; ++d) {
+          o[d] = __uint_as_float(o0[d]);
+          o[32 + d] = __uint_as_float(o1[d]);
+        }
+        l = __uint_as_float(o2[0]);
+      }
+    }
+    const int r = (x ? qt1 : qt0) * kBM + row;
+    if (ok && r < p.Lq) {
+      const int h = x ? hd1 : hd0;
+      if (p.splits == 1) {
+        const float inv = 1.0f / l;
+        uint4* dst = reinterpret_cast<uint4*>(p.out + static_cast<size_t>(r) * p.ld_out +
+                                              h * kHeadDim);
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          dst[k] = make_uint4(pack_bf16x2(o[8 * k] * inv, o[8 * k + 1] * inv),
+                              pack_bf16x2(o[8 * k + 2] * inv, o[8 * k + 3] * inv),
+                              pack_bf16x2(o[8 * k + 4] * inv, o[8 * k + 5] * inv),
+                              pack_bf16x2(o[8 * k + 6] * inv, o[8 * k + 7] * inv));
+      } else {
+        const size_t idx = (static_cast<size_t>(blockIdx.z) * p.heads + h) * p.Lq + r;
+        float4* dst = reinterpret_cast<float4*>(p.part_o + idx * kHeadDim);
+#pragma unroll
+        for (int k = 0; k < 16; ++k)
+          dst[k] = make_float4(o[4 * k], o[4 * k + 1], o[4 * k + 2], o[4 * k + 3]);
+        reinterpret_cast<float2*>(p.part_ml)[idx] = make_float2(nblk > 0 ? m_used : -INFINITY, l);
+      }
+    }
   }
 
-  // teardown: every MMA of this CTA has completed and no TMA load is still in flight
-  if (tid == 0 && issued_any) {
-    mma_commit(bar_done);
-    mbar_wait(bar_done, 0, p.err, ERR_WAIT_MMA);
-    for (int st = 0; st < 2; ++st)
-      if (last_loaded[st] > last_waited[st])
-        mbar_wait(bar_kv + 8 * st, (last_loaded[st] >> 1) & 1, p.err, ERR_WAIT_TMA);
-  }
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
+}
+
+// One warp per (row, head): O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s.
+__global__ void attn_combine_kernel(const float* __restrict__ part_o,
+                                    const float* __restrict__ part_ml, int splits, int Lq,
+                                    int heads, __nv_bfloat16* __restrict__ out, int ld_out) {
+  const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (wid >= Lq * heads) return;
+  const int r = wid / heads, h = wid - r * heads;
+  const float2* ml = reinterpret_cast<const float2*>(part_ml);
+  float M = -INFINITY;
+  for (int s = 0; s < splits; ++s)
+    M = fmaxf(M, ml[(static_cast<size_t>(s) * heads + h) * Lq + r].x);
+  float a0 = 0.f, a1 = 0.f, l = 0.f;
+  for (int s = 0; s < splits; ++s) {
+    const size_t idx = (static_cast<size_t>(s) * heads + h) * Lq + r;
+    const float2 v = ml[idx];
+    const float w = ex2_approx(v.x - M);
+    l = fmaf(w, v.y, l);
+    const float2 o = reinterpret_cast<const float2*>(part_o + idx * kHeadDim)[lane];
+    a0 = fmaf(w, o.x, a0);
+    a1 = fmaf(w, o.y, a1);
+  }
+  const float inv = 1.0f / l;
+  reinterpret_cast<uint32_t*>(out + static_cast<size_t>(r) * ld_out + h * kHeadDim)[lane] =
+      pack_bf16x2(a0 * inv, a1 * inv);
+}
+
+int attention_splits(int units, int nblk, int num_sms) {
+  int best = 1;
+  long long best_cost = -1;
+  for (int s = 1; s <= 4; ++s) {
+    const long long ctas = static_cast<long long>(units) * s;
+    const long long waves = (ctas + num_sms - 1) / num_sms;
+    const long long cost = waves * ((nblk + s - 1) / s) * 100 + (s > 1 ? 150 : 0);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = s;
+    }
+  }
+  return best;
 }
 
 cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmK,
@@ -248,8 +383,15 @@ cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmK,
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  dim3 grid((p.Lq + kBM - 1) / kBM, p.heads);
-  attn_kernel<<<grid, 128, attn::kSmem, s>>>(tmQ, tmK, tmVt, p);
+  const int qtiles = (p.Lq + kBM - 1) / kBM;
+  dim3 grid = p.pair_heads ? dim3(qtiles, p.heads / 2, p.splits)
+                           : dim3((qtiles + 1) / 2, p.heads, p.splits);
+  attn_kernel<<<grid, attn::kThreads, attn::kSmem, s>>>(tmQ, tmK, tmVt, p);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || p.splits == 1) return e;
+  const long long warps = static_cast<long long>(p.Lq) * p.heads;
+  attn_combine_kernel<<<static_cast<int>((warps + 7) / 8), 256, 0, s>>>(
+      p.part_o, p.part_ml, p.splits, p.Lq, p.heads, p.out, p.ld_out);
   return cudaGetLastError();
 }
 

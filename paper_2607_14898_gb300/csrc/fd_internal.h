@@ -65,13 +65,24 @@ struct AttnParams {
   int ld_out;
   float scale_log2;          // log2(e) / sqrt(D_h)
   int* err;
+  int pair_heads;            // 1: a CTA takes heads 2p, 2p+1 of one q tile; 0: q tiles 2i, 2i+1
+  int splits;                // key-range splits per (q tile, head); > 1 writes partials
+  float* part_o;             // [splits][heads][Lq][64] unnormalised O   (splits > 1)
+  float* part_ml;            // [splits][heads][Lq][2]  (max used, row sum) (splits > 1)
 };
 
 // launch wrappers; return cudaGetLastError() of the launch
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p,
                         int bn, int num_sms, cudaStream_t s);
+// Attention (+ the combine of key-range splits when p.splits > 1).
 cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmK,
                              const CUtensorMap& tmVt, const AttnParams& p, cudaStream_t s);
+// Key-range splits that balance (units x splits) CTAs over the SMs for nblk key blocks.
+int attention_splits(int units, int nblk, int num_sms);
+// Workspace floats needed by a split attention of Lq rows.
+inline size_t attention_workspace_floats(int splits, int heads, int Lq) {
+  return splits <= 1 ? 0 : static_cast<size_t>(splits) * heads * Lq * (64 + 2);
+}
 cudaError_t launch_unshuffle(const float* z, int C, int H, int W, int p, __nv_bfloat16* x0,
                              cudaStream_t s);
 cudaError_t launch_rmsnorm(const float* h, const float* g, int M, int D, float eps,

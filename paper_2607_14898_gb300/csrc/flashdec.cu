@@ -212,6 +212,10 @@ struct fd_handle_s {
   float *h = nullptr, *hf = nullptr, *F = nullptr;
   int pitchB = 0, pitchR = 0;
   std::vector<Ring> ringB, ringR;
+  // attention key-range splits (fixed per stack for the steady-state window) and their
+  // partial-result workspace
+  int splitsB = 1, splitsR = 1;
+  float* attn_ws = nullptr;
   // A-operand / Q descriptors
   CUtensorMap tm_x0, tm_uB, tm_uR, tm_oB, tm_oR, tm_hidB, tm_hidR, tm_hidH, tm_qB, tm_qR;
   // host-buffer decode: library-owned device copies of the latent and the pixels
@@ -273,6 +277,15 @@ fd_status traced(fd_handle h, int kind, cudaStream_t s, Fn&& fn) {
   return FD_OK;
 }
 
+int pair_heads(int heads, int groups) { return (heads / groups) % 2 == 0 ? 1 : 0; }
+
+// key-range splits for an attention of Lq rows over n_keys keys
+int choose_splits(int Lq, int heads, int groups, int n_keys) {
+  const int qtiles = (Lq + 127) / 128;
+  const int units = pair_heads(heads, groups) ? qtiles * (heads / 2) : ((qtiles + 1) / 2) * heads;
+  return fd::attention_splits(units, (n_keys + 127) / 128, num_sms());
+}
+
 fd_status run_linear(fd_handle h, int kind, const CUtensorMap& tmA, const Linear& lin, int M,
                      fd::GemmParams p, cudaStream_t s) {
   p.M = M;
@@ -313,6 +326,10 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
   a.window = d.Wn; a.step_dev = h->state; a.n_keys_host = 0; a.out = h->o;
   a.ld_out = d.N * kHeadDim; a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
   a.err = h->state + 1;
+  a.pair_heads = pair_heads(d.N, d.G);
+  a.splits = refine ? h->splitsR : h->splitsB;
+  a.part_o = h->attn_ws;
+  a.part_ml = h->attn_ws + static_cast<size_t>(a.splits) * d.N * rows * kHeadDim;
   if ((st = traced(h, refine ? FD_K_ATTN_R : FD_K_ATTN_B, s,
                    [&] { return fd::launch_attention(tm_q, r.tm_k, r.tm_vt, a, s); })))
     return st;
@@ -422,12 +439,21 @@ size_t fd_pixels_bytes(const fd_config* cfg) {
   return static_cast<size_t>(d.Cout) * d.rt * d.gh * d.rs * d.gw * d.rs * (d.u8 ? 1 : 4);
 }
 
-static size_t handle_layout(const Dims& d, size_t* off /* 14 offsets */, int* pitchB,
+static size_t attn_ws_floats(const Dims& d) {
+  const int R = d.rt * d.L;
+  const int sB = choose_splits(d.L, d.N, d.G, d.Wn * d.L);
+  const int sR = choose_splits(R, d.N, d.G, d.Wn * R);
+  const size_t a = fd::attention_workspace_floats(sB, d.N, d.L);
+  const size_t b = d.nr > 0 ? fd::attention_workspace_floats(sR, d.N, R) : 0;
+  return a > b ? a : b;
+}
+
+static size_t handle_layout(const Dims& d, size_t* off /* 15 offsets */, int* pitchB,
                             int* pitchR) {
   const size_t R = static_cast<size_t>(d.rt) * d.L;
   *pitchB = static_cast<int>(align_up(static_cast<size_t>(d.Wn) * d.L, 128));
   *pitchR = static_cast<int>(align_up(static_cast<size_t>(d.Wn) * R, 128));
-  size_t sizes[13] = {
+  size_t sizes[14] = {
       16,                                              // state
       static_cast<size_t>(d.L) * d.cin * 2,            // x0
       R * d.D * 2,                                     // u
@@ -441,19 +467,20 @@ static size_t handle_layout(const Dims& d, size_t* off /* 14 offsets */, int* pi
       static_cast<size_t>(d.nr) * 2 * d.G * *pitchR * kHeadDim * 2,  // refinement rings
       static_cast<size_t>(d.C) * d.H * d.W * 4,                      // latent (host decode)
       static_cast<size_t>(d.Cout) * d.rt * d.gh * d.rs * d.gw * d.rs * (d.u8 ? 1 : 4),  // pixels
+      attn_ws_floats(d) * 4,                                         // attention partials
   };
   size_t cur = 0;
-  for (int i = 0; i < 13; ++i) {
+  for (int i = 0; i < 14; ++i) {
     off[i] = cur;
     cur = align_up(cur + sizes[i], 1024);
   }
-  off[13] = cur;
+  off[14] = cur;
   return cur;
 }
 
 size_t fd_handle_device_bytes(const fd_config* cfg) {
   if (!valid_cfg(cfg)) return 0;
-  size_t off[14];
+  size_t off[15];
   int a, b;
   return handle_layout(dims_of(cfg), off, &a, &b);
 }
@@ -580,7 +607,7 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   h->d = dims_of(cfg);
   h->w = w;
   const Dims& d = h->d;
-  size_t off[14];
+  size_t off[15];
   h->arena_bytes = handle_layout(d, off, &h->pitchB, &h->pitchR);
   if (cudaMalloc(&h->arena, h->arena_bytes) != cudaSuccess) {
     delete h;
@@ -598,6 +625,9 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   h->F = reinterpret_cast<float*>(b + off[8]);
   h->latent_buf = reinterpret_cast<float*>(b + off[11]);
   h->pixel_buf = b + off[12];
+  h->attn_ws = reinterpret_cast<float*>(b + off[13]);
+  h->splitsB = choose_splits(d.L, d.N, d.G, d.Wn * d.L);
+  h->splitsR = choose_splits(d.rt * d.L, d.N, d.G, d.Wn * d.rt * d.L);
   const size_t ringB_elems = static_cast<size_t>(d.G) * h->pitchB * kHeadDim;
   const size_t ringR_elems = static_cast<size_t>(d.G) * h->pitchR * kHeadDim;
   h->ringB.resize(d.nb);
@@ -855,13 +885,22 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
   return launch_ok(fd::launch_gemm(ta, tb, p, bn, num_sms(), static_cast<cudaStream_t>(stream)));
 }
 
+size_t fd_attention_workspace_bytes(int Lq, int heads, int groups, int n_keys, int splits) {
+  if (Lq < 1 || heads < 1 || groups < 1 || heads % groups || n_keys < 1 || splits < 0)
+    return 0;
+  if (splits == 0) splits = choose_splits(Lq, heads, groups, n_keys);
+  return fd::attention_workspace_floats(splits, heads, Lq) * 4;
+}
+
 fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const void* k_ring,
                           const void* vt_ring, int ring_pitch, int n_keys, void* out,
-                          int* err_dev, void* stream) {
+                          int splits, void* workspace, int* err_dev, void* stream) {
   if (!q || !k_ring || !vt_ring || !out || !err_dev) return FD_ERR_INVALID_ARG;
   if (Lq < 1 || heads < 1 || groups < 1 || heads % groups || n_keys < 1 ||
-      n_keys > ring_pitch || ring_pitch % 128)
+      n_keys > ring_pitch || ring_pitch % 128 || splits < 0 || splits > 16)
     return FD_ERR_INVALID_ARG;
+  if (splits == 0) splits = choose_splits(Lq, heads, groups, n_keys);
+  if (splits > 1 && (workspace == nullptr || !aligned16(workspace))) return FD_ERR_INVALID_ARG;
   fd_status st = check_device();
   if (st) return st;
   const uint64_t NQ = static_cast<uint64_t>(heads) * kHeadDim;
@@ -878,6 +917,10 @@ fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const vo
   a.out = static_cast<__nv_bfloat16*>(out); a.ld_out = static_cast<int>(NQ);
   a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
   a.err = err_dev;
+  a.pair_heads = pair_heads(heads, groups);
+  a.splits = splits;
+  a.part_o = static_cast<float*>(workspace);
+  a.part_ml = a.part_o + static_cast<size_t>(splits) * heads * Lq * kHeadDim;
   return launch_ok(fd::launch_attention(tq, tk, tv, a, static_cast<cudaStream_t>(stream)));
 }
 

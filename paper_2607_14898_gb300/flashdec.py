@@ -69,7 +69,8 @@ _SIGS = {
     "fd_op_linear": (_I, [_I, _I, _I, _I, _P, _P, _P, _P, _I, _I, _P, _P]),
     "fd_op_qkv": (_I, [_I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _F, _F,
                        _P, _P, _P, _I, _I, _P, _P]),
-    "fd_op_attention": (_I, [_I, _I, _I, _P, _P, _P, _I, _I, _P, _P, _P]),
+    "fd_attention_workspace_bytes": (ctypes.c_size_t, [_I, _I, _I, _I, _I]),
+    "fd_op_attention": (_I, [_I, _I, _I, _P, _P, _P, _I, _I, _P, _I, _P, _P, _P]),
     "fd_op_kv_append": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _P, _P]),
     "fd_op_rmsnorm": (_I, [_P, _P, _I, _I, _F, _P, _P]),
     "fd_op_unshuffle": (_I, [_P, _I, _I, _I, _I, _P, _P]),
@@ -274,12 +275,16 @@ def op_qkv(A, Wqkv, bqkv, knorm_g, vnorm_g, heads, groups, tokens, grid_w, frame
                            _ptr(err), _stream_ptr(stream)), "fd_op_qkv")
 
 
-def op_attention(q, k_ring, vt_ring, heads, groups, ring_pitch, n_keys, out, err=None,
-                 stream=None) -> None:
+def attention_workspace_bytes(Lq, heads, groups, n_keys, splits=0) -> int:
+    return lib().fd_attention_workspace_bytes(Lq, heads, groups, n_keys, splits)
+
+
+def op_attention(q, k_ring, vt_ring, heads, groups, ring_pitch, n_keys, out, splits=0,
+                 workspace=None, err=None, stream=None) -> None:
     Lq = q.shape[0]
     _check(lib().fd_op_attention(Lq, heads, groups, _ptr(q), _ptr(k_ring), _ptr(vt_ring),
-                                 ring_pitch, n_keys, _ptr(out), _ptr(err), _stream_ptr(stream)),
-           "fd_op_attention")
+                                 ring_pitch, n_keys, _ptr(out), splits, _ptr(workspace),
+                                 _ptr(err), _stream_ptr(stream)), "fd_op_attention")
 
 
 def op_kv_append(k, v, window, t, ring_pitch, k_ring, vt_ring, stream=None) -> None:

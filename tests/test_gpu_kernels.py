@@ -147,28 +147,33 @@ def attention_case(Lq, heads, groups, pitch, n_keys, seed, qscale=1.5):
     return q, k, v
 
 
-def run_attention(q, k, v, heads, groups, pitch, n_keys):
+def run_attention(q, k, v, heads, groups, pitch, n_keys, splits=0):
     Lq = q.shape[0]
     out = torch.zeros(Lq, heads * 64, dtype=torch.bfloat16, device="cuda")
     vt = np.ascontiguousarray(np.transpose(v, (0, 2, 1)))
+    ws_bytes = fdp.attention_workspace_bytes(Lq, heads, groups, n_keys, splits)
+    ws = torch.full((max(1, ws_bytes // 4),), float("nan"), device="cuda")
     err = err_word()
     fdp.op_attention(dev(q, torch.bfloat16), dev(k, torch.bfloat16), dev(vt, torch.bfloat16),
-                     heads, groups, pitch, n_keys, out, err=err)
+                     heads, groups, pitch, n_keys, out, splits=splits, workspace=ws, err=err)
     check_err(err)
     return out.float().cpu()
 
 
-@pytest.mark.parametrize("Lq,heads,groups,n_keys", [
-    (520, 4, 2, 520),       # one chunk, ragged query tail
-    (520, 4, 2, 1300),      # ragged last key block
-    (130, 4, 1, 390),       # multi-query (G = 1)
-    (128, 4, 4, 128),       # MHA (G = N), exactly one block
-    (64, 2, 1, 1),          # a single key
+@pytest.mark.parametrize("Lq,heads,groups,n_keys,splits", [
+    (520, 4, 2, 520, 1),      # one chunk, ragged query tail
+    (520, 4, 2, 1300, 1),     # ragged last key block
+    (520, 4, 2, 1300, 3),     # key range split in 3, partials combined
+    (130, 4, 1, 390, 2),      # multi-query (G = 1)
+    (128, 4, 4, 128, 1),      # MHA (G = N): N/G odd, query tiles paired, second tile empty
+    (128, 4, 4, 128, 2),      # one key block split in 2: the second split is empty
+    (300, 3, 3, 700, 0),      # N/G = 1 with 3 query tiles: last pair half out of range
+    (64, 2, 1, 1, 1),         # a single key
 ])
-def test_attention_small(Lq, heads, groups, n_keys):
+def test_attention_small(Lq, heads, groups, n_keys, splits):
     pitch = max(128, -(-n_keys // 128) * 128 + 128)
     q, k, v = attention_case(Lq, heads, groups, pitch, n_keys, seed=Lq + n_keys)
-    got = run_attention(q, k, v, heads, groups, pitch, n_keys)
+    got = run_attention(q, k, v, heads, groups, pitch, n_keys, splits)
     qh = f64(q).reshape(Lq, heads, 64).transpose(0, 1)
     want = oracle.attention(qh, f64(k)[:, :n_keys], f64(v)[:, :n_keys])
     assert_close_scaled(got.reshape(Lq, heads, 64).transpose(0, 1), want, 1.5e-2, "attention")
