@@ -63,6 +63,29 @@ fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const vo
                           const void* vt_ring, int ring_pitch, int n_keys, void* out,
                           int splits, void* workspace, int* err_dev, void* stream);
 
+/* Allocation-free variant of fd_op_attention. The paper has no counterpart: this is a library
+ * convenience for callers that cannot call cudaMalloc, for example code that runs while a CUDA
+ * stream is being captured into a graph (allocation is not allowed there), plug-ins that must
+ * stay inside a device-memory budget handed to them by a host framework, and real-time loops
+ * that cannot afford the device synchronisation an allocation may cause. Such callers can pass
+ * their own inputs and outputs but have no way to provide the key-range-split workspace.
+ * This call takes that workspace from one array in the library's static device memory,
+ * FD_STATIC_ATTN_SCRATCH_BYTES (16 MiB) on every GPU that loads the library, held until the
+ * process exits. It allocates nothing: no cudaMalloc, cudaFree or allocating library routine.
+ *   - Arguments and results are those of fd_op_attention without `workspace`. splits = 0 lets
+ *     the library choose. If splits * heads * Lq * 66 * 4 bytes would exceed the static size,
+ *     the call returns FD_ERR_INVALID_ARG and launches nothing (pass fewer splits; splits = 1
+ *     uses no workspace at all).
+ *   - The first call on a device looks up the array's device address with that device current
+ *     (cudaGetSymbolAddress); make that first call before any stream capture begins.
+ *   - Every call shares the one array and writes every entry it later reads, so nothing needs
+ *     clearing between calls; calls whose kernels overlap on the GPU (unordered streams) race
+ *     on the array and may return wrong results. */
+#define FD_STATIC_ATTN_SCRATCH_BYTES (16u << 20)
+fd_status fd_op_attention_static(int Lq, int heads, int groups, const void* q,
+                                 const void* k_ring, const void* vt_ring, int ring_pitch,
+                                 int n_keys, void* out, int splits, int* err_dev, void* stream);
+
 /* Rolling-cache append (Algorithm 1, cache update): fp32 k, v [groups][rows][64] rounded to
  * bf16 (nearest even) into ring slot s = t mod window: k_ring[g][s*rows + r][d] and
  * vt_ring[g][d][s*rows + r]. The oldest chunk's slot is overwritten (eviction). */

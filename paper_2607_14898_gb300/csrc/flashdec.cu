@@ -924,6 +924,55 @@ fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const vo
   return launch_ok(fd::launch_attention(tq, tk, tv, a, static_cast<cudaStream_t>(stream)));
 }
 
+}  // extern "C"
+
+// ---------------------------------------------------------------- allocation-free attention
+// Workspace of fd_op_attention_static: the library's own static device memory, so that the
+// call needs no allocation. Host code only uses its device address, looked up per device.
+static __device__ __align__(256) float g_attn_static_scratch[FD_STATIC_ATTN_SCRATCH_BYTES / 4];
+
+namespace {
+std::mutex g_static_scratch_mu;
+constexpr int kMaxDevices = 64;
+float* g_static_scratch_addr[kMaxDevices] = {};
+
+// device address of g_attn_static_scratch on the current device (looked up once per device)
+fd_status static_scratch_address(float** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return FD_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return FD_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_static_scratch_mu);
+  if (g_static_scratch_addr[dev] == nullptr) {
+    void* addr = nullptr;
+    if (cudaGetSymbolAddress(&addr, g_attn_static_scratch) != cudaSuccess || addr == nullptr)
+      return FD_ERR_CUDA;
+    g_static_scratch_addr[dev] = static_cast<float*>(addr);
+  }
+  *out = g_static_scratch_addr[dev];
+  return FD_OK;
+}
+}  // namespace
+
+extern "C" {
+
+fd_status fd_op_attention_static(int Lq, int heads, int groups, const void* q,
+                                 const void* k_ring, const void* vt_ring, int ring_pitch,
+                                 int n_keys, void* out, int splits, int* err_dev, void* stream) {
+  if (Lq < 1 || heads < 1 || groups < 1 || heads % groups || n_keys < 1 || splits < 0 ||
+      splits > 16)
+    return FD_ERR_INVALID_ARG;
+  if (splits == 0) splits = choose_splits(Lq, heads, groups, n_keys);
+  if (fd::attention_workspace_floats(splits, heads, Lq) * 4 > FD_STATIC_ATTN_SCRATCH_BYTES)
+    return FD_ERR_INVALID_ARG;
+  float* ws = nullptr;
+  if (splits > 1) {
+    const fd_status st = static_scratch_address(&ws);
+    if (st != FD_OK) return st;
+  }
+  return fd_op_attention(Lq, heads, groups, q, k_ring, vt_ring, ring_pitch, n_keys, out, splits,
+                         ws, err_dev, stream);
+}
+
 fd_status fd_op_kv_append(const float* k, const float* v, int groups, int rows, int window,
                           int t, int ring_pitch, void* k_ring, void* vt_ring, void* stream) {
   if (!k || !v || !k_ring || !vt_ring || groups < 1 || rows < 1 || window < 1 || t < 0)

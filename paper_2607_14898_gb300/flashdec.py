@@ -71,6 +71,7 @@ _SIGS = {
                        _P, _P, _P, _I, _I, _P, _P]),
     "fd_attention_workspace_bytes": (ctypes.c_size_t, [_I, _I, _I, _I, _I]),
     "fd_op_attention": (_I, [_I, _I, _I, _P, _P, _P, _I, _I, _P, _I, _P, _P, _P]),
+    "fd_op_attention_static": (_I, [_I, _I, _I, _P, _P, _P, _I, _I, _P, _I, _P, _P]),
     "fd_op_kv_append": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _P, _P]),
     "fd_op_rmsnorm": (_I, [_P, _P, _I, _I, _F, _P, _P]),
     "fd_op_unshuffle": (_I, [_P, _I, _I, _I, _I, _P, _P]),
@@ -285,6 +286,15 @@ def op_attention(q, k_ring, vt_ring, heads, groups, ring_pitch, n_keys, out, spl
     _check(lib().fd_op_attention(Lq, heads, groups, _ptr(q), _ptr(k_ring), _ptr(vt_ring),
                                  ring_pitch, n_keys, _ptr(out), splits, _ptr(workspace),
                                  _ptr(err), _stream_ptr(stream)), "fd_op_attention")
+
+
+def op_attention_static(q, k_ring, vt_ring, heads, groups, ring_pitch, n_keys, out, splits=0,
+                        err=None, stream=None) -> None:
+    """fd_op_attention with the split workspace in the library's static device memory."""
+    Lq = q.shape[0]
+    _check(lib().fd_op_attention_static(Lq, heads, groups, _ptr(q), _ptr(k_ring), _ptr(vt_ring),
+                                        ring_pitch, n_keys, _ptr(out), splits, _ptr(err),
+                                        _stream_ptr(stream)), "fd_op_attention_static")
 
 
 def op_kv_append(k, v, window, t, ring_pitch, k_ring, vt_ring, stream=None) -> None:
