@@ -163,7 +163,7 @@ const char* fd_status_str(fd_status s);
 typedef enum {
   FD_K_UNSHUFFLE = 0, FD_K_EMBED = 1, FD_K_RMSNORM = 2, FD_K_QKV = 3, FD_K_ATTN_B = 4,
   FD_K_ATTN_R = 5, FD_K_OUT = 6, FD_K_MLP1 = 7, FD_K_MLP2 = 8, FD_K_TUP = 9, FD_K_HEAD1 = 10,
-  FD_K_HEAD2 = 11, FD_K_PIXEL = 12, FD_K_ADVANCE = 13, FD_K_COUNT = 14
+  FD_K_HEAD2 = 11, FD_K_PIXEL = 12, FD_K_ADVANCE = 13, FD_K_ROPE = 14, FD_K_COUNT = 15
 } fd_kernel_kind;
 
 /* Per-kernel profile (tracing): while enabled, every kernel the handle launches is bracketed

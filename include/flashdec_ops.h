@@ -30,24 +30,32 @@ typedef enum {
 /* Linear layer on the tensor cores (tcgen05, bf16 in, fp32 accumulate).
  * A bf16 [M][K] row-major; W bf16 [N][K] row-major (nn.Linear); bias fp32 [N].
  * Requires N % 32 == 0, K % 8 == 0, 16-byte aligned A / W / out. bn = output tile width
- * (64, 128 or 256; 0 = library choice). */
+ * (64, 128, 192 or 256; 0 = library choice). */
 fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const void* W,
                        const float* bias, void* out, int tup_hidden, int bn, int* err_dev,
                        void* stream);
 
+/* Temporal 3D-RoPE table of chunk t (Sec. 3.2, reading of Algorithm 1's "RoPE offset"):
+ * table[tau][i] = (cos, sin)((t * frames_per_chunk + tau) * rope_base^(-2i/24)) for the
+ * frames_per_chunk frames of the chunk and the 12 temporal pairs (fp32 values of an fp64
+ * evaluation). table: device float [frames_per_chunk][12][2]. */
+fd_status fd_op_rope_table(int t, int frames_per_chunk, float rope_base, float* table,
+                           void* stream);
+
 /* Fused QKV projection of one attention block (Sec. 3.2, Sec. 3.3 step (2)):
  *   [Q | K | V] = A Wqkv^T + b   (Wqkv rows: heads*64 query, groups*64 key, groups*64 value)
  *   K, V <- RMSNorm over the 64 head dims with gains knorm_g / vnorm_g (KV-norm)
- *   Q, K <- 3D-RoPE at temporal index t*frames_per_chunk + row / tokens, row and column of
- *           token (row % tokens) in a grid of width grid_w (rope_base; bands 24/20/20 dims)
+ *   Q, K <- 3D-RoPE at temporal index t*frames_per_chunk + row / tokens (cos / sin from
+ *           rope_t, the fd_op_rope_table of chunk t), row and column of token (row % tokens)
+ *           in a grid of width grid_w (rope_base; bands 24/20/20 dims)
  *   q_out bf16 [M][heads*64];  K -> k_ring bf16 [groups][ring_pitch][64] rows
  *   (t mod window)*M + row;  V -> vt_ring bf16 [groups][64][ring_pitch] (transposed), same
  *   key index.  M = frames_per_chunk * tokens; ring_pitch % 128 == 0, >= window * M. */
 fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* bqkv,
                     const float* knorm_g, const float* vnorm_g, int heads, int groups,
                     int tokens, int grid_w, int frames_per_chunk, int window, int t, float eps,
-                    float rope_base, void* q_out, void* k_ring, void* vt_ring, int ring_pitch,
-                    int bn, int* err_dev, void* stream);
+                    float rope_base, const float* rope_t, void* q_out, void* k_ring,
+                    void* vt_ring, int ring_pitch, int bn, int* err_dev, void* stream);
 
 /* Attention of Lq queries over the first n_keys keys of a ring (Sec. 3.3, Eq. kv_cache):
  *   out[r][n*64 + d] = sum_j softmax_j(q_n . k_j / 8) v_j[d],  KV group g = n / (heads/groups)

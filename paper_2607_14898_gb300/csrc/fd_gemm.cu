@@ -7,8 +7,11 @@
 //   warp 1 (one lane)  MMA issuer: 4 x tcgen05.mma (K = 16 each) per stage into a TMEM
 //                      accumulator; two accumulators so the epilogue of tile i overlaps the
 //                      MMAs of tile i+1
-//   warps 2-5          epilogue: each thread owns one accumulator row (TMEM lane) and
-//                      applies the fused epilogue while storing it
+//   warps 2-5          epilogue: each thread owns one accumulator row (TMEM lane), applies
+//                      the fused epilogue, and writes its row of a 32-row slab into a
+//                      128-byte-swizzled staging buffer; one lane then stores the slab with a
+//                      TMA bulk tensor store (a bulk reduce-add for the residual), so global
+//                      writes are whole lines and rows past M are clipped by the tensor map
 // Fused epilogues (the linear layers of Sec. 3.2 / 3.4 and Eq. projection / temporal_upsample):
 //   EPI_F32    out = acc + b                    (patch-embed, head layer 2)
 //   EPI_RESID  h  += acc + b                    (out-projection, MLP layer 2: residual)
@@ -23,37 +26,57 @@ namespace fd {
 
 template <int BN>
 struct GemmCfg {
-  static constexpr int kStages = BN >= 256 ? 4 : 6;
+  static constexpr int kStages = BN >= 192 ? 4 : 6;
   static constexpr int kABytes = kBM * kBK * 2;  // 16 KB
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kTmemCols = 2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512);
-  static constexpr int kBarOffset = kStages * kStageBytes;
+  static constexpr int kStgOffset = kStages * kStageBytes;   // 4 warps x 2 x 4 KB staging
+  static constexpr int kBarOffset = kStgOffset + 4 * 2 * 4096;
   static constexpr int kSmem = kBarOffset + 256;
   static_assert(kSmem <= 227 * 1024, "shared memory");
 };
+
+// one 128-byte row (8 x 16 B) of a 32-row slab in the 128-byte-swizzled layout of a TMA box
+__device__ __forceinline__ void put_row_sw128(uint8_t* buf, int row, const uint32_t* w) {
+#pragma unroll
+  for (int k = 0; k < 8; ++k)
+    *reinterpret_cast<uint4*>(buf + row * 128 + ((k ^ (row & 7)) << 4)) =
+        make_uint4(w[4 * k], w[4 * k + 1], w[4 * k + 2], w[4 * k + 3]);
+}
 
 __device__ __forceinline__ float gelu_erf(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
 }
 
-// cos / sin of the 32 rotation pairs of one token (3D-RoPE, reading: temporal pairs first,
-// then row, then column; angle = position * base^(-2i/d_band)), argument reduced in fp64.
-__device__ __forceinline__ void rope_table(const QkvEpi& q, int f, int y, int x, float* c,
+// cos / sin of the 32 rotation pairs of one token (3D-RoPE: temporal pairs first, then row,
+// then column; angle = position * base^(-2i/d_band)). Temporal values come from the chunk's
+// table (fp64-evaluated, any stream length); row / column angles are below 2^12 rad, reduced to
+// [-pi, pi] in fp32 (2 pi split in two parts) and evaluated with the fast sin / cos.
+__device__ __forceinline__ void rope_table(const QkvEpi& q, int tau, int y, int x, float* c,
                                            float* s) {
 #pragma unroll
   for (int i = 0; i < kRopePairs; ++i) {
-    const int pos = i < q.band_t ? f : (i < q.band_t + q.band_s ? y : x);
-    double a = static_cast<double>(pos) * q.inv_freq[i];
-    a -= 6.283185307179586 * rint(a * 0.15915494309189535);
-    sincosf(static_cast<float>(a), &s[i], &c[i]);
+    if (i < q.band_t) {
+      const float2 v = __ldg(q.rope_t + tau * q.band_t + i);
+      c[i] = v.x;
+      s[i] = v.y;
+    } else {
+      const int pos = i < q.band_t + q.band_s ? y : x;
+      const float a = static_cast<float>(pos) * q.inv_freq_s[i];
+      const float k = rintf(a * 0.159154943091895336f);
+      float r = fmaf(-k, 6.28318548202514648f, a);
+      r = fmaf(-k, -1.74845553e-7f, r);
+      __sincosf(r, &s[i], &c[i]);
+    }
   }
 }
 
 template <int BN>
 __global__ void __launch_bounds__(192, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                const __grid_constant__ GemmParams p) {
+                const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmK,
+                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ GemmParams p) {
   using C = GemmCfg<BN>;
   extern __shared__ __align__(1024) uint8_t smem[];
   const int warp = threadIdx.x >> 5;
@@ -150,6 +173,27 @@ __global__ void __launch_bounds__(192, 1)
     // ------------------------------------------------------------ epilogue
     const int quarter = warp & 3;  // TMEM lanes this warp may read
     const int rloc = quarter * 32 + lane;
+    uint8_t* stg = smem + C::kStgOffset + (warp - 2) * 8192;
+    int sb = 0;
+    // a free 4 KB staging buffer: the store issued from it two stores ago has read it
+    auto acquire = [&]() -> uint8_t* {
+      if (lane == 0) bulk_wait_read_1();
+      __syncwarp();
+      uint8_t* b = stg + sb * 4096;
+      sb ^= 1;
+      return b;
+    };
+    auto publish = [&]() {  // make the slab visible to the TMA engine
+      fence_proxy_async_smem();
+      __syncwarp();
+    };
+    if (lane == 0) {
+      prefetch_tmap(&tmO);
+      if (p.epi == EPI_QKV) {
+        prefetch_tmap(&tmK);
+        if (p.v_tma) prefetch_tmap(&tmV);
+      }
+    }
     int t = 0;
     if (p.epi == EPI_QKV) t = p.qkv.step_dev ? *p.qkv.step_dev : p.qkv.step_host;
     int tc = 0;
@@ -160,6 +204,7 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_after();
       const int m0 = (tile / n_tiles) * kBM;
       const int n0 = (tile % n_tiles) * BN;
+      const int row0 = m0 + quarter * 32;  // first row of this warp's slab
       const int row = m0 + rloc;
       const bool row_ok = row < p.M;
       const uint32_t tbase =
@@ -172,18 +217,17 @@ __global__ void __launch_bounds__(192, 1)
         const int slot = t % q.window;
         if (row_ok) {
           const int l = row % q.tokens;
-          const int f = t * q.frames_per_chunk + row / q.tokens;
-          rope_table(q, f, l / q.grid_w, l % q.grid_w, rc, rsn);
+          rope_table(q, row / q.tokens, l / q.grid_w, l % q.grid_w, rc, rsn);
         }
 #pragma unroll 1
         for (int c = 0; c < BN; c += 64) {
+          const int col = n0 + c;
+          if (col >= p.N) break;  // warp-uniform
           uint32_t r0[32], r1[32];
           __syncwarp();  // tcgen05.ld is warp-collective: reconverge first
           tmem_ld_32x32b_x32(tbase + c, r0);
           tmem_ld_32x32b_x32(tbase + c + 32, r1);
           tmem_ld_wait();
-          const int col = n0 + c;
-          if (!row_ok || col >= p.N) continue;
           float v[64];
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
@@ -209,28 +253,32 @@ __global__ void __launch_bounds__(192, 1)
               v[2 * i] = a * rc[i] - b * rsn[i];
               v[2 * i + 1] = a * rsn[i] + b * rc[i];
             }
-          }
-          if (is_q) {
-            uint4* dst = reinterpret_cast<uint4*>(q.q_out + static_cast<size_t>(row) *
-                                                                (q.heads * kHeadDim) +
-                                                  hidx * kHeadDim);
+            uint32_t w[32];
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
-              dst[j] = make_uint4(pack_bf16x2(v[8 * j], v[8 * j + 1]),
-                                  pack_bf16x2(v[8 * j + 2], v[8 * j + 3]),
-                                  pack_bf16x2(v[8 * j + 4], v[8 * j + 5]),
-                                  pack_bf16x2(v[8 * j + 6], v[8 * j + 7]));
-          } else if (is_k) {
-            const int g = hidx - q.heads;
-            const size_t krow = static_cast<size_t>(g) * q.ring_pitch + slot * rows_chunk + row;
-            uint4* dst = reinterpret_cast<uint4*>(q.k_ring + krow * kHeadDim);
+            for (int j = 0; j < 32; ++j) w[j] = pack_bf16x2(v[2 * j], v[2 * j + 1]);
+            uint8_t* buf = acquire();
+            put_row_sw128(buf, lane, w);
+            publish();
+            if (lane == 0 && row0 < p.M) {  // a slab wholly past M stores nothing
+              if (is_q) {
+                tma_store_2d(&tmO, smem_u32(buf), hidx * kHeadDim, row0);
+              } else {
+                tma_store_4d(&tmK, smem_u32(buf), 0, row0, slot, hidx - q.heads);
+              }
+              bulk_commit();
+            }
+          } else if (p.v_tma) {
+            // V transposed: slab [64 dims][32 keys] bf16, stored into the ring's V^T slot view
+            uint8_t* buf = acquire();
+            __nv_bfloat16* sv = reinterpret_cast<__nv_bfloat16*>(buf);
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
-              dst[j] = make_uint4(pack_bf16x2(v[8 * j], v[8 * j + 1]),
-                                  pack_bf16x2(v[8 * j + 2], v[8 * j + 3]),
-                                  pack_bf16x2(v[8 * j + 4], v[8 * j + 5]),
-                                  pack_bf16x2(v[8 * j + 6], v[8 * j + 7]));
-          } else {
+            for (int j = 0; j < 64; ++j) sv[j * 32 + lane] = __float2bfloat16_rn(v[j]);
+            publish();
+            if (lane == 0 && row0 < p.M) {
+              tma_store_4d(&tmV, smem_u32(buf), row0, slot, 0, hidx - q.heads - q.groups);
+              bulk_commit();
+            }
+          } else if (row_ok) {
             const int g = hidx - q.heads - q.groups;
             __nv_bfloat16* dst = q.vt_ring + static_cast<size_t>(g) * kHeadDim * q.ring_pitch +
                                  slot * rows_chunk + row;
@@ -239,52 +287,60 @@ __global__ void __launch_bounds__(192, 1)
               dst[static_cast<size_t>(j) * q.ring_pitch] = __float2bfloat16_rn(v[j]);
           }
         }
-      } else {
+      } else if (p.epi == EPI_GELU) {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 64) {
+          const int col = n0 + c;
+          if (col >= p.N) break;
+          uint32_t r0[32], r1[32];
+          __syncwarp();
+          tmem_ld_32x32b_x32(tbase + c, r0);
+          tmem_ld_32x32b_x32(tbase + c + 32, r1);
+          tmem_ld_wait();
+          uint32_t w[32];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            w[j] = pack_bf16x2(gelu_erf(__uint_as_float(r0[2 * j]) + __ldg(p.bias + col + 2 * j)),
+                               gelu_erf(__uint_as_float(r0[2 * j + 1]) +
+                                        __ldg(p.bias + col + 2 * j + 1)));
+            w[16 + j] = pack_bf16x2(
+                gelu_erf(__uint_as_float(r1[2 * j]) + __ldg(p.bias + col + 32 + 2 * j)),
+                gelu_erf(__uint_as_float(r1[2 * j + 1]) + __ldg(p.bias + col + 33 + 2 * j)));
+          }
+          uint8_t* buf = acquire();
+          put_row_sw128(buf, lane, w);
+          publish();
+          if (lane == 0 && row0 < p.M) {
+            tma_store_2d(&tmO, smem_u32(buf), col, row0);
+            bulk_commit();
+          }
+        }
+      } else {  // EPI_F32, EPI_RESID, EPI_TUP: fp32 slabs of 32 columns
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
+          const int col = n0 + c;
+          if (col >= p.N) break;
           uint32_t r[32];
-          __syncwarp();  // tcgen05.ld is warp-collective: reconverge first
+          __syncwarp();
           tmem_ld_32x32b_x32(tbase + c, r);
           tmem_ld_wait();
-          const int col = n0 + c;
-          if (!row_ok || col >= p.N) continue;
-          float v[32];
+          uint32_t w[32];
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]) + __ldg(p.bias + col + j);
-          if (p.epi == EPI_GELU) {
-            uint4* dst =
-                reinterpret_cast<uint4*>(p.out_bf16 + static_cast<size_t>(row) * p.ld_out + col);
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              dst[j] = make_uint4(pack_bf16x2(gelu_erf(v[8 * j]), gelu_erf(v[8 * j + 1])),
-                                  pack_bf16x2(gelu_erf(v[8 * j + 2]), gelu_erf(v[8 * j + 3])),
-                                  pack_bf16x2(gelu_erf(v[8 * j + 4]), gelu_erf(v[8 * j + 5])),
-                                  pack_bf16x2(gelu_erf(v[8 * j + 6]), gelu_erf(v[8 * j + 7])));
-          } else {
-            float* dst;
-            if (p.epi == EPI_TUP) {
-              const int tau = col / p.tup_hidden;
-              dst = p.out_f32 + (static_cast<size_t>(tau) * p.tup_tokens + row) * p.tup_hidden +
-                    (col - tau * p.tup_hidden);
-            } else {
-              dst = p.out_f32 + static_cast<size_t>(row) * p.ld_out + col;
-            }
-            float4* d4 = reinterpret_cast<float4*>(dst);
+          for (int j = 0; j < 32; ++j)
+            w[j] = __float_as_uint(__uint_as_float(r[j]) + __ldg(p.bias + col + j));
+          uint8_t* buf = acquire();
+          put_row_sw128(buf, lane, w);
+          publish();
+          if (lane == 0 && row0 < p.M) {
             if (p.epi == EPI_RESID) {
-#pragma unroll
-              for (int j = 0; j < 8; ++j) {
-                float4 o = d4[j];
-                o.x += v[4 * j];
-                o.y += v[4 * j + 1];
-                o.z += v[4 * j + 2];
-                o.w += v[4 * j + 3];
-                d4[j] = o;
-              }
+              tma_reduce_add_2d(&tmO, smem_u32(buf), col, row0);
+            } else if (p.epi == EPI_TUP) {
+              const int tau = col / p.tup_hidden;
+              tma_store_3d(&tmO, smem_u32(buf), col - tau * p.tup_hidden, row0, tau);
             } else {
-#pragma unroll
-              for (int j = 0; j < 8; ++j)
-                d4[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+              tma_store_2d(&tmO, smem_u32(buf), col, row0);
             }
+            bulk_commit();
           }
         }
       }
@@ -292,6 +348,8 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_before();
       mbar_arrive(bar_tempty + 8 * acc);
     }
+    if (lane == 0) bulk_wait_all();  // every store has landed before the CTA exits
+    __syncwarp();
   }
   tc_fence_before();
   __syncthreads();
@@ -302,8 +360,10 @@ __global__ void __launch_bounds__(192, 1)
 }
 
 template <int BN>
-static cudaError_t launch_bn(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p,
-                             int num_sms, cudaStream_t s) {
+static cudaError_t launch_bn(const CUtensorMap& tmA, const CUtensorMap& tmB,
+                             const CUtensorMap& tmO, const CUtensorMap& tmK,
+                             const CUtensorMap& tmV, const GemmParams& p, int num_sms,
+                             cudaStream_t s) {
   using C = GemmCfg<BN>;
   static bool attr_set = false;
   if (!attr_set) {
@@ -314,16 +374,18 @@ static cudaError_t launch_bn(const CUtensorMap& tmA, const CUtensorMap& tmB, con
   }
   const int tiles = ((p.M + kBM - 1) / kBM) * ((p.N + BN - 1) / BN);
   const int grid = tiles < num_sms ? tiles : num_sms;
-  gemm_kernel<BN><<<grid, 192, C::kSmem, s>>>(tmA, tmB, p);
+  gemm_kernel<BN><<<grid, 192, C::kSmem, s>>>(tmA, tmB, tmO, tmK, tmV, p);
   return cudaGetLastError();
 }
 
-cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p,
+cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmO,
+                        const CUtensorMap& tmK, const CUtensorMap& tmV, const GemmParams& p,
                         int bn, int num_sms, cudaStream_t s) {
   switch (bn) {
-    case 64: return launch_bn<64>(tmA, tmB, p, num_sms, s);
-    case 128: return launch_bn<128>(tmA, tmB, p, num_sms, s);
-    case 256: return launch_bn<256>(tmA, tmB, p, num_sms, s);
+    case 64: return launch_bn<64>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+    case 128: return launch_bn<128>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+    case 192: return launch_bn<192>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+    case 256: return launch_bn<256>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
     default: return cudaErrorInvalidValue;
   }
 }

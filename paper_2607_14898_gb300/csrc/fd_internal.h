@@ -38,12 +38,23 @@ struct QkvEpi {
   int step_host;
   float eps;
   int band_t, band_s;        // pairs in the temporal band and in each spatial band
-  double inv_freq[kRopePairs];  // base^(-2i/d_band), temporal pairs first, then row, column
+  const float2* rope_t;      // [frames_per_chunk][band_t] (cos, sin) of this chunk's frames
+  float inv_freq_s[kRopePairs];  // base^(-2i/d_band) of the row / column pairs (fp32)
 };
 
+// Output of the GEMM epilogue goes through TMA bulk stores with these tensor maps (all boxes
+// are 32-row slabs, 128-byte swizzled unless noted):
+//   EPI_F32 / EPI_RESID  tmO: fp32 [M][ld_out], box {32, 32} (RESID uses a bulk reduce-add)
+//   EPI_GELU             tmO: bf16 [M][ld_out], box {64, 32}
+//   EPI_TUP              tmO: fp32 3D {D, L, r_t}, box {32, 32, 1}
+//   EPI_QKV              tmO: Q bf16 [M][heads*64], box {64, 32};
+//                        tmK: K ring 4D {64, M, W, G} (row, slot, group strides), box {64,32,1,1};
+//                        tmV: V^T ring 4D {M, W, 64, G}, box {32, 1, 64, 1}, no swizzle
+//                        (used when v_tma; needs M % 8 == 0), else direct stores
 struct GemmParams {
   int M, N, K;
   int epi;
+  int v_tma;
   const float* bias;         // [N]
   float* out_f32;            // EPI_F32 / EPI_RESID / EPI_TUP
   int ld_out;                // row pitch of out_f32 / out_bf16 (elements)
@@ -72,7 +83,8 @@ struct AttnParams {
 };
 
 // launch wrappers; return cudaGetLastError() of the launch
-cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p,
+cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmO,
+                        const CUtensorMap& tmK, const CUtensorMap& tmV, const GemmParams& p,
                         int bn, int num_sms, cudaStream_t s);
 // Attention (+ the combine of key-range splits when p.splits > 1).
 cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmK,
@@ -93,8 +105,17 @@ cudaError_t launch_kv_append(const float* k, const float* v, int groups, int row
                              int ring_pitch, __nv_bfloat16* k_ring, __nv_bfloat16* vt_ring,
                              cudaStream_t s);
 cudaError_t launch_advance(int* step_dev, cudaStream_t s);
+// Temporal RoPE table of one chunk: for each block of `frames[k]` frames per chunk (k < nsets),
+// entries [off_k + tau][i] = (cos, sin)((t * frames[k] + tau) * inv_freq[i]), i < band_t,
+// computed in fp64 (t read from step_dev, or t_host when step_dev is null).
+cudaError_t launch_rope_table(const int* step_dev, int t_host, int nsets, const int* frames,
+                              int band_t, const double* inv_freq, float2* table,
+                              cudaStream_t s);
+constexpr int kMaxRopeSets = 2;
 
 // GEMM tile widths compiled in
-inline bool gemm_bn_supported(int bn) { return bn == 64 || bn == 128 || bn == 256; }
+inline bool gemm_bn_supported(int bn) {
+  return bn == 64 || bn == 128 || bn == 192 || bn == 256;
+}
 
 }  // namespace fd

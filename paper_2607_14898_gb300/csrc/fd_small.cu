@@ -120,6 +120,29 @@ __global__ void kv_append_kernel(const float* __restrict__ k, const float* __res
 
 __global__ void advance_kernel(int* step) { *step += 1; }
 
+struct RopeSets {
+  int frames[kMaxRopeSets];
+  double inv_freq[kRopePairs];
+};
+
+// one thread per (set, frame, pair): angles reduced and evaluated in fp64, stored as fp32
+__global__ void rope_table_kernel(const int* step_dev, int t_host, int nsets, int band_t,
+                                  RopeSets sets, float2* table) {
+  const int t = step_dev ? *step_dev : t_host;
+  int off = 0;
+  for (int k = 0; k < nsets; ++k) {
+    const int n = sets.frames[k] * band_t;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+      const int tau = i / band_t, pair = i - tau * band_t;
+      const double f = static_cast<double>(t) * sets.frames[k] + tau;
+      double sn, cs;
+      sincos(f * sets.inv_freq[pair], &sn, &cs);
+      table[off + i] = make_float2(static_cast<float>(cs), static_cast<float>(sn));
+    }
+    off += n;
+  }
+}
+
 static int grid_for(long long work, int threads) {
   long long b = (work + threads - 1) / threads;
   if (b > 152LL * 16) b = 152LL * 16;
@@ -151,6 +174,18 @@ cudaError_t launch_kv_append(const float* k, const float* v, int groups, int row
                              cudaStream_t s) {
   dim3 grid((rows + 31) / 32, groups);
   kv_append_kernel<<<grid, dim3(32, 8), 0, s>>>(k, v, rows, slot, ring_pitch, k_ring, vt_ring);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rope_table(const int* step_dev, int t_host, int nsets, const int* frames,
+                              int band_t, const double* inv_freq, float2* table,
+                              cudaStream_t s) {
+  if (nsets < 1 || nsets > kMaxRopeSets || band_t < 1 || band_t > kRopePairs)
+    return cudaErrorInvalidValue;
+  RopeSets sets{};
+  for (int k = 0; k < nsets; ++k) sets.frames[k] = frames[k];
+  for (int i = 0; i < band_t; ++i) sets.inv_freq[i] = inv_freq[i];
+  rope_table_kernel<<<1, 128, 0, s>>>(step_dev, t_host, nsets, band_t, sets, table);
   return cudaGetLastError();
 }
 

@@ -51,6 +51,63 @@ bool tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// N-d tensor map (rank <= 5): dims innermost first, strides in bytes for dims 1..rank-1
+bool tmap_nd(CUtensorMap* m, CUtensorMapDataType dt, int rank, const void* base,
+             const uint64_t* dims, const uint64_t* strides, const uint32_t* box,
+             CUtensorMapSwizzle sw) {
+  if (!load_encode()) return false;
+  cuuint64_t d[5], st[4];
+  cuuint32_t b[5], es[5];
+  for (int i = 0; i < rank; ++i) {
+    d[i] = dims[i];
+    b[i] = box[i];
+    es[i] = 1;
+    if (i > 0) st[i - 1] = strides[i - 1];
+  }
+  return g_encode(m, dt, rank, const_cast<void*>(base), d, st, b, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// GEMM epilogue store maps (32-row slabs)
+bool tmap_out_f32(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t ld) {
+  const uint64_t dims[2] = {cols, rows}, strides[1] = {ld * 4};
+  const uint32_t box[2] = {32, 32};
+  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box,
+                 CU_TENSOR_MAP_SWIZZLE_128B);
+}
+bool tmap_out_bf16(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t ld) {
+  const uint64_t dims[2] = {cols, rows}, strides[1] = {ld * 2};
+  const uint32_t box[2] = {64, 32};
+  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box,
+                 CU_TENSOR_MAP_SWIZZLE_128B);
+}
+// temporal upsampling output viewed as [r_t][L][D]
+bool tmap_out_tup(CUtensorMap* m, const void* base, uint64_t D, uint64_t L, uint64_t rt) {
+  const uint64_t dims[3] = {D, L, rt}, strides[2] = {D * 4, L * D * 4};
+  const uint32_t box[3] = {32, 32, 1};
+  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base, dims, strides, box,
+                 CU_TENSOR_MAP_SWIZZLE_128B);
+}
+// K ring [G][pitch][64] viewed as {64, M rows of a slot, W slots, G}
+bool tmap_kring_store(CUtensorMap* m, const void* base, uint64_t M, uint64_t W, uint64_t G,
+                      uint64_t pitch) {
+  const uint64_t dims[4] = {64, M, W, G};
+  const uint64_t strides[3] = {128, M * 128, pitch * 128};
+  const uint32_t box[4] = {64, 32, 1, 1};
+  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, base, dims, strides, box,
+                 CU_TENSOR_MAP_SWIZZLE_128B);
+}
+// V^T ring [G][64][pitch] viewed as {M keys of a slot, W slots, 64 dims, G}; needs M % 8 == 0
+bool tmap_vring_store(CUtensorMap* m, const void* base, uint64_t M, uint64_t W, uint64_t G,
+                      uint64_t pitch) {
+  const uint64_t dims[4] = {M, W, 64, G};
+  const uint64_t strides[3] = {M * 2, pitch * 2, 64 * pitch * 2};
+  const uint32_t box[4] = {32, 1, 64, 1};
+  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, base, dims, strides, box,
+                 CU_TENSOR_MAP_SWIZZLE_NONE);
+}
+
 int g_num_sms = 0;
 int num_sms() {
   if (g_num_sms == 0) {
@@ -148,17 +205,21 @@ float bf16_to_f32(uint16_t b) {
   return f;
 }
 
-// GEMM tile width for an M x N problem: fewest "waves x width" on the SM count
+// GEMM tile width for an M x N problem: a tile costs about (128 + BN) (a fixed part plus its
+// width) and a persistent grid runs ceil(tiles / SMs) rounds; pick the cheapest, the wider tile
+// on ties. Matches the measured best width on the decoder's shapes.
 int pick_bn(int M, int N) {
   const int sms = num_sms();
   int best = 128;
   long long best_cost = -1;
-  for (int bn : {128, 256}) {
-    if (N % bn && bn != 128) continue;
+  for (int bn : {128, 192, 256}) {
     const long long tiles = static_cast<long long>((M + 127) / 128) * ((N + bn - 1) / bn);
-    const long long waves = (tiles + sms - 1) / sms;
-    const long long cost = waves * bn * 100 + bn;  // prefer the narrower tile on ties
-    if (best_cost < 0 || cost < best_cost) { best_cost = cost; best = bn; }
+    const long long rounds = (tiles + sms - 1) / sms;
+    const long long cost = rounds * (128 + bn);
+    if (best_cost < 0 || cost <= best_cost) {
+      best_cost = cost;
+      best = bn;
+    }
   }
   return best;
 }
@@ -192,7 +253,8 @@ namespace {
 struct Ring {
   __nv_bfloat16* k = nullptr;   // [G][pitch][64]
   __nv_bfloat16* vt = nullptr;  // [G][64][pitch]
-  CUtensorMap tm_k, tm_vt;
+  CUtensorMap tm_k, tm_vt;      // attention loads
+  CUtensorMap st_k, st_vt;      // QKV epilogue stores into ring slots
 };
 
 }  // namespace
@@ -216,8 +278,12 @@ struct fd_handle_s {
   // partial-result workspace
   int splitsB = 1, splitsR = 1;
   float* attn_ws = nullptr;
+  // temporal RoPE (cos, sin) of the current chunk: backbone frame, then the r_t refined frames
+  float2* rope_tab = nullptr;
   // A-operand / Q descriptors
   CUtensorMap tm_x0, tm_uB, tm_uR, tm_oB, tm_oR, tm_hidB, tm_hidR, tm_hidH, tm_qB, tm_qR;
+  // epilogue store descriptors
+  CUtensorMap so_h, so_hf, so_tup, so_hidB, so_hidR, so_hidH, so_F, so_qB, so_qR;
   // host-buffer decode: library-owned device copies of the latent and the pixels
   float* latent_buf = nullptr;
   void* pixel_buf = nullptr;
@@ -244,7 +310,15 @@ void fill_rope(fd::QkvEpi& q, float base) {
   q.band_s = kHeadDim / 6;                 // pairs per spatial band (10 at D_h = 64)
   q.band_t = kHeadDim / 2 - 2 * q.band_s;  // temporal pairs (12)
   for (int i = 0; i < fd::kRopePairs; ++i)
-    q.inv_freq[i] = rope_inv_freq(i, q.band_t, q.band_s, static_cast<double>(base));
+    q.inv_freq_s[i] =
+        static_cast<float>(rope_inv_freq(i, q.band_t, q.band_s, static_cast<double>(base)));
+}
+
+int rope_band_t() { return kHeadDim / 2 - 2 * (kHeadDim / 6); }
+
+void temporal_inv_freq(float base, double* out) {
+  const int bt = rope_band_t(), bs = kHeadDim / 6;
+  for (int i = 0; i < bt; ++i) out[i] = rope_inv_freq(i, bt, bs, static_cast<double>(base));
 }
 
 fd_status launch_ok(cudaError_t e) { return e == cudaSuccess ? FD_OK : FD_ERR_CUDA; }
@@ -287,13 +361,18 @@ int choose_splits(int Lq, int heads, int groups, int n_keys) {
 }
 
 fd_status run_linear(fd_handle h, int kind, const CUtensorMap& tmA, const Linear& lin, int M,
-                     fd::GemmParams p, cudaStream_t s) {
+                     fd::GemmParams p, const CUtensorMap& tmO, cudaStream_t s,
+                     const CUtensorMap* tmK = nullptr, const CUtensorMap* tmV = nullptr) {
   p.M = M;
   p.N = lin.N;
   p.K = lin.K;
   p.bias = lin.b;
   p.err = h->state + 1;
-  return traced(h, kind, s, [&] { return fd::launch_gemm(tmA, lin.tm, p, lin.bn, num_sms(), s); });
+  const CUtensorMap& k = tmK ? *tmK : tmO;
+  const CUtensorMap& v = tmV ? *tmV : tmO;
+  return traced(h, kind, s, [&] {
+    return fd::launch_gemm(tmA, lin.tm, tmO, k, v, p, lin.bn, num_sms(), s);
+  });
 }
 
 fd_status run_norm(fd_handle h, const float* x, const float* g, int rows, cudaStream_t s) {
@@ -306,7 +385,8 @@ fd_status run_norm(fd_handle h, const float* x, const float* g, int rows, cudaSt
 // one Transformer block (Sec. 3.2) on `rows` tokens of residual stream hbuf, with ring r
 fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int rows, int fpc,
                     int pitch, const CUtensorMap& tm_u, const CUtensorMap& tm_q,
-                    const CUtensorMap& tm_o, const CUtensorMap& tm_hid, bool refine,
+                    const CUtensorMap& tm_o, const CUtensorMap& tm_hid, const CUtensorMap& so_h,
+                    const CUtensorMap& so_q, const CUtensorMap& so_hid, bool refine,
                     cudaStream_t s) {
   const Dims& d = h->d;
   fd_status st;
@@ -319,7 +399,10 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
   q.frames_per_chunk = fpc; q.window = d.Wn; q.step_dev = h->state; q.step_host = 0;
   q.eps = h->cfg.norm_eps;
   fill_rope(q, h->cfg.rope_base);
-  if ((st = run_linear(h, FD_K_QKV, tm_u, lw.qkv, rows, p, s))) return st;
+  q.rope_t = h->rope_tab + (refine ? q.band_t : 0);
+  p.v_tma = rows % 8 == 0 ? 1 : 0;
+  if ((st = run_linear(h, FD_K_QKV, tm_u, lw.qkv, rows, p, so_q, s, &r.st_k, &r.st_vt)))
+    return st;
 
   fd::AttnParams a{};
   a.Lq = rows; a.heads = d.N; a.groups = d.G; a.ring_pitch = pitch; a.rows_per_chunk = rows;
@@ -338,20 +421,31 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
   po.epi = fd::EPI_RESID;
   po.out_f32 = hbuf;
   po.ld_out = d.D;
-  if ((st = run_linear(h, FD_K_OUT, tm_o, lw.out, rows, po, s))) return st;
+  if ((st = run_linear(h, FD_K_OUT, tm_o, lw.out, rows, po, so_h, s))) return st;
   if ((st = run_norm(h, hbuf, lw.g2, rows, s))) return st;
   fd::GemmParams p1{};
   p1.epi = fd::EPI_GELU;
   p1.out_bf16 = h->hid;
   p1.ld_out = d.Mr * d.D;
-  if ((st = run_linear(h, FD_K_MLP1, tm_u, lw.mlp1, rows, p1, s))) return st;
-  return run_linear(h, FD_K_MLP2, tm_hid, lw.mlp2, rows, po, s);
+  if ((st = run_linear(h, FD_K_MLP1, tm_u, lw.mlp1, rows, p1, so_hid, s))) return st;
+  return run_linear(h, FD_K_MLP2, tm_hid, lw.mlp2, rows, po, so_h, s);
 }
 
 fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_t s) {
   const Dims& d = h->d;
   const fd_weights w = h->w;
   fd_status st;
+  {
+    const int frames[2] = {1, d.rt};
+    double inv[fd::kRopePairs];
+    temporal_inv_freq(h->cfg.rope_base, inv);
+    const int* step = h->state;
+    float2* tab = h->rope_tab;
+    if ((st = traced(h, FD_K_ROPE, s, [&] {
+           return fd::launch_rope_table(step, 0, 2, frames, rope_band_t(), inv, tab, s);
+         })))
+      return st;
+  }
   __nv_bfloat16* x0 = h->x0;
   if ((st = traced(h, FD_K_UNSHUFFLE, s,
                    [&] { return fd::launch_unshuffle(latent, d.C, d.H, d.W, d.p, x0, s); })))
@@ -360,10 +454,10 @@ fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_
   pe.epi = fd::EPI_F32;
   pe.out_f32 = h->h;
   pe.ld_out = d.D;
-  if ((st = run_linear(h, FD_K_EMBED, h->tm_x0, w->embed, d.L, pe, s))) return st;
+  if ((st = run_linear(h, FD_K_EMBED, h->tm_x0, w->embed, d.L, pe, h->so_h, s))) return st;
   for (int b = 0; b < d.nb; ++b)
     if ((st = run_block(h, w->blocks[b], h->ringB[b], h->h, d.L, 1, h->pitchB, h->tm_uB, h->tm_qB,
-                        h->tm_oB, h->tm_hidB, false, s)))
+                        h->tm_oB, h->tm_hidB, h->so_h, h->so_qB, h->so_hidB, false, s)))
       return st;
   // temporal upsampling: RMSNorm, Linear D -> r_t D, channel block tau -> refined frame tau
   if ((st = run_norm(h, h->h, w->g_f, d.L, s))) return st;
@@ -372,11 +466,11 @@ fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_
   pt.out_f32 = h->hf;
   pt.tup_tokens = d.L;
   pt.tup_hidden = d.D;
-  if ((st = run_linear(h, FD_K_TUP, h->tm_uB, w->tup, d.L, pt, s))) return st;
+  if ((st = run_linear(h, FD_K_TUP, h->tm_uB, w->tup, d.L, pt, h->so_tup, s))) return st;
   const int R = d.rt * d.L;
   for (int b = 0; b < d.nr; ++b)
     if ((st = run_block(h, w->refine[b], h->ringR[b], h->hf, R, d.rt, h->pitchR, h->tm_uR,
-                        h->tm_qR, h->tm_oR, h->tm_hidR, true, s)))
+                        h->tm_qR, h->tm_oR, h->tm_hidR, h->so_hf, h->so_qR, h->so_hidR, true, s)))
       return st;
   // spatial upsampling head: RMSNorm, Linear D->D + GELU, Linear D -> C r_s^2, PixelShuffle
   if ((st = run_norm(h, h->hf, w->g_h, R, s))) return st;
@@ -384,12 +478,12 @@ fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_
   ph.epi = fd::EPI_GELU;
   ph.out_bf16 = h->hid;
   ph.ld_out = d.D;
-  if ((st = run_linear(h, FD_K_HEAD1, h->tm_uR, w->head1, R, ph, s))) return st;
+  if ((st = run_linear(h, FD_K_HEAD1, h->tm_uR, w->head1, R, ph, h->so_hidH, s))) return st;
   fd::GemmParams pf{};
   pf.epi = fd::EPI_F32;
   pf.out_f32 = h->F;
   pf.ld_out = d.head_out;
-  if ((st = run_linear(h, FD_K_HEAD2, h->tm_hidH, w->head2, R, pf, s))) return st;
+  if ((st = run_linear(h, FD_K_HEAD2, h->tm_hidH, w->head2, R, pf, h->so_F, s))) return st;
   const float* F = h->F;
   if ((st = traced(h, FD_K_PIXEL, s, [&] {
          return fd::launch_pixel_head(F, d.rt, d.gh, d.gw, d.Cout, d.rs, d.u8 ? 1 : 0, pixels, s);
@@ -448,12 +542,12 @@ static size_t attn_ws_floats(const Dims& d) {
   return a > b ? a : b;
 }
 
-static size_t handle_layout(const Dims& d, size_t* off /* 15 offsets */, int* pitchB,
+static size_t handle_layout(const Dims& d, size_t* off /* 16 offsets */, int* pitchB,
                             int* pitchR) {
   const size_t R = static_cast<size_t>(d.rt) * d.L;
   *pitchB = static_cast<int>(align_up(static_cast<size_t>(d.Wn) * d.L, 128));
   *pitchR = static_cast<int>(align_up(static_cast<size_t>(d.Wn) * R, 128));
-  size_t sizes[14] = {
+  size_t sizes[15] = {
       16,                                              // state
       static_cast<size_t>(d.L) * d.cin * 2,            // x0
       R * d.D * 2,                                     // u
@@ -468,19 +562,20 @@ static size_t handle_layout(const Dims& d, size_t* off /* 15 offsets */, int* pi
       static_cast<size_t>(d.C) * d.H * d.W * 4,                      // latent (host decode)
       static_cast<size_t>(d.Cout) * d.rt * d.gh * d.rs * d.gw * d.rs * (d.u8 ? 1 : 4),  // pixels
       attn_ws_floats(d) * 4,                                         // attention partials
+      static_cast<size_t>(1 + d.rt) * kHeadDim / 2 * sizeof(float2),  // temporal RoPE table
   };
   size_t cur = 0;
-  for (int i = 0; i < 14; ++i) {
+  for (int i = 0; i < 15; ++i) {
     off[i] = cur;
     cur = align_up(cur + sizes[i], 1024);
   }
-  off[14] = cur;
+  off[15] = cur;
   return cur;
 }
 
 size_t fd_handle_device_bytes(const fd_config* cfg) {
   if (!valid_cfg(cfg)) return 0;
-  size_t off[15];
+  size_t off[16];
   int a, b;
   return handle_layout(dims_of(cfg), off, &a, &b);
 }
@@ -607,7 +702,7 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   h->d = dims_of(cfg);
   h->w = w;
   const Dims& d = h->d;
-  size_t off[15];
+  size_t off[16];
   h->arena_bytes = handle_layout(d, off, &h->pitchB, &h->pitchR);
   if (cudaMalloc(&h->arena, h->arena_bytes) != cudaSuccess) {
     delete h;
@@ -626,6 +721,7 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   h->latent_buf = reinterpret_cast<float*>(b + off[11]);
   h->pixel_buf = b + off[12];
   h->attn_ws = reinterpret_cast<float*>(b + off[13]);
+  h->rope_tab = reinterpret_cast<float2*>(b + off[14]);
   h->splitsB = choose_splits(d.L, d.N, d.G, d.Wn * d.L);
   h->splitsR = choose_splits(d.rt * d.L, d.N, d.G, d.Wn * d.rt * d.L);
   const size_t ringB_elems = static_cast<size_t>(d.G) * h->pitchB * kHeadDim;
@@ -641,6 +737,9 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
                          kHeadDim * 2, 64, 128);
     ok = ok && tmap_bf16(&r.tm_vt, r.vt, h->pitchB, static_cast<uint64_t>(d.G) * kHeadDim,
                          static_cast<uint64_t>(h->pitchB) * 2, 64, 64);
+    ok = ok && tmap_kring_store(&r.st_k, r.k, d.L, d.Wn, d.G, h->pitchB);
+    if (d.L % 8 == 0) ok = ok && tmap_vring_store(&r.st_vt, r.vt, d.L, d.Wn, d.G, h->pitchB);
+    else r.st_vt = r.st_k;
   }
   for (int i = 0; i < d.nr; ++i) {
     Ring& r = h->ringR[i];
@@ -650,6 +749,10 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
                          kHeadDim * 2, 64, 128);
     ok = ok && tmap_bf16(&r.tm_vt, r.vt, h->pitchR, static_cast<uint64_t>(d.G) * kHeadDim,
                          static_cast<uint64_t>(h->pitchR) * 2, 64, 64);
+    const uint64_t R = static_cast<uint64_t>(d.rt) * d.L;
+    ok = ok && tmap_kring_store(&r.st_k, r.k, R, d.Wn, d.G, h->pitchR);
+    if (R % 8 == 0) ok = ok && tmap_vring_store(&r.st_vt, r.vt, R, d.Wn, d.G, h->pitchR);
+    else r.st_vt = r.st_k;
   }
   const uint64_t R = static_cast<uint64_t>(d.rt) * d.L;
   const uint64_t NQ = static_cast<uint64_t>(d.N) * kHeadDim;
@@ -664,6 +767,15 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   ok = ok && tmap_bf16(&h->tm_hidB, h->hid, Dm, d.L, Dm * 2, 64, 128);
   ok = ok && tmap_bf16(&h->tm_hidR, h->hid, Dm, R, Dm * 2, 64, 128);
   ok = ok && tmap_bf16(&h->tm_hidH, h->hid, d.D, R, static_cast<uint64_t>(d.D) * 2, 64, 128);
+  ok = ok && tmap_out_f32(&h->so_h, h->h, d.D, d.L, d.D);
+  ok = ok && tmap_out_f32(&h->so_hf, h->hf, d.D, R, d.D);
+  ok = ok && tmap_out_tup(&h->so_tup, h->hf, d.D, d.L, d.rt);
+  ok = ok && tmap_out_bf16(&h->so_hidB, h->hid, Dm, d.L, Dm);
+  ok = ok && tmap_out_bf16(&h->so_hidR, h->hid, Dm, R, Dm);
+  ok = ok && tmap_out_bf16(&h->so_hidH, h->hid, d.D, R, d.D);
+  ok = ok && tmap_out_f32(&h->so_F, h->F, d.head_out, R, d.head_out);
+  ok = ok && tmap_out_bf16(&h->so_qB, h->q, NQ, d.L, NQ);
+  ok = ok && tmap_out_bf16(&h->so_qR, h->q, NQ, R, NQ);
   if (!ok || cudaMemset(h->arena, 0, h->arena_bytes) != cudaSuccess ||
       cudaDeviceSynchronize() != cudaSuccess) {
     cudaFree(h->arena);
@@ -837,6 +949,12 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
   if (!tmap_bf16(&ta, A, K, M, static_cast<uint64_t>(K) * 2, 64, 128) ||
       !tmap_bf16(&tb, W, K, N, static_cast<uint64_t>(K) * 2, 64, bn))
     return FD_ERR_CUDA;
+  CUtensorMap to;
+  bool ok;
+  if (epilogue == FD_EPI_GELU) ok = tmap_out_bf16(&to, out, N, M, N);
+  else if (epilogue == FD_EPI_TUP) ok = tmap_out_tup(&to, out, tup_hidden, M, N / tup_hidden);
+  else ok = tmap_out_f32(&to, out, N, M, N);
+  if (!ok) return FD_ERR_CUDA;
   fd::GemmParams p{};
   p.M = M; p.N = N; p.K = K; p.epi = epilogue; p.bias = bias; p.err = err_dev;
   if (epilogue == FD_EPI_GELU) {
@@ -847,21 +965,24 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
   p.ld_out = N;
   p.tup_tokens = M;
   p.tup_hidden = tup_hidden;
-  return launch_ok(fd::launch_gemm(ta, tb, p, bn, num_sms(), static_cast<cudaStream_t>(stream)));
+  return launch_ok(fd::launch_gemm(ta, tb, to, to, to, p, bn, num_sms(),
+                                   static_cast<cudaStream_t>(stream)));
 }
 
 fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* bqkv,
                     const float* knorm_g, const float* vnorm_g, int heads, int groups,
                     int tokens, int grid_w, int frames_per_chunk, int window, int t, float eps,
-                    float rope_base, void* q_out, void* k_ring, void* vt_ring, int ring_pitch,
-                    int bn, int* err_dev, void* stream) {
-  if (!A || !Wqkv || !bqkv || !knorm_g || !vnorm_g || !q_out || !k_ring || !vt_ring || !err_dev)
+                    float rope_base, const float* rope_t, void* q_out, void* k_ring,
+                    void* vt_ring, int ring_pitch, int bn, int* err_dev, void* stream) {
+  if (!A || !Wqkv || !bqkv || !knorm_g || !vnorm_g || !q_out || !k_ring || !vt_ring ||
+      !err_dev || !rope_t)
     return FD_ERR_INVALID_ARG;
   if (heads < 1 || groups < 1 || heads % groups || tokens < 1 || grid_w < 1 ||
       tokens % grid_w || frames_per_chunk < 1 || window < 1 || t < 0 || K < 8 || K % 8)
     return FD_ERR_INVALID_ARG;
   if (M != frames_per_chunk * tokens) return FD_ERR_INVALID_ARG;
   if (ring_pitch < window * M || ring_pitch % 128) return FD_ERR_INVALID_ARG;
+  if (!aligned16(q_out) || !aligned16(k_ring) || !aligned16(vt_ring)) return FD_ERR_INVALID_ARG;
   if (bn == 0) bn = 128;
   if (!fd::gemm_bn_supported(bn)) return FD_ERR_INVALID_ARG;
   fd_status st = check_device();
@@ -882,7 +1003,20 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
   q.frames_per_chunk = frames_per_chunk; q.window = window; q.step_dev = nullptr;
   q.step_host = t; q.eps = eps;
   fill_rope(q, rope_base);
-  return launch_ok(fd::launch_gemm(ta, tb, p, bn, num_sms(), static_cast<cudaStream_t>(stream)));
+  q.rope_t = reinterpret_cast<const float2*>(rope_t);
+  p.v_tma = M % 8 == 0 ? 1 : 0;
+  CUtensorMap tq, tk, tv;
+  if (!tmap_out_bf16(&tq, q_out, static_cast<uint64_t>(heads) * kHeadDim, M,
+                     static_cast<uint64_t>(heads) * kHeadDim) ||
+      !tmap_kring_store(&tk, k_ring, M, window, groups, ring_pitch))
+    return FD_ERR_CUDA;
+  if (p.v_tma) {
+    if (!tmap_vring_store(&tv, vt_ring, M, window, groups, ring_pitch)) return FD_ERR_CUDA;
+  } else {
+    tv = tk;
+  }
+  return launch_ok(fd::launch_gemm(ta, tb, tq, tk, tv, p, bn, num_sms(),
+                                   static_cast<cudaStream_t>(stream)));
 }
 
 size_t fd_attention_workspace_bytes(int Lq, int heads, int groups, int n_keys, int splits) {
@@ -971,6 +1105,20 @@ fd_status fd_op_attention_static(int Lq, int heads, int groups, const void* q,
   }
   return fd_op_attention(Lq, heads, groups, q, k_ring, vt_ring, ring_pitch, n_keys, out, splits,
                          ws, err_dev, stream);
+}
+
+fd_status fd_op_rope_table(int t, int frames_per_chunk, float rope_base, float* table,
+                           void* stream) {
+  if (t < 0 || frames_per_chunk < 1 || table == nullptr || !(rope_base > 1.f))
+    return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  double inv[fd::kRopePairs];
+  temporal_inv_freq(rope_base, inv);
+  const int frames[1] = {frames_per_chunk};
+  return launch_ok(fd::launch_rope_table(nullptr, t, 1, frames, rope_band_t(), inv,
+                                         reinterpret_cast<float2*>(table),
+                                         static_cast<cudaStream_t>(stream)));
 }
 
 fd_status fd_op_kv_append(const float* k, const float* v, int groups, int rows, int window,

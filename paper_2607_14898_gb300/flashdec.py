@@ -24,7 +24,7 @@ DTYPE_F32, DTYPE_BF16, DTYPE_U8 = 0, 1, 2
 EPI_F32, EPI_RESID, EPI_GELU, EPI_TUP = 0, 1, 2, 3
 # fd_kernel_kind order
 KERNEL_KINDS = ["unshuffle", "embed", "rmsnorm", "qkv", "attn_backbone", "attn_refine", "out",
-                "mlp1", "mlp2", "tup", "head1", "head2", "pixel", "advance"]
+                "mlp1", "mlp2", "tup", "head1", "head2", "pixel", "advance", "rope"]
 
 
 class FdError(RuntimeError):
@@ -67,8 +67,9 @@ _SIGS = {
     "fd_sync_status": (_I, [_P]),
     "fd_debug_read_ring": (_I, [_P, _I, _I, _P, ctypes.c_size_t]),
     "fd_op_linear": (_I, [_I, _I, _I, _I, _P, _P, _P, _P, _I, _I, _P, _P]),
+    "fd_op_rope_table": (_I, [_I, _I, _F, _P, _P]),
     "fd_op_qkv": (_I, [_I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _F, _F,
-                       _P, _P, _P, _I, _I, _P, _P]),
+                       _P, _P, _P, _P, _I, _I, _P, _P]),
     "fd_attention_workspace_bytes": (ctypes.c_size_t, [_I, _I, _I, _I, _I]),
     "fd_op_attention": (_I, [_I, _I, _I, _P, _P, _P, _I, _I, _P, _I, _P, _P, _P]),
     "fd_op_attention_static": (_I, [_I, _I, _I, _P, _P, _P, _I, _I, _P, _I, _P, _P]),
@@ -266,14 +267,19 @@ def op_linear(epi, A, W, bias, out, tup_hidden=0, bn=0, err=None, stream=None) -
                               tup_hidden, bn, _ptr(err), _stream_ptr(stream)), "fd_op_linear")
 
 
+def op_rope_table(t, frames_per_chunk, rope_base, table, stream=None) -> None:
+    _check(lib().fd_op_rope_table(t, frames_per_chunk, rope_base, _ptr(table),
+                                  _stream_ptr(stream)), "fd_op_rope_table")
+
+
 def op_qkv(A, Wqkv, bqkv, knorm_g, vnorm_g, heads, groups, tokens, grid_w, frames_per_chunk,
-           window, t, eps, rope_base, q_out, k_ring, vt_ring, ring_pitch, bn=0, err=None,
+           window, t, eps, rope_base, rope_t, q_out, k_ring, vt_ring, ring_pitch, bn=0, err=None,
            stream=None) -> None:
     M, K = A.shape
     _check(lib().fd_op_qkv(M, K, _ptr(A), _ptr(Wqkv), _ptr(bqkv), _ptr(knorm_g), _ptr(vnorm_g),
                            heads, groups, tokens, grid_w, frames_per_chunk, window, t, eps,
-                           rope_base, _ptr(q_out), _ptr(k_ring), _ptr(vt_ring), ring_pitch, bn,
-                           _ptr(err), _stream_ptr(stream)), "fd_op_qkv")
+                           rope_base, _ptr(rope_t), _ptr(q_out), _ptr(k_ring), _ptr(vt_ring),
+                           ring_pitch, bn, _ptr(err), _stream_ptr(stream)), "fd_op_qkv")
 
 
 def attention_workspace_bytes(Lq, heads, groups, n_keys, splits=0) -> int:

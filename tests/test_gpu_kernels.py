@@ -39,6 +39,7 @@ def linear_case(M, N, K, seed):
 # ------------------------------------------------------------------ tcgen05 GEMM
 @pytest.mark.parametrize("M,N,K,bn", [
     (130, 256, 256, 128),     # ragged M (2 tiles), one K tile of 4 x 64
+    (520, 768, 1024, 192),    # 192-wide tiles
     (64, 192, 16, 64),        # K < 64 (tiny patch-embed), zero-filled K tail
     (520, 1024, 256, 256),    # 256-wide tiles
     (1560, 1536, 1024, 128),  # 480p QKV shape: 13 x 12 tiles, persistent (> 1 tile per CTA)
@@ -88,12 +89,14 @@ class Cfg:
         self.__dict__.update(kw)
 
 
-@pytest.mark.parametrize("heads,groups,grid_h,grid_w,fpc,window,t,K", [
-    (4, 2, 10, 13, 4, 3, 5, 256),       # refinement-like: 4 frames per chunk, ragged rows
-    (16, 4, 30, 52, 1, 4, 7, 1024),     # 480p backbone block
-    (24, 3, 3, 5, 1, 8, 130, 1536),     # wide model, long stream (large temporal index)
+@pytest.mark.parametrize("heads,groups,grid_h,grid_w,fpc,window,t,K,bn", [
+    (4, 2, 10, 13, 4, 3, 5, 256, 128),       # refinement-like: 4 frames per chunk, ragged rows
+    (16, 4, 30, 52, 1, 4, 7, 1024, 192),     # 480p backbone block, 192-wide tiles
+    (16, 4, 30, 52, 1, 4, 7, 1024, 256),     # same, 256-wide tiles
+    (24, 3, 3, 5, 1, 8, 130, 1536, 64),      # wide model, long stream (large temporal index)
+    (4, 2, 8, 8, 4, 2, 40000, 256, 0),       # very long stream: temporal index 160000
 ])
-def test_qkv_fused(heads, groups, grid_h, grid_w, fpc, window, t, K):
+def test_qkv_fused(heads, groups, grid_h, grid_w, fpc, window, t, K, bn):
     dh, eps, base = 64, 1e-6, 10000.0
     tokens = grid_h * grid_w
     M = fpc * tokens
@@ -106,9 +109,11 @@ def test_qkv_fused(heads, groups, grid_h, grid_w, fpc, window, t, K):
     k_ring = torch.zeros(groups, pitch, dh, dtype=torch.bfloat16, device="cuda")
     vt_ring = torch.zeros(groups, dh, pitch, dtype=torch.bfloat16, device="cuda")
     err = err_word()
+    rope_t = torch.zeros(fpc, 12, 2, device="cuda")
+    fdp.op_rope_table(t, fpc, base, rope_t)
     fdp.op_qkv(dev(A, torch.bfloat16), dev(W, torch.bfloat16), dev(b), dev(kg), dev(vg), heads,
-               groups, tokens, grid_w, fpc, window, t, eps, base, q_out, k_ring, vt_ring, pitch,
-               err=err)
+               groups, tokens, grid_w, fpc, window, t, eps, base, rope_t, q_out, k_ring, vt_ring,
+               pitch, bn=bn, err=err)
     check_err(err)
     # oracle: Linear, KV-norm, 3D-RoPE at (t*fpc + row // tokens, y, x)
     qkv = oracle.linear(f64(A), f64(W), f64(b))
