@@ -115,7 +115,8 @@ fd_status fd_weights_destroy(fd_weights w);
 /* ------------------------------------------------------------------ streams */
 
 /* Create a decoder stream state for cfg (must equal the weights' cfg): KV rings for every
- * layer (backbone G x W L x 64 per K and V; refinement G x r_t W L x 64), activation scratch
+ * layer (backbone G x W L x 64 per K and V; refinement G x r_t W L x 64; K bf16, V fp16
+ * stored transposed), activation scratch
  * and a device chunk counter t = 0. Zero-fills the rings. Synchronous. */
 fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out);
 
@@ -178,7 +179,7 @@ fd_status fd_profile_collect(fd_handle h, int64_t* launches, double* ms);
 int64_t fd_launch_count(fd_handle h);
 
 /* Copy layer `layer` of the backbone (which = 0) or refinement (which = 1) ring into host
- * memory: K as [G][W * rows][64] bf16 bits, then V as [G][W * rows][64] bf16 bits (rows =
+ * memory: K as [G][W * rows][64] bf16 bits, then V as [G][W * rows][64] fp16 bits (rows =
  * L backbone, r_t L refinement; row slot*rows + r holds token r of the chunk in ring slot
  * `slot` = chunk index mod W). dst_bytes must be >= 2 * G * W * rows * 64 * 2. Synchronous.
  * For tests of the cache indexing. */

@@ -49,7 +49,7 @@ fd_status fd_op_rope_table(int t, int frames_per_chunk, float rope_base, float* 
  *           rope_t, the fd_op_rope_table of chunk t), row and column of token (row % tokens)
  *           in a grid of width grid_w (rope_base; bands 24/20/20 dims)
  *   q_out bf16 [M][heads*64];  K -> k_ring bf16 [groups][ring_pitch][64] rows
- *   (t mod window)*M + row;  V -> vt_ring bf16 [groups][64][ring_pitch] (transposed), same
+ *   (t mod window)*M + row;  V -> vt_ring fp16 [groups][64][ring_pitch] (transposed), same
  *   key index.  M = frames_per_chunk * tokens; ring_pitch % 128 == 0, >= window * M. */
 fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* bqkv,
                     const float* knorm_g, const float* vnorm_g, int heads, int groups,
@@ -59,7 +59,7 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
 
 /* Attention of Lq queries over the first n_keys keys of a ring (Sec. 3.3, Eq. kv_cache):
  *   out[r][n*64 + d] = sum_j softmax_j(q_n . k_j / 8) v_j[d],  KV group g = n / (heads/groups)
- * q bf16 [Lq][heads*64]; k_ring bf16 [groups][ring_pitch][64]; vt_ring bf16
+ * q bf16 [Lq][heads*64]; k_ring bf16 [groups][ring_pitch][64]; vt_ring fp16
  * [groups][64][ring_pitch]; out bf16 [Lq][heads*64]. 1 <= n_keys <= ring_pitch,
  * ring_pitch % 128 == 0. Ring entries past n_keys must hold finite values.
  * splits: the key range is divided over `splits` CTAs per (query tile, head) whose partial
@@ -95,8 +95,8 @@ fd_status fd_op_attention_static(int Lq, int heads, int groups, const void* q,
                                  int n_keys, void* out, int splits, int* err_dev, void* stream);
 
 /* Rolling-cache append (Algorithm 1, cache update): fp32 k, v [groups][rows][64] rounded to
- * bf16 (nearest even) into ring slot s = t mod window: k_ring[g][s*rows + r][d] and
- * vt_ring[g][d][s*rows + r]. The oldest chunk's slot is overwritten (eviction). */
+ * nearest even into ring slot s = t mod window: k_ring[g][s*rows + r][d] (bf16) and
+ * vt_ring[g][d][s*rows + r] (fp16). The oldest chunk's slot is overwritten (eviction). */
 fd_status fd_op_kv_append(const float* k, const float* v, int groups, int rows, int window,
                           int t, int ring_pitch, void* k_ring, void* vt_ring, void* stream);
 

@@ -18,7 +18,8 @@
 //   EPI_GELU   out = bf16(GELU(acc + b))        (MLP layer 1, head layer 1)
 //   EPI_TUP    channel block tau of token l -> refined token tau*L + l   (Eq. temporal_upsample)
 //   EPI_QKV    bias; KV-norm (RMS over D_h) on K and V; 3D-RoPE on Q and K; Q to its buffer,
-//              K and V (transposed) into ring slot t mod W of the layer's cache (Sec. 3.3)
+//              K (bf16) and V (transposed, fp16) into ring slot t mod W of the layer's cache
+//              (Sec. 3.3)
 #include "fd_internal.h"
 #include "fd_ptx.cuh"
 
@@ -268,11 +269,11 @@ __global__ void __launch_bounds__(192, 1)
               bulk_commit();
             }
           } else if (p.v_tma) {
-            // V transposed: slab [64 dims][32 keys] bf16, stored into the ring's V^T slot view
+            // V transposed: slab [64 dims][32 keys] fp16, stored into the ring's V^T slot view
             uint8_t* buf = acquire();
-            __nv_bfloat16* sv = reinterpret_cast<__nv_bfloat16*>(buf);
+            __half* sv = reinterpret_cast<__half*>(buf);
 #pragma unroll
-            for (int j = 0; j < 64; ++j) sv[j * 32 + lane] = __float2bfloat16_rn(v[j]);
+            for (int j = 0; j < 64; ++j) sv[j * 32 + lane] = __float2half_rn(v[j]);
             publish();
             if (lane == 0 && row0 < p.M) {
               tma_store_4d(&tmV, smem_u32(buf), row0, slot, 0, hidx - q.heads - q.groups);
@@ -280,11 +281,11 @@ __global__ void __launch_bounds__(192, 1)
             }
           } else if (row_ok) {
             const int g = hidx - q.heads - q.groups;
-            __nv_bfloat16* dst = q.vt_ring + static_cast<size_t>(g) * kHeadDim * q.ring_pitch +
-                                 slot * rows_chunk + row;
+            __half* dst = q.vt_ring + static_cast<size_t>(g) * kHeadDim * q.ring_pitch +
+                          slot * rows_chunk + row;
 #pragma unroll
             for (int j = 0; j < 64; ++j)
-              dst[static_cast<size_t>(j) * q.ring_pitch] = __float2bfloat16_rn(v[j]);
+              dst[static_cast<size_t>(j) * q.ring_pitch] = __float2half_rn(v[j]);
           }
         }
       } else if (p.epi == EPI_GELU) {

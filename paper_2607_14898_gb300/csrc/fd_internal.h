@@ -3,6 +3,7 @@
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <cstdint>
 
@@ -28,7 +29,7 @@ struct QkvEpi {
   const float* vnorm_g;      // [64] KV-norm gain for V
   __nv_bfloat16* q_out;      // [M][heads * 64]
   __nv_bfloat16* k_ring;     // [groups][ring_pitch][64]
-  __nv_bfloat16* vt_ring;    // [groups][64][ring_pitch]   (V stored transposed)
+  __half* vt_ring;           // [groups][64][ring_pitch]   (V stored transposed, fp16)
   int ring_pitch;            // key rows per group (>= window * rows_per_chunk, multiple of 128)
   int tokens;                // L_frm
   int grid_w;                // token-grid width W'/p
@@ -102,7 +103,7 @@ cudaError_t launch_rmsnorm(const float* h, const float* g, int M, int D, float e
 cudaError_t launch_pixel_head(const float* F, int frames, int gh, int gw, int C, int rs,
                               int out_u8, void* pix, cudaStream_t s);
 cudaError_t launch_kv_append(const float* k, const float* v, int groups, int rows, int slot,
-                             int ring_pitch, __nv_bfloat16* k_ring, __nv_bfloat16* vt_ring,
+                             int ring_pitch, __nv_bfloat16* k_ring, __half* vt_ring,
                              cudaStream_t s);
 cudaError_t launch_advance(int* step_dev, cudaStream_t s);
 // Temporal RoPE table of one chunk: for each block of `frames[k]` frames per chunk (k < nsets),

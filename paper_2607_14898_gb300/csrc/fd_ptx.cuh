@@ -5,6 +5,7 @@
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cstdint>
 
 namespace fd {
@@ -266,6 +267,11 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
          (static_cast<uint32_t>(M >> 4) << 24);
 }
 
+// Same for fp16 A and B (both operands must share one type).
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
+  return (1u << 4) | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
 // Shared-memory matrix descriptor for a K-major operand stored with the 128-byte swizzle
 // (rows of 64 bf16 = 128 B, 8-row atoms of 1024 B, atoms 1024 B apart). Start address and
 // offsets are encoded >> 4; bit 46 is the descriptor version; bits 61-63 = 2 selects the
@@ -285,6 +291,36 @@ __device__ __forceinline__ uint32_t sw128_offset(uint32_t row, uint32_t k) {
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// exp2 of (a * scale + neg, b * scale + neg): the fp32 pair from one packed FMA is rounded to
+// fp16 and both powers come from one packed ex2; result fp16x2 with a in the low half
+__device__ __forceinline__ uint32_t exp2_pair_f16(float a, float b, uint64_t scale2,
+                                                  uint64_t neg2) {
+  uint64_t ab, r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(ab) : "f"(a), "f"(b));
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(ab), "l"(scale2), "l"(neg2));
+  float xa, xb;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(xa), "=f"(xb) : "l"(r));
+  uint32_t h, e;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(h) : "f"(xb), "f"(xa));
+  asm("ex2.approx.f16x2 %0, %1;" : "=r"(e) : "r"(h));
+  return e;
+}
+__device__ __forceinline__ uint64_t pack_f32x2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ uint32_t hadd2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("add.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+// sum of the two fp16 halves, in fp32
+__device__ __forceinline__ float f16x2_sum(uint32_t a) {
+  __half2 h = *reinterpret_cast<__half2*>(&a);
+  return __low2float(h) + __high2float(h);
 }
 
 __device__ __forceinline__ float ex2_approx(float x) {

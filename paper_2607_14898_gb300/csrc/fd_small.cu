@@ -4,7 +4,7 @@
 //   rmsnorm      h fp32 [M][D] -> bf16(h / sqrt(mean(h^2) + eps) * g)  (pre-norm, Sec. 3.2)
 //   pixel_head   F fp32 [frames*L][C r_s^2] -> PixelShuffle(r_s) + clamp to [-1, 1], fp32 or
 //                uint8 (Sec. 3.4 "Step 3"); one thread per 4 consecutive output pixels
-//   kv_append    fp32 K, V of one chunk -> bf16 ring slot (K rows, V transposed) (Sec. 3.3)
+//   kv_append    fp32 K, V of one chunk -> ring slot (K rows bf16, V transposed fp16) (Sec. 3.3)
 //   advance      chunk counter t += 1 (device-resident, so a captured graph can be replayed)
 #include "fd_internal.h"
 #include "fd_ptx.cuh"
@@ -90,12 +90,12 @@ __global__ void pixel_head_kernel(const float* __restrict__ F, int frames, int g
   }
 }
 
-// K, V fp32 [groups][rows][64] -> k_ring[g][slot*rows + r][d], vt_ring[g][d][slot*rows + r]
-// (bf16, round to nearest even). Block: 32 x 8 threads over a 32-row x 64-dim tile; V goes
+// K, V fp32 [groups][rows][64] -> k_ring[g][slot*rows + r][d] (bf16) and
+// vt_ring[g][d][slot*rows + r] (fp16), both rounded to nearest even. Block: 32 x 8 threads over a 32-row x 64-dim tile; V goes
 // through shared memory so both the read and the transposed write are coalesced.
 __global__ void kv_append_kernel(const float* __restrict__ k, const float* __restrict__ v,
                                  int rows, int slot, int pitch, __nv_bfloat16* __restrict__ k_ring,
-                                 __nv_bfloat16* __restrict__ vt_ring) {
+                                 __half* __restrict__ vt_ring) {
   __shared__ float tile[64][33];
   const int g = blockIdx.y;
   const int r0 = blockIdx.x * 32;
@@ -114,7 +114,7 @@ __global__ void kv_append_kernel(const float* __restrict__ k, const float* __res
     const int r = r0 + threadIdx.x;
     if (r < rows)
       vt_ring[(static_cast<size_t>(g) * kHeadDim + d) * pitch + slot * static_cast<size_t>(rows) +
-              r] = __float2bfloat16_rn(tile[d][threadIdx.x]);
+              r] = __float2half_rn(tile[d][threadIdx.x]);
   }
 }
 
@@ -170,7 +170,7 @@ cudaError_t launch_pixel_head(const float* F, int frames, int gh, int gw, int C,
 }
 
 cudaError_t launch_kv_append(const float* k, const float* v, int groups, int rows, int slot,
-                             int ring_pitch, __nv_bfloat16* k_ring, __nv_bfloat16* vt_ring,
+                             int ring_pitch, __nv_bfloat16* k_ring, __half* vt_ring,
                              cudaStream_t s) {
   dim3 grid((rows + 31) / 32, groups);
   kv_append_kernel<<<grid, dim3(32, 8), 0, s>>>(k, v, rows, slot, ring_pitch, k_ring, vt_ring);

@@ -38,17 +38,27 @@ bool load_encode() {
 
 // 2D bf16 tensor [outer][inner] with row pitch row_bytes, 128-byte swizzled box
 // {box_inner (<= 64), box_outer}.
-bool tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
-               uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+bool tmap_16bit(CUtensorMap* m, CUtensorMapDataType dt, const void* base, uint64_t inner,
+                uint64_t outer, uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
   if (!load_encode()) return false;
   cuuint64_t dims[2] = {inner, outer};
   cuuint64_t strides[1] = {row_bytes};
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t es[2] = {1, 1};
-  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
-                  box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+  return g_encode(m, dt, 2, const_cast<void*>(base), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+bool tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+               uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  return tmap_16bit(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, base, inner, outer, row_bytes,
+                    box_inner, box_outer);
+}
+bool tmap_f16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+              uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  return tmap_16bit(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base, inner, outer, row_bytes,
+                    box_inner, box_outer);
 }
 
 // N-d tensor map (rank <= 5): dims innermost first, strides in bytes for dims 1..rank-1
@@ -98,13 +108,14 @@ bool tmap_kring_store(CUtensorMap* m, const void* base, uint64_t M, uint64_t W, 
   return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, base, dims, strides, box,
                  CU_TENSOR_MAP_SWIZZLE_128B);
 }
-// V^T ring [G][64][pitch] viewed as {M keys of a slot, W slots, 64 dims, G}; needs M % 8 == 0
+// V^T ring [G][64][pitch] (fp16) viewed as {M keys of a slot, W slots, 64 dims, G};
+// needs M % 8 == 0
 bool tmap_vring_store(CUtensorMap* m, const void* base, uint64_t M, uint64_t W, uint64_t G,
                       uint64_t pitch) {
   const uint64_t dims[4] = {M, W, 64, G};
   const uint64_t strides[3] = {M * 2, pitch * 2, 64 * pitch * 2};
   const uint32_t box[4] = {32, 1, 64, 1};
-  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, base, dims, strides, box,
+  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, base, dims, strides, box,
                  CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
@@ -252,7 +263,7 @@ namespace {
 
 struct Ring {
   __nv_bfloat16* k = nullptr;   // [G][pitch][64]
-  __nv_bfloat16* vt = nullptr;  // [G][64][pitch]
+  __half* vt = nullptr;         // [G][64][pitch] fp16
   CUtensorMap tm_k, tm_vt;      // attention loads
   CUtensorMap st_k, st_vt;      // QKV epilogue stores into ring slots
 };
@@ -732,10 +743,10 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   for (int i = 0; i < d.nb; ++i) {
     Ring& r = h->ringB[i];
     r.k = reinterpret_cast<__nv_bfloat16*>(b + off[9]) + 2 * i * ringB_elems;
-    r.vt = r.k + ringB_elems;
+    r.vt = reinterpret_cast<__half*>(r.k + ringB_elems);
     ok = ok && tmap_bf16(&r.tm_k, r.k, kHeadDim, static_cast<uint64_t>(d.G) * h->pitchB,
                          kHeadDim * 2, 64, 128);
-    ok = ok && tmap_bf16(&r.tm_vt, r.vt, h->pitchB, static_cast<uint64_t>(d.G) * kHeadDim,
+    ok = ok && tmap_f16(&r.tm_vt, r.vt, h->pitchB, static_cast<uint64_t>(d.G) * kHeadDim,
                          static_cast<uint64_t>(h->pitchB) * 2, 64, 64);
     ok = ok && tmap_kring_store(&r.st_k, r.k, d.L, d.Wn, d.G, h->pitchB);
     if (d.L % 8 == 0) ok = ok && tmap_vring_store(&r.st_vt, r.vt, d.L, d.Wn, d.G, h->pitchB);
@@ -744,10 +755,10 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   for (int i = 0; i < d.nr; ++i) {
     Ring& r = h->ringR[i];
     r.k = reinterpret_cast<__nv_bfloat16*>(b + off[10]) + 2 * i * ringR_elems;
-    r.vt = r.k + ringR_elems;
+    r.vt = reinterpret_cast<__half*>(r.k + ringR_elems);
     ok = ok && tmap_bf16(&r.tm_k, r.k, kHeadDim, static_cast<uint64_t>(d.G) * h->pitchR,
                          kHeadDim * 2, 64, 128);
-    ok = ok && tmap_bf16(&r.tm_vt, r.vt, h->pitchR, static_cast<uint64_t>(d.G) * kHeadDim,
+    ok = ok && tmap_f16(&r.tm_vt, r.vt, h->pitchR, static_cast<uint64_t>(d.G) * kHeadDim,
                          static_cast<uint64_t>(h->pitchR) * 2, 64, 64);
     const uint64_t R = static_cast<uint64_t>(d.rt) * d.L;
     ok = ok && tmap_kring_store(&r.st_k, r.k, R, d.Wn, d.G, h->pitchR);
@@ -998,7 +1009,7 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
   q.heads = heads; q.groups = groups; q.knorm_g = knorm_g; q.vnorm_g = vnorm_g;
   q.q_out = static_cast<__nv_bfloat16*>(q_out);
   q.k_ring = static_cast<__nv_bfloat16*>(k_ring);
-  q.vt_ring = static_cast<__nv_bfloat16*>(vt_ring);
+  q.vt_ring = static_cast<__half*>(vt_ring);
   q.ring_pitch = ring_pitch; q.tokens = tokens; q.grid_w = grid_w;
   q.frames_per_chunk = frames_per_chunk; q.window = window; q.step_dev = nullptr;
   q.step_host = t; q.eps = eps;
@@ -1042,7 +1053,7 @@ fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const vo
   if (!tmap_bf16(&tq, q, NQ, Lq, NQ * 2, 64, 128) ||
       !tmap_bf16(&tk, k_ring, kHeadDim, static_cast<uint64_t>(groups) * ring_pitch, kHeadDim * 2,
                  64, 128) ||
-      !tmap_bf16(&tv, vt_ring, ring_pitch, static_cast<uint64_t>(groups) * kHeadDim,
+      !tmap_f16(&tv, vt_ring, ring_pitch, static_cast<uint64_t>(groups) * kHeadDim,
                  static_cast<uint64_t>(ring_pitch) * 2, 64, 64))
     return FD_ERR_CUDA;
   fd::AttnParams a{};
@@ -1130,7 +1141,7 @@ fd_status fd_op_kv_append(const float* k, const float* v, int groups, int rows, 
   if (st) return st;
   return launch_ok(fd::launch_kv_append(k, v, groups, rows, t % window, ring_pitch,
                                         static_cast<__nv_bfloat16*>(k_ring),
-                                        static_cast<__nv_bfloat16*>(vt_ring),
+                                        static_cast<__half*>(vt_ring),
                                         static_cast<cudaStream_t>(stream)));
 }
 

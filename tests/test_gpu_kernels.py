@@ -107,7 +107,7 @@ def test_qkv_fused(heads, groups, grid_h, grid_w, fpc, window, t, K, bn):
     pitch = -(-window * M // 128) * 128
     q_out = torch.zeros(M, heads * dh, dtype=torch.bfloat16, device="cuda")
     k_ring = torch.zeros(groups, pitch, dh, dtype=torch.bfloat16, device="cuda")
-    vt_ring = torch.zeros(groups, dh, pitch, dtype=torch.bfloat16, device="cuda")
+    vt_ring = torch.zeros(groups, dh, pitch, dtype=torch.float16, device="cuda")
     err = err_word()
     rope_t = torch.zeros(fpc, 12, 2, device="cuda")
     fdp.op_rope_table(t, fpc, base, rope_t)
@@ -145,7 +145,7 @@ def attention_case(Lq, heads, groups, pitch, n_keys, seed, qscale=1.5):
     dh = 64
     q = bf16_values(randn((Lq, heads * dh), seed, qscale))
     k = bf16_values(randn((groups, pitch, dh), seed + 1))
-    v = bf16_values(randn((groups, pitch, dh), seed + 2))
+    v = randn((groups, pitch, dh), seed + 2).astype(np.float16).astype(np.float32)  # fp16 V
     # entries past n_keys hold large stale values: they must not leak in
     k[:, n_keys:] *= 50
     v[:, n_keys:] *= 50
@@ -159,7 +159,7 @@ def run_attention(q, k, v, heads, groups, pitch, n_keys, splits=0):
     ws_bytes = fdp.attention_workspace_bytes(Lq, heads, groups, n_keys, splits)
     ws = torch.full((max(1, ws_bytes // 4),), float("nan"), device="cuda")
     err = err_word()
-    fdp.op_attention(dev(q, torch.bfloat16), dev(k, torch.bfloat16), dev(vt, torch.bfloat16),
+    fdp.op_attention(dev(q, torch.bfloat16), dev(k, torch.bfloat16), dev(vt, torch.float16),
                      heads, groups, pitch, n_keys, out, splits=splits, workspace=ws, err=err)
     check_err(err)
     return out.float().cpu()
@@ -203,11 +203,11 @@ def test_attention_full_size_sampled(Lq, heads, groups, n_keys):
 # ------------------------------------------------------------------ cache append (bit-exact)
 def test_kv_append_ring_indexing_bit_exact():
     """After appending chunk t, ring slot s holds chunk j with j = s mod W, t-W < j <= t, bit
-    for bit equal to the bf16 (nearest-even) rounding of its fp32 K / V."""
+    for bit equal to the nearest-even rounding of its fp32 K (bf16) and V (fp16)."""
     G, rows, W, dh = 3, 200, 3, 64
     pitch = -(-W * rows // 128) * 128
     k_ring = torch.zeros(G, pitch, dh, dtype=torch.bfloat16, device="cuda")
-    vt_ring = torch.zeros(G, dh, pitch, dtype=torch.bfloat16, device="cuda")
+    vt_ring = torch.zeros(G, dh, pitch, dtype=torch.float16, device="cuda")
     chunks = []
     for t in range(7):
         k = randn((G, rows, dh), 100 + t)
@@ -220,7 +220,7 @@ def test_kv_append_ring_indexing_bit_exact():
         for j in range(max(0, t - W + 1), t + 1):
             s = j % W
             kb = torch.from_numpy(chunks[j][0]).to(torch.bfloat16).view(torch.int16).numpy()
-            vb = torch.from_numpy(chunks[j][1]).to(torch.bfloat16).view(torch.int16).numpy()
+            vb = torch.from_numpy(chunks[j][1]).to(torch.float16).view(torch.int16).numpy()
             assert np.array_equal(kr[:, s * rows:(s + 1) * rows], kb), (t, j)
             assert np.array_equal(vr[:, :, s * rows:(s + 1) * rows], vb.transpose(0, 2, 1)), (t, j)
         assert not kr[:, W * rows:].any()   # padding rows never written
