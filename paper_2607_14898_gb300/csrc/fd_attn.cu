@@ -83,16 +83,6 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
   const int hd0 = p.pair_heads ? 2 * blockIdx.y : blockIdx.y;
   const int hd1 = p.pair_heads ? 2 * blockIdx.y + 1 : blockIdx.y;
   const int g = hd0 / (p.heads / p.groups);
-  int n_keys = p.n_keys_host;
-  if (p.step_dev != nullptr) {
-    const int t = *p.step_dev;
-    n_keys = (t + 1 < p.window ? t + 1 : p.window) * p.rows_per_chunk;
-  }
-  const int nblk_all = (n_keys + 127) / 128;
-  const int per = (nblk_all + p.splits - 1) / p.splits;
-  const int kb0 = blockIdx.z * per;
-  const int kb_end = kb0 + per < nblk_all ? kb0 + per : nblk_all;
-  const int nblk = kb_end > kb0 ? kb_end - kb0 : 0;
 
   if (threadIdx.x == 0) {
     if (!aligned) atomicOr(p.err, ERR_SMEM_ALIGN);
@@ -110,6 +100,17 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
     }
     fence_barrier_init();
   }
+  grid_dep_wait();  // Q and the ring written by the previous kernels; TMEM freed by their CTAs
+  int n_keys = p.n_keys_host;
+  if (p.step_dev != nullptr) {
+    const int t = *p.step_dev;
+    n_keys = (t + 1 < p.window ? t + 1 : p.window) * p.rows_per_chunk;
+  }
+  const int nblk_all = (n_keys + 127) / 128;
+  const int per = (nblk_all + p.splits - 1) / p.splits;
+  const int kb0 = blockIdx.z * per;
+  const int kb_end = kb0 + per < nblk_all ? kb0 + per : nblk_all;
+  const int nblk = kb_end > kb0 ? kb_end - kb0 : 0;
   if (warp == 0) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
     tmem_relinquish();
@@ -346,6 +347,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
     }
   }
 
+  grid_dep_launch();
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
@@ -358,6 +360,8 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
 __global__ void attn_combine_kernel(const float* __restrict__ part_o,
                                     const float* __restrict__ part_ml, int splits, int Lq,
                                     int heads, __nv_bfloat16* __restrict__ out, int ld_out) {
+  grid_dep_wait();
+  grid_dep_launch();
   const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (wid >= Lq * heads) return;
@@ -408,13 +412,13 @@ cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmK,
   const int qtiles = (p.Lq + kBM - 1) / kBM;
   dim3 grid = p.pair_heads ? dim3(qtiles, p.heads / 2, p.splits)
                            : dim3((qtiles + 1) / 2, p.heads, p.splits);
-  attn_kernel<<<grid, attn::kThreads, attn::kSmem, s>>>(tmQ, tmK, tmVt, p);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_pdl(attn_kernel, grid, dim3(attn::kThreads), attn::kSmem, s, tmQ, tmK,
+                             tmVt, p);
   if (e != cudaSuccess || p.splits == 1) return e;
   const long long warps = static_cast<long long>(p.Lq) * p.heads;
-  attn_combine_kernel<<<static_cast<int>((warps + 7) / 8), 256, 0, s>>>(
-      p.part_o, p.part_ml, p.splits, p.Lq, p.heads, p.out, p.ld_out);
-  return cudaGetLastError();
+  return launch_pdl(attn_combine_kernel, dim3(static_cast<int>((warps + 7) / 8)), dim3(256), 0,
+                    s, static_cast<const float*>(p.part_o), static_cast<const float*>(p.part_ml),
+                    p.splits, p.Lq, p.heads, p.out, p.ld_out);
 }
 
 }  // namespace fd

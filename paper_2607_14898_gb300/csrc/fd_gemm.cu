@@ -113,6 +113,7 @@ __global__ void __launch_bounds__(192, 1)
     prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
   }
+  grid_dep_wait();  // inputs written by the previous kernel; TMEM freed by its CTAs
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
     tmem_relinquish();
@@ -352,6 +353,7 @@ __global__ void __launch_bounds__(192, 1)
     if (lane == 0) bulk_wait_all();  // every store has landed before the CTA exits
     __syncwarp();
   }
+  grid_dep_launch();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -375,8 +377,8 @@ static cudaError_t launch_bn(const CUtensorMap& tmA, const CUtensorMap& tmB,
   }
   const int tiles = ((p.M + kBM - 1) / kBM) * ((p.N + BN - 1) / BN);
   const int grid = tiles < num_sms ? tiles : num_sms;
-  gemm_kernel<BN><<<grid, 192, C::kSmem, s>>>(tmA, tmB, tmO, tmK, tmV, p);
-  return cudaGetLastError();
+  return launch_pdl(gemm_kernel<BN>, dim3(grid), dim3(192), C::kSmem, s, tmA, tmB, tmO, tmK,
+                    tmV, p);
 }
 
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmO,

@@ -9,6 +9,24 @@
 
 namespace fd {
 
+// Launch with programmatic stream serialization (the kernel must call grid_dep_wait before it
+// touches memory written by the previous kernel of the stream).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 constexpr int kHeadDim = 64;     // D_h: every model size of the paper uses D / N = 64
 constexpr int kRopePairs = 32;   // D_h / 2 rotation pairs: 12 temporal, 10 row, 10 column
 constexpr int kBM = 128;         // GEMM / attention tile rows (one TMEM lane per row)

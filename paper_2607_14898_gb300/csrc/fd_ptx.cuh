@@ -31,6 +31,20 @@ __device__ __forceinline__ unsigned long long globaltimer() {
   return t;
 }
 
+// ---------------------------------------------------------------- dependent launch
+// Programmatic dependent launch: the next kernel of the stream may start (its prologue runs
+// while this one finishes) once every CTA of this kernel has called grid_dep_launch() or
+// exited; grid_dep_wait() blocks until the previous kernel has completed and its memory
+// writes are visible. Both are no-ops for a launch without the attribute. Every kernel waits
+// before its first global memory access and before allocating TMEM (a CTA that held TMEM
+// while waiting could starve the CTAs it waits for).
+__device__ __forceinline__ void grid_dep_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dep_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");

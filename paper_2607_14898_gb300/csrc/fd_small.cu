@@ -13,6 +13,8 @@ namespace fd {
 
 __global__ void unshuffle_kernel(const float* __restrict__ z, int C, int H, int W, int p,
                                  __nv_bfloat16* __restrict__ x0) {
+  grid_dep_wait();
+  grid_dep_launch();
   const int gw = W / p;
   const int cin = C * p * p;
   const int total = (H / p) * gw * cin;
@@ -29,6 +31,8 @@ __global__ void unshuffle_kernel(const float* __restrict__ z, int C, int H, int 
 // one warp per row; D % 128 == 0
 __global__ void rmsnorm_kernel(const float* __restrict__ h, const float* __restrict__ g, int M,
                                int D, float eps, __nv_bfloat16* __restrict__ u) {
+  grid_dep_wait();
+  grid_dep_launch();
   const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= M) return;
@@ -60,6 +64,8 @@ __device__ __forceinline__ uint32_t quant_u8(float x) {
 // pix[c][tau][y][x] = clamp(F[tau*L + (y/rs)*gw + x/rs][c*rs*rs + (y%rs)*rs + x%rs]); rs % 4 == 0
 __global__ void pixel_head_kernel(const float* __restrict__ F, int frames, int gh, int gw, int C,
                                   int rs, int out_u8, void* __restrict__ pix) {
+  grid_dep_wait();
+  grid_dep_launch();
   const int Wo = gw * rs, Ho = gh * rs;
   const int L = gh * gw;
   const int ld = C * rs * rs;
@@ -97,6 +103,8 @@ __global__ void kv_append_kernel(const float* __restrict__ k, const float* __res
                                  int rows, int slot, int pitch, __nv_bfloat16* __restrict__ k_ring,
                                  __half* __restrict__ vt_ring) {
   __shared__ float tile[64][33];
+  grid_dep_wait();
+  grid_dep_launch();
   const int g = blockIdx.y;
   const int r0 = blockIdx.x * 32;
   const size_t src = static_cast<size_t>(g) * rows * kHeadDim;
@@ -118,7 +126,11 @@ __global__ void kv_append_kernel(const float* __restrict__ k, const float* __res
   }
 }
 
-__global__ void advance_kernel(int* step) { *step += 1; }
+__global__ void advance_kernel(int* step) {
+  grid_dep_wait();
+  grid_dep_launch();
+  *step += 1;
+}
 
 struct RopeSets {
   int frames[kMaxRopeSets];
@@ -128,6 +140,8 @@ struct RopeSets {
 // one thread per (set, frame, pair): angles reduced and evaluated in fp64, stored as fp32
 __global__ void rope_table_kernel(const int* step_dev, int t_host, int nsets, int band_t,
                                   RopeSets sets, float2* table) {
+  grid_dep_wait();
+  grid_dep_launch();
   const int t = step_dev ? *step_dev : t_host;
   int off = 0;
   for (int k = 0; k < nsets; ++k) {
@@ -152,29 +166,28 @@ static int grid_for(long long work, int threads) {
 cudaError_t launch_unshuffle(const float* z, int C, int H, int W, int p, __nv_bfloat16* x0,
                              cudaStream_t s) {
   const long long total = static_cast<long long>(H / p) * (W / p) * C * p * p;
-  unshuffle_kernel<<<grid_for(total, 256), 256, 0, s>>>(z, C, H, W, p, x0);
-  return cudaGetLastError();
+  return launch_pdl(unshuffle_kernel, dim3(grid_for(total, 256)), dim3(256), 0, s, z, C, H, W, p,
+                    x0);
 }
 
 cudaError_t launch_rmsnorm(const float* h, const float* g, int M, int D, float eps,
                            __nv_bfloat16* u, cudaStream_t s) {
-  rmsnorm_kernel<<<(M + 7) / 8, 256, 0, s>>>(h, g, M, D, eps, u);
-  return cudaGetLastError();
+  return launch_pdl(rmsnorm_kernel, dim3((M + 7) / 8), dim3(256), 0, s, h, g, M, D, eps, u);
 }
 
 cudaError_t launch_pixel_head(const float* F, int frames, int gh, int gw, int C, int rs,
                               int out_u8, void* pix, cudaStream_t s) {
   const long long total = static_cast<long long>(C) * frames * gh * rs * gw * rs / 4;
-  pixel_head_kernel<<<grid_for(total, 256), 256, 0, s>>>(F, frames, gh, gw, C, rs, out_u8, pix);
-  return cudaGetLastError();
+  return launch_pdl(pixel_head_kernel, dim3(grid_for(total, 256)), dim3(256), 0, s, F, frames, gh,
+                    gw, C, rs, out_u8, pix);
 }
 
 cudaError_t launch_kv_append(const float* k, const float* v, int groups, int rows, int slot,
                              int ring_pitch, __nv_bfloat16* k_ring, __half* vt_ring,
                              cudaStream_t s) {
   dim3 grid((rows + 31) / 32, groups);
-  kv_append_kernel<<<grid, dim3(32, 8), 0, s>>>(k, v, rows, slot, ring_pitch, k_ring, vt_ring);
-  return cudaGetLastError();
+  return launch_pdl(kv_append_kernel, grid, dim3(32, 8), 0, s, k, v, rows, slot, ring_pitch,
+                    k_ring, vt_ring);
 }
 
 cudaError_t launch_rope_table(const int* step_dev, int t_host, int nsets, const int* frames,
@@ -185,13 +198,12 @@ cudaError_t launch_rope_table(const int* step_dev, int t_host, int nsets, const 
   RopeSets sets{};
   for (int k = 0; k < nsets; ++k) sets.frames[k] = frames[k];
   for (int i = 0; i < band_t; ++i) sets.inv_freq[i] = inv_freq[i];
-  rope_table_kernel<<<1, 128, 0, s>>>(step_dev, t_host, nsets, band_t, sets, table);
-  return cudaGetLastError();
+  return launch_pdl(rope_table_kernel, dim3(1), dim3(128), 0, s, step_dev, t_host, nsets, band_t,
+                    sets, table);
 }
 
 cudaError_t launch_advance(int* step_dev, cudaStream_t s) {
-  advance_kernel<<<1, 1, 0, s>>>(step_dev);
-  return cudaGetLastError();
+  return launch_pdl(advance_kernel, dim3(1), dim3(1), 0, s, step_dev);
 }
 
 }  // namespace fd
