@@ -28,7 +28,30 @@ __global__ void unshuffle_kernel(const float* __restrict__ z, int C, int H, int 
   }
 }
 
-// one warp per row; D % 128 == 0
+// one warp per row, the row held in registers (D / 128 float4 per lane, D % 128 == 0,
+// D <= 128 * kMaxChunks): one pass over h
+constexpr int kMaxChunks = 16;
+template <int CH>
+__device__ __forceinline__ void rmsnorm_row(const float4* hr, const float4* g4, int lane,
+                                            float inv_d, float eps, uint2* ur) {
+  float4 v[CH];
+  float ss = 0.f;
+#pragma unroll
+  for (int c = 0; c < CH; ++c) {
+    v[c] = hr[lane + 32 * c];
+    ss = fmaf(v[c].x, v[c].x, fmaf(v[c].y, v[c].y, fmaf(v[c].z, v[c].z, fmaf(v[c].w, v[c].w, ss))));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  const float r = rsqrtf(ss * inv_d + eps);
+#pragma unroll
+  for (int c = 0; c < CH; ++c) {
+    const float4 gg = g4[lane + 32 * c];
+    ur[lane + 32 * c] = make_uint2(pack_bf16x2(v[c].x * r * gg.x, v[c].y * r * gg.y),
+                                   pack_bf16x2(v[c].z * r * gg.z, v[c].w * r * gg.w));
+  }
+}
+
 __global__ void rmsnorm_kernel(const float* __restrict__ h, const float* __restrict__ g, int M,
                                int D, float eps, __nv_bfloat16* __restrict__ u) {
   grid_dep_wait();
@@ -38,20 +61,30 @@ __global__ void rmsnorm_kernel(const float* __restrict__ h, const float* __restr
   if (row >= M) return;
   const float4* hr = reinterpret_cast<const float4*>(h + static_cast<size_t>(row) * D);
   const float4* g4 = reinterpret_cast<const float4*>(g);
-  float ss = 0.f;
-  for (int c = lane; c < D / 4; c += 32) {
-    const float4 v = hr[c];
-    ss = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, ss))));
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-  const float r = rsqrtf(ss / static_cast<float>(D) + eps);
   uint2* ur = reinterpret_cast<uint2*>(u + static_cast<size_t>(row) * D);
-  for (int c = lane; c < D / 4; c += 32) {
-    const float4 v = hr[c];
-    const float4 gg = g4[c];
-    ur[c] = make_uint2(pack_bf16x2(v.x * r * gg.x, v.y * r * gg.y),
-                       pack_bf16x2(v.z * r * gg.z, v.w * r * gg.w));
+  const float inv_d = 1.0f / static_cast<float>(D);
+  switch (D / 128) {  // chunks of 128 elements per lane-row
+    case 2: rmsnorm_row<2>(hr, g4, lane, inv_d, eps, ur); break;
+    case 4: rmsnorm_row<4>(hr, g4, lane, inv_d, eps, ur); break;
+    case 8: rmsnorm_row<8>(hr, g4, lane, inv_d, eps, ur); break;
+    case 12: rmsnorm_row<12>(hr, g4, lane, inv_d, eps, ur); break;
+    case 16: rmsnorm_row<16>(hr, g4, lane, inv_d, eps, ur); break;
+    default: {  // any other multiple of 128: two passes
+      float ss = 0.f;
+      for (int c = lane; c < D / 4; c += 32) {
+        const float4 v = hr[c];
+        ss = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, ss))));
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+      const float r = rsqrtf(ss * inv_d + eps);
+      for (int c = lane; c < D / 4; c += 32) {
+        const float4 v = hr[c];
+        const float4 gg = g4[c];
+        ur[c] = make_uint2(pack_bf16x2(v.x * r * gg.x, v.y * r * gg.y),
+                           pack_bf16x2(v.z * r * gg.z, v.w * r * gg.w));
+      }
+    }
   }
 }
 
