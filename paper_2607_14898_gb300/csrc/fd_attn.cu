@@ -24,8 +24,8 @@
 //                 tile's softmax has read S(j), then P V of block j once P(j) is written
 //   warps 0-3 / 4-7  softmax of tile 0 / 1, one query row (TMEM lane) per thread: load S,
 //                 release it, running max in the log2 domain and running row sum in
-//                 registers, P = exp2(s - m) as fp16 into P_X (after the previous P V has read
-//                 it). O_X is rescaled in TMEM (load, multiply, store) only when a row's max
+//                 registers, P = exp2(s - m) as fp16 in registers, then into P_X once the
+//                 previous P V has read it. O_X is rescaled in TMEM (load, multiply, store) only when a row's max
 //                 grows by more than 2^8, so P stays <= 256 and the rescale is rare.
 #include "fd_internal.h"
 #include "fd_ptx.cuh"
@@ -248,6 +248,32 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       const float mb = mx * sl2;
       const bool grow = mb > m_used + kRescaleLog2;
       const float m_new = grow ? mb : m_used;
+      // P = exp2(s * scale - m) in fp16 pairs: one packed FMA, one rounding to fp16 and one
+      // packed ex2 per two keys; the row sum is a pairwise fp16x2 tree per 64 keys (sums stay
+      // below 2^15 because P <= 2^8) added into fp32. This runs while the tensor core may
+      // still be reading P_X(j-1): only the store of P(j) and the rescale of O wait for it.
+      const uint64_t sc2 = pack_f32x2(sl2, sl2);
+      const uint64_t ng2 = pack_f32x2(-m_new, -m_new);
+      float lsum = 0.f;
+      uint32_t pk[2][32];
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc)
+#pragma unroll
+          for (int e = 0; e < 32; e += 2)
+            pk[half][cc * 16 + (e >> 1)] =
+                exp2_pair_f16(__uint_as_float(sr[2 * half + cc][e]),
+                              __uint_as_float(sr[2 * half + cc][e + 1]), sc2, ng2);
+        uint32_t t16[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) t16[i] = hadd2(pk[half][2 * i], pk[half][2 * i + 1]);
+#pragma unroll
+        for (int stride = 8; stride > 0; stride >>= 1)
+#pragma unroll
+          for (int i = 0; i < stride; ++i) t16[i] = hadd2(t16[i], t16[i + stride]);
+        lsum += f16x2_sum(t16[0]);
+      }
       // P_X and O_X are free once the P V of the previous block has completed
       if (j > 0) {
         const bool pv = mbar_wait(bar(kBarPv + x), (j - 1) & 1, p.err, ERR_WAIT_MMA);
@@ -271,32 +297,8 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         }
       }
       m_used = m_new;
-      // P = exp2(s * scale - m) in fp16 pairs: one packed FMA, one rounding to fp16 and one
-      // packed ex2 per two keys; the row sum is a pairwise fp16x2 tree per 64 keys (sums stay
-      // below 2^15 because P <= 2^8) added into fp32
-      const uint64_t sc2 = pack_f32x2(sl2, sl2);
-      const uint64_t ng2 = pack_f32x2(-m_used, -m_used);
-      float lsum = 0.f;
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        uint32_t pk[32];
-#pragma unroll
-        for (int cc = 0; cc < 2; ++cc)
-#pragma unroll
-          for (int e = 0; e < 32; e += 2)
-            pk[cc * 16 + (e >> 1)] = exp2_pair_f16(__uint_as_float(sr[2 * half + cc][e]),
-                                                   __uint_as_float(sr[2 * half + cc][e + 1]),
-                                                   sc2, ng2);
-        tmem_st_32x32b_x32(p_col + 32 * half, pk);
-        uint32_t t16[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) t16[i] = hadd2(pk[2 * i], pk[2 * i + 1]);
-#pragma unroll
-        for (int stride = 8; stride > 0; stride >>= 1)
-#pragma unroll
-          for (int i = 0; i < stride; ++i) t16[i] = hadd2(t16[i], t16[i + stride]);
-        lsum += f16x2_sum(t16[0]);
-      }
+      tmem_st_32x32b_x32(p_col, pk[0]);
+      tmem_st_32x32b_x32(p_col + 32, pk[1]);
       l_run += lsum;
       tmem_st_wait();
       tc_fence_before();
