@@ -25,7 +25,8 @@
 //   warps 0-3 / 4-7  softmax of tile 0 / 1, one query row (TMEM lane) per thread: load S,
 //                 release it, running max in the log2 domain and running row sum in
 //                 registers, P = exp2(s - m) as fp16 in registers, then into P_X once the
-//                 previous P V has read it. O_X is rescaled in TMEM (load, multiply, store) only when a row's max
+//                 previous P V has read it. The two tiles' warps on one SMSP alternate on the
+//                 exponentials. O_X is rescaled in TMEM (load, multiply, store) only when a row's max
 //                 grows by more than 2^8, so P stays <= 256 and the rescale is rare.
 #include "fd_internal.h"
 #include "fd_ptx.cuh"
@@ -54,7 +55,9 @@ constexpr int kBarQ = 0, kBarKvFull = 1, kBarKvEmpty = kBarKvFull + kStages,
               kBarP = kBarSFree + 2,           // [tile] P_X(j) written
               kBarPv = kBarP + 2,              // [tile] P V of block j completed
               kBarDone = kBarPv + 2,           // [tile] every MMA of the tile's issuer completed
-              kNumBars = kBarDone + 2;
+              kBarTurn = kBarDone + 2,  // [tile][quarter] the other tile's warp of this SMSP
+                                        // has finished its exponentials: this tile's turn
+              kNumBars = kBarTurn + 8;
 static_assert(kNumBars * 8 + 4 <= 256, "barrier area");
 static_assert(kSmem <= 227 * 1024, "shared memory");
 }  // namespace attn
@@ -98,6 +101,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       mbar_init(bar(kBarPv + x), 1);
       mbar_init(bar(kBarDone + x), 1);
     }
+    for (int i = 0; i < 8; ++i) mbar_init(bar(kBarTurn + i), 1);
     fence_barrier_init();
   }
   grid_dep_wait();  // Q and the ring written by the previous kernels; TMEM freed by their CTAs
@@ -252,6 +256,18 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       // packed ex2 per two keys; the row sum is a pairwise fp16x2 tree per 64 keys (sums stay
       // below 2^15 because P <= 2^8) added into fp32. This runs while the tensor core may
       // still be reading P_X(j-1): only the store of P(j) and the rescale of O wait for it.
+      // Warp q of tile 0 and warp q of tile 1 share one SMSP, whose conversion and ex2 units
+      // bound this loop. They take turns on the exponentials (tile 0 block j, tile 1 block j,
+      // tile 0 block j+1, ...), so each one's S load, P V wait and P store run while the other
+      // computes instead of both stalling at once.
+      if (x == 1 || j > 0) {
+        const bool turn = mbar_wait(bar(kBarTurn + 4 * x + quarter), (x == 1 ? j : j - 1) & 1,
+                                    p.err, ERR_WAIT_EPI);
+        if (!__all_sync(0xffffffffu, turn)) {
+          ok = false;
+          break;
+        }
+      }
       const uint64_t sc2 = pack_f32x2(sl2, sl2);
       const uint64_t ng2 = pack_f32x2(-m_new, -m_new);
       float lsum = 0.f;
@@ -274,6 +290,8 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
           for (int i = 0; i < stride; ++i) t16[i] = hadd2(t16[i], t16[i + stride]);
         lsum += f16x2_sum(t16[0]);
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(kBarTurn + 4 * (1 - x) + quarter));
       // P_X and O_X are free once the P V of the previous block has completed
       if (j > 0) {
         const bool pv = mbar_wait(bar(kBarPv + x), (j - 1) & 1, p.err, ERR_WAIT_MMA);
