@@ -5,8 +5,10 @@
 // softmax does not depend on key order, so no mask tensor is needed; only the ragged last key
 // block is cut at n_keys. GQA: head n reads KV group n / (N / G).
 //
-// One CTA = two 128-row tiles X = 0, 1 sharing one KV group (two heads of the group on one
-// query tile, or two query tiles of one head), so each K / V block is loaded once for both.
+// GQA row packing: the query rows of the heads sharing KV group g form one row space (head
+// after head, each head's Lq rows padded to lq_pad, a multiple of 8). One CTA = two consecutive
+// 128-row tiles X = 0, 1 of one group's row space, so each K / V block is loaded once for both
+// and the only padding is at the end of the group, not at the end of every head.
 // Optionally the key range is split over `splits` CTAs whose partial results a second kernel
 // combines (balances the grid over the SMs).
 //
@@ -67,7 +69,8 @@ __device__ __forceinline__ float add_pair(uint32_t a, uint32_t b) {
 }
 
 __global__ void __launch_bounds__(attn::kThreads, 1)
-    attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+    attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQ8,
+                const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
   using namespace attn;
   extern __shared__ __align__(1024) uint8_t smem[];
@@ -80,12 +83,9 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
   auto bar = [&](int i) { return bar0 + 8u * static_cast<uint32_t>(i); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kNumBars);
 
-  // the two tiles of this CTA: (query tile qt0, head hd0) and (qt1, hd1)
-  const int qt0 = p.pair_heads ? blockIdx.x : 2 * blockIdx.x;
-  const int qt1 = p.pair_heads ? blockIdx.x : 2 * blockIdx.x + 1;
-  const int hd0 = p.pair_heads ? 2 * blockIdx.y : blockIdx.y;
-  const int hd1 = p.pair_heads ? 2 * blockIdx.y + 1 : blockIdx.y;
-  const int g = hd0 / (p.heads / p.groups);
+  // the two tiles of this CTA: packed rows (2 blockIdx.x + X) * 128 + i of KV group g
+  const int g = blockIdx.y;
+  const int hpg = p.heads / p.groups;
 
   if (threadIdx.x == 0) {
     if (!aligned) atomicOr(p.err, ERR_SMEM_ALIGN);
@@ -128,11 +128,33 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
     // ------------------------------------------------------------ TMA loads
     if (lane == 0 && aligned && nblk > 0) {
       prefetch_tmap(&tmQ);
+      prefetch_tmap(&tmQ8);
       prefetch_tmap(&tmK);
       prefetch_tmap(&tmV);
       mbar_expect_tx(bar(kBarQ), 2 * kQBytes);
-      tma_load_2d(base + kOffQ, &tmQ, bar(kBarQ), hd0 * kHeadDim, qt0 * kBM);
-      tma_load_2d(base + kOffQ + kQBytes, &tmQ, bar(kBarQ), hd1 * kHeadDim, qt1 * kBM);
+      // A tile inside one head's rows is one 128-row box (rows past Lq read the fill value);
+      // a tile across two heads is loaded in boxes of 8 rows (one 1024-byte swizzle atom
+      // each, same shared-memory layout). Rows past the group's last head load head 0's
+      // first rows; their outputs are not written.
+      for (int x = 0; x < 2; ++x) {
+        const int rho0 = (2 * blockIdx.x + x) * kBM;
+        const int hl0 = rho0 / p.lq_pad;
+        const int hl1 = (rho0 + kBM - 1) / p.lq_pad;
+        const uint32_t dst = base + kOffQ + x * kQBytes;
+        if (hl0 >= hpg) {
+          tma_load_2d(dst, &tmQ, bar(kBarQ), g * hpg * kHeadDim, 0);
+        } else if (hl1 == hl0 || hl1 >= hpg) {
+          tma_load_2d(dst, &tmQ, bar(kBarQ), (g * hpg + hl0) * kHeadDim, rho0 - hl0 * p.lq_pad);
+        } else {
+          for (int b = 0; b < kBM / 8; ++b) {
+            const int rho = rho0 + 8 * b;
+            int hl = rho / p.lq_pad;
+            int r = rho - hl * p.lq_pad;
+            if (hl >= hpg) hl = r = 0;
+            tma_load_2d(dst + b * 1024, &tmQ8, bar(kBarQ), (g * hpg + hl) * kHeadDim, r);
+          }
+        }
+      }
       int j = 0;
       for (; j < nblk; ++j) {
         const int st = j % kStages;
@@ -342,9 +364,11 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         }
       }
     }
-    const int r = (x ? qt1 : qt0) * kBM + row;
-    if (ok && r < p.Lq) {
-      const int h = x ? hd1 : hd0;
+    const int rho = (2 * blockIdx.x + x) * kBM + row;
+    const int hl = rho / p.lq_pad;
+    const int r = rho - hl * p.lq_pad;
+    if (ok && hl < hpg && r < p.Lq) {
+      const int h = g * hpg + hl;
       if (p.splits == 1) {
         const float inv = 1.0f / l_run;
         uint4* dst = reinterpret_cast<uint4*>(p.out + static_cast<size_t>(r) * p.ld_out +
@@ -420,7 +444,8 @@ int attention_splits(int units, int nblk, int num_sms) {
   return best;
 }
 
-cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmK,
+cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmQ8,
+                             const CUtensorMap& tmK,
                              const CUtensorMap& tmVt, const AttnParams& p, cudaStream_t s) {
   static bool attr_set = false;
   if (!attr_set) {
@@ -429,10 +454,9 @@ cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmK,
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  const int qtiles = (p.Lq + kBM - 1) / kBM;
-  dim3 grid = p.pair_heads ? dim3(qtiles, p.heads / 2, p.splits)
-                           : dim3((qtiles + 1) / 2, p.heads, p.splits);
-  cudaError_t e = launch_pdl(attn_kernel, grid, dim3(attn::kThreads), attn::kSmem, s, tmQ, tmK,
+  const int tiles = attention_tiles_per_group(p.Lq, p.heads, p.groups);
+  const dim3 grid((tiles + 1) / 2, p.groups, p.splits);
+  cudaError_t e = launch_pdl(attn_kernel, grid, dim3(attn::kThreads), attn::kSmem, s, tmQ, tmQ8, tmK,
                              tmVt, p);
   if (e != cudaSuccess || p.splits == 1) return e;
   const long long warps = static_cast<long long>(p.Lq) * p.heads;

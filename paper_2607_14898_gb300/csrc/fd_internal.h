@@ -95,7 +95,7 @@ struct AttnParams {
   int ld_out;
   float scale_log2;          // log2(e) / sqrt(D_h)
   int* err;
-  int pair_heads;            // 1: a CTA takes heads 2p, 2p+1 of one q tile; 0: q tiles 2i, 2i+1
+  int lq_pad;                // query rows per head in the packed row space (Lq rounded up to 8)
   int splits;                // key-range splits per (q tile, head); > 1 writes partials
   float* part_o;             // [splits][heads][Lq][64] unnormalised O   (splits > 1)
   float* part_ml;            // [splits][heads][Lq][2]  (max used, row sum) (splits > 1)
@@ -106,8 +106,21 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CU
                         const CUtensorMap& tmK, const CUtensorMap& tmV, const GemmParams& p,
                         int bn, int num_sms, cudaStream_t s);
 // Attention (+ the combine of key-range splits when p.splits > 1).
-cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmK,
+// tmQ: Q [Lq][heads * 64] bf16 in boxes of 64 x 128 rows; tmQ8: the same in boxes of 64 x 8.
+cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmQ8,
+                             const CUtensorMap& tmK,
                              const CUtensorMap& tmVt, const AttnParams& p, cudaStream_t s);
+// GQA row packing: the query rows of the heads that share KV group g form one row space,
+// head after head, each head's rows padded to a multiple of 8 (so a TMA box of 8 rows never
+// holds two heads); 128-row tiles run over that space and a CTA takes two tiles of one group.
+inline int attention_lq_pad(int Lq) { return (Lq + 7) / 8 * 8; }
+inline int attention_tiles_per_group(int Lq, int heads, int groups) {
+  return ((heads / groups) * attention_lq_pad(Lq) + 127) / 128;
+}
+// CTAs per key-range split
+inline int attention_units(int Lq, int heads, int groups) {
+  return groups * ((attention_tiles_per_group(Lq, heads, groups) + 1) / 2);
+}
 // Key-range splits that balance (units x splits) CTAs over the SMs for nblk key blocks.
 int attention_splits(int units, int nblk, int num_sms);
 // Workspace floats needed by a split attention of Lq rows.

@@ -293,6 +293,7 @@ struct fd_handle_s {
   float2* rope_tab = nullptr;
   // A-operand / Q descriptors
   CUtensorMap tm_x0, tm_uB, tm_uR, tm_oB, tm_oR, tm_hidB, tm_hidR, tm_hidH, tm_qB, tm_qR;
+  CUtensorMap tm_q8B, tm_q8R;  // attention Q in 8-row boxes (tiles across two heads)
   // epilogue store descriptors
   CUtensorMap so_h, so_hf, so_tup, so_hidB, so_hidR, so_hidH, so_F, so_qB, so_qR;
   // host-buffer decode: library-owned device copies of the latent and the pixels
@@ -362,13 +363,10 @@ fd_status traced(fd_handle h, int kind, cudaStream_t s, Fn&& fn) {
   return FD_OK;
 }
 
-int pair_heads(int heads, int groups) { return (heads / groups) % 2 == 0 ? 1 : 0; }
-
 // key-range splits for an attention of Lq rows over n_keys keys
 int choose_splits(int Lq, int heads, int groups, int n_keys) {
-  const int qtiles = (Lq + 127) / 128;
-  const int units = pair_heads(heads, groups) ? qtiles * (heads / 2) : ((qtiles + 1) / 2) * heads;
-  return fd::attention_splits(units, (n_keys + 127) / 128, num_sms());
+  return fd::attention_splits(fd::attention_units(Lq, heads, groups), (n_keys + 127) / 128,
+                              num_sms());
 }
 
 fd_status run_linear(fd_handle h, int kind, const CUtensorMap& tmA, const Linear& lin, int M,
@@ -420,12 +418,15 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
   a.window = d.Wn; a.step_dev = h->state; a.n_keys_host = 0; a.out = h->o;
   a.ld_out = d.N * kHeadDim; a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
   a.err = h->state + 1;
-  a.pair_heads = pair_heads(d.N, d.G);
+  a.lq_pad = fd::attention_lq_pad(rows);
   a.splits = refine ? h->splitsR : h->splitsB;
   a.part_o = h->attn_ws;
   a.part_ml = h->attn_ws + static_cast<size_t>(a.splits) * d.N * rows * kHeadDim;
   if ((st = traced(h, refine ? FD_K_ATTN_R : FD_K_ATTN_B, s,
-                   [&] { return fd::launch_attention(tm_q, r.tm_k, r.tm_vt, a, s); })))
+                   [&] {
+                     return fd::launch_attention(tm_q, refine ? h->tm_q8R : h->tm_q8B, r.tm_k,
+                                                 r.tm_vt, a, s);
+                   })))
     return st;
 
   fd::GemmParams po{};
@@ -775,6 +776,8 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   ok = ok && tmap_bf16(&h->tm_oR, h->o, NQ, R, NQ * 2, 64, 128);
   ok = ok && tmap_bf16(&h->tm_qB, h->q, NQ, d.L, NQ * 2, 64, 128);
   ok = ok && tmap_bf16(&h->tm_qR, h->q, NQ, R, NQ * 2, 64, 128);
+  ok = ok && tmap_bf16(&h->tm_q8B, h->q, NQ, d.L, NQ * 2, 64, 8);
+  ok = ok && tmap_bf16(&h->tm_q8R, h->q, NQ, R, NQ * 2, 64, 8);
   ok = ok && tmap_bf16(&h->tm_hidB, h->hid, Dm, d.L, Dm * 2, 64, 128);
   ok = ok && tmap_bf16(&h->tm_hidR, h->hid, Dm, R, Dm * 2, 64, 128);
   ok = ok && tmap_bf16(&h->tm_hidH, h->hid, d.D, R, static_cast<uint64_t>(d.D) * 2, 64, 128);
@@ -1049,8 +1052,8 @@ fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const vo
   fd_status st = check_device();
   if (st) return st;
   const uint64_t NQ = static_cast<uint64_t>(heads) * kHeadDim;
-  CUtensorMap tq, tk, tv;
-  if (!tmap_bf16(&tq, q, NQ, Lq, NQ * 2, 64, 128) ||
+  CUtensorMap tq, tq8, tk, tv;
+  if (!tmap_bf16(&tq, q, NQ, Lq, NQ * 2, 64, 128) || !tmap_bf16(&tq8, q, NQ, Lq, NQ * 2, 64, 8) ||
       !tmap_bf16(&tk, k_ring, kHeadDim, static_cast<uint64_t>(groups) * ring_pitch, kHeadDim * 2,
                  64, 128) ||
       !tmap_f16(&tv, vt_ring, ring_pitch, static_cast<uint64_t>(groups) * kHeadDim,
@@ -1062,11 +1065,11 @@ fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const vo
   a.out = static_cast<__nv_bfloat16*>(out); a.ld_out = static_cast<int>(NQ);
   a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
   a.err = err_dev;
-  a.pair_heads = pair_heads(heads, groups);
+  a.lq_pad = fd::attention_lq_pad(Lq);
   a.splits = splits;
   a.part_o = static_cast<float*>(workspace);
   a.part_ml = a.part_o + static_cast<size_t>(splits) * heads * Lq * kHeadDim;
-  return launch_ok(fd::launch_attention(tq, tk, tv, a, static_cast<cudaStream_t>(stream)));
+  return launch_ok(fd::launch_attention(tq, tq8, tk, tv, a, static_cast<cudaStream_t>(stream)));
 }
 
 }  // extern "C"
