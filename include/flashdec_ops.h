@@ -62,37 +62,41 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
  * q bf16 [Lq][heads*64]; k_ring bf16 [groups][ring_pitch][64]; vt_ring fp16
  * [groups][64][ring_pitch]; out bf16 [Lq][heads*64]. 1 <= n_keys <= ring_pitch,
  * ring_pitch % 128 == 0. Ring entries past n_keys must hold finite values.
- * splits: the key range is divided over `splits` CTAs per (query tile, head) whose partial
- * results a second kernel combines (0 = library choice, 1..16). With more than one split,
- * `workspace` is a caller-owned device buffer of fd_attention_workspace_bytes(...) bytes
- * (16-byte aligned) that the call overwrites; calls sharing it must not overlap. */
-size_t fd_attention_workspace_bytes(int Lq, int heads, int groups, int n_keys, int splits);
+ * parts: CTAs of the launch (0 = library choice, one per SM; 1..4096). The launch is
+ * persistent: the query rows of the heads of each KV group are packed into 128-row tiles, the
+ * (tile pair x 128-key block) units are cut into `parts` equal runs, one per CTA, and a tile
+ * pair whose keys fall into several runs is finished by combining partial results. With
+ * parts > 1, `workspace` is a caller-owned device buffer of fd_attention_workspace_bytes(...)
+ * bytes (16-byte aligned) that the call overwrites (its counters are cleared on `stream` first);
+ * calls sharing it must not overlap. The combine order is fixed: results do not depend on
+ * which CTA finishes first. */
+size_t fd_attention_workspace_bytes(int Lq, int heads, int groups, int n_keys, int parts);
 fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const void* k_ring,
                           const void* vt_ring, int ring_pitch, int n_keys, void* out,
-                          int splits, void* workspace, int* err_dev, void* stream);
+                          int parts, void* workspace, int* err_dev, void* stream);
 
 /* Allocation-free variant of fd_op_attention. The paper has no counterpart: this is a library
  * convenience for callers that cannot call cudaMalloc, for example code that runs while a CUDA
  * stream is being captured into a graph (allocation is not allowed there), plug-ins that must
  * stay inside a device-memory budget handed to them by a host framework, and real-time loops
  * that cannot afford the device synchronisation an allocation may cause. Such callers can pass
- * their own inputs and outputs but have no way to provide the key-range-split workspace.
+ * their own inputs and outputs but have no way to provide the partial-result workspace.
  * This call takes that workspace from one array in the library's static device memory,
- * FD_STATIC_ATTN_SCRATCH_BYTES (16 MiB) on every GPU that loads the library, held until the
+ * FD_STATIC_ATTN_SCRATCH_BYTES (32 MiB) on every GPU that loads the library, held until the
  * process exits. It allocates nothing: no cudaMalloc, cudaFree or allocating library routine.
- *   - Arguments and results are those of fd_op_attention without `workspace`. splits = 0 lets
- *     the library choose. If splits * heads * Lq * 66 * 4 bytes would exceed the static size,
- *     the call returns FD_ERR_INVALID_ARG and launches nothing (pass fewer splits; splits = 1
- *     uses no workspace at all).
+ *   - Arguments and results are those of fd_op_attention without `workspace`. parts = 0 lets
+ *     the library choose (one CTA per SM: about 135 KB per SM). If
+ *     fd_attention_workspace_bytes(..., parts) would exceed the static size, the call returns
+ *     FD_ERR_INVALID_ARG and launches nothing (pass fewer parts; parts = 1 uses no workspace).
  *   - The first call on a device looks up the array's device address with that device current
  *     (cudaGetSymbolAddress); make that first call before any stream capture begins.
- *   - Every call shares the one array and writes every entry it later reads, so nothing needs
- *     clearing between calls; calls whose kernels overlap on the GPU (unordered streams) race
- *     on the array and may return wrong results. */
-#define FD_STATIC_ATTN_SCRATCH_BYTES (16u << 20)
+ *   - Every call shares the one array; it clears the array's counters on `stream` (a memset,
+ *     not an allocation) and writes every other entry it later reads. Calls whose kernels
+ *     overlap on the GPU (unordered streams) race on the array and may return wrong results. */
+#define FD_STATIC_ATTN_SCRATCH_BYTES (32u << 20)
 fd_status fd_op_attention_static(int Lq, int heads, int groups, const void* q,
                                  const void* k_ring, const void* vt_ring, int ring_pitch,
-                                 int n_keys, void* out, int splits, int* err_dev, void* stream);
+                                 int n_keys, void* out, int parts, int* err_dev, void* stream);
 
 /* Rolling-cache append (Algorithm 1, cache update): fp32 k, v [groups][rows][64] rounded to
  * nearest even into ring slot s = t mod window: k_ring[g][s*rows + r][d] (bf16) and

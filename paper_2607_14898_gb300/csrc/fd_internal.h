@@ -96,9 +96,11 @@ struct AttnParams {
   float scale_log2;          // log2(e) / sqrt(D_h)
   int* err;
   int lq_pad;                // query rows per head in the packed row space (Lq rounded up to 8)
-  int splits;                // key-range splits per (q tile, head); > 1 writes partials
-  float* part_o;             // [splits][heads][Lq][64] unnormalised O   (splits > 1)
-  float* part_ml;            // [splits][heads][Lq][2]  (max used, row sum) (splits > 1)
+  int parts;                 // CTAs of the persistent launch; each takes an equal run of the
+                             // (tile pair, key block) units
+  float* part_o;             // [parts][2 slots][2 tiles][16][128 rows] float4 partial O
+  float* part_ml;            // [parts][2][2][128] (running max, row sum)
+  int* counters;             // [pairs] partial results stored per pair; zero between launches
 };
 
 // launch wrappers; return cudaGetLastError() of the launch
@@ -113,19 +115,28 @@ cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmQ8,
 // GQA row packing: the query rows of the heads that share KV group g form one row space,
 // head after head, each head's rows padded to a multiple of 8 (so a TMA box of 8 rows never
 // holds two heads); 128-row tiles run over that space and a CTA takes two tiles of one group.
-inline int attention_lq_pad(int Lq) { return (Lq + 7) / 8 * 8; }
-inline int attention_tiles_per_group(int Lq, int heads, int groups) {
+__host__ __device__ inline int attention_lq_pad(int Lq) { return (Lq + 7) / 8 * 8; }
+__host__ __device__ inline int attention_tiles_per_group(int Lq, int heads, int groups) {
   return ((heads / groups) * attention_lq_pad(Lq) + 127) / 128;
 }
-// CTAs per key-range split
+// tile pairs (two 128-row tiles of one KV group) of an attention
 inline int attention_units(int Lq, int heads, int groups) {
   return groups * ((attention_tiles_per_group(Lq, heads, groups) + 1) / 2);
 }
-// Key-range splits that balance (units x splits) CTAs over the SMs for nblk key blocks.
-int attention_splits(int units, int nblk, int num_sms);
-// Workspace floats needed by a split attention of Lq rows.
-inline size_t attention_workspace_floats(int splits, int heads, int Lq) {
-  return splits <= 1 ? 0 : static_cast<size_t>(splits) * heads * Lq * (64 + 2);
+// CTAs of an attention launch over `units` tile pairs with nblk key blocks each
+int attention_parts(int units, int nblk, int num_sms);
+// Workspace of an attention launch with `parts` CTAs: one int counter per tile pair (room for
+// `pairs` pairs, at the start so that launches with other part counts find them in place),
+// then partial O and (max, sum) for two slots of two tiles per CTA.
+constexpr size_t kAttnPartFloats = 4 * (64 * 128 + 2 * 128);
+inline size_t attention_counter_floats(int pairs) { return (static_cast<size_t>(pairs) + 3) / 4 * 4; }
+inline size_t attention_workspace_floats(int parts, int pairs) {
+  return parts <= 1 ? 0 : attention_counter_floats(pairs) + static_cast<size_t>(parts) * kAttnPartFloats;
+}
+inline void attention_workspace_split(float* ws, int parts, int pairs, AttnParams& a) {
+  a.counters = reinterpret_cast<int*>(ws);
+  a.part_o = ws ? ws + attention_counter_floats(pairs) : nullptr;
+  a.part_ml = ws ? a.part_o + static_cast<size_t>(parts) * 4 * 64 * 128 : nullptr;
 }
 cudaError_t launch_unshuffle(const float* z, int C, int H, int W, int p, __nv_bfloat16* x0,
                              cudaStream_t s);

@@ -287,7 +287,7 @@ struct fd_handle_s {
   std::vector<Ring> ringB, ringR;
   // attention key-range splits (fixed per stack for the steady-state window) and their
   // partial-result workspace
-  int splitsB = 1, splitsR = 1;
+  int partsB = 1, partsR = 1;  // CTAs of the backbone / refinement attention launches
   float* attn_ws = nullptr;
   // temporal RoPE (cos, sin) of the current chunk: backbone frame, then the r_t refined frames
   float2* rope_tab = nullptr;
@@ -363,10 +363,17 @@ fd_status traced(fd_handle h, int kind, cudaStream_t s, Fn&& fn) {
   return FD_OK;
 }
 
-// key-range splits for an attention of Lq rows over n_keys keys
-int choose_splits(int Lq, int heads, int groups, int n_keys) {
-  return fd::attention_splits(fd::attention_units(Lq, heads, groups), (n_keys + 127) / 128,
-                              num_sms());
+// tile pairs the attention counters must cover (the larger of backbone and refinement)
+static int attn_pairs(const Dims& d) {
+  const int a = fd::attention_units(d.L, d.N, d.G);
+  const int b = d.nr > 0 ? fd::attention_units(d.rt * d.L, d.N, d.G) : 0;
+  return a > b ? a : b;
+}
+
+// CTAs of an attention of Lq rows over n_keys keys
+int choose_parts(int Lq, int heads, int groups, int n_keys) {
+  return fd::attention_parts(fd::attention_units(Lq, heads, groups), (n_keys + 127) / 128,
+                             num_sms());
 }
 
 fd_status run_linear(fd_handle h, int kind, const CUtensorMap& tmA, const Linear& lin, int M,
@@ -419,9 +426,8 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
   a.ld_out = d.N * kHeadDim; a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
   a.err = h->state + 1;
   a.lq_pad = fd::attention_lq_pad(rows);
-  a.splits = refine ? h->splitsR : h->splitsB;
-  a.part_o = h->attn_ws;
-  a.part_ml = h->attn_ws + static_cast<size_t>(a.splits) * d.N * rows * kHeadDim;
+  a.parts = refine ? h->partsR : h->partsB;
+  fd::attention_workspace_split(h->attn_ws, a.parts, attn_pairs(d), a);
   if ((st = traced(h, refine ? FD_K_ATTN_R : FD_K_ATTN_B, s,
                    [&] {
                      return fd::launch_attention(tm_q, refine ? h->tm_q8R : h->tm_q8B, r.tm_k,
@@ -507,6 +513,8 @@ fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+constexpr int kMaxAttnParts = 4096;  // CTAs of one attention launch (fd_op_attention)
+
 }  // namespace
 
 extern "C" {
@@ -547,11 +555,9 @@ size_t fd_pixels_bytes(const fd_config* cfg) {
 
 static size_t attn_ws_floats(const Dims& d) {
   const int R = d.rt * d.L;
-  const int sB = choose_splits(d.L, d.N, d.G, d.Wn * d.L);
-  const int sR = choose_splits(R, d.N, d.G, d.Wn * R);
-  const size_t a = fd::attention_workspace_floats(sB, d.N, d.L);
-  const size_t b = d.nr > 0 ? fd::attention_workspace_floats(sR, d.N, R) : 0;
-  return a > b ? a : b;
+  const int sB = choose_parts(d.L, d.N, d.G, d.Wn * d.L);
+  const int sR = d.nr > 0 ? choose_parts(R, d.N, d.G, d.Wn * R) : 1;
+  return fd::attention_workspace_floats(sB > sR ? sB : sR, attn_pairs(d));
 }
 
 static size_t handle_layout(const Dims& d, size_t* off /* 16 offsets */, int* pitchB,
@@ -734,8 +740,8 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   h->pixel_buf = b + off[12];
   h->attn_ws = reinterpret_cast<float*>(b + off[13]);
   h->rope_tab = reinterpret_cast<float2*>(b + off[14]);
-  h->splitsB = choose_splits(d.L, d.N, d.G, d.Wn * d.L);
-  h->splitsR = choose_splits(d.rt * d.L, d.N, d.G, d.Wn * d.rt * d.L);
+  h->partsB = choose_parts(d.L, d.N, d.G, d.Wn * d.L);
+  h->partsR = choose_parts(d.rt * d.L, d.N, d.G, d.Wn * d.rt * d.L);
   const size_t ringB_elems = static_cast<size_t>(d.G) * h->pitchB * kHeadDim;
   const size_t ringR_elems = static_cast<size_t>(d.G) * h->pitchR * kHeadDim;
   h->ringB.resize(d.nb);
@@ -850,6 +856,11 @@ fd_status fd_decode_chunk_host(fd_handle h, const float* latent_host, void* pixe
 fd_status fd_reset(fd_handle h) {
   if (h == nullptr) return FD_ERR_INVALID_ARG;
   if (cudaMemsetAsync(h->state, 0, 2 * sizeof(int), h->last_stream) != cudaSuccess)
+    return FD_ERR_CUDA;
+  // a launch stopped by an error may leave attention counters non-zero
+  if (attn_ws_floats(h->d) > 0 &&
+      cudaMemsetAsync(h->attn_ws, 0, sizeof(int) * attn_pairs(h->d), h->last_stream) !=
+          cudaSuccess)
     return FD_ERR_CUDA;
   h->t_host = 0;
   h->error = false;
@@ -1033,22 +1044,23 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
                                    static_cast<cudaStream_t>(stream)));
 }
 
-size_t fd_attention_workspace_bytes(int Lq, int heads, int groups, int n_keys, int splits) {
-  if (Lq < 1 || heads < 1 || groups < 1 || heads % groups || n_keys < 1 || splits < 0)
+size_t fd_attention_workspace_bytes(int Lq, int heads, int groups, int n_keys, int parts) {
+  if (Lq < 1 || heads < 1 || groups < 1 || heads % groups || n_keys < 1 || parts < 0 ||
+      parts > kMaxAttnParts)
     return 0;
-  if (splits == 0) splits = choose_splits(Lq, heads, groups, n_keys);
-  return fd::attention_workspace_floats(splits, heads, Lq) * 4;
+  if (parts == 0) parts = choose_parts(Lq, heads, groups, n_keys);
+  return fd::attention_workspace_floats(parts, fd::attention_units(Lq, heads, groups)) * 4;
 }
 
 fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const void* k_ring,
                           const void* vt_ring, int ring_pitch, int n_keys, void* out,
-                          int splits, void* workspace, int* err_dev, void* stream) {
+                          int parts, void* workspace, int* err_dev, void* stream) {
   if (!q || !k_ring || !vt_ring || !out || !err_dev) return FD_ERR_INVALID_ARG;
   if (Lq < 1 || heads < 1 || groups < 1 || heads % groups || n_keys < 1 ||
-      n_keys > ring_pitch || ring_pitch % 128 || splits < 0 || splits > 16)
+      n_keys > ring_pitch || ring_pitch % 128 || parts < 0 || parts > kMaxAttnParts)
     return FD_ERR_INVALID_ARG;
-  if (splits == 0) splits = choose_splits(Lq, heads, groups, n_keys);
-  if (splits > 1 && (workspace == nullptr || !aligned16(workspace))) return FD_ERR_INVALID_ARG;
+  if (parts == 0) parts = choose_parts(Lq, heads, groups, n_keys);
+  if (parts > 1 && (workspace == nullptr || !aligned16(workspace))) return FD_ERR_INVALID_ARG;
   fd_status st = check_device();
   if (st) return st;
   const uint64_t NQ = static_cast<uint64_t>(heads) * kHeadDim;
@@ -1066,10 +1078,17 @@ fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const vo
   a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
   a.err = err_dev;
   a.lq_pad = fd::attention_lq_pad(Lq);
-  a.splits = splits;
-  a.part_o = static_cast<float*>(workspace);
-  a.part_ml = a.part_o + static_cast<size_t>(splits) * heads * Lq * kHeadDim;
-  return launch_ok(fd::launch_attention(tq, tq8, tk, tv, a, static_cast<cudaStream_t>(stream)));
+  a.parts = parts;
+  const int pairs = fd::attention_units(Lq, heads, groups);
+  fd::attention_workspace_split(parts > 1 ? static_cast<float*>(workspace) : nullptr, parts,
+                                pairs, a);
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the per-pair counters must start at zero (each launch leaves them at zero)
+  if (a.counters != nullptr &&
+      cudaMemsetAsync(a.counters, 0, sizeof(int) * pairs, s) !=
+          cudaSuccess)
+    return FD_ERR_CUDA;
+  return launch_ok(fd::launch_attention(tq, tq8, tk, tv, a, s));
 }
 
 }  // extern "C"
@@ -1105,19 +1124,20 @@ extern "C" {
 
 fd_status fd_op_attention_static(int Lq, int heads, int groups, const void* q,
                                  const void* k_ring, const void* vt_ring, int ring_pitch,
-                                 int n_keys, void* out, int splits, int* err_dev, void* stream) {
-  if (Lq < 1 || heads < 1 || groups < 1 || heads % groups || n_keys < 1 || splits < 0 ||
-      splits > 16)
+                                 int n_keys, void* out, int parts, int* err_dev, void* stream) {
+  if (Lq < 1 || heads < 1 || groups < 1 || heads % groups || n_keys < 1 || parts < 0 ||
+      parts > kMaxAttnParts)
     return FD_ERR_INVALID_ARG;
-  if (splits == 0) splits = choose_splits(Lq, heads, groups, n_keys);
-  if (fd::attention_workspace_floats(splits, heads, Lq) * 4 > FD_STATIC_ATTN_SCRATCH_BYTES)
+  if (parts == 0) parts = choose_parts(Lq, heads, groups, n_keys);
+  if (fd::attention_workspace_floats(parts, fd::attention_units(Lq, heads, groups)) * 4 >
+      FD_STATIC_ATTN_SCRATCH_BYTES)
     return FD_ERR_INVALID_ARG;
   float* ws = nullptr;
-  if (splits > 1) {
+  if (parts > 1) {
     const fd_status st = static_scratch_address(&ws);
     if (st != FD_OK) return st;
   }
-  return fd_op_attention(Lq, heads, groups, q, k_ring, vt_ring, ring_pitch, n_keys, out, splits,
+  return fd_op_attention(Lq, heads, groups, q, k_ring, vt_ring, ring_pitch, n_keys, out, parts,
                          ws, err_dev, stream);
 }
 

@@ -282,24 +282,25 @@ def op_qkv(A, Wqkv, bqkv, knorm_g, vnorm_g, heads, groups, tokens, grid_w, frame
                            ring_pitch, bn, _ptr(err), _stream_ptr(stream)), "fd_op_qkv")
 
 
-def attention_workspace_bytes(Lq, heads, groups, n_keys, splits=0) -> int:
-    return lib().fd_attention_workspace_bytes(Lq, heads, groups, n_keys, splits)
+def attention_workspace_bytes(Lq, heads, groups, n_keys, parts=0) -> int:
+    return lib().fd_attention_workspace_bytes(Lq, heads, groups, n_keys, parts)
 
 
-def op_attention(q, k_ring, vt_ring, heads, groups, ring_pitch, n_keys, out, splits=0,
+def op_attention(q, k_ring, vt_ring, heads, groups, ring_pitch, n_keys, out, parts=0,
                  workspace=None, err=None, stream=None) -> None:
+    """fd_op_attention; parts = CTAs of the persistent launch (0: one per SM)."""
     Lq = q.shape[0]
     _check(lib().fd_op_attention(Lq, heads, groups, _ptr(q), _ptr(k_ring), _ptr(vt_ring),
-                                 ring_pitch, n_keys, _ptr(out), splits, _ptr(workspace),
+                                 ring_pitch, n_keys, _ptr(out), parts, _ptr(workspace),
                                  _ptr(err), _stream_ptr(stream)), "fd_op_attention")
 
 
-def op_attention_static(q, k_ring, vt_ring, heads, groups, ring_pitch, n_keys, out, splits=0,
+def op_attention_static(q, k_ring, vt_ring, heads, groups, ring_pitch, n_keys, out, parts=0,
                         err=None, stream=None) -> None:
-    """fd_op_attention with the split workspace in the library's static device memory."""
+    """fd_op_attention with its workspace in the library's static device memory."""
     Lq = q.shape[0]
     _check(lib().fd_op_attention_static(Lq, heads, groups, _ptr(q), _ptr(k_ring), _ptr(vt_ring),
-                                        ring_pitch, n_keys, _ptr(out), splits, _ptr(err),
+                                        ring_pitch, n_keys, _ptr(out), parts, _ptr(err),
                                         _stream_ptr(stream)), "fd_op_attention_static")
 
 

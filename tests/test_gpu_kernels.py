@@ -152,33 +152,42 @@ def attention_case(Lq, heads, groups, pitch, n_keys, seed, qscale=1.5):
     return q, k, v
 
 
-def run_attention(q, k, v, heads, groups, pitch, n_keys, splits=0):
+def run_attention(q, k, v, heads, groups, pitch, n_keys, parts=0, runs=1):
     Lq = q.shape[0]
-    out = torch.zeros(Lq, heads * 64, dtype=torch.bfloat16, device="cuda")
     vt = np.ascontiguousarray(np.transpose(v, (0, 2, 1)))
-    ws_bytes = fdp.attention_workspace_bytes(Lq, heads, groups, n_keys, splits)
+    ws_bytes = fdp.attention_workspace_bytes(Lq, heads, groups, n_keys, parts)
+    # the workspace starts as NaN garbage: the call must clear what it relies on
     ws = torch.full((max(1, ws_bytes // 4),), float("nan"), device="cuda")
     err = err_word()
-    fdp.op_attention(dev(q, torch.bfloat16), dev(k, torch.bfloat16), dev(vt, torch.float16),
-                     heads, groups, pitch, n_keys, out, splits=splits, workspace=ws, err=err)
+    outs = []
+    for _ in range(runs):
+        out = torch.zeros(Lq, heads * 64, dtype=torch.bfloat16, device="cuda")
+        fdp.op_attention(dev(q, torch.bfloat16), dev(k, torch.bfloat16), dev(vt, torch.float16),
+                         heads, groups, pitch, n_keys, out, parts=parts, workspace=ws, err=err)
+        outs.append(out)
     check_err(err)
-    return out.float().cpu()
+    return outs[0].float().cpu() if runs == 1 else [o.float().cpu() for o in outs]
 
 
-@pytest.mark.parametrize("Lq,heads,groups,n_keys,splits", [
-    (520, 4, 2, 520, 1),      # one chunk, ragged query tail
+# parts = CTAs of the persistent launch: each takes an equal run of the (tile pair, key block)
+# units, so runs start and end inside pairs and partial results are combined
+@pytest.mark.parametrize("Lq,heads,groups,n_keys,parts", [
+    (520, 4, 2, 520, 1),      # one CTA takes every pair: many segments, no partials
     (520, 4, 2, 1300, 1),     # ragged last key block
-    (520, 4, 2, 1300, 3),     # key range split in 3, partials combined
+    (520, 4, 2, 1300, 3),     # runs of ~37 blocks: partial first / last pairs, whole pairs between
+    (520, 4, 2, 1300, 25),    # runs of ~4 blocks: each pair cut into 3-4 partials
     (130, 4, 1, 390, 2),      # multi-query (G = 1)
-    (128, 4, 4, 128, 1),      # MHA (G = N): N/G odd, query tiles paired, second tile empty
-    (128, 4, 4, 128, 2),      # one key block split in 2: the second split is empty
+    (128, 4, 4, 128, 1),      # MHA (G = N): one tile per group, second tile of each pair empty
+    (128, 4, 4, 128, 7),      # more CTAs than units: some CTAs have nothing to do
+    (520, 4, 2, 1300, 200),   # 110 units on 200 CTAs: a pair's parts lie between empty CTAs
     (300, 3, 3, 700, 0),      # N/G = 1 with 3 query tiles: last pair half out of range
+    (300, 4, 2, 700, 5),      # Lq % 8 != 0: heads padded to 304 rows in the packed space
     (64, 2, 1, 1, 1),         # a single key
 ])
-def test_attention_small(Lq, heads, groups, n_keys, splits):
+def test_attention_small(Lq, heads, groups, n_keys, parts):
     pitch = max(128, -(-n_keys // 128) * 128 + 128)
     q, k, v = attention_case(Lq, heads, groups, pitch, n_keys, seed=Lq + n_keys)
-    got = run_attention(q, k, v, heads, groups, pitch, n_keys, splits)
+    got = run_attention(q, k, v, heads, groups, pitch, n_keys, parts)
     qh = f64(q).reshape(Lq, heads, 64).transpose(0, 1)
     want = oracle.attention(qh, f64(k)[:, :n_keys], f64(v)[:, :n_keys])
     assert_close_scaled(got.reshape(Lq, heads, 64).transpose(0, 1), want, 1.5e-2, "attention")
@@ -186,12 +195,16 @@ def test_attention_small(Lq, heads, groups, n_keys, splits):
 
 @pytest.mark.parametrize("Lq,heads,groups,n_keys", [
     (6240, 16, 4, 24960),   # 480p refinement, steady state (4 chunks x 4 frames x 1560)
+    (1560, 16, 4, 6240),    # 480p backbone, steady state
     (3600, 16, 4, 14400),   # 720p backbone, steady state
 ])
 def test_attention_full_size_sampled(Lq, heads, groups, n_keys):
+    """The launch configuration of the decode (one CTA per SM); two launches in a row on one
+    workspace give identical bits (the combine order is fixed and the counters are reset)."""
     pitch = -(-n_keys // 128) * 128
     q, k, v = attention_case(Lq, heads, groups, pitch, n_keys, seed=7, qscale=1.0)
-    got = run_attention(q, k, v, heads, groups, pitch, n_keys)
+    got, again = run_attention(q, k, v, heads, groups, pitch, n_keys, runs=2)
+    assert torch.equal(got, again)
     rows = np.random.default_rng(0).choice(Lq, 48, replace=False)
     rows = np.concatenate([rows, [0, Lq - 1]])
     qh = f64(q[rows]).reshape(len(rows), heads, 64).transpose(0, 1)

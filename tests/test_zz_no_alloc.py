@@ -16,7 +16,7 @@ pytestmark = pytest.mark.gpu
 
 fdp = pytest.importorskip("paper_2607_14898_gb300.flashdec")
 
-STATIC_BYTES = 16 << 20  # FD_STATIC_ATTN_SCRATCH_BYTES
+STATIC_BYTES = 32 << 20  # FD_STATIC_ATTN_SCRATCH_BYTES
 
 
 def case(Lq, heads, groups, n_keys, seed):
@@ -28,16 +28,16 @@ def case(Lq, heads, groups, n_keys, seed):
     return (dev(q, torch.bfloat16), dev(k, torch.bfloat16), dev(vt, torch.float16), pitch)
 
 
-def run_both(Lq, heads, groups, n_keys, splits, seed):
+def run_both(Lq, heads, groups, n_keys, parts, seed):
     q, k, vt, pitch = case(Lq, heads, groups, n_keys, seed)
     err = torch.zeros(2, dtype=torch.int32, device="cuda")
     ref = torch.zeros(Lq, heads * 64, dtype=torch.bfloat16, device="cuda")
-    ws_bytes = fdp.attention_workspace_bytes(Lq, heads, groups, n_keys, splits)
+    ws_bytes = fdp.attention_workspace_bytes(Lq, heads, groups, n_keys, parts)
     ws = torch.empty(max(1, ws_bytes // 4), dtype=torch.float32, device="cuda")
-    fdp.op_attention(q, k, vt, heads, groups, pitch, n_keys, ref, splits=splits, workspace=ws,
+    fdp.op_attention(q, k, vt, heads, groups, pitch, n_keys, ref, parts=parts, workspace=ws,
                      err=err[0:1])
     got = torch.zeros_like(ref)
-    fdp.op_attention_static(q, k, vt, heads, groups, pitch, n_keys, got, splits=splits,
+    fdp.op_attention_static(q, k, vt, heads, groups, pitch, n_keys, got, parts=parts,
                             err=err[1:2])
     torch.cuda.synchronize()
     assert err.cpu().tolist() == [0, 0]
@@ -47,10 +47,10 @@ def run_both(Lq, heads, groups, n_keys, splits, seed):
 def test_static_workspace_attention_matches_allocated_workspace():
     torch.cuda.set_device(0)
     # two calls in a row through the shared static array, different shapes and inputs; both
-    # use key-range splits, so the static workspace really carries the partial results
-    for Lq, heads, groups, n_keys, splits, seed in [(520, 4, 2, 1300, 3, 31),
-                                                    (1560, 16, 4, 6240, 2, 37)]:
-        got, ref, ws_bytes = run_both(Lq, heads, groups, n_keys, splits, seed)
+    # cut tile pairs across CTAs, so the static workspace really carries partial results
+    for Lq, heads, groups, n_keys, parts, seed in [(520, 4, 2, 1300, 3, 31),
+                                                   (1560, 16, 4, 6240, 0, 37)]:
+        got, ref, ws_bytes = run_both(Lq, heads, groups, n_keys, parts, seed)
         assert 0 < ws_bytes <= STATIC_BYTES
         assert_close_scaled(got, ref, 1.5e-2, f"static vs allocated workspace, Lq={Lq}")
 
@@ -58,6 +58,6 @@ def test_static_workspace_attention_matches_allocated_workspace():
 def test_static_workspace_rejects_oversize_requests():
     L = fdp.lib()
     Lq, heads, groups, n_keys = 6240, 16, 4, 24960
-    assert fdp.attention_workspace_bytes(Lq, heads, groups, n_keys, 4) > STATIC_BYTES
+    assert fdp.attention_workspace_bytes(Lq, heads, groups, n_keys, 300) > STATIC_BYTES
     # rejected before any launch: pointers are never touched
-    assert L.fd_op_attention_static(Lq, heads, groups, 0, 0, 0, 24960, n_keys, 0, 4, 0, 0) == 1
+    assert L.fd_op_attention_static(Lq, heads, groups, 0, 0, 0, 24960, n_keys, 0, 300, 0, 0) == 1
