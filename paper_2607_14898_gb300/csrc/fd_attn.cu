@@ -199,11 +199,34 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       prefetch_tmap(&tmQ8);
       prefetch_tmap(&tmK);
       prefetch_tmap(&tmV);
+      // Count this CTA's partial results once the softmax warps have stored them. The stores
+      // reach this thread through the barrier (CTA scope); the gpu-scope fence before the
+      // counter update publishes them all (fences are cumulative). The CTA that stores a
+      // pair's last part combines the pair. Slot 0 is polled between loads, so that a CTA
+      // that finished its first segment early does not end up combining that pair too.
+      const PartialSlots ps(wr, u0, len, nblk);
+      bool counted[2] = {!ps.has[0], !ps.has[1]};
+      decision[0] = decision[1] = 0;
+      auto count_slot = [&](int sl) {
+        counted[sl] = true;
+        const int pr = ps.pair[sl];
+        int owners = 0;  // CTAs holding a part of the pair
+        for (int c = wr.cta_of(pr * nblk); c <= wr.cta_of(pr * nblk + nblk - 1); ++c)
+          owners += wr.empty(c) ? 0 : 1;
+        __threadfence();
+        const int prev = atomicAdd(p.counters + pr, 1);
+        if (prev == owners - 1) {
+          p.counters[pr] = 0;  // every part has arrived: ready for the next launch
+          __threadfence();
+          decision[sl] = 1;
+        }
+      };
       Cursor cur;
       cur.begin(u0, len, nblk);
       int J = 0;
       bool ok = true;
       for (; J < len && ok; ++J) {
+        if (!counted[0] && mbar_test_wait(bar(kBarPartDone), 0)) count_slot(0);
         const int g = cur.pair / pairs_per_group;
         if (cur.first) {
           // Q of the segment's pair into buffer seg & 1, once the segment two back has done
@@ -259,26 +282,9 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         mbar_wait(bar(kBarQFull + (sg & 1)), (sg >> 1) & 1, p.err, ERR_WAIT_TMA);
       for (int i = J - 1; i >= 0 && i >= J - kStages; --i)
         mbar_wait(bar(kBarKvFull + i % kStages), (i / kStages) & 1, p.err, ERR_WAIT_TMA);
-      // Count this CTA's partial results, once the softmax warps have stored them. The
-      // stores reach this thread through the barrier (CTA scope); the gpu-scope fence before
-      // the counter update publishes them all (fences are cumulative). The CTA that stores a
-      // pair's last part combines the pair.
-      const PartialSlots ps(wr, u0, len, nblk);
-      for (int sl = 0; sl < 2; ++sl) {
-        decision[sl] = 0;
-        if (!ps.has[sl] || !mbar_wait(bar(kBarPartDone + sl), 0, p.err, ERR_WAIT_EPI)) continue;
-        const int pr = ps.pair[sl];
-        int owners = 0;  // CTAs holding a part of the pair
-        for (int c = wr.cta_of(pr * nblk); c <= wr.cta_of(pr * nblk + nblk - 1); ++c)
-          owners += wr.empty(c) ? 0 : 1;
-        __threadfence();
-        const int prev = atomicAdd(p.counters + pr, 1);
-        if (prev == owners - 1) {
-          p.counters[pr] = 0;  // every part has arrived: ready for the next launch
-          __threadfence();
-          decision[sl] = 1;
-        }
-      }
+      for (int sl = 0; sl < 2; ++sl)
+        if (!counted[sl] && mbar_wait(bar(kBarPartDone + sl), 0, p.err, ERR_WAIT_EPI))
+          count_slot(sl);
       mbar_arrive(bar(kBarDecided));
     }
   } else if (warp == 9 || warp == 10) {
