@@ -29,8 +29,9 @@ typedef enum {
 
 /* Linear layer on the tensor cores (tcgen05, bf16 in, fp32 accumulate).
  * A bf16 [M][K] row-major; W bf16 [N][K] row-major (nn.Linear); bias fp32 [N].
- * Requires N % 32 == 0, K % 8 == 0, 16-byte aligned A / W / out. bn = output tile width
- * (64, 128, 192 or 256; 0 = library choice). */
+ * Requires N % 32 == 0 (N % 64 == 0 for FD_EPI_GELU), K % 8 == 0, 16-byte aligned A / W /
+ * out. bn = output tile width (64, 96, 128, 192 or 256; 96 only for the fp32 epilogues;
+ * 0 = library choice). */
 fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const void* W,
                        const float* bias, void* out, int tup_hidden, int bn, int* err_dev,
                        void* stream);

@@ -386,6 +386,7 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CU
                         int bn, int num_sms, cudaStream_t s) {
   switch (bn) {
     case 64: return launch_bn<64>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+    case 96: return launch_bn<96>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
     case 128: return launch_bn<128>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
     case 192: return launch_bn<192>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
     case 256: return launch_bn<256>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);

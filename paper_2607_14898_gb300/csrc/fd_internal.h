@@ -158,7 +158,12 @@ constexpr int kMaxRopeSets = 2;
 
 // GEMM tile widths compiled in
 inline bool gemm_bn_supported(int bn) {
-  return bn == 64 || bn == 128 || bn == 192 || bn == 256;
+  return bn == 64 || bn == 96 || bn == 128 || bn == 192 || bn == 256;
+}
+// the QKV and GELU epilogues work on 64-column slabs (one head / one 128-byte bf16 row),
+// the fp32 epilogues on 32-column slabs
+inline bool gemm_bn_fits_epilogue(int bn, int epi) {
+  return (epi == EPI_QKV || epi == EPI_GELU) ? bn % 64 == 0 : bn % 32 == 0;
 }
 
 }  // namespace fd

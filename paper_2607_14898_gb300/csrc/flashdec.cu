@@ -219,11 +219,12 @@ float bf16_to_f32(uint16_t b) {
 // GEMM tile width for an M x N problem: a tile costs about (128 + BN) (a fixed part plus its
 // width) and a persistent grid runs ceil(tiles / SMs) rounds; pick the cheapest, the wider tile
 // on ties. Matches the measured best width on the decoder's shapes.
-int pick_bn(int M, int N) {
+int pick_bn(int M, int N, bool fp32_epilogue) {
   const int sms = num_sms();
   int best = 128;
   long long best_cost = -1;
-  for (int bn : {128, 192, 256}) {
+  for (int bn : {96, 128, 192, 256}) {
+    if (bn == 96 && !fp32_epilogue) continue;  // 64-column slabs need a multiple of 64
     const long long tiles = static_cast<long long>((M + 127) / 128) * ((N + bn - 1) / bn);
     const long long rounds = (tiles + sms - 1) / sms;
     const long long cost = rounds * (128 + bn);
@@ -662,34 +663,36 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
   uint8_t* base = static_cast<uint8_t*>(w->arena);
   size_t idx = 0;
   auto next = [&]() { return base + doff[idx++]; };
-  auto linear = [&](Linear& lin, int N, int K, int M) -> bool {
+  // fp32_epi: the layer's epilogue stores fp32 (patch-embed, out-projection, MLP down, temporal
+  // upsampling, head layer 2), which allows the narrower 96-wide tiles
+  auto linear = [&](Linear& lin, int N, int K, int M, bool fp32_epi) -> bool {
     lin.w = reinterpret_cast<__nv_bfloat16*>(next());
     lin.b = reinterpret_cast<float*>(next());
     lin.N = N;
     lin.K = K;
-    lin.bn = pick_bn(M, N);
+    lin.bn = pick_bn(M, N, fp32_epi);
     return tmap_bf16(&lin.tm, lin.w, K, N, static_cast<uint64_t>(K) * 2, fd::kBK, lin.bn);
   };
-  bool ok = linear(w->embed, d.D, d.cin, d.L);
+  bool ok = linear(w->embed, d.D, d.cin, d.L, true);
   auto block = [&](LayerW& lw, int M) {
     lw.g1 = reinterpret_cast<float*>(next());
-    ok = ok && linear(lw.qkv, d.qkv_out, d.D, M);
+    ok = ok && linear(lw.qkv, d.qkv_out, d.D, M, false);
     lw.kg = reinterpret_cast<float*>(next());
     lw.vg = reinterpret_cast<float*>(next());
-    ok = ok && linear(lw.out, d.D, d.N * kHeadDim, M);
+    ok = ok && linear(lw.out, d.D, d.N * kHeadDim, M, true);
     lw.g2 = reinterpret_cast<float*>(next());
-    ok = ok && linear(lw.mlp1, d.Mr * d.D, d.D, M);
-    ok = ok && linear(lw.mlp2, d.D, d.Mr * d.D, M);
+    ok = ok && linear(lw.mlp1, d.Mr * d.D, d.D, M, false);
+    ok = ok && linear(lw.mlp2, d.D, d.Mr * d.D, M, true);
   };
   w->blocks.resize(d.nb);
   for (auto& lw : w->blocks) block(lw, d.L);
   w->g_f = reinterpret_cast<float*>(next());
-  ok = ok && linear(w->tup, d.rt * d.D, d.D, d.L);
+  ok = ok && linear(w->tup, d.rt * d.D, d.D, d.L, true);
   w->refine.resize(d.nr);
   for (auto& lw : w->refine) block(lw, d.rt * d.L);
   w->g_h = reinterpret_cast<float*>(next());
-  ok = ok && linear(w->head1, d.D, d.D, d.rt * d.L);
-  ok = ok && linear(w->head2, d.head_out, d.D, d.rt * d.L);
+  ok = ok && linear(w->head1, d.D, d.D, d.rt * d.L, false);
+  ok = ok && linear(w->head2, d.head_out, d.D, d.rt * d.L, true);
   if (!ok || idx != layout.size()) {
     cudaFree(w->arena);
     delete w;
@@ -963,9 +966,11 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
     return FD_ERR_INVALID_ARG;
   if (N % 32 || K % 8 || !aligned16(A) || !aligned16(W) || !aligned16(out))
     return FD_ERR_INVALID_ARG;
-  if (bn == 0) bn = pick_bn(M, N);
-  if (!fd::gemm_bn_supported(bn)) return FD_ERR_INVALID_ARG;
   if (epilogue < FD_EPI_F32 || epilogue > FD_EPI_TUP) return FD_ERR_INVALID_ARG;
+  if (epilogue == FD_EPI_GELU && N % 64) return FD_ERR_INVALID_ARG;
+  if (bn == 0) bn = pick_bn(M, N, epilogue != FD_EPI_GELU);
+  if (!fd::gemm_bn_supported(bn) || !fd::gemm_bn_fits_epilogue(bn, epilogue))
+    return FD_ERR_INVALID_ARG;
   if (epilogue == FD_EPI_TUP && (tup_hidden < 32 || tup_hidden % 32 || N % tup_hidden))
     return FD_ERR_INVALID_ARG;
   fd_status st = check_device();
@@ -1009,7 +1014,8 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
   if (ring_pitch < window * M || ring_pitch % 128) return FD_ERR_INVALID_ARG;
   if (!aligned16(q_out) || !aligned16(k_ring) || !aligned16(vt_ring)) return FD_ERR_INVALID_ARG;
   if (bn == 0) bn = 128;
-  if (!fd::gemm_bn_supported(bn)) return FD_ERR_INVALID_ARG;
+  if (!fd::gemm_bn_supported(bn) || !fd::gemm_bn_fits_epilogue(bn, fd::EPI_QKV))
+    return FD_ERR_INVALID_ARG;
   fd_status st = check_device();
   if (st) return st;
   const int N = (heads + 2 * groups) * kHeadDim;

@@ -43,7 +43,9 @@ def linear_case(M, N, K, seed):
     (64, 192, 16, 64),        # K < 64 (tiny patch-embed), zero-filled K tail
     (520, 1024, 256, 256),    # 256-wide tiles
     (1560, 1536, 1024, 128),  # 480p QKV shape: 13 x 12 tiles, persistent (> 1 tile per CTA)
-    (1560, 1024, 4096, 0),    # 480p MLP-down shape, library tile choice
+    (1560, 1024, 4096, 0),    # 480p MLP-down shape, library tile choice (96-wide tiles)
+    (1560, 1024, 1024, 96),   # 480p out-projection shape: 13 x 11 tiles of 96, ragged N
+    (300, 608, 512, 96),      # ragged M and N with 96-wide tiles
     (6240, 768, 1024, 0),     # 480p head layer 2 on r_t L tokens
 ])
 def test_linear_f32(M, N, K, bn):
