@@ -28,6 +28,8 @@ Readings where the paper leaves a choice (each listed in the design notes):
   R6  Reshape after temporal upsampling: channel block tau (channels tau*D .. tau*D + D - 1)
       becomes refined frame tau; refined token tau*L + l.
   R7  MLP = Linear(D, 4D) -> GELU (erf form) -> Linear(4D, D); biases on every linear (R13).
+      Gated option (the XL layout): Linear(D, 4D) gate and Linear(D, 4D) up, SiLU(gate) * up,
+      then Linear(4D, D); the first weight stores the gate rows, then the up rows.
   R8  Head MLP: Linear(D, D) -> GELU -> Linear(D, C r_s^2).
   R9  Pixels clamped to [-1, 1]; uint8 = round-half-even(fl32(fl32(x + 1) * 127.5)).
   R12 RMSNorm with a learned gain before the temporal upsampling and before the head.
@@ -67,6 +69,11 @@ def rms_norm(x: torch.Tensor, g: torch.Tensor, eps: float) -> torch.Tensor:
 def gelu(x: torch.Tensor) -> torch.Tensor:
     """GELU, exact erf form: x * Phi(x) = 0.5 x (1 + erf(x / sqrt 2))."""
     return 0.5 * x * (1.0 + torch.erf(x / math.sqrt(2.0)))
+
+
+def silu(x: torch.Tensor) -> torch.Tensor:
+    """SiLU (swish): x * sigmoid(x) = x / (1 + exp(-x))."""
+    return x / (1.0 + torch.exp(-x))
 
 
 def linear(x: torch.Tensor, w: torch.Tensor, b: torch.Tensor | None) -> torch.Tensor:
@@ -190,8 +197,13 @@ def _block_rest(h, o, w, p, cfg):
     o = o.transpose(0, 1).reshape(L, -1)
     h = h + linear(o, w[p + "out.w"], w[p + "out.b"])
     u = rms_norm(h, w[p + "norm2.g"], cfg.norm_eps)
-    return h + linear(gelu(linear(u, w[p + "mlp1.w"], w[p + "mlp1.b"])),
-                      w[p + "mlp2.w"], w[p + "mlp2.b"])
+    z = linear(u, w[p + "mlp1.w"], w[p + "mlp1.b"])
+    if cfg.mlp_gated:
+        dm = z.shape[1] // 2
+        a = silu(z[:, :dm]) * z[:, dm:]
+    else:
+        a = gelu(z)
+    return h + linear(a, w[p + "mlp2.w"], w[p + "mlp2.b"])
 
 
 def _positions(cfg, frames: list[int], tokens_per_frame: int):

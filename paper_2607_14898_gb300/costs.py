@@ -22,7 +22,9 @@ def chunk_flops(cfg, t: int) -> dict[str, int]:
 
     def block(rows: int, keys: int) -> dict[str, int]:
         return {"qkv": 2 * rows * D * qkv_out, "attn": 4 * rows * keys * DH * N,
-                "out": 2 * rows * N * DH * D, "mlp1": 2 * rows * D * Dm, "mlp2": 2 * rows * Dm * D}
+                "out": 2 * rows * N * DH * D,
+                "mlp1": 2 * rows * D * Dm * (2 if cfg.mlp_gated else 1),  # gated: gate + up
+                "mlp2": 2 * rows * Dm * D}
 
     f = {"embed": 2 * L * cfg.c_in * D, "qkv": 0, "attn_backbone": 0, "attn_refine": 0,
          "out": 0, "mlp1": 0, "mlp2": 0, "tup": 2 * L * D * cfg.r_t * D,

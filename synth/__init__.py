@@ -39,6 +39,7 @@ class FDConfig:
     heads: int = 4                 # N
     kv_groups: int = 2             # G
     mlp_ratio: int = 4
+    mlp_gated: bool = False        # MLP: False = Linear, GELU, Linear; True = gated SiLU
     n_blocks: int = 2              # backbone blocks
     n_refine: int = 0              # temporal-refinement blocks
     window: int = 2                # W_frm, counts the current chunk
@@ -134,6 +135,21 @@ PRESETS: dict[str, FDConfig] = {
     "small_u8": FDConfig(latent_h=20, latent_w=26, patch=2, hidden=256, heads=4, kv_groups=1,
                          n_blocks=1, n_refine=1, window=2, r_t=4, out_u8=True,
                          name="small_u8", chunks=4),
+    # XL layout at tiny size: 48-channel 16x latent, patch 1, gated-SiLU MLP, refinement
+    "tiny_gated": FDConfig(latent_channels=48, latent_h=10, latent_w=13, vae_spatial=16,
+                           mlp_gated=True, n_refine=1, r_t=2, name="tiny_gated", chunks=3),
+    # FlashDecoder-XL as the paper's configuration table gives it: Wan2.2 latents (48
+    # channels, 16x spatial), patch 1, D=1536, 24 heads / 3 KV groups, 20 + 2 blocks, W=2,
+    # r_t=4, gated-SiLU MLP 4x; 480p (30x52 latent), 720p (45x80), 1080p (68x120)
+    "xl_480p": FDConfig(latent_channels=48, latent_h=30, latent_w=52, vae_spatial=16,
+                        hidden=1536, heads=24, kv_groups=3, mlp_gated=True, n_blocks=20,
+                        n_refine=2, window=2, r_t=4, name="xl_480p", chunks=16),
+    "xl_720p": FDConfig(latent_channels=48, latent_h=45, latent_w=80, vae_spatial=16,
+                        hidden=1536, heads=24, kv_groups=3, mlp_gated=True, n_blocks=20,
+                        n_refine=2, window=2, r_t=4, out_u8=True, name="xl_720p", chunks=16),
+    "xl_1080p": FDConfig(latent_channels=48, latent_h=68, latent_w=120, vae_spatial=16,
+                         hidden=1536, heads=24, kv_groups=3, mlp_gated=True, n_blocks=20,
+                         n_refine=2, window=2, r_t=4, out_u8=True, name="xl_1080p", chunks=8),
 }
 
 
@@ -145,6 +161,7 @@ def weight_layout(cfg: FDConfig) -> list[tuple[str, tuple[int, ...], str]]:
     """
     D, Dh, N, G = cfg.hidden, cfg.head_dim, cfg.heads, cfg.kv_groups
     Dm = cfg.mlp_ratio * D
+    D1 = 2 * Dm if cfg.mlp_gated else Dm  # gated: gate rows, then up rows
     out: list[tuple[str, tuple[int, ...], str]] = [
         ("embed.w", (D, cfg.c_in), "w"), ("embed.b", (D,), "b")]
 
@@ -158,8 +175,8 @@ def weight_layout(cfg: FDConfig) -> list[tuple[str, tuple[int, ...], str]]:
             (f"{prefix}.out.w", (D, N * Dh), "w"),
             (f"{prefix}.out.b", (D,), "b"),
             (f"{prefix}.norm2.g", (D,), "g"),
-            (f"{prefix}.mlp1.w", (Dm, D), "w"),
-            (f"{prefix}.mlp1.b", (Dm,), "b"),
+            (f"{prefix}.mlp1.w", (D1, D), "w"),
+            (f"{prefix}.mlp1.b", (D1,), "b"),
             (f"{prefix}.mlp2.w", (D, Dm), "w"),
             (f"{prefix}.mlp2.b", (D,), "b"),
         ])
