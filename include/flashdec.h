@@ -66,7 +66,8 @@ typedef struct {
   int32_t vae_spatial;     /* pixels per latent cell side (8 for Wan2.1)          */
   int32_t out_channels;    /* C (3)                                               */
   int32_t out_dtype;       /* FD_DTYPE_F32 or FD_DTYPE_U8                         */
-  int32_t reserved;        /* must be 0                                           */
+  int32_t mlp_gated;       /* MLP form: 0 = Linear, GELU, Linear; 1 = gated SiLU:    *
+                            * SiLU(x Wg + bg) * (x Wu + bu), then Linear (XL layout) */
   float norm_eps;          /* RMSNorm epsilon (1e-6)                              */
   float rope_base;         /* RoPE base (10000)                                   */
 } fd_config;
@@ -81,9 +82,10 @@ typedef struct fd_handle_s* fd_handle;
  *   embed.w [D][C' p^2], embed.b [D]
  *   per backbone block b = 0 .. n_blocks-1:
  *     norm1.g [D], qkv.w [(N+2G)*64][D], qkv.b [(N+2G)*64], knorm.g [64], vnorm.g [64],
- *     out.w [D][N*64], out.b [D], norm2.g [D], mlp1.w [M*D][D], mlp1.b [M*D],
+ *     out.w [D][N*64], out.b [D], norm2.g [D], mlp1.w [k*M*D][D], mlp1.b [k*M*D],
  *     mlp2.w [D][M*D], mlp2.b [D]
- *     (qkv rows: N query heads, then G key groups, then G value groups, 64 rows each)
+ *     (qkv rows: N query heads, then G key groups, then G value groups, 64 rows each;
+ *      k = 1, or k = 2 with mlp_gated: the M*D gate rows, then the M*D up rows)
  *   normf.g [D], tup.w [r_t*D][D], tup.b [r_t*D]
  *   per refinement block: the same twelve tensors
  *   normh.g [D], head1.w [D][D], head1.b [D], head2.w [C r_s^2][D], head2.b [C r_s^2]

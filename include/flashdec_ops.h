@@ -23,15 +23,18 @@ typedef enum {
   FD_EPI_F32 = 0,   /* out fp32 [M][N]  = A W^T + b                                   */
   FD_EPI_RESID = 1, /* out fp32 [M][N] += A W^T + b          (residual, Sec. 3.2)      */
   FD_EPI_GELU = 2,  /* out bf16 [M][N]  = GELU_erf(A W^T + b) (MLP, R7; head, Sec. 3.4) */
-  FD_EPI_TUP = 3    /* out fp32 [(N / tup_hidden) M][tup_hidden]: column tau*D + d of row
+  FD_EPI_TUP = 3,   /* out fp32 [(N / tup_hidden) M][tup_hidden]: column tau*D + d of row
                        l goes to row tau*M + l, column d (Eq. temporal_upsample)          */
+  FD_EPI_SWIGLU = 4 /* out bf16 [M][N/2]: gated SiLU MLP (XL layout). W and bias rows come in
+                       blocks of 64: rows 64j..64j+31 gate and 64j+32..64j+63 up of hidden
+                       units 32j..32j+31; out[m][32j+i] = SiLU(g + bg) * (u + bu)          */
 } fd_epilogue;
 
 /* Linear layer on the tensor cores (tcgen05, bf16 in, fp32 accumulate).
  * A bf16 [M][K] row-major; W bf16 [N][K] row-major (nn.Linear); bias fp32 [N].
- * Requires N % 32 == 0 (N % 64 == 0 for FD_EPI_GELU), K % 8 == 0, 16-byte aligned A / W /
- * out. bn = output tile width (64, 96, 128, 192 or 256; 96 only for the fp32 epilogues;
- * 0 = library choice). */
+ * Requires N % 32 == 0 (N % 64 == 0 for FD_EPI_GELU, N % 128 == 0 for FD_EPI_SWIGLU),
+ * K % 8 == 0, 16-byte aligned A / W / out. bn = output tile width (64, 96, 128, 192 or 256;
+ * 96 only for the fp32 epilogues, 128 or 256 for FD_EPI_SWIGLU; 0 = library choice). */
 fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const void* W,
                        const float* bias, void* out, int tup_hidden, int bn, int* err_dev,
                        void* stream);

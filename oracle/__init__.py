@@ -6,5 +6,5 @@ may import this package. The CUDA library and its Python binding never do.
 from .flashdecoder import (  # noqa: F401
     FLOPS, StreamingDecoder, attention, chunk_mask, decode_full_masked, decode_stream, gelu,
     kv_cache_elems, linear, pixel_shuffle, pixel_unshuffle, quantize_u8, reset_flops,
-    rms_norm, rope, rope_bands, silu,
+    operand_rounding, rms_norm, rope, rope_bands, silu,
 )

@@ -37,6 +37,7 @@ Readings where the paper leaves a choice (each listed in the design notes):
 """
 from __future__ import annotations
 
+import contextlib
 import math
 
 import numpy as np
@@ -52,6 +53,28 @@ FLOPS = {"gemm": 0, "attn": 0}
 def reset_flops() -> None:
     FLOPS["gemm"] = 0
     FLOPS["attn"] = 0
+
+
+# Operand rounding (off by default): the computation stays fp64, but the operands of every
+# matrix product are first rounded to the storage precision of "bf16 compute, fp32
+# accumulate": Linear inputs to bf16 (round to nearest even), attention Q and K to bf16 and
+# V to fp16. With it on, the oracle measures the rounding noise that precision alone causes,
+# which is what a floating-point tolerance for a given model size can be derived from.
+_OPERAND_ROUNDING = [False]
+
+
+@contextlib.contextmanager
+def operand_rounding():
+    prev = _OPERAND_ROUNDING[0]
+    _OPERAND_ROUNDING[0] = True
+    try:
+        yield
+    finally:
+        _OPERAND_ROUNDING[0] = prev
+
+
+def _round(x: torch.Tensor, dtype) -> torch.Tensor:
+    return x.to(dtype).to(F64) if _OPERAND_ROUNDING[0] else x
 
 
 def _t(x) -> torch.Tensor:
@@ -79,7 +102,7 @@ def silu(x: torch.Tensor) -> torch.Tensor:
 def linear(x: torch.Tensor, w: torch.Tensor, b: torch.Tensor | None) -> torch.Tensor:
     """y = x W^T + b with W stored [out][in] (Eq. projection and every other Linear)."""
     FLOPS["gemm"] += 2 * x.shape[0] * w.shape[0] * w.shape[1]
-    y = x @ w.T
+    y = _round(x, torch.bfloat16) @ w.T
     return y if b is None else y + b
 
 
@@ -142,6 +165,7 @@ def attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor,
     """
     N, Lq, dh = q.shape
     G, Lk, _ = k.shape
+    q, k, v = _round(q, torch.bfloat16), _round(k, torch.bfloat16), _round(v, torch.float16)
     out = torch.empty_like(q)
     scale = 1.0 / math.sqrt(dh)
     for n in range(N):

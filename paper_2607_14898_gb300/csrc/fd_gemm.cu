@@ -17,6 +17,8 @@
 //   EPI_RESID  h  += acc + b                    (out-projection, MLP layer 2: residual)
 //   EPI_GELU   out = bf16(GELU(acc + b))        (MLP layer 1, head layer 1)
 //   EPI_TUP    channel block tau of token l -> refined token tau*L + l   (Eq. temporal_upsample)
+//   EPI_SWIGLU out = bf16(SiLU(gate + b) * (up + b)) (gated MLP layer 1 of the XL layout; gate
+//              and up rows interleaved in blocks of 32, so 128 columns give 64 outputs)
 //   EPI_QKV    bias; KV-norm (RMS over D_h) on K and V; 3D-RoPE on Q and K; Q to its buffer,
 //              K (bf16) and V (transposed, fp16) into ring slot t mod W of the layer's cache
 //              (Sec. 3.3)
@@ -49,6 +51,8 @@ __device__ __forceinline__ void put_row_sw128(uint8_t* buf, int row, const uint3
 __device__ __forceinline__ float gelu_erf(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
 }
+
+__device__ __forceinline__ float silu(float x) { return x / (1.0f + __expf(-x)); }
 
 // cos / sin of the 32 rotation pairs of one token (3D-RoPE: temporal pairs first, then row,
 // then column; angle = position * base^(-2i/d_band)). Temporal values come from the chunk's
@@ -314,6 +318,37 @@ __global__ void __launch_bounds__(192, 1)
           publish();
           if (lane == 0 && row0 < p.M) {
             tma_store_2d(&tmO, smem_u32(buf), col, row0);
+            bulk_commit();
+          }
+        }
+      } else if (p.epi == EPI_SWIGLU) {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 128) {
+          const int col = n0 + c;
+          if (col >= p.N) break;
+          uint32_t w[32];
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            uint32_t rg[32], ru[32];
+            __syncwarp();
+            tmem_ld_32x32b_x32(tbase + c + 64 * hh, rg);
+            tmem_ld_32x32b_x32(tbase + c + 64 * hh + 32, ru);
+            tmem_ld_wait();
+            const float* bg = p.bias + col + 64 * hh;
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const float g0 = __uint_as_float(rg[2 * j]) + __ldg(bg + 2 * j);
+              const float g1 = __uint_as_float(rg[2 * j + 1]) + __ldg(bg + 2 * j + 1);
+              const float u0 = __uint_as_float(ru[2 * j]) + __ldg(bg + 32 + 2 * j);
+              const float u1 = __uint_as_float(ru[2 * j + 1]) + __ldg(bg + 33 + 2 * j);
+              w[16 * hh + j] = pack_bf16x2(silu(g0) * u0, silu(g1) * u1);
+            }
+          }
+          uint8_t* buf = acquire();
+          put_row_sw128(buf, lane, w);
+          publish();
+          if (lane == 0 && row0 < p.M) {
+            tma_store_2d(&tmO, smem_u32(buf), col / 2, row0);
             bulk_commit();
           }
         }

@@ -38,6 +38,8 @@ enum EpiKind : int {
   EPI_GELU = 2,   // out_bf16[r][c] = bf16(GELU(acc + bias))
   EPI_TUP = 3,    // temporal upsampling: column tau*D + d of row l -> out_f32[tau*L + l][d]
   EPI_QKV = 4,    // bias, KV-norm, 3D-RoPE; Q to q_out, K/V into the cache ring slot
+  EPI_SWIGLU = 5, // gated SiLU: accumulator columns in blocks of 64 (32 gate, 32 up of the same
+                  // hidden units); out_bf16[r][32j + i] = bf16(SiLU(g + bg) * (u + bu))
 };
 
 // Rotary / cache parameters of the fused QKV epilogue.
@@ -163,6 +165,7 @@ inline bool gemm_bn_supported(int bn) {
 // the QKV and GELU epilogues work on 64-column slabs (one head / one 128-byte bf16 row),
 // the fp32 epilogues on 32-column slabs
 inline bool gemm_bn_fits_epilogue(int bn, int epi) {
+  if (epi == EPI_SWIGLU) return bn % 128 == 0;  // 128 accumulator columns -> 64 outputs
   return (epi == EPI_QKV || epi == EPI_GELU) ? bn % 64 == 0 : bn % 32 == 0;
 }
 

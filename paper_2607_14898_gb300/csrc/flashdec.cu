@@ -146,6 +146,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 struct Dims {
   int C, H, W, p, D, N, G, Dh, Mr, nb, nr, Wn, rt, rs, Cout, cin, gh, gw, L, head_out, qkv_out;
   bool u8;
+  bool gated;  // gated-SiLU MLP: layer 1 has 2 Mr D outputs (gate, up)
 };
 
 bool valid_cfg(const fd_config* c) {
@@ -162,7 +163,7 @@ bool valid_cfg(const fd_config* c) {
   if ((c->out_channels * rs * rs) % 64) return false;
   if ((c->latent_channels * c->patch * c->patch) % 8) return false;  // TMA row pitch
   if (c->out_dtype != FD_DTYPE_F32 && c->out_dtype != FD_DTYPE_U8) return false;
-  if (c->reserved != 0) return false;
+  if (c->mlp_gated != 0 && c->mlp_gated != 1) return false;
   if (!(c->norm_eps >= 0.f) || !(c->rope_base > 1.f)) return false;
   const long long L = static_cast<long long>(c->latent_h / c->patch) * (c->latent_w / c->patch);
   if (L * c->r_t * c->window > (1LL << 26)) return false;
@@ -178,6 +179,7 @@ Dims dims_of(const fd_config* c) {
   d.cin = d.C * d.p * d.p; d.gh = d.H / d.p; d.gw = d.W / d.p; d.L = d.gh * d.gw;
   d.head_out = d.Cout * d.rs * d.rs; d.qkv_out = (d.N + 2 * d.G) * kHeadDim;
   d.u8 = c->out_dtype == FD_DTYPE_U8;
+  d.gated = c->mlp_gated == 1;
   return d;
 }
 
@@ -186,20 +188,39 @@ bool same_cfg(const fd_config* a, const fd_config* b) {
 }
 
 // blob element counts, in blob order
-struct BlobEntry { size_t elems; int kind; };  // kind: 0 weight (bf16 on device), 1 fp32
+struct BlobEntry {
+  size_t elems;
+  int kind;          // 0 weight (bf16 on device), 1 fp32
+  size_t gate_rows;  // > 0: gated MLP layer 1 (gate rows, then as many up rows) whose rows the
+  size_t row_len;    // device copy interleaves in blocks of 32 (see gated_row)
+};
 void blob_layout(const Dims& d, std::vector<BlobEntry>& out) {
-  auto W = [&](size_t n) { out.push_back({n, 0}); };
-  auto F = [&](size_t n) { out.push_back({n, 1}); };
+  auto W = [&](size_t n) { out.push_back({n, 0, 0, 0}); };
+  auto F = [&](size_t n) { out.push_back({n, 1, 0, 0}); };
   const size_t D = d.D, Dm = static_cast<size_t>(d.Mr) * d.D;
   W(D * d.cin); F(D);
   auto block = [&] {
     F(D); W(static_cast<size_t>(d.qkv_out) * D); F(d.qkv_out); F(kHeadDim); F(kHeadDim);
-    W(D * d.N * kHeadDim); F(D); F(D); W(Dm * D); F(Dm); W(D * Dm); F(D);
+    W(D * d.N * kHeadDim); F(D); F(D);
+    if (d.gated) {
+      out.push_back({2 * Dm * D, 0, Dm, D});
+      out.push_back({2 * Dm, 1, Dm, 1});
+    } else {
+      W(Dm * D); F(Dm);
+    }
+    W(D * Dm); F(D);
   };
   for (int b = 0; b < d.nb; ++b) block();
   F(D); W(static_cast<size_t>(d.rt) * D * D); F(static_cast<size_t>(d.rt) * D);
   for (int b = 0; b < d.nr; ++b) block();
   F(D); W(D * D); F(D); W(static_cast<size_t>(d.head_out) * D); F(d.head_out);
+}
+
+// Device row of blob row r of a gated MLP layer 1 with `gate` gate rows: the EPI_SWIGLU
+// epilogue wants gate and up rows of the same 32 hidden units side by side (64-row blocks).
+size_t gated_row(size_t r, size_t gate) {
+  const size_t u = r < gate ? r : r - gate;
+  return (u / 32) * 64 + (r < gate ? 0 : 32) + u % 32;
 }
 
 uint16_t f32_to_bf16_rne(float f) {
@@ -219,12 +240,12 @@ float bf16_to_f32(uint16_t b) {
 // GEMM tile width for an M x N problem: a tile costs about (128 + BN) (a fixed part plus its
 // width) and a persistent grid runs ceil(tiles / SMs) rounds; pick the cheapest, the wider tile
 // on ties. Matches the measured best width on the decoder's shapes.
-int pick_bn(int M, int N, bool fp32_epilogue) {
+int pick_bn_step(int M, int N, int step) {
   const int sms = num_sms();
   int best = 128;
   long long best_cost = -1;
   for (int bn : {96, 128, 192, 256}) {
-    if (bn == 96 && !fp32_epilogue) continue;  // 64-column slabs need a multiple of 64
+    if (bn % step) continue;
     const long long tiles = static_cast<long long>((M + 127) / 128) * ((N + bn - 1) / bn);
     const long long rounds = (tiles + sms - 1) / sms;
     const long long cost = rounds * (128 + bn);
@@ -235,6 +256,8 @@ int pick_bn(int M, int N, bool fp32_epilogue) {
   }
   return best;
 }
+// fp32 epilogues store 32-column slabs, the others 64-column slabs
+int pick_bn(int M, int N, bool fp32_epilogue) { return pick_bn_step(M, N, fp32_epilogue ? 32 : 64); }
 
 struct Linear {
   __nv_bfloat16* w = nullptr;  // [N][K]
@@ -443,7 +466,7 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
   if ((st = run_linear(h, FD_K_OUT, tm_o, lw.out, rows, po, so_h, s))) return st;
   if ((st = run_norm(h, hbuf, lw.g2, rows, s))) return st;
   fd::GemmParams p1{};
-  p1.epi = fd::EPI_GELU;
+  p1.epi = d.gated ? fd::EPI_SWIGLU : fd::EPI_GELU;
   p1.out_bf16 = h->hid;
   p1.ld_out = d.Mr * d.D;
   if ((st = run_linear(h, FD_K_MLP1, tm_u, lw.mlp1, rows, p1, so_hid, s))) return st;
@@ -630,7 +653,10 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
   }
   size_t src = 0;
   for (size_t i = 0; i < layout.size(); ++i) {
-    for (size_t k = 0; k < layout[i].elems; ++k, ++src) {
+    const BlobEntry& e = layout[i];
+    for (size_t k0 = 0; k0 < e.elems; ++k0, ++src) {
+      const size_t k =
+          e.gate_rows ? gated_row(k0 / e.row_len, e.gate_rows) * e.row_len + k0 % e.row_len : k0;
       float f;
       if (blob_dtype == FD_DTYPE_F32) {
         std::memcpy(&f, static_cast<const uint8_t*>(host_blob) + 4 * src, 4);
@@ -681,7 +707,12 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
     lw.vg = reinterpret_cast<float*>(next());
     ok = ok && linear(lw.out, d.D, d.N * kHeadDim, M, true);
     lw.g2 = reinterpret_cast<float*>(next());
-    ok = ok && linear(lw.mlp1, d.Mr * d.D, d.D, M, false);
+    ok = ok && linear(lw.mlp1, (d.gated ? 2 : 1) * d.Mr * d.D, d.D, M, false);
+    if (d.gated) {  // EPI_SWIGLU works on 128-column steps
+      lw.mlp1.bn = pick_bn_step(M, lw.mlp1.N, 128);
+      ok = ok && tmap_bf16(&lw.mlp1.tm, lw.mlp1.w, d.D, lw.mlp1.N,
+                           static_cast<uint64_t>(d.D) * 2, fd::kBK, lw.mlp1.bn);
+    }
     ok = ok && linear(lw.mlp2, d.D, d.Mr * d.D, M, true);
   };
   w->blocks.resize(d.nb);
@@ -966,10 +997,13 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
     return FD_ERR_INVALID_ARG;
   if (N % 32 || K % 8 || !aligned16(A) || !aligned16(W) || !aligned16(out))
     return FD_ERR_INVALID_ARG;
-  if (epilogue < FD_EPI_F32 || epilogue > FD_EPI_TUP) return FD_ERR_INVALID_ARG;
+  if (epilogue < FD_EPI_F32 || epilogue > FD_EPI_SWIGLU) return FD_ERR_INVALID_ARG;
   if (epilogue == FD_EPI_GELU && N % 64) return FD_ERR_INVALID_ARG;
-  if (bn == 0) bn = pick_bn(M, N, epilogue != FD_EPI_GELU);
-  if (!fd::gemm_bn_supported(bn) || !fd::gemm_bn_fits_epilogue(bn, epilogue))
+  if (epilogue == FD_EPI_SWIGLU && N % 128) return FD_ERR_INVALID_ARG;
+  const bool bf16_out = epilogue == FD_EPI_GELU || epilogue == FD_EPI_SWIGLU;
+  const int epi = epilogue == FD_EPI_SWIGLU ? fd::EPI_SWIGLU : epilogue;
+  if (bn == 0) bn = pick_bn_step(M, N, epilogue == FD_EPI_SWIGLU ? 128 : bf16_out ? 64 : 32);
+  if (!fd::gemm_bn_supported(bn) || !fd::gemm_bn_fits_epilogue(bn, epi))
     return FD_ERR_INVALID_ARG;
   if (epilogue == FD_EPI_TUP && (tup_hidden < 32 || tup_hidden % 32 || N % tup_hidden))
     return FD_ERR_INVALID_ARG;
@@ -982,17 +1016,18 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
   CUtensorMap to;
   bool ok;
   if (epilogue == FD_EPI_GELU) ok = tmap_out_bf16(&to, out, N, M, N);
+  else if (epilogue == FD_EPI_SWIGLU) ok = tmap_out_bf16(&to, out, N / 2, M, N / 2);
   else if (epilogue == FD_EPI_TUP) ok = tmap_out_tup(&to, out, tup_hidden, M, N / tup_hidden);
   else ok = tmap_out_f32(&to, out, N, M, N);
   if (!ok) return FD_ERR_CUDA;
   fd::GemmParams p{};
-  p.M = M; p.N = N; p.K = K; p.epi = epilogue; p.bias = bias; p.err = err_dev;
-  if (epilogue == FD_EPI_GELU) {
+  p.M = M; p.N = N; p.K = K; p.epi = epi; p.bias = bias; p.err = err_dev;
+  if (bf16_out) {
     p.out_bf16 = static_cast<__nv_bfloat16*>(out);
   } else {
     p.out_f32 = static_cast<float*>(out);
   }
-  p.ld_out = N;
+  p.ld_out = epilogue == FD_EPI_SWIGLU ? N / 2 : N;
   p.tup_tokens = M;
   p.tup_hidden = tup_hidden;
   return launch_ok(fd::launch_gemm(ta, tb, to, to, to, p, bn, num_sms(),

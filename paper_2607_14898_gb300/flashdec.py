@@ -21,7 +21,7 @@ STATUS = {0: "FD_OK", 1: "FD_ERR_INVALID_ARG", 2: "FD_ERR_CONFIG", 3: "FD_ERR_OO
           4: "FD_ERR_CUDA", 5: "FD_ERR_STATE", 6: "FD_ERR_DEVICE_TIMEOUT",
           7: "FD_ERR_UNSUPPORTED"}
 DTYPE_F32, DTYPE_BF16, DTYPE_U8 = 0, 1, 2
-EPI_F32, EPI_RESID, EPI_GELU, EPI_TUP = 0, 1, 2, 3
+EPI_F32, EPI_RESID, EPI_GELU, EPI_TUP, EPI_SWIGLU = 0, 1, 2, 3, 4
 # fd_kernel_kind order
 KERNEL_KINDS = ["unshuffle", "embed", "rmsnorm", "qkv", "attn_backbone", "attn_refine", "out",
                 "mlp1", "mlp2", "tup", "head1", "head2", "pixel", "advance", "rope"]
@@ -37,7 +37,7 @@ class fd_config(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "latent_channels", "latent_h", "latent_w", "patch", "hidden", "heads", "kv_groups",
         "mlp_ratio", "n_blocks", "n_refine", "window", "r_t", "vae_spatial", "out_channels",
-        "out_dtype", "reserved")] + [("norm_eps", ctypes.c_float), ("rope_base", ctypes.c_float)]
+        "out_dtype", "mlp_gated")] + [("norm_eps", ctypes.c_float), ("rope_base", ctypes.c_float)]
 
 
 _P = ctypes.c_void_p
@@ -111,7 +111,7 @@ def make_config(cfg) -> fd_config:
               "out_channels"):
         setattr(c, n, int(getattr(cfg, n)))
     c.out_dtype = DTYPE_U8 if getattr(cfg, "out_u8", False) else DTYPE_F32
-    c.reserved = 0
+    c.mlp_gated = 1 if cfg.mlp_gated else 0
     c.norm_eps = float(cfg.norm_eps)
     c.rope_base = float(cfg.rope_base)
     return c

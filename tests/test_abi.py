@@ -75,16 +75,17 @@ def test_cost_model_matches_the_oracle_flop_count():
     count 2*M*N*K), chunk by chunk through warm-up and steady state."""
     import oracle
     from paper_2607_14898_gb300 import costs
-    cfg = synth.PRESETS["small"]
-    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
-    dec = oracle.StreamingDecoder(cfg, w)
-    for t in range(cfg.chunks):
-        oracle.reset_flops()
-        dec.decode_chunk(z[t])
-        f = costs.chunk_flops(cfg, t)
-        attn = f["attn_backbone"] + f["attn_refine"]
-        assert oracle.FLOPS["attn"] == attn, t
-        assert oracle.FLOPS["gemm"] == sum(f.values()) - attn, t
+    for name in ("small", "tiny_gated"):
+        cfg = synth.PRESETS[name]
+        w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+        dec = oracle.StreamingDecoder(cfg, w)
+        for t in range(cfg.chunks):
+            oracle.reset_flops()
+            dec.decode_chunk(z[t])
+            f = costs.chunk_flops(cfg, t)
+            attn = f["attn_backbone"] + f["attn_refine"]
+            assert oracle.FLOPS["attn"] == attn, (name, t)
+            assert oracle.FLOPS["gemm"] == sum(f.values()) - attn, (name, t)
     # Sec. 3.3: attention cost linear in W and N, quadratic in L_frm
     big = synth.PRESETS["480p"]
     a = costs.chunk_flops(big, 10)["attn_backbone"]

@@ -14,6 +14,11 @@ fdp = pytest.importorskip("paper_2607_14898_gb300.flashdec")
 
 # Tolerance on pixels in [-1, 1]: bf16 compute with fp32 accumulation against the fp64 oracle.
 MAX_ABS, MEAN_ABS = 2e-2, 2e-3
+# The XL layout (D = 1536, gated MLP) is outside the configurations that bar was set for: with
+# its operands rounded to bf16 / fp16 (oracle.operand_rounding) the fp64 oracle itself moves by
+# max-abs 1.6e-2, mean-abs 2.4e-3 on 480p chunk 0 (the L model at 480p: 5.6e-3 / 8.4e-4), so no
+# bf16-operand computation of it meets 2e-3. Its bar is derived from that noise.
+XL_MAX_ABS, XL_MEAN_ABS = 2e-2, 3e-3
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -44,21 +49,22 @@ def gpu_stream(cfg, w, z, chunks=None, reset_and_repeat=False):
     return runs if reset_and_repeat else runs[0]
 
 
-def compare(cfg, got, want, what):
+def compare(cfg, got, want, what, max_abs=MAX_ABS, mean_abs=MEAN_ABS):
     for t, (g, o) in enumerate(zip(got, want)):
         if cfg.out_u8:
             wc = oracle.quantize_u8(o.float().numpy()).astype(np.int32)
             gc = g.numpy().astype(np.int32)
             d = np.abs(gc - wc)
             assert d.max() <= 3, f"{what} chunk {t}: max code diff {d.max()}"
-            assert d.mean() / 127.5 <= MEAN_ABS, f"{what} chunk {t}: mean {d.mean() / 127.5:.2e}"
+            assert d.mean() / 127.5 <= mean_abs, f"{what} chunk {t}: mean {d.mean() / 127.5:.2e}"
         else:
             mx, mean = pixel_errors(g, o)
-            assert mx <= MAX_ABS and mean <= MEAN_ABS, \
+            print(f"{what} chunk {t}: max-abs {mx:.3e} mean-abs {mean:.3e}")
+            assert mx <= max_abs and mean <= mean_abs, \
                 f"{what} chunk {t}: max-abs {mx:.3e} mean-abs {mean:.3e}"
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8", "tiny_gated"])
 def test_decode_matches_oracle(name):
     cfg = synth.PRESETS[name]
     w, z = synth.make_weights(cfg), synth.make_latents(cfg)
@@ -155,3 +161,21 @@ def test_decode_full_size(name, chunks):
     want = [ref.decode_chunk(z[t]) for t in range(chunks)]
     got = gpu_stream(cfg, w, z, chunks=chunks)
     compare(cfg, got, want, name)
+
+
+@pytest.mark.slow
+def test_decode_xl_layout():
+    """The paper's XL layout at 480p (48-channel latents, patch 1, D = 1536, gated MLP, W = 2:
+    chunk 2 evicts chunk 0) against the fp64 oracle. The bar is the one that the oracle itself
+    needs once its matrix operands are rounded to bf16 / fp16, which is checked first."""
+    cfg, chunks = synth.PRESETS["xl_480p"], 3
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg, chunks=chunks)
+    ref = oracle.StreamingDecoder(cfg, w)
+    want = [ref.decode_chunk(z[t]) for t in range(chunks)]
+    with oracle.operand_rounding():
+        ref_r = oracle.StreamingDecoder(cfg, w)
+        want_r = [ref_r.decode_chunk(z[t]) for t in range(chunks)]
+    compare(cfg, want_r, want, "xl_480p operand-rounded oracle vs fp64", XL_MAX_ABS, XL_MEAN_ABS)
+    assert max(float((a - b).abs().mean()) for a, b in zip(want_r, want)) > MEAN_ABS
+    got = gpu_stream(cfg, w, z, chunks=chunks)
+    compare(cfg, got, want, "xl_480p vs fp64", XL_MAX_ABS, XL_MEAN_ABS)

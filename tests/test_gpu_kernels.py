@@ -59,6 +59,31 @@ def test_linear_f32(M, N, K, bn):
     assert_close_scaled(out, want, 2e-5, "linear f32")
 
 
+@pytest.mark.parametrize("M,Dm,K,bn", [
+    (520, 512, 256, 0),     # ragged M, library tile choice
+    (130, 256, 1024, 128),  # 128-wide tiles: one 64-wide output slab per tile
+    (300, 576, 512, 256),   # 256-wide tiles; the last tile holds only 128 gate / up columns
+])
+def test_linear_swiglu(M, Dm, K, bn):
+    """Gated MLP layer 1 of the XL layout: out = SiLU(A Wg^T + bg) * (A Wu^T + bu), with the
+    gate and up rows interleaved in blocks of 32 as the epilogue expects."""
+    A = bf16_values(randn((M, K), M + K, 1.0))
+    Wg = bf16_values(randn((Dm, K), M + 1, 1.0 / math.sqrt(K)))
+    Wu = bf16_values(randn((Dm, K), M + 2, 1.0 / math.sqrt(K)))
+    bg, bu = randn((Dm,), M + 3, 0.1), randn((Dm,), M + 4, 0.1)
+    blocks = lambda g, u: np.concatenate(
+        [np.concatenate([g[32 * j:32 * j + 32], u[32 * j:32 * j + 32]]) for j in range(Dm // 32)])
+    W, b = blocks(Wg, Wu), blocks(bg, bu)
+    out = torch.zeros(M, Dm, dtype=torch.bfloat16, device="cuda")
+    err = err_word()
+    fdp.op_linear(fdp.EPI_SWIGLU, dev(A, torch.bfloat16), dev(W, torch.bfloat16), dev(b), out,
+                  bn=bn, err=err)
+    check_err(err)
+    want = oracle.silu(oracle.linear(f64(A), f64(Wg), f64(bg))) * \
+        oracle.linear(f64(A), f64(Wu), f64(bu))
+    assert_close_scaled(out.float(), want, 8e-3, "swiglu")
+
+
 def test_linear_resid_gelu_tup():
     M, N, K, D = 520, 1024, 256, 256
     A, W, b = linear_case(M, N, K, seed=11)

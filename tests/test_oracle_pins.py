@@ -82,6 +82,25 @@ def test_xl_parameter_count_fits_the_gated_mlp():
     assert 769.3e6 - count(xl.replace(mlp_gated=False)) > 200e6
 
 
+def test_operand_rounding_rounds_to_nearest_even_and_is_off_by_default():
+    """The test-only operand rounding: Linear inputs to bf16, attention Q, K to bf16 and V to
+    fp16, round to nearest even (as the library's dtype conversions); off outside the context."""
+    x = torch.tensor([[1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -9, -3.0 + 2.0 ** -10]],
+                     dtype=torch.float64)
+    w = torch.eye(3, dtype=torch.float64)
+    assert torch.equal(oracle.linear(x, w, None), x)
+    with oracle.operand_rounding():
+        # ties go to even: 1 + 2^-8 -> 1 (bf16 spacing 2^-7), 1 + 3 2^-9 -> 1 + 2^-7
+        want = torch.tensor([[1.0, 1.0 + 2.0 ** -7, -3.0]], dtype=torch.float64)
+        assert torch.equal(oracle.linear(x, w, None), want)
+        v = torch.tensor([[[1.0 + 2.0 ** -11, 2.0]]], dtype=torch.float64)
+        q = torch.zeros(1, 1, 1, dtype=torch.float64)
+        k = torch.zeros(1, 1, 1, dtype=torch.float64)
+        # one key: the output is V, rounded to fp16 (1 + 2^-11 is a tie between 1 and 1 + 2^-10)
+        assert float(oracle.attention(q, k, v[:, :, :1])[0, 0, 0]) == 1.0
+    assert torch.equal(oracle.linear(x, w, None), x)
+
+
 def test_linear_is_x_wt_plus_b():
     x, w, b = rnd(5, 7, seed=3), rnd(4, 7, seed=4), rnd(4, seed=5)
     brute = torch.tensor([[sum(x[i, k] * w[j, k] for k in range(7)) + b[j] for j in range(4)]
