@@ -164,26 +164,40 @@ def run_ours(args, rank: int, world: int):
 
     cfg = synth.PRESETS[args.workload]
     chunks = cfg.chunks
-    frames_per_step = chunks * cfg.r_t
+    S = cfg.streams  # independent streams on this GPU (480p x 8: 8)
+    frames_per_step = S * chunks * cfg.r_t
     w = synth.make_weights(cfg)
     blob = fdp.pack_blob(cfg, w)
     weights = fdp.Weights(cfg, blob)
-    dec = fdp.Decoder(cfg, weights)
-    # replicas: rank r decodes its own stream (latent seed r)
-    z = torch.from_numpy(synth.make_latents(cfg, seed=cfg.latent_seed + rank)).cuda()
+    decs = [fdp.Decoder(cfg, weights) for _ in range(S)]
+    dec = decs[0]
+    # replicas: rank r decodes its own streams (latent seeds r*S .. r*S + S - 1)
+    zs = [torch.from_numpy(synth.make_latents(cfg, seed=cfg.latent_seed + rank * S + i)).cuda()
+          for i in range(S)]
+    z = zs[0]
     out_dtype = torch.uint8 if cfg.out_u8 else torch.float32
-    pix = [torch.empty(cfg.out_channels, cfg.r_t, cfg.out_h, cfg.out_w, dtype=out_dtype,
-                       device="cuda") for _ in range(chunks)]
+    pixs = [[torch.empty(cfg.out_channels, cfg.r_t, cfg.out_h, cfg.out_w, dtype=out_dtype,
+                         device="cuda") for _ in range(chunks)] for _ in range(S)]
+    pix = pixs[0]
     stream = torch.cuda.Stream()
 
     def step(events=None):
-        dec.reset()
+        for d in decs:
+            d.reset()
         for t in range(chunks):
             if events is not None:
                 events[t][0].record(stream)
-            dec.decode_chunk(z[t], pix[t], stream)
+            if S == 1:
+                dec.decode_chunk(z[t], pix[t], stream)
+            else:  # chunk t of every stream, concurrently (fd_decode_chunks)
+                fdp.decode_chunks(decs, [zz[t] for zz in zs], [pp[t] for pp in pixs], stream)
             if events is not None:
                 events[t][1].record(stream)
+
+    def step_single():  # stream 0 alone, for the per-kernel profile
+        dec.reset()
+        for t in range(chunks):
+            dec.decode_chunk(z[t], pix[t], stream)
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -197,7 +211,7 @@ def run_ours(args, rank: int, world: int):
           for _ in range(args.steps)]
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
-    launches0 = dec.launch_count
+    launches0 = sum(d.launch_count for d in decs)
     barrier()
     torch.cuda.synchronize()
     try:
@@ -212,22 +226,22 @@ def run_ours(args, rank: int, world: int):
             t1.record(stream)
         torch.cuda.synchronize()
     barrier()
-    gpu_launches = dec.launch_count - launches0
+    gpu_launches = sum(d.launch_count for d in decs) - launches0
     ms_total = t0.elapsed_time(t1)
     ms_max = max_over_ranks(ms_total)
     frames_all = sum_over_ranks(frames_per_step * args.steps)
     lat = [ev[k][t][0].elapsed_time(ev[k][t][1]) for k in range(args.steps) for t in range(chunks)]
     lat_steady = [ev[k][t][0].elapsed_time(ev[k][t][1]) for k in range(args.steps)
                   for t in range(cfg.window - 1, chunks)]
-    if dec.sync_status() != fdp.FD_OK:
+    if any(d.sync_status() != fdp.FD_OK for d in decs):
         raise RuntimeError("device error in the timed region")
-    flops_step = costs.stream_flops(cfg, chunks)
+    flops_step = S * costs.stream_flops(cfg, chunks)
 
     # ---------------------------------------------------------------- per-kernel profile
     dec.profile(True)
     with torch.cuda.stream(stream):
         for _ in range(args.steps):
-            step()
+            step_single()
     torch.cuda.synchronize()
     prof = dec.profile_collect()
     dec.profile(False)
@@ -260,13 +274,17 @@ def run_ours(args, rank: int, world: int):
     prof_ms_step = sum(ms for _, ms in prof.values()) / args.steps
 
     # ---------------------------------------------------------------- end to end (host buffers)
-    lat_host = torch.from_numpy(synth.make_latents(cfg, seed=cfg.latent_seed + rank)).pin_memory()
-    pix_host = [torch.empty(pix[0].shape, dtype=out_dtype).pin_memory() for _ in range(chunks)]
+    lat_host = [torch.from_numpy(synth.make_latents(cfg, seed=cfg.latent_seed + rank * S + i))
+                .pin_memory() for i in range(S)]
+    pix_host = [[torch.empty(pix[0].shape, dtype=out_dtype).pin_memory() for _ in range(chunks)]
+                for _ in range(S)]
 
-    def step_host():
-        dec.reset()
+    def step_host():  # streams one after another through the host-buffer call
+        for d in decs:
+            d.reset()
         for t in range(chunks):
-            dec.decode_chunk_host(lat_host[t], pix_host[t], stream)
+            for i, d in enumerate(decs):
+                d.decode_chunk_host(lat_host[i][t], pix_host[i][t], stream)
 
     with torch.cuda.stream(stream):
         step_host()
@@ -301,10 +319,12 @@ def run_ours(args, rank: int, world: int):
         "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) latents, random-init N(0,0.02) bf16 weights)",
         "config": {
-            "workload": f"{cfg.name} single stream per GPU: latent 16x{cfg.latent_h}x"
-                        f"{cfg.latent_w}, patch 2 ({cfg.tokens} tokens/chunk), {chunks} chunks "
-                        f"per step, {cfg.n_blocks}+{cfg.n_refine} blocks, D={cfg.hidden}, "
-                        f"{cfg.heads} heads / {cfg.kv_groups} KV groups, W={cfg.window}, r_t="
+            "workload": f"{cfg.name} {S} stream{'s' if S > 1 else ''} per GPU: latent "
+                        f"{cfg.latent_channels}x{cfg.latent_h}x{cfg.latent_w}, patch {cfg.patch} "
+                        f"({cfg.tokens} tokens/chunk), {chunks} chunks per step, "
+                        f"{cfg.n_blocks}+{cfg.n_refine} blocks, D={cfg.hidden}, "
+                        f"{cfg.heads} heads / {cfg.kv_groups} KV groups, "
+                        f"{'gated-SiLU' if cfg.mlp_gated else 'GELU'} MLP, W={cfg.window}, r_t="
                         f"{cfg.r_t}, output {cfg.out_h}x{cfg.out_w} "
                         f"{'uint8' if cfg.out_u8 else 'fp32'}",
             "frames_per_step": frames_per_step,
@@ -314,15 +334,15 @@ def run_ours(args, rank: int, world: int):
         "latency_ms": {"p50": round(statistics.median(lat), 3),
                        "p99": round(sorted(lat)[max(0, int(0.99 * len(lat)) - 1)], 3),
                        "steady_p50": round(statistics.median(lat_steady), 3),
-                       "steady_frames_per_s": round(cfg.r_t / (statistics.median(lat_steady)
+                       "steady_frames_per_s": round(S * cfg.r_t / (statistics.median(lat_steady)
                                                                * 1e-3), 2)},
         "tensor_tflops_step": round(flops_step * args.steps / (ms_total * 1e-3) / 1e12, 1),
         "tensor_frac_step": round(flops_step * args.steps / (ms_total * 1e-3) / 1e12
                                   / sustained, 3),
         "clocks": clocks.summary(),
         "e2e": {"value": round(frames_all / (e2e_ms * 1e-3), 2), "unit": "frames/s",
-                "h2d_bytes_per_step": chunks * latent_bytes,
-                "d2h_bytes_per_step": chunks * pixel_bytes,
+                "h2d_bytes_per_step": S * chunks * latent_bytes,
+                "d2h_bytes_per_step": S * chunks * pixel_bytes,
                 "call": "fd_decode_chunk_host (pinned host latents / pixels)"},
         "gpu_launches": int(gpu_launches),
         "roofline": {"kernel": "attention (attn_kernel, backbone + refinement launches)",
@@ -347,7 +367,8 @@ def run_ours(args, rank: int, world: int):
         line["secondary"] = secondary_720p(args, stream, blob)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(cfg, w)
-    dec.close()
+    for d in decs:
+        d.close()
     weights.close()
     if dist is not None:
         dist.destroy_process_group()

@@ -131,8 +131,11 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out);
  * synchronisation). Attention at chunk t covers the min(t+1, W) most recent chunks. */
 fd_status fd_decode_chunk(fd_handle h, const float* latent_dev, void* pixels_dev, void* stream);
 
-/* Decode one chunk for each of n handles (independent streams sharing one weights object),
- * in order, on one CUDA stream. */
+/* Decode one chunk for each of n distinct handles (independent streams, e.g. sharing one
+ * weights object). Ordered on `stream` as one operation: it starts after the work already on
+ * `stream`, and work enqueued on `stream` afterwards sees every chunk's pixels. Inside, each
+ * handle's chunk runs on a library-owned stream forked from and joined back to `stream`, so
+ * the chunks run concurrently. All arguments are checked before anything is enqueued. */
 fd_status fd_decode_chunks(fd_handle* hs, int n, const float* const* latents_dev,
                            void* const* pixels_dev, void* stream);
 

@@ -304,6 +304,10 @@ struct fd_handle_s {
   int64_t t_host = 0;
   bool error = false;
   cudaStream_t last_stream = nullptr;
+  // fd_decode_chunks: a library-owned stream on which this handle's chunk runs beside the
+  // other handles', forked from and joined back to the caller's stream (created on first use)
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   // activations (rows: L for the backbone, r_t L for refinement / head)
   __nv_bfloat16 *x0 = nullptr, *u = nullptr, *q = nullptr, *o = nullptr, *hid = nullptr;
   float *h = nullptr, *hf = nullptr, *F = nullptr;
@@ -861,10 +865,40 @@ fd_status fd_decode_chunks(fd_handle* hs, int n, const float* const* latents_dev
                            void* const* pixels_dev, void* stream) {
   if (hs == nullptr || n < 0 || (n > 0 && (latents_dev == nullptr || pixels_dev == nullptr)))
     return FD_ERR_INVALID_ARG;
-  for (int i = 0; i < n; ++i) {
-    fd_status st = fd_decode_chunk(hs[i], latents_dev[i], pixels_dev[i], stream);
-    if (st != FD_OK) return st;
+  for (int i = 0; i < n; ++i) {  // check everything before enqueueing anything
+    fd_handle h = hs[i];
+    if (h == nullptr || latents_dev[i] == nullptr || pixels_dev[i] == nullptr)
+      return FD_ERR_INVALID_ARG;
+    if (!aligned16(latents_dev[i]) || !aligned16(pixels_dev[i])) return FD_ERR_INVALID_ARG;
+    for (int j = 0; j < i; ++j)
+      if (hs[j] == h) return FD_ERR_INVALID_ARG;
+    if (h->error || h->t_host >= (1LL << 30)) return FD_ERR_STATE;
+    if (h->side == nullptr &&
+        (cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) != cudaSuccess ||
+         cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+         cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess))
+      return FD_ERR_CUDA;
   }
+  if (n == 1) return fd_decode_chunk(hs[0], latents_dev[0], pixels_dev[0], stream);
+  // fork: every handle's side stream starts after the work already on the caller's stream;
+  // join: the caller's stream continues once every chunk is done. The independent streams'
+  // kernels fill each other's launch gaps and idle SMs.
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (n > 0 && cudaEventRecord(hs[0]->ev_fork, s) != cudaSuccess) return FD_ERR_CUDA;
+  for (int i = 0; i < n; ++i) {
+    fd_handle h = hs[i];
+    if (cudaStreamWaitEvent(h->side, hs[0]->ev_fork, 0) != cudaSuccess) return FD_ERR_CUDA;
+    fd_status st = decode_one(h, latents_dev[i], pixels_dev[i], h->side);
+    if (st == FD_OK && cudaEventRecord(h->ev_join, h->side) != cudaSuccess) st = FD_ERR_CUDA;
+    if (st != FD_OK) {
+      h->error = true;
+      return st;
+    }
+    h->t_host++;
+    h->last_stream = s;  // ordered on the caller's stream once joined
+  }
+  for (int i = 0; i < n; ++i)
+    if (cudaStreamWaitEvent(s, hs[i]->ev_join, 0) != cudaSuccess) return FD_ERR_CUDA;
   return FD_OK;
 }
 
@@ -904,6 +938,12 @@ fd_status fd_reset(fd_handle h) {
 fd_status fd_destroy(fd_handle h) {
   if (h == nullptr) return FD_ERR_INVALID_ARG;
   cudaStreamSynchronize(h->last_stream);
+  if (h->side != nullptr) {
+    cudaStreamSynchronize(h->side);
+    cudaStreamDestroy(h->side);
+  }
+  if (h->ev_fork != nullptr) cudaEventDestroy(h->ev_fork);
+  if (h->ev_join != nullptr) cudaEventDestroy(h->ev_join);
   for (size_t i = 0; i < h->ev_start.size(); ++i) {
     cudaEventDestroy(h->ev_start[i]);
     cudaEventDestroy(h->ev_stop[i]);

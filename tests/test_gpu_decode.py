@@ -81,6 +81,37 @@ def test_decode_deterministic_after_reset():
         assert torch.equal(x, y)
 
 
+def test_decode_chunks_concurrent_streams_match_single_stream_decodes():
+    """fd_decode_chunks runs independent streams (one weights object, three handles, seeds s)
+    concurrently on forked streams; each stream's pixels are bit-identical to decoding it alone
+    with fd_decode_chunk, chunk after chunk, and the caller's stream sees all of them."""
+    cfg = synth.PRESETS["small"]
+    w = synth.make_weights(cfg)
+    zs = [synth.make_latents(cfg, seed=s) for s in range(3)]
+    alone = [gpu_stream(cfg, w, z) for z in zs]
+    W = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    decs = [fdp.Decoder(cfg, W) for _ in zs]
+    stream = torch.cuda.Stream()
+    shape = (cfg.out_channels, cfg.r_t, cfg.out_h, cfg.out_w)
+    got = [[] for _ in zs]
+    with torch.cuda.stream(stream):
+        for t in range(cfg.chunks):
+            lat = [dev(z[t]) for z in zs]
+            pix = [torch.empty(shape, device="cuda") for _ in zs]
+            fdp.decode_chunks(decs, lat, pix, stream)
+            copies = [p.to("cpu", non_blocking=False) for p in pix]  # ordered on `stream`
+            for s, c in enumerate(copies):
+                got[s].append(c)
+    torch.cuda.synchronize()
+    for d in decs:
+        assert d.sync_status() == fdp.FD_OK
+        d.close()
+    W.close()
+    for s in range(len(zs)):
+        for t in range(cfg.chunks):
+            assert torch.equal(got[s][t], alone[s][t]), (s, t)
+
+
 def test_decode_causality_on_gpu():
     """Outputs of chunks < 3 are bit-identical when chunks >= 3 change."""
     cfg = synth.PRESETS["small"]
