@@ -70,6 +70,9 @@ typedef struct {
                             * SiLU(x Wg + bg) * (x Wu + bu), then Linear (XL layout) */
   float norm_eps;          /* RMSNorm epsilon (1e-6)                              */
   float rope_base;         /* RoPE base (10000)                                   */
+  int32_t qk_norm;         /* per-head RMSNorm on: 0 = K and V (KV-norm, Sec. 3.2); *
+                            * 1 = Q and K (QK-norm); the blob's second D_h gain is  *
+                            * then Q's                                              */
 } fd_config;
 
 typedef struct fd_weights_s* fd_weights;
@@ -81,7 +84,8 @@ typedef struct fd_handle_s* fd_handle;
  * linear weight stored [out][in] row-major (nn.Linear layout):
  *   embed.w [D][C' p^2], embed.b [D]
  *   per backbone block b = 0 .. n_blocks-1:
- *     norm1.g [D], qkv.w [(N+2G)*64][D], qkv.b [(N+2G)*64], knorm.g [64], vnorm.g [64],
+ *     norm1.g [D], qkv.w [(N+2G)*64][D], qkv.b [(N+2G)*64], knorm.g [64], vnorm.g [64]
+ *     (qnorm.g with qk_norm),
  *     out.w [D][N*64], out.b [D], norm2.g [D], mlp1.w [k*M*D][D], mlp1.b [k*M*D],
  *     mlp2.w [D][M*D], mlp2.b [D]
  *     (qkv rows: N query heads, then G key groups, then G value groups, 64 rows each;
@@ -182,6 +186,23 @@ fd_status fd_profile_collect(fd_handle h, int64_t* launches, double* ms);
 
 /* Number of kernels this handle has launched since fd_create. */
 int64_t fd_launch_count(fd_handle h);
+
+/* Streaming state, for checkpoint / resume and for moving a stream to another handle (no
+ * counterpart in the paper, whose decode keeps this state in the process): the chunk index t
+ * and every layer's rolling cache (backbone and refinement rings, K bf16 and V^T fp16, as the
+ * device holds them). It contains no weights.
+ *   fd_state_bytes: size of the state of a handle of configuration cfg (0 if cfg is invalid).
+ *   fd_save_state: copy the handle's state into host_buf (exactly fd_state_bytes bytes), ordered
+ *     on `stream` after the decodes already enqueued there (use the decode stream): the buffer
+ *     is complete once the stream reaches this point. Pinned memory makes the copy asynchronous.
+ *     FD_ERR_STATE if the handle is in error.
+ *   fd_load_state: restore a saved state into a handle created with an identical configuration
+ *     (checked against the header; FD_ERR_INVALID_ARG otherwise), ordered on `stream`; the next
+ *     fd_decode_chunk on that stream continues the saved stream exactly as the original handle
+ *     would have. Clears the handle's error state. */
+size_t fd_state_bytes(const fd_config* cfg);
+fd_status fd_save_state(fd_handle h, void* host_buf, size_t bytes, void* stream);
+fd_status fd_load_state(fd_handle h, const void* host_buf, size_t bytes, void* stream);
 
 /* Copy layer `layer` of the backbone (which = 0) or refinement (which = 1) ring into host
  * memory: K as [G][W * rows][64] bf16 bits, then V as [G][W * rows][64] fp16 bits (rows =

@@ -48,7 +48,8 @@ fd_status fd_op_rope_table(int t, int frames_per_chunk, float rope_base, float* 
 
 /* Fused QKV projection of one attention block (Sec. 3.2, Sec. 3.3 step (2)):
  *   [Q | K | V] = A Wqkv^T + b   (Wqkv rows: heads*64 query, groups*64 key, groups*64 value)
- *   K, V <- RMSNorm over the 64 head dims with gains knorm_g / vnorm_g (KV-norm)
+ *   K, V <- RMSNorm over the 64 head dims with gains knorm_g / norm2_g (KV-norm), or with
+ *           qk_norm = 1: Q, K <- RMSNorm with gains norm2_g / knorm_g (QK-norm), V as is
  *   Q, K <- 3D-RoPE at temporal index t*frames_per_chunk + row / tokens (cos / sin from
  *           rope_t, the fd_op_rope_table of chunk t), row and column of token (row % tokens)
  *           in a grid of width grid_w (rope_base; bands 24/20/20 dims)
@@ -56,7 +57,7 @@ fd_status fd_op_rope_table(int t, int frames_per_chunk, float rope_base, float* 
  *   (t mod window)*M + row;  V -> vt_ring fp16 [groups][64][ring_pitch] (transposed), same
  *   key index.  M = frames_per_chunk * tokens; ring_pitch % 128 == 0, >= window * M. */
 fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* bqkv,
-                    const float* knorm_g, const float* vnorm_g, int heads, int groups,
+                    const float* knorm_g, const float* norm2_g, int qk_norm, int heads, int groups,
                     int tokens, int grid_w, int frames_per_chunk, int window, int t, float eps,
                     float rope_base, const float* rope_t, void* q_out, void* k_ring,
                     void* vt_ring, int ring_pitch, int bn, int* err_dev, void* stream);

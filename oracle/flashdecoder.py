@@ -18,7 +18,8 @@ Everything here is written straight from the paper, in fp64 with PyTorch CPU ten
 
 Readings where the paper leaves a choice (each listed in the design notes):
   R3  KV-norm = RMSNorm over the head dimension of K and of V (learned gain of length D_h,
-      shared by all groups), applied before RoPE; Q is not normalised.
+      shared by all groups), applied before RoPE; Q is not normalised. Option qk_norm: the
+      usual QK-norm instead, on Q and K (gains qnorm.g, knorm.g), V not normalised.
   R4  3D-RoPE bands: D_h split [temporal | height | width] = [D_h - 2*2*floor(D_h/6) | 2*floor(D_h/6)
       | 2*floor(D_h/6)] dims (24/20/20 at D_h = 64); rotation of interleaved pairs
       (2i, 2i+1) by angle pos * base^(-2i/d_band).
@@ -208,7 +209,10 @@ def _block_qkv(h, w, p, cfg, pos):
     k = qkv[:, N * dh:(N + G) * dh].reshape(L, G, dh).transpose(0, 1)
     v = qkv[:, (N + G) * dh:].reshape(L, G, dh).transpose(0, 1)
     k = rms_norm(k, w[p + "knorm.g"], cfg.norm_eps)
-    v = rms_norm(v, w[p + "vnorm.g"], cfg.norm_eps)
+    if cfg.qk_norm:
+        q = rms_norm(q, w[p + "qnorm.g"], cfg.norm_eps)
+    else:
+        v = rms_norm(v, w[p + "vnorm.g"], cfg.norm_eps)
     if pos is not None:
         q = rope(q, *pos, cfg.rope_base)
         k = rope(k, *pos, cfg.rope_base)

@@ -19,7 +19,8 @@
 //   EPI_TUP    channel block tau of token l -> refined token tau*L + l   (Eq. temporal_upsample)
 //   EPI_SWIGLU out = bf16(SiLU(gate + b) * (up + b)) (gated MLP layer 1 of the XL layout; gate
 //              and up rows interleaved in blocks of 32, so 128 columns give 64 outputs)
-//   EPI_QKV    bias; KV-norm (RMS over D_h) on K and V; 3D-RoPE on Q and K; Q to its buffer,
+//   EPI_QKV    bias; KV-norm (RMS over D_h) on K and V (or QK-norm on Q and K); 3D-RoPE on Q
+//              and K; Q to its buffer,
 //              K (bf16) and V (transposed, fp16) into ring slot t mod W of the layer's cache
 //              (Sec. 3.3)
 #include "fd_internal.h"
@@ -243,7 +244,7 @@ __global__ void __launch_bounds__(192, 1)
           const int hidx = col / kHeadDim;
           const bool is_q = hidx < q.heads;
           const bool is_k = !is_q && hidx < q.heads + q.groups;
-          if (!is_q) {  // KV-norm: RMS over the head dimension, learned gain
+          if (q.qk_norm ? (is_q || is_k) : !is_q) {  // per-head RMSNorm, learned gain
             float ss = 0.f;
 #pragma unroll
             for (int j = 0; j < 64; ++j) ss = fmaf(v[j], v[j], ss);

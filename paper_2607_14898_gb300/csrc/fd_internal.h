@@ -44,6 +44,7 @@ enum EpiKind : int {
 
 // Rotary / cache parameters of the fused QKV epilogue.
 struct QkvEpi {
+  int qk_norm;  // 0: RMSNorm K (knorm_g) and V (vnorm_g); 1: Q (vnorm_g holds Q's gain) and K
   int heads, groups;
   const float* knorm_g;      // [64] KV-norm gain for K
   const float* vnorm_g;      // [64] KV-norm gain for V

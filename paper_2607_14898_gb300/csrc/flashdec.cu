@@ -147,6 +147,7 @@ struct Dims {
   int C, H, W, p, D, N, G, Dh, Mr, nb, nr, Wn, rt, rs, Cout, cin, gh, gw, L, head_out, qkv_out;
   bool u8;
   bool gated;  // gated-SiLU MLP: layer 1 has 2 Mr D outputs (gate, up)
+  bool qk;     // QK-norm instead of KV-norm
 };
 
 bool valid_cfg(const fd_config* c) {
@@ -164,6 +165,7 @@ bool valid_cfg(const fd_config* c) {
   if ((c->latent_channels * c->patch * c->patch) % 8) return false;  // TMA row pitch
   if (c->out_dtype != FD_DTYPE_F32 && c->out_dtype != FD_DTYPE_U8) return false;
   if (c->mlp_gated != 0 && c->mlp_gated != 1) return false;
+  if (c->qk_norm != 0 && c->qk_norm != 1) return false;
   if (!(c->norm_eps >= 0.f) || !(c->rope_base > 1.f)) return false;
   const long long L = static_cast<long long>(c->latent_h / c->patch) * (c->latent_w / c->patch);
   if (L * c->r_t * c->window > (1LL << 26)) return false;
@@ -180,6 +182,7 @@ Dims dims_of(const fd_config* c) {
   d.head_out = d.Cout * d.rs * d.rs; d.qkv_out = (d.N + 2 * d.G) * kHeadDim;
   d.u8 = c->out_dtype == FD_DTYPE_U8;
   d.gated = c->mlp_gated == 1;
+  d.qk = c->qk_norm == 1;
   return d;
 }
 
@@ -439,6 +442,7 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
   p.epi = fd::EPI_QKV;
   fd::QkvEpi& q = p.qkv;
   q.heads = d.N; q.groups = d.G; q.knorm_g = lw.kg; q.vnorm_g = lw.vg; q.q_out = h->q;
+  q.qk_norm = d.qk ? 1 : 0;
   q.k_ring = r.k; q.vt_ring = r.vt; q.ring_pitch = pitch; q.tokens = d.L; q.grid_w = d.gw;
   q.frames_per_chunk = fpc; q.window = d.Wn; q.step_dev = h->state; q.step_host = 0;
   q.eps = h->cfg.norm_eps;
@@ -980,6 +984,98 @@ int64_t fd_launch_count(fd_handle h) { return h ? h->launches : -1; }
 
 int64_t fd_chunk_index(fd_handle h) { return h ? h->t_host : -1; }
 
+}  // extern "C"
+
+namespace {
+// Header of a saved streaming state; the rings follow (per backbone layer, then per refinement
+// layer: K [G][pitch][64] bf16, then V^T [G][64][pitch] fp16).
+struct StateHeader {
+  char magic[8];
+  int64_t version;
+  int64_t t;
+  int64_t payload_bytes;
+  fd_config cfg;
+};
+constexpr char kStateMagic[8] = {'F', 'D', 'S', 'T', 'A', 'T', 'E', '\0'};
+constexpr int64_t kStateVersion = 1;
+
+size_t ring_bytes(const Dims& d, int pitch) {  // K or V^T of one layer
+  return static_cast<size_t>(d.G) * pitch * kHeadDim * 2;
+}
+size_t state_payload(const Dims& d) {
+  const int pitchB = static_cast<int>(align_up(static_cast<size_t>(d.Wn) * d.L, 128));
+  const int pitchR = static_cast<int>(align_up(static_cast<size_t>(d.Wn) * d.rt * d.L, 128));
+  return 2 * (d.nb * ring_bytes(d, pitchB) + d.nr * ring_bytes(d, pitchR));
+}
+}  // namespace
+
+extern "C" {
+
+size_t fd_state_bytes(const fd_config* cfg) {
+  if (!valid_cfg(cfg)) return 0;
+  return sizeof(StateHeader) + state_payload(dims_of(cfg));
+}
+
+fd_status fd_save_state(fd_handle h, void* host_buf, size_t bytes, void* stream) {
+  if (h == nullptr || host_buf == nullptr) return FD_ERR_INVALID_ARG;
+  if (bytes != fd_state_bytes(&h->cfg)) return FD_ERR_INVALID_ARG;
+  if (h->error) return FD_ERR_STATE;
+  StateHeader hd;
+  std::memset(&hd, 0, sizeof(hd));
+  std::memcpy(hd.magic, kStateMagic, 8);
+  hd.version = kStateVersion;
+  hd.t = h->t_host;
+  hd.payload_bytes = static_cast<int64_t>(state_payload(h->d));
+  hd.cfg = h->cfg;
+  std::memcpy(host_buf, &hd, sizeof(hd));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint8_t* dst = static_cast<uint8_t*>(host_buf) + sizeof(hd);
+  auto copy_out = [&](const std::vector<Ring>& rings, int pitch) -> bool {
+    const size_t n = ring_bytes(h->d, pitch);
+    for (const Ring& r : rings) {
+      if (cudaMemcpyAsync(dst, r.k, n, cudaMemcpyDeviceToHost, s) != cudaSuccess) return false;
+      dst += n;
+      if (cudaMemcpyAsync(dst, r.vt, n, cudaMemcpyDeviceToHost, s) != cudaSuccess) return false;
+      dst += n;
+    }
+    return true;
+  };
+  if (!copy_out(h->ringB, h->pitchB) || !copy_out(h->ringR, h->pitchR)) return FD_ERR_CUDA;
+  return FD_OK;
+}
+
+fd_status fd_load_state(fd_handle h, const void* host_buf, size_t bytes, void* stream) {
+  if (h == nullptr || host_buf == nullptr) return FD_ERR_INVALID_ARG;
+  if (bytes != fd_state_bytes(&h->cfg)) return FD_ERR_INVALID_ARG;
+  StateHeader hd;
+  std::memcpy(&hd, host_buf, sizeof(hd));
+  if (std::memcmp(hd.magic, kStateMagic, 8) != 0 || hd.version != kStateVersion ||
+      hd.payload_bytes != static_cast<int64_t>(state_payload(h->d)) ||
+      !same_cfg(&hd.cfg, &h->cfg) || hd.t < 0 || hd.t >= (1LL << 30))
+    return FD_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const uint8_t* src = static_cast<const uint8_t*>(host_buf) + sizeof(hd);
+  auto copy_in = [&](std::vector<Ring>& rings, int pitch) -> bool {
+    const size_t n = ring_bytes(h->d, pitch);
+    for (Ring& r : rings) {
+      if (cudaMemcpyAsync(r.k, src, n, cudaMemcpyHostToDevice, s) != cudaSuccess) return false;
+      src += n;
+      if (cudaMemcpyAsync(r.vt, src, n, cudaMemcpyHostToDevice, s) != cudaSuccess) return false;
+      src += n;
+    }
+    return true;
+  };
+  // device chunk index and a clear error word; pageable source: staged before the call returns
+  const int st[2] = {static_cast<int>(hd.t), 0};
+  if (!copy_in(h->ringB, h->pitchB) || !copy_in(h->ringR, h->pitchR) ||
+      cudaMemcpyAsync(h->state, st, sizeof(st), cudaMemcpyHostToDevice, s) != cudaSuccess)
+    return FD_ERR_CUDA;
+  h->t_host = hd.t;
+  h->error = false;
+  h->last_stream = s;
+  return FD_OK;
+}
+
 fd_status fd_sync_status(fd_handle h) {
   if (h == nullptr) return FD_ERR_INVALID_ARG;
   if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) {
@@ -1075,12 +1171,12 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
 }
 
 fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* bqkv,
-                    const float* knorm_g, const float* vnorm_g, int heads, int groups,
-                    int tokens, int grid_w, int frames_per_chunk, int window, int t, float eps,
-                    float rope_base, const float* rope_t, void* q_out, void* k_ring,
+                    const float* knorm_g, const float* norm2_g, int qk_norm, int heads,
+                    int groups, int tokens, int grid_w, int frames_per_chunk, int window, int t,
+                    float eps, float rope_base, const float* rope_t, void* q_out, void* k_ring,
                     void* vt_ring, int ring_pitch, int bn, int* err_dev, void* stream) {
-  if (!A || !Wqkv || !bqkv || !knorm_g || !vnorm_g || !q_out || !k_ring || !vt_ring ||
-      !err_dev || !rope_t)
+  if (!A || !Wqkv || !bqkv || !knorm_g || !norm2_g || !q_out || !k_ring || !vt_ring ||
+      !err_dev || !rope_t || (qk_norm != 0 && qk_norm != 1))
     return FD_ERR_INVALID_ARG;
   if (heads < 1 || groups < 1 || heads % groups || tokens < 1 || grid_w < 1 ||
       tokens % grid_w || frames_per_chunk < 1 || window < 1 || t < 0 || K < 8 || K % 8)
@@ -1101,7 +1197,8 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
   fd::GemmParams p{};
   p.M = M; p.N = N; p.K = K; p.epi = fd::EPI_QKV; p.bias = bqkv; p.err = err_dev;
   fd::QkvEpi& q = p.qkv;
-  q.heads = heads; q.groups = groups; q.knorm_g = knorm_g; q.vnorm_g = vnorm_g;
+  q.heads = heads; q.groups = groups; q.knorm_g = knorm_g; q.vnorm_g = norm2_g;
+  q.qk_norm = qk_norm;
   q.q_out = static_cast<__nv_bfloat16*>(q_out);
   q.k_ring = static_cast<__nv_bfloat16*>(k_ring);
   q.vt_ring = static_cast<__half*>(vt_ring);

@@ -37,7 +37,8 @@ class fd_config(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "latent_channels", "latent_h", "latent_w", "patch", "hidden", "heads", "kv_groups",
         "mlp_ratio", "n_blocks", "n_refine", "window", "r_t", "vae_spatial", "out_channels",
-        "out_dtype", "mlp_gated")] + [("norm_eps", ctypes.c_float), ("rope_base", ctypes.c_float)]
+        "out_dtype", "mlp_gated")] + [("norm_eps", ctypes.c_float), ("rope_base", ctypes.c_float),
+                                      ("qk_norm", ctypes.c_int32)]
 
 
 _P = ctypes.c_void_p
@@ -66,9 +67,12 @@ _SIGS = {
     "fd_chunk_index": (ctypes.c_int64, [_P]),
     "fd_sync_status": (_I, [_P]),
     "fd_debug_read_ring": (_I, [_P, _I, _I, _P, ctypes.c_size_t]),
+    "fd_state_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
+    "fd_save_state": (_I, [_P, _P, ctypes.c_size_t, _P]),
+    "fd_load_state": (_I, [_P, _P, ctypes.c_size_t, _P]),
     "fd_op_linear": (_I, [_I, _I, _I, _I, _P, _P, _P, _P, _I, _I, _P, _P]),
     "fd_op_rope_table": (_I, [_I, _I, _F, _P, _P]),
-    "fd_op_qkv": (_I, [_I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _F, _F,
+    "fd_op_qkv": (_I, [_I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _F, _F,
                        _P, _P, _P, _P, _I, _I, _P, _P]),
     "fd_attention_workspace_bytes": (ctypes.c_size_t, [_I, _I, _I, _I, _I]),
     "fd_op_attention": (_I, [_I, _I, _I, _P, _P, _P, _I, _I, _P, _I, _P, _P, _P]),
@@ -112,6 +116,7 @@ def make_config(cfg) -> fd_config:
         setattr(c, n, int(getattr(cfg, n)))
     c.out_dtype = DTYPE_U8 if getattr(cfg, "out_u8", False) else DTYPE_F32
     c.mlp_gated = 1 if cfg.mlp_gated else 0
+    c.qk_norm = 1 if cfg.qk_norm else 0
     c.norm_eps = float(cfg.norm_eps)
     c.rope_base = float(cfg.rope_base)
     return c
@@ -119,7 +124,8 @@ def make_config(cfg) -> fd_config:
 
 def weight_names(cfg) -> list[str]:
     """Tensor names in weight-blob order (the order documented in include/flashdec.h)."""
-    blk = ["norm1.g", "qkv.w", "qkv.b", "knorm.g", "vnorm.g", "out.w", "out.b", "norm2.g",
+    second = "qnorm.g" if getattr(cfg, "qk_norm", False) else "vnorm.g"
+    blk = ["norm1.g", "qkv.w", "qkv.b", "knorm.g", second, "out.w", "out.b", "norm2.g",
            "mlp1.w", "mlp1.b", "mlp2.w", "mlp2.b"]
     names = ["embed.w", "embed.b"]
     names += [f"blocks.{b}.{n}" for b in range(cfg.n_blocks) for n in blk]
@@ -145,6 +151,8 @@ def _stream_ptr(stream) -> int:
 def _ptr(x) -> int:
     if x is None:
         return 0
+    if isinstance(x, np.ndarray):
+        return int(x.ctypes.data)
     return int(x.data_ptr()) if hasattr(x, "data_ptr") else int(x)
 
 
@@ -239,6 +247,20 @@ class Decoder:
                "fd_debug_read_ring")
         return (buf[:n].reshape(groups, window * rows, 64), buf[n:].reshape(groups, window * rows, 64))
 
+    def state_bytes(self) -> int:
+        return lib().fd_state_bytes(ctypes.byref(self.cfg))
+
+    def save_state(self, buf, stream=None) -> None:
+        """Copy the streaming state (chunk index, rolling caches) into buf (host memory of
+        state_bytes() bytes: a numpy uint8 array or a pinned torch tensor), ordered on stream."""
+        _check(lib().fd_save_state(self.handle, _ptr(buf), self.state_bytes(),
+                                   _stream_ptr(stream)), "fd_save_state")
+
+    def load_state(self, buf, stream=None) -> None:
+        """Restore a state saved by a decoder of the same configuration."""
+        _check(lib().fd_load_state(self.handle, _ptr(buf), self.state_bytes(),
+                                   _stream_ptr(stream)), "fd_load_state")
+
     def close(self) -> None:
         if getattr(self, "handle", None):
             _check(lib().fd_destroy(self.handle), "fd_destroy")
@@ -272,11 +294,13 @@ def op_rope_table(t, frames_per_chunk, rope_base, table, stream=None) -> None:
                                   _stream_ptr(stream)), "fd_op_rope_table")
 
 
-def op_qkv(A, Wqkv, bqkv, knorm_g, vnorm_g, heads, groups, tokens, grid_w, frames_per_chunk,
+def op_qkv(A, Wqkv, bqkv, knorm_g, norm2_g, heads, groups, tokens, grid_w, frames_per_chunk,
            window, t, eps, rope_base, rope_t, q_out, k_ring, vt_ring, ring_pitch, bn=0, err=None,
-           stream=None) -> None:
+           stream=None, qk_norm=False) -> None:
+    """norm2_g: V's gain (KV-norm) or, with qk_norm, Q's gain."""
     M, K = A.shape
-    _check(lib().fd_op_qkv(M, K, _ptr(A), _ptr(Wqkv), _ptr(bqkv), _ptr(knorm_g), _ptr(vnorm_g),
+    _check(lib().fd_op_qkv(M, K, _ptr(A), _ptr(Wqkv), _ptr(bqkv), _ptr(knorm_g), _ptr(norm2_g),
+                           1 if qk_norm else 0,
                            heads, groups, tokens, grid_w, frames_per_chunk, window, t, eps,
                            rope_base, _ptr(rope_t), _ptr(q_out), _ptr(k_ring), _ptr(vt_ring),
                            ring_pitch, bn, _ptr(err), _stream_ptr(stream)), "fd_op_qkv")

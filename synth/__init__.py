@@ -40,6 +40,7 @@ class FDConfig:
     kv_groups: int = 2             # G
     mlp_ratio: int = 4
     mlp_gated: bool = False        # MLP: False = Linear, GELU, Linear; True = gated SiLU
+    qk_norm: bool = False          # per-head RMSNorm on Q and K instead of on K and V
     n_blocks: int = 2              # backbone blocks
     n_refine: int = 0              # temporal-refinement blocks
     window: int = 2                # W_frm, counts the current chunk
@@ -135,6 +136,8 @@ PRESETS: dict[str, FDConfig] = {
     "small_u8": FDConfig(latent_h=20, latent_w=26, patch=2, hidden=256, heads=4, kv_groups=1,
                          n_blocks=1, n_refine=1, window=2, r_t=4, out_u8=True,
                          name="small_u8", chunks=4),
+    # the QK-norm reading of "KV-norm" at tiny size, with refinement
+    "tiny_qk": FDConfig(qk_norm=True, n_refine=1, r_t=2, name="tiny_qk", chunks=3),
     # XL layout at tiny size: 48-channel 16x latent, patch 1, gated-SiLU MLP, refinement
     "tiny_gated": FDConfig(latent_channels=48, latent_h=10, latent_w=13, vae_spatial=16,
                            mlp_gated=True, n_refine=1, r_t=2, name="tiny_gated", chunks=3),
@@ -171,7 +174,7 @@ def weight_layout(cfg: FDConfig) -> list[tuple[str, tuple[int, ...], str]]:
             (f"{prefix}.qkv.w", ((N + 2 * G) * Dh, D), "w"),
             (f"{prefix}.qkv.b", ((N + 2 * G) * Dh,), "b"),
             (f"{prefix}.knorm.g", (Dh,), "g"),
-            (f"{prefix}.vnorm.g", (Dh,), "g"),
+            (f"{prefix}.{'qnorm' if cfg.qk_norm else 'vnorm'}.g", (Dh,), "g"),
             (f"{prefix}.out.w", (D, N * Dh), "w"),
             (f"{prefix}.out.b", (D,), "b"),
             (f"{prefix}.norm2.g", (D,), "g"),

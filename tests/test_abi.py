@@ -49,6 +49,25 @@ def test_sizes_follow_the_compression_factors():
     assert L.fd_pixels_bytes(ctypes.byref(c)) == 3 * 4 * 720 * 1280
 
 
+def test_state_size_is_header_plus_every_ring():
+    """Saved streaming state: a header (magic, version, t, payload size, the config) and, per
+    layer, K [G][pitch][64] bf16 and V^T [G][64][pitch] fp16 with pitch = round_up(W rows, 128)
+    (rows = L backbone, r_t L refinement)."""
+    L = fdp.lib()
+    cfg = synth.PRESETS["480p"]
+    c = fdp.make_config(cfg)
+    up = lambda x: -(-x // 128) * 128
+    ring = lambda rows: cfg.kv_groups * up(cfg.window * rows) * 64 * 2
+    payload = 2 * (cfg.n_blocks * ring(cfg.tokens) + cfg.n_refine * ring(cfg.r_t * cfg.tokens))
+    header = -(-(8 + 3 * 8 + ctypes.sizeof(fdp.fd_config)) // 8) * 8  # 8-byte aligned struct
+    assert L.fd_state_bytes(ctypes.byref(c)) == header + payload
+    bad = fdp.make_config(synth.PRESETS["small"].replace(heads=3))
+    assert L.fd_state_bytes(ctypes.byref(bad)) == 0
+    buf = ctypes.create_string_buffer(16)
+    assert L.fd_save_state(None, buf, 16, None) == 1
+    assert L.fd_load_state(None, buf, 16, None) == 1
+
+
 @pytest.mark.parametrize("field,value", [("hidden", 320), ("heads", 3), ("kv_groups", 3),
                                          ("patch", 3), ("window", 0), ("r_t", 0),
                                          ("n_blocks", 0), ("latent_channels", 1)])

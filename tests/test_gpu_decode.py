@@ -64,7 +64,8 @@ def compare(cfg, got, want, what, max_abs=MAX_ABS, mean_abs=MEAN_ABS):
                 f"{what} chunk {t}: max-abs {mx:.3e} mean-abs {mean:.3e}"
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8", "tiny_gated"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8", "tiny_gated",
+                                  "tiny_qk"])
 def test_decode_matches_oracle(name):
     cfg = synth.PRESETS[name]
     w, z = synth.make_weights(cfg), synth.make_latents(cfg)
@@ -110,6 +111,46 @@ def test_decode_chunks_concurrent_streams_match_single_stream_decodes():
     for s in range(len(zs)):
         for t in range(cfg.chunks):
             assert torch.equal(got[s][t], alone[s][t]), (s, t)
+
+
+def test_state_save_load_resumes_the_stream_bit_exactly():
+    """Checkpoint / resume: decode chunks 0..k-1, save the state, load it into a fresh handle
+    (same configuration and weights) and decode chunks k.. there: every pixel equals the
+    uninterrupted stream's, and the saving handle continues unaffected. A state of another
+    configuration, a wrong size or a damaged header is refused."""
+    cfg = synth.PRESETS["small"]          # W = 3: the resumed chunks evict saved ones
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    want = gpu_stream(cfg, w, z)
+    W = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    a = fdp.Decoder(cfg, W)
+    shape = (cfg.out_channels, cfg.r_t, cfg.out_h, cfg.out_w)
+    k = 2
+    for t in range(k):
+        a.decode_chunk(dev(z[t]), torch.empty(shape, device="cuda"))
+    buf = torch.empty(a.state_bytes(), dtype=torch.uint8).pin_memory()
+    a.save_state(buf)
+    torch.cuda.synchronize()
+    b = fdp.Decoder(cfg, W)
+    b.load_state(buf)
+    assert b.chunk_index == k
+    for t in range(k, cfg.chunks):
+        pa, pb = torch.empty(shape, device="cuda"), torch.empty(shape, device="cuda")
+        a.decode_chunk(dev(z[t]), pa)
+        b.decode_chunk(dev(z[t]), pb)
+        torch.cuda.synchronize()
+        assert torch.equal(pb.cpu(), want[t]), t
+        assert torch.equal(pa.cpu(), want[t]), t
+    assert a.sync_status() == fdp.FD_OK and b.sync_status() == fdp.FD_OK
+    L = fdp.lib()
+    other = synth.PRESETS["small"].replace(window=2)
+    c = fdp.Decoder(other, fdp.Weights(other, fdp.pack_blob(other, synth.make_weights(other))))
+    assert L.fd_load_state(c.handle, fdp._ptr(buf), a.state_bytes(), None) == 1  # size differs
+    bad = buf.clone()
+    bad[0] = ord("X")
+    assert L.fd_load_state(b.handle, fdp._ptr(bad), b.state_bytes(), None) == 1
+    for d in (a, b, c):
+        d.close()
+    W.close()
 
 
 def test_decode_causality_on_gpu():

@@ -116,14 +116,16 @@ class Cfg:
         self.__dict__.update(kw)
 
 
-@pytest.mark.parametrize("heads,groups,grid_h,grid_w,fpc,window,t,K,bn", [
-    (4, 2, 10, 13, 4, 3, 5, 256, 128),       # refinement-like: 4 frames per chunk, ragged rows
-    (16, 4, 30, 52, 1, 4, 7, 1024, 192),     # 480p backbone block, 192-wide tiles
-    (16, 4, 30, 52, 1, 4, 7, 1024, 256),     # same, 256-wide tiles
-    (24, 3, 3, 5, 1, 8, 130, 1536, 64),      # wide model, long stream (large temporal index)
-    (4, 2, 8, 8, 4, 2, 40000, 256, 0),       # very long stream: temporal index 160000
+@pytest.mark.parametrize("heads,groups,grid_h,grid_w,fpc,window,t,K,bn,qk", [
+    (4, 2, 10, 13, 4, 3, 5, 256, 128, False),    # refinement-like: 4 frames per chunk, ragged
+    (16, 4, 30, 52, 1, 4, 7, 1024, 192, False),  # 480p backbone block, 192-wide tiles
+    (16, 4, 30, 52, 1, 4, 7, 1024, 256, False),  # same, 256-wide tiles
+    (24, 3, 3, 5, 1, 8, 130, 1536, 64, False),   # wide model, long stream (large temporal index)
+    (4, 2, 8, 8, 4, 2, 40000, 256, 0, False),    # very long stream: temporal index 160000
+    (16, 4, 30, 52, 1, 4, 7, 1024, 192, True),   # QK-norm instead of KV-norm
+    (4, 2, 10, 13, 4, 3, 5, 256, 128, True),     # QK-norm, refinement-like
 ])
-def test_qkv_fused(heads, groups, grid_h, grid_w, fpc, window, t, K, bn):
+def test_qkv_fused(heads, groups, grid_h, grid_w, fpc, window, t, K, bn, qk):
     dh, eps, base = 64, 1e-6, 10000.0
     tokens = grid_h * grid_w
     M = fpc * tokens
@@ -140,15 +142,19 @@ def test_qkv_fused(heads, groups, grid_h, grid_w, fpc, window, t, K, bn):
     fdp.op_rope_table(t, fpc, base, rope_t)
     fdp.op_qkv(dev(A, torch.bfloat16), dev(W, torch.bfloat16), dev(b), dev(kg), dev(vg), heads,
                groups, tokens, grid_w, fpc, window, t, eps, base, rope_t, q_out, k_ring, vt_ring,
-               pitch, bn=bn, err=err)
+               pitch, bn=bn, err=err, qk_norm=qk)
     check_err(err)
-    # oracle: Linear, KV-norm, 3D-RoPE at (t*fpc + row // tokens, y, x)
+    # oracle: Linear, KV-norm (or QK-norm, vg then Q's gain), 3D-RoPE at (t*fpc + row // tokens,
+    # y, x)
     qkv = oracle.linear(f64(A), f64(W), f64(b))
     q = qkv[:, :heads * dh].reshape(M, heads, dh).transpose(0, 1)
     k = qkv[:, heads * dh:(heads + groups) * dh].reshape(M, groups, dh).transpose(0, 1)
     v = qkv[:, (heads + groups) * dh:].reshape(M, groups, dh).transpose(0, 1)
     k = oracle.rms_norm(k, f64(kg), eps)
-    v = oracle.rms_norm(v, f64(vg), eps)
+    if qk:
+        q = oracle.rms_norm(q, f64(vg), eps)
+    else:
+        v = oracle.rms_norm(v, f64(vg), eps)
     r = torch.arange(M)
     pos = ((t * fpc + r // tokens).double(), ((r % tokens) // grid_w).double(),
            ((r % tokens) % grid_w).double())

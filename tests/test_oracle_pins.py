@@ -101,6 +101,36 @@ def test_operand_rounding_rounds_to_nearest_even_and_is_off_by_default():
     assert torch.equal(oracle.linear(x, w, None), x)
 
 
+def test_qk_norm_bounds_every_score():
+    """QK-norm option: with unit gains every query and key head vector has length sqrt(D_h), so
+    by Cauchy-Schwarz every scaled score q.k / sqrt(D_h) lies in [-sqrt(D_h), sqrt(D_h)] = [-8, 8],
+    whatever the activations; V keeps its scale. KV-norm normalises V instead of Q."""
+    from oracle.flashdecoder import _block_qkv
+    base = synth.PRESETS["tiny_qk"]
+    Dh, N, G, D = base.head_dim, base.heads, base.kv_groups, base.hidden
+    torch.manual_seed(0)
+    h = torch.randn(16, D, dtype=torch.float64) * 3
+    w = {"x.norm1.g": torch.ones(D, dtype=torch.float64),
+         "x.qkv.w": torch.randn((N + 2 * G) * Dh, D, dtype=torch.float64) * 5,
+         "x.qkv.b": torch.zeros((N + 2 * G) * Dh, dtype=torch.float64),
+         "x.knorm.g": torch.ones(Dh, dtype=torch.float64),
+         "x.qnorm.g": torch.ones(Dh, dtype=torch.float64),
+         "x.vnorm.g": torch.ones(Dh, dtype=torch.float64)}
+    for qk in (True, False):
+        cfg = base.replace(qk_norm=qk, norm_eps=0.0)
+        q, k, v = _block_qkv(h, w, "x.", cfg, None)
+        qn, kn, vn = (x.norm(dim=-1) for x in (q, k, v))
+        assert torch.allclose(kn, torch.full_like(kn, math.sqrt(Dh)), atol=1e-9)
+        if qk:
+            assert torch.allclose(qn, torch.full_like(qn, math.sqrt(Dh)), atol=1e-9)
+            s = torch.einsum("nld,nmd->nlm", q, k.repeat_interleave(N // G, 0)) / math.sqrt(Dh)
+            assert float(s.abs().max()) <= math.sqrt(Dh) + 1e-9
+            assert float(vn.max()) > 2 * math.sqrt(Dh)   # V left as projected
+        else:
+            assert torch.allclose(vn, torch.full_like(vn, math.sqrt(Dh)), atol=1e-9)
+            assert float(qn.max()) > 2 * math.sqrt(Dh)
+
+
 def test_linear_is_x_wt_plus_b():
     x, w, b = rnd(5, 7, seed=3), rnd(4, 7, seed=4), rnd(4, seed=5)
     brute = torch.tensor([[sum(x[i, k] * w[j, k] for k in range(7)) + b[j] for j in range(4)]
@@ -261,7 +291,7 @@ def test_fig2_visibility_golden():
             assert torch.equal(K[:, slot * cfg.tokens:(slot + 1) * cfg.tokens], keys_of_chunk[c])
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8", "tiny_qk", "tiny_gated"])
 def test_streaming_equals_masked_full_sequence(name):
     """Sec. 3.3: sequential decoding with the rolling cache equals one pass under the block
     sliding-window mask (the paper's training-inference consistency)."""
