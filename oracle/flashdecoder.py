@@ -31,6 +31,12 @@ Readings where the paper leaves a choice (each listed in the design notes):
   R7  MLP = Linear(D, 4D) -> GELU (erf form) -> Linear(4D, D); biases on every linear (R13).
       Gated option (the XL layout): Linear(D, 4D) gate and Linear(D, 4D) up, SiLU(gate) * up,
       then Linear(4D, D); the first weight stores the gate rows, then the up rows.
+      FP8 option (Sec. 4.6, "static-calibrated FP8 quantization of all MLP layers"): both MLP
+      matrix products take e4m3 operands with power-of-two scales fixed before decoding:
+      per weight row s = 2^ceil(log2(max|w| / 448)); the MLP input u = RMSNorm(h) g obeys
+      |u_i| <= sqrt(D) max|g|, its scale s_u covers that; the MLP hidden a = GELU(z) obeys
+      |a_j| <= max(1, max_j 1.125 sqrt(D) max|g| ||w1_j|| + |b1_j|), its scale s_h covers that.
+      So no value leaves the e4m3 range (448) for any input.
   R8  Head MLP: Linear(D, D) -> GELU -> Linear(D, C r_s^2).
   R9  Pixels clamped to [-1, 1]; uint8 = round-half-even(fl32(fl32(x + 1) * 127.5)).
   R12 RMSNorm with a learned gain before the temporal upsampling and before the head.
@@ -93,6 +99,35 @@ def rms_norm(x: torch.Tensor, g: torch.Tensor, eps: float) -> torch.Tensor:
 def gelu(x: torch.Tensor) -> torch.Tensor:
     """GELU, exact erf form: x * Phi(x) = 0.5 x (1 + erf(x / sqrt 2))."""
     return 0.5 * x * (1.0 + torch.erf(x / math.sqrt(2.0)))
+
+
+def e4m3(x: torch.Tensor) -> torch.Tensor:
+    """Round to the nearest FP8 E4M3 value (OCP: 3 mantissa bits, bias 7, largest 448,
+    subnormals down to 2^-9), ties to even."""
+    return x.to(torch.float8_e4m3fn).to(F64)
+
+
+def pow2_ceil(x: float) -> float:
+    """Smallest power of two >= x (x > 0), exactly."""
+    m, e = math.frexp(x)          # x = m 2^e, 0.5 <= m < 1
+    return math.ldexp(1.0, e - 1) if m == 0.5 else math.ldexp(1.0, e)
+
+
+def fp8_weight(w: torch.Tensor) -> torch.Tensor:
+    """Per-row FP8 quantisation of a Linear weight [out][in], returned dequantised."""
+    amax = w.abs().max(dim=1).values
+    s = torch.tensor([pow2_ceil(float(a) / 448.0) if a > 0 else 1.0 for a in amax], dtype=F64)
+    return e4m3(w / s[:, None]) * s[:, None]
+
+
+def fp8_mlp_scales(g2: torch.Tensor, w1_deq: torch.Tensor, b1: torch.Tensor):
+    """Static activation scales (s_u, s_h) of one FP8 MLP from its weights (see R7)."""
+    D = g2.shape[0]
+    gmax = float(g2.abs().max())
+    s_u = pow2_ceil(math.sqrt(D) * gmax / 448.0)
+    bz = float((1.125 * math.sqrt(D) * gmax * w1_deq.norm(dim=1) + b1.abs()).max())
+    s_h = pow2_ceil(max(bz, 1.0) / 448.0)
+    return s_u, s_h
 
 
 def silu(x: torch.Tensor) -> torch.Tensor:
@@ -225,6 +260,11 @@ def _block_rest(h, o, w, p, cfg):
     o = o.transpose(0, 1).reshape(L, -1)
     h = h + linear(o, w[p + "out.w"], w[p + "out.b"])
     u = rms_norm(h, w[p + "norm2.g"], cfg.norm_eps)
+    if getattr(cfg, "mlp_fp8", False):
+        w1, w2 = fp8_weight(w[p + "mlp1.w"]), fp8_weight(w[p + "mlp2.w"])
+        s_u, s_h = fp8_mlp_scales(w[p + "norm2.g"], w1, w[p + "mlp1.b"])
+        a = gelu(linear(e4m3(u / s_u) * s_u, w1, w[p + "mlp1.b"]))
+        return h + linear(e4m3(a / s_h) * s_h, w2, w[p + "mlp2.b"])
     z = linear(u, w[p + "mlp1.w"], w[p + "mlp1.b"])
     if cfg.mlp_gated:
         dm = z.shape[1] // 2

@@ -131,6 +131,50 @@ def test_qk_norm_bounds_every_score():
             assert float(qn.max()) > 2 * math.sqrt(Dh)
 
 
+def test_e4m3_rounding_worked_values():
+    """FP8 E4M3 (3 mantissa bits, exponent bias 7, max 448, subnormal step 2^-9), ties to even,
+    on values worked out by hand: 1 + 2^-4 lies halfway between 1 and 1.125 -> 1 (even
+    mantissa); 1.1875 halfway between 1.125 and 1.25 -> 1.25; 3 * 2^-10 halfway between the
+    subnormals 2^-9 and 2^-8 -> 2^-8; 2^-10 halfway between 0 and 2^-9 -> 0; 449 -> 448."""
+    cases = [(0.5, 0.5), (1.0625, 1.0), (1.1875, 1.25), (-1.0625, -1.0), (13.0, 13.0),
+             (448.0, 448.0), (449.0, 448.0), (2.0 ** -9, 2.0 ** -9), (3 * 2.0 ** -10, 2.0 ** -8),
+             (2.0 ** -10, 0.0), (248.0, 256.0), (0.0, 0.0)]
+    x = torch.tensor([c[0] for c in cases], dtype=torch.float64)
+    assert oracle.e4m3(x).tolist() == [c[1] for c in cases]
+
+
+def test_pow2_ceil_is_exact():
+    assert [oracle.pow2_ceil(v) for v in (3.0, 4.0, 0.3, 1.0, 4.000001, 2.0 ** -20)] == \
+        [4.0, 4.0, 0.5, 1.0, 8.0, 2.0 ** -20]
+
+
+def test_fp8_static_scales_never_overflow_and_are_tight():
+    """The static MLP scales keep every scaled FP8 operand within the e4m3 range (448) for any
+    input, including a row whose RMSNorm puts all its weight in one coordinate (|u_i| =
+    sqrt(D) g_i, the bound), and that row uses more than half of the range."""
+    from oracle.flashdecoder import gelu, linear
+    cfg = synth.PRESETS["small_fp8"]
+    w = {k: torch.from_numpy(v).to(torch.float64) for k, v in synth.make_weights(cfg).items()}
+    D = cfg.hidden
+    g2, w1, b1 = w["blocks.0.norm2.g"], oracle.fp8_weight(w["blocks.0.mlp1.w"]), w["blocks.0.mlp1.b"]
+    s_u, s_h = oracle.fp8_mlp_scales(g2, w1, b1)
+    h = torch.randn(64, D, dtype=torch.float64) * 3
+    i = int(g2.abs().argmax())
+    h[0] = 0.0
+    h[0, i] = 5.0                                 # one-hot row: |u_i| = sqrt(D) |g_i|
+    u = oracle.rms_norm(h, g2, 0.0)
+    assert float((u / s_u).abs().max()) <= 448.0
+    assert float((u[0] / s_u).abs().max()) > 224.0
+    a = gelu(linear(oracle.e4m3(u / s_u) * s_u, w1, b1))
+    assert float((a / s_h).abs().max()) <= 448.0
+    # the FP8 MLP output differs from the exact one by FP8-sized amounts, not more
+    w2 = w["blocks.0.mlp2.w"]
+    exact = linear(gelu(linear(u, w["blocks.0.mlp1.w"], b1)), w2, None)
+    q = linear(oracle.e4m3(a / s_h) * s_h, oracle.fp8_weight(w2), None)
+    rel = float((q - exact).norm() / exact.norm())
+    assert 1e-3 < rel < 0.1, rel
+
+
 def test_linear_is_x_wt_plus_b():
     x, w, b = rnd(5, 7, seed=3), rnd(4, 7, seed=4), rnd(4, seed=5)
     brute = torch.tensor([[sum(x[i, k] * w[j, k] for k in range(7)) + b[j] for j in range(4)]
@@ -291,7 +335,8 @@ def test_fig2_visibility_golden():
             assert torch.equal(K[:, slot * cfg.tokens:(slot + 1) * cfg.tokens], keys_of_chunk[c])
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8", "tiny_qk", "tiny_gated"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8", "tiny_qk", "tiny_gated",
+                                  "small_fp8"])
 def test_streaming_equals_masked_full_sequence(name):
     """Sec. 3.3: sequential decoding with the rolling cache equals one pass under the block
     sliding-window mask (the paper's training-inference consistency)."""
