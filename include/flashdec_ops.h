@@ -113,6 +113,25 @@ fd_status fd_op_kv_append(const float* k, const float* v, int groups, int rows, 
 fd_status fd_op_rmsnorm(const float* h, const float* g, int M, int D, float eps, void* u,
                         void* stream);
 
+/* The same with e4m3 output (the input of an FP8 MLP, Sec. 4.6):
+ * u e4m3 [M][D] = e4m3(h / sqrt(mean(h^2) + eps) * g * out_scale), round to nearest even,
+ * saturating at +-448. */
+fd_status fd_op_rmsnorm_e4m3(const float* h, const float* g, int M, int D, float eps,
+                             float out_scale, void* u, void* stream);
+
+/* FP8 linear layer (the MLP products of the FP8 option, Sec. 4.6): A e4m3 [M][K], W e4m3
+ * [N][K] (nn.Linear layout), col_scale fp32 [N] (the dequantisation s_A * s_W[n]), bias fp32
+ * [N]; acc = sum_k A[m][k] W[n][k], exact e4m3 products accumulated in fp32 (tcgen05
+ * kind::f8f6f4):
+ *   FD_EPI_F32    out fp32 [M][N]  = acc * col_scale + bias
+ *   FD_EPI_RESID  out fp32 [M][N] += acc * col_scale + bias
+ *   FD_EPI_GELU   out e4m3 [M][N]  = e4m3(GELU(acc * col_scale + bias) * out_scale)
+ * K % 16 == 0, N % 32 == 0 (N % 128 == 0 for FD_EPI_GELU), 16-byte aligned A / W / out.
+ * bn = output tile width (96 / 128 / 192 / 256, 128 or 256 for FD_EPI_GELU; 0 = choice). */
+fd_status fd_op_linear_e4m3(int epilogue, int M, int N, int K, const void* A, const void* W,
+                            const float* col_scale, const float* bias, void* out,
+                            float out_scale, int bn, int* err_dev, void* stream);
+
 /* PixelUnshuffle(p) of a latent frame z fp32 [C][H][W] into tokens x0 bf16 [(H/p)(W/p)][C p^2]
  * (Sec. 4.3; raster token order of Eq. projection). */
 fd_status fd_op_unshuffle(const float* z, int C, int H, int W, int p, void* x0, void* stream);

@@ -19,6 +19,10 @@
 //   EPI_TUP    channel block tau of token l -> refined token tau*L + l   (Eq. temporal_upsample)
 //   EPI_SWIGLU out = bf16(SiLU(gate + b) * (up + b)) (gated MLP layer 1 of the XL layout; gate
 //              and up rows interleaved in blocks of 32, so 128 columns give 64 outputs)
+//   EPI_GELU_F8 out = e4m3(GELU(acc s_col + b) s_out)  (FP8 MLP layer 1, Sec. 4.6)
+// FP8 operands (p.fp8): A and W are e4m3 with a K-block of 128 elements (the same 128-byte
+// swizzled rows), tcgen05.mma kind::f8f6f4 with K = 32 per instruction; the fp32 epilogues
+// then scale the accumulator per column by s_A s_W[n] (p.col_scale).
 //   EPI_QKV    bias; KV-norm (RMS over D_h) on K and V (or QK-norm on Q and K); 3D-RoPE on Q
 //              and K; Q to its buffer,
 //              K (bf16) and V (transposed, fp16) into ring slot t mod W of the layer's cache
@@ -101,7 +105,8 @@ __global__ void __launch_bounds__(192, 1)
   const int m_tiles = (p.M + kBM - 1) / kBM;
   const int n_tiles = (p.N + BN - 1) / BN;
   const int tiles = m_tiles * n_tiles;
-  const int nk = (p.K + kBK - 1) / kBK;
+  const int kel = p.fp8 ? 2 * kBK : kBK;  // K elements per 128-byte stage row
+  const int nk = (p.K + kel - 1) / kel;
 
   if (threadIdx.x == 0) {
     if (!aligned) atomicOr(p.err, ERR_SMEM_ALIGN);
@@ -140,8 +145,8 @@ __global__ void __launch_bounds__(192, 1)
         const uint32_t ph = (it / C::kStages) & 1;
         if (!mbar_wait(bar_empty + 8 * s, ph ^ 1, p.err, ERR_WAIT_MMA)) { ok = false; break; }
         mbar_expect_tx(bar_full + 8 * s, C::kStageBytes);
-        tma_load_2d(sA + s * C::kABytes, &tmA, bar_full + 8 * s, kb * kBK, m0);
-        tma_load_2d(sB + s * C::kBBytes, &tmB, bar_full + 8 * s, kb * kBK, n0);
+        tma_load_2d(sA + s * C::kABytes, &tmA, bar_full + 8 * s, kb * kel, m0);
+        tma_load_2d(sB + s * C::kBBytes, &tmB, bar_full + 8 * s, kb * kel, n0);
       }
     }
     // drain: the loads issued last must land before the CTA may exit
@@ -149,7 +154,7 @@ __global__ void __launch_bounds__(192, 1)
       mbar_wait(bar_full + 8 * (j % C::kStages), (j / C::kStages) & 1, p.err, ERR_WAIT_TMA);
   } else if (aligned && warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA issuer
-    const uint32_t idesc = idesc_bf16_f32(kBM, BN);
+    const uint32_t idesc = p.fp8 ? idesc_e4m3_f32(kBM, BN) : idesc_bf16_f32(kBM, BN);
     int it = 0, tc = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++tc) {
@@ -166,10 +171,17 @@ __global__ void __launch_bounds__(192, 1)
         tc_fence_after();
         const uint32_t a0 = sA + s * C::kABytes;
         const uint32_t b0 = sB + s * C::kBBytes;
+        if (p.fp8) {
 #pragma unroll
-        for (int k = 0; k < kBK / 16; ++k)
-          mma_bf16_ss(d_tmem, sdesc_k_sw128(a0 + 32 * k), sdesc_k_sw128(b0 + 32 * k), idesc,
-                      (kb | k) != 0);
+          for (int k = 0; k < 4; ++k)  // 4 x 32 e4m3 = one 128-byte row
+            mma_e4m3_ss(d_tmem, sdesc_k_sw128(a0 + 32 * k), sdesc_k_sw128(b0 + 32 * k), idesc,
+                        (kb | k) != 0);
+        } else {
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+            mma_bf16_ss(d_tmem, sdesc_k_sw128(a0 + 32 * k), sdesc_k_sw128(b0 + 32 * k), idesc,
+                        (kb | k) != 0);
+        }
         mma_commit(bar_empty + 8 * s);  // stage s free once these MMAs have read it
       }
       if (ok) mma_commit(bar_tfull + 8 * acc);
@@ -322,6 +334,40 @@ __global__ void __launch_bounds__(192, 1)
             bulk_commit();
           }
         }
+      } else if (p.epi == EPI_GELU_F8) {
+        // 128 accumulator columns -> one 128-byte row of e4m3 per slab
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 128) {
+          const int col = n0 + c;
+          if (col >= p.N) break;
+          uint32_t w[32];
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4) {
+            uint32_t r[32];
+            __syncwarp();
+            tmem_ld_32x32b_x32(tbase + c + 32 * q4, r);
+            tmem_ld_wait();
+            const int cb = col + 32 * q4;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              float f[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int cc = cb + 4 * j + e;
+                f[e] = gelu_erf(fmaf(__uint_as_float(r[4 * j + e]), __ldg(p.col_scale + cc),
+                                     __ldg(p.bias + cc))) * p.out_scale;
+              }
+              w[8 * q4 + j] = pack_e4m3x4(f[0], f[1], f[2], f[3]);
+            }
+          }
+          uint8_t* buf = acquire();
+          put_row_sw128(buf, lane, w);
+          publish();
+          if (lane == 0 && row0 < p.M) {
+            tma_store_2d(&tmO, smem_u32(buf), col, row0);
+            bulk_commit();
+          }
+        }
       } else if (p.epi == EPI_SWIGLU) {
 #pragma unroll 1
         for (int c = 0; c < BN; c += 128) {
@@ -363,9 +409,16 @@ __global__ void __launch_bounds__(192, 1)
           tmem_ld_32x32b_x32(tbase + c, r);
           tmem_ld_wait();
           uint32_t w[32];
+          if (p.col_scale != nullptr) {  // FP8 operands: dequantise per column
 #pragma unroll
-          for (int j = 0; j < 32; ++j)
-            w[j] = __float_as_uint(__uint_as_float(r[j]) + __ldg(p.bias + col + j));
+            for (int j = 0; j < 32; ++j)
+              w[j] = __float_as_uint(fmaf(__uint_as_float(r[j]), __ldg(p.col_scale + col + j),
+                                          __ldg(p.bias + col + j)));
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              w[j] = __float_as_uint(__uint_as_float(r[j]) + __ldg(p.bias + col + j));
+          }
           uint8_t* buf = acquire();
           put_row_sw128(buf, lane, w);
           publish();

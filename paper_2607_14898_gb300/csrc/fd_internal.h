@@ -40,6 +40,7 @@ enum EpiKind : int {
   EPI_QKV = 4,    // bias, KV-norm, 3D-RoPE; Q to q_out, K/V into the cache ring slot
   EPI_SWIGLU = 5, // gated SiLU: accumulator columns in blocks of 64 (32 gate, 32 up of the same
                   // hidden units); out_bf16[r][32j + i] = bf16(SiLU(g + bg) * (u + bu))
+  EPI_GELU_F8 = 6,  // out_f8[r][c] = e4m3(GELU(acc * col_scale + bias) * out_scale)
 };
 
 // Rotary / cache parameters of the fused QKV epilogue.
@@ -84,6 +85,13 @@ struct GemmParams {
   int tup_tokens, tup_hidden;
   QkvEpi qkv;
   int* err;
+  // FP8 operands: A and W are e4m3 (K-blocks of 128 elements, kind::f8f6f4 MMAs); the
+  // accumulator is dequantised per output column by col_scale (s_A * s_W[n]) in the fp32 and
+  // GELU_F8 epilogues. out_scale: multiplier before the e4m3 rounding of EPI_GELU_F8.
+  int fp8;
+  const float* col_scale;
+  uint8_t* out_f8;
+  float out_scale;
 };
 
 struct AttnParams {
@@ -145,6 +153,9 @@ cudaError_t launch_unshuffle(const float* z, int C, int H, int W, int p, __nv_bf
                              cudaStream_t s);
 cudaError_t launch_rmsnorm(const float* h, const float* g, int M, int D, float eps,
                            __nv_bfloat16* u, cudaStream_t s);
+// u[r][c] = e4m3(rmsnorm(h)[r][c] * oscale)  (FP8 MLP input)
+cudaError_t launch_rmsnorm_e4m3(const float* h, const float* g, int M, int D, float eps,
+                                uint8_t* u, float oscale, cudaStream_t s);
 cudaError_t launch_pixel_head(const float* F, int frames, int gh, int gw, int C, int rs,
                               int out_u8, void* pix, cudaStream_t s);
 cudaError_t launch_kv_append(const float* k, const float* v, int groups, int rows, int slot,
@@ -167,6 +178,7 @@ inline bool gemm_bn_supported(int bn) {
 // the fp32 epilogues on 32-column slabs
 inline bool gemm_bn_fits_epilogue(int bn, int epi) {
   if (epi == EPI_SWIGLU) return bn % 128 == 0;  // 128 accumulator columns -> 64 outputs
+  if (epi == EPI_GELU_F8) return bn % 128 == 0;  // 128 e4m3 outputs per 128-byte slab row
   return (epi == EPI_QKV || epi == EPI_GELU) ? bn % 64 == 0 : bn % 32 == 0;
 }
 

@@ -1,7 +1,8 @@
 // Bandwidth-bound kernels of the decode path.
 //   unshuffle    latent [C'][H'][W'] fp32 -> tokens [L][C' p^2] bf16 (PixelUnshuffle, Sec. 4.3;
 //                raster token order of Eq. projection)
-//   rmsnorm      h fp32 [M][D] -> bf16(h / sqrt(mean(h^2) + eps) * g)  (pre-norm, Sec. 3.2)
+//   rmsnorm      h fp32 [M][D] -> bf16(h / sqrt(mean(h^2) + eps) * g)  (pre-norm, Sec. 3.2),
+//                or e4m3 of that times a scale (input of an FP8 MLP)
 //   pixel_head   F fp32 [frames*L][C r_s^2] -> PixelShuffle(r_s) + clamp to [-1, 1], fp32 or
 //                uint8 (Sec. 3.4 "Step 3"); one thread per 4 consecutive output pixels
 //   kv_append    fp32 K, V of one chunk -> ring slot (K rows bf16, V transposed fp16) (Sec. 3.3)
@@ -28,12 +29,13 @@ __global__ void unshuffle_kernel(const float* __restrict__ z, int C, int H, int 
   }
 }
 
-// one warp per row, the row held in registers (D / 128 float4 per lane, D % 128 == 0,
-// D <= 128 * kMaxChunks): one pass over h
-constexpr int kMaxChunks = 16;
-template <int CH>
+// one warp per row, the row held in registers (D / 128 float4 per lane for D / 128 in
+// {2, 4, 8, 12, 16}, one pass over h; any other multiple of 128 takes two passes); output bf16,
+// or e4m3 of (y * oscale) when F8
+template <int CH, bool F8>
 __device__ __forceinline__ void rmsnorm_row(const float4* hr, const float4* g4, int lane,
-                                            float inv_d, float eps, uint2* ur) {
+                                            float inv_d, float eps, void* out_row,
+                                            float oscale) {
   float4 v[CH];
   float ss = 0.f;
 #pragma unroll
@@ -47,13 +49,21 @@ __device__ __forceinline__ void rmsnorm_row(const float4* hr, const float4* g4, 
 #pragma unroll
   for (int c = 0; c < CH; ++c) {
     const float4 gg = g4[lane + 32 * c];
-    ur[lane + 32 * c] = make_uint2(pack_bf16x2(v[c].x * r * gg.x, v[c].y * r * gg.y),
-                                   pack_bf16x2(v[c].z * r * gg.z, v[c].w * r * gg.w));
+    const float y0 = v[c].x * r * gg.x, y1 = v[c].y * r * gg.y;
+    const float y2 = v[c].z * r * gg.z, y3 = v[c].w * r * gg.w;
+    if (F8) {
+      reinterpret_cast<uint32_t*>(out_row)[lane + 32 * c] =
+          pack_e4m3x4(y0 * oscale, y1 * oscale, y2 * oscale, y3 * oscale);
+    } else {
+      reinterpret_cast<uint2*>(out_row)[lane + 32 * c] =
+          make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
+    }
   }
 }
 
+template <bool F8>
 __global__ void rmsnorm_kernel(const float* __restrict__ h, const float* __restrict__ g, int M,
-                               int D, float eps, __nv_bfloat16* __restrict__ u) {
+                               int D, float eps, void* __restrict__ u, float oscale) {
   grid_dep_wait();
   grid_dep_launch();
   const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -61,14 +71,14 @@ __global__ void rmsnorm_kernel(const float* __restrict__ h, const float* __restr
   if (row >= M) return;
   const float4* hr = reinterpret_cast<const float4*>(h + static_cast<size_t>(row) * D);
   const float4* g4 = reinterpret_cast<const float4*>(g);
-  uint2* ur = reinterpret_cast<uint2*>(u + static_cast<size_t>(row) * D);
+  void* ur = static_cast<uint8_t*>(u) + static_cast<size_t>(row) * D * (F8 ? 1 : 2);
   const float inv_d = 1.0f / static_cast<float>(D);
   switch (D / 128) {  // chunks of 128 elements per lane-row
-    case 2: rmsnorm_row<2>(hr, g4, lane, inv_d, eps, ur); break;
-    case 4: rmsnorm_row<4>(hr, g4, lane, inv_d, eps, ur); break;
-    case 8: rmsnorm_row<8>(hr, g4, lane, inv_d, eps, ur); break;
-    case 12: rmsnorm_row<12>(hr, g4, lane, inv_d, eps, ur); break;
-    case 16: rmsnorm_row<16>(hr, g4, lane, inv_d, eps, ur); break;
+    case 2: rmsnorm_row<2, F8>(hr, g4, lane, inv_d, eps, ur, oscale); break;
+    case 4: rmsnorm_row<4, F8>(hr, g4, lane, inv_d, eps, ur, oscale); break;
+    case 8: rmsnorm_row<8, F8>(hr, g4, lane, inv_d, eps, ur, oscale); break;
+    case 12: rmsnorm_row<12, F8>(hr, g4, lane, inv_d, eps, ur, oscale); break;
+    case 16: rmsnorm_row<16, F8>(hr, g4, lane, inv_d, eps, ur, oscale); break;
     default: {  // any other multiple of 128: two passes
       float ss = 0.f;
       for (int c = lane; c < D / 4; c += 32) {
@@ -81,8 +91,14 @@ __global__ void rmsnorm_kernel(const float* __restrict__ h, const float* __restr
       for (int c = lane; c < D / 4; c += 32) {
         const float4 v = hr[c];
         const float4 gg = g4[c];
-        ur[c] = make_uint2(pack_bf16x2(v.x * r * gg.x, v.y * r * gg.y),
-                           pack_bf16x2(v.z * r * gg.z, v.w * r * gg.w));
+        const float y0 = v.x * r * gg.x, y1 = v.y * r * gg.y;
+        const float y2 = v.z * r * gg.z, y3 = v.w * r * gg.w;
+        if (F8) {
+          reinterpret_cast<uint32_t*>(ur)[c] =
+              pack_e4m3x4(y0 * oscale, y1 * oscale, y2 * oscale, y3 * oscale);
+        } else {
+          reinterpret_cast<uint2*>(ur)[c] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
+        }
       }
     }
   }
@@ -205,7 +221,14 @@ cudaError_t launch_unshuffle(const float* z, int C, int H, int W, int p, __nv_bf
 
 cudaError_t launch_rmsnorm(const float* h, const float* g, int M, int D, float eps,
                            __nv_bfloat16* u, cudaStream_t s) {
-  return launch_pdl(rmsnorm_kernel, dim3((M + 7) / 8), dim3(256), 0, s, h, g, M, D, eps, u);
+  return launch_pdl(rmsnorm_kernel<false>, dim3((M + 7) / 8), dim3(256), 0, s, h, g, M, D, eps,
+                    static_cast<void*>(u), 1.0f);
+}
+
+cudaError_t launch_rmsnorm_e4m3(const float* h, const float* g, int M, int D, float eps,
+                                uint8_t* u, float oscale, cudaStream_t s) {
+  return launch_pdl(rmsnorm_kernel<true>, dim3((M + 7) / 8), dim3(256), 0, s, h, g, M, D, eps,
+                    static_cast<void*>(u), oscale);
 }
 
 cudaError_t launch_pixel_head(const float* F, int frames, int gh, int gw, int C, int rs,

@@ -79,7 +79,22 @@ bool tmap_nd(CUtensorMap* m, CUtensorMapDataType dt, int rank, const void* base,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// e4m3 K-major operand [outer][inner] bytes in boxes of 128 bytes x box_outer rows
+bool tmap_e4m3(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+               uint64_t row_bytes, uint32_t box_outer) {
+  const uint64_t dims[2] = {inner, outer}, strides[1] = {row_bytes};
+  const uint32_t box[2] = {128, box_outer};
+  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, base, dims, strides, box,
+                 CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
 // GEMM epilogue store maps (32-row slabs)
+bool tmap_out_e4m3(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t ld) {
+  const uint64_t dims[2] = {cols, rows}, strides[1] = {ld};
+  const uint32_t box[2] = {128, 32};
+  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, base, dims, strides, box,
+                 CU_TENSOR_MAP_SWIZZLE_128B);
+}
 bool tmap_out_f32(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t ld) {
   const uint64_t dims[2] = {cols, rows}, strides[1] = {ld * 4};
   const uint32_t box[2] = {32, 32};
@@ -1354,6 +1369,50 @@ fd_status fd_op_rmsnorm(const float* h, const float* g, int M, int D, float eps,
   if (st) return st;
   return launch_ok(fd::launch_rmsnorm(h, g, M, D, eps, static_cast<__nv_bfloat16*>(u),
                                       static_cast<cudaStream_t>(stream)));
+}
+
+fd_status fd_op_rmsnorm_e4m3(const float* h, const float* g, int M, int D, float eps,
+                             float out_scale, void* u, void* stream) {
+  if (!h || !g || !u || M < 1 || D < 128 || D % 128 || !aligned16(h) || !aligned16(g) ||
+      !aligned16(u) || !(out_scale > 0.f))
+    return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  return launch_ok(fd::launch_rmsnorm_e4m3(h, g, M, D, eps, static_cast<uint8_t*>(u), out_scale,
+                                           static_cast<cudaStream_t>(stream)));
+}
+
+fd_status fd_op_linear_e4m3(int epilogue, int M, int N, int K, const void* A, const void* W,
+                            const float* col_scale, const float* bias, void* out,
+                            float out_scale, int bn, int* err_dev, void* stream) {
+  if (M < 1 || N < 1 || K < 16 || !A || !W || !col_scale || !bias || !out || !err_dev)
+    return FD_ERR_INVALID_ARG;
+  if (N % 32 || K % 16 || !aligned16(A) || !aligned16(W) || !aligned16(out))
+    return FD_ERR_INVALID_ARG;
+  if (epilogue != FD_EPI_F32 && epilogue != FD_EPI_RESID && epilogue != FD_EPI_GELU)
+    return FD_ERR_INVALID_ARG;
+  const bool f8_out = epilogue == FD_EPI_GELU;
+  if (f8_out && (N % 128 || !(out_scale > 0.f))) return FD_ERR_INVALID_ARG;
+  const int epi = f8_out ? fd::EPI_GELU_F8 : epilogue;
+  if (bn == 0) bn = pick_bn_step(M, N, f8_out ? 128 : 32);
+  if (!fd::gemm_bn_supported(bn) || !fd::gemm_bn_fits_epilogue(bn, epi))
+    return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  CUtensorMap ta, tb, to;
+  if (!tmap_e4m3(&ta, A, K, M, K, 128) || !tmap_e4m3(&tb, W, K, N, K, bn)) return FD_ERR_CUDA;
+  if (!(f8_out ? tmap_out_e4m3(&to, out, N, M, N) : tmap_out_f32(&to, out, N, M, N)))
+    return FD_ERR_CUDA;
+  fd::GemmParams p{};
+  p.M = M; p.N = N; p.K = K; p.epi = epi; p.bias = bias; p.err = err_dev;
+  p.fp8 = 1;
+  p.col_scale = col_scale;
+  p.out_scale = out_scale;
+  if (f8_out) p.out_f8 = static_cast<uint8_t*>(out);
+  else p.out_f32 = static_cast<float*>(out);
+  p.ld_out = N;
+  return launch_ok(fd::launch_gemm(ta, tb, to, to, to, p, bn, num_sms(),
+                                   static_cast<cudaStream_t>(stream)));
 }
 
 fd_status fd_op_unshuffle(const float* z, int C, int H, int W, int p, void* x0, void* stream) {

@@ -79,6 +79,8 @@ _SIGS = {
     "fd_op_attention_static": (_I, [_I, _I, _I, _P, _P, _P, _I, _I, _P, _I, _P, _P]),
     "fd_op_kv_append": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _P, _P]),
     "fd_op_rmsnorm": (_I, [_P, _P, _I, _I, _F, _P, _P]),
+    "fd_op_rmsnorm_e4m3": (_I, [_P, _P, _I, _I, _F, _F, _P, _P]),
+    "fd_op_linear_e4m3": (_I, [_I, _I, _I, _I, _P, _P, _P, _P, _P, _F, _I, _P, _P]),
     "fd_op_unshuffle": (_I, [_P, _I, _I, _I, _I, _P, _P]),
     "fd_op_pixel_head": (_I, [_P, _I, _I, _I, _I, _I, _I, _P, _P]),
 }
@@ -338,6 +340,23 @@ def op_rmsnorm(h, g, eps, u, stream=None) -> None:
     M, D = h.shape
     _check(lib().fd_op_rmsnorm(_ptr(h), _ptr(g), M, D, eps, _ptr(u), _stream_ptr(stream)),
            "fd_op_rmsnorm")
+
+
+def op_rmsnorm_e4m3(h, g, eps, out_scale, u, stream=None) -> None:
+    """u (uint8 tensor holding e4m3 codes) = e4m3(RMSNorm(h) g out_scale)."""
+    M, D = h.shape
+    _check(lib().fd_op_rmsnorm_e4m3(_ptr(h), _ptr(g), M, D, eps, out_scale, _ptr(u),
+                                    _stream_ptr(stream)), "fd_op_rmsnorm_e4m3")
+
+
+def op_linear_e4m3(epi, A, W, col_scale, bias, out, out_scale=1.0, bn=0, err=None,
+                   stream=None) -> None:
+    """FP8 linear: A [M][K], W [N][K] e4m3 codes (uint8 tensors), fp32 col_scale / bias."""
+    M, K = A.shape
+    N = W.shape[0]
+    _check(lib().fd_op_linear_e4m3(epi, M, N, K, _ptr(A), _ptr(W), _ptr(col_scale), _ptr(bias),
+                                   _ptr(out), out_scale, bn, _ptr(err), _stream_ptr(stream)),
+           "fd_op_linear_e4m3")
 
 
 def op_unshuffle(z, p, x0, stream=None) -> None:

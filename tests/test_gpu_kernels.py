@@ -84,6 +84,77 @@ def test_linear_swiglu(M, Dm, K, bn):
     assert_close_scaled(out.float(), want, 8e-3, "swiglu")
 
 
+def e4m3_codes(x):
+    """fp64 values -> (e4m3 codes as uint8, the values they stand for)."""
+    q = torch.as_tensor(x, dtype=torch.float64).to(torch.float8_e4m3fn)
+    return q.view(torch.uint8), q.to(torch.float64)
+
+
+def assert_e4m3_close(got_codes, want_values, what):
+    """e4m3 outputs computed in fp32 (GPU) vs fp64 (oracle): equal codes except where the exact
+    value sits at a rounding boundary, and then one step apart (relative 2^-3, or one
+    subnormal step)."""
+    got = got_codes.cpu().view(torch.float8_e4m3fn).to(torch.float64)
+    want = want_values.to(torch.float8_e4m3fn).to(torch.float64)
+    diff = (got - want).abs()
+    assert float((diff > 0).double().mean()) < 0.01, f"{what}: too many codes differ"
+    assert bool((diff <= 2.0 ** -3 * want.abs() + 2.0 ** -9).all()), f"{what}: more than a step"
+
+
+@pytest.mark.parametrize("M,N,K,bn", [
+    (520, 1024, 256, 0),     # ragged M, library tile choice
+    (1560, 1024, 4096, 96),  # 480p MLP-down shape, 96-wide tiles, 32 K-blocks of 128
+    (300, 640, 208, 128),    # K not a multiple of 128: zero-filled K tail
+])
+def test_linear_e4m3_fp32_epilogues(M, N, K, bn):
+    """FP8 MLP products (Sec. 4.6): e4m3 operands make every product exact, so the fp32 and
+    residual epilogues match the oracle's dequantised matrix product to fp32 accumulation."""
+    torch.manual_seed(M + N + K)
+    a_c, a = e4m3_codes(torch.randn(M, K, dtype=torch.float64) * 3)
+    w_c, wv = e4m3_codes(torch.randn(N, K, dtype=torch.float64) * 40)
+    cs = torch.tensor([2.0 ** -int(e) for e in torch.randint(4, 12, (N,))], dtype=torch.float32)
+    b = torch.randn(N, dtype=torch.float32) * 0.1
+    want = oracle.linear(a, wv, None) * cs.double() + b.double()
+    err = err_word()
+    out = torch.zeros(M, N, device="cuda")
+    fdp.op_linear_e4m3(fdp.EPI_F32, a_c.cuda(), w_c.cuda(), cs.cuda(), b.cuda(), out, bn=bn,
+                       err=err)
+    check_err(err)
+    assert_close_scaled(out, want, 2e-5, "e4m3 linear f32")
+    h0 = torch.randn(M, N, dtype=torch.float32)
+    h = h0.cuda()
+    fdp.op_linear_e4m3(fdp.EPI_RESID, a_c.cuda(), w_c.cuda(), cs.cuda(), b.cuda(), h, bn=bn,
+                       err=err)
+    check_err(err)
+    assert_close_scaled(h, h0.double() + want, 2e-5, "e4m3 linear residual")
+
+
+def test_linear_e4m3_gelu_to_e4m3_and_rmsnorm_e4m3():
+    """The two FP8 producers of the MLP: GELU epilogue to e4m3 (layer 1 output) and RMSNorm to
+    e4m3 (layer 1 input), each against the oracle's rounding of the same formula."""
+    M, N, K = 520, 1024, 512
+    torch.manual_seed(5)
+    a_c, a = e4m3_codes(torch.randn(M, K, dtype=torch.float64) * 2)
+    w_c, wv = e4m3_codes(torch.randn(N, K, dtype=torch.float64) * 30)
+    cs = torch.full((N,), 2.0 ** -10, dtype=torch.float32)
+    b = torch.randn(N, dtype=torch.float32) * 0.1
+    z = oracle.linear(a, wv, None) * cs.double() + b.double()
+    for bn in (128, 256):
+        out = torch.zeros(M, N, dtype=torch.uint8, device="cuda")
+        err = err_word()
+        fdp.op_linear_e4m3(fdp.EPI_GELU, a_c.cuda(), w_c.cuda(), cs.cuda(), b.cuda(), out,
+                           out_scale=32.0, bn=bn, err=err)
+        check_err(err)
+        assert_e4m3_close(out, oracle.gelu(z) * 32.0, f"gelu e4m3 bn={bn}")
+    D = 1024
+    h = torch.from_numpy(randn((M, D), 9, 2.0))
+    g = torch.from_numpy(bf16_values(1 + randn((D,), 10, 0.1)))
+    u = torch.zeros(M, D, dtype=torch.uint8, device="cuda")
+    fdp.op_rmsnorm_e4m3(h.cuda(), g.cuda(), 1e-6, 8.0, u)
+    torch.cuda.synchronize()
+    assert_e4m3_close(u, oracle.rms_norm(h.double(), g.double(), 1e-6) * 8.0, "rmsnorm e4m3")
+
+
 def test_linear_resid_gelu_tup():
     M, N, K, D = 520, 1024, 256, 256
     A, W, b = linear_case(M, N, K, seed=11)
