@@ -73,6 +73,13 @@ typedef struct {
   int32_t qk_norm;         /* per-head RMSNorm on: 0 = K and V (KV-norm, Sec. 3.2); *
                             * 1 = Q and K (QK-norm); the blob's second D_h gain is  *
                             * then Q's                                              */
+  int32_t mlp_fp8;         /* 1: both products of every block MLP in FP8 (Sec. 4.6, *
+                            * "static-calibrated FP8 quantization"): e4m3 weights   *
+                            * with a power-of-two scale per row, e4m3 activations   *
+                            * with static power-of-two scales derived from the      *
+                            * weights at fd_weights_create (bounds that no input    *
+                            * can exceed), fp32 accumulation. Needs mlp_gated = 0.  *
+                            * The blob is unchanged.                                */
 } fd_config;
 
 typedef struct fd_weights_s* fd_weights;

@@ -3,6 +3,7 @@
 // descriptors, and the per-chunk kernel sequence of Algorithm 1.
 #include <cuda.h>
 #include <cudaTypedefs.h>
+#include <cuda_fp8.h>
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -163,6 +164,7 @@ struct Dims {
   bool u8;
   bool gated;  // gated-SiLU MLP: layer 1 has 2 Mr D outputs (gate, up)
   bool qk;     // QK-norm instead of KV-norm
+  bool fp8;    // block MLPs in FP8 (e4m3 operands, static scales)
 };
 
 bool valid_cfg(const fd_config* c) {
@@ -181,6 +183,8 @@ bool valid_cfg(const fd_config* c) {
   if (c->out_dtype != FD_DTYPE_F32 && c->out_dtype != FD_DTYPE_U8) return false;
   if (c->mlp_gated != 0 && c->mlp_gated != 1) return false;
   if (c->qk_norm != 0 && c->qk_norm != 1) return false;
+  if (c->mlp_fp8 != 0 && c->mlp_fp8 != 1) return false;
+  if (c->mlp_fp8 == 1 && c->mlp_gated == 1) return false;  // FP8 gated MLP not built
   if (!(c->norm_eps >= 0.f) || !(c->rope_base > 1.f)) return false;
   const long long L = static_cast<long long>(c->latent_h / c->patch) * (c->latent_w / c->patch);
   if (L * c->r_t * c->window > (1LL << 26)) return false;
@@ -198,6 +202,7 @@ Dims dims_of(const fd_config* c) {
   d.u8 = c->out_dtype == FD_DTYPE_U8;
   d.gated = c->mlp_gated == 1;
   d.qk = c->qk_norm == 1;
+  d.fp8 = c->mlp_fp8 == 1;
   return d;
 }
 
@@ -208,7 +213,8 @@ bool same_cfg(const fd_config* a, const fd_config* b) {
 // blob element counts, in blob order
 struct BlobEntry {
   size_t elems;
-  int kind;          // 0 weight (bf16 on device), 1 fp32
+  int kind;          // 0 weight (bf16 on device), 1 fp32, 2 weight (e4m3 on device, one
+                     // power-of-two scale per row of row_len elements)
   size_t gate_rows;  // > 0: gated MLP layer 1 (gate rows, then as many up rows) whose rows the
   size_t row_len;    // device copy interleaves in blocks of 32 (see gated_row)
 };
@@ -223,10 +229,18 @@ void blob_layout(const Dims& d, std::vector<BlobEntry>& out) {
     if (d.gated) {
       out.push_back({2 * Dm * D, 0, Dm, D});
       out.push_back({2 * Dm, 1, Dm, 1});
+    } else if (d.fp8) {
+      out.push_back({Dm * D, 2, 0, D});
+      F(Dm);
     } else {
       W(Dm * D); F(Dm);
     }
-    W(D * Dm); F(D);
+    if (d.fp8) {
+      out.push_back({D * Dm, 2, 0, Dm});
+    } else {
+      W(D * Dm);
+    }
+    F(D);
   };
   for (int b = 0; b < d.nb; ++b) block();
   F(D); W(static_cast<size_t>(d.rt) * D * D); F(static_cast<size_t>(d.rt) * D);
@@ -239,6 +253,22 @@ void blob_layout(const Dims& d, std::vector<BlobEntry>& out) {
 size_t gated_row(size_t r, size_t gate) {
   const size_t u = r < gate ? r : r - gate;
   return (u / 32) * 64 + (r < gate ? 0 : 32) + u % 32;
+}
+
+// smallest power of two >= x (x > 0), exactly
+double pow2_ceil(double x) {
+  int e = 0;
+  const double m = std::frexp(x, &e);  // x = m 2^e, 0.5 <= m < 1
+  return m == 0.5 ? std::ldexp(1.0, e - 1) : std::ldexp(1.0, e);
+}
+
+// value of an FP8 E4M3 code (OCP: sign, 4 exponent bits with bias 7, 3 mantissa bits;
+// exponent 0 = subnormal, steps of 2^-9); the NaN codes never occur here
+double e4m3_value(uint8_t c) {
+  const int e = (c >> 3) & 15, m = c & 7;
+  const double v = e == 0 ? std::ldexp(static_cast<double>(m), -9)
+                          : std::ldexp(1.0 + m / 8.0, e - 7);
+  return (c & 0x80) ? -v : v;
 }
 
 uint16_t f32_to_bf16_rne(float f) {
@@ -287,6 +317,10 @@ struct Linear {
 struct LayerW {
   float *g1 = nullptr, *g2 = nullptr, *kg = nullptr, *vg = nullptr;
   Linear qkv, out, mlp1, mlp2;
+  // FP8 MLP (mlp1 / mlp2 weights are e4m3): per-column dequantisation scales of the two
+  // products and the reciprocal activation scales 1 / s_u, 1 / s_h
+  float *cs1 = nullptr, *cs2 = nullptr;
+  float inv_su = 1.f, inv_sh = 1.f;
 };
 
 }  // namespace
@@ -342,6 +376,8 @@ struct fd_handle_s {
   CUtensorMap tm_q8B, tm_q8R;  // attention Q in 8-row boxes (tiles across two heads)
   // epilogue store descriptors
   CUtensorMap so_h, so_hf, so_tup, so_hidB, so_hidR, so_hidH, so_F, so_qB, so_qR;
+  // FP8 MLP: e4m3 views of u (MLP input) and hid (MLP hidden), A operands and store map
+  CUtensorMap tm_u8B, tm_u8R, tm_hid8B, tm_hid8R, so_hid8B, so_hid8R;
   // host-buffer decode: library-owned device copies of the latent and the pixels
   float* latent_buf = nullptr;
   void* pixel_buf = nullptr;
@@ -487,6 +523,33 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
   po.out_f32 = hbuf;
   po.ld_out = d.D;
   if ((st = run_linear(h, FD_K_OUT, tm_o, lw.out, rows, po, so_h, s))) return st;
+  if (d.fp8) {
+    // FP8 MLP (Sec. 4.6): u8 = e4m3(RMSNorm(h) g / s_u); hid8 = e4m3(GELU(u8 W1 s_u s_w1 + b1)
+    // / s_h); h += hid8 W2 s_h s_w2 + b2
+    const float* gain = lw.g2;
+    const float eps = h->cfg.norm_eps, inv_su = lw.inv_su;
+    uint8_t* u8 = reinterpret_cast<uint8_t*>(h->u);
+    const int D = d.D;
+    if ((st = traced(h, FD_K_RMSNORM, s, [&] {
+           return fd::launch_rmsnorm_e4m3(hbuf, gain, rows, D, eps, u8, inv_su, s);
+         })))
+      return st;
+    fd::GemmParams p1{};
+    p1.epi = fd::EPI_GELU_F8;
+    p1.fp8 = 1;
+    p1.col_scale = lw.cs1;
+    p1.out_scale = lw.inv_sh;
+    p1.out_f8 = reinterpret_cast<uint8_t*>(h->hid);
+    p1.ld_out = d.Mr * d.D;
+    if ((st = run_linear(h, FD_K_MLP1, refine ? h->tm_u8R : h->tm_u8B, lw.mlp1, rows, p1,
+                         refine ? h->so_hid8R : h->so_hid8B, s)))
+      return st;
+    fd::GemmParams p2 = po;
+    p2.fp8 = 1;
+    p2.col_scale = lw.cs2;
+    return run_linear(h, FD_K_MLP2, refine ? h->tm_hid8R : h->tm_hid8B, lw.mlp2, rows, p2, so_h,
+                      s);
+  }
   if ((st = run_norm(h, hbuf, lw.g2, rows, s))) return st;
   fd::GemmParams p1{};
   p1.epi = d.gated ? fd::EPI_SWIGLU : fd::EPI_GELU;
@@ -661,33 +724,69 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
   const Dims d = dims_of(cfg);
   std::vector<BlobEntry> layout;
   blob_layout(d, layout);
-  // device arena: bf16 weights then fp32 vectors, each 256-byte aligned
+  // device arena: bf16 (or e4m3) weights and fp32 vectors in blob order, each 256-byte
+  // aligned, then the FP8 column scales of every block (FP8 MLPs only)
   std::vector<size_t> doff(layout.size());
   size_t cur = 0;
   for (size_t i = 0; i < layout.size(); ++i) {
     doff[i] = cur;
-    cur = align_up(cur + layout[i].elems * (layout[i].kind == 0 ? 2 : 4), 256);
+    const size_t esz_dev = layout[i].kind == 0 ? 2 : (layout[i].kind == 1 ? 4 : 1);
+    cur = align_up(cur + layout[i].elems * esz_dev, 256);
   }
+  const size_t Dm = static_cast<size_t>(d.Mr) * d.D;
+  const size_t fp8_cs_bytes = align_up((Dm + d.D) * 4, 256);  // per block: mlp1, mlp2 scales
+  const size_t fp8_off = cur;
+  if (d.fp8) cur += static_cast<size_t>(d.nb + d.nr) * fp8_cs_bytes;
   std::vector<uint8_t> stage;
+  std::vector<std::vector<double>> row_scale(layout.size()), row_norm(layout.size());
   try {
     stage.assign(cur, 0);
   } catch (...) {
     return FD_ERR_OOM;
   }
+  auto blob_value = [&](size_t i) -> float {
+    float f;
+    if (blob_dtype == FD_DTYPE_F32) {
+      std::memcpy(&f, static_cast<const uint8_t*>(host_blob) + 4 * i, 4);
+    } else {
+      uint16_t b;
+      std::memcpy(&b, static_cast<const uint8_t*>(host_blob) + 2 * i, 2);
+      f = bf16_to_f32(b);
+    }
+    return f;
+  };
   size_t src = 0;
   for (size_t i = 0; i < layout.size(); ++i) {
     const BlobEntry& e = layout[i];
+    if (e.kind == 2) {
+      // FP8 weight (Sec. 4.6): per row, s = 2^ceil(log2(max|w| / 448)) and code = e4m3(w / s)
+      // (round to nearest even; |w / s| <= 448, so nothing saturates). Keeps s and the norm of
+      // the dequantised row for the static activation scales.
+      const size_t rows = e.elems / e.row_len;
+      row_scale[i].resize(rows);
+      row_norm[i].resize(rows);
+      for (size_t r = 0; r < rows; ++r, src += e.row_len) {
+        double amax = 0.0;
+        for (size_t k = 0; k < e.row_len; ++k)
+          amax = std::fmax(amax, std::fabs(static_cast<double>(blob_value(src + k))));
+        const double sc = amax > 0.0 ? pow2_ceil(amax / 448.0) : 1.0;
+        double ss = 0.0;
+        for (size_t k = 0; k < e.row_len; ++k) {
+          const float x = static_cast<float>(static_cast<double>(blob_value(src + k)) / sc);
+          const uint8_t code = __nv_cvt_float_to_fp8(x, __NV_SATFINITE, __NV_E4M3);
+          stage[doff[i] + r * e.row_len + k] = code;
+          const double dq = e4m3_value(code) * sc;
+          ss += dq * dq;
+        }
+        row_scale[i][r] = sc;
+        row_norm[i][r] = std::sqrt(ss);
+      }
+      continue;
+    }
     for (size_t k0 = 0; k0 < e.elems; ++k0, ++src) {
       const size_t k =
           e.gate_rows ? gated_row(k0 / e.row_len, e.gate_rows) * e.row_len + k0 % e.row_len : k0;
-      float f;
-      if (blob_dtype == FD_DTYPE_F32) {
-        std::memcpy(&f, static_cast<const uint8_t*>(host_blob) + 4 * src, 4);
-      } else {
-        uint16_t b;
-        std::memcpy(&b, static_cast<const uint8_t*>(host_blob) + 2 * src, 2);
-        f = bf16_to_f32(b);
-      }
+      const float f = blob_value(src);
       if (layout[i].kind == 0) {
         const uint16_t b = f32_to_bf16_rne(f);
         std::memcpy(&stage[doff[i] + 2 * k], &b, 2);
@@ -704,14 +803,11 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
     delete w;
     return FD_ERR_OOM;
   }
-  if (cudaMemcpy(w->arena, stage.data(), cur, cudaMemcpyHostToDevice) != cudaSuccess) {
-    cudaFree(w->arena);
-    delete w;
-    return FD_ERR_CUDA;
-  }
   uint8_t* base = static_cast<uint8_t*>(w->arena);
   size_t idx = 0;
   auto next = [&]() { return base + doff[idx++]; };
+  auto host_f32 = [&](size_t entry) { return reinterpret_cast<const float*>(&stage[doff[entry]]); };
+  int fp8_block = 0;
   // fp32_epi: the layer's epilogue stores fp32 (patch-embed, out-projection, MLP down, temporal
   // upsampling, head layer 2), which allows the narrower 96-wide tiles
   auto linear = [&](Linear& lin, int N, int K, int M, bool fp32_epi) -> bool {
@@ -722,6 +818,15 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
     lin.bn = pick_bn(M, N, fp32_epi);
     return tmap_bf16(&lin.tm, lin.w, K, N, static_cast<uint64_t>(K) * 2, fd::kBK, lin.bn);
   };
+  // FP8 linear: e4m3 weight [N][K] in boxes of 128 bytes (= 128 K elements)
+  auto linear_e4m3 = [&](Linear& lin, int N, int K, int M, int step) -> bool {
+    lin.w = reinterpret_cast<__nv_bfloat16*>(next());
+    lin.b = reinterpret_cast<float*>(next());
+    lin.N = N;
+    lin.K = K;
+    lin.bn = pick_bn_step(M, N, step);
+    return tmap_e4m3(&lin.tm, lin.w, K, N, K, lin.bn);
+  };
   bool ok = linear(w->embed, d.D, d.cin, d.L, true);
   auto block = [&](LayerW& lw, int M) {
     lw.g1 = reinterpret_cast<float*>(next());
@@ -729,7 +834,37 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
     lw.kg = reinterpret_cast<float*>(next());
     lw.vg = reinterpret_cast<float*>(next());
     ok = ok && linear(lw.out, d.D, d.N * kHeadDim, M, true);
+    const size_t e_g2 = idx;
     lw.g2 = reinterpret_cast<float*>(next());
+    if (d.fp8) {
+      // Static scales (Sec. 4.6 "static-calibrated"), from bounds no input can exceed:
+      //   u = RMSNorm(h) g has |u_i| <= sqrt(D) max|g|          -> s_u = 2^ceil(log2(./448))
+      //   |GELU(z_j)| <= max(1, |z_j|) and |z_j| <= 1.125 sqrt(D) max|g| ||w1_j|| + |b1_j|
+      //   (with the e4m3 rounding of u, at most 1 + 2^-3)         -> s_h likewise
+      // Columns are dequantised by s_u s_w1[n] (layer 1) and s_h s_w2[n] (layer 2).
+      const size_t e_w1 = idx, e_b1 = idx + 1, e_w2 = idx + 2;
+      ok = ok && linear_e4m3(lw.mlp1, static_cast<int>(Dm), d.D, M, 128);
+      ok = ok && linear_e4m3(lw.mlp2, d.D, static_cast<int>(Dm), M, 32);
+      const float* g2 = host_f32(e_g2);
+      const float* b1 = host_f32(e_b1);
+      double gmax = 0.0;
+      for (int i = 0; i < d.D; ++i) gmax = std::fmax(gmax, std::fabs(static_cast<double>(g2[i])));
+      const double sq = std::sqrt(static_cast<double>(d.D));
+      const double s_u = pow2_ceil(sq * gmax / 448.0);
+      double bz = 0.0;
+      for (size_t j = 0; j < Dm; ++j)
+        bz = std::fmax(bz, 1.125 * sq * gmax * row_norm[e_w1][j] + std::fabs(double(b1[j])));
+      const double s_h = pow2_ceil(std::fmax(bz, 1.0) / 448.0);
+      const size_t off = fp8_off + static_cast<size_t>(fp8_block++) * fp8_cs_bytes;
+      float* cs = reinterpret_cast<float*>(&stage[off]);
+      for (size_t n = 0; n < Dm; ++n) cs[n] = static_cast<float>(s_u * row_scale[e_w1][n]);
+      for (int n = 0; n < d.D; ++n) cs[Dm + n] = static_cast<float>(s_h * row_scale[e_w2][n]);
+      lw.cs1 = reinterpret_cast<float*>(base + off);
+      lw.cs2 = lw.cs1 + Dm;
+      lw.inv_su = static_cast<float>(1.0 / s_u);
+      lw.inv_sh = static_cast<float>(1.0 / s_h);
+      return;
+    }
     ok = ok && linear(lw.mlp1, (d.gated ? 2 : 1) * d.Mr * d.D, d.D, M, false);
     if (d.gated) {  // EPI_SWIGLU works on 128-column steps
       lw.mlp1.bn = pick_bn_step(M, lw.mlp1.N, 128);
@@ -747,7 +882,8 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
   w->g_h = reinterpret_cast<float*>(next());
   ok = ok && linear(w->head1, d.D, d.D, d.rt * d.L, false);
   ok = ok && linear(w->head2, d.head_out, d.D, d.rt * d.L, true);
-  if (!ok || idx != layout.size()) {
+  if (!ok || idx != layout.size() ||
+      cudaMemcpy(w->arena, stage.data(), cur, cudaMemcpyHostToDevice) != cudaSuccess) {
     cudaFree(w->arena);
     delete w;
     return FD_ERR_CUDA;
@@ -853,6 +989,14 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   ok = ok && tmap_out_f32(&h->so_F, h->F, d.head_out, R, d.head_out);
   ok = ok && tmap_out_bf16(&h->so_qB, h->q, NQ, d.L, NQ);
   ok = ok && tmap_out_bf16(&h->so_qR, h->q, NQ, R, NQ);
+  if (d.fp8) {
+    ok = ok && tmap_e4m3(&h->tm_u8B, h->u, d.D, d.L, d.D, 128);
+    ok = ok && tmap_e4m3(&h->tm_u8R, h->u, d.D, R, d.D, 128);
+    ok = ok && tmap_e4m3(&h->tm_hid8B, h->hid, Dm, d.L, Dm, 128);
+    ok = ok && tmap_e4m3(&h->tm_hid8R, h->hid, Dm, R, Dm, 128);
+    ok = ok && tmap_out_e4m3(&h->so_hid8B, h->hid, Dm, d.L, Dm);
+    ok = ok && tmap_out_e4m3(&h->so_hid8R, h->hid, Dm, R, Dm);
+  }
   if (!ok || cudaMemset(h->arena, 0, h->arena_bytes) != cudaSuccess ||
       cudaDeviceSynchronize() != cudaSuccess) {
     cudaFree(h->arena);
