@@ -33,8 +33,8 @@ typedef enum {
 /* Linear layer on the tensor cores (tcgen05, bf16 in, fp32 accumulate).
  * A bf16 [M][K] row-major; W bf16 [N][K] row-major (nn.Linear); bias fp32 [N].
  * Requires N % 32 == 0 (N % 64 == 0 for FD_EPI_GELU, N % 128 == 0 for FD_EPI_SWIGLU),
- * K % 8 == 0, 16-byte aligned A / W / out. bn = output tile width (64, 96, 128, 192 or 256;
- * 96 only for the fp32 epilogues, 128 or 256 for FD_EPI_SWIGLU; 0 = library choice). */
+ * K % 8 == 0, 16-byte aligned A / W / out / bias. bn = output tile width (64, 96, 128, 192
+ * or 256; 96 only for the fp32 epilogues, 128 or 256 for FD_EPI_SWIGLU; 0 = library choice). */
 fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const void* W,
                        const float* bias, void* out, int tup_hidden, int bn, int* err_dev,
                        void* stream);
@@ -55,7 +55,8 @@ fd_status fd_op_rope_table(int t, int frames_per_chunk, float rope_base, float* 
  *           in a grid of width grid_w (rope_base; bands 24/20/20 dims)
  *   q_out bf16 [M][heads*64];  K -> k_ring bf16 [groups][ring_pitch][64] rows
  *   (t mod window)*M + row;  V -> vt_ring fp16 [groups][64][ring_pitch] (transposed), same
- *   key index.  M = frames_per_chunk * tokens; ring_pitch % 128 == 0, >= window * M. */
+ *   key index.  M = frames_per_chunk * tokens; ring_pitch % 128 == 0, >= window * M;
+ *   bqkv, q_out and the rings 16-byte aligned. */
 fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* bqkv,
                     const float* knorm_g, const float* norm2_g, int qk_norm, int heads, int groups,
                     int tokens, int grid_w, int frames_per_chunk, int window, int t, float eps,
@@ -126,7 +127,8 @@ fd_status fd_op_rmsnorm_e4m3(const float* h, const float* g, int M, int D, float
  *   FD_EPI_F32    out fp32 [M][N]  = acc * col_scale + bias
  *   FD_EPI_RESID  out fp32 [M][N] += acc * col_scale + bias
  *   FD_EPI_GELU   out e4m3 [M][N]  = e4m3(GELU(acc * col_scale + bias) * out_scale)
- * K % 16 == 0, N % 32 == 0 (N % 128 == 0 for FD_EPI_GELU), 16-byte aligned A / W / out.
+ * K % 16 == 0, N % 32 == 0 (N % 128 == 0 for FD_EPI_GELU), 16-byte aligned A / W / out /
+ * bias / col_scale.
  * bn = output tile width (96 / 128 / 192 / 256, 128 or 256 for FD_EPI_GELU; 0 = choice). */
 fd_status fd_op_linear_e4m3(int epilogue, int M, int N, int K, const void* A, const void* W,
                             const float* col_scale, const float* bias, void* out,

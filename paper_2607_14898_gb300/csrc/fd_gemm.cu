@@ -53,8 +53,39 @@ __device__ __forceinline__ void put_row_sw128(uint8_t* buf, int row, const uint3
         make_uint4(w[4 * k], w[4 * k + 1], w[4 * k + 2], w[4 * k + 3]);
 }
 
+// 1 + erf(a), after Abramowitz & Stegun, Handbook of Mathematical Functions, formula 7.1.26:
+// for b = |a|, erf(b) = 1 - (a1 t + a2 t^2 + a3 t^3 + a4 t^4 + a5 t^5) e^(-b^2) with
+// t = 1 / (1 + p b), absolute error at most 1.5e-7. With E = the polynomial times e^(-b^2),
+// 1 + erf(a) = 2 - E for a >= 0 and E for a < 0 (erf is odd), so the negative side has no
+// cancellation. In fp32 with the hardware reciprocal and exp2 (a few ulp each) the error stays
+// near 1e-7, far below the bf16 (2^-9) and e4m3 (2^-4) rounding of the GELU outputs.
+__device__ __forceinline__ float one_plus_erf(float a) {
+  const float b = fabsf(a);
+  float t;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(t) : "f"(fmaf(0.3275911f, b, 1.0f)));
+  float y = fmaf(1.061405429f, t, -1.453152027f);
+  y = fmaf(y, t, 1.421413741f);
+  y = fmaf(y, t, -0.284496736f);
+  y = fmaf(y, t, 0.254829592f);
+  const float e = y * t * ex2_approx(-(b * b) * 1.44269504088896341f);  // erfc(b)
+  return a >= 0.f ? 2.0f - e : e;
+}
+
+// GELU, exact (erf) form: x Phi(x) = 0.5 x (1 + erf(x / sqrt 2))
 __device__ __forceinline__ float gelu_erf(float x) {
-  return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
+  return 0.5f * x * one_plus_erf(x * 0.70710678118654752f);
+}
+
+// 32 consecutive fp32 values (16-byte aligned) as eight vector loads; the same for every lane
+__device__ __forceinline__ void load32(const float* p, float (&v)[32]) {
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const float4 q = __ldg(reinterpret_cast<const float4*>(p) + k);
+    v[4 * k] = q.x;
+    v[4 * k + 1] = q.y;
+    v[4 * k + 2] = q.z;
+    v[4 * k + 3] = q.w;
+  }
 }
 
 __device__ __forceinline__ float silu(float x) { return x / (1.0f + __expf(-x)); }
@@ -123,6 +154,19 @@ __global__ void __launch_bounds__(192, 1)
     prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
   }
+  // Weights that no kernel of the stream writes (p.w_static) are loaded into the first stages
+  // while the previous kernel is still finishing; only the activations wait for it. Thread 0
+  // is the TMA producer and initialised the barriers above.
+  const int pre = (p.w_static && aligned && static_cast<int>(blockIdx.x) < tiles)
+                      ? (nk < C::kStages ? nk : C::kStages)
+                      : 0;
+  if (threadIdx.x == 0) {
+    const int n0 = (static_cast<int>(blockIdx.x) % n_tiles) * BN;
+    for (int kb = 0; kb < pre; ++kb) {
+      mbar_expect_tx(bar_full + 8 * kb, C::kStageBytes);
+      tma_load_2d(sB + kb * C::kBBytes, &tmB, bar_full + 8 * kb, kb * kel, n0);
+    }
+  }
   grid_dep_wait();  // inputs written by the previous kernel; TMEM freed by its CTAs
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
@@ -143,6 +187,10 @@ __global__ void __launch_bounds__(192, 1)
       for (int kb = 0; kb < nk; ++kb, ++it) {
         const int s = it % C::kStages;
         const uint32_t ph = (it / C::kStages) & 1;
+        if (it < pre) {  // W already on its way: the activation half of the stage
+          tma_load_2d(sA + s * C::kABytes, &tmA, bar_full + 8 * s, kb * kel, m0);
+          continue;
+        }
         if (!mbar_wait(bar_empty + 8 * s, ph ^ 1, p.err, ERR_WAIT_MMA)) { ok = false; break; }
         mbar_expect_tx(bar_full + 8 * s, C::kStageBytes);
         tma_load_2d(sA + s * C::kABytes, &tmA, bar_full + 8 * s, kb * kel, m0);
@@ -248,10 +296,15 @@ __global__ void __launch_bounds__(192, 1)
           tmem_ld_32x32b_x32(tbase + c + 32, r1);
           tmem_ld_wait();
           float v[64];
+          {
+            float b0[32], b1[32];
+            load32(p.bias + col, b0);
+            load32(p.bias + col + 32, b1);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            v[j] = __uint_as_float(r0[j]) + __ldg(p.bias + col + j);
-            v[32 + j] = __uint_as_float(r1[j]) + __ldg(p.bias + col + 32 + j);
+            for (int j = 0; j < 32; ++j) {
+              v[j] = __uint_as_float(r0[j]) + b0[j];
+              v[32 + j] = __uint_as_float(r1[j]) + b1[j];
+            }
           }
           const int hidx = col / kHeadDim;
           const bool is_q = hidx < q.heads;
@@ -317,14 +370,17 @@ __global__ void __launch_bounds__(192, 1)
           tmem_ld_32x32b_x32(tbase + c + 32, r1);
           tmem_ld_wait();
           uint32_t w[32];
+          {
+            float b0[32], b1[32];
+            load32(p.bias + col, b0);
+            load32(p.bias + col + 32, b1);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            w[j] = pack_bf16x2(gelu_erf(__uint_as_float(r0[2 * j]) + __ldg(p.bias + col + 2 * j)),
-                               gelu_erf(__uint_as_float(r0[2 * j + 1]) +
-                                        __ldg(p.bias + col + 2 * j + 1)));
-            w[16 + j] = pack_bf16x2(
-                gelu_erf(__uint_as_float(r1[2 * j]) + __ldg(p.bias + col + 32 + 2 * j)),
-                gelu_erf(__uint_as_float(r1[2 * j + 1]) + __ldg(p.bias + col + 33 + 2 * j)));
+            for (int j = 0; j < 16; ++j) {
+              w[j] = pack_bf16x2(gelu_erf(__uint_as_float(r0[2 * j]) + b0[2 * j]),
+                                 gelu_erf(__uint_as_float(r0[2 * j + 1]) + b0[2 * j + 1]));
+              w[16 + j] = pack_bf16x2(gelu_erf(__uint_as_float(r1[2 * j]) + b1[2 * j]),
+                                      gelu_erf(__uint_as_float(r1[2 * j + 1]) + b1[2 * j + 1]));
+            }
           }
           uint8_t* buf = acquire();
           put_row_sw128(buf, lane, w);
@@ -348,15 +404,16 @@ __global__ void __launch_bounds__(192, 1)
             tmem_ld_32x32b_x32(tbase + c + 32 * q4, r);
             tmem_ld_wait();
             const int cb = col + 32 * q4;
+            float cs[32], bb[32];
+            load32(p.col_scale + cb, cs);
+            load32(p.bias + cb, bb);
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
               float f[4];
 #pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const int cc = cb + 4 * j + e;
-                f[e] = gelu_erf(fmaf(__uint_as_float(r[4 * j + e]), __ldg(p.col_scale + cc),
-                                     __ldg(p.bias + cc))) * p.out_scale;
-              }
+              for (int e = 0; e < 4; ++e)
+                f[e] = gelu_erf(fmaf(__uint_as_float(r[4 * j + e]), cs[4 * j + e], bb[4 * j + e])) *
+                       p.out_scale;
               w[8 * q4 + j] = pack_e4m3x4(f[0], f[1], f[2], f[3]);
             }
           }
@@ -381,13 +438,15 @@ __global__ void __launch_bounds__(192, 1)
             tmem_ld_32x32b_x32(tbase + c + 64 * hh, rg);
             tmem_ld_32x32b_x32(tbase + c + 64 * hh + 32, ru);
             tmem_ld_wait();
-            const float* bg = p.bias + col + 64 * hh;
+            float bgv[32], buv[32];
+            load32(p.bias + col + 64 * hh, bgv);
+            load32(p.bias + col + 64 * hh + 32, buv);
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
-              const float g0 = __uint_as_float(rg[2 * j]) + __ldg(bg + 2 * j);
-              const float g1 = __uint_as_float(rg[2 * j + 1]) + __ldg(bg + 2 * j + 1);
-              const float u0 = __uint_as_float(ru[2 * j]) + __ldg(bg + 32 + 2 * j);
-              const float u1 = __uint_as_float(ru[2 * j + 1]) + __ldg(bg + 33 + 2 * j);
+              const float g0 = __uint_as_float(rg[2 * j]) + bgv[2 * j];
+              const float g1 = __uint_as_float(rg[2 * j + 1]) + bgv[2 * j + 1];
+              const float u0 = __uint_as_float(ru[2 * j]) + buv[2 * j];
+              const float u1 = __uint_as_float(ru[2 * j + 1]) + buv[2 * j + 1];
               w[16 * hh + j] = pack_bf16x2(silu(g0) * u0, silu(g1) * u1);
             }
           }
@@ -409,15 +468,17 @@ __global__ void __launch_bounds__(192, 1)
           tmem_ld_32x32b_x32(tbase + c, r);
           tmem_ld_wait();
           uint32_t w[32];
+          float bb[32];
+          load32(p.bias + col, bb);
           if (p.col_scale != nullptr) {  // FP8 operands: dequantise per column
+            float cs[32];
+            load32(p.col_scale + col, cs);
 #pragma unroll
             for (int j = 0; j < 32; ++j)
-              w[j] = __float_as_uint(fmaf(__uint_as_float(r[j]), __ldg(p.col_scale + col + j),
-                                          __ldg(p.bias + col + j)));
+              w[j] = __float_as_uint(fmaf(__uint_as_float(r[j]), cs[j], bb[j]));
           } else {
 #pragma unroll
-            for (int j = 0; j < 32; ++j)
-              w[j] = __float_as_uint(__uint_as_float(r[j]) + __ldg(p.bias + col + j));
+            for (int j = 0; j < 32; ++j) w[j] = __float_as_uint(__uint_as_float(r[j]) + bb[j]);
           }
           uint8_t* buf = acquire();
           put_row_sw128(buf, lane, w);

@@ -92,6 +92,9 @@ struct GemmParams {
   const float* col_scale;
   uint8_t* out_f8;
   float out_scale;
+  // W is never written by a kernel of the stream (the decoder's weights): its first stages may
+  // load before the dependency on the previous kernel is resolved
+  int w_static;
 };
 
 struct AttnParams {

@@ -287,8 +287,9 @@ float bf16_to_f32(uint16_t b) {
 
 // GEMM tile width for an M x N problem: a tile costs about (128 + BN) (a fixed part plus its
 // width) and a persistent grid runs ceil(tiles / SMs) rounds; pick the cheapest, the wider tile
-// on ties. Matches the measured best width on the decoder's shapes.
-int pick_bn_step(int M, int N, int step) {
+// on ties (the narrower one for epilogue-bound layers). Matches the measured best width on the
+// decoder's shapes.
+int pick_bn_step(int M, int N, int step, bool narrow_on_ties = false) {
   const int sms = num_sms();
   int best = 128;
   long long best_cost = -1;
@@ -297,7 +298,7 @@ int pick_bn_step(int M, int N, int step) {
     const long long tiles = static_cast<long long>((M + 127) / 128) * ((N + bn - 1) / bn);
     const long long rounds = (tiles + sms - 1) / sms;
     const long long cost = rounds * (128 + bn);
-    if (best_cost < 0 || cost <= best_cost) {
+    if (best_cost < 0 || cost < best_cost || (cost == best_cost && !narrow_on_ties)) {
       best_cost = cost;
       best = bn;
     }
@@ -466,6 +467,7 @@ fd_status run_linear(fd_handle h, int kind, const CUtensorMap& tmA, const Linear
   p.K = lin.K;
   p.bias = lin.b;
   p.err = h->state + 1;
+  p.w_static = 1;  // written once by fd_weights_create (synchronous copy)
   const CUtensorMap& k = tmK ? *tmK : tmO;
   const CUtensorMap& v = tmV ? *tmV : tmO;
   return traced(h, kind, s, [&] {
@@ -824,7 +826,8 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
     lin.b = reinterpret_cast<float*>(next());
     lin.N = N;
     lin.K = K;
-    lin.bn = pick_bn_step(M, N, step);
+    // the e4m3 GELU epilogue outweighs the FP8 MMAs: narrower tiles overlap it better
+    lin.bn = pick_bn_step(M, N, step, step == 128);
     return tmap_e4m3(&lin.tm, lin.w, K, N, K, lin.bn);
   };
   bool ok = linear(w->embed, d.D, d.cin, d.L, true);
@@ -1290,7 +1293,7 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
   if (M < 1 || N < 1 || K < 1 || A == nullptr || W == nullptr || bias == nullptr ||
       out == nullptr || err_dev == nullptr)
     return FD_ERR_INVALID_ARG;
-  if (N % 32 || K % 8 || !aligned16(A) || !aligned16(W) || !aligned16(out))
+  if (N % 32 || K % 8 || !aligned16(A) || !aligned16(W) || !aligned16(out) || !aligned16(bias))
     return FD_ERR_INVALID_ARG;
   if (epilogue < FD_EPI_F32 || epilogue > FD_EPI_SWIGLU) return FD_ERR_INVALID_ARG;
   if (epilogue == FD_EPI_GELU && N % 64) return FD_ERR_INVALID_ARG;
@@ -1342,7 +1345,8 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
     return FD_ERR_INVALID_ARG;
   if (M != frames_per_chunk * tokens) return FD_ERR_INVALID_ARG;
   if (ring_pitch < window * M || ring_pitch % 128) return FD_ERR_INVALID_ARG;
-  if (!aligned16(q_out) || !aligned16(k_ring) || !aligned16(vt_ring)) return FD_ERR_INVALID_ARG;
+  if (!aligned16(q_out) || !aligned16(k_ring) || !aligned16(vt_ring) || !aligned16(bqkv))
+    return FD_ERR_INVALID_ARG;
   if (bn == 0) bn = 128;
   if (!fd::gemm_bn_supported(bn) || !fd::gemm_bn_fits_epilogue(bn, fd::EPI_QKV))
     return FD_ERR_INVALID_ARG;
@@ -1531,7 +1535,8 @@ fd_status fd_op_linear_e4m3(int epilogue, int M, int N, int K, const void* A, co
                             float out_scale, int bn, int* err_dev, void* stream) {
   if (M < 1 || N < 1 || K < 16 || !A || !W || !col_scale || !bias || !out || !err_dev)
     return FD_ERR_INVALID_ARG;
-  if (N % 32 || K % 16 || !aligned16(A) || !aligned16(W) || !aligned16(out))
+  if (N % 32 || K % 16 || !aligned16(A) || !aligned16(W) || !aligned16(out) ||
+      !aligned16(bias) || !aligned16(col_scale))
     return FD_ERR_INVALID_ARG;
   if (epilogue != FD_EPI_F32 && epilogue != FD_EPI_RESID && epilogue != FD_EPI_GELU)
     return FD_ERR_INVALID_ARG;

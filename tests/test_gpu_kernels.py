@@ -59,6 +59,36 @@ def test_linear_f32(M, N, K, bn):
     assert_close_scaled(out, want, 2e-5, "linear f32")
 
 
+def test_gelu_epilogue_is_the_exact_erf_gelu_at_bf16():
+    """The GELU epilogue evaluates erf with Abramowitz & Stegun 7.1.26 (error <= 1.5e-7): on a
+    grid of pre-activations from -8 to 8 (A holds x in one column, W picks it, the bias shifts
+    it) every bf16 output is within one bf16 step of bf16(GELU(z)) computed in fp64 with the
+    exact erf (or, in the far negative tail, within 1e-6 of the exact value), and at least 99 %
+    of the outputs above 1e-3 in magnitude are equal to it (the rest are round-to-nearest
+    ties decided by the last fp32 bits)."""
+    M, N, K = 512, 64, 64
+    x = bf16_values(np.linspace(-8.0, 8.0, M).astype(np.float32))
+    A = np.zeros((M, K), np.float32)
+    A[:, 0] = x
+    W = np.zeros((N, K), np.float32)
+    W[:, 0] = 1.0
+    b = ((np.arange(N) - 32) / 32.0).astype(np.float32)
+    out = torch.zeros(M, N, dtype=torch.bfloat16, device="cuda")
+    err = err_word()
+    fdp.op_linear(fdp.EPI_GELU, dev(A, torch.bfloat16), dev(W, torch.bfloat16), dev(b), out,
+                  err=err)
+    check_err(err)
+    z = f64(x)[:, None] + f64(b)[None, :]
+    exact = oracle.gelu(z)
+    want = exact.to(torch.bfloat16)
+    got = out.cpu()
+    big = exact.abs() > 1e-3
+    steps = (got.view(torch.int16).int() - want.view(torch.int16).int()).abs()
+    assert int(steps[big].max()) <= 1
+    assert float((steps[big] == 0).double().mean()) >= 0.99
+    assert bool(((steps <= 1) | ((f64(got) - exact).abs() <= 1e-6)).all())
+
+
 @pytest.mark.parametrize("M,Dm,K,bn", [
     (520, 512, 256, 0),     # ragged M, library tile choice
     (130, 256, 1024, 128),  # 128-wide tiles: one 64-wide output slab per tile
