@@ -80,6 +80,11 @@ typedef struct {
                             * weights at fd_weights_create (bounds that no input    *
                             * can exceed), fp32 accumulation. Needs mlp_gated = 0.  *
                             * The blob is unchanged.                                */
+  int32_t first_chunk_frames; /* 0: every chunk emits r_t frames. 1: the causal frame *
+                            * count of Fig. 2 (T' latent frames -> 1 + r_t (T'-1)   *
+                            * frames): chunk 0 emits only its first refined frame   *
+                            * (tau = 0; which one is kept is our reading), written  *
+                            * as [C][1][H][W]; its cache entries are unchanged      */
 } fd_config;
 
 typedef struct fd_weights_s* fd_weights;
@@ -107,7 +112,8 @@ size_t fd_weights_blob_elems(const fd_config* cfg);
 size_t fd_latent_bytes(const fd_config* cfg);
 
 /* Bytes of one chunk of pixels: C * r_t * (H' 8) * (W' 8) elements of out_dtype, layout
- * [C][r_t][H][W] row-major (planar channels, then frames; Sec. 3.4 Step 3). */
+ * [C][r_t][H][W] row-major (planar channels, then frames; Sec. 3.4 Step 3). With
+ * first_chunk_frames = 1, chunk 0 writes only the first 1/r_t of this ([C][1][H][W]). */
 size_t fd_pixels_bytes(const fd_config* cfg);
 
 /* Device bytes a handle allocates (rings, scratch), excluding the shared weights. */

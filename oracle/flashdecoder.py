@@ -40,6 +40,9 @@ Readings where the paper leaves a choice (each listed in the design notes):
   R8  Head MLP: Linear(D, D) -> GELU -> Linear(D, C r_s^2).
   R9  Pixels clamped to [-1, 1]; uint8 = round-half-even(fl32(fl32(x + 1) * 127.5)).
   R12 RMSNorm with a learned gain before the temporal upsampling and before the head.
+  R16 Frame count: every chunk emits r_t frames; option first_chunk_frames = 1 follows Fig. 2's
+      causal count (T' latent frames -> 1 + r_t (T' - 1) frames): chunk 0 emits refined frame
+      tau = 0 only (the paper does not say which one is kept); nothing else changes.
   R14 RMSNorm: x / sqrt(mean(x^2) + eps) * g with eps = 1e-6.
 """
 from __future__ import annotations
@@ -354,6 +357,8 @@ class StreamingDecoder:
         y = rms_norm(hf, w["normh.g"], cfg.norm_eps)
         F = linear(gelu(linear(y, w["head1.w"], w["head1.b"])), w["head2.w"], w["head2.b"])
         pix = pixel_shuffle(F, rt, cfg.grid_h, cfg.grid_w, cfg.out_channels, cfg.r_s)
+        if t == 0 and getattr(cfg, "first_chunk_frames", 0) == 1:
+            pix = pix[:, :1]                                        # R16
         self.t += 1
         return pix.clamp(-1.0, 1.0)
 
@@ -403,8 +408,11 @@ def decode_full_masked(cfg, weights, latents) -> list[torch.Tensor]:
     hf = stack(hf, "refine", cfg.n_refine, rt)
     y = rms_norm(hf, w["normh.g"], cfg.norm_eps)
     F = linear(gelu(linear(y, w["head1.w"], w["head1.b"])), w["head2.w"], w["head2.b"])
-    return [pixel_shuffle(F[c * rt * L:(c + 1) * rt * L], rt, cfg.grid_h, cfg.grid_w,
-                          cfg.out_channels, cfg.r_s).clamp(-1.0, 1.0) for c in range(T)]
+    out = [pixel_shuffle(F[c * rt * L:(c + 1) * rt * L], rt, cfg.grid_h, cfg.grid_w,
+                         cfg.out_channels, cfg.r_s).clamp(-1.0, 1.0) for c in range(T)]
+    if getattr(cfg, "first_chunk_frames", 0) == 1:
+        out[0] = out[0][:, :1]                                      # R16
+    return out
 
 
 # --------------------------------------------------------------------------------------

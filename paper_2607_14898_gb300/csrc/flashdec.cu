@@ -165,6 +165,7 @@ struct Dims {
   bool gated;  // gated-SiLU MLP: layer 1 has 2 Mr D outputs (gate, up)
   bool qk;     // QK-norm instead of KV-norm
   bool fp8;    // block MLPs in FP8 (e4m3 operands, static scales)
+  bool f1;     // chunk 0 emits one frame (first_chunk_frames = 1)
 };
 
 bool valid_cfg(const fd_config* c) {
@@ -185,6 +186,7 @@ bool valid_cfg(const fd_config* c) {
   if (c->qk_norm != 0 && c->qk_norm != 1) return false;
   if (c->mlp_fp8 != 0 && c->mlp_fp8 != 1) return false;
   if (c->mlp_fp8 == 1 && c->mlp_gated == 1) return false;  // FP8 gated MLP not built
+  if (c->first_chunk_frames != 0 && c->first_chunk_frames != 1) return false;
   if (!(c->norm_eps >= 0.f) || !(c->rope_base > 1.f)) return false;
   const long long L = static_cast<long long>(c->latent_h / c->patch) * (c->latent_w / c->patch);
   if (L * c->r_t * c->window > (1LL << 26)) return false;
@@ -203,6 +205,7 @@ Dims dims_of(const fd_config* c) {
   d.gated = c->mlp_gated == 1;
   d.qk = c->qk_norm == 1;
   d.fp8 = c->mlp_fp8 == 1;
+  d.f1 = c->first_chunk_frames == 1;
   return d;
 }
 
@@ -615,8 +618,11 @@ fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_
   pf.ld_out = d.head_out;
   if ((st = run_linear(h, FD_K_HEAD2, h->tm_hidH, w->head2, R, pf, h->so_F, s))) return st;
   const float* F = h->F;
+  // the causal frame count (Fig. 2): chunk 0 emits refined frame 0 only (rows 0 .. L-1 of F)
+  const int frames = d.f1 && h->t_host == 0 ? 1 : d.rt;
   if ((st = traced(h, FD_K_PIXEL, s, [&] {
-         return fd::launch_pixel_head(F, d.rt, d.gh, d.gw, d.Cout, d.rs, d.u8 ? 1 : 0, pixels, s);
+         return fd::launch_pixel_head(F, frames, d.gh, d.gw, d.Cout, d.rs, d.u8 ? 1 : 0, pixels,
+                                      s);
        })))
     return st;
   int* state = h->state;
@@ -1073,7 +1079,8 @@ fd_status fd_decode_chunk_host(fd_handle h, const float* latent_host, void* pixe
   if (h == nullptr || latent_host == nullptr || pixels_host == nullptr) return FD_ERR_INVALID_ARG;
   if (h->error) return FD_ERR_STATE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const size_t lb = fd_latent_bytes(&h->cfg), pb = fd_pixels_bytes(&h->cfg);
+  const size_t lb = fd_latent_bytes(&h->cfg);
+  const size_t pb = fd_pixels_bytes(&h->cfg) / (h->d.f1 && h->t_host == 0 ? h->d.rt : 1);
   if (cudaMemcpyAsync(h->latent_buf, latent_host, lb, cudaMemcpyHostToDevice, s) != cudaSuccess) {
     h->error = true;
     return FD_ERR_CUDA;

@@ -38,7 +38,8 @@ class fd_config(ctypes.Structure):
         "latent_channels", "latent_h", "latent_w", "patch", "hidden", "heads", "kv_groups",
         "mlp_ratio", "n_blocks", "n_refine", "window", "r_t", "vae_spatial", "out_channels",
         "out_dtype", "mlp_gated")] + [("norm_eps", ctypes.c_float), ("rope_base", ctypes.c_float),
-                                      ("qk_norm", ctypes.c_int32), ("mlp_fp8", ctypes.c_int32)]
+                                      ("qk_norm", ctypes.c_int32), ("mlp_fp8", ctypes.c_int32),
+                                      ("first_chunk_frames", ctypes.c_int32)]
 
 
 _P = ctypes.c_void_p
@@ -120,6 +121,7 @@ def make_config(cfg) -> fd_config:
     c.mlp_gated = 1 if cfg.mlp_gated else 0
     c.qk_norm = 1 if cfg.qk_norm else 0
     c.mlp_fp8 = 1 if getattr(cfg, "mlp_fp8", False) else 0
+    c.first_chunk_frames = int(getattr(cfg, "first_chunk_frames", 0))
     c.norm_eps = float(cfg.norm_eps)
     c.rope_base = float(cfg.rope_base)
     return c

@@ -42,6 +42,7 @@ class FDConfig:
     mlp_gated: bool = False        # MLP: False = Linear, GELU, Linear; True = gated SiLU
     qk_norm: bool = False          # per-head RMSNorm on Q and K instead of on K and V
     mlp_fp8: bool = False          # MLP GEMMs in FP8 (e4m3) with static scales
+    first_chunk_frames: int = 0    # 1: chunk 0 emits one frame (causal frame count, Fig. 2)
     n_blocks: int = 2              # backbone blocks
     n_refine: int = 0              # temporal-refinement blocks
     window: int = 2                # W_frm, counts the current chunk
@@ -144,6 +145,10 @@ PRESETS: dict[str, FDConfig] = {
     "480p_fp8": FDConfig(latent_h=60, latent_w=104, patch=2, hidden=1024, heads=16,
                          kv_groups=4, n_blocks=24, n_refine=2, window=4, r_t=4, mlp_fp8=True,
                          name="480p_fp8", chunks=16),
+    # the causal frame count of Fig. 2 (T' latents -> 1 + r_t (T' - 1) frames), r_t = 4
+    "small_f1": FDConfig(latent_h=20, latent_w=26, patch=2, hidden=256, heads=4, kv_groups=2,
+                         n_blocks=2, n_refine=1, window=3, r_t=4, first_chunk_frames=1,
+                         name="small_f1", chunks=3),
     # the QK-norm reading of "KV-norm" at tiny size, with refinement
     "tiny_qk": FDConfig(qk_norm=True, n_refine=1, r_t=2, name="tiny_qk", chunks=3),
     # XL layout at tiny size: 48-channel 16x latent, patch 1, gated-SiLU MLP, refinement

@@ -437,6 +437,23 @@ def test_output_shapes_follow_compression_factors():
     assert tuple(oracle.decode_stream(cfg, w, z)[0].shape) == (3, 1, 64, 64)
 
 
+def test_causal_frame_count_of_fig2():
+    """Fig. 2 caption: at r_t = 4, 3 latent frames decode to 9 output frames (1 + r_t (T'-1)).
+    With first_chunk_frames = 1 chunk 0 keeps refined frame 0 only; every other output, and
+    chunk 0's kept frame, equal the r_t-frames-per-chunk decode of the same stream."""
+    cfg, w, z = _setup("small_f1")
+    got = oracle.decode_stream(cfg, w, z)
+    assert cfg.r_t == 4 and len(got) == 3
+    assert sum(p.shape[1] for p in got) == 9
+    full = oracle.decode_stream(cfg.replace(first_chunk_frames=0), w, z)
+    assert torch.equal(got[0], full[0][:, :1])
+    for a, b in zip(got[1:], full[1:]):
+        assert torch.equal(a, b)
+    masked = oracle.decode_full_masked(cfg, w, z)
+    for a, b in zip(got, masked):
+        assert a.shape == b.shape and torch.allclose(a, b, atol=1e-12)
+
+
 def test_kv_cache_size_formula():
     """Eq. kv_cache: G x (W L) x D_h per layer for K and V; refinement r_t W L (Sec. 3.3)."""
     cfg = synth.PRESETS["480p"]
