@@ -36,6 +36,9 @@ Readings where the paper leaves a choice (each listed in the design notes):
       per weight row s = 2^ceil(log2(max|w| / 448)); the MLP input u = RMSNorm(h) g obeys
       |u_i| <= sqrt(D) max|g|, its scale s_u covers that; the MLP hidden a = GELU(z) obeys
       |a_j| <= max(1, max_j 1.125 sqrt(D) max|g| ||w1_j|| + |b1_j|), its scale s_h covers that.
+      With the gated MLP, a_j = SiLU(z_gate_j) z_up_j and |SiLU(x)| <= max(|x|, 0.28) (SiLU is
+      below x for x > 0 and its negative branch never reaches -0.2785), so
+      |a_j| <= max(B_gate_j, 0.28) B_up_j with B the same per-row bound on |z|.
       So no value leaves the e4m3 range (448) for any input.
   R8  Head MLP: Linear(D, D) -> GELU -> Linear(D, C r_s^2).
   R9  Pixels clamped to [-1, 1]; uint8 = round-half-even(fl32(fl32(x + 1) * 127.5)).
@@ -123,13 +126,19 @@ def fp8_weight(w: torch.Tensor) -> torch.Tensor:
     return e4m3(w / s[:, None]) * s[:, None]
 
 
-def fp8_mlp_scales(g2: torch.Tensor, w1_deq: torch.Tensor, b1: torch.Tensor):
+def fp8_mlp_scales(g2: torch.Tensor, w1_deq: torch.Tensor, b1: torch.Tensor,
+                   gated: bool = False):
     """Static activation scales (s_u, s_h) of one FP8 MLP from its weights (see R7)."""
     D = g2.shape[0]
     gmax = float(g2.abs().max())
     s_u = pow2_ceil(math.sqrt(D) * gmax / 448.0)
-    bz = float((1.125 * math.sqrt(D) * gmax * w1_deq.norm(dim=1) + b1.abs()).max())
-    s_h = pow2_ceil(max(bz, 1.0) / 448.0)
+    bz = 1.125 * math.sqrt(D) * gmax * w1_deq.norm(dim=1) + b1.abs()   # |z_j| <= bz_j
+    if gated:
+        dm = bz.shape[0] // 2
+        bound = float((torch.clamp(bz[:dm], min=0.28) * bz[dm:]).max())
+    else:
+        bound = float(bz.max())
+    s_h = pow2_ceil(max(bound, 1.0) / 448.0)
     return s_u, s_h
 
 
@@ -265,8 +274,13 @@ def _block_rest(h, o, w, p, cfg):
     u = rms_norm(h, w[p + "norm2.g"], cfg.norm_eps)
     if getattr(cfg, "mlp_fp8", False):
         w1, w2 = fp8_weight(w[p + "mlp1.w"]), fp8_weight(w[p + "mlp2.w"])
-        s_u, s_h = fp8_mlp_scales(w[p + "norm2.g"], w1, w[p + "mlp1.b"])
-        a = gelu(linear(e4m3(u / s_u) * s_u, w1, w[p + "mlp1.b"]))
+        s_u, s_h = fp8_mlp_scales(w[p + "norm2.g"], w1, w[p + "mlp1.b"], cfg.mlp_gated)
+        z = linear(e4m3(u / s_u) * s_u, w1, w[p + "mlp1.b"])
+        if cfg.mlp_gated:
+            dm = z.shape[1] // 2
+            a = silu(z[:, :dm]) * z[:, dm:]
+        else:
+            a = gelu(z)
         return h + linear(e4m3(a / s_h) * s_h, w2, w[p + "mlp2.b"])
     z = linear(u, w[p + "mlp1.w"], w[p + "mlp1.b"])
     if cfg.mlp_gated:

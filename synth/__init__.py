@@ -145,6 +145,10 @@ PRESETS: dict[str, FDConfig] = {
     "480p_fp8": FDConfig(latent_h=60, latent_w=104, patch=2, hidden=1024, heads=16,
                          kv_groups=4, n_blocks=24, n_refine=2, window=4, r_t=4, mlp_fp8=True,
                          name="480p_fp8", chunks=16),
+    # gated (XL-layout) MLP in FP8 at tiny size, with refinement
+    "tiny_gated_fp8": FDConfig(latent_channels=48, latent_h=10, latent_w=13, vae_spatial=16,
+                               mlp_gated=True, mlp_fp8=True, n_refine=1, r_t=2,
+                               name="tiny_gated_fp8", chunks=3),
     # the causal frame count of Fig. 2 (T' latents -> 1 + r_t (T' - 1) frames), r_t = 4
     "small_f1": FDConfig(latent_h=20, latent_w=26, patch=2, hidden=256, heads=4, kv_groups=2,
                          n_blocks=2, n_refine=1, window=3, r_t=4, first_chunk_frames=1,
@@ -163,6 +167,15 @@ PRESETS: dict[str, FDConfig] = {
     "xl_720p": FDConfig(latent_channels=48, latent_h=45, latent_w=80, vae_spatial=16,
                         hidden=1536, heads=24, kv_groups=3, mlp_gated=True, n_blocks=20,
                         n_refine=2, window=2, r_t=4, out_u8=True, name="xl_720p", chunks=16),
+    # the XL layout with FP8 MLPs (the paper's lossy "XL-Opt" setting, Sec. 4.6)
+    "xl_480p_fp8": FDConfig(latent_channels=48, latent_h=30, latent_w=52, vae_spatial=16,
+                            hidden=1536, heads=24, kv_groups=3, mlp_gated=True, mlp_fp8=True,
+                            n_blocks=20, n_refine=2, window=2, r_t=4, name="xl_480p_fp8",
+                            chunks=16),
+    "xl_720p_fp8": FDConfig(latent_channels=48, latent_h=45, latent_w=80, vae_spatial=16,
+                            hidden=1536, heads=24, kv_groups=3, mlp_gated=True, mlp_fp8=True,
+                            n_blocks=20, n_refine=2, window=2, r_t=4, out_u8=True,
+                            name="xl_720p_fp8", chunks=16),
     "xl_1080p": FDConfig(latent_channels=48, latent_h=68, latent_w=120, vae_spatial=16,
                          hidden=1536, heads=24, kv_groups=3, mlp_gated=True, n_blocks=20,
                          n_refine=2, window=2, r_t=4, out_u8=True, name="xl_1080p", chunks=8),

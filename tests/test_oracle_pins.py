@@ -175,6 +175,46 @@ def test_fp8_static_scales_never_overflow_and_are_tight():
     assert 1e-3 < rel < 0.1, rel
 
 
+def test_silu_bound_used_by_the_gated_fp8_scale():
+    """|SiLU(x)| <= max(|x|, 0.28): SiLU lies below x for x > 0, and its negative branch has
+    its minimum near x = -1.2785 at about -0.2785 (so the 0.28 floor is nearly reached)."""
+    x = torch.linspace(-40.0, 40.0, 400001, dtype=F64)
+    y = oracle.silu(x)
+    assert bool((y.abs() <= torch.clamp(x.abs(), min=0.28)).all())
+    assert -0.2786 < float(y.min()) < -0.2784
+    assert abs(float(x[int(y.argmin())]) + 1.2785) < 1e-3
+
+
+def test_gated_fp8_scales_never_overflow():
+    """The gated FP8 MLP's hidden scale covers SiLU(gate) * up for any input: adversarial
+    one-hot rows that put all of u into the coordinate with the largest gain, and random
+    rows, stay within the e4m3 range after scaling; the FP8 gated MLP differs from the exact
+    one by FP8-sized amounts."""
+    from oracle.flashdecoder import linear
+    cfg = synth.PRESETS["tiny_gated_fp8"]
+    w = {k: torch.from_numpy(v).to(torch.float64) for k, v in synth.make_weights(cfg).items()}
+    D = cfg.hidden
+    g2, b1 = w["blocks.0.norm2.g"], w["blocks.0.mlp1.b"]
+    w1 = oracle.fp8_weight(w["blocks.0.mlp1.w"])
+    s_u, s_h = oracle.fp8_mlp_scales(g2, w1, b1, gated=True)
+    h = torch.randn(64, D, dtype=torch.float64) * 3
+    for r, i in enumerate(g2.abs().argsort(descending=True)[:8].tolist()):
+        h[r] = 0.0
+        h[r, i] = (-1.0) ** r * 5.0
+    u = oracle.rms_norm(h, g2, 0.0)
+    assert float((u / s_u).abs().max()) <= 448.0
+    z = linear(oracle.e4m3(u / s_u) * s_u, w1, b1)
+    dm = z.shape[1] // 2
+    a = oracle.silu(z[:, :dm]) * z[:, dm:]
+    assert float((a / s_h).abs().max()) <= 448.0
+    w2 = w["blocks.0.mlp2.w"]
+    zx = linear(u, w["blocks.0.mlp1.w"], b1)
+    exact = linear(oracle.silu(zx[:, :dm]) * zx[:, dm:], w2, None)
+    q = linear(oracle.e4m3(a / s_h) * s_h, oracle.fp8_weight(w2), None)
+    rel = float((q - exact).norm() / exact.norm())
+    assert 1e-3 < rel < 0.2, rel
+
+
 def test_linear_is_x_wt_plus_b():
     x, w, b = rnd(5, 7, seed=3), rnd(4, 7, seed=4), rnd(4, seed=5)
     brute = torch.tensor([[sum(x[i, k] * w[j, k] for k in range(7)) + b[j] for j in range(4)]
@@ -336,7 +376,7 @@ def test_fig2_visibility_golden():
 
 
 @pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8", "tiny_qk", "tiny_gated",
-                                  "small_fp8"])
+                                  "small_fp8", "tiny_gated_fp8"])
 def test_streaming_equals_masked_full_sequence(name):
     """Sec. 3.3: sequential decoding with the rolling cache equals one pass under the block
     sliding-window mask (the paper's training-inference consistency)."""
