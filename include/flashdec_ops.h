@@ -127,6 +127,9 @@ fd_status fd_op_rmsnorm_e4m3(const float* h, const float* g, int M, int D, float
  *   FD_EPI_F32    out fp32 [M][N]  = acc * col_scale + bias
  *   FD_EPI_RESID  out fp32 [M][N] += acc * col_scale + bias
  *   FD_EPI_GELU   out e4m3 [M][N]  = e4m3(GELU(acc * col_scale + bias) * out_scale)
+ *   FD_EPI_SWIGLU out e4m3 [M][N/2] = e4m3(SiLU(g) u * out_scale), g / u = acc * col_scale +
+ *                 bias of the gate / up rows, interleaved in blocks of 32 as for fd_op_linear
+ *                 (the FP8 gated MLP layer 1); N % 256 == 0
  * K % 16 == 0, N % 32 == 0 (N % 128 == 0 for FD_EPI_GELU), 16-byte aligned A / W / out /
  * bias / col_scale.
  * bn = output tile width (96 / 128 / 192 / 256, 128 or 256 for FD_EPI_GELU; 0 = choice). */

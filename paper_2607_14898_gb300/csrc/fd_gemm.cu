@@ -20,6 +20,8 @@
 //   EPI_SWIGLU out = bf16(SiLU(gate + b) * (up + b)) (gated MLP layer 1 of the XL layout; gate
 //              and up rows interleaved in blocks of 32, so 128 columns give 64 outputs)
 //   EPI_GELU_F8 out = e4m3(GELU(acc s_col + b) s_out)  (FP8 MLP layer 1, Sec. 4.6)
+//   EPI_SWIGLU_F8 out = e4m3(SiLU(gate) up s_out), gate / up = acc s_col + b in the interleaved
+//              blocks of EPI_SWIGLU (the FP8 gated MLP layer 1; 256 columns -> 128 outputs)
 // FP8 operands (p.fp8): A and W are e4m3 with a K-block of 128 elements (the same 128-byte
 // swizzled rows), tcgen05.mma kind::f8f6f4 with K = 32 per instruction; the fp32 epilogues
 // then scale the accumulator per column by s_A s_W[n] (p.col_scale).
@@ -88,7 +90,9 @@ __device__ __forceinline__ void load32(const float* p, float (&v)[32]) {
   }
 }
 
-__device__ __forceinline__ float silu(float x) { return x / (1.0f + __expf(-x)); }
+// SiLU(x) = x / (1 + e^-x) with the fast division (a few ulp; for x -> -inf the denominator
+// overflows and the quotient goes to 0, the correct limit)
+__device__ __forceinline__ float silu(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
 
 // cos / sin of the 32 rotation pairs of one token (3D-RoPE: temporal pairs first, then row,
 // then column; angle = position * base^(-2i/d_band)). Temporal values come from the chunk's
@@ -422,6 +426,46 @@ __global__ void __launch_bounds__(192, 1)
           publish();
           if (lane == 0 && row0 < p.M) {
             tma_store_2d(&tmO, smem_u32(buf), col, row0);
+            bulk_commit();
+          }
+        }
+      } else if (p.epi == EPI_SWIGLU_F8) {
+        // 256 accumulator columns (4 blocks of 32 gate + 32 up) -> one 128-byte e4m3 row
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 256) {
+          const int col = n0 + c;
+          if (col >= p.N) break;
+          uint32_t w[32];
+#pragma unroll
+          for (int hh = 0; hh < 4; ++hh) {
+            uint32_t rg[32], ru[32];
+            __syncwarp();
+            tmem_ld_32x32b_x32(tbase + c + 64 * hh, rg);
+            tmem_ld_32x32b_x32(tbase + c + 64 * hh + 32, ru);
+            tmem_ld_wait();
+            const int cb = col + 64 * hh;
+            float v[32];
+            {
+              float cs[32], bb[32];
+              load32(p.col_scale + cb, cs);
+              load32(p.bias + cb, bb);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) v[j] = silu(fmaf(__uint_as_float(rg[j]), cs[j], bb[j]));
+              load32(p.col_scale + cb + 32, cs);
+              load32(p.bias + cb + 32, bb);
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                v[j] *= fmaf(__uint_as_float(ru[j]), cs[j], bb[j]) * p.out_scale;
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              w[8 * hh + j] = pack_e4m3x4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+          }
+          uint8_t* buf = acquire();
+          put_row_sw128(buf, lane, w);
+          publish();
+          if (lane == 0 && row0 < p.M) {
+            tma_store_2d(&tmO, smem_u32(buf), col / 2, row0);
             bulk_commit();
           }
         }

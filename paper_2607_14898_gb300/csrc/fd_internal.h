@@ -41,6 +41,8 @@ enum EpiKind : int {
   EPI_SWIGLU = 5, // gated SiLU: accumulator columns in blocks of 64 (32 gate, 32 up of the same
                   // hidden units); out_bf16[r][32j + i] = bf16(SiLU(g + bg) * (u + bu))
   EPI_GELU_F8 = 6,  // out_f8[r][c] = e4m3(GELU(acc * col_scale + bias) * out_scale)
+  EPI_SWIGLU_F8 = 7,  // gated: out_f8[r][32j + i] = e4m3(SiLU(g) u out_scale) with g, u the
+                      // (acc * col_scale + bias) of the interleaved gate / up columns
 };
 
 // Rotary / cache parameters of the fused QKV epilogue.
@@ -182,6 +184,7 @@ inline bool gemm_bn_supported(int bn) {
 inline bool gemm_bn_fits_epilogue(int bn, int epi) {
   if (epi == EPI_SWIGLU) return bn % 128 == 0;  // 128 accumulator columns -> 64 outputs
   if (epi == EPI_GELU_F8) return bn % 128 == 0;  // 128 e4m3 outputs per 128-byte slab row
+  if (epi == EPI_SWIGLU_F8) return bn % 256 == 0;  // 256 accumulator columns -> 128 outputs
   return (epi == EPI_QKV || epi == EPI_GELU) ? bn % 64 == 0 : bn % 32 == 0;
 }
 

@@ -185,7 +185,6 @@ bool valid_cfg(const fd_config* c) {
   if (c->mlp_gated != 0 && c->mlp_gated != 1) return false;
   if (c->qk_norm != 0 && c->qk_norm != 1) return false;
   if (c->mlp_fp8 != 0 && c->mlp_fp8 != 1) return false;
-  if (c->mlp_fp8 == 1 && c->mlp_gated == 1) return false;  // FP8 gated MLP not built
   if (c->first_chunk_frames != 0 && c->first_chunk_frames != 1) return false;
   if (!(c->norm_eps >= 0.f) || !(c->rope_base > 1.f)) return false;
   const long long L = static_cast<long long>(c->latent_h / c->patch) * (c->latent_w / c->patch);
@@ -230,7 +229,7 @@ void blob_layout(const Dims& d, std::vector<BlobEntry>& out) {
     F(D); W(static_cast<size_t>(d.qkv_out) * D); F(d.qkv_out); F(kHeadDim); F(kHeadDim);
     W(D * d.N * kHeadDim); F(D); F(D);
     if (d.gated) {
-      out.push_back({2 * Dm * D, 0, Dm, D});
+      out.push_back({2 * Dm * D, d.fp8 ? 2 : 0, Dm, D});
       out.push_back({2 * Dm, 1, Dm, 1});
     } else if (d.fp8) {
       out.push_back({Dm * D, 2, 0, D});
@@ -540,7 +539,7 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
          })))
       return st;
     fd::GemmParams p1{};
-    p1.epi = fd::EPI_GELU_F8;
+    p1.epi = d.gated ? fd::EPI_SWIGLU_F8 : fd::EPI_GELU_F8;
     p1.fp8 = 1;
     p1.col_scale = lw.cs1;
     p1.out_scale = lw.inv_sh;
@@ -742,7 +741,8 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
     cur = align_up(cur + layout[i].elems * esz_dev, 256);
   }
   const size_t Dm = static_cast<size_t>(d.Mr) * d.D;
-  const size_t fp8_cs_bytes = align_up((Dm + d.D) * 4, 256);  // per block: mlp1, mlp2 scales
+  const size_t fp8_cs_bytes =  // per block: mlp1 (gate and up when gated), mlp2 column scales
+      align_up(((d.gated ? 2 : 1) * Dm + d.D) * 4, 256);
   const size_t fp8_off = cur;
   if (d.fp8) cur += static_cast<size_t>(d.nb + d.nr) * fp8_cs_bytes;
   std::vector<uint8_t> stage;
@@ -770,10 +770,13 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
       // FP8 weight (Sec. 4.6): per row, s = 2^ceil(log2(max|w| / 448)) and code = e4m3(w / s)
       // (round to nearest even; |w / s| <= 448, so nothing saturates). Keeps s and the norm of
       // the dequantised row for the static activation scales.
+      // (row_scale in device row order, row_norm in blob row order; the gated layer's rows are
+      // interleaved on the device like the bf16 one's)
       const size_t rows = e.elems / e.row_len;
       row_scale[i].resize(rows);
       row_norm[i].resize(rows);
       for (size_t r = 0; r < rows; ++r, src += e.row_len) {
+        const size_t dr = e.gate_rows ? gated_row(r, e.gate_rows) : r;
         double amax = 0.0;
         for (size_t k = 0; k < e.row_len; ++k)
           amax = std::fmax(amax, std::fabs(static_cast<double>(blob_value(src + k))));
@@ -782,11 +785,11 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
         for (size_t k = 0; k < e.row_len; ++k) {
           const float x = static_cast<float>(static_cast<double>(blob_value(src + k)) / sc);
           const uint8_t code = __nv_cvt_float_to_fp8(x, __NV_SATFINITE, __NV_E4M3);
-          stage[doff[i] + r * e.row_len + k] = code;
+          stage[doff[i] + dr * e.row_len + k] = code;
           const double dq = e4m3_value(code) * sc;
           ss += dq * dq;
         }
-        row_scale[i][r] = sc;
+        row_scale[i][dr] = sc;
         row_norm[i][r] = std::sqrt(ss);
       }
       continue;
@@ -851,25 +854,32 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
       //   |GELU(z_j)| <= max(1, |z_j|) and |z_j| <= 1.125 sqrt(D) max|g| ||w1_j|| + |b1_j|
       //   (with the e4m3 rounding of u, at most 1 + 2^-3)         -> s_h likewise
       // Columns are dequantised by s_u s_w1[n] (layer 1) and s_h s_w2[n] (layer 2).
+      // Gated: |SiLU(x)| <= max(|x|, 0.28), so |SiLU(gate_j) up_j| <= max(B_gate_j, 0.28) B_up_j.
       const size_t e_w1 = idx, e_b1 = idx + 1, e_w2 = idx + 2;
-      ok = ok && linear_e4m3(lw.mlp1, static_cast<int>(Dm), d.D, M, 128);
+      const size_t N1 = (d.gated ? 2 : 1) * Dm;
+      ok = ok && linear_e4m3(lw.mlp1, static_cast<int>(N1), d.D, M, d.gated ? 256 : 128);
       ok = ok && linear_e4m3(lw.mlp2, d.D, static_cast<int>(Dm), M, 32);
       const float* g2 = host_f32(e_g2);
-      const float* b1 = host_f32(e_b1);
+      const float* b1 = host_f32(e_b1);  // device (interleaved) order when gated
       double gmax = 0.0;
       for (int i = 0; i < d.D; ++i) gmax = std::fmax(gmax, std::fabs(static_cast<double>(g2[i])));
       const double sq = std::sqrt(static_cast<double>(d.D));
       const double s_u = pow2_ceil(sq * gmax / 448.0);
-      double bz = 0.0;
+      // bound on |z_j| of blob row j
+      auto bz = [&](size_t j) {
+        const size_t dj = d.gated ? gated_row(j, Dm) : j;
+        return 1.125 * sq * gmax * row_norm[e_w1][j] + std::fabs(static_cast<double>(b1[dj]));
+      };
+      double bound = 0.0;
       for (size_t j = 0; j < Dm; ++j)
-        bz = std::fmax(bz, 1.125 * sq * gmax * row_norm[e_w1][j] + std::fabs(double(b1[j])));
-      const double s_h = pow2_ceil(std::fmax(bz, 1.0) / 448.0);
+        bound = std::fmax(bound, d.gated ? std::fmax(bz(j), 0.28) * bz(Dm + j) : bz(j));
+      const double s_h = pow2_ceil(std::fmax(bound, 1.0) / 448.0);
       const size_t off = fp8_off + static_cast<size_t>(fp8_block++) * fp8_cs_bytes;
       float* cs = reinterpret_cast<float*>(&stage[off]);
-      for (size_t n = 0; n < Dm; ++n) cs[n] = static_cast<float>(s_u * row_scale[e_w1][n]);
-      for (int n = 0; n < d.D; ++n) cs[Dm + n] = static_cast<float>(s_h * row_scale[e_w2][n]);
+      for (size_t n = 0; n < N1; ++n) cs[n] = static_cast<float>(s_u * row_scale[e_w1][n]);
+      for (int n = 0; n < d.D; ++n) cs[N1 + n] = static_cast<float>(s_h * row_scale[e_w2][n]);
       lw.cs1 = reinterpret_cast<float*>(base + off);
-      lw.cs2 = lw.cs1 + Dm;
+      lw.cs2 = lw.cs1 + N1;
       lw.inv_su = static_cast<float>(1.0 / s_u);
       lw.inv_sh = static_cast<float>(1.0 / s_h);
       return;
@@ -1545,19 +1555,22 @@ fd_status fd_op_linear_e4m3(int epilogue, int M, int N, int K, const void* A, co
   if (N % 32 || K % 16 || !aligned16(A) || !aligned16(W) || !aligned16(out) ||
       !aligned16(bias) || !aligned16(col_scale))
     return FD_ERR_INVALID_ARG;
-  if (epilogue != FD_EPI_F32 && epilogue != FD_EPI_RESID && epilogue != FD_EPI_GELU)
+  if (epilogue != FD_EPI_F32 && epilogue != FD_EPI_RESID && epilogue != FD_EPI_GELU &&
+      epilogue != FD_EPI_SWIGLU)
     return FD_ERR_INVALID_ARG;
-  const bool f8_out = epilogue == FD_EPI_GELU;
-  if (f8_out && (N % 128 || !(out_scale > 0.f))) return FD_ERR_INVALID_ARG;
-  const int epi = f8_out ? fd::EPI_GELU_F8 : epilogue;
-  if (bn == 0) bn = pick_bn_step(M, N, f8_out ? 128 : 32);
+  const bool gated = epilogue == FD_EPI_SWIGLU;
+  const bool f8_out = epilogue == FD_EPI_GELU || gated;
+  if (f8_out && (N % (gated ? 256 : 128) || !(out_scale > 0.f))) return FD_ERR_INVALID_ARG;
+  const int epi = gated ? fd::EPI_SWIGLU_F8 : f8_out ? fd::EPI_GELU_F8 : epilogue;
+  if (bn == 0) bn = pick_bn_step(M, N, gated ? 256 : f8_out ? 128 : 32, f8_out);
   if (!fd::gemm_bn_supported(bn) || !fd::gemm_bn_fits_epilogue(bn, epi))
     return FD_ERR_INVALID_ARG;
   fd_status st = check_device();
   if (st) return st;
   CUtensorMap ta, tb, to;
   if (!tmap_e4m3(&ta, A, K, M, K, 128) || !tmap_e4m3(&tb, W, K, N, K, bn)) return FD_ERR_CUDA;
-  if (!(f8_out ? tmap_out_e4m3(&to, out, N, M, N) : tmap_out_f32(&to, out, N, M, N)))
+  const int n_out = gated ? N / 2 : N;
+  if (!(f8_out ? tmap_out_e4m3(&to, out, n_out, M, n_out) : tmap_out_f32(&to, out, N, M, N)))
     return FD_ERR_CUDA;
   fd::GemmParams p{};
   p.M = M; p.N = N; p.K = K; p.epi = epi; p.bias = bias; p.err = err_dev;
@@ -1566,7 +1579,7 @@ fd_status fd_op_linear_e4m3(int epilogue, int M, int N, int K, const void* A, co
   p.out_scale = out_scale;
   if (f8_out) p.out_f8 = static_cast<uint8_t*>(out);
   else p.out_f32 = static_cast<float*>(out);
-  p.ld_out = N;
+  p.ld_out = n_out;
   return launch_ok(fd::launch_gemm(ta, tb, to, to, to, p, bn, num_sms(),
                                    static_cast<cudaStream_t>(stream)));
 }

@@ -185,6 +185,36 @@ def test_linear_e4m3_gelu_to_e4m3_and_rmsnorm_e4m3():
     assert_e4m3_close(u, oracle.rms_norm(h.double(), g.double(), 1e-6) * 8.0, "rmsnorm e4m3")
 
 
+def test_linear_e4m3_swiglu_to_e4m3():
+    """The FP8 gated MLP's layer 1: gate and up rows interleaved in blocks of 32 as for the
+    bf16 gated epilogue, out = e4m3(SiLU(g) u out_scale) against the oracle's rounding of the
+    same formula; two launches in a row give the same codes."""
+    M, Dm, K = 300, 512, 384
+    torch.manual_seed(11)
+    a_c, a = e4m3_codes(torch.randn(M, K, dtype=torch.float64) * 2)
+    wg_c, wg = e4m3_codes(torch.randn(Dm, K, dtype=torch.float64) * 30)
+    wu_c, wu = e4m3_codes(torch.randn(Dm, K, dtype=torch.float64) * 30)
+    csg = torch.full((Dm,), 2.0 ** -10, dtype=torch.float32)
+    csu = torch.full((Dm,), 2.0 ** -11, dtype=torch.float32)
+    bg, bu = torch.randn(Dm) * 0.1, torch.randn(Dm) * 0.1
+    blocks = lambda g, u: torch.cat([torch.cat([g[32 * j:32 * j + 32], u[32 * j:32 * j + 32]])
+                                     for j in range(Dm // 32)])
+    W, cs, b = blocks(wg_c, wu_c), blocks(csg, csu), blocks(bg, bu)
+    zg = oracle.linear(a, wg, None) * csg.double() + bg.double()
+    zu = oracle.linear(a, wu, None) * csu.double() + bu.double()
+    want = oracle.silu(zg) * zu * 4.0
+    outs = []
+    for _ in range(2):
+        out = torch.zeros(M, Dm, dtype=torch.uint8, device="cuda")
+        err = err_word()
+        fdp.op_linear_e4m3(fdp.EPI_SWIGLU, a_c.cuda(), W.contiguous().cuda(), cs.cuda(),
+                           b.cuda(), out, out_scale=4.0, err=err)
+        check_err(err)
+        assert_e4m3_close(out, want, "swiglu e4m3")
+        outs.append(out.cpu())
+    assert torch.equal(outs[0], outs[1])
+
+
 def test_linear_resid_gelu_tup():
     M, N, K, D = 520, 1024, 256, 256
     A, W, b = linear_case(M, N, K, seed=11)
