@@ -39,6 +39,15 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
                        const float* bias, void* out, int tup_hidden, int bn, int* err_dev,
                        void* stream);
 
+/* The same with the launch shape chosen by the caller: bn as above (0 = library choice of
+ * everything), pair = 1 for 128-row tiles on single CTAs, 2 for 256-row tiles on CTA pairs
+ * (tcgen05 cta_group::2: each CTA of the pair holds its 128 rows of A and half of W's bn rows,
+ * the even CTA issues the pair's MMAs; bn 96 / 128 / 192 / 256), 0 = library choice. Results
+ * do not depend on the shape. fd_op_linear runs an explicit bn on single CTAs. */
+fd_status fd_op_linear_tiled(int epilogue, int M, int N, int K, const void* A, const void* W,
+                             const float* bias, void* out, int tup_hidden, int bn, int pair,
+                             int* err_dev, void* stream);
+
 /* Temporal 3D-RoPE table of chunk t (Sec. 3.2, reading of Algorithm 1's "RoPE offset"):
  * table[tau][i] = (cos, sin)((t * frames_per_chunk + tau) * rope_base^(-2i/24)) for the
  * frames_per_chunk frames of the chunk and the 12 temporal pairs (fp32 values of an fp64

@@ -34,17 +34,25 @@
 
 namespace fd {
 
-template <int BN>
+// PAIR: the tile is 256 x BN, computed by a cluster of two CTAs with tcgen05 cta_group::2
+// MMAs issued by the even CTA: each CTA holds its 128 rows of A and half (BN/2 rows) of W per
+// stage, the pair's tensor cores read both halves, and each CTA's TMEM receives its 128 rows of
+// the accumulator. Per SM, a stage then needs 16 KB + 64 BN bytes for 2 BN MMA cycles instead of
+// 16 KB + 128 BN, which is what bounds the single-CTA kernel (shared-memory intake per SM).
+template <int BN, bool PAIR>
 struct GemmCfg {
-  static constexpr int kStages = BN >= 192 ? 4 : 6;
   static constexpr int kABytes = kBM * kBK * 2;  // 16 KB
-  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kBRows = PAIR ? BN / 2 : BN;
+  static constexpr int kBBytes = kBRows * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kRoom = (227 * 1024 - 4 * 2 * 4096 - 256) / kStageBytes;
+  static constexpr int kStages = PAIR ? (kRoom > 8 ? 8 : kRoom) : (BN >= 192 ? 4 : 6);
   static constexpr int kTmemCols = 2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512);
   static constexpr int kStgOffset = kStages * kStageBytes;   // 4 warps x 2 x 4 KB staging
   static constexpr int kBarOffset = kStgOffset + 4 * 2 * 4096;
   static constexpr int kSmem = kBarOffset + 256;
   static_assert(kSmem <= 227 * 1024, "shared memory");
+  static_assert((kBRows * 128) % 1024 == 0, "W stages start on a swizzle atom");
 };
 
 // one 128-byte row (8 x 16 B) of a 32-row slab in the 128-byte-swizzled layout of a TMA box
@@ -117,12 +125,12 @@ __device__ __forceinline__ void rope_table(const QkvEpi& q, int tau, int y, int 
   }
 }
 
-template <int BN>
+template <int BN, bool PAIR>
 __global__ void __launch_bounds__(192, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ GemmParams p) {
-  using C = GemmCfg<BN>;
+  using C = GemmCfg<BN, PAIR>;
   extern __shared__ __align__(1024) uint8_t smem[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -137,11 +145,24 @@ __global__ void __launch_bounds__(192, 1)
   const uint32_t sB = sA + C::kStages * C::kABytes;
   const bool aligned = (sA & 1023u) == 0;
 
-  const int m_tiles = (p.M + kBM - 1) / kBM;
+  // CTA pairs: rank 0 issues the MMAs; every load of the pair completes on rank 0's full
+  // barrier; the MMA commits arrive in both CTAs (stage release, accumulator ready); both CTAs'
+  // epilogue warps release the accumulator on rank 0's barrier
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0;
+  const int tile_rows = PAIR ? 2 * kBM : kBM;
+  const int m_tiles = (p.M + tile_rows - 1) / tile_rows;
   const int n_tiles = (p.N + BN - 1) / BN;
   const int tiles = m_tiles * n_tiles;
+  const int cta0 = PAIR ? static_cast<int>(blockIdx.x) / 2 : static_cast<int>(blockIdx.x);
+  const int ctas = PAIR ? static_cast<int>(gridDim.x) / 2 : static_cast<int>(gridDim.x);
   const int kel = p.fp8 ? 2 * kBK : kBK;  // K elements per 128-byte stage row
   const int nk = (p.K + kel - 1) / kel;
+  const uint32_t full_tx = PAIR ? 2 * C::kStageBytes : C::kStageBytes;  // on rank 0's barrier
+  const uint32_t bar_full0 = PAIR ? mapa_rank(bar_full, 0) : bar_full;
+  auto load = [&](uint32_t dst, const CUtensorMap* m, int s, int x, int y) {
+    if (PAIR) tma_load_2d_pair(dst, m, bar_full0 + 8 * s, x, y);
+    else tma_load_2d(dst, m, bar_full + 8 * s, x, y);
+  };
 
   if (threadIdx.x == 0) {
     if (!aligned) atomicOr(p.err, ERR_SMEM_ALIGN);
@@ -151,30 +172,36 @@ __global__ void __launch_bounds__(192, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(bar_tfull + 8 * a, 1);
-      mbar_init(bar_tempty + 8 * a, 128);
+      mbar_init(bar_tempty + 8 * a, PAIR ? 8 : 128);  // pairs: one arrive per epilogue warp
     }
     mbar_init(bar_done, 1);
     fence_barrier_init();
     prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
   }
+  if (PAIR) cluster_sync();  // both CTAs' barriers exist before any load or commit reaches them
   // Weights that no kernel of the stream writes (p.w_static) are loaded into the first stages
   // while the previous kernel is still finishing; only the activations wait for it. Thread 0
   // is the TMA producer and initialised the barriers above.
-  const int pre = (p.w_static && aligned && static_cast<int>(blockIdx.x) < tiles)
+  const int pre = (p.w_static && aligned && cta0 < tiles)
                       ? (nk < C::kStages ? nk : C::kStages)
                       : 0;
   if (threadIdx.x == 0) {
-    const int n0 = (static_cast<int>(blockIdx.x) % n_tiles) * BN;
+    const int nb0 = (cta0 % n_tiles) * BN + static_cast<int>(rank) * C::kBRows;
     for (int kb = 0; kb < pre; ++kb) {
-      mbar_expect_tx(bar_full + 8 * kb, C::kStageBytes);
-      tma_load_2d(sB + kb * C::kBBytes, &tmB, bar_full + 8 * kb, kb * kel, n0);
+      if (rank == 0) mbar_expect_tx(bar_full + 8 * kb, full_tx);
+      load(sB + kb * C::kBBytes, &tmB, kb, kb * kel, nb0);
     }
   }
   grid_dep_wait();  // inputs written by the previous kernel; TMEM freed by its CTAs
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
-    tmem_relinquish();
+    if (PAIR) {
+      tmem_alloc_pair(smem_u32(tmem_slot), C::kTmemCols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -185,31 +212,37 @@ __global__ void __launch_bounds__(192, 1)
     // ------------------------------------------------------------ TMA producer
     int it = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
-      const int m0 = (tile / n_tiles) * kBM;
-      const int n0 = (tile % n_tiles) * BN;
+    for (int tile = cta0; tile < tiles && ok; tile += ctas) {
+      const int m0 = (tile / n_tiles) * tile_rows + static_cast<int>(rank) * kBM;
+      const int nb0 = (tile % n_tiles) * BN + static_cast<int>(rank) * C::kBRows;
       for (int kb = 0; kb < nk; ++kb, ++it) {
         const int s = it % C::kStages;
         const uint32_t ph = (it / C::kStages) & 1;
         if (it < pre) {  // W already on its way: the activation half of the stage
-          tma_load_2d(sA + s * C::kABytes, &tmA, bar_full + 8 * s, kb * kel, m0);
+          load(sA + s * C::kABytes, &tmA, s, kb * kel, m0);
           continue;
         }
         if (!mbar_wait(bar_empty + 8 * s, ph ^ 1, p.err, ERR_WAIT_MMA)) { ok = false; break; }
-        mbar_expect_tx(bar_full + 8 * s, C::kStageBytes);
-        tma_load_2d(sA + s * C::kABytes, &tmA, bar_full + 8 * s, kb * kel, m0);
-        tma_load_2d(sB + s * C::kBBytes, &tmB, bar_full + 8 * s, kb * kel, n0);
+        if (rank == 0) mbar_expect_tx(bar_full + 8 * s, full_tx);
+        load(sA + s * C::kABytes, &tmA, s, kb * kel, m0);
+        load(sB + s * C::kBBytes, &tmB, s, kb * kel, nb0);
       }
     }
-    // drain: the loads issued last must land before the CTA may exit
-    for (int j = it - 1; j >= 0 && j >= it - C::kStages; --j)
-      mbar_wait(bar_full + 8 * (j % C::kStages), (j / C::kStages) & 1, p.err, ERR_WAIT_TMA);
-  } else if (aligned && warp == 1 && lane == 0) {
+    // drain: the loads issued last must land before the CTA may exit (pairs: they have once
+    // rank 0's MMAs have read their stages, which releases the stage in both CTAs)
+    for (int j = it - 1; j >= 0 && j >= it - C::kStages; --j) {
+      if (PAIR)
+        mbar_wait(bar_empty + 8 * (j % C::kStages), (j / C::kStages) & 1, p.err, ERR_WAIT_MMA);
+      else
+        mbar_wait(bar_full + 8 * (j % C::kStages), (j / C::kStages) & 1, p.err, ERR_WAIT_TMA);
+    }
+  } else if (aligned && warp == 1 && lane == 0 && rank == 0) {
     // ------------------------------------------------------------ MMA issuer
-    const uint32_t idesc = p.fp8 ? idesc_e4m3_f32(kBM, BN) : idesc_bf16_f32(kBM, BN);
+    const uint32_t idesc =
+        p.fp8 ? idesc_e4m3_f32(tile_rows, BN) : idesc_bf16_f32(tile_rows, BN);
     int it = 0, tc = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++tc) {
+    for (int tile = cta0; tile < tiles && ok; tile += ctas, ++tc) {
       const int acc = tc & 1;
       if (!mbar_wait(bar_tempty + 8 * acc, ((tc >> 1) & 1) ^ 1, p.err, ERR_WAIT_EPI)) break;
       tc_fence_after();
@@ -225,20 +258,30 @@ __global__ void __launch_bounds__(192, 1)
         const uint32_t b0 = sB + s * C::kBBytes;
         if (p.fp8) {
 #pragma unroll
-          for (int k = 0; k < 4; ++k)  // 4 x 32 e4m3 = one 128-byte row
-            mma_e4m3_ss(d_tmem, sdesc_k_sw128(a0 + 32 * k), sdesc_k_sw128(b0 + 32 * k), idesc,
-                        (kb | k) != 0);
+          for (int k = 0; k < 4; ++k) {  // 4 x 32 e4m3 = one 128-byte row
+            const uint64_t da = sdesc_k_sw128(a0 + 32 * k), db = sdesc_k_sw128(b0 + 32 * k);
+            if (PAIR) mma_e4m3_ss_pair(d_tmem, da, db, idesc, (kb | k) != 0);
+            else mma_e4m3_ss(d_tmem, da, db, idesc, (kb | k) != 0);
+          }
         } else {
 #pragma unroll
-          for (int k = 0; k < kBK / 16; ++k)
-            mma_bf16_ss(d_tmem, sdesc_k_sw128(a0 + 32 * k), sdesc_k_sw128(b0 + 32 * k), idesc,
-                        (kb | k) != 0);
+          for (int k = 0; k < kBK / 16; ++k) {
+            const uint64_t da = sdesc_k_sw128(a0 + 32 * k), db = sdesc_k_sw128(b0 + 32 * k);
+            if (PAIR) mma_bf16_ss_pair(d_tmem, da, db, idesc, (kb | k) != 0);
+            else mma_bf16_ss(d_tmem, da, db, idesc, (kb | k) != 0);
+          }
         }
-        mma_commit(bar_empty + 8 * s);  // stage s free once these MMAs have read it
+        // stage s free (in both CTAs of a pair) once these MMAs have read it
+        if (PAIR) mma_commit_pair(bar_empty + 8 * s, 3);
+        else mma_commit(bar_empty + 8 * s);
       }
-      if (ok) mma_commit(bar_tfull + 8 * acc);
+      if (ok) {
+        if (PAIR) mma_commit_pair(bar_tfull + 8 * acc, 3);
+        else mma_commit(bar_tfull + 8 * acc);
+      }
     }
-    mma_commit(bar_done);
+    if (PAIR) mma_commit_pair(bar_done, 1);
+    else mma_commit(bar_done);
     mbar_wait(bar_done, 0, p.err, ERR_WAIT_MMA);
   } else if (aligned && warp >= 2) {
     // ------------------------------------------------------------ epilogue
@@ -268,12 +311,13 @@ __global__ void __launch_bounds__(192, 1)
     int t = 0;
     if (p.epi == EPI_QKV) t = p.qkv.step_dev ? *p.qkv.step_dev : p.qkv.step_host;
     int tc = 0;
-    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++tc) {
+    const uint32_t bar_tempty0 = PAIR ? mapa_rank(bar_tempty, 0) : bar_tempty;
+    for (int tile = cta0; tile < tiles; tile += ctas, ++tc) {
       const int acc = tc & 1;
       const bool got = mbar_wait(bar_tfull + 8 * acc, (tc >> 1) & 1, p.err, ERR_WAIT_MMA);
       if (!__all_sync(0xffffffffu, got)) break;  // leave together: TMEM loads are collective
       tc_fence_after();
-      const int m0 = (tile / n_tiles) * kBM;
+      const int m0 = (tile / n_tiles) * tile_rows + static_cast<int>(rank) * kBM;
       const int n0 = (tile % n_tiles) * BN;
       const int row0 = m0 + quarter * 32;  // first row of this warp's slab
       const int row = m0 + rloc;
@@ -542,48 +586,88 @@ __global__ void __launch_bounds__(192, 1)
       }
       __syncwarp();
       tc_fence_before();
-      mbar_arrive(bar_tempty + 8 * acc);
+      if (PAIR) {  // one arrive per warp on rank 0's barrier
+        if (lane == 0) mbar_arrive_remote(bar_tempty0 + 8 * acc);
+      } else {
+        mbar_arrive(bar_tempty + 8 * acc);
+      }
     }
     if (lane == 0) bulk_wait_all();  // every store has landed before the CTA exits
     __syncwarp();
   }
   grid_dep_launch();
   tc_fence_before();
-  __syncthreads();
+  // pairs: neither CTA leaves (or frees the TMEM columns both hold) before the other is done
+  if (PAIR) cluster_sync();
+  else __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, C::kTmemCols);
+    if (PAIR) tmem_dealloc_pair(tmem, C::kTmemCols);
+    else tmem_dealloc(tmem, C::kTmemCols);
   }
 }
 
-template <int BN>
+template <int BN, bool PAIR>
 static cudaError_t launch_bn(const CUtensorMap& tmA, const CUtensorMap& tmB,
                              const CUtensorMap& tmO, const CUtensorMap& tmK,
                              const CUtensorMap& tmV, const GemmParams& p, int num_sms,
                              cudaStream_t s) {
-  using C = GemmCfg<BN>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
+  using C = GemmCfg<BN, PAIR>;
+  static const cudaError_t attr = cudaFuncSetAttribute(
+      gemm_kernel<BN, PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+  if (attr != cudaSuccess) return attr;
+  const int rows = PAIR ? 2 * kBM : kBM;
+  const int tiles = ((p.M + rows - 1) / rows) * ((p.N + BN - 1) / BN);
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = C::kSmem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[1].id = cudaLaunchAttributeClusterDimension;
+  at[1].val.clusterDim.x = 2;
+  at[1].val.clusterDim.y = 1;
+  at[1].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = PAIR ? 2 : 1;
+  int slots = num_sms;  // CTAs (pairs: CTA pairs) resident at once
+  if (PAIR) {
+    static int pairs = 0;  // CTA pairs that fit at once (one CTA per SM), asked once
+    if (pairs == 0) {
+      cfg.gridDim = dim3(2 * (num_sms / 2));
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel<BN, PAIR>, &cfg) != cudaSuccess || n < 1) {
+        cudaGetLastError();
+        n = num_sms / 2;
+      }
+      pairs = n;
+    }
+    slots = pairs;
   }
-  const int tiles = ((p.M + kBM - 1) / kBM) * ((p.N + BN - 1) / BN);
-  const int grid = tiles < num_sms ? tiles : num_sms;
-  return launch_pdl(gemm_kernel<BN>, dim3(grid), dim3(192), C::kSmem, s, tmA, tmB, tmO, tmK,
-                    tmV, p);
+  const int units = tiles < slots ? tiles : slots;
+  cfg.gridDim = dim3(PAIR ? 2 * units : units);
+  return cudaLaunchKernelEx(&cfg, gemm_kernel<BN, PAIR>, tmA, tmB, tmO, tmK, tmV, p);
 }
 
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmO,
                         const CUtensorMap& tmK, const CUtensorMap& tmV, const GemmParams& p,
-                        int bn, int num_sms, cudaStream_t s) {
+                        int bn, bool pair, int num_sms, cudaStream_t s) {
+  if (pair) {
+    switch (bn) {
+      case 96: return launch_bn<96, true>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+      case 128: return launch_bn<128, true>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+      case 192: return launch_bn<192, true>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+      case 256: return launch_bn<256, true>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   switch (bn) {
-    case 64: return launch_bn<64>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
-    case 96: return launch_bn<96>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
-    case 128: return launch_bn<128>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
-    case 192: return launch_bn<192>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
-    case 256: return launch_bn<256>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+    case 64: return launch_bn<64, false>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+    case 96: return launch_bn<96, false>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+    case 128: return launch_bn<128, false>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+    case 192: return launch_bn<192, false>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
+    case 256: return launch_bn<256, false>(tmA, tmB, tmO, tmK, tmV, p, num_sms, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -120,9 +120,11 @@ struct AttnParams {
 };
 
 // launch wrappers; return cudaGetLastError() of the launch
+// pair: 256-row tiles computed by CTA pairs (cta_group::2; bn 96 / 128 / 192 / 256): tmA
+// boxes of 128 rows as for single CTAs, tmB boxes of bn / 2 rows (each CTA loads half of W)
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmO,
                         const CUtensorMap& tmK, const CUtensorMap& tmV, const GemmParams& p,
-                        int bn, int num_sms, cudaStream_t s);
+                        int bn, bool pair, int num_sms, cudaStream_t s);
 // Attention (+ the combine of key-range splits when p.splits > 1).
 // tmQ: Q [Lq][heads * 64] bf16 in boxes of 64 x 128 rows; tmQ8: the same in boxes of 64 x 8.
 cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmQ8,

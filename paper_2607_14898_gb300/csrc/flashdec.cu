@@ -307,15 +307,33 @@ int pick_bn_step(int M, int N, int step, bool narrow_on_ties = false) {
   }
   return best;
 }
-// fp32 epilogues store 32-column slabs, the others 64-column slabs
-int pick_bn(int M, int N, bool fp32_epilogue) { return pick_bn_step(M, N, fp32_epilogue ? 32 : 64); }
 
 struct Linear {
   __nv_bfloat16* w = nullptr;  // [N][K]
   float* b = nullptr;          // [N]
   int N = 0, K = 0, bn = 128;
+  bool pair = false;           // 256-row tiles on CTA pairs (W boxes of bn / 2 rows)
   CUtensorMap tm;
 };
+
+// Launch shape of an M x N x K product. CTA pairs (256 x 256 tiles, each SM holding half of W)
+// measured 4-10 % faster than the best single-CTA tile once there are at least 2.5 rounds of
+// pair tiles, and slower on the smaller products, where a tile's fixed costs dominate; there
+// the single-CTA width model of pick_bn_step (which matches the measured best width) decides.
+struct TileChoice {
+  int bn;
+  bool pair;
+};
+TileChoice pick_tile(int M, int N, int K, int step, bool fp8, int force_pair = 0) {
+  (void)K;
+  (void)fp8;
+  const int sms = num_sms();
+  const long long pair_tiles = static_cast<long long>((M + 255) / 256) * ((N + 255) / 256);
+  const bool pair = force_pair == 2 ||
+                    (force_pair == 0 && 256 % step == 0 && 2 * pair_tiles >= 5LL * (sms / 2));
+  if (pair) return {256, true};
+  return {pick_bn_step(M, N, step), false};
+}
 
 struct LayerW {
   float *g1 = nullptr, *g2 = nullptr, *kg = nullptr, *vg = nullptr;
@@ -473,7 +491,7 @@ fd_status run_linear(fd_handle h, int kind, const CUtensorMap& tmA, const Linear
   const CUtensorMap& k = tmK ? *tmK : tmO;
   const CUtensorMap& v = tmV ? *tmV : tmO;
   return traced(h, kind, s, [&] {
-    return fd::launch_gemm(tmA, lin.tm, tmO, k, v, p, lin.bn, num_sms(), s);
+    return fd::launch_gemm(tmA, lin.tm, tmO, k, v, p, lin.bn, lin.pair, num_sms(), s);
   });
 }
 
@@ -826,8 +844,11 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
     lin.b = reinterpret_cast<float*>(next());
     lin.N = N;
     lin.K = K;
-    lin.bn = pick_bn(M, N, fp32_epi);
-    return tmap_bf16(&lin.tm, lin.w, K, N, static_cast<uint64_t>(K) * 2, fd::kBK, lin.bn);
+    const TileChoice t = pick_tile(M, N, K, fp32_epi ? 32 : 64, false);
+    lin.bn = t.bn;
+    lin.pair = t.pair;
+    return tmap_bf16(&lin.tm, lin.w, K, N, static_cast<uint64_t>(K) * 2, fd::kBK,
+                     lin.pair ? lin.bn / 2 : lin.bn);
   };
   // FP8 linear: e4m3 weight [N][K] in boxes of 128 bytes (= 128 K elements)
   auto linear_e4m3 = [&](Linear& lin, int N, int K, int M, int step) -> bool {
@@ -837,6 +858,7 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
     lin.K = K;
     // the e4m3 GELU epilogue outweighs the FP8 MMAs: narrower tiles overlap it better
     lin.bn = pick_bn_step(M, N, step, step == 128);
+    lin.pair = false;
     return tmap_e4m3(&lin.tm, lin.w, K, N, K, lin.bn);
   };
   bool ok = linear(w->embed, d.D, d.cin, d.L, true);
@@ -886,9 +908,12 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
     }
     ok = ok && linear(lw.mlp1, (d.gated ? 2 : 1) * d.Mr * d.D, d.D, M, false);
     if (d.gated) {  // EPI_SWIGLU works on 128-column steps
-      lw.mlp1.bn = pick_bn_step(M, lw.mlp1.N, 128);
+      const TileChoice t = pick_tile(M, lw.mlp1.N, d.D, 128, false);
+      lw.mlp1.bn = t.bn;
+      lw.mlp1.pair = t.pair;
       ok = ok && tmap_bf16(&lw.mlp1.tm, lw.mlp1.w, d.D, lw.mlp1.N,
-                           static_cast<uint64_t>(d.D) * 2, fd::kBK, lw.mlp1.bn);
+                           static_cast<uint64_t>(d.D) * 2, fd::kBK,
+                           lw.mlp1.pair ? lw.mlp1.bn / 2 : lw.mlp1.bn);
     }
     ok = ok && linear(lw.mlp2, d.D, d.Mr * d.D, M, true);
   };
@@ -1307,6 +1332,14 @@ fd_status fd_debug_read_ring(fd_handle h, int which, int layer, void* dst_host,
 fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const void* W,
                        const float* bias, void* out, int tup_hidden, int bn, int* err_dev,
                        void* stream) {
+  return fd_op_linear_tiled(epilogue, M, N, K, A, W, bias, out, tup_hidden, bn, bn ? 1 : 0,
+                            err_dev, stream);
+}
+
+fd_status fd_op_linear_tiled(int epilogue, int M, int N, int K, const void* A, const void* W,
+                             const float* bias, void* out, int tup_hidden, int bn, int pair,
+                             int* err_dev, void* stream) {
+  if (pair < 0 || pair > 2) return FD_ERR_INVALID_ARG;
   if (M < 1 || N < 1 || K < 1 || A == nullptr || W == nullptr || bias == nullptr ||
       out == nullptr || err_dev == nullptr)
     return FD_ERR_INVALID_ARG;
@@ -1317,8 +1350,14 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
   if (epilogue == FD_EPI_SWIGLU && N % 128) return FD_ERR_INVALID_ARG;
   const bool bf16_out = epilogue == FD_EPI_GELU || epilogue == FD_EPI_SWIGLU;
   const int epi = epilogue == FD_EPI_SWIGLU ? fd::EPI_SWIGLU : epilogue;
-  if (bn == 0) bn = pick_bn_step(M, N, epilogue == FD_EPI_SWIGLU ? 128 : bf16_out ? 64 : 32);
-  if (!fd::gemm_bn_supported(bn) || !fd::gemm_bn_fits_epilogue(bn, epi))
+  const int step = epilogue == FD_EPI_SWIGLU ? 128 : bf16_out ? 64 : 32;
+  if (bn == 0) {
+    const TileChoice t = pick_tile(M, N, K, step, false, pair);
+    bn = t.bn;
+    pair = t.pair ? 2 : 1;
+  }
+  if (pair == 0) pair = 1;
+  if (!fd::gemm_bn_supported(bn) || !fd::gemm_bn_fits_epilogue(bn, epi) || (pair == 2 && bn < 96))
     return FD_ERR_INVALID_ARG;
   if (epilogue == FD_EPI_TUP && (tup_hidden < 32 || tup_hidden % 32 || N % tup_hidden))
     return FD_ERR_INVALID_ARG;
@@ -1326,7 +1365,7 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
   if (st) return st;
   CUtensorMap ta, tb;
   if (!tmap_bf16(&ta, A, K, M, static_cast<uint64_t>(K) * 2, 64, 128) ||
-      !tmap_bf16(&tb, W, K, N, static_cast<uint64_t>(K) * 2, 64, bn))
+      !tmap_bf16(&tb, W, K, N, static_cast<uint64_t>(K) * 2, 64, pair == 2 ? bn / 2 : bn))
     return FD_ERR_CUDA;
   CUtensorMap to;
   bool ok;
@@ -1345,7 +1384,7 @@ fd_status fd_op_linear(int epilogue, int M, int N, int K, const void* A, const v
   p.ld_out = epilogue == FD_EPI_SWIGLU ? N / 2 : N;
   p.tup_tokens = M;
   p.tup_hidden = tup_hidden;
-  return launch_ok(fd::launch_gemm(ta, tb, to, to, to, p, bn, num_sms(),
+  return launch_ok(fd::launch_gemm(ta, tb, to, to, to, p, bn, pair == 2, num_sms(),
                                    static_cast<cudaStream_t>(stream)));
 }
 
@@ -1364,15 +1403,20 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
   if (ring_pitch < window * M || ring_pitch % 128) return FD_ERR_INVALID_ARG;
   if (!aligned16(q_out) || !aligned16(k_ring) || !aligned16(vt_ring) || !aligned16(bqkv))
     return FD_ERR_INVALID_ARG;
-  if (bn == 0) bn = 128;
+  const int N = (heads + 2 * groups) * kHeadDim;
+  bool pair = false;  // an explicit width runs on single CTAs; 0 = the launch-shape model
+  if (bn == 0) {
+    const TileChoice t = pick_tile(M, N, K, 64, false);
+    bn = t.bn;
+    pair = t.pair;
+  }
   if (!fd::gemm_bn_supported(bn) || !fd::gemm_bn_fits_epilogue(bn, fd::EPI_QKV))
     return FD_ERR_INVALID_ARG;
   fd_status st = check_device();
   if (st) return st;
-  const int N = (heads + 2 * groups) * kHeadDim;
   CUtensorMap ta, tb;
   if (!tmap_bf16(&ta, A, K, M, static_cast<uint64_t>(K) * 2, 64, 128) ||
-      !tmap_bf16(&tb, Wqkv, K, N, static_cast<uint64_t>(K) * 2, 64, bn))
+      !tmap_bf16(&tb, Wqkv, K, N, static_cast<uint64_t>(K) * 2, 64, pair ? bn / 2 : bn))
     return FD_ERR_CUDA;
   fd::GemmParams p{};
   p.M = M; p.N = N; p.K = K; p.epi = fd::EPI_QKV; p.bias = bqkv; p.err = err_dev;
@@ -1398,7 +1442,7 @@ fd_status fd_op_qkv(int M, int K, const void* A, const void* Wqkv, const float* 
   } else {
     tv = tk;
   }
-  return launch_ok(fd::launch_gemm(ta, tb, tq, tk, tv, p, bn, num_sms(),
+  return launch_ok(fd::launch_gemm(ta, tb, tq, tk, tv, p, bn, pair, num_sms(),
                                    static_cast<cudaStream_t>(stream)));
 }
 
@@ -1580,7 +1624,7 @@ fd_status fd_op_linear_e4m3(int epilogue, int M, int N, int K, const void* A, co
   if (f8_out) p.out_f8 = static_cast<uint8_t*>(out);
   else p.out_f32 = static_cast<float*>(out);
   p.ld_out = n_out;
-  return launch_ok(fd::launch_gemm(ta, tb, to, to, to, p, bn, num_sms(),
+  return launch_ok(fd::launch_gemm(ta, tb, to, to, to, p, bn, false, num_sms(),
                                    static_cast<cudaStream_t>(stream)));
 }
 

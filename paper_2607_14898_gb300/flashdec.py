@@ -72,6 +72,7 @@ _SIGS = {
     "fd_save_state": (_I, [_P, _P, ctypes.c_size_t, _P]),
     "fd_load_state": (_I, [_P, _P, ctypes.c_size_t, _P]),
     "fd_op_linear": (_I, [_I, _I, _I, _I, _P, _P, _P, _P, _I, _I, _P, _P]),
+    "fd_op_linear_tiled": (_I, [_I, _I, _I, _I, _P, _P, _P, _P, _I, _I, _I, _P, _P]),
     "fd_op_rope_table": (_I, [_I, _I, _F, _P, _P]),
     "fd_op_qkv": (_I, [_I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _F, _F,
                        _P, _P, _P, _P, _I, _I, _P, _P]),
@@ -287,11 +288,18 @@ def decode_chunks(decoders, latents, pixels, stream=None) -> None:
 
 
 # ------------------------------------------------------------------ kernel-level entry points
-def op_linear(epi, A, W, bias, out, tup_hidden=0, bn=0, err=None, stream=None) -> None:
+def op_linear(epi, A, W, bias, out, tup_hidden=0, bn=0, err=None, stream=None, pair=None
+              ) -> None:
+    """pair: None (fd_op_linear), or 0 / 1 / 2 (library choice / single CTAs / CTA pairs)."""
     M, K = A.shape
     N = W.shape[0]
-    _check(lib().fd_op_linear(epi, M, N, K, _ptr(A), _ptr(W), _ptr(bias), _ptr(out),
-                              tup_hidden, bn, _ptr(err), _stream_ptr(stream)), "fd_op_linear")
+    if pair is None:
+        _check(lib().fd_op_linear(epi, M, N, K, _ptr(A), _ptr(W), _ptr(bias), _ptr(out),
+                                  tup_hidden, bn, _ptr(err), _stream_ptr(stream)), "fd_op_linear")
+    else:
+        _check(lib().fd_op_linear_tiled(epi, M, N, K, _ptr(A), _ptr(W), _ptr(bias), _ptr(out),
+                                        tup_hidden, bn, pair, _ptr(err), _stream_ptr(stream)),
+               "fd_op_linear_tiled")
 
 
 def op_rope_table(t, frames_per_chunk, rope_base, table, stream=None) -> None:

@@ -59,6 +59,42 @@ def test_linear_f32(M, N, K, bn):
     assert_close_scaled(out, want, 2e-5, "linear f32")
 
 
+@pytest.mark.parametrize("M,N,K,bn", [
+    (1560, 4096, 1024, 256),  # 480p MLP layer 1 shape: 7 pair tiles of 256 rows, ragged last
+    (1560, 1024, 4096, 128),  # 480p MLP layer 2 shape, long K
+    (300, 608, 512, 96),      # ragged M and N; the second CTA of the last pair has no rows
+    (6240, 1536, 1024, 192),  # refinement QKV shape, several tiles per pair (persistent)
+    (130, 256, 64, 128),      # one K block
+])
+def test_linear_cta_pairs(M, N, K, bn):
+    """256-row tiles on CTA pairs (tcgen05 cta_group::2; each CTA holds half of W) compute the
+    same products as single CTAs: fp32, residual and GELU epilogues against the oracle, and
+    bit-identical to the single-CTA launch of the same width."""
+    A, W, b = linear_case(M, N, K, seed=M + 5 * N + K)
+    Ad, Wd, bd = dev(A, torch.bfloat16), dev(W, torch.bfloat16), dev(b)
+    err = err_word()
+    out = {}
+    for pair in (1, 2):
+        o = torch.zeros(M, N, device="cuda")
+        fdp.op_linear(fdp.EPI_F32, Ad, Wd, bd, o, bn=bn, err=err, pair=pair)
+        check_err(err)
+        out[pair] = o
+    want = oracle.linear(f64(A), f64(W), f64(b))
+    assert_close_scaled(out[2], want, 2e-5, f"pair linear f32 bn={bn}")
+    assert torch.equal(out[1], out[2])
+    h = torch.ones(M, N, device="cuda")
+    fdp.op_linear(fdp.EPI_RESID, Ad, Wd, bd, h, bn=bn, err=err, pair=2)
+    check_err(err)
+    assert torch.equal(h, out[1] + 1.0)
+    if bn % 64 == 0:
+        g1 = torch.zeros(M, N, dtype=torch.bfloat16, device="cuda")
+        g2 = torch.zeros(M, N, dtype=torch.bfloat16, device="cuda")
+        fdp.op_linear(fdp.EPI_GELU, Ad, Wd, bd, g1, bn=bn, err=err, pair=1)
+        fdp.op_linear(fdp.EPI_GELU, Ad, Wd, bd, g2, bn=bn, err=err, pair=2)
+        check_err(err)
+        assert torch.equal(g1, g2)
+
+
 def test_gelu_epilogue_is_the_exact_erf_gelu_at_bf16():
     """The GELU epilogue evaluates erf with Abramowitz & Stegun 7.1.26 (error <= 1.5e-7): on a
     grid of pre-activations from -8 to 8 (A holds x in one column, W picks it, the bias shifts
