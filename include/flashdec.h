@@ -89,6 +89,7 @@ typedef struct {
 
 typedef struct fd_weights_s* fd_weights;
 typedef struct fd_handle_s* fd_handle;
+typedef struct fd_batch_s* fd_batch;
 
 /* ------------------------------------------------------------------ sizes */
 
@@ -155,6 +156,27 @@ fd_status fd_decode_chunk(fd_handle h, const float* latent_dev, void* pixels_dev
  * the chunks run concurrently. All arguments are checked before anything is enqueued. */
 fd_status fd_decode_chunks(fd_handle* hs, int n, const float* const* latents_dev,
                            void* const* pixels_dev, void* stream);
+
+/* Batched decode (Sec. 4.6: independent streams share one set of weights). A batch object
+ * owns stacked activation scratch for up to max_streams (1..64) streams of cfg: each stream's
+ * L tokens are padded to Lp = 128 * ceil(L / 128) rows per frame, so every GEMM of a chunk
+ * runs once on the rows of all streams, while attention and the pixel head run per stream on
+ * that stream's own KV cache. The streams' states (KV rings, chunk counters) stay in their
+ * fd_handles, created with the same weights object. Synchronous; counts as a user of w. */
+fd_status fd_batch_create(const fd_config* cfg, fd_weights w, int max_streams, fd_batch* out);
+
+/* Decode chunk t_i of each of n (1..max_streams) distinct handles through the batch object
+ * and advance each t_i; the handles may be at different t. Pixels and latents as for
+ * fd_decode_chunk (device, 16-byte aligned). Stream-ordered on `stream`, no host wait except
+ * when the set of handles differs from the previous call (the batch's per-layer stream table
+ * is then rewritten after a stream synchronisation). All arguments are checked before
+ * anything is enqueued; a launch failure puts every handle of the call in the error state.
+ * Calls with the same batch object must not overlap on different streams. */
+fd_status fd_decode_batch(fd_batch b, fd_handle* hs, int n, const float* const* latents_dev,
+                          void* const* pixels_dev, void* stream);
+
+/* Free the batch object (after a device synchronisation). */
+fd_status fd_batch_destroy(fd_batch b);
 
 /* Like fd_decode_chunk, with the latent and the pixels in HOST memory (pinned for
  * asynchronous copies): the latent is copied into a library-owned device buffer, decoded, and

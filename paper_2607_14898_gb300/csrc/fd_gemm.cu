@@ -106,12 +106,12 @@ __device__ __forceinline__ float silu(float x) { return __fdividef(x, 1.0f + __e
 // then column; angle = position * base^(-2i/d_band)). Temporal values come from the chunk's
 // table (fp64-evaluated, any stream length); row / column angles are below 2^12 rad, reduced to
 // [-pi, pi] in fp32 (2 pi split in two parts) and evaluated with the fast sin / cos.
-__device__ __forceinline__ void rope_table(const QkvEpi& q, int tau, int y, int x, float* c,
-                                           float* s) {
+__device__ __forceinline__ void rope_table(const QkvEpi& q, const float2* rope_t, int tau, int y,
+                                           int x, float* c, float* s) {
 #pragma unroll
   for (int i = 0; i < kRopePairs; ++i) {
     if (i < q.band_t) {
-      const float2 v = __ldg(q.rope_t + tau * q.band_t + i);
+      const float2 v = __ldcg(rope_t + tau * q.band_t + i);
       c[i] = v.x;
       s[i] = v.y;
     } else {
@@ -327,12 +327,33 @@ __global__ void __launch_bounds__(192, 1)
 
       if (p.epi == EPI_QKV) {
         const QkvEpi& q = p.qkv;
-        float rc[kRopePairs], rsn[kRopePairs];
-        const int rows_chunk = q.frames_per_chunk * q.tokens;  // = M
-        const int slot = t % q.window;
-        if (row_ok) {
+        float rc[kRopePairs], rsn[kRopePairs];  // identity rotation for rows past M / padding
+#pragma unroll
+        for (int i = 0; i < kRopePairs; ++i) {
+          rc[i] = 1.0f;
+          rsn[i] = 0.0f;
+        }
+        const int rows_chunk = q.frames_per_chunk * q.tokens;  // = M (single stream)
+        int slot = t % q.window;
+        // batched: this row's stream, frame and token, its ring row (or -1 for padding)
+        int ring_row = -1;
+        __nv_bfloat16* k_ring = q.k_ring;
+        __half* vt_ring = q.vt_ring;
+        if (q.streams > 0) {
+          const int si = row / q.stream_rows, loc = row - si * q.stream_rows;
+          const int tau = loc / q.frame_rows, l = loc - tau * q.frame_rows;
+          if (row_ok && si < q.streams && l < q.tokens) {
+            const QkvStream st = q.stream[si];
+            slot = *st.step_dev % q.window;
+            ring_row = slot * rows_chunk + tau * q.tokens + l;
+            k_ring = st.k_ring;
+            vt_ring = st.vt_ring;
+            rope_table(q, st.rope_t, tau, l / q.grid_w, l % q.grid_w, rc, rsn);
+          }
+        } else if (row_ok) {
           const int l = row % q.tokens;
-          rope_table(q, row / q.tokens, l / q.grid_w, l % q.grid_w, rc, rsn);
+          rope_table(q, q.rope_t, row / q.tokens, l / q.grid_w, l % q.grid_w, rc, rsn);
+          ring_row = slot * rows_chunk + row;
         }
 #pragma unroll 1
         for (int c = 0; c < BN; c += 64) {
@@ -376,6 +397,17 @@ __global__ void __launch_bounds__(192, 1)
             uint32_t w[32];
 #pragma unroll
             for (int j = 0; j < 32; ++j) w[j] = pack_bf16x2(v[2 * j], v[2 * j + 1]);
+            if (!is_q && q.streams > 0) {  // batched: K row straight into its stream's ring
+              if (ring_row >= 0) {
+                uint4* dst = reinterpret_cast<uint4*>(
+                    k_ring + (static_cast<size_t>(hidx - q.heads) * q.ring_pitch + ring_row) *
+                                 kHeadDim);
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                  dst[k] = make_uint4(w[4 * k], w[4 * k + 1], w[4 * k + 2], w[4 * k + 3]);
+              }
+              continue;
+            }
             uint8_t* buf = acquire();
             put_row_sw128(buf, lane, w);
             publish();
@@ -387,7 +419,7 @@ __global__ void __launch_bounds__(192, 1)
               }
               bulk_commit();
             }
-          } else if (p.v_tma) {
+          } else if (p.v_tma && q.streams == 0) {
             // V transposed: slab [64 dims][32 keys] fp16, stored into the ring's V^T slot view
             uint8_t* buf = acquire();
             __half* sv = reinterpret_cast<__half*>(buf);
@@ -398,10 +430,9 @@ __global__ void __launch_bounds__(192, 1)
               tma_store_4d(&tmV, smem_u32(buf), row0, slot, 0, hidx - q.heads - q.groups);
               bulk_commit();
             }
-          } else if (row_ok) {
+          } else if (ring_row >= 0) {  // V^T column by column (keys of a warp are adjacent)
             const int g = hidx - q.heads - q.groups;
-            __half* dst = q.vt_ring + static_cast<size_t>(g) * kHeadDim * q.ring_pitch +
-                          slot * rows_chunk + row;
+            __half* dst = vt_ring + static_cast<size_t>(g) * kHeadDim * q.ring_pitch + ring_row;
 #pragma unroll
             for (int j = 0; j < 64; ++j)
               dst[static_cast<size_t>(j) * q.ring_pitch] = __float2half_rn(v[j]);
@@ -576,7 +607,9 @@ __global__ void __launch_bounds__(192, 1)
               tma_reduce_add_2d(&tmO, smem_u32(buf), col, row0);
             } else if (p.epi == EPI_TUP) {
               const int tau = col / p.tup_hidden;
-              tma_store_3d(&tmO, smem_u32(buf), col - tau * p.tup_hidden, row0, tau);
+              // rows stack streams of tup_tokens rows each: [stream][tau][token][channel]
+              tma_store_4d(&tmO, smem_u32(buf), col - tau * p.tup_hidden, row0 % p.tup_tokens,
+                           tau, row0 / p.tup_tokens);
             } else {
               tma_store_2d(&tmO, smem_u32(buf), col, row0);
             }

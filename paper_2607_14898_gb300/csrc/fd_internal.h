@@ -45,6 +45,14 @@ enum EpiKind : int {
                       // (acc * col_scale + bias) of the interleaved gate / up columns
 };
 
+// One stream of a batched QKV launch: its cache ring, chunk counter and temporal RoPE table.
+struct QkvStream {
+  __nv_bfloat16* k_ring;     // [groups][ring_pitch][64]
+  __half* vt_ring;           // [groups][64][ring_pitch]
+  const int* step_dev;       // chunk index t of the stream
+  const float2* rope_t;      // [frames_per_chunk][band_t] of the stream's chunk
+};
+
 // Rotary / cache parameters of the fused QKV epilogue.
 struct QkvEpi {
   int qk_norm;  // 0: RMSNorm K (knorm_g) and V (vnorm_g); 1: Q (vnorm_g holds Q's gain) and K
@@ -65,6 +73,12 @@ struct QkvEpi {
   int band_t, band_s;        // pairs in the temporal band and in each spatial band
   const float2* rope_t;      // [frames_per_chunk][band_t] (cos, sin) of this chunk's frames
   float inv_freq_s[kRopePairs];  // base^(-2i/d_band) of the row / column pairs (fp32)
+  // batched launch (streams > 0): the rows stack `streams` independent streams, stream_rows rows
+  // each (frames_per_chunk blocks of frame_rows >= tokens rows; rows past `tokens` in a block
+  // are padding and append nothing); ring, counter and RoPE table come from stream[i], and K /
+  // V are stored row by row (the single-stream fields above are unused)
+  int streams, stream_rows, frame_rows;
+  const QkvStream* stream;
 };
 
 // Output of the GEMM epilogue goes through TMA bulk stores with these tensor maps (all boxes
@@ -163,8 +177,9 @@ cudaError_t launch_rmsnorm(const float* h, const float* g, int M, int D, float e
 // u[r][c] = e4m3(rmsnorm(h)[r][c] * oscale)  (FP8 MLP input)
 cudaError_t launch_rmsnorm_e4m3(const float* h, const float* g, int M, int D, float eps,
                                 uint8_t* u, float oscale, cudaStream_t s);
+// frame_rows: F rows per refined frame (0 = gh gw, the tokens of a frame)
 cudaError_t launch_pixel_head(const float* F, int frames, int gh, int gw, int C, int rs,
-                              int out_u8, void* pix, cudaStream_t s);
+                              int out_u8, void* pix, cudaStream_t s, int frame_rows = 0);
 cudaError_t launch_kv_append(const float* k, const float* v, int groups, int rows, int slot,
                              int ring_pitch, __nv_bfloat16* k_ring, __half* vt_ring,
                              cudaStream_t s);

@@ -111,12 +111,12 @@ __device__ __forceinline__ uint32_t quant_u8(float x) {
 }
 
 // pix[c][tau][y][x] = clamp(F[tau*L + (y/rs)*gw + x/rs][c*rs*rs + (y%rs)*rs + x%rs]); rs % 4 == 0
-__global__ void pixel_head_kernel(const float* __restrict__ F, int frames, int gh, int gw, int C,
-                                  int rs, int out_u8, void* __restrict__ pix) {
+// frame tau's tokens are rows tau * frame_rows .. + gh gw - 1 of F (frame_rows >= gh gw)
+__global__ void pixel_head_kernel(const float* __restrict__ F, int frames, int frame_rows, int gh,
+                                  int gw, int C, int rs, int out_u8, void* __restrict__ pix) {
   grid_dep_wait();
   grid_dep_launch();
   const int Wo = gw * rs, Ho = gh * rs;
-  const int L = gh * gw;
   const int ld = C * rs * rs;
   const int q_per_row = Wo / 4;
   const long long total = static_cast<long long>(C) * frames * Ho * q_per_row;
@@ -129,7 +129,7 @@ __global__ void pixel_head_kernel(const float* __restrict__ F, int frames, int g
     const int tau = static_cast<int>(r % frames);
     const int c = static_cast<int>(r / frames);
     const int x = 4 * xq;
-    const int tok = tau * L + (y / rs) * gw + x / rs;
+    const int tok = tau * frame_rows + (y / rs) * gw + x / rs;
     const int ch = c * rs * rs + (y % rs) * rs + (x % rs);
     const float4 v = *reinterpret_cast<const float4*>(F + static_cast<size_t>(tok) * ld + ch);
     const size_t o = ((static_cast<size_t>(c) * frames + tau) * Ho + y) * Wo + x;
@@ -232,10 +232,11 @@ cudaError_t launch_rmsnorm_e4m3(const float* h, const float* g, int M, int D, fl
 }
 
 cudaError_t launch_pixel_head(const float* F, int frames, int gh, int gw, int C, int rs,
-                              int out_u8, void* pix, cudaStream_t s) {
+                              int out_u8, void* pix, cudaStream_t s, int frame_rows) {
   const long long total = static_cast<long long>(C) * frames * gh * rs * gw * rs / 4;
-  return launch_pdl(pixel_head_kernel, dim3(grid_for(total, 256)), dim3(256), 0, s, F, frames, gh,
-                    gw, C, rs, out_u8, pix);
+  if (frame_rows == 0) frame_rows = gh * gw;
+  return launch_pdl(pixel_head_kernel, dim3(grid_for(total, 256)), dim3(256), 0, s, F, frames,
+                    frame_rows, gh, gw, C, rs, out_u8, pix);
 }
 
 cudaError_t launch_kv_append(const float* k, const float* v, int groups, int rows, int slot,

@@ -6,6 +6,7 @@
 #include <cuda_fp8.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
@@ -108,11 +109,13 @@ bool tmap_out_bf16(CUtensorMap* m, const void* base, uint64_t cols, uint64_t row
   return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box,
                  CU_TENSOR_MAP_SWIZZLE_128B);
 }
-// temporal upsampling output viewed as [r_t][L][D]
-bool tmap_out_tup(CUtensorMap* m, const void* base, uint64_t D, uint64_t L, uint64_t rt) {
-  const uint64_t dims[3] = {D, L, rt}, strides[2] = {D * 4, L * D * 4};
-  const uint32_t box[3] = {32, 32, 1};
-  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base, dims, strides, box,
+// temporal upsampling output viewed as [streams][r_t][L][D] (L rows per refined frame)
+bool tmap_out_tup(CUtensorMap* m, const void* base, uint64_t D, uint64_t L, uint64_t rt,
+                  uint64_t streams = 1) {
+  const uint64_t dims[4] = {D, L, rt, streams};
+  const uint64_t strides[3] = {D * 4, L * D * 4, rt * L * D * 4};
+  const uint32_t box[4] = {32, 32, 1, 1};
+  return tmap_nd(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, base, dims, strides, box,
                  CU_TENSOR_MAP_SWIZZLE_128B);
 }
 // K ring [G][pitch][64] viewed as {64, M rows of a slot, W slots, G}
@@ -410,6 +413,33 @@ struct fd_handle_s {
   size_t ev_used = 0;
 };
 
+// Batched decode of independent streams (fd_decode_batch): the streams' tokens are stacked,
+// each stream's rows padded to a multiple of 128 (Lp per frame), so that every GEMM runs once
+// on all of them and no tile or 32-row slab holds two streams; attention and the pixel head
+// run per stream on the streams' own caches.
+struct fd_batch_s {
+  fd_config cfg;
+  Dims d;
+  fd_weights w = nullptr;
+  int nmax = 0, Lp = 0, Rp = 0;  // streams; padded rows per stream (backbone, refinement)
+  void* arena = nullptr;
+  __nv_bfloat16 *x0 = nullptr, *u = nullptr, *q = nullptr, *o = nullptr, *hid = nullptr;
+  float *h = nullptr, *hf = nullptr, *F = nullptr, *attn_ws = nullptr;
+  float2* rope = nullptr;               // [nmax][(1 + r_t) band_t] temporal RoPE per stream
+  fd::QkvStream* table = nullptr;       // [n_blocks + n_refine][nmax] on the device
+  fd::QkvStream* table_host = nullptr;  // pinned copy
+  std::vector<fd_handle> table_for;     // handles the table was written for
+  int partsB = 1, partsR = 1;
+  CUtensorMap tm_x0, tm_uB, tm_uR, tm_oB, tm_oR, tm_hidB, tm_hidR, tm_hidH;
+  CUtensorMap so_h, so_hf, so_tup, so_hidB, so_hidR, so_hidH, so_F, so_qB, so_qR;
+  CUtensorMap tm_u8B, tm_u8R, tm_hid8B, tm_hid8R, so_hid8B, so_hid8R;
+  std::vector<CUtensorMap> tm_qB, tm_q8B, tm_qR, tm_q8R;  // each stream's Q rows
+  // the weights' products with launch shapes re-chosen for the stacked row counts (same
+  // device weights; only the tile width, CTA pairing and W descriptor differ)
+  Linear embed, tup, head1, head2;
+  std::vector<LayerW> blocks, refine;
+};
+
 namespace {
 
 double rope_inv_freq(int i, int band_t, int band_s, double base) {
@@ -647,6 +677,225 @@ fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Re-choose the launch shape of a product of the weights for M rows (as fd_weights_create
+// does for one stream's rows); step: the epilogue's column step, e4m3: FP8 weight
+bool retile(Linear& lin, int M, int step, bool e4m3) {
+  if (e4m3) {
+    lin.bn = pick_bn_step(M, lin.N, step, step == 128);
+    lin.pair = false;
+    return tmap_e4m3(&lin.tm, lin.w, lin.K, lin.N, lin.K, lin.bn);
+  }
+  const TileChoice t = pick_tile(M, lin.N, lin.K, step, false);
+  lin.bn = t.bn;
+  lin.pair = t.pair;
+  return tmap_bf16(&lin.tm, lin.w, lin.K, lin.N, static_cast<uint64_t>(lin.K) * 2, fd::kBK,
+                   lin.pair ? lin.bn / 2 : lin.bn);
+}
+
+bool retile_block(LayerW& lw, const Dims& d, int M) {
+  bool ok = retile(lw.qkv, M, 64, false) && retile(lw.out, M, 32, false);
+  if (d.fp8)
+    return ok && retile(lw.mlp1, M, d.gated ? 256 : 128, true) && retile(lw.mlp2, M, 32, true);
+  return ok && retile(lw.mlp1, M, d.gated ? 128 : 64, false) && retile(lw.mlp2, M, 32, false);
+}
+
+// ---------------------------------------------------------------- batched decode
+// One Transformer block on the stacked rows of n streams (see fd_batch_s): the GEMMs and the
+// norms run once on n * rows_s rows; the QKV epilogue appends each stream's K / V to its own
+// ring (padding rows append nothing); attention runs once per stream on its own cache.
+fd_status batch_block(fd_batch b, fd_handle* hs, int n, int layer, bool refine, cudaStream_t s) {
+  const Dims& d = b->d;
+  fd_handle h0 = hs[0];  // launches of the stacked kernels are traced on the first stream
+  const LayerW& lw = refine ? b->refine[layer] : b->blocks[layer];
+  const int rows_s = refine ? b->Rp : b->Lp;
+  const int M = n * rows_s;
+  float* hbuf = refine ? b->hf : b->h;
+  const int D = d.D;
+  const float eps = h0->cfg.norm_eps;
+  const uint64_t NQ = static_cast<uint64_t>(d.N) * kHeadDim;
+  fd_status st;
+  {
+    const float* g1 = lw.g1;
+    __nv_bfloat16* u = b->u;
+    if ((st = traced(h0, FD_K_RMSNORM, s,
+                     [&] { return fd::launch_rmsnorm(hbuf, g1, M, D, eps, u, s); })))
+      return st;
+  }
+  fd::GemmParams p{};
+  p.epi = fd::EPI_QKV;
+  fd::QkvEpi& q = p.qkv;
+  q.heads = d.N; q.groups = d.G; q.knorm_g = lw.kg; q.vnorm_g = lw.vg; q.q_out = b->q;
+  q.qk_norm = d.qk ? 1 : 0;
+  q.ring_pitch = refine ? h0->pitchR : h0->pitchB; q.tokens = d.L; q.grid_w = d.gw;
+  q.frames_per_chunk = refine ? d.rt : 1; q.window = d.Wn; q.eps = eps;
+  fill_rope(q, h0->cfg.rope_base);
+  q.streams = n;
+  q.stream_rows = rows_s;
+  q.frame_rows = b->Lp;
+  q.stream = b->table + static_cast<size_t>(refine ? d.nb + layer : layer) * b->nmax;
+  p.v_tma = 0;
+  const CUtensorMap& so_q = refine ? b->so_qR : b->so_qB;
+  if ((st = run_linear(h0, FD_K_QKV, refine ? b->tm_uR : b->tm_uB, lw.qkv, M, p, so_q, s, &so_q,
+                       &so_q)))
+    return st;
+  const int pairs = std::max(fd::attention_units(d.L, d.N, d.G),
+                             fd::attention_units(b->Rp, d.N, d.G));
+  for (int i = 0; i < n; ++i) {
+    fd_handle hi = hs[i];
+    Ring& r = refine ? hi->ringR[layer] : hi->ringB[layer];
+    fd::AttnParams a{};
+    a.Lq = refine ? b->Rp : d.L;
+    a.heads = d.N; a.groups = d.G; a.ring_pitch = q.ring_pitch;
+    a.rows_per_chunk = refine ? d.rt * d.L : d.L;
+    a.window = d.Wn; a.step_dev = hi->state; a.n_keys_host = 0;
+    a.out = b->o + static_cast<size_t>(i) * rows_s * NQ;
+    a.ld_out = static_cast<int>(NQ); a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
+    a.err = hi->state + 1;
+    a.lq_pad = fd::attention_lq_pad(a.Lq);
+    a.parts = refine ? b->partsR : b->partsB;
+    fd::attention_workspace_split(b->attn_ws, a.parts, pairs, a);
+    const CUtensorMap& tq = refine ? b->tm_qR[i] : b->tm_qB[i];
+    const CUtensorMap& tq8 = refine ? b->tm_q8R[i] : b->tm_q8B[i];
+    if ((st = traced(hi, refine ? FD_K_ATTN_R : FD_K_ATTN_B, s,
+                     [&] { return fd::launch_attention(tq, tq8, r.tm_k, r.tm_vt, a, s); })))
+      return st;
+  }
+  fd::GemmParams po{};
+  po.epi = fd::EPI_RESID;
+  po.out_f32 = hbuf;
+  po.ld_out = D;
+  const CUtensorMap& so_h = refine ? b->so_hf : b->so_h;
+  if ((st = run_linear(h0, FD_K_OUT, refine ? b->tm_oR : b->tm_oB, lw.out, M, po, so_h, s)))
+    return st;
+  if (d.fp8) {  // as in run_block (Sec. 4.6)
+    const float* gain = lw.g2;
+    const float inv_su = lw.inv_su;
+    uint8_t* u8 = reinterpret_cast<uint8_t*>(b->u);
+    if ((st = traced(h0, FD_K_RMSNORM, s, [&] {
+           return fd::launch_rmsnorm_e4m3(hbuf, gain, M, D, eps, u8, inv_su, s);
+         })))
+      return st;
+    fd::GemmParams p1{};
+    p1.epi = d.gated ? fd::EPI_SWIGLU_F8 : fd::EPI_GELU_F8;
+    p1.fp8 = 1;
+    p1.col_scale = lw.cs1;
+    p1.out_scale = lw.inv_sh;
+    p1.out_f8 = reinterpret_cast<uint8_t*>(b->hid);
+    p1.ld_out = d.Mr * d.D;
+    if ((st = run_linear(h0, FD_K_MLP1, refine ? b->tm_u8R : b->tm_u8B, lw.mlp1, M, p1,
+                         refine ? b->so_hid8R : b->so_hid8B, s)))
+      return st;
+    fd::GemmParams p2 = po;
+    p2.fp8 = 1;
+    p2.col_scale = lw.cs2;
+    return run_linear(h0, FD_K_MLP2, refine ? b->tm_hid8R : b->tm_hid8B, lw.mlp2, M, p2, so_h, s);
+  }
+  {
+    const float* g2 = lw.g2;
+    __nv_bfloat16* u = b->u;
+    if ((st = traced(h0, FD_K_RMSNORM, s,
+                     [&] { return fd::launch_rmsnorm(hbuf, g2, M, D, eps, u, s); })))
+      return st;
+  }
+  fd::GemmParams p1{};
+  p1.epi = d.gated ? fd::EPI_SWIGLU : fd::EPI_GELU;
+  p1.out_bf16 = b->hid;
+  p1.ld_out = d.Mr * d.D;
+  if ((st = run_linear(h0, FD_K_MLP1, refine ? b->tm_uR : b->tm_uB, lw.mlp1, M, p1,
+                       refine ? b->so_hidR : b->so_hidB, s)))
+    return st;
+  return run_linear(h0, FD_K_MLP2, refine ? b->tm_hidR : b->tm_hidB, lw.mlp2, M, po, so_h, s);
+}
+
+// Algorithm 1 for chunk t_i of each of n streams at once (streams may be at different t)
+fd_status decode_batch(fd_batch b, fd_handle* hs, int n, const float* const* latents,
+                       void* const* pixels, cudaStream_t s) {
+  const Dims& d = b->d;
+  const fd_weights w = b->w;
+  fd_handle h0 = hs[0];
+  fd_status st;
+  const int bt = rope_band_t();
+  for (int i = 0; i < n; ++i) {
+    const int frames[2] = {1, d.rt};
+    double inv[fd::kRopePairs];
+    temporal_inv_freq(h0->cfg.rope_base, inv);
+    const int* step = hs[i]->state;
+    float2* tab = b->rope + static_cast<size_t>(i) * (1 + d.rt) * bt;
+    if ((st = traced(hs[i], FD_K_ROPE, s, [&] {
+           return fd::launch_rope_table(step, 0, 2, frames, bt, inv, tab, s);
+         })))
+      return st;
+    __nv_bfloat16* x0 = b->x0 + static_cast<size_t>(i) * b->Lp * d.cin;
+    const float* z = latents[i];
+    if ((st = traced(hs[i], FD_K_UNSHUFFLE, s,
+                     [&] { return fd::launch_unshuffle(z, d.C, d.H, d.W, d.p, x0, s); })))
+      return st;
+  }
+  const int MB = n * b->Lp, MR = n * b->Rp;
+  fd::GemmParams pe{};
+  pe.epi = fd::EPI_F32;
+  pe.out_f32 = b->h;
+  pe.ld_out = d.D;
+  if ((st = run_linear(h0, FD_K_EMBED, b->tm_x0, b->embed, MB, pe, b->so_h, s))) return st;
+  for (int l = 0; l < d.nb; ++l)
+    if ((st = batch_block(b, hs, n, l, false, s))) return st;
+  {
+    const float* g = w->g_f;
+    __nv_bfloat16* u = b->u;
+    float* hb = b->h;
+    const int D = d.D;
+    const float eps = h0->cfg.norm_eps;
+    if ((st = traced(h0, FD_K_RMSNORM, s,
+                     [&] { return fd::launch_rmsnorm(hb, g, MB, D, eps, u, s); })))
+      return st;
+  }
+  fd::GemmParams pt{};
+  pt.epi = fd::EPI_TUP;
+  pt.out_f32 = b->hf;
+  pt.tup_tokens = b->Lp;  // stream i's token l: row i Lp + l; refined: i Rp + tau Lp + l
+  pt.tup_hidden = d.D;
+  if ((st = run_linear(h0, FD_K_TUP, b->tm_uB, b->tup, MB, pt, b->so_tup, s))) return st;
+  for (int l = 0; l < d.nr; ++l)
+    if ((st = batch_block(b, hs, n, l, true, s))) return st;
+  {
+    const float* g = w->g_h;
+    __nv_bfloat16* u = b->u;
+    float* hb = b->hf;
+    const int D = d.D;
+    const float eps = h0->cfg.norm_eps;
+    if ((st = traced(h0, FD_K_RMSNORM, s,
+                     [&] { return fd::launch_rmsnorm(hb, g, MR, D, eps, u, s); })))
+      return st;
+  }
+  fd::GemmParams ph{};
+  ph.epi = fd::EPI_GELU;
+  ph.out_bf16 = b->hid;
+  ph.ld_out = d.D;
+  if ((st = run_linear(h0, FD_K_HEAD1, b->tm_uR, b->head1, MR, ph, b->so_hidH, s))) return st;
+  fd::GemmParams pf{};
+  pf.epi = fd::EPI_F32;
+  pf.out_f32 = b->F;
+  pf.ld_out = d.head_out;
+  if ((st = run_linear(h0, FD_K_HEAD2, b->tm_hidH, b->head2, MR, pf, b->so_F, s))) return st;
+  for (int i = 0; i < n; ++i) {
+    const float* F = b->F + static_cast<size_t>(i) * b->Rp * d.head_out;
+    const int frames = d.f1 && hs[i]->t_host == 0 ? 1 : d.rt;
+    void* pix = pixels[i];
+    const int Lp = b->Lp;
+    if ((st = traced(hs[i], FD_K_PIXEL, s, [&] {
+           return fd::launch_pixel_head(F, frames, d.gh, d.gw, d.Cout, d.rs, d.u8 ? 1 : 0, pix, s,
+                                        Lp);
+         })))
+      return st;
+    int* state = hs[i]->state;
+    if ((st = traced(hs[i], FD_K_ADVANCE, s, [&] { return fd::launch_advance(state, s); })))
+      return st;
+  }
+  return FD_OK;
+}
+
+
 
 constexpr int kMaxAttnParts = 4096;  // CTAs of one attention launch (fd_op_attention)
 
@@ -1106,6 +1355,193 @@ fd_status fd_decode_chunks(fd_handle* hs, int n, const float* const* latents_dev
   }
   for (int i = 0; i < n; ++i)
     if (cudaStreamWaitEvent(s, hs[i]->ev_join, 0) != cudaSuccess) return FD_ERR_CUDA;
+  return FD_OK;
+}
+
+fd_status fd_batch_create(const fd_config* cfg, fd_weights w, int max_streams, fd_batch* out) {
+  if (out == nullptr || w == nullptr || max_streams < 1 || max_streams > 64)
+    return FD_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!valid_cfg(cfg) || !same_cfg(cfg, &w->cfg)) return FD_ERR_CONFIG;
+  fd_status st = check_device();
+  if (st) return st;
+  fd_batch b = new (std::nothrow) fd_batch_s;
+  if (b == nullptr) return FD_ERR_OOM;
+  b->cfg = *cfg;
+  b->d = dims_of(cfg);
+  b->w = w;
+  b->nmax = max_streams;
+  const Dims& d = b->d;
+  b->Lp = static_cast<int>(align_up(static_cast<size_t>(d.L), 128));
+  b->Rp = d.rt * b->Lp;
+  const size_t RB = static_cast<size_t>(max_streams) * b->Lp;  // stacked backbone rows
+  const size_t RR = static_cast<size_t>(max_streams) * b->Rp;  // stacked refinement rows
+  const uint64_t NQ = static_cast<uint64_t>(d.N) * kHeadDim;
+  const uint64_t Dm = static_cast<uint64_t>(d.Mr) * d.D;
+  const int bt = rope_band_t();
+  b->partsB = choose_parts(d.L, d.N, d.G, d.Wn * d.L);
+  b->partsR = choose_parts(b->Rp, d.N, d.G, d.Wn * d.rt * d.L);
+  const int pairs = std::max(fd::attention_units(d.L, d.N, d.G),
+                             fd::attention_units(b->Rp, d.N, d.G));
+  const size_t ws = fd::attention_workspace_floats(std::max(b->partsB, b->partsR), pairs);
+  const size_t sizes[12] = {
+      RB * d.cin * 2,                                                  // x0
+      RR * d.D * 2,                                                    // u
+      RR * NQ * 2,                                                     // q
+      RR * NQ * 2,                                                     // o
+      RR * Dm * 2,                                                     // hid
+      RB * d.D * 4,                                                    // h
+      RR * d.D * 4,                                                    // hf
+      RR * d.head_out * 4,                                             // F
+      ws * 4,                                                          // attention partials
+      static_cast<size_t>(max_streams) * (1 + d.rt) * bt * sizeof(float2),  // RoPE tables
+      static_cast<size_t>(d.nb + d.nr) * max_streams * sizeof(fd::QkvStream),  // stream table
+      0};
+  size_t off[12], cur = 0;
+  for (int i = 0; i < 12; ++i) {
+    off[i] = cur;
+    cur = align_up(cur + sizes[i], 1024);
+  }
+  if (cudaMalloc(&b->arena, cur) != cudaSuccess) {
+    delete b;
+    return FD_ERR_OOM;
+  }
+  if (cudaMallocHost(&b->table_host, sizes[10]) != cudaSuccess) {
+    cudaFree(b->arena);
+    delete b;
+    return FD_ERR_OOM;
+  }
+  uint8_t* a = static_cast<uint8_t*>(b->arena);
+  b->x0 = reinterpret_cast<__nv_bfloat16*>(a + off[0]);
+  b->u = reinterpret_cast<__nv_bfloat16*>(a + off[1]);
+  b->q = reinterpret_cast<__nv_bfloat16*>(a + off[2]);
+  b->o = reinterpret_cast<__nv_bfloat16*>(a + off[3]);
+  b->hid = reinterpret_cast<__nv_bfloat16*>(a + off[4]);
+  b->h = reinterpret_cast<float*>(a + off[5]);
+  b->hf = reinterpret_cast<float*>(a + off[6]);
+  b->F = reinterpret_cast<float*>(a + off[7]);
+  b->attn_ws = reinterpret_cast<float*>(a + off[8]);
+  b->rope = reinterpret_cast<float2*>(a + off[9]);
+  b->table = reinterpret_cast<fd::QkvStream*>(a + off[10]);
+  bool ok = true;
+  b->embed = w->embed;
+  b->tup = w->tup;
+  b->head1 = w->head1;
+  b->head2 = w->head2;
+  b->blocks = w->blocks;
+  b->refine = w->refine;
+  ok = ok && retile(b->embed, static_cast<int>(RB), 32, false);
+  ok = ok && retile(b->tup, static_cast<int>(RB), 32, false);
+  ok = ok && retile(b->head1, static_cast<int>(RR), 64, false);
+  ok = ok && retile(b->head2, static_cast<int>(RR), 32, false);
+  for (auto& lw : b->blocks) ok = ok && retile_block(lw, d, static_cast<int>(RB));
+  for (auto& lw : b->refine) ok = ok && retile_block(lw, d, static_cast<int>(RR));
+  ok = ok && tmap_bf16(&b->tm_x0, b->x0, d.cin, RB, d.cin * 2, 64, 128);
+  ok = ok && tmap_bf16(&b->tm_uB, b->u, d.D, RB, d.D * 2, 64, 128);
+  ok = ok && tmap_bf16(&b->tm_uR, b->u, d.D, RR, d.D * 2, 64, 128);
+  ok = ok && tmap_bf16(&b->tm_oB, b->o, NQ, RB, NQ * 2, 64, 128);
+  ok = ok && tmap_bf16(&b->tm_oR, b->o, NQ, RR, NQ * 2, 64, 128);
+  ok = ok && tmap_bf16(&b->tm_hidB, b->hid, Dm, RB, Dm * 2, 64, 128);
+  ok = ok && tmap_bf16(&b->tm_hidR, b->hid, Dm, RR, Dm * 2, 64, 128);
+  ok = ok && tmap_bf16(&b->tm_hidH, b->hid, d.D, RR, static_cast<uint64_t>(d.D) * 2, 64, 128);
+  ok = ok && tmap_out_f32(&b->so_h, b->h, d.D, RB, d.D);
+  ok = ok && tmap_out_f32(&b->so_hf, b->hf, d.D, RR, d.D);
+  ok = ok && tmap_out_tup(&b->so_tup, b->hf, d.D, b->Lp, d.rt, max_streams);
+  ok = ok && tmap_out_bf16(&b->so_hidB, b->hid, Dm, RB, Dm);
+  ok = ok && tmap_out_bf16(&b->so_hidR, b->hid, Dm, RR, Dm);
+  ok = ok && tmap_out_bf16(&b->so_hidH, b->hid, d.D, RR, d.D);
+  ok = ok && tmap_out_f32(&b->so_F, b->F, d.head_out, RR, d.head_out);
+  ok = ok && tmap_out_bf16(&b->so_qB, b->q, NQ, RB, NQ);
+  ok = ok && tmap_out_bf16(&b->so_qR, b->q, NQ, RR, NQ);
+  if (d.fp8) {
+    ok = ok && tmap_e4m3(&b->tm_u8B, b->u, d.D, RB, d.D, 128);
+    ok = ok && tmap_e4m3(&b->tm_u8R, b->u, d.D, RR, d.D, 128);
+    ok = ok && tmap_e4m3(&b->tm_hid8B, b->hid, Dm, RB, Dm, 128);
+    ok = ok && tmap_e4m3(&b->tm_hid8R, b->hid, Dm, RR, Dm, 128);
+    ok = ok && tmap_out_e4m3(&b->so_hid8B, b->hid, Dm, RB, Dm);
+    ok = ok && tmap_out_e4m3(&b->so_hid8R, b->hid, Dm, RR, Dm);
+  }
+  b->tm_qB.resize(max_streams);
+  b->tm_q8B.resize(max_streams);
+  b->tm_qR.resize(max_streams);
+  b->tm_q8R.resize(max_streams);
+  for (int i = 0; i < max_streams; ++i) {  // stream i's Q rows (attention reads them alone)
+    const __nv_bfloat16* qb = b->q + static_cast<size_t>(i) * b->Lp * NQ;
+    const __nv_bfloat16* qr = b->q + static_cast<size_t>(i) * b->Rp * NQ;
+    ok = ok && tmap_bf16(&b->tm_qB[i], qb, NQ, d.L, NQ * 2, 64, 128);
+    ok = ok && tmap_bf16(&b->tm_q8B[i], qb, NQ, d.L, NQ * 2, 64, 8);
+    ok = ok && tmap_bf16(&b->tm_qR[i], qr, NQ, b->Rp, NQ * 2, 64, 128);
+    ok = ok && tmap_bf16(&b->tm_q8R[i], qr, NQ, b->Rp, NQ * 2, 64, 8);
+  }
+  // padding rows start (and, being outputs of row-wise kernels on zero inputs, stay) finite
+  if (!ok || cudaMemset(b->arena, 0, cur) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
+    cudaFreeHost(b->table_host);
+    cudaFree(b->arena);
+    delete b;
+    return FD_ERR_CUDA;
+  }
+  w->live_handles++;
+  *out = b;
+  return FD_OK;
+}
+
+fd_status fd_decode_batch(fd_batch b, fd_handle* hs, int n, const float* const* latents_dev,
+                          void* const* pixels_dev, void* stream) {
+  if (b == nullptr || hs == nullptr || n < 1 || n > b->nmax || latents_dev == nullptr ||
+      pixels_dev == nullptr)
+    return FD_ERR_INVALID_ARG;
+  for (int i = 0; i < n; ++i) {  // check everything before enqueueing anything
+    fd_handle h = hs[i];
+    if (h == nullptr || latents_dev[i] == nullptr || pixels_dev[i] == nullptr)
+      return FD_ERR_INVALID_ARG;
+    if (!aligned16(latents_dev[i]) || !aligned16(pixels_dev[i])) return FD_ERR_INVALID_ARG;
+    if (h->w != b->w) return FD_ERR_CONFIG;
+    for (int j = 0; j < i; ++j)
+      if (hs[j] == h) return FD_ERR_INVALID_ARG;
+    if (h->error || h->t_host >= (1LL << 30)) return FD_ERR_STATE;
+  }
+  const Dims& d = b->d;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the per-layer stream table (rings, counters, RoPE tables) for this set of handles
+  if (b->table_for.size() != static_cast<size_t>(n) ||
+      !std::equal(b->table_for.begin(), b->table_for.end(), hs)) {
+    if (cudaStreamSynchronize(s) != cudaSuccess) return FD_ERR_CUDA;  // table not in use
+    const int bt = rope_band_t();
+    for (int l = 0; l < d.nb + d.nr; ++l)
+      for (int i = 0; i < n; ++i) {
+        const bool refine = l >= d.nb;
+        const Ring& r = refine ? hs[i]->ringR[l - d.nb] : hs[i]->ringB[l];
+        fd::QkvStream& e = b->table_host[static_cast<size_t>(l) * b->nmax + i];
+        e.k_ring = r.k;
+        e.vt_ring = r.vt;
+        e.step_dev = hs[i]->state;
+        e.rope_t = b->rope + static_cast<size_t>(i) * (1 + d.rt) * bt + (refine ? bt : 0);
+      }
+    if (cudaMemcpyAsync(b->table, b->table_host,
+                        static_cast<size_t>(d.nb + d.nr) * b->nmax * sizeof(fd::QkvStream),
+                        cudaMemcpyHostToDevice, s) != cudaSuccess)
+      return FD_ERR_CUDA;
+    b->table_for.assign(hs, hs + n);
+  }
+  const fd_status st = decode_batch(b, hs, n, latents_dev, pixels_dev, s);
+  for (int i = 0; i < n; ++i) {
+    if (st != FD_OK) {
+      hs[i]->error = true;
+    } else {
+      hs[i]->t_host++;
+      hs[i]->last_stream = s;
+    }
+  }
+  return st;
+}
+
+fd_status fd_batch_destroy(fd_batch b) {
+  if (b == nullptr) return FD_ERR_INVALID_ARG;
+  cudaDeviceSynchronize();
+  cudaFreeHost(b->table_host);
+  cudaFree(b->arena);
+  if (b->w) b->w->live_handles--;
+  delete b;
   return FD_OK;
 }
 

@@ -59,6 +59,10 @@ _SIGS = {
     "fd_decode_chunks": (_I, [ctypes.POINTER(_P), _I, ctypes.POINTER(_P), ctypes.POINTER(_P),
                               _P]),
     "fd_decode_chunk_host": (_I, [_P, _P, _P, _P]),
+    "fd_batch_create": (_I, [ctypes.POINTER(fd_config), _P, _I, ctypes.POINTER(_P)]),
+    "fd_decode_batch": (_I, [_P, ctypes.POINTER(_P), _I, ctypes.POINTER(_P),
+                             ctypes.POINTER(_P), _P]),
+    "fd_batch_destroy": (_I, [_P]),
     "fd_reset": (_I, [_P]),
     "fd_profile_enable": (_I, [_P, _I]),
     "fd_profile_collect": (_I, [_P, ctypes.POINTER(ctypes.c_int64),
@@ -285,6 +289,39 @@ def decode_chunks(decoders, latents, pixels, stream=None) -> None:
     ls = (_P * n)(*[_ptr(x) for x in latents])
     ps = (_P * n)(*[_ptr(x) for x in pixels])
     _check(lib().fd_decode_chunks(hs, n, ls, ps, _stream_ptr(stream)), "fd_decode_chunks")
+
+
+class Batch:
+    """Stacked decode of up to max_streams decoders of one weights object (fd_batch_create):
+    the GEMMs of a chunk run once on all streams' rows."""
+
+    def __init__(self, cfg, weights: Weights, max_streams: int):
+        self.cfg = make_config(cfg)
+        self.weights = weights
+        out = _P()
+        _check(lib().fd_batch_create(ctypes.byref(self.cfg), weights.handle, int(max_streams),
+                                     ctypes.byref(out)), "fd_batch_create")
+        self.handle = out
+
+    def decode(self, decoders, latents, pixels, stream=None) -> None:
+        """One chunk for each decoder (fd_decode_batch)."""
+        n = len(decoders)
+        hs = (_P * n)(*[d.handle for d in decoders])
+        ls = (_P * n)(*[_ptr(x) for x in latents])
+        ps = (_P * n)(*[_ptr(x) for x in pixels])
+        _check(lib().fd_decode_batch(self.handle, hs, n, ls, ps, _stream_ptr(stream)),
+               "fd_decode_batch")
+
+    def close(self) -> None:
+        if getattr(self, "handle", None):
+            _check(lib().fd_batch_destroy(self.handle), "fd_batch_destroy")
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 # ------------------------------------------------------------------ kernel-level entry points
