@@ -130,11 +130,46 @@ struct Cursor {
   }
 };
 
+// kBatched: grid y = stream of p.streams (K / V maps, counter and error word from there; Q,
+// output and workspace offset by the stream)
+template <bool kBatched>
 __global__ void __launch_bounds__(attn::kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQ8,
                 const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
   using namespace attn;
+  // the stream's own pointers in a batched launch; the single-stream kernel reads p directly
+  struct {
+    const CUtensorMap *k, *v;
+    int* err;
+    const int* step;
+    __nv_bfloat16* out;
+    float *po, *pml;
+    int* cnt;
+    int q_row0;
+  } bs{};
+  if constexpr (kBatched) {
+    const int y = blockIdx.y;
+    const AttnStream* as = p.streams + y;
+    bs.k = &as->k;
+    bs.v = &as->vt;
+    bs.err = as->err;
+    bs.step = as->step_dev;
+    bs.q_row0 = y * p.q_rows_stream;
+    bs.out = p.out + static_cast<size_t>(bs.q_row0) * p.ld_out;
+    bs.po = p.part_o + y * p.ws_stride;
+    bs.pml = p.part_ml + y * p.ws_stride;
+    bs.cnt = p.counters + y * p.ws_stride;
+  }
+  const CUtensorMap* const mK = kBatched ? bs.k : &tmK;
+  const CUtensorMap* const mV = kBatched ? bs.v : &tmV;
+#define ERR_WORD (kBatched ? bs.err : p.err)
+#define STEP_DEV (kBatched ? bs.step : p.step_dev)
+#define OUT_ROWS (kBatched ? bs.out : p.out)
+#define PART_O (kBatched ? bs.po : p.part_o)
+#define PART_ML (kBatched ? bs.pml : p.part_ml)
+#define COUNTERS (kBatched ? bs.cnt : p.counters)
+#define Q_ROW0 (kBatched ? bs.q_row0 : 0)
   extern __shared__ __align__(1024) uint8_t smem[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -150,7 +185,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
   const int pairs_per_group = (attention_tiles_per_group(p.Lq, p.heads, p.groups) + 1) / 2;
 
   if (threadIdx.x == 0) {
-    if (!aligned) atomicOr(p.err, ERR_SMEM_ALIGN);
+    if (!aligned) atomicOr(ERR_WORD, ERR_SMEM_ALIGN);
     for (int b = 0; b < 2; ++b) {
       mbar_init(bar(kBarQFull + b), 1);
       mbar_init(bar(kBarQFree + b), 2);  // both tiles' issuers
@@ -175,8 +210,8 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
   }
   grid_dep_wait();  // Q and the ring written by the previous kernels; TMEM freed by their CTAs
   int n_keys = p.n_keys_host;
-  if (p.step_dev != nullptr) {
-    const int t = *p.step_dev;
+  if (STEP_DEV != nullptr) {
+    const int t = *STEP_DEV;
     n_keys = (t + 1 < p.window ? t + 1 : p.window) * p.rows_per_chunk;
   }
   const int nblk = (n_keys + 127) / 128;
@@ -197,8 +232,8 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
     if (lane == 0 && aligned && len > 0) {
       prefetch_tmap(&tmQ);
       prefetch_tmap(&tmQ8);
-      prefetch_tmap(&tmK);
-      prefetch_tmap(&tmV);
+      prefetch_tmap(mK);
+      prefetch_tmap(mV);
       // Count this CTA's partial results once the softmax warps have stored them. The stores
       // reach this thread through the barrier (CTA scope); the gpu-scope fence before the
       // counter update publishes them all (fences are cumulative). The CTA that stores a
@@ -214,9 +249,9 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         for (int c = wr.cta_of(pr * nblk); c <= wr.cta_of(pr * nblk + nblk - 1); ++c)
           owners += wr.empty(c) ? 0 : 1;
         __threadfence();
-        const int prev = atomicAdd(p.counters + pr, 1);
+        const int prev = atomicAdd(COUNTERS + pr, 1);
         if (prev == owners - 1) {
-          p.counters[pr] = 0;  // every part has arrived: ready for the next launch
+          COUNTERS[pr] = 0;  // every part has arrived: ready for the next launch
           __threadfence();
           decision[sl] = 1;
         }
@@ -233,7 +268,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
           // its S MMAs
           const int qb = cur.seg & 1;
           if (cur.seg >= 2 &&
-              !mbar_wait(bar(kBarQFree + qb), ((cur.seg >> 1) - 1) & 1, p.err, ERR_WAIT_MMA)) {
+              !mbar_wait(bar(kBarQFree + qb), ((cur.seg >> 1) - 1) & 1, ERR_WORD, ERR_WAIT_MMA)) {
             ok = false;
             break;
           }
@@ -249,41 +284,42 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
             const uint32_t dst = base + kOffQ + (2 * qb + x) * kQBytes;
             const uint32_t qbar = bar(kBarQFull + qb);
             if (hl0 >= hpg) {
-              tma_load_2d(dst, &tmQ, qbar, g * hpg * kHeadDim, 0);
+              tma_load_2d(dst, &tmQ, qbar, g * hpg * kHeadDim, Q_ROW0);
             } else if (hl1 == hl0 || hl1 >= hpg) {
-              tma_load_2d(dst, &tmQ, qbar, (g * hpg + hl0) * kHeadDim, rho0 - hl0 * p.lq_pad);
+              tma_load_2d(dst, &tmQ, qbar, (g * hpg + hl0) * kHeadDim,
+                          Q_ROW0 + rho0 - hl0 * p.lq_pad);
             } else {
               for (int b = 0; b < kBM / 8; ++b) {
                 const int rho = rho0 + 8 * b;
                 int hl = rho / p.lq_pad;
                 int r = rho - hl * p.lq_pad;
                 if (hl >= hpg) hl = r = 0;
-                tma_load_2d(dst + b * 1024, &tmQ8, qbar, (g * hpg + hl) * kHeadDim, r);
+                tma_load_2d(dst + b * 1024, &tmQ8, qbar, (g * hpg + hl) * kHeadDim, Q_ROW0 + r);
               }
             }
           }
         }
         const int st = J % kStages;
-        if (!mbar_wait(bar(kBarKvEmpty + st), ((J / kStages) & 1) ^ 1, p.err, ERR_WAIT_MMA)) {
+        if (!mbar_wait(bar(kBarKvEmpty + st), ((J / kStages) & 1) ^ 1, ERR_WORD, ERR_WAIT_MMA)) {
           ok = false;
           break;
         }
         const uint32_t b = bar(kBarKvFull + st);
         mbar_expect_tx(b, kKBytes + kVBytes);
-        tma_load_2d(base + kOffK + st * kKBytes, &tmK, b, 0, g * p.ring_pitch + cur.kb * 128);
-        tma_load_2d(base + kOffV + st * kVBytes, &tmV, b, cur.kb * 128, g * kHeadDim);
-        tma_load_2d(base + kOffV + st * kVBytes + kVSub, &tmV, b, cur.kb * 128 + 64,
+        tma_load_2d(base + kOffK + st * kKBytes, mK, b, 0, g * p.ring_pitch + cur.kb * 128);
+        tma_load_2d(base + kOffV + st * kVBytes, mV, b, cur.kb * 128, g * kHeadDim);
+        tma_load_2d(base + kOffV + st * kVBytes + kVSub, mV, b, cur.kb * 128 + 64,
                     g * kHeadDim);
         if (J + 1 < len) cur.next(len - J - 2, nblk);
       }
       // nothing may be in flight when the CTA exits: the last two Q loads, the last KV loads
       const int nseg = cur.seg + 1;
       for (int sg = nseg - 1; sg >= 0 && sg >= nseg - 2; --sg)
-        mbar_wait(bar(kBarQFull + (sg & 1)), (sg >> 1) & 1, p.err, ERR_WAIT_TMA);
+        mbar_wait(bar(kBarQFull + (sg & 1)), (sg >> 1) & 1, ERR_WORD, ERR_WAIT_TMA);
       for (int i = J - 1; i >= 0 && i >= J - kStages; --i)
-        mbar_wait(bar(kBarKvFull + i % kStages), (i / kStages) & 1, p.err, ERR_WAIT_TMA);
+        mbar_wait(bar(kBarKvFull + i % kStages), (i / kStages) & 1, ERR_WORD, ERR_WAIT_TMA);
       for (int sl = 0; sl < 2; ++sl)
-        if (!counted[sl] && mbar_wait(bar(kBarPartDone + sl), 0, p.err, ERR_WAIT_EPI))
+        if (!counted[sl] && mbar_wait(bar(kBarPartDone + sl), 0, ERR_WORD, ERR_WAIT_EPI))
           count_slot(sl);
       mbar_arrive(bar(kBarDecided));
     }
@@ -306,9 +342,9 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       // S_X(J) = Q_X K_J^T; after the last block of a segment, release its Q buffer
       auto issue_s = [&](int J, const Cursor& c) -> bool {
         const int qb = c.seg & 1;
-        if (c.first && !mbar_wait(bar(kBarQFull + qb), (c.seg >> 1) & 1, p.err, ERR_WAIT_TMA))
+        if (c.first && !mbar_wait(bar(kBarQFull + qb), (c.seg >> 1) & 1, ERR_WORD, ERR_WAIT_TMA))
           return false;
-        if (!mbar_wait(bar(kBarKvFull + J % kStages), (J / kStages) & 1, p.err, ERR_WAIT_TMA))
+        if (!mbar_wait(bar(kBarKvFull + J % kStages), (J / kStages) & 1, ERR_WORD, ERR_WAIT_TMA))
           return false;
         tc_fence_after();
         const uint64_t dq = dq0 + static_cast<uint64_t>((2 * qb * kQBytes) >> 4);
@@ -328,14 +364,14 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         // S of the next block as soon as the softmax has read S(J)
         if (J + 1 < len) {
           cur.next(len - J - 2, nblk);
-          ok = mbar_wait(bar(kBarSFree + x), J & 1, p.err, ERR_WAIT_EPI) && issue_s(J + 1, cur);
+          ok = mbar_wait(bar(kBarSFree + x), J & 1, ERR_WORD, ERR_WAIT_EPI) && issue_s(J + 1, cur);
           if (!ok) break;
         }
         // P V of this block once P(J) is written; the first block of a segment overwrites O,
         // so it also waits until the softmax has read the previous segment's O
-        ok = mbar_wait(bar(kBarP + x), J & 1, p.err, ERR_WAIT_EPI);
+        ok = mbar_wait(bar(kBarP + x), J & 1, ERR_WORD, ERR_WAIT_EPI);
         if (ok && here.first && here.seg > 0)
-          ok = mbar_wait(bar(kBarOFree + x), (here.seg - 1) & 1, p.err, ERR_WAIT_EPI);
+          ok = mbar_wait(bar(kBarOFree + x), (here.seg - 1) & 1, ERR_WORD, ERR_WAIT_EPI);
         tc_fence_after();
         if (!ok) break;
         const uint64_t dv = dv0 + static_cast<uint64_t>((st * kVBytes) >> 4);
@@ -348,7 +384,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         mma_commit(bar(kBarKvEmpty + st));  // one of the two arrivals that free the stage
       }
       mma_commit(bar(kBarDone + x));
-      mbar_wait(bar(kBarDone + x), 0, p.err, ERR_WAIT_MMA);
+      mbar_wait(bar(kBarDone + x), 0, ERR_WORD, ERR_WAIT_MMA);
     }
   } else {
     // ------------------------------------------------------------ softmax, tile x
@@ -370,7 +406,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         m_used = -INFINITY;
         l_run = 0.f;
       }
-      const bool got = mbar_wait(bar(kBarS + x), J & 1, p.err, ERR_WAIT_MMA);
+      const bool got = mbar_wait(bar(kBarS + x), J & 1, ERR_WORD, ERR_WAIT_MMA);
       if (!__all_sync(0xffffffffu, got)) {
         ok = false;
         break;
@@ -415,7 +451,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       // load, P V wait and P store run while the other computes.
       if (x == 1 || J > 0) {
         const bool turn = mbar_wait(bar(kBarTurn + 4 * x + quarter), (x == 1 ? J : J - 1) & 1,
-                                    p.err, ERR_WAIT_EPI);
+                                    ERR_WORD, ERR_WAIT_EPI);
         if (!__all_sync(0xffffffffu, turn)) {
           ok = false;
           break;
@@ -448,7 +484,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       // P_X and O_X are free once the P V of the previous block has completed (for the
       // first block of a segment the previous segment's output already waited for it)
       if (!cur.first) {
-        const bool pv = mbar_wait(bar(kBarPv + x), (J - 1) & 1, p.err, ERR_WAIT_MMA);
+        const bool pv = mbar_wait(bar(kBarPv + x), (J - 1) & 1, ERR_WORD, ERR_WAIT_MMA);
         if (!__all_sync(0xffffffffu, pv)) {
           ok = false;
           break;
@@ -479,7 +515,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       if (!cur.last) continue;
 
       // -------------------------------------------------------- output of the segment
-      const bool done = mbar_wait(bar(kBarPv + x), J & 1, p.err, ERR_WAIT_MMA);
+      const bool done = mbar_wait(bar(kBarPv + x), J & 1, ERR_WORD, ERR_WAIT_MMA);
       if (!__all_sync(0xffffffffu, done)) {
         ok = false;
         break;
@@ -505,7 +541,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       const int r = rho - hl * p.lq_pad;
       const bool valid_row = hl < hpg && r < p.Lq;
       __nv_bfloat16* out_row =
-          p.out + static_cast<size_t>(r) * p.ld_out + (g * hpg + hl) * kHeadDim;
+          OUT_ROWS + static_cast<size_t>(r) * p.ld_out + (g * hpg + hl) * kHeadDim;
       const int c_lo = wr.cta_of(cur.pair * nblk);
       const int c_hi = wr.cta_of(cur.pair * nblk + nblk - 1);
       if (c_lo == c_hi) {  // the whole pair was done here
@@ -525,11 +561,11 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       const int slot = wr.start(blockIdx.x) >= cur.pair * nblk ? 0 : 1;
       {
         const size_t pb = (static_cast<size_t>(blockIdx.x) * 2 + slot) * 2 + x;
-        float4* po = reinterpret_cast<float4*>(p.part_o) + pb * (kPartO / 4) + row;
+        float4* po = reinterpret_cast<float4*>(PART_O) + pb * (kPartO / 4) + row;
 #pragma unroll
         for (int k = 0; k < 16; ++k)
           po[k * 128] = make_float4(o[4 * k], o[4 * k + 1], o[4 * k + 2], o[4 * k + 3]);
-        reinterpret_cast<float2*>(p.part_ml)[pb * 128 + row] = make_float2(m_used, l_run);
+        reinterpret_cast<float2*>(PART_ML)[pb * 128 + row] = make_float2(m_used, l_run);
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(bar(kBarPartDone + slot));
@@ -539,7 +575,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
     // O = sum_c 2^(m_c - M) O_c / sum_c 2^(m_c - M) l_c over the CTAs c holding a part of it
     const PartialSlots ps(wr, u0, len, nblk);
     if (ok && (ps.has[0] || ps.has[1])) {
-      const bool decided = mbar_wait(bar(kBarDecided), 0, p.err, ERR_WAIT_EPI);
+      const bool decided = mbar_wait(bar(kBarDecided), 0, ERR_WORD, ERR_WAIT_EPI);
       ok = __all_sync(0xffffffffu, decided);
       for (int sl = 0; sl < 2 && ok; ++sl) {
         if (!ps.has[sl] || !decision[sl]) continue;
@@ -555,7 +591,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         for (int c = c_lo; c <= c_hi; ++c) {
           if (wr.empty(c)) continue;
           const size_t pb = (static_cast<size_t>(c) * 2 + (wr.start(c) >= pr * nblk ? 0 : 1)) * 2 + x;
-          M = fmaxf(M, __ldcg(reinterpret_cast<const float2*>(p.part_ml) + pb * 128 + row).x);
+          M = fmaxf(M, __ldcg(reinterpret_cast<const float2*>(PART_ML) + pb * 128 + row).x);
         }
         float acc[64];
 #pragma unroll
@@ -564,10 +600,10 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         for (int c = c_lo; c <= c_hi; ++c) {
           if (wr.empty(c)) continue;
           const size_t pb = (static_cast<size_t>(c) * 2 + (wr.start(c) >= pr * nblk ? 0 : 1)) * 2 + x;
-          const float2 ml = __ldcg(reinterpret_cast<const float2*>(p.part_ml) + pb * 128 + row);
+          const float2 ml = __ldcg(reinterpret_cast<const float2*>(PART_ML) + pb * 128 + row);
           const float w = ex2_approx(ml.x - M);
           l = fmaf(w, ml.y, l);
-          const float4* po = reinterpret_cast<const float4*>(p.part_o) + pb * (kPartO / 4) + row;
+          const float4* po = reinterpret_cast<const float4*>(PART_O) + pb * (kPartO / 4) + row;
 #pragma unroll
           for (int k = 0; k < 16; ++k) {
             const float4 v = __ldcg(po + k * 128);
@@ -578,7 +614,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
           }
         }
         const float inv = 1.0f / l;
-        uint4* dst = reinterpret_cast<uint4*>(p.out + static_cast<size_t>(r) * p.ld_out +
+        uint4* dst = reinterpret_cast<uint4*>(OUT_ROWS + static_cast<size_t>(r) * p.ld_out +
                                               (g * hpg + hl) * kHeadDim);
 #pragma unroll
         for (int k = 0; k < 8; ++k)
@@ -599,6 +635,14 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
   }
 }
 
+#undef ERR_WORD
+#undef STEP_DEV
+#undef OUT_ROWS
+#undef PART_O
+#undef PART_ML
+#undef COUNTERS
+#undef Q_ROW0
+
 int attention_parts(int units, int nblk, int num_sms) {
   const long long w = static_cast<long long>(units) * nblk;
   return static_cast<int>(w < num_sms ? (w > 0 ? w : 1) : num_sms);
@@ -609,13 +653,19 @@ cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmQ8,
                              const CUtensorMap& tmVt, const AttnParams& p, cudaStream_t s) {
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         attn::kSmem);
+    cudaError_t e = cudaFuncSetAttribute(attn_kernel<false>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, attn::kSmem);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(attn_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               attn::kSmem);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  return launch_pdl(attn_kernel, dim3(p.parts), dim3(attn::kThreads), attn::kSmem, s, tmQ, tmQ8,
-                    tmK, tmVt, p);
+  if (p.streams != nullptr)
+    return launch_pdl(attn_kernel<true>, dim3(p.parts, p.n_streams), dim3(attn::kThreads),
+                      attn::kSmem, s, tmQ, tmQ8, tmK, tmVt, p);
+  return launch_pdl(attn_kernel<false>, dim3(p.parts), dim3(attn::kThreads), attn::kSmem, s, tmQ,
+                    tmQ8, tmK, tmVt, p);
 }
 
 }  // namespace fd

@@ -113,6 +113,14 @@ struct GemmParams {
   int w_static;
 };
 
+// one stream of a batched attention launch (grid y = stream): its ring's K and V^T maps, its
+// chunk counter and error word
+struct AttnStream {
+  CUtensorMap k, vt;
+  const int* step_dev;
+  int* err;
+};
+
 struct AttnParams {
   int Lq;                    // query rows
   int heads, groups;
@@ -131,6 +139,13 @@ struct AttnParams {
   float* part_o;             // [parts][2 slots][2 tiles][16][128 rows] float4 partial O
   float* part_ml;            // [parts][2][2][128] (running max, row sum)
   int* counters;             // [pairs] partial results stored per pair; zero between launches
+  // batched launch over n_streams streams (null: one stream, the maps passed to the launch):
+  // stream y's Q rows start at row y * q_rows_stream of tmQ, its output rows likewise in out,
+  // its partial results and counters at y * ws_stride floats past part_o / part_ml / counters
+  const AttnStream* streams;
+  int n_streams;
+  int q_rows_stream;
+  size_t ws_stride;
 };
 
 // launch wrappers; return cudaGetLastError() of the launch
@@ -139,6 +154,11 @@ struct AttnParams {
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmO,
                         const CUtensorMap& tmK, const CUtensorMap& tmV, const GemmParams& p,
                         int bn, bool pair, int num_sms, cudaStream_t s);
+// the EPI_QKV instances (launch_gemm forwards to it for that epilogue)
+cudaError_t launch_gemm_qkv(const CUtensorMap& tmA, const CUtensorMap& tmB,
+                            const CUtensorMap& tmO, const CUtensorMap& tmK,
+                            const CUtensorMap& tmV, const GemmParams& p, int bn, bool pair,
+                            int num_sms, cudaStream_t s);
 // Attention (+ the combine of key-range splits when p.splits > 1).
 // tmQ: Q [Lq][heads * 64] bf16 in boxes of 64 x 128 rows; tmQ8: the same in boxes of 64 x 8.
 cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmQ8,

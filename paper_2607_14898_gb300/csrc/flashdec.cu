@@ -428,12 +428,14 @@ struct fd_batch_s {
   float2* rope = nullptr;               // [nmax][(1 + r_t) band_t] temporal RoPE per stream
   fd::QkvStream* table = nullptr;       // [n_blocks + n_refine][nmax] on the device
   fd::QkvStream* table_host = nullptr;  // pinned copy
-  std::vector<fd_handle> table_for;     // handles the table was written for
-  int partsB = 1, partsR = 1;
+  fd::AttnStream* attn_table = nullptr;       // [n_blocks + n_refine][nmax]: rings' K / V maps
+  fd::AttnStream* attn_table_host = nullptr;  // pinned copy
+  std::vector<fd_handle> table_for;     // handles the tables were written for
+  size_t ws_stride = 0;                 // attention workspace floats per stream
   CUtensorMap tm_x0, tm_uB, tm_uR, tm_oB, tm_oR, tm_hidB, tm_hidR, tm_hidH;
   CUtensorMap so_h, so_hf, so_tup, so_hidB, so_hidR, so_hidH, so_F, so_qB, so_qR;
   CUtensorMap tm_u8B, tm_u8R, tm_hid8B, tm_hid8R, so_hid8B, so_hid8R;
-  std::vector<CUtensorMap> tm_qB, tm_q8B, tm_qR, tm_q8R;  // each stream's Q rows
+  CUtensorMap tm_qB, tm_q8B, tm_qR, tm_q8R;  // stacked Q in boxes of 128 and 8 rows
   // the weights' products with launch shapes re-chosen for the stacked row counts (same
   // device weights; only the tile width, CTA pairing and W descriptor differ)
   Linear embed, tup, head1, head2;
@@ -700,6 +702,16 @@ bool retile_block(LayerW& lw, const Dims& d, int M) {
   return ok && retile(lw.mlp1, M, d.gated ? 128 : 64, false) && retile(lw.mlp2, M, 32, false);
 }
 
+// CTAs per stream of a batched attention launch over n streams: the GPU's SMs shared out
+// (the launch is persistent, one CTA per SM), at most one per (tile pair, key block) unit of
+// the full window
+int batch_parts(int Lq, int n_keys, const Dims& d, int n) {
+  const long long units =
+      static_cast<long long>(fd::attention_units(Lq, d.N, d.G)) * ((n_keys + 127) / 128);
+  const int share = std::max(1, num_sms() / n);
+  return static_cast<int>(std::min<long long>(share, std::max(1LL, units)));
+}
+
 // ---------------------------------------------------------------- batched decode
 // One Transformer block on the stacked rows of n streams (see fd_batch_s): the GEMMs and the
 // norms run once on n * rows_s rows; the QKV epilogue appends each stream's K / V to its own
@@ -739,26 +751,29 @@ fd_status batch_block(fd_batch b, fd_handle* hs, int n, int layer, bool refine, 
   if ((st = run_linear(h0, FD_K_QKV, refine ? b->tm_uR : b->tm_uB, lw.qkv, M, p, so_q, s, &so_q,
                        &so_q)))
     return st;
-  const int pairs = std::max(fd::attention_units(d.L, d.N, d.G),
-                             fd::attention_units(b->Rp, d.N, d.G));
-  for (int i = 0; i < n; ++i) {
-    fd_handle hi = hs[i];
-    Ring& r = refine ? hi->ringR[layer] : hi->ringB[layer];
+  {  // one launch for all streams: grid y = stream, parts_s CTAs each
+    const int pairs = std::max(fd::attention_units(d.L, d.N, d.G),
+                               fd::attention_units(b->Rp, d.N, d.G));
+    Ring& r0 = refine ? h0->ringR[layer] : h0->ringB[layer];
     fd::AttnParams a{};
     a.Lq = refine ? b->Rp : d.L;
     a.heads = d.N; a.groups = d.G; a.ring_pitch = q.ring_pitch;
     a.rows_per_chunk = refine ? d.rt * d.L : d.L;
-    a.window = d.Wn; a.step_dev = hi->state; a.n_keys_host = 0;
-    a.out = b->o + static_cast<size_t>(i) * rows_s * NQ;
+    a.window = d.Wn; a.step_dev = h0->state; a.n_keys_host = 0;
+    a.out = b->o;
     a.ld_out = static_cast<int>(NQ); a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
-    a.err = hi->state + 1;
+    a.err = h0->state + 1;
     a.lq_pad = fd::attention_lq_pad(a.Lq);
-    a.parts = refine ? b->partsR : b->partsB;
+    a.parts = batch_parts(a.Lq, d.Wn * a.rows_per_chunk, d, n);
     fd::attention_workspace_split(b->attn_ws, a.parts, pairs, a);
-    const CUtensorMap& tq = refine ? b->tm_qR[i] : b->tm_qB[i];
-    const CUtensorMap& tq8 = refine ? b->tm_q8R[i] : b->tm_q8B[i];
-    if ((st = traced(hi, refine ? FD_K_ATTN_R : FD_K_ATTN_B, s,
-                     [&] { return fd::launch_attention(tq, tq8, r.tm_k, r.tm_vt, a, s); })))
+    a.streams = b->attn_table + static_cast<size_t>(refine ? d.nb + layer : layer) * b->nmax;
+    a.n_streams = n;
+    a.q_rows_stream = rows_s;
+    a.ws_stride = b->ws_stride;
+    const CUtensorMap& tq = refine ? b->tm_qR : b->tm_qB;
+    const CUtensorMap& tq8 = refine ? b->tm_q8R : b->tm_q8B;
+    if ((st = traced(h0, refine ? FD_K_ATTN_R : FD_K_ATTN_B, s,
+                     [&] { return fd::launch_attention(tq, tq8, r0.tm_k, r0.tm_vt, a, s); })))
       return st;
   }
   fd::GemmParams po{};
@@ -1379,11 +1394,11 @@ fd_status fd_batch_create(const fd_config* cfg, fd_weights w, int max_streams, f
   const uint64_t NQ = static_cast<uint64_t>(d.N) * kHeadDim;
   const uint64_t Dm = static_cast<uint64_t>(d.Mr) * d.D;
   const int bt = rope_band_t();
-  b->partsB = choose_parts(d.L, d.N, d.G, d.Wn * d.L);
-  b->partsR = choose_parts(b->Rp, d.N, d.G, d.Wn * d.rt * d.L);
   const int pairs = std::max(fd::attention_units(d.L, d.N, d.G),
                              fd::attention_units(b->Rp, d.N, d.G));
-  const size_t ws = fd::attention_workspace_floats(std::max(b->partsB, b->partsR), pairs);
+  // per stream: partial results of up to one CTA per SM (a batch of one stream)
+  b->ws_stride = align_up(fd::attention_workspace_floats(num_sms(), pairs), 64);
+  const size_t ws = b->ws_stride * max_streams;
   const size_t sizes[12] = {
       RB * d.cin * 2,                                                  // x0
       RR * d.D * 2,                                                    // u
@@ -1396,7 +1411,7 @@ fd_status fd_batch_create(const fd_config* cfg, fd_weights w, int max_streams, f
       ws * 4,                                                          // attention partials
       static_cast<size_t>(max_streams) * (1 + d.rt) * bt * sizeof(float2),  // RoPE tables
       static_cast<size_t>(d.nb + d.nr) * max_streams * sizeof(fd::QkvStream),  // stream table
-      0};
+      static_cast<size_t>(d.nb + d.nr) * max_streams * sizeof(fd::AttnStream)};  // ring maps
   size_t off[12], cur = 0;
   for (int i = 0; i < 12; ++i) {
     off[i] = cur;
@@ -1407,6 +1422,12 @@ fd_status fd_batch_create(const fd_config* cfg, fd_weights w, int max_streams, f
     return FD_ERR_OOM;
   }
   if (cudaMallocHost(&b->table_host, sizes[10]) != cudaSuccess) {
+    cudaFree(b->arena);
+    delete b;
+    return FD_ERR_OOM;
+  }
+  if (cudaMallocHost(&b->attn_table_host, sizes[11]) != cudaSuccess) {
+    cudaFreeHost(b->table_host);
     cudaFree(b->arena);
     delete b;
     return FD_ERR_OOM;
@@ -1423,6 +1444,7 @@ fd_status fd_batch_create(const fd_config* cfg, fd_weights w, int max_streams, f
   b->attn_ws = reinterpret_cast<float*>(a + off[8]);
   b->rope = reinterpret_cast<float2*>(a + off[9]);
   b->table = reinterpret_cast<fd::QkvStream*>(a + off[10]);
+  b->attn_table = reinterpret_cast<fd::AttnStream*>(a + off[11]);
   bool ok = true;
   b->embed = w->embed;
   b->tup = w->tup;
@@ -1461,20 +1483,13 @@ fd_status fd_batch_create(const fd_config* cfg, fd_weights w, int max_streams, f
     ok = ok && tmap_out_e4m3(&b->so_hid8B, b->hid, Dm, RB, Dm);
     ok = ok && tmap_out_e4m3(&b->so_hid8R, b->hid, Dm, RR, Dm);
   }
-  b->tm_qB.resize(max_streams);
-  b->tm_q8B.resize(max_streams);
-  b->tm_qR.resize(max_streams);
-  b->tm_q8R.resize(max_streams);
-  for (int i = 0; i < max_streams; ++i) {  // stream i's Q rows (attention reads them alone)
-    const __nv_bfloat16* qb = b->q + static_cast<size_t>(i) * b->Lp * NQ;
-    const __nv_bfloat16* qr = b->q + static_cast<size_t>(i) * b->Rp * NQ;
-    ok = ok && tmap_bf16(&b->tm_qB[i], qb, NQ, d.L, NQ * 2, 64, 128);
-    ok = ok && tmap_bf16(&b->tm_q8B[i], qb, NQ, d.L, NQ * 2, 64, 8);
-    ok = ok && tmap_bf16(&b->tm_qR[i], qr, NQ, b->Rp, NQ * 2, 64, 128);
-    ok = ok && tmap_bf16(&b->tm_q8R[i], qr, NQ, b->Rp, NQ * 2, 64, 8);
-  }
+  ok = ok && tmap_bf16(&b->tm_qB, b->q, NQ, RB, NQ * 2, 64, 128);
+  ok = ok && tmap_bf16(&b->tm_q8B, b->q, NQ, RB, NQ * 2, 64, 8);
+  ok = ok && tmap_bf16(&b->tm_qR, b->q, NQ, RR, NQ * 2, 64, 128);
+  ok = ok && tmap_bf16(&b->tm_q8R, b->q, NQ, RR, NQ * 2, 64, 8);
   // padding rows start (and, being outputs of row-wise kernels on zero inputs, stay) finite
   if (!ok || cudaMemset(b->arena, 0, cur) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
+    cudaFreeHost(b->attn_table_host);
     cudaFreeHost(b->table_host);
     cudaFree(b->arena);
     delete b;
@@ -1516,9 +1531,16 @@ fd_status fd_decode_batch(fd_batch b, fd_handle* hs, int n, const float* const* 
         e.vt_ring = r.vt;
         e.step_dev = hs[i]->state;
         e.rope_t = b->rope + static_cast<size_t>(i) * (1 + d.rt) * bt + (refine ? bt : 0);
+        fd::AttnStream& m = b->attn_table_host[static_cast<size_t>(l) * b->nmax + i];
+        m.k = r.tm_k;
+        m.vt = r.tm_vt;
+        m.step_dev = hs[i]->state;
+        m.err = hs[i]->state + 1;
       }
-    if (cudaMemcpyAsync(b->table, b->table_host,
-                        static_cast<size_t>(d.nb + d.nr) * b->nmax * sizeof(fd::QkvStream),
+    const size_t entries = static_cast<size_t>(d.nb + d.nr) * b->nmax;
+    if (cudaMemcpyAsync(b->table, b->table_host, entries * sizeof(fd::QkvStream),
+                        cudaMemcpyHostToDevice, s) != cudaSuccess ||
+        cudaMemcpyAsync(b->attn_table, b->attn_table_host, entries * sizeof(fd::AttnStream),
                         cudaMemcpyHostToDevice, s) != cudaSuccess)
       return FD_ERR_CUDA;
     b->table_for.assign(hs, hs + n);
@@ -1538,6 +1560,7 @@ fd_status fd_decode_batch(fd_batch b, fd_handle* hs, int n, const float* const* 
 fd_status fd_batch_destroy(fd_batch b) {
   if (b == nullptr) return FD_ERR_INVALID_ARG;
   cudaDeviceSynchronize();
+  cudaFreeHost(b->attn_table_host);
   cudaFreeHost(b->table_host);
   cudaFree(b->arena);
   if (b->w) b->w->live_handles--;
