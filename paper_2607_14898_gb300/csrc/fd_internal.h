@@ -1,5 +1,5 @@
 // Internal launch interface between the host runtime (flashdec.cu) and the kernels
-// (fd_gemm.cu, fd_attn.cu, fd_small.cu). Not part of the public C ABI.
+// (fd_gemm_kernel.cuh and its instances, fd_attn.cu, fd_small.cu). Not part of the public C ABI.
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
