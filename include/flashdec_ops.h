@@ -91,11 +91,11 @@ fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const vo
                           int parts, void* workspace, int* err_dev, void* stream);
 
 /* Allocation-free variant of fd_op_attention. The paper has no counterpart: this is a library
- * convenience for callers that cannot call cudaMalloc, for example code that runs while a CUDA
- * stream is being captured into a graph (allocation is not allowed there), plug-ins that must
- * stay inside a device-memory budget handed to them by a host framework, and real-time loops
- * that cannot afford the device synchronisation an allocation may cause. Such callers can pass
- * their own inputs and outputs but have no way to provide the partial-result workspace.
+ * convenience for callers that cannot call cudaMalloc, for example plug-ins that must stay
+ * inside a device-memory budget handed to them by a host framework (which owns every
+ * allocation), and real-time loops that cannot afford the device synchronisation an allocation
+ * may cause. Such callers can pass their own inputs and outputs but have no way to provide the
+ * partial-result workspace.
  * This call takes that workspace from one array in the library's static device memory,
  * FD_STATIC_ATTN_SCRATCH_BYTES (32 MiB) on every GPU that loads the library, held until the
  * process exits. It allocates nothing: no cudaMalloc, cudaFree or allocating library routine.

@@ -1,8 +1,8 @@
 """fd_op_attention_static: attention whose key-range-split workspace lives in the library's
-static device memory, for callers that cannot allocate device memory (for example while a
-stream is being captured into a CUDA graph, or inside a fixed memory budget). Its results must
-match fd_op_attention run with a caller-allocated workspace, call after call, since every call
-reuses the same static array.
+static device memory, for callers that cannot allocate device memory (a plug-in held to a
+device-memory budget owned by its host framework, or a real-time loop that cannot take an
+allocation's device synchronisation). Its results must match fd_op_attention run with a
+caller-allocated workspace, call after call, since every call reuses the same static array.
 
 This file is collected last on purpose: it must pass in a fresh process and after every other
 test has run in the same process."""
