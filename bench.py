@@ -139,31 +139,15 @@ def run_ours(args, rank: int, world: int):
     import synth
     from paper_2607_14898_gb300 import costs
     from paper_2607_14898_gb300 import flashdec as fdp
+    from paper_2607_14898_gb300.replicas import RankGroup, rank_env, stream_seeds
 
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    local = rank_env().local_rank
     torch.cuda.set_device(local)
     dist = None
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-
-    def barrier():
-        if dist is not None:
-            dist.barrier()
-
-    def max_over_ranks(x: float) -> float:
-        if dist is None:
-            return x
-        t = torch.tensor([x], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
-
-    def sum_over_ranks(x: float) -> float:
-        if dist is None:
-            return x
-        t = torch.tensor([x], device="cuda", dtype=torch.float64)
-        dist.all_reduce(t)
-        return float(t.item())
+    group = RankGroup(dist, "cuda")
 
     cfg = synth.PRESETS[args.workload]
     chunks = cfg.chunks
@@ -175,8 +159,8 @@ def run_ours(args, rank: int, world: int):
     decs = [fdp.Decoder(cfg, weights) for _ in range(S)]
     dec = decs[0]
     # replicas: rank r decodes its own streams (latent seeds r*S .. r*S + S - 1)
-    zs = [torch.from_numpy(synth.make_latents(cfg, seed=cfg.latent_seed + rank * S + i)).cuda()
-          for i in range(S)]
+    seeds = stream_seeds(cfg.latent_seed, rank, S)
+    zs = [torch.from_numpy(synth.make_latents(cfg, seed=sd)).cuda() for sd in seeds]
     z = zs[0]
     out_dtype = torch.uint8 if cfg.out_u8 else torch.float32
     pixs = [[torch.empty(cfg.out_channels, cfg.r_t, cfg.out_h, cfg.out_w, dtype=out_dtype,
@@ -218,7 +202,7 @@ def run_ours(args, rank: int, world: int):
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     launches0 = sum(d.launch_count for d in decs)
-    barrier()
+    group.barrier()
     torch.cuda.synchronize()
     try:
         gpu_id = "GPU-" + str(torch.cuda.get_device_properties(local).uuid)
@@ -231,11 +215,10 @@ def run_ours(args, rank: int, world: int):
                 step(ev[k])
             t1.record(stream)
         torch.cuda.synchronize()
-    barrier()
+    group.barrier()
     gpu_launches = sum(d.launch_count for d in decs) - launches0
     ms_total = t0.elapsed_time(t1)
-    ms_max = max_over_ranks(ms_total)
-    frames_all = sum_over_ranks(frames_per_step * args.steps)
+    value, frames_all, ms_max = group.throughput(frames_per_step * args.steps, ms_total)
     lat = [ev[k][t][0].elapsed_time(ev[k][t][1]) for k in range(args.steps) for t in range(chunks)]
     lat_steady = [ev[k][t][0].elapsed_time(ev[k][t][1]) for k in range(args.steps)
                   for t in range(cfg.window - 1, chunks)]
@@ -286,8 +269,7 @@ def run_ours(args, rank: int, world: int):
     prof_ms_step = sum(ms for _, ms in prof.values()) / args.steps
 
     # ---------------------------------------------------------------- end to end (host buffers)
-    lat_host = [torch.from_numpy(synth.make_latents(cfg, seed=cfg.latent_seed + rank * S + i))
-                .pin_memory() for i in range(S)]
+    lat_host = [torch.from_numpy(synth.make_latents(cfg, seed=sd)).pin_memory() for sd in seeds]
     pix_host = [[torch.empty(pix[0].shape, dtype=out_dtype).pin_memory() for _ in range(chunks)]
                 for _ in range(S)]
 
@@ -303,7 +285,7 @@ def run_ours(args, rank: int, world: int):
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
-    barrier()
+    group.barrier()
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         e0.record(stream)
@@ -311,12 +293,11 @@ def run_ours(args, rank: int, world: int):
             step_host()
         e1.record(stream)
     torch.cuda.synchronize()
-    barrier()
-    e2e_ms = max_over_ranks(e0.elapsed_time(e1))
+    group.barrier()
+    e2e_value, _, _ = group.throughput(frames_per_step * args.steps, e0.elapsed_time(e1))
     latent_bytes = cfg.latent_channels * cfg.latent_h * cfg.latent_w * 4
     pixel_bytes = pix[0].numel() * pix[0].element_size()
 
-    value = frames_all / (ms_max * 1e-3)
     line = {
         "metric": METRIC,
         "value": round(value, 2),
@@ -355,7 +336,7 @@ def run_ours(args, rank: int, world: int):
         "tensor_frac_step": round(flops_step * args.steps / (ms_total * 1e-3) / 1e12
                                   / sustained, 3),
         "clocks": clocks.summary(),
-        "e2e": {"value": round(frames_all / (e2e_ms * 1e-3), 2), "unit": "frames/s",
+        "e2e": {"value": round(e2e_value, 2), "unit": "frames/s",
                 "h2d_bytes_per_step": S * chunks * latent_bytes,
                 "d2h_bytes_per_step": S * chunks * pixel_bytes,
                 "call": "fd_decode_chunk_host (pinned host latents / pixels)"},
@@ -495,8 +476,9 @@ def run_reference(args):
 
 def main():
     args = parse()
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
+    from paper_2607_14898_gb300.replicas import rank_env
+    env = rank_env()
+    rank, world = env.rank, env.world
     if args.impl == "reference":
         if rank != 0:
             return
