@@ -129,6 +129,13 @@ PRESETS: dict[str, FDConfig] = {
     "720p_wide": FDConfig(latent_h=90, latent_w=160, patch=2, hidden=1536, heads=24,
                           kv_groups=3, n_blocks=32, n_refine=2, window=8, r_t=4, out_u8=True,
                           name="720p_wide", chunks=128, latent_mode="ar1"),
+    # the 720p wide model's structure (D=1536, 24 heads / 3 KV groups, 32 + 2 blocks, W=8,
+    # AR(1) latents, uint8) on a 10x13-token frame, 10 chunks: the W=8 window fills and evicts
+    "wide_small": FDConfig(latent_h=20, latent_w=26, patch=2, hidden=1536, heads=24,
+                           kv_groups=3, n_blocks=32, n_refine=2, window=8, r_t=4, out_u8=True,
+                           name="wide_small", chunks=10, latent_mode="ar1"),
+    # degenerate window W=1: every chunk attends to itself only (no temporal context)
+    "tiny_w1": FDConfig(window=1, n_refine=1, r_t=2, name="tiny_w1", chunks=3),
     # refinement exercised at tiny size: r_t=2, one refinement block, 3 chunks
     "tiny_rt": FDConfig(r_t=2, n_refine=1, name="tiny_rt", chunks=3),
     # several M tiles with ragged tails: 10x13=130 tokens (4L = 520), W=3 so eviction runs

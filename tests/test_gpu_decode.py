@@ -56,6 +56,7 @@ def compare(cfg, got, want, what, max_abs=MAX_ABS, mean_abs=MEAN_ABS):
             wc = oracle.quantize_u8(o.float().numpy()).astype(np.int32)
             gc = g.numpy().astype(np.int32)
             d = np.abs(gc - wc)
+            print(f"{what} chunk {t}: max code diff {d.max()} mean {d.mean() / 127.5:.3e}")
             assert d.max() <= 3, f"{what} chunk {t}: max code diff {d.max()}"
             assert d.mean() / 127.5 <= mean_abs, f"{what} chunk {t}: mean {d.mean() / 127.5:.2e}"
         else:
@@ -66,7 +67,8 @@ def compare(cfg, got, want, what, max_abs=MAX_ABS, mean_abs=MEAN_ABS):
 
 
 @pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "small_u8", "tiny_gated",
-                                  "tiny_qk", "small_fp8", "small_f1", "tiny_gated_fp8"])
+                                  "tiny_qk", "small_fp8", "small_f1", "tiny_gated_fp8",
+                                  "tiny_w1"])
 def test_decode_matches_oracle(name):
     cfg = synth.PRESETS[name]
     w, z = synth.make_weights(cfg), synth.make_latents(cfg)
@@ -234,6 +236,21 @@ def test_decode_full_size(name, chunks):
     want = [ref.decode_chunk(z[t]) for t in range(chunks)]
     got = gpu_stream(cfg, w, z, chunks=chunks)
     compare(cfg, got, want, name)
+
+
+@pytest.mark.slow
+def test_decode_wide_model_structure():
+    """The 720p wide model (D = 1536, 24 heads / 3 KV groups, 32 + 2 blocks, W = 8, AR(1)
+    latents, uint8 pixels) on a 130-token frame, 10 chunks: the 8-chunk window fills, then
+    evicts twice. Its full-size stream is too large for the fp64 oracle; every shape that
+    differs from this case (token count) is covered at full size by the kernel tests and the
+    480p / 720p decodes. The oracle's own bf16 / fp16 operand-rounding noise on this case is
+    mean-abs 1.45e-3, so the configurations' bar (2e-3) applies."""
+    cfg = synth.PRESETS["wide_small"]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    want = oracle.decode_stream(cfg, w, z)
+    got = gpu_stream(cfg, w, z)
+    compare(cfg, got, want, "wide_small")
 
 
 @pytest.mark.slow

@@ -419,6 +419,18 @@ def test_eviction_one_block():
     assert torch.allclose(a[3], b[3], atol=1e-13)
 
 
+def test_window_of_one_chunk_decodes_each_chunk_alone():
+    """Degenerate window W = 1: every layer attends to the current chunk only, and RoPE scores
+    depend only on position differences (Sec. 3.2), so chunk t decodes exactly as if it were
+    chunk 0 of a new stream, whatever came before."""
+    cfg, w, z = _setup("tiny_w1")
+    stream = oracle.decode_stream(cfg, w, z)
+    for t in range(cfg.chunks):
+        alone = oracle.decode_stream(cfg, w, z[t:t + 1])[0]
+        assert torch.allclose(stream[t], alone, atol=1e-12)
+    assert not torch.allclose(stream[0], stream[1])   # the chunks themselves differ
+
+
 @pytest.mark.parametrize("name", ["tiny_rt", "small"])
 def test_window_relative_rope_equals_absolute(name):
     """Sec. 4.3: RoPE positions relative to the window give the same scores."""
