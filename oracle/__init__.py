@@ -1,4 +1,5 @@
-"""CPU oracle for the FlashDecoder streaming decode (test infrastructure only).
+"""CPU oracle for the FlashDecoder streaming decode and its training step (test
+infrastructure only; the training step is the submodule ``oracle.training``).
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline / reference arm
 may import this package. The CUDA library and its Python binding never do.

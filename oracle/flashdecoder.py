@@ -309,12 +309,15 @@ class StreamingDecoder:
     (Sec. 4.3 "Long Video Decoding").
     """
 
-    def __init__(self, cfg, weights: dict, rope_mode: str = "abs"):
+    def __init__(self, cfg, weights: dict, rope_mode: str = "abs", detach_cache: bool = False):
         self.cfg = cfg
         self.w = {k: _t(v) for k, v in weights.items()}
         if rope_mode not in ("abs", "window"):
             raise ValueError(rope_mode)
         self.rope_mode = rope_mode
+        # training option (oracle/training.py): keep the cached K / V out of the autograd
+        # graph, so a chunk's gradient stops at the cache; no effect on the values
+        self.detach_cache = detach_cache
         self.reset()
 
     def reset(self) -> None:
@@ -339,7 +342,7 @@ class StreamingDecoder:
             # cache update: concat(tail_{(W-1) L}(K), K_t)  (Algorithm 1)
             K = torch.cat([kc[b][:, max(0, kc[b].shape[1] - tail):], k], dim=1)
             V = torch.cat([vc[b][:, max(0, vc[b].shape[1] - tail):], v], dim=1)
-            kc[b], vc[b] = K, V
+            kc[b], vc[b] = (K.detach(), V.detach()) if self.detach_cache else (K, V)
             if window_rel:
                 n_frames = K.shape[1] // L             # frames now in the window
                 first = frames[-1] + 1 - n_frames      # absolute index of the oldest one
@@ -350,8 +353,9 @@ class StreamingDecoder:
             h = _block_rest(h, o, self.w, p, cfg)
         return h
 
-    def decode_chunk(self, z_t) -> torch.Tensor:
-        """Decode latent frame z_t [C'][H'][W'] -> clamped pixels [C][r_t][H][W] (fp64)."""
+    def decode_chunk(self, z_t, clamp: bool = True) -> torch.Tensor:
+        """Decode latent frame z_t [C'][H'][W'] -> clamped pixels [C][r_t][H][W] (fp64).
+        clamp=False returns the head's output before the clamp (the training loss's input)."""
         cfg, w, t = self.cfg, self.w, self.t
         L, D, rt = cfg.tokens, cfg.hidden, cfg.r_t
         # Project (Eq. projection, with PixelUnshuffle(p) of Sec. 4.3)
@@ -374,7 +378,7 @@ class StreamingDecoder:
         if t == 0 and getattr(cfg, "first_chunk_frames", 0) == 1:
             pix = pix[:, :1]                                        # R16
         self.t += 1
-        return pix.clamp(-1.0, 1.0)
+        return pix.clamp(-1.0, 1.0) if clamp else pix
 
 
 def decode_stream(cfg, weights, latents, rope_mode: str = "abs") -> list[torch.Tensor]:
@@ -394,7 +398,7 @@ def chunk_mask(chunk_of_tok: torch.Tensor, window: int) -> torch.Tensor:
     return (j <= i) & (j > i - window)
 
 
-def decode_full_masked(cfg, weights, latents) -> list[torch.Tensor]:
+def decode_full_masked(cfg, weights, latents, clamp: bool = True) -> list[torch.Tensor]:
     w = {k: _t(v) for k, v in weights.items()}
     T = len(latents)
     L, D, rt = cfg.tokens, cfg.hidden, cfg.r_t
@@ -423,7 +427,9 @@ def decode_full_masked(cfg, weights, latents) -> list[torch.Tensor]:
     y = rms_norm(hf, w["normh.g"], cfg.norm_eps)
     F = linear(gelu(linear(y, w["head1.w"], w["head1.b"])), w["head2.w"], w["head2.b"])
     out = [pixel_shuffle(F[c * rt * L:(c + 1) * rt * L], rt, cfg.grid_h, cfg.grid_w,
-                         cfg.out_channels, cfg.r_s).clamp(-1.0, 1.0) for c in range(T)]
+                         cfg.out_channels, cfg.r_s) for c in range(T)]
+    if clamp:
+        out = [o.clamp(-1.0, 1.0) for o in out]
     if getattr(cfg, "first_chunk_frames", 0) == 1:
         out[0] = out[0][:, :1]                                      # R16
     return out

@@ -23,7 +23,7 @@ import numpy as np
 
 __all__ = [
     "FDConfig", "PRESETS", "weight_layout", "make_weights", "make_latents",
-    "normal", "to_bf16_values",
+    "normal", "to_bf16_values", "frames_of_chunk", "make_target_pixels",
 ]
 
 
@@ -292,3 +292,26 @@ def make_latents(cfg: FDConfig, chunks: int | None = None, seed: int | None = No
     for t in range(1, chunks):
         z[t] = a * z[t - 1] + b * e[t]
     return z
+
+
+def frames_of_chunk(cfg: FDConfig, t: int) -> int:
+    """Output frames of chunk t: r_t, or 1 for chunk 0 under the causal count of Fig. 2."""
+    return 1 if t == 0 and cfg.first_chunk_frames == 1 else cfg.r_t
+
+
+def make_target_pixels(cfg: FDConfig, chunks: int | None = None, seed: int = 77,
+                       min_abs: float = 0.0) -> list[np.ndarray]:
+    """Synthetic ground-truth video for a training step: per chunk fp32
+    [C][frames][H][W] with values in [-1, 1] (normalised pixels). Magnitudes are uniform on
+    [min_abs, 1] with a random sign (min_abs = 0: uniform on [-1, 1])."""
+    chunks = cfg.chunks if chunks is None else chunks
+    out = []
+    for t in range(chunks):
+        shape = (cfg.out_channels, frames_of_chunk(cfg, t), cfg.out_h, cfg.out_w)
+        n = int(np.prod(shape))
+        key = (int(seed) << 32) | (0x7FFE0000 + t)
+        gen = np.random.Generator(np.random.Philox(key=key))
+        mag = gen.uniform(min_abs, 1.0, n).astype(np.float32)
+        sign = np.where(gen.integers(0, 2, n) == 1, np.float32(1.0), np.float32(-1.0))
+        out.append((mag * sign).reshape(shape))
+    return out
