@@ -7,6 +7,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
@@ -378,6 +379,9 @@ struct fd_handle_s {
   size_t arena_bytes = 0;
   int* state = nullptr;  // [0] chunk index t, [1] error bits
   int64_t t_host = 0;
+  // unique for the life of the process: a destroyed handle's address can be reused by a new
+  // one, so tables built for a set of handles remember serials, not addresses
+  uint64_t serial = 0;
   bool error = false;
   cudaStream_t last_stream = nullptr;
   // fd_decode_chunks: a library-owned stream on which this handle's chunk runs beside the
@@ -430,7 +434,7 @@ struct fd_batch_s {
   fd::QkvStream* table_host = nullptr;  // pinned copy
   fd::AttnStream* attn_table = nullptr;       // [n_blocks + n_refine][nmax]: rings' K / V maps
   fd::AttnStream* attn_table_host = nullptr;  // pinned copy
-  std::vector<fd_handle> table_for;     // handles the tables were written for
+  std::vector<uint64_t> table_for;      // serials of the handles the tables were written for
   size_t ws_stride = 0;                 // attention workspace floats per stream
   CUtensorMap tm_x0, tm_uB, tm_uR, tm_oB, tm_oR, tm_hidB, tm_hidR, tm_hidH;
   CUtensorMap so_h, so_hf, so_tup, so_hidB, so_hidR, so_hidH, so_F, so_qB, so_qR;
@@ -1217,6 +1221,8 @@ fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   if (st) return st;
   fd_handle h = new (std::nothrow) fd_handle_s;
   if (h == nullptr) return FD_ERR_OOM;
+  static std::atomic<uint64_t> next_serial{0};
+  h->serial = ++next_serial;
   h->cfg = *cfg;
   h->d = dims_of(cfg);
   h->w = w;
@@ -1518,8 +1524,9 @@ fd_status fd_decode_batch(fd_batch b, fd_handle* hs, int n, const float* const* 
   const Dims& d = b->d;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // the per-layer stream table (rings, counters, RoPE tables) for this set of handles
-  if (b->table_for.size() != static_cast<size_t>(n) ||
-      !std::equal(b->table_for.begin(), b->table_for.end(), hs)) {
+  bool same_set = b->table_for.size() == static_cast<size_t>(n);
+  for (int i = 0; i < n && same_set; ++i) same_set = b->table_for[i] == hs[i]->serial;
+  if (!same_set) {
     if (cudaStreamSynchronize(s) != cudaSuccess) return FD_ERR_CUDA;  // table not in use
     const int bt = rope_band_t();
     for (int l = 0; l < d.nb + d.nr; ++l)
@@ -1543,7 +1550,8 @@ fd_status fd_decode_batch(fd_batch b, fd_handle* hs, int n, const float* const* 
         cudaMemcpyAsync(b->attn_table, b->attn_table_host, entries * sizeof(fd::AttnStream),
                         cudaMemcpyHostToDevice, s) != cudaSuccess)
       return FD_ERR_CUDA;
-    b->table_for.assign(hs, hs + n);
+    b->table_for.resize(n);
+    for (int i = 0; i < n; ++i) b->table_for[i] = hs[i]->serial;
   }
   const fd_status st = decode_batch(b, hs, n, latents_dev, pixels_dev, s);
   for (int i = 0; i < n; ++i) {

@@ -81,6 +81,43 @@ def test_batch_of_one_and_changing_membership():
         compare(cfg, got[s], oracle.decode_stream(cfg, w, z), f"stream {s}")
 
 
+def test_batch_replaced_handle_gets_its_own_rings():
+    """A handle destroyed and replaced by a new one (whose address the allocator may well
+    reuse) in the same batch slot: the batch must rebuild its per-stream tables, so the new
+    stream writes and reads its own rings and matches its own oracle decode."""
+    cfg = synth.PRESETS["tiny_rt"]
+    w = synth.make_weights(cfg)
+    W = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    B = fdp.Batch(cfg, W, 2)
+    za, zb, zc = (synth.make_latents(cfg, seed=s) for s in (20, 21, 22))
+    a, b = fdp.Decoder(cfg, W), fdp.Decoder(cfg, W)
+    got_a, got_c = [], []
+    for t in range(2):
+        pa, pb = pixel_buffer(cfg, t), pixel_buffer(cfg, t)
+        B.decode([a, b], [dev(za[t]), dev(zb[t])], [pa, pb])
+        got_a.append(pa)
+    torch.cuda.synchronize()
+    b.close()
+    c = fdp.Decoder(cfg, W)
+    for t in range(cfg.chunks):
+        if t + 2 < cfg.chunks:
+            pa, pc = pixel_buffer(cfg, t + 2), pixel_buffer(cfg, t)
+            B.decode([a, c], [dev(za[t + 2]), dev(zc[t])], [pa, pc])
+            got_a.append(pa)
+        else:
+            pc = pixel_buffer(cfg, t)
+            B.decode([c], [dev(zc[t])], [pc])
+        got_c.append(pc)
+    torch.cuda.synchronize()
+    assert a.sync_status() == fdp.FD_OK and c.sync_status() == fdp.FD_OK
+    compare(cfg, [p.cpu() for p in got_a], oracle.decode_stream(cfg, w, za), "kept stream")
+    compare(cfg, [p.cpu() for p in got_c], oracle.decode_stream(cfg, w, zc), "new stream")
+    B.close()
+    a.close()
+    c.close()
+    W.close()
+
+
 def test_batch_api_errors():
     cfg = synth.PRESETS["tiny"]
     w = synth.make_weights(cfg)
