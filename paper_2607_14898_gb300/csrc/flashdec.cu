@@ -174,6 +174,13 @@ struct Dims {
 
 bool valid_cfg(const fd_config* c) {
   if (c == nullptr) return false;
+  // upper bounds first, so that the int products below (heads x 64, C' p^2, C r_s^2, ...)
+  // cannot overflow; every real decoder sits far inside them
+  if (c->latent_channels > 4096 || c->patch > 16 || c->heads > 256 || c->kv_groups > 256 ||
+      c->mlp_ratio > 16 || c->n_blocks > 1024 || c->n_refine > 1024 || c->window > 4096 ||
+      c->r_t > 64 || c->vae_spatial > 64 || c->out_channels > 64 || c->latent_h > (1 << 16) ||
+      c->latent_w > (1 << 16))
+    return false;
   if (c->latent_channels < 1 || c->latent_h < 1 || c->latent_w < 1 || c->patch < 1) return false;
   if (c->latent_h % c->patch || c->latent_w % c->patch) return false;
   if (c->heads < 1 || c->kv_groups < 1 || c->heads % c->kv_groups) return false;
@@ -1740,6 +1747,10 @@ fd_status fd_load_state(fd_handle h, const void* host_buf, size_t bytes, void* s
   const int st[2] = {static_cast<int>(hd.t), 0};
   if (!copy_in(h->ringB, h->pitchB) || !copy_in(h->ringR, h->pitchR) ||
       cudaMemcpyAsync(h->state, st, sizeof(st), cudaMemcpyHostToDevice, s) != cudaSuccess)
+    return FD_ERR_CUDA;
+  // as in fd_reset: an attention launch stopped by an error may have left pair counters set
+  if (attn_ws_floats(h->d) > 0 &&
+      cudaMemsetAsync(h->attn_ws, 0, sizeof(int) * attn_pairs(h->d), s) != cudaSuccess)
     return FD_ERR_CUDA;
   h->t_host = hd.t;
   h->error = false;

@@ -70,7 +70,11 @@ def test_state_size_is_header_plus_every_ring():
 
 @pytest.mark.parametrize("field,value", [("hidden", 320), ("heads", 3), ("kv_groups", 3),
                                          ("patch", 3), ("window", 0), ("r_t", 0),
-                                         ("n_blocks", 0), ("latent_channels", 1)])
+                                         ("n_blocks", 0), ("latent_channels", 1),
+                                         # beyond the upper bounds (no int overflow inside)
+                                         ("heads", 1 << 26), ("mlp_ratio", 1 << 20),
+                                         ("vae_spatial", 1 << 12), ("r_t", 1 << 20),
+                                         ("out_channels", 1 << 16)])
 def test_invalid_configs_rejected(field, value):
     L = fdp.lib()
     cfg = synth.PRESETS["small"].replace(**{field: value})
