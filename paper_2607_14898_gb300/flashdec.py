@@ -166,6 +166,34 @@ def _ptr(x) -> int:
     return int(x.data_ptr()) if hasattr(x, "data_ptr") else int(x)
 
 
+def check_buffer(x, what: str, nbytes: int, dtype: str, on_device: bool,
+                 device: int | None = None) -> None:
+    """Refuse a buffer that the library would overrun or misread. The C ABI receives raw
+    pointers and cannot see sizes, so the binding checks, for the stream-level calls, that each
+    buffer is where the call expects it (CUDA device / host), contiguous, of the element type
+    (dtype "float32" or "uint8") and of exactly nbytes bytes."""
+    import torch
+    if isinstance(x, np.ndarray):
+        if on_device:
+            raise TypeError(f"{what}: a CUDA tensor is required, not a numpy array")
+        if x.dtype != np.dtype(dtype) or not x.flags.c_contiguous:
+            raise TypeError(f"{what}: a C-contiguous {dtype} array is required")
+        size = x.nbytes
+    elif isinstance(x, torch.Tensor):
+        if x.is_cuda != on_device:
+            raise TypeError(f"{what}: a {'CUDA' if on_device else 'host'} tensor is required")
+        if on_device and device is not None and x.device.index != device:
+            raise ValueError(f"{what}: on cuda:{x.device.index}, the decoder is on cuda:{device}")
+        if x.dtype != getattr(torch, dtype) or not x.is_contiguous():
+            raise TypeError(f"{what}: a contiguous {dtype} tensor is required")
+        size = x.numel() * x.element_size()
+    else:
+        raise TypeError(f"{what}: a torch tensor{'' if on_device else ' or numpy array'} "
+                        "is required")
+    if size != nbytes:
+        raise ValueError(f"{what}: {size} bytes, the call reads or writes {nbytes}")
+
+
 class Weights:
     """Device copy of the decoder weights (fd_weights_create); shareable by several Decoders."""
 
@@ -204,6 +232,21 @@ class Decoder:
         _check(L.fd_create(ctypes.byref(self.cfg), weights.handle, ctypes.byref(out)),
                "fd_create")
         self.handle = out
+        import torch
+        self.device = torch.cuda.current_device()
+        self._latent_bytes = L.fd_latent_bytes(ctypes.byref(self.cfg))
+        self._pixels_bytes = L.fd_pixels_bytes(ctypes.byref(self.cfg))
+
+    def _check_buffers(self, latent, pixels, on_device: bool) -> None:
+        """The latent of one chunk and the pixels of the next chunk this decoder emits (one
+        frame instead of r_t for chunk 0 under the causal frame count)."""
+        pix = self._pixels_bytes
+        if self.cfg.first_chunk_frames == 1 and self.chunk_index == 0:
+            pix //= self.cfg.r_t
+        dev = self.device if on_device else None
+        check_buffer(latent, "latent", self._latent_bytes, "float32", on_device, dev)
+        check_buffer(pixels, "pixels", pix,
+                     "uint8" if self.cfg.out_dtype == DTYPE_U8 else "float32", on_device, dev)
 
     @property
     def pixels_bytes(self) -> int:
@@ -214,11 +257,13 @@ class Decoder:
         return lib().fd_latent_bytes(ctypes.byref(self.cfg))
 
     def decode_chunk(self, latent, pixels, stream=None) -> None:
+        self._check_buffers(latent, pixels, True)
         _check(lib().fd_decode_chunk(self.handle, _ptr(latent), _ptr(pixels),
                                      _stream_ptr(stream)), "fd_decode_chunk")
 
     def decode_chunk_host(self, latent_host, pixels_host, stream=None) -> None:
         """Decode from / to host buffers (numpy arrays or pinned torch tensors)."""
+        self._check_buffers(latent_host, pixels_host, False)
         lp = latent_host.ctypes.data if isinstance(latent_host, np.ndarray) else _ptr(latent_host)
         pp = pixels_host.ctypes.data if isinstance(pixels_host, np.ndarray) else _ptr(pixels_host)
         _check(lib().fd_decode_chunk_host(self.handle, lp, pp, _stream_ptr(stream)),
@@ -285,6 +330,10 @@ class Decoder:
 
 def decode_chunks(decoders, latents, pixels, stream=None) -> None:
     n = len(decoders)
+    if len(latents) != n or len(pixels) != n:
+        raise ValueError("one latent and one pixel buffer per decoder")
+    for d, z, p in zip(decoders, latents, pixels):
+        d._check_buffers(z, p, True)
     hs = (_P * n)(*[d.handle for d in decoders])
     ls = (_P * n)(*[_ptr(x) for x in latents])
     ps = (_P * n)(*[_ptr(x) for x in pixels])
@@ -306,6 +355,10 @@ class Batch:
     def decode(self, decoders, latents, pixels, stream=None) -> None:
         """One chunk for each decoder (fd_decode_batch)."""
         n = len(decoders)
+        if len(latents) != n or len(pixels) != n:
+            raise ValueError("one latent and one pixel buffer per decoder")
+        for d, z, p in zip(decoders, latents, pixels):
+            d._check_buffers(z, p, True)
         hs = (_P * n)(*[d.handle for d in decoders])
         ls = (_P * n)(*[_ptr(x) for x in latents])
         ps = (_P * n)(*[_ptr(x) for x in pixels])

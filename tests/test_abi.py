@@ -113,3 +113,29 @@ def test_cost_model_matches_the_oracle_flop_count():
     big = synth.PRESETS["480p"]
     a = costs.chunk_flops(big, 10)["attn_backbone"]
     assert a == 24 * 4 * 1560 * (4 * 1560) * 64 * 16
+
+
+def test_binding_refuses_buffers_the_library_would_overrun():
+    """The C ABI takes raw pointers; the binding's stream-level calls check place, type,
+    layout and size of every buffer first (here: the host-buffer rules, checkable without a
+    GPU)."""
+    import numpy as np
+    import torch
+    chk = fdp.check_buffer
+    chk(np.zeros(16, np.float32), "x", 64, "float32", False)
+    chk(torch.zeros(4, 4), "x", 64, "float32", False)
+    chk(torch.zeros(64, dtype=torch.uint8), "x", 64, "uint8", False)
+    bad = [
+        (np.zeros(15, np.float32), "float32", False),          # too small
+        (np.zeros(17, np.float32), "float32", False),          # too large
+        (np.zeros(16, np.float64)[::2].copy(), "float32", False),  # wrong type
+        (np.zeros((4, 8), np.float32)[:, ::2], "float32", False),  # not contiguous
+        (torch.zeros(8, 4).t(), "float32", False),              # not contiguous
+        (torch.zeros(16, dtype=torch.float64), "float32", False),
+        (np.zeros(16, np.float32), "float32", True),            # host array for a device call
+        (torch.zeros(16), "float32", True),                     # host tensor for a device call
+        ([0.0] * 16, "float32", False),                         # not a buffer
+    ]
+    for x, dt, on_dev in bad:
+        with pytest.raises((TypeError, ValueError)):
+            chk(x, "x", 64, dt, on_dev)
