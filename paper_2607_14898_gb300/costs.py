@@ -53,3 +53,14 @@ def chunk_bytes(cfg, t: int) -> dict[str, int]:
 
 def stream_flops(cfg, chunks: int) -> int:
     return sum(sum(chunk_flops(cfg, t).values()) for t in range(chunks))
+
+
+def training_step_flops(cfg, chunks: int) -> dict[str, int]:
+    """Contraction FLOPs of one streaming training step over `chunks` latent frames (the
+    forward passes of Algorithm 1, the L1 pixel loss, every parameter's gradient). Each
+    product's backward is two products of its size (the input and the weight gradient; in
+    attention dQ and dK for the scores, dP and dV for P V), except the patch-embedding, whose
+    input is the latent and needs no gradient."""
+    fwd = stream_flops(cfg, chunks)
+    emb = sum(chunk_flops(cfg, t)["embed"] for t in range(chunks))
+    return {"forward": fwd, "backward": 2 * fwd - emb}

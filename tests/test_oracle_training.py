@@ -186,3 +186,22 @@ def test_causal_training_gradient_of_a_frame_ignores_later_frames():
         acc.append(tr.gradients(loss, ws))
     for k in ga[0]:
         assert torch.equal(ga[0][k], gb[0][k]), k
+
+
+@pytest.mark.parametrize("name", ["tiny_rt", "small", "tiny_gated"])
+def test_training_cost_model_matches_counted_products(name):
+    """costs.training_step_flops against the products the oracle's step actually runs, as
+    PyTorch's FlopCounterMode counts them (forward and autograd's backward separately)."""
+    from torch.utils.flop_counter import FlopCounterMode
+
+    from paper_2607_14898_gb300 import costs
+    cfg, w, z, x = _setup(name)
+    ws = tr.leaf_weights(w)
+    fwd, bwd = FlopCounterMode(display=False), FlopCounterMode(display=False)
+    with fwd:
+        loss = tr.streaming_loss(cfg, ws, z, x)
+    with bwd:
+        tr.gradients(loss, ws)
+    want = costs.training_step_flops(cfg, cfg.chunks)
+    assert fwd.get_total_flops() == want["forward"]
+    assert bwd.get_total_flops() == want["backward"]
