@@ -139,3 +139,22 @@ def test_binding_refuses_buffers_the_library_would_overrun():
     for x, dt, on_dev in bad:
         with pytest.raises((TypeError, ValueError)):
             chk(x, "x", 64, dt, on_dev)
+
+
+def test_empty_inputs_are_refused_before_any_launch():
+    """Zero-sized problems are argument errors, returned before the library touches the
+    device (so this runs without a GPU); an empty list of streams is a no-op."""
+    import ctypes
+    L = fdp.lib()
+    assert L.fd_op_linear(0, 0, 128, 64, 0, 0, 0, 0, 0, 0, 0, 0) == 1      # M = 0
+    assert L.fd_op_linear(0, 128, 0, 64, 0, 0, 0, 0, 0, 0, 0, 0) == 1      # N = 0
+    assert L.fd_op_linear(0, 128, 128, 0, 0, 0, 0, 0, 0, 0, 0, 0) == 1     # K = 0
+    assert L.fd_op_attention(0, 4, 2, 0, 0, 0, 128, 1, 0, 0, 0, 0, 0) == 1  # no queries
+    assert L.fd_op_attention(128, 4, 2, 0, 0, 0, 128, 0, 0, 0, 0, 0, 0) == 1  # no keys
+    assert L.fd_op_attention_static(0, 4, 2, 0, 0, 0, 128, 1, 0, 0, 0, 0) == 1
+    assert L.fd_op_rmsnorm(0, 0, 0, 128, 1e-6, 0, 0) == 1
+    assert L.fd_op_kv_append(0, 0, 2, 0, 2, 0, 128, 0, 0, 0) == 1
+    assert L.fd_op_unshuffle(0, 0, 8, 8, 1, 0, 0) == 1
+    assert L.fd_op_pixel_head(0, 0, 8, 8, 3, 8, 0, 0, 0) == 1
+    assert L.fd_decode_chunks(None, 0, None, None, None) == 1       # no handle array at all
+    assert L.fd_decode_chunks((ctypes.c_void_p * 1)(), 0, None, None, None) == 0  # no streams
