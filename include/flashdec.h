@@ -18,6 +18,9 @@
  *   - Device pointers are CUDA device addresses on the current device; a stream argument is a
  *     cudaStream_t passed as void* (NULL = the legacy default stream).
  *   - A handle is not thread-safe; distinct handles may be used from distinct threads.
+ *   - One GPU per process: the library caches the SM count, the kernels' shared-memory
+ *     attributes and the cluster occupancy for the first device it runs on. Serve several GPUs
+ *     with one process each (independent streams share nothing but the weights).
  *   - Asynchronous device errors (a kernel's bounded wait giving up, a CUDA launch error)
  *     put the handle in the FD_ERR_STATE state: later decode calls fail until fd_reset.
  */
