@@ -116,9 +116,10 @@ def source_hash(*names: str) -> str:
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(kernel_file: str, workload: str):
-    """DRAM bytes per launch of a kernel from the committed ncu summary, if the kernel source
-    has not changed since the counters were taken (else None)."""
+def ncu_traffic(kernel_file: str, workload: str, launch: str):
+    """DRAM bytes of one launch of a kernel (launch = which of its launches was captured) from
+    the committed ncu summary, if the kernel source has not changed since the counters were
+    taken (else None)."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
@@ -126,9 +127,21 @@ def ncu_traffic(kernel_file: str, workload: str):
     with open(path) as fh:
         for line in fh:
             f = line.split()
-            if len(f) >= 4 and f[0] == kernel_file and f[1] == workload and f[2] == cur:
+            if (len(f) >= 5 and f[0] == kernel_file and f[1] == workload and f[2] == cur
+                    and f[4] == launch):
                 return float(f[3])
     return None
+
+
+def attention_traffic(workload: str, prof: dict):
+    """DRAM bytes per attention launch, averaged over the same launches as the achieved rate:
+    the backbone and refinement captures weighted by how many of each were profiled."""
+    tb = ncu_traffic("fd_attn.cu", workload, "backbone")
+    tr = ncu_traffic("fd_attn.cu", workload, "refine")
+    nb, nr = prof["attn_backbone"][0], prof["attn_refine"][0]
+    if tb is None or tr is None or nb + nr == 0:
+        return None
+    return round((tb * nb + tr * nr) / (nb + nr))
 
 
 # ---------------------------------------------------------------------------------- GPU arm
@@ -347,9 +360,11 @@ def run_ours(args, rank: int, world: int):
                      "frac": round(att_tflops / sustained, 3),
                      "peak_source": f"bf16_tflops_sustained ({peak_src}); kernel timed inside "
                                     "a long step",
-                     "traffic": ncu_traffic("fd_attn.cu", cfg.name),
-                     "traffic_launch": "ncu DRAM read+write bytes of one steady-state "
-                                       "refinement launch (profiles/traffic.txt)",
+                     "traffic": attention_traffic(cfg.name, prof),
+                     "traffic_launch": "ncu DRAM read+write bytes per attention launch: one "
+                                       "steady-state backbone and one refinement capture "
+                                       "(profiles/traffic.txt), weighted by the launches "
+                                       "profiled",
                      "flops_per_launch": round(att_flops / att_n),
                      "us_per_launch": round(1e3 * att_ms / att_n, 2),
                      "measured_over": f"{args.steps} profiled steps of the same workload "

@@ -103,3 +103,20 @@ def test_bench_reference_arm_under_torchrun_prints_once(tmp_path):
     assert line["value"] > 0 and line["unit"] == "frames/s"
     assert line["cpu_baseline"]["kind"] == "oracle"
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
+
+
+def test_bench_attention_traffic_is_the_launch_weighted_capture_mean():
+    """The roofline's traffic is per attention launch over the same launch mix as its achieved
+    rate: the committed backbone and refinement captures weighted by launch counts."""
+    import bench
+    tb = bench.ncu_traffic("fd_attn.cu", "480p", "backbone")
+    tr = bench.ncu_traffic("fd_attn.cu", "480p", "refine")
+    prof = {"attn_backbone": (24, 1.0), "attn_refine": (2, 1.0)}
+    if tb is None or tr is None:  # the kernel changed since the captures: no traffic claimed
+        assert bench.attention_traffic("480p", prof) is None
+        return
+    assert tr > tb > 0
+    assert bench.attention_traffic("480p", prof) == round((24 * tb + 2 * tr) / 26)
+    assert bench.attention_traffic("720p", prof) is None          # no capture for 720p
+    assert bench.attention_traffic("480p", {"attn_backbone": (0, 0.0),
+                                            "attn_refine": (0, 0.0)}) is None
