@@ -205,3 +205,18 @@ def test_training_cost_model_matches_counted_products(name):
     want = costs.training_step_flops(cfg, cfg.chunks)
     assert fwd.get_total_flops() == want["forward"]
     assert bwd.get_total_flops() == want["backward"]
+
+
+def test_target_pixels_are_seeded_normalised_frames():
+    """Synthetic ground truth: one [C][frames][H][W] array per chunk in [-1, 1] (one frame
+    for chunk 0 under the causal frame count), magnitudes at least min_abs, same seed same
+    values."""
+    cfg = synth.PRESETS["small_f1"]
+    a, b = synth.make_target_pixels(cfg, min_abs=0.6), synth.make_target_pixels(cfg, min_abs=0.6)
+    assert [x.shape for x in a] == [(3, 1, 160, 208)] + [(3, 4, 160, 208)] * (cfg.chunks - 1)
+    for x, y in zip(a, b):
+        assert np.array_equal(x, y) and x.dtype == np.float32
+        assert float(np.abs(x).min()) >= 0.6 and float(np.abs(x).max()) <= 1.0
+        assert abs(float((x > 0).mean()) - 0.5) < 0.02          # both signs, evenly
+    c = synth.make_target_pixels(cfg, seed=78)
+    assert not np.array_equal(c[1], synth.make_target_pixels(cfg)[1])
