@@ -120,3 +120,42 @@ def test_bench_attention_traffic_is_the_launch_weighted_capture_mean():
     assert bench.attention_traffic("720p", prof) is None          # no capture for 720p
     assert bench.attention_traffic("480p", {"attn_backbone": (0, 0.0),
                                             "attn_refine": (0, 0.0)}) is None
+
+
+def _rank_dies(rank, world, port, out_dir):
+    import datetime
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world,
+                            timeout=datetime.timedelta(seconds=10))
+    if rank == 1:
+        os._exit(3)  # the rank is lost between steps, without any goodbye
+    g = RankGroup(dist, "cpu")
+    try:
+        g.barrier()
+        g.max(1.0)
+        outcome = "no error"
+    except Exception as e:  # the survivors learn of it through the failed collective
+        outcome = "error: " + type(e).__name__
+    with open(os.path.join(out_dir, "rank0.txt"), "w") as fh:
+        fh.write(outcome)
+    os._exit(0)
+
+
+def test_a_lost_rank_fails_the_next_collective_instead_of_hanging(tmp_path):
+    """Failure detection of the replica bookkeeping, on the host: a rank that dies between
+    steps makes the surviving rank's next barrier / reduction raise (connection loss or the
+    process group's timeout) rather than wait forever."""
+    import multiprocessing
+    ctx = multiprocessing.get_context("spawn")
+    port = free_port()
+    procs = [ctx.Process(target=_rank_dies, args=(r, 2, port, str(tmp_path))) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=120)
+    alive = [p for p in procs if p.is_alive()]
+    for p in alive:
+        p.kill()
+    assert not alive, "a rank hung"
+    assert procs[1].exitcode == 3
+    assert (tmp_path / "rank0.txt").read_text().startswith("error")
