@@ -530,3 +530,56 @@ def test_weights_and_latents_are_seeded_and_bf16_exact():
     z = synth.make_latents(synth.PRESETS["720p_wide"].replace(latent_h=4, latent_w=4), chunks=400)
     c = np.corrcoef(z[:-1].ravel(), z[1:].ravel())[0, 1]
     assert abs(c - 0.9) < 0.02                  # AR(1), rho = 0.9
+
+
+def test_uniform_attention_decode_closed_form():
+    """With the query projection zeroed every score is 0, so attention averages the values of
+    the cached window: head n returns the mean over the window's keys of group n // (N/G)'s
+    normalised V (KV-norm, Sec. 3.2). The whole stream (cache windows, out-projection,
+    residuals, MLPs, temporal upsampling, refinement, head) is then written here with plain
+    numpy and compared with the oracle."""
+    cfg, w, z = _setup("tiny_rt", chunks=3)
+    N, G, dh, D, L, rt = cfg.heads, cfg.kv_groups, 64, cfg.hidden, cfg.tokens, cfg.r_t
+    hpg = N // G
+    for k in list(w):
+        if k.endswith("qkv.w") or k.endswith("qkv.b"):
+            w[k] = w[k].copy()
+            w[k][:N * dh] = 0.0                        # Q = 0 (and RoPE of 0 is 0)
+    got = oracle.decode_stream(cfg, w, z)
+    ww = {k: v.astype(np.float64) for k, v in w.items()}
+    erf = np.vectorize(math.erf)
+    eps = cfg.norm_eps
+
+    def rms(a, g):
+        return a / np.sqrt((a ** 2).mean(-1, keepdims=True) + eps) * g
+
+    def gelu(a):
+        return 0.5 * a * (1 + erf(a / math.sqrt(2)))
+
+    def stack(h, prefix, n, cache, t, per_chunk):
+        for b in range(n):
+            p = f"{prefix}.{b}."
+            qkv = rms(h, ww[p + "norm1.g"]) @ ww[p + "qkv.w"].T + ww[p + "qkv.b"]
+            v = qkv[:, (N + G) * dh:].reshape(-1, G, dh)
+            v = rms(v, ww[p + "vnorm.g"])                                 # [rows][G][64]
+            cache.setdefault(p, []).append(v)
+            window = np.concatenate(cache[p][max(0, t - cfg.window + 1):t + 1])
+            mean_v = window.mean(axis=0)                                  # [G][64]
+            o = np.concatenate([mean_v[n_ // hpg] for n_ in range(N)])    # [N * 64]
+            h = h + o @ ww[p + "out.w"].T + ww[p + "out.b"]
+            u2 = rms(h, ww[p + "norm2.g"])
+            h = h + gelu(u2 @ ww[p + "mlp1.w"].T + ww[p + "mlp1.b"]) @ ww[p + "mlp2.w"].T + ww[p + "mlp2.b"]
+        return h
+
+    cache = {}
+    for t in range(cfg.chunks):
+        x0 = oracle.pixel_unshuffle(torch.from_numpy(z[t]).double(), cfg.patch).numpy()
+        h = x0 @ ww["embed.w"].T + ww["embed.b"]
+        h = stack(h, "blocks", cfg.n_blocks, cache, t, L)
+        e = rms(h, ww["normf.g"]) @ ww["tup.w"].T + ww["tup.b"]
+        hf = np.concatenate([e[:, tau * D:(tau + 1) * D] for tau in range(rt)])
+        hf = stack(hf, "refine", cfg.n_refine, cache, t, rt * L)
+        F = gelu(rms(hf, ww["normh.g"]) @ ww["head1.w"].T + ww["head1.b"]) @ ww["head2.w"].T + ww["head2.b"]
+        pix = oracle.pixel_shuffle(torch.from_numpy(F), rt, cfg.grid_h, cfg.grid_w,
+                                   cfg.out_channels, cfg.r_s).numpy()
+        assert np.allclose(got[t].numpy(), np.clip(pix, -1, 1), atol=1e-12), t
