@@ -183,3 +183,83 @@ def test_a_wrong_cache_window_fails_a_pin(delta):
                       pins.test_eviction_one_block)
     finally:
         fd.StreamingDecoder._stack = _orig_stack
+
+
+# ---------------------------------------------------------------- training-step oracle
+import test_oracle_training as tpins  # noqa: E402
+from oracle import backward as bw  # noqa: E402
+from oracle import training as tr  # noqa: E402
+
+_orig_l1 = tr.l1_loss
+_orig_streaming_outputs = tr.streaming_outputs
+
+
+def _l1_sum_not_mean(pixels, targets):
+    return _orig_l1(pixels, targets) * sum(p.numel() for p in pixels)
+
+
+def _outputs_cache_detached(cfg, w, latents, detach_cache=False):
+    return _orig_streaming_outputs(cfg, w, latents, True)
+
+
+TRAIN_MUTATIONS = [
+    ("L1 summed instead of averaged", "l1_loss", _l1_sum_not_mean,
+     [tpins.test_last_layer_gradient_closed_form]),
+    ("gradient stopped at the cache", "streaming_outputs", _outputs_cache_detached,
+     [lambda: tpins.test_streaming_gradients_equal_masked_full_sequence("tiny_rt")]),
+]
+
+
+@pytest.mark.parametrize("what,name,fn,checks", TRAIN_MUTATIONS, ids=[m[0] for m in TRAIN_MUTATIONS])
+def test_a_planted_training_mistake_fails_a_pin(what, name, fn, checks):
+    saved = getattr(tr, name)
+    setattr(tr, name, fn)
+    try:
+        assert caught(*checks), f"no pin caught: {what}"
+    finally:
+        setattr(tr, name, saved)
+
+
+_orig_rms_bwd = bw.rms_norm_bwd
+_orig_attn_bwd = bw.attention_bwd
+
+
+def _rms_bwd_no_projection(x, g, eps, dy):
+    r = 1.0 / torch.sqrt((x * x).mean(dim=-1, keepdim=True) + eps)
+    dx, dg = _orig_rms_bwd(x, g, eps, dy)
+    return r * dy * g, dg                  # the term through r dropped
+
+
+def _attn_bwd_no_delta(q, k, v, do, allowed=None):
+    N, Lq, dh = q.shape
+    G = k.shape[0]
+    scale = 1.0 / math.sqrt(dh)
+    dq, dk, dv = torch.zeros_like(q), torch.zeros_like(k), torch.zeros_like(v)
+    for n in range(N):
+        g = n // (N // G)
+        s = (q[n] @ k[g].T) * scale
+        if allowed is not None:
+            s = s.masked_fill(~allowed, float("-inf"))
+        p = torch.softmax(s, dim=-1)
+        dv[g] += p.T @ do[n]
+        ds = p * (do[n] @ v[g].T)          # the softmax's - delta term dropped
+        dq[n] = ds @ k[g] * scale
+        dk[g] += ds.T @ q[n] * scale
+    return dq, dk, dv
+
+
+BWD_MUTATIONS = [
+    ("RMSNorm backward without the normaliser's term", "rms_norm_bwd", _rms_bwd_no_projection),
+    ("attention backward without delta", "attention_bwd", _attn_bwd_no_delta),
+]
+
+
+@pytest.mark.parametrize("what,name,fn", BWD_MUTATIONS, ids=[m[0] for m in BWD_MUTATIONS])
+def test_a_planted_backward_mistake_fails_a_pin(what, name, fn):
+    import test_oracle_backward as bpins
+    saved = getattr(bw, name)
+    setattr(bw, name, fn)
+    try:
+        assert caught(lambda: bpins.test_explicit_step_equals_autograd_step("tiny_rt")), what
+    finally:
+        setattr(bw, name, saved)
