@@ -263,3 +263,38 @@ def test_a_planted_backward_mistake_fails_a_pin(what, name, fn):
         assert caught(lambda: bpins.test_explicit_step_equals_autograd_step("tiny_rt")), what
     finally:
         setattr(bw, name, saved)
+
+
+# ---------------------------------------------------------------- mistakes inside decode_chunk
+def _mutant_decode_chunk(old, new):
+    """decode_chunk with one line of its source replaced (a planted mistake)."""
+    import inspect
+    import textwrap
+    src = textwrap.dedent(inspect.getsource(fd.StreamingDecoder.decode_chunk))
+    assert src.count(old) == 1, old
+    ns = {}
+    exec(compile(src.replace(old, new), "<mutant>", "exec"), vars(fd), ns)
+    return ns["decode_chunk"]
+
+
+CHUNK_MUTATIONS = [
+    ("upsampled channels read token-major (reading R6 broken)",
+     "hf = e.reshape(L, rt, D).transpose(0, 1).reshape(rt * L, D)",
+     "hf = e.reshape(rt * L, D)",
+     pins.test_identity_blocks_reduce_to_closed_form),
+    ("refined frames all at temporal index t",
+     "[t * rt + tau for tau in range(rt)]",
+     "[t for tau in range(rt)]",
+     lambda: pins.test_streaming_equals_masked_full_sequence("tiny_rt")),
+]
+
+
+@pytest.mark.parametrize("what,old,new,check", CHUNK_MUTATIONS, ids=[m[0] for m in CHUNK_MUTATIONS])
+def test_a_planted_mistake_in_the_chunk_step_fails_a_pin(what, old, new, check):
+    saved = fd.StreamingDecoder.decode_chunk
+    fd.StreamingDecoder.decode_chunk = _mutant_decode_chunk(old, new)
+    try:
+        assert caught(check), f"no pin caught: {what}"
+    finally:
+        fd.StreamingDecoder.decode_chunk = saved
+    check()
