@@ -158,3 +158,20 @@ def test_empty_inputs_are_refused_before_any_launch():
     assert L.fd_op_pixel_head(0, 0, 8, 8, 3, 8, 0, 0, 0) == 1
     assert L.fd_decode_chunks(None, 0, None, None, None) == 1       # no handle array at all
     assert L.fd_decode_chunks((ctypes.c_void_p * 1)(), 0, None, None, None) == 0  # no streams
+
+
+def test_library_is_rebuilt_when_a_source_or_header_changes():
+    """build() recompiles when any kernel source or header is newer than the library, so a
+    stale libflashdec.so is never loaded (checked on the mtimes, without compiling)."""
+    import os
+    from paper_2607_14898_gb300 import build as b
+    fdp.lib()                                   # built and current
+    assert b.up_to_date()
+    hdr = os.path.join(b.INCLUDE, "flashdec.h")
+    st = os.stat(hdr)
+    try:
+        os.utime(hdr, (st.st_atime, os.path.getmtime(b.LIB) + 10))
+        assert not b.up_to_date()
+    finally:
+        os.utime(hdr, (st.st_atime, st.st_mtime))
+    assert b.up_to_date()
