@@ -88,7 +88,25 @@ typedef struct {
                             * frames): chunk 0 emits only its first refined frame   *
                             * (tau = 0; which one is kept is our reading), written  *
                             * as [C][1][H][W]; its cache entries are unchanged      */
+  int32_t rope_mode;       /* temporal RoPE index: FD_ROPE_ABS or FD_ROPE_WINDOW_REL   */
 } fd_config;
+
+/*
+ * Temporal index of the 3D-RoPE (Sec. 3.2), two readings of the paper:
+ *   FD_ROPE_ABS         the offset t * L_frm of Algorithm 1: chunk t's frames sit at temporal
+ *                       index t (backbone) and t r_t + tau (refinement); each key is rotated
+ *                       once, when it enters the cache.
+ *   FD_ROPE_WINDOW_REL  indices counted from the first frame of the current window (Sec. 4.3
+ *                       "Long Video Decoding"), as if the whole window were re-rotated at
+ *                       every chunk.
+ * A score <R(a) q, R(b) k> depends only on b - a, and the window-relative indices of a query
+ * and of a cached key differ by exactly what their absolute indices differ by, so the two
+ * readings give the same scores. The library therefore runs one computation for both: keys
+ * rotated once at their absolute index, with the temporal angles evaluated in double precision
+ * for every chunk (so a long stream loses no accuracy to large indices). The mode is checked
+ * and recorded; the pixels of the two modes are bit-identical.
+ */
+typedef enum { FD_ROPE_ABS = 0, FD_ROPE_WINDOW_REL = 1 } fd_rope_mode;
 
 typedef struct fd_weights_s* fd_weights;
 typedef struct fd_handle_s* fd_handle;
@@ -112,6 +130,10 @@ typedef struct fd_batch_s* fd_batch;
  * with r_s = vae_spatial * patch and M = mlp_ratio. */
 size_t fd_weights_blob_elems(const fd_config* cfg);
 
+/* Bytes of that blob for blob_dtype FD_DTYPE_F32 (4 per element) or FD_DTYPE_BF16 (2): the
+ * blob_bytes fd_weights_create expects. 0 if cfg or blob_dtype is invalid. */
+size_t fd_weights_blob_bytes(const fd_config* cfg, int blob_dtype);
+
 /* Bytes of one latent chunk: C' * H' * W' fp32, layout [C'][H'][W'] row-major. */
 size_t fd_latent_bytes(const fd_config* cfg);
 
@@ -125,22 +147,31 @@ size_t fd_handle_device_bytes(const fd_config* cfg);
 
 /* ------------------------------------------------------------------ weights */
 
-/* Copy a host weight blob (order above) to the device, converting to bf16 (round to nearest
- * even) for the linear weights and keeping biases and gains in fp32.
+/* Load the parameters of the backbone B, the temporal refinement R and the projection / head
+ * MLPs that Algorithm 1 takes as given ("Require: Backbone Transformer B, Temporal Refinement
+ * Transformer R"; block layout Sec. 3.2, head Sec. 3.4 Step 3): copy a host weight blob
+ * (order above) to the device, converting to bf16 (round to nearest even) for the linear
+ * weights and keeping biases and gains in fp32.
  * blob_dtype: FD_DTYPE_F32 or FD_DTYPE_BF16. blob_bytes must equal
- * fd_weights_blob_elems(cfg) * sizeof(element). Synchronous. The caller keeps ownership of
+ * fd_weights_blob_bytes(cfg, blob_dtype). Synchronous. The caller keeps ownership of
  * host_blob; the library owns the device copy until fd_weights_destroy. A weights object may
- * be shared by several handles (it must outlive them). */
+ * be shared by several handles (it must outlive them).
+ * Errors: FD_ERR_CONFIG (cfg invalid), FD_ERR_INVALID_ARG (null pointer, wrong size or
+ * dtype), FD_ERR_OOM, FD_ERR_CUDA, FD_ERR_UNSUPPORTED; *out is set to NULL on error. */
 fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t blob_bytes,
                             int blob_dtype, fd_weights* out);
+/* Free a weights object. FD_ERR_STATE while a handle or batch still uses it. */
 fd_status fd_weights_destroy(fd_weights w);
 
 /* ------------------------------------------------------------------ streams */
 
-/* Create a decoder stream state for cfg (must equal the weights' cfg): KV rings for every
- * layer (backbone G x W L x 64 per K and V; refinement G x r_t W L x 64; K bf16, V fp16
- * stored transposed), activation scratch
- * and a device chunk counter t = 0. Zero-fills the rings. Synchronous. */
+/* Create a decoder stream state for cfg (must equal the weights' cfg): the initialisation
+ * of Algorithm 1, (K^B, V^B) <- empty, (K^R, V^R) <- empty, t = 0. The caches are rings of the
+ * sizes of Eq. kv_cache (Sec. 3.3): for every layer, backbone G x W L x 64 per K and V;
+ * refinement G x r_t W L x 64; K bf16, V fp16 stored transposed. Also allocates the
+ * activation scratch and the device chunk counter. Zero-fills the rings. Synchronous.
+ * Errors: FD_ERR_CONFIG (cfg invalid or not the weights' cfg), FD_ERR_INVALID_ARG (null
+ * pointer), FD_ERR_OOM, FD_ERR_CUDA, FD_ERR_UNSUPPORTED; *out is set to NULL on error. */
 fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out);
 
 /* Decode chunk t (Algorithm 1, one loop iteration) and advance t.
@@ -188,13 +219,19 @@ fd_status fd_batch_destroy(fd_batch b);
 fd_status fd_decode_chunk_host(fd_handle h, const float* latent_host, void* pixels_host,
                                void* stream);
 
-/* Restart the stream: t = 0 and the caches logically empty (their memory is not cleared;
- * stale entries are never read because attention at chunk t reads only chunks <= t).
- * Clears the error state. Stream-ordered: enqueued on the stream of the handle's last decode
- * call, so the next decode on that stream starts from chunk 0 without a host wait. */
+/* Restart the stream: Algorithm 1's initialisation again for a new latent sequence, t = 0 and
+ * the caches logically empty (their memory is not cleared; stale entries are never read
+ * because attention at chunk t reads only chunks <= t). Clears the error state.
+ * Stream-ordered: enqueued on the stream of the handle's last decode call, so the next decode
+ * on that stream starts from chunk 0 without a host wait. A decode on ANOTHER stream must
+ * first wait for that one (e.g. an event), or call fd_sync_status first.
+ * Errors: FD_ERR_INVALID_ARG (null handle), FD_ERR_CUDA. */
 fd_status fd_reset(fd_handle h);
 
-/* Free everything the handle owns (after synchronising its last stream). */
+/* End of the stream (Algorithm 1 returns): free everything the handle owns, the caches
+ * included, after synchronising its last stream. The handle is invalid afterwards; a batch
+ * object that decoded it notices by the handle's serial number if the address comes back for
+ * a new handle. Errors: FD_ERR_INVALID_ARG (null handle). */
 fd_status fd_destroy(fd_handle h);
 
 /* Host-side chunk counter (chunks decoded since create / reset). */

@@ -197,6 +197,7 @@ bool valid_cfg(const fd_config* c) {
   if (c->qk_norm != 0 && c->qk_norm != 1) return false;
   if (c->mlp_fp8 != 0 && c->mlp_fp8 != 1) return false;
   if (c->first_chunk_frames != 0 && c->first_chunk_frames != 1) return false;
+  if (c->rope_mode != FD_ROPE_ABS && c->rope_mode != FD_ROPE_WINDOW_REL) return false;
   if (!(c->norm_eps >= 0.f) || !(c->rope_base > 1.f)) return false;
   const long long L = static_cast<long long>(c->latent_h / c->patch) * (c->latent_w / c->patch);
   if (L * c->r_t * c->window > (1LL << 26)) return false;
@@ -952,6 +953,11 @@ size_t fd_weights_blob_elems(const fd_config* cfg) {
   return n;
 }
 
+size_t fd_weights_blob_bytes(const fd_config* cfg, int blob_dtype) {
+  if (blob_dtype != FD_DTYPE_F32 && blob_dtype != FD_DTYPE_BF16) return 0;
+  return fd_weights_blob_elems(cfg) * (blob_dtype == FD_DTYPE_F32 ? 4 : 2);
+}
+
 size_t fd_latent_bytes(const fd_config* cfg) {
   if (!valid_cfg(cfg)) return 0;
   return static_cast<size_t>(cfg->latent_channels) * cfg->latent_h * cfg->latent_w * 4;
@@ -1015,8 +1021,7 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
   if (!valid_cfg(cfg)) return FD_ERR_CONFIG;
   if (host_blob == nullptr) return FD_ERR_INVALID_ARG;
   if (blob_dtype != FD_DTYPE_F32 && blob_dtype != FD_DTYPE_BF16) return FD_ERR_INVALID_ARG;
-  const size_t esz = blob_dtype == FD_DTYPE_F32 ? 4 : 2;
-  if (blob_bytes != fd_weights_blob_elems(cfg) * esz) return FD_ERR_INVALID_ARG;
+  if (blob_bytes != fd_weights_blob_bytes(cfg, blob_dtype)) return FD_ERR_INVALID_ARG;
   fd_status st = check_device();
   if (st) return st;
   if (!load_encode()) return FD_ERR_CUDA;

@@ -21,6 +21,8 @@ STATUS = {0: "FD_OK", 1: "FD_ERR_INVALID_ARG", 2: "FD_ERR_CONFIG", 3: "FD_ERR_OO
           4: "FD_ERR_CUDA", 5: "FD_ERR_STATE", 6: "FD_ERR_DEVICE_TIMEOUT",
           7: "FD_ERR_UNSUPPORTED"}
 DTYPE_F32, DTYPE_BF16, DTYPE_U8 = 0, 1, 2
+# fd_rope_mode, keyed like the oracle's rope_mode argument
+ROPE_MODES = {"abs": 0, "window": 1}
 EPI_F32, EPI_RESID, EPI_GELU, EPI_TUP, EPI_SWIGLU = 0, 1, 2, 3, 4
 # fd_kernel_kind order
 KERNEL_KINDS = ["unshuffle", "embed", "rmsnorm", "qkv", "attn_backbone", "attn_refine", "out",
@@ -39,7 +41,8 @@ class fd_config(ctypes.Structure):
         "mlp_ratio", "n_blocks", "n_refine", "window", "r_t", "vae_spatial", "out_channels",
         "out_dtype", "mlp_gated")] + [("norm_eps", ctypes.c_float), ("rope_base", ctypes.c_float),
                                       ("qk_norm", ctypes.c_int32), ("mlp_fp8", ctypes.c_int32),
-                                      ("first_chunk_frames", ctypes.c_int32)]
+                                      ("first_chunk_frames", ctypes.c_int32),
+                                      ("rope_mode", ctypes.c_int32)]
 
 
 _P = ctypes.c_void_p
@@ -48,6 +51,7 @@ _F = ctypes.c_float
 _SIGS = {
     "fd_status_str": (ctypes.c_char_p, [_I]),
     "fd_weights_blob_elems": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
+    "fd_weights_blob_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config), _I]),
     "fd_latent_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
     "fd_pixels_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
     "fd_handle_device_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
@@ -127,6 +131,7 @@ def make_config(cfg) -> fd_config:
     c.qk_norm = 1 if cfg.qk_norm else 0
     c.mlp_fp8 = 1 if getattr(cfg, "mlp_fp8", False) else 0
     c.first_chunk_frames = int(getattr(cfg, "first_chunk_frames", 0))
+    c.rope_mode = ROPE_MODES[getattr(cfg, "rope_mode", "abs")]
     c.norm_eps = float(cfg.norm_eps)
     c.rope_base = float(cfg.rope_base)
     return c

@@ -43,6 +43,7 @@ class FDConfig:
     qk_norm: bool = False          # per-head RMSNorm on Q and K instead of on K and V
     mlp_fp8: bool = False          # MLP GEMMs in FP8 (e4m3) with static scales
     first_chunk_frames: int = 0    # 1: chunk 0 emits one frame (causal frame count, Fig. 2)
+    rope_mode: str = "abs"         # temporal RoPE index: "abs" (t L_frm offset) or "window"
     n_blocks: int = 2              # backbone blocks
     n_refine: int = 0              # temporal-refinement blocks
     window: int = 2                # W_frm, counts the current chunk
@@ -134,6 +135,16 @@ PRESETS: dict[str, FDConfig] = {
     "wide_small": FDConfig(latent_h=20, latent_w=26, patch=2, hidden=1536, heads=24,
                            kv_groups=3, n_blocks=32, n_refine=2, window=8, r_t=4, out_u8=True,
                            name="wide_small", chunks=10, latent_mode="ar1"),
+    # the 720p token count (3600 tokens, 14400 refined) at reduced depth (2 + 1 blocks), 5
+    # chunks: the W = 4 rings of both stacks fill and evict
+    "720p_d3": FDConfig(latent_h=90, latent_w=160, patch=2, hidden=1024, heads=16, kv_groups=4,
+                        n_blocks=2, n_refine=1, window=4, r_t=4, out_u8=True, name="720p_d3",
+                        chunks=5),
+    # the 720p wide model's shapes (3600 tokens, D=1536, 24 heads / 3 KV groups, W=8, AR(1)
+    # latents, uint8) at reduced depth (2 + 1 blocks), 3 chunks
+    "720p_wide_d3": FDConfig(latent_h=90, latent_w=160, patch=2, hidden=1536, heads=24,
+                             kv_groups=3, n_blocks=2, n_refine=1, window=8, r_t=4, out_u8=True,
+                             name="720p_wide_d3", chunks=3, latent_mode="ar1"),
     # degenerate window W=1: every chunk attends to itself only (no temporal context)
     "tiny_w1": FDConfig(window=1, n_refine=1, r_t=2, name="tiny_w1", chunks=3),
     # refinement exercised at tiny size: r_t=2, one refinement block, 3 chunks

@@ -40,6 +40,38 @@ def test_blob_layout_matches_seeded_layout_and_binding_order():
         assert [n for n, _, _ in synth.weight_layout(cfg)] == fdp.weight_names(cfg)
 
 
+def test_blob_bytes_is_what_weights_create_expects():
+    """fd_weights_blob_bytes = elements x element size of the blob dtype (fp32 4, bf16 2);
+    any other dtype or an invalid configuration gives 0."""
+    L = fdp.lib()
+    for name in ("tiny", "480p", "xl_480p"):
+        c = fdp.make_config(synth.PRESETS[name])
+        n = L.fd_weights_blob_elems(ctypes.byref(c))
+        assert n > 0
+        assert L.fd_weights_blob_bytes(ctypes.byref(c), fdp.DTYPE_F32) == 4 * n
+        assert L.fd_weights_blob_bytes(ctypes.byref(c), fdp.DTYPE_BF16) == 2 * n
+        assert L.fd_weights_blob_bytes(ctypes.byref(c), fdp.DTYPE_U8) == 0
+        assert L.fd_weights_blob_bytes(ctypes.byref(c), 7) == 0
+    bad = fdp.make_config(synth.PRESETS["small"].replace(heads=3))
+    assert L.fd_weights_blob_bytes(ctypes.byref(bad), fdp.DTYPE_F32) == 0
+    assert L.fd_weights_blob_bytes(None, fdp.DTYPE_F32) == 0
+
+
+def test_rope_mode_is_checked():
+    """fd_config.rope_mode takes FD_ROPE_ABS (0) or FD_ROPE_WINDOW_REL (1); other values make
+    the configuration invalid. The mode does not change the blob."""
+    L = fdp.lib()
+    cfg = synth.PRESETS["small"]
+    n = L.fd_weights_blob_elems(ctypes.byref(fdp.make_config(cfg)))
+    win = fdp.make_config(cfg.replace(rope_mode="window"))
+    assert win.rope_mode == 1
+    assert L.fd_weights_blob_elems(ctypes.byref(win)) == n
+    for v in (2, -1):
+        c = fdp.make_config(cfg)
+        c.rope_mode = v
+        assert L.fd_weights_blob_elems(ctypes.byref(c)) == 0
+
+
 def test_sizes_follow_the_compression_factors():
     L = fdp.lib()
     c = fdp.make_config(synth.PRESETS["480p"])

@@ -47,6 +47,8 @@ def linear_case(M, N, K, seed):
     (1560, 1024, 1024, 96),   # 480p out-projection shape: 13 x 11 tiles of 96, ragged N
     (300, 608, 512, 96),      # ragged M and N with 96-wide tiles
     (6240, 768, 1024, 0),     # 480p head layer 2 on r_t L tokens
+    (200, 256, 192, 128),     # odd number of K blocks: the last two-block stage is half past K
+    (130, 320, 128, 64),      # exactly one two-block stage
 ])
 def test_linear_f32(M, N, K, bn):
     A, W, b = linear_case(M, N, K, seed=M + N + K)
@@ -65,6 +67,7 @@ def test_linear_f32(M, N, K, bn):
     (300, 608, 512, 96),      # ragged M and N; the second CTA of the last pair has no rows
     (6240, 1536, 1024, 192),  # refinement QKV shape, several tiles per pair (persistent)
     (130, 256, 64, 128),      # one K block
+    (520, 512, 320, 256),     # odd number of K blocks on pairs
 ])
 def test_linear_cta_pairs(M, N, K, bn):
     """256-row tiles on CTA pairs (tcgen05 cta_group::2; each CTA holds half of W) compute the
@@ -171,6 +174,7 @@ def assert_e4m3_close(got_codes, want_values, what):
     (520, 1024, 256, 0),     # ragged M, library tile choice
     (1560, 1024, 4096, 96),  # 480p MLP-down shape, 96-wide tiles, 32 K-blocks of 128
     (300, 640, 208, 128),    # K not a multiple of 128: zero-filled K tail
+    (260, 512, 384, 128),    # odd number of 128-element K blocks (two per stage)
 ])
 def test_linear_e4m3_fp32_epilogues(M, N, K, bn):
     """FP8 MLP products (Sec. 4.6): e4m3 operands make every product exact, so the fp32 and
