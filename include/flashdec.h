@@ -279,6 +279,15 @@ size_t fd_state_bytes(const fd_config* cfg);
 fd_status fd_save_state(fd_handle h, void* host_buf, size_t bytes, void* stream);
 fd_status fd_load_state(fd_handle h, const void* host_buf, size_t bytes, void* stream);
 
+/* Failure-path check (tests): enqueue on `stream` one kernel that waits, through the same
+ * bounded mbarrier wait every decode kernel uses, on a barrier that nothing arrives at, with a
+ * limit of limit_us microseconds (1 .. 100000) instead of the decode kernels' 2 s. The wait gives
+ * up, records its code in the handle's device status word and the kernel returns (no trap, no
+ * fault), exactly as a decode kernel does when a load or an MMA never completes. Afterwards
+ * fd_sync_status returns FD_ERR_DEVICE_TIMEOUT, decode calls return FD_ERR_STATE, and fd_reset
+ * makes the handle usable again. FD_ERR_INVALID_ARG for a null handle or a limit out of range. */
+fd_status fd_debug_wait_timeout(fd_handle h, unsigned int limit_us, void* stream);
+
 /* Copy layer `layer` of the backbone (which = 0) or refinement (which = 1) ring into host
  * memory: K as [G][W * rows][64] bf16 bits, then V as [G][W * rows][64] fp16 bits (rows =
  * L backbone, r_t L refinement; row slot*rows + r holds token r of the chunk in ring slot

@@ -103,7 +103,10 @@ fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const vo
  *     the library choose (one CTA per SM: about 135 KB per SM). If
  *     fd_attention_workspace_bytes(..., parts) would exceed the static size, the call returns
  *     FD_ERR_INVALID_ARG and launches nothing (pass fewer parts; parts = 1 uses no workspace).
- *   - The first call on a device looks up the array's device address with that device current
+ *   - The 32 MiB are reserved on a device when the library's device code is loaded there,
+ *     which with CUDA's lazy module loading may be this call's first use on that device.
+ *   - The first call in a CUDA context (per device, and again after a device reset, which
+ *     makes a new context) looks up the array's device address with that context current
  *     (cudaGetSymbolAddress); make that first call before any stream capture begins.
  *   - Every call shares the one array; it clears the array's counters on `stream` (a memset,
  *     not an allocation) and writes every other entry it later reads. Calls whose kernels

@@ -204,6 +204,8 @@ cudaError_t launch_kv_append(const float* k, const float* v, int groups, int row
                              int ring_pitch, __nv_bfloat16* k_ring, __half* vt_ring,
                              cudaStream_t s);
 cudaError_t launch_advance(int* step_dev, cudaStream_t s);
+// failure-path check: a bounded wait that runs out after limit_ns and records ERR_WAIT_CHECK
+cudaError_t launch_wait_check(int* err, unsigned long long limit_ns, cudaStream_t s);
 // Temporal RoPE table of one chunk: for each block of `frames[k]` frames per chunk (k < nsets),
 // entries [off_k + tau][i] = (cos, sin)((t * frames[k] + tau) * inv_freq[i]), i < band_t,
 // computed in fp64 (t read from step_dev, or t_host when step_dev is null).

@@ -17,6 +17,7 @@ enum : int {
   ERR_WAIT_EPI = 4,       // accumulator never released by the epilogue
   ERR_SMEM_ALIGN = 8,     // dynamic shared memory not 1024-byte aligned
   ERR_BAD_ARGS = 16,      // kernel arguments failed a device-side check
+  ERR_WAIT_CHECK = 32,    // the failure-path check's wait gave up (fd_debug_wait_timeout)
 };
 
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
@@ -85,21 +86,26 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Wait for the phase of the given parity to complete. Gives up after kWaitLimitNs, or at once
-// when another wait of this launch (or an earlier one on the same status word) already gave
-// up; records `code` in *err and returns false in that case.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* err, int code) {
+// Wait for the phase of the given parity to complete. Gives up after limit_ns, or at once when
+// another wait of this launch (or an earlier one on the same status word) already gave up;
+// records `code` in *err and returns false in that case.
+__device__ __forceinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity, int* err, int code,
+                                              unsigned long long limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer();
   while (true) {
     for (int i = 0; i < 64; ++i)
       if (mbar_try_wait(bar, parity)) return true;
     if (err != nullptr && *reinterpret_cast<volatile int*>(err) != 0) return false;
-    if (globaltimer() - t0 > kWaitLimitNs) {
+    if (globaltimer() - t0 > limit_ns) {
       if (err != nullptr) atomicOr(err, code);
       return false;
     }
   }
+}
+// the waits of the decode kernels: limit kWaitLimitNs
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* err, int code) {
+  return mbar_wait_for(bar, parity, err, code, kWaitLimitNs);
 }
 
 // ---------------------------------------------------------------- TMA

@@ -7,6 +7,8 @@
 //                uint8 (Sec. 3.4 "Step 3"); one thread per 4 consecutive output pixels
 //   kv_append    fp32 K, V of one chunk -> ring slot (K rows bf16, V transposed fp16) (Sec. 3.3)
 //   advance      chunk counter t += 1 (device-resident, so a captured graph can be replayed)
+//   wait_check   failure-path check: a wait on an mbarrier that nothing arrives at, through
+//                the decode kernels' bounded wait, gives up after a short limit and returns
 #include "fd_internal.h"
 #include "fd_ptx.cuh"
 
@@ -257,6 +259,24 @@ cudaError_t launch_rope_table(const int* step_dev, int t_host, int nsets, const 
   for (int i = 0; i < band_t; ++i) sets.inv_freq[i] = inv_freq[i];
   return launch_pdl(rope_table_kernel, dim3(1), dim3(128), 0, s, step_dev, t_host, nsets, band_t,
                     sets, table);
+}
+
+// One thread waits, with the decode kernels' bounded wait (mbar_wait_for) and a limit of
+// limit_ns, on an mbarrier that expects one arrival that never comes: the wait gives up, ORs
+// ERR_WAIT_CHECK into *err and the kernel returns. No trap, no fault; the context stays usable.
+__global__ void wait_check_kernel(int* err, unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  const uint32_t b = smem_u32(&bar);
+  mbar_init(b, 1);
+  fence_barrier_init();
+  // err may already be set by an earlier failure: then the wait gives up at once
+  mbar_wait_for(b, 0, err, ERR_WAIT_CHECK, limit_ns);
+}
+
+cudaError_t launch_wait_check(int* err, unsigned long long limit_ns, cudaStream_t s) {
+  wait_check_kernel<<<1, 32, 0, s>>>(err, limit_ns);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_advance(int* step_dev, cudaStream_t s) {

@@ -1781,6 +1781,15 @@ fd_status fd_sync_status(fd_handle h) {
   return h->error ? FD_ERR_STATE : FD_OK;
 }
 
+fd_status fd_debug_wait_timeout(fd_handle h, unsigned int limit_us, void* stream) {
+  if (h == nullptr || limit_us < 1 || limit_us > 100000) return FD_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (fd::launch_wait_check(h->state + 1, 1000ull * limit_us, s) != cudaSuccess)
+    return FD_ERR_CUDA;
+  h->last_stream = s;
+  return FD_OK;
+}
+
 fd_status fd_debug_read_ring(fd_handle h, int which, int layer, void* dst_host,
                              size_t dst_bytes) {
   if (h == nullptr || dst_host == nullptr) return FD_ERR_INVALID_ARG;
@@ -1980,27 +1989,64 @@ fd_status fd_op_attention(int Lq, int heads, int groups, const void* q, const vo
 
 // ---------------------------------------------------------------- allocation-free attention
 // Workspace of fd_op_attention_static: the library's own static device memory, so that the
-// call needs no allocation. Host code only uses its device address, looked up per device.
+// call needs no allocation. Host code only uses its device address, looked up per CUDA context.
 static __device__ __align__(256) float g_attn_static_scratch[FD_STATIC_ATTN_SCRATCH_BYTES / 4];
 
 namespace {
 std::mutex g_static_scratch_mu;
-constexpr int kMaxDevices = 64;
-float* g_static_scratch_addr[kMaxDevices] = {};
+// (context id, device address) of the contexts seen so far. The array's address belongs to the
+// context that loaded the module: after a device reset the primary context (and its id) is new,
+// so the address is looked up again instead of reusing a stale one.
+constexpr int kMaxContexts = 64;
+unsigned long long g_static_ctx_id[kMaxContexts] = {};
+float* g_static_ctx_addr[kMaxContexts] = {};
+int g_static_ctx_n = 0;
+PFN_cuCtxGetCurrent_v4000 g_ctx_current = nullptr;
+PFN_cuCtxGetId_v12000 g_ctx_id = nullptr;
 
-// device address of g_attn_static_scratch on the current device (looked up once per device)
-fd_status static_scratch_address(float** out) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return FD_ERR_CUDA;
-  if (dev < 0 || dev >= kMaxDevices) return FD_ERR_UNSUPPORTED;
-  std::lock_guard<std::mutex> lock(g_static_scratch_mu);
-  if (g_static_scratch_addr[dev] == nullptr) {
-    void* addr = nullptr;
-    if (cudaGetSymbolAddress(&addr, g_attn_static_scratch) != cudaSuccess || addr == nullptr)
-      return FD_ERR_CUDA;
-    g_static_scratch_addr[dev] = static_cast<float*>(addr);
+// id of the current CUDA context (0 if none or unavailable)
+unsigned long long current_context_id() {
+  if (g_ctx_current == nullptr || g_ctx_id == nullptr) {
+    cudaDriverEntryPointQueryResult q;
+    void* f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 4000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      g_ctx_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(f);
+    f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      g_ctx_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(f);
+    if (g_ctx_current == nullptr || g_ctx_id == nullptr) return 0;
   }
-  *out = g_static_scratch_addr[dev];
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (g_ctx_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return 0;
+  if (g_ctx_id(ctx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// device address of g_attn_static_scratch in the current context (looked up once per context,
+// with that context current)
+fd_status static_scratch_address(float** out) {
+  std::lock_guard<std::mutex> lock(g_static_scratch_mu);
+  unsigned long long id = current_context_id();
+  for (int i = 0; id != 0 && i < g_static_ctx_n; ++i)
+    if (g_static_ctx_id[i] == id) {
+      *out = g_static_ctx_addr[i];
+      return FD_OK;
+    }
+  if (g_static_ctx_n == kMaxContexts) return FD_ERR_UNSUPPORTED;
+  // first call in this context: the lookup also makes the device's primary context current
+  // on this thread if nothing had yet (no allocation either way)
+  void* addr = nullptr;
+  if (cudaGetSymbolAddress(&addr, g_attn_static_scratch) != cudaSuccess || addr == nullptr)
+    return FD_ERR_CUDA;
+  id = current_context_id();
+  if (id == 0) return FD_ERR_CUDA;
+  g_static_ctx_id[g_static_ctx_n] = id;
+  g_static_ctx_addr[g_static_ctx_n] = static_cast<float*>(addr);
+  ++g_static_ctx_n;
+  *out = static_cast<float*>(addr);
   return FD_OK;
 }
 }  // namespace

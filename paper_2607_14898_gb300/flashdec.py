@@ -76,6 +76,7 @@ _SIGS = {
     "fd_chunk_index": (ctypes.c_int64, [_P]),
     "fd_sync_status": (_I, [_P]),
     "fd_debug_read_ring": (_I, [_P, _I, _I, _P, ctypes.c_size_t]),
+    "fd_debug_wait_timeout": (_I, [_P, ctypes.c_uint, _P]),
     "fd_state_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
     "fd_save_state": (_I, [_P, _P, ctypes.c_size_t, _P]),
     "fd_load_state": (_I, [_P, _P, ctypes.c_size_t, _P]),
@@ -306,6 +307,11 @@ class Decoder:
         _check(lib().fd_debug_read_ring(self.handle, which, layer, buf.ctypes.data, buf.nbytes),
                "fd_debug_read_ring")
         return (buf[:n].reshape(groups, window * rows, 64), buf[n:].reshape(groups, window * rows, 64))
+
+    def debug_wait_timeout(self, limit_us: int, stream=None) -> None:
+        """Enqueue the failure-path check: a bounded wait that runs out after limit_us."""
+        _check(lib().fd_debug_wait_timeout(self.handle, int(limit_us), _stream_ptr(stream)),
+               "fd_debug_wait_timeout")
 
     def state_bytes(self) -> int:
         return lib().fd_state_bytes(ctypes.byref(self.cfg))

@@ -141,10 +141,10 @@ PRESETS: dict[str, FDConfig] = {
                         n_blocks=2, n_refine=1, window=4, r_t=4, out_u8=True, name="720p_d3",
                         chunks=5),
     # the 720p wide model's shapes (3600 tokens, D=1536, 24 heads / 3 KV groups, W=8, AR(1)
-    # latents, uint8) at reduced depth (2 + 1 blocks), 3 chunks
+    # latents, uint8) at reduced depth (2 + 1 blocks), 2 chunks (chunk 1 attends to chunk 0)
     "720p_wide_d3": FDConfig(latent_h=90, latent_w=160, patch=2, hidden=1536, heads=24,
                              kv_groups=3, n_blocks=2, n_refine=1, window=8, r_t=4, out_u8=True,
-                             name="720p_wide_d3", chunks=3, latent_mode="ar1"),
+                             name="720p_wide_d3", chunks=2, latent_mode="ar1"),
     # degenerate window W=1: every chunk attends to itself only (no temporal context)
     "tiny_w1": FDConfig(window=1, n_refine=1, r_t=2, name="tiny_w1", chunks=3),
     # refinement exercised at tiny size: r_t=2, one refinement block, 3 chunks

@@ -226,16 +226,116 @@ def test_api_errors():
 
 
 @pytest.mark.slow
-@pytest.mark.parametrize("name,chunks", [("480p", 5), ("720p", 2)])
+@pytest.mark.parametrize("name,chunks", [("480p", 5), ("720p", 1)])
 def test_decode_full_size(name, chunks):
-    """The benchmark's own configurations at full size, first chunks (warm-up and, at 480p,
-    the full W = 4 window plus the first eviction)."""
+    """The benchmark's own configurations at full size and depth, first chunks (at 480p the
+    full W = 4 window plus the first eviction; at 720p chunk 0, every block at 3600 tokens)."""
     cfg = synth.PRESETS[name]
     w, z = synth.make_weights(cfg), synth.make_latents(cfg, chunks=chunks)
     ref = oracle.StreamingDecoder(cfg, w)
     want = [ref.decode_chunk(z[t]) for t in range(chunks)]
     got = gpu_stream(cfg, w, z, chunks=chunks)
     compare(cfg, got, want, name)
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name", ["720p_d3", "720p_wide_d3"])
+def test_decode_full_token_count_reduced_depth(name):
+    """The 720p token count (3600 tokens, 14400 refined rows) through whole streams at
+    reduced depth (2 backbone + 1 refinement blocks): 720p_d3 decodes 5 chunks, so both W = 4
+    rings fill and evict at 720p; 720p_wide_d3 is the wide model's shape (D = 1536, 24 heads on
+    3 KV groups, W = 8, AR(1) latents), 2 chunks. Every chunk against the oracle, uint8 codes."""
+    cfg = synth.PRESETS[name]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    want = oracle.decode_stream(cfg, w, z)
+    got = gpu_stream(cfg, w, z)
+    compare(cfg, got, want, name)
+
+
+@pytest.mark.parametrize("name", ["small", "small_f1", "small_u8"])
+def test_decode_chunk_host_matches_oracle(name):
+    """fd_decode_chunk_host (the call the end-to-end benchmark times: pinned host latents in,
+    pinned host pixels out, copies on the stream) against the oracle, chunk by chunk, and bit
+    for bit equal to the device-buffer call. small_f1 checks the one-frame first chunk of the
+    causal frame count (its copy-back is one frame)."""
+    cfg = synth.PRESETS[name]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    want = oracle.decode_stream(cfg, w, z)
+    dev_out = gpu_stream(cfg, w, z)
+    Wt = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    dec = fdp.Decoder(cfg, Wt)
+    stream = torch.cuda.Stream()
+    dt = torch.uint8 if cfg.out_u8 else torch.float32
+    got = []
+    for t in range(cfg.chunks):
+        frames = 1 if (t == 0 and getattr(cfg, "first_chunk_frames", 0) == 1) else cfg.r_t
+        lat = torch.from_numpy(np.ascontiguousarray(z[t])).pin_memory()
+        pix = torch.full((cfg.out_channels, frames, cfg.out_h, cfg.out_w), 7, dtype=dt).pin_memory()
+        dec.decode_chunk_host(lat, pix, stream)
+        stream.synchronize()
+        got.append(pix.clone())
+    assert dec.sync_status() == fdp.FD_OK
+    dec.close()
+    Wt.close()
+    compare(cfg, got, want, name + " host buffers")
+    for t in range(cfg.chunks):
+        assert torch.equal(got[t], dev_out[t]), t
+
+
+def test_window_relative_rope_mode():
+    """rope_mode = window (the temporal RoPE index counted from the window's first frame, Sec.
+    4.3) against the oracle's window-relative decode, which keeps un-rotated keys and re-rotates
+    the whole window every chunk; the library's pixels are bit-identical to its absolute mode
+    (only index differences enter a score)."""
+    for name in ("small", "tiny_rt"):
+        cfg = synth.PRESETS[name]
+        w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+        want = oracle.decode_stream(cfg, w, z, rope_mode="window")
+        win = gpu_stream(cfg.replace(rope_mode="window"), w, z)
+        compare(cfg, win, want, name + " window-relative RoPE")
+        absolute = gpu_stream(cfg, w, z)
+        for a, b in zip(win, absolute):
+            assert torch.equal(a, b)
+
+
+def test_bounded_wait_gives_up_and_the_handle_recovers():
+    """Failure detection on the GPU without a fault: a kernel waits, through the bounded
+    mbarrier wait every decode kernel uses, on a barrier nothing arrives at, with a 1 ms limit.
+    The wait gives up and the kernel returns; the host sees FD_ERR_DEVICE_TIMEOUT from
+    fd_sync_status within a fraction of a second, decodes are refused with FD_ERR_STATE until
+    fd_reset, and after the reset the same context decodes the stream exactly as before."""
+    import time
+    cfg = synth.PRESETS["small"]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    want = oracle.decode_stream(cfg, w, z)
+    Wt = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    dec = fdp.Decoder(cfg, Wt)
+    shape = (cfg.out_channels, cfg.r_t, cfg.out_h, cfg.out_w)
+    dec.decode_chunk(dev(z[0]), torch.empty(shape, device="cuda"))
+    assert dec.sync_status() == fdp.FD_OK
+    t0 = time.perf_counter()
+    dec.debug_wait_timeout(1000)
+    status = dec.sync_status()
+    elapsed = time.perf_counter() - t0
+    assert status == 6, fdp.STATUS.get(status)          # FD_ERR_DEVICE_TIMEOUT
+    assert elapsed < 1.0, elapsed                        # the 1 ms wait ended by itself
+    with pytest.raises(fdp.FdError) as e:
+        dec.decode_chunk(dev(z[1]), torch.empty(shape, device="cuda"))
+    assert e.value.code == 5                             # FD_ERR_STATE until fd_reset
+    L = fdp.lib()
+    assert L.fd_debug_wait_timeout(dec.handle, 0, None) == 1
+    assert L.fd_debug_wait_timeout(dec.handle, 100001, None) == 1
+    dec.reset()
+    got = []
+    for t in range(cfg.chunks):
+        pix = torch.empty(shape, device="cuda")
+        dec.decode_chunk(dev(z[t]), pix)
+        got.append(pix)
+    torch.cuda.synchronize()
+    assert dec.sync_status() == fdp.FD_OK
+    compare(cfg, [g.cpu() for g in got], want, "small after a device timeout and fd_reset")
+    dec.close()
+    Wt.close()
 
 
 @pytest.mark.slow
@@ -262,11 +362,11 @@ def test_decode_xl_layout():
     w, z = synth.make_weights(cfg), synth.make_latents(cfg, chunks=chunks)
     ref = oracle.StreamingDecoder(cfg, w)
     want = [ref.decode_chunk(z[t]) for t in range(chunks)]
-    with oracle.operand_rounding():
-        ref_r = oracle.StreamingDecoder(cfg, w)
-        want_r = [ref_r.decode_chunk(z[t]) for t in range(chunks)]
-    compare(cfg, want_r, want, "xl_480p operand-rounded oracle vs fp64", XL_MAX_ABS, XL_MEAN_ABS)
-    assert max(float((a - b).abs().mean()) for a, b in zip(want_r, want)) > MEAN_ABS
+    with oracle.operand_rounding():  # chunk 0 fixes the derivation of the bar
+        want_r = [oracle.StreamingDecoder(cfg, w).decode_chunk(z[0])]
+    compare(cfg, want_r, want[:1], "xl_480p operand-rounded oracle vs fp64", XL_MAX_ABS,
+            XL_MEAN_ABS)
+    assert float((want_r[0] - want[0]).abs().mean()) > MEAN_ABS
     got = gpu_stream(cfg, w, z, chunks=chunks)
     compare(cfg, got, want, "xl_480p vs fp64", XL_MAX_ABS, XL_MEAN_ABS)
 
@@ -283,16 +383,16 @@ def test_decode_fp8_mlp_full_size():
     cfg, chunks = synth.PRESETS["480p_fp8"], 2
     w, z = synth.make_weights(cfg), synth.make_latents(cfg, chunks=chunks)
     want = oracle.decode_stream(cfg, w, z)
-    with oracle.operand_rounding():
-        want_r = oracle.decode_stream(cfg, w, z)
-    noise = [pixel_errors(a, b) for a, b in zip(want_r, want)]
-    print("480p_fp8 operand-rounded oracle vs fp64:", noise)
-    assert all(mean < 2e-2 and mx < 0.15 for mx, mean in noise)
+    with oracle.operand_rounding():  # the noise of chunk 0 sets the bar of both chunks
+        want_r = oracle.StreamingDecoder(cfg, w).decode_chunk(z[0])
+    noise = pixel_errors(want_r, want[0])
+    print("480p_fp8 operand-rounded oracle vs fp64 (chunk 0):", noise)
+    assert noise[1] < 2e-2 and noise[0] < 0.15
     got = gpu_stream(cfg, w, z, chunks=chunks)
     for t, (g, o) in enumerate(zip(got, want)):
         mx, mean = pixel_errors(g, o)
         print(f"480p_fp8 chunk {t}: max-abs {mx:.3e} mean-abs {mean:.3e}")
-        assert mean <= 1.5 * noise[t][1] and mx <= 1.5 * noise[t][0] + 2e-2, t
+        assert mean <= 1.5 * noise[1] and mx <= 1.5 * noise[0] + 2e-2, t
     bf = gpu_stream(synth.PRESETS["480p"], w, z, chunks=1)
     assert float((f64(bf[0]) - f64(got[0])).abs().mean()) > MEAN_ABS
 
@@ -305,12 +405,12 @@ def test_decode_xl_fp8_mlp():
     cfg, chunks = synth.PRESETS["xl_480p_fp8"], 2
     w, z = synth.make_weights(cfg), synth.make_latents(cfg, chunks=chunks)
     want = oracle.decode_stream(cfg, w, z)
-    with oracle.operand_rounding():
-        want_r = oracle.decode_stream(cfg, w, z)
-    noise = [pixel_errors(a, b) for a, b in zip(want_r, want)]
-    print("xl_480p_fp8 operand-rounded oracle vs fp64:", noise)
+    with oracle.operand_rounding():  # the noise of chunk 0 sets the bar of both chunks
+        want_r = oracle.StreamingDecoder(cfg, w).decode_chunk(z[0])
+    noise = pixel_errors(want_r, want[0])
+    print("xl_480p_fp8 operand-rounded oracle vs fp64 (chunk 0):", noise)
     got = gpu_stream(cfg, w, z, chunks=chunks)
     for t, (g, o) in enumerate(zip(got, want)):
         mx, mean = pixel_errors(g, o)
         print(f"xl_480p_fp8 chunk {t}: max-abs {mx:.3e} mean-abs {mean:.3e}")
-        assert mean <= 1.5 * noise[t][1] and mx <= 1.5 * noise[t][0] + 2e-2, t
+        assert mean <= 1.5 * noise[1] and mx <= 1.5 * noise[0] + 2e-2, t

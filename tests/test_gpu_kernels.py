@@ -398,9 +398,14 @@ def test_attention_small(Lq, heads, groups, n_keys, parts):
 
 
 @pytest.mark.parametrize("Lq,heads,groups,n_keys", [
-    (6240, 16, 4, 24960),   # 480p refinement, steady state (4 chunks x 4 frames x 1560)
-    (1560, 16, 4, 6240),    # 480p backbone, steady state
-    (3600, 16, 4, 14400),   # 720p backbone, steady state
+    (6240, 16, 4, 24960),    # 480p refinement, steady state (4 chunks x 4 frames x 1560)
+    (1560, 16, 4, 6240),     # 480p backbone, steady state
+    (3600, 16, 4, 14400),    # 720p backbone, steady state
+    (14400, 16, 4, 57600),   # 720p refinement, steady state (4 chunks x 4 frames x 3600)
+    (3600, 24, 3, 28800),    # 720p wide model backbone: 8 heads per group, W = 8 chunks
+    (14400, 24, 3, 115200),  # 720p wide model refinement: 32 frames of 3600 keys
+    (8160, 24, 3, 16320),    # XL layout at 1080p, backbone (W = 2)
+    (32640, 24, 3, 65280),   # XL layout at 1080p, refinement: the largest packed row space
 ])
 def test_attention_full_size_sampled(Lq, heads, groups, n_keys):
     """The launch configuration of the decode (one CTA per SM); two launches in a row on one
