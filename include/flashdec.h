@@ -288,6 +288,37 @@ fd_status fd_load_state(fd_handle h, const void* host_buf, size_t bytes, void* s
  * makes the handle usable again. FD_ERR_INVALID_ARG for a null handle or a limit out of range. */
 fd_status fd_debug_wait_timeout(fd_handle h, unsigned int limit_us, void* stream);
 
+/* ------------------------------------------------------------------ training step */
+
+/* One streaming training step (Sec. 3.3 "Training--Inference Consistency"; Sec. 3.5 Eq. loss,
+ * its L1 term): the loss of a clip of T latent frames against its target video and the
+ * gradient of every decoder parameter. Training through the rolling cache has the gradient of
+ * one pass over the clip under the block sliding-window mask, and the step computes exactly
+ * that: every chunk's forward with its activations kept (the attention of query chunk i over
+ * key chunks i-W < j <= i), the L1 term, then the backward, all in the library's kernels (the
+ * products on the tcgen05 GEMM, bf16 operands, fp32 accumulation).
+ * Readings: the loss takes the head's output before the clamp (T1); the mean of |x_hat - x|
+ * over every pixel of the clip (T3); the gradient flows through the cache (T2).
+ *   fd_train_create: a trainer for clips of `chunks` (1 .. 256) latent frames of cfg (equal to
+ *     the weights' cfg; the GELU MLP in bf16 with r_t frames from every chunk: mlp_gated,
+ *     mlp_fp8 and first_chunk_frames give FD_ERR_CONFIG). Allocates the saved activations and
+ *     scratch, transposes the weights; synchronous. The trainer is a user of w.
+ *   fd_train_step: latents device fp32 [T][C'][H'][W']; targets device fp32
+ *     [T][C][r_t][H' 8][W' 8] (the pixels of each chunk, fd_pixels_bytes apart); loss: one
+ *     device fp32; grads: device fp32 of fd_train_grad_elems(cfg) elements, written in the
+ *     weight-blob order (each tensor's gradient where its weights sit in the blob). 16-byte
+ *     aligned buffers. Enqueued on `stream`; a trainer runs one step at a time.
+ *   fd_train_status: synchronise `stream`, then FD_OK, or FD_ERR_DEVICE_TIMEOUT if a kernel's
+ *     bounded wait gave up during the last step.
+ * Errors: FD_ERR_INVALID_ARG, FD_ERR_CONFIG, FD_ERR_OOM, FD_ERR_CUDA. */
+typedef struct fd_trainer_s* fd_trainer;
+size_t fd_train_grad_elems(const fd_config* cfg);
+fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_trainer* out);
+fd_status fd_train_step(fd_trainer tr, const float* latents, const float* targets, float* loss,
+                        float* grads, void* stream);
+fd_status fd_train_status(fd_trainer tr, void* stream);
+fd_status fd_train_destroy(fd_trainer tr);
+
 /* Copy layer `layer` of the backbone (which = 0) or refinement (which = 1) ring into host
  * memory: K as [G][W * rows][64] bf16 bits, then V as [G][W * rows][64] fp16 bits (rows =
  * L backbone, r_t L refinement; row slot*rows + r holds token r of the chunk in ring slot

@@ -1,6 +1,6 @@
 """Build the CUDA library libflashdec.so in-tree (sm_103a only).
 
-Five translation units compiled in parallel with nvcc, then linked into
+Six translation units compiled in parallel with nvcc, then linked into
 ``paper_2607_14898_gb300/_build/libflashdec.so``. Rebuilds only when a source or header is
 newer than the library.
 """
@@ -17,7 +17,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libflashdec.so")
-SOURCES = ["flashdec.cu", "fd_gemm.cu", "fd_gemm_qkv.cu", "fd_attn.cu", "fd_small.cu"]
+SOURCES = ["flashdec.cu", "fd_gemm.cu", "fd_gemm_qkv.cu", "fd_attn.cu", "fd_small.cu",
+           "fd_train.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

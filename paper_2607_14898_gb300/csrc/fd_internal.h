@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <cstdint>
 
+#include "flashdec.h"
+
 namespace fd {
 
 // Launch with programmatic stream serialization (the kernel must call grid_dep_wait before it
@@ -213,6 +215,19 @@ cudaError_t launch_rope_table(const int* step_dev, int t_host, int nsets, const 
                               int band_t, const double* inv_freq, float2* table,
                               cudaStream_t s);
 constexpr int kMaxRopeSets = 2;
+
+// ---- hooks of the training step (fd_train.cu) into the runtime (flashdec.cu)
+// the weights object's configuration; device address of every blob tensor in blob order
+// (returns the number of tensors); the weights object counts one more / one less user
+const fd_config* weights_config(fd_weights w);
+size_t weights_entries(fd_weights w, const void** ptrs, size_t n);
+void weights_add_user(fd_weights w, int delta);
+// out[M][N] (fp32, row pitch ldo) = A[M][K] (bf16, row pitch lda) W[N][K]^T (bf16, row pitch
+// ldw) + bias, stored (EPI_F32) or added into out (EPI_RESID); pitches in elements, N % 32 == 0,
+// lda, ldw % 8 == 0, ldo % 4 == 0, 16-byte aligned pointers
+cudaError_t gemm_view(int epi, int M, int N, int K, const __nv_bfloat16* A, int lda,
+                      const __nv_bfloat16* W, int ldw, const float* bias, float* out, int ldo,
+                      int* err, cudaStream_t s);
 
 // GEMM tile widths compiled in
 inline bool gemm_bn_supported(int bn) {

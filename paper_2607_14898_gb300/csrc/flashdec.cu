@@ -362,6 +362,7 @@ struct fd_weights_s {
   fd_config cfg;
   Dims d;
   void* arena = nullptr;
+  std::vector<void*> entry;  // device address of every blob tensor, in blob order
   Linear embed, tup, head1, head2;
   float *g_f = nullptr, *g_h = nullptr;
   std::vector<LayerW> blocks, refine;
@@ -1113,6 +1114,7 @@ fd_status fd_weights_create(const fd_config* cfg, const void* host_blob, size_t 
     return FD_ERR_OOM;
   }
   uint8_t* base = static_cast<uint8_t*>(w->arena);
+  for (size_t i = 0; i < layout.size(); ++i) w->entry.push_back(base + doff[i]);
   size_t idx = 0;
   auto next = [&]() { return base + doff[idx++]; };
   auto host_f32 = [&](size_t entry) { return reinterpret_cast<const float*>(&stage[doff[entry]]); };
@@ -1223,6 +1225,52 @@ fd_status fd_weights_destroy(fd_weights w) {
   delete w;
   return FD_OK;
 }
+
+}  // extern "C"
+
+// ---------------------------------------------------------------- hooks of the training step
+namespace fd {
+
+const fd_config* weights_config(fd_weights w) { return w ? &w->cfg : nullptr; }
+
+size_t weights_entries(fd_weights w, const void** ptrs, size_t n) {
+  if (w == nullptr) return 0;
+  for (size_t i = 0; i < n && i < w->entry.size(); ++i) ptrs[i] = w->entry[i];
+  return w->entry.size();
+}
+
+void weights_add_user(fd_weights w, int delta) {
+  if (w) w->live_handles += delta;
+}
+
+cudaError_t gemm_view(int epi, int M, int N, int K, const __nv_bfloat16* A, int lda,
+                      const __nv_bfloat16* W, int ldw, const float* bias, float* out, int ldo,
+                      int* err, cudaStream_t s) {
+  if ((epi != EPI_F32 && epi != EPI_RESID) || M < 1 || N < 1 || K < 1 || N % 32 || lda % 8 ||
+      ldw % 8 || ldo % 4 || K > lda || K > ldw || N > ldo || !aligned16(A) || !aligned16(W) ||
+      !aligned16(out) || !aligned16(bias))
+    return cudaErrorInvalidValue;
+  const TileChoice t = pick_tile(M, N, K, 32, false);
+  CUtensorMap ta, tb, to;
+  if (!tmap_bf16(&ta, A, K, M, static_cast<uint64_t>(lda) * 2, 64, 128) ||
+      !tmap_bf16(&tb, W, K, N, static_cast<uint64_t>(ldw) * 2, 64, t.pair ? t.bn / 2 : t.bn) ||
+      !tmap_out_f32(&to, out, N, M, ldo))
+    return cudaErrorInvalidValue;
+  GemmParams p{};
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.epi = epi;
+  p.bias = bias;
+  p.out_f32 = out;
+  p.ld_out = ldo;
+  p.err = err;
+  return launch_gemm(ta, tb, to, to, to, p, t.bn, t.pair, num_sms(), s);
+}
+
+}  // namespace fd
+
+extern "C" {
 
 fd_status fd_create(const fd_config* cfg, fd_weights w, fd_handle* out) {
   if (out == nullptr || w == nullptr) return FD_ERR_INVALID_ARG;

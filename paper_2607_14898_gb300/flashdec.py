@@ -77,6 +77,11 @@ _SIGS = {
     "fd_sync_status": (_I, [_P]),
     "fd_debug_read_ring": (_I, [_P, _I, _I, _P, ctypes.c_size_t]),
     "fd_debug_wait_timeout": (_I, [_P, ctypes.c_uint, _P]),
+    "fd_train_grad_elems": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
+    "fd_train_create": (_I, [ctypes.POINTER(fd_config), _P, _I, ctypes.POINTER(_P)]),
+    "fd_train_step": (_I, [_P, _P, _P, _P, _P, _P]),
+    "fd_train_status": (_I, [_P, _P]),
+    "fd_train_destroy": (_I, [_P]),
     "fd_state_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
     "fd_save_state": (_I, [_P, _P, ctypes.c_size_t, _P]),
     "fd_load_state": (_I, [_P, _P, ctypes.c_size_t, _P]),
@@ -330,6 +335,52 @@ class Decoder:
     def close(self) -> None:
         if getattr(self, "handle", None):
             _check(lib().fd_destroy(self.handle), "fd_destroy")
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class Trainer:
+    """Streaming training step over clips of `chunks` latent frames (fd_train_create)."""
+
+    def __init__(self, cfg, weights: Weights, chunks: int):
+        L = lib()
+        self.cfg = make_config(cfg)
+        self.weights = weights
+        self.chunks = int(chunks)
+        out = _P()
+        _check(L.fd_train_create(ctypes.byref(self.cfg), weights.handle, self.chunks,
+                                 ctypes.byref(out)), "fd_train_create")
+        self.handle = out
+        import torch
+        self.device = torch.cuda.current_device()
+        self.grad_elems = L.fd_train_grad_elems(ctypes.byref(self.cfg))
+        self._latent_bytes = self.chunks * L.fd_latent_bytes(ctypes.byref(self.cfg))
+        self._target_bytes = self.chunks * L.fd_pixels_bytes(ctypes.byref(self.cfg))
+
+    def step(self, latents, targets, loss, grads, stream=None) -> None:
+        """latents fp32 [T][C'][H'][W'], targets fp32 [T][C][r_t][H][W], loss fp32 [1], grads
+        fp32 [grad_elems], all on the trainer's device."""
+        dev = self.device
+        check_buffer(latents, "latents", self._latent_bytes, "float32", True, dev)
+        check_buffer(targets, "targets", self._target_bytes * (4 if self.cfg.out_dtype ==
+                                                                DTYPE_U8 else 1),
+                     "float32", True, dev)
+        check_buffer(loss, "loss", 4, "float32", True, dev)
+        check_buffer(grads, "grads", 4 * self.grad_elems, "float32", True, dev)
+        _check(lib().fd_train_step(self.handle, _ptr(latents), _ptr(targets), _ptr(loss),
+                                   _ptr(grads), _stream_ptr(stream)), "fd_train_step")
+
+    def status(self, stream=None) -> int:
+        return lib().fd_train_status(self.handle, _stream_ptr(stream))
+
+    def close(self) -> None:
+        if getattr(self, "handle", None):
+            _check(lib().fd_train_destroy(self.handle), "fd_train_destroy")
             self.handle = None
 
     def __del__(self):
