@@ -159,6 +159,28 @@ fd_status fd_op_unshuffle(const float* z, int C, int H, int W, int p, void* x0, 
 fd_status fd_op_pixel_head(const float* F, int frames, int grid_h, int grid_w, int channels,
                            int rs, int out_dtype, void* pixels, void* stream);
 
+/* ---- single kernels of the training step (fd_train_step), for per-kernel checks ---- */
+
+/* RMSNorm backward (the derivative of y = x r g, r = (mean(x^2) + eps)^(-1/2), Sec. 3.2):
+ * dx = r (dy g) - x r^3 sum_j(dy_j g_j x_j) / D and dg = sum over rows of dy x r.
+ * x, dy, dx fp32 [M][D]; g, dg fp32 [D]; work: fp32 [M][D] scratch of the caller. */
+fd_status fd_op_rmsnorm_bwd(const float* x, const float* g, const float* dy, int M, int D,
+                            float eps, float* dx, float* dg, float* work, void* stream);
+
+/* GELU backward, exact form: dz = da (Phi(z) + z phi(z)); fp32 z, da, dz and a bf16 copy of dz
+ * (the operand of the next products), n elements each. */
+fd_status fd_op_gelu_bwd(const float* z, const float* da, int64_t n, float* dz, void* dz_bf16,
+                         void* stream);
+
+/* The L1 term of one chunk's pixels through the pixel shuffle (Sec. 3.4 Step 3, Sec. 3.5 Eq.
+ * loss): F fp32 [frames grid_h grid_w][channels rs^2] (refined token tau L + l), target fp32
+ * [channels][frames][grid_h rs][grid_w rs]; loss = mean |PixelShuffle(F) - target| (one fp32)
+ * and dF = sign(F - target) / (pixel count) in F's layout. work: fp32 scratch of
+ * ceil(frames L channels rs^2 / 256) elements. */
+fd_status fd_op_l1_pixel_bwd(const float* F, const float* target, int frames, int grid_h,
+                             int grid_w, int channels, int rs, float* dF, float* loss,
+                             float* work, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

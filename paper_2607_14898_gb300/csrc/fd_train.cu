@@ -994,6 +994,46 @@ fd_status fd_train_step(fd_trainer tr, const float* latents, const float* target
   return r.ok ? FD_OK : FD_ERR_CUDA;
 }
 
+// ---- single kernels of the step, for per-kernel checks (include/flashdec_ops.h)
+fd_status fd_op_rmsnorm_bwd(const float* x, const float* g, const float* dy, int M, int D,
+                            float eps, float* dx, float* dg, float* work, void* stream) {
+  if (!x || !g || !dy || !dx || !dg || !work || M < 1 || D < 1 || D > 65536)
+    return FD_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  fd::train::rmsnorm_bwd_kernel<<<(M + 7) / 8, 256, 0, s>>>(x, g, dy, nullptr, M, D, eps, dx,
+                                                            work);
+  if (cudaGetLastError() != cudaSuccess) return FD_ERR_CUDA;
+  fd::train::colsum_kernel<<<(D + 127) / 128, 128, 0, s>>>(work, M, D, D, dg);
+  return cudaGetLastError() == cudaSuccess ? FD_OK : FD_ERR_CUDA;
+}
+
+fd_status fd_op_gelu_bwd(const float* z, const float* da, int64_t n, float* dz, void* dz_bf16,
+                         void* stream) {
+  if (!z || !da || !dz || !dz_bf16 || n < 1) return FD_ERR_INVALID_ARG;
+  fd::train::gelu_bwd_kernel<<<blocks_for(n, 256), 256, 0, static_cast<cudaStream_t>(stream)>>>(
+      z, da, n, dz, static_cast<bf16*>(dz_bf16));
+  return cudaGetLastError() == cudaSuccess ? FD_OK : FD_ERR_CUDA;
+}
+
+fd_status fd_op_l1_pixel_bwd(const float* F, const float* target, int frames, int grid_h,
+                             int grid_w, int channels, int rs, float* dF, float* loss,
+                             float* work, void* stream) {
+  if (!F || !target || !dF || !loss || !work || frames < 1 || grid_h < 1 || grid_w < 1 ||
+      channels < 1 || rs < 1)
+    return FD_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int L = grid_h * grid_w;
+  const long long n = static_cast<long long>(frames) * L * channels * rs * rs;
+  const int blocks = static_cast<int>((n + 255) / 256);
+  const float inv_total = static_cast<float>(1.0 / static_cast<double>(n));
+  // one chunk of `frames` refined frames, rows unpadded (Lp = L)
+  fd::train::l1_head_kernel<<<blocks, 256, 0, s>>>(F, target, 1, frames, L, L, grid_h, grid_w,
+                                                   channels, rs, inv_total, dF, work);
+  if (cudaGetLastError() != cudaSuccess) return FD_ERR_CUDA;
+  fd::train::finish_loss_kernel<<<1, 32, 0, s>>>(work, blocks, inv_total, loss);
+  return cudaGetLastError() == cudaSuccess ? FD_OK : FD_ERR_CUDA;
+}
+
 fd_status fd_train_status(fd_trainer tr, void* stream) {
   if (tr == nullptr) return FD_ERR_INVALID_ARG;
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return FD_ERR_CUDA;

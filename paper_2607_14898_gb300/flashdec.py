@@ -78,6 +78,9 @@ _SIGS = {
     "fd_debug_read_ring": (_I, [_P, _I, _I, _P, ctypes.c_size_t]),
     "fd_debug_wait_timeout": (_I, [_P, ctypes.c_uint, _P]),
     "fd_train_grad_elems": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
+    "fd_op_rmsnorm_bwd": (_I, [_P, _P, _P, _I, _I, _F, _P, _P, _P, _P]),
+    "fd_op_gelu_bwd": (_I, [_P, _P, ctypes.c_int64, _P, _P, _P]),
+    "fd_op_l1_pixel_bwd": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P]),
     "fd_train_create": (_I, [ctypes.POINTER(fd_config), _P, _I, ctypes.POINTER(_P)]),
     "fd_train_step": (_I, [_P, _P, _P, _P, _P, _P]),
     "fd_train_status": (_I, [_P, _P]),
@@ -531,3 +534,25 @@ def op_unshuffle(z, p, x0, stream=None) -> None:
 def op_pixel_head(F, frames, grid_h, grid_w, channels, rs, out_dtype, pixels, stream=None) -> None:
     _check(lib().fd_op_pixel_head(_ptr(F), frames, grid_h, grid_w, channels, rs, out_dtype,
                                   _ptr(pixels), _stream_ptr(stream)), "fd_op_pixel_head")
+
+
+def op_rmsnorm_bwd(x, g, dy, eps, dx, dg, stream=None) -> None:
+    M, D = x.shape
+    import torch
+    work = torch.empty(M, D, dtype=torch.float32, device=x.device)
+    _check(lib().fd_op_rmsnorm_bwd(_ptr(x), _ptr(g), _ptr(dy), M, D, eps, _ptr(dx), _ptr(dg),
+                                   _ptr(work), _stream_ptr(stream)), "fd_op_rmsnorm_bwd")
+
+
+def op_gelu_bwd(z, da, dz, dz_bf16, stream=None) -> None:
+    _check(lib().fd_op_gelu_bwd(_ptr(z), _ptr(da), z.numel(), _ptr(dz), _ptr(dz_bf16),
+                                _stream_ptr(stream)), "fd_op_gelu_bwd")
+
+
+def op_l1_pixel_bwd(F, target, frames, grid_h, grid_w, channels, rs, dF, loss,
+                    stream=None) -> None:
+    import torch
+    work = torch.empty((F.numel() + 255) // 256, dtype=torch.float32, device=F.device)
+    _check(lib().fd_op_l1_pixel_bwd(_ptr(F), _ptr(target), frames, grid_h, grid_w, channels, rs,
+                                    _ptr(dF), _ptr(loss), _ptr(work), _stream_ptr(stream)),
+           "fd_op_l1_pixel_bwd")
