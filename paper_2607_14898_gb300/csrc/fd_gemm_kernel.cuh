@@ -321,9 +321,6 @@ __global__ void __launch_bounds__(192, 1)
     const uint32_t bar_tempty0 = PAIR ? mapa_rank(bar_tempty, 0) : bar_tempty;
     for (int tile = cta0; tile < tiles; tile += ctas, ++tc) {
       const int acc = tc & 1;
-      const bool got = mbar_wait(bar_tfull + 8 * acc, (tc >> 1) & 1, p.err, ERR_WAIT_MMA);
-      if (!__all_sync(0xffffffffu, got)) break;  // leave together: TMEM loads are collective
-      tc_fence_after();
       const int m0 = (tile / n_tiles) * tile_rows + static_cast<int>(rank) * kBM;
       const int n0 = (tile % n_tiles) * BN;
       const int row0 = m0 + quarter * 32;  // first row of this warp's slab
@@ -331,6 +328,20 @@ __global__ void __launch_bounds__(192, 1)
       const bool row_ok = row < p.M;
       const uint32_t tbase =
           tmem + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      // The tile's bias (and column-scale) lines go into L1 while its MMAs still run, so the
+      // per-chunk loads below do not each wait a round trip to L2 after the accumulator is ready.
+      if (lane < BN / 32 && n0 + 32 * lane < p.N) {
+        prefetch_l1(p.bias + n0 + 32 * lane);
+        if (p.col_scale != nullptr) prefetch_l1(p.col_scale + n0 + 32 * lane);
+      }
+      // wait for the tile's accumulator; all lanes leave together (TMEM loads are collective)
+      auto acc_ready = [&]() -> bool {
+        const bool got = mbar_wait(bar_tfull + 8 * acc, (tc >> 1) & 1, p.err, ERR_WAIT_MMA);
+        if (!__all_sync(0xffffffffu, got)) return false;
+        tc_fence_after();
+        return true;
+      };
+      if (!QKV && !acc_ready()) break;
 
       if (QKV) {
         const QkvEpi& q = p.qkv;
@@ -362,6 +373,13 @@ __global__ void __launch_bounds__(192, 1)
           rope_table(q, q.rope_t, row / q.tokens, l / q.grid_w, l % q.grid_w, rc, rsn);
           ring_row = slot * rows_chunk + row;
         }
+        if (lane < 2) {  // the per-head norm gains (64 floats each)
+          if (q.knorm_g != nullptr) prefetch_l1(q.knorm_g + 32 * lane);
+          if (q.vnorm_g != nullptr) prefetch_l1(q.vnorm_g + 32 * lane);
+        }
+        // the rotation and ring position above depend only on the row: computed while the
+        // MMAs of the tile still run
+        if (!acc_ready()) break;
 #pragma unroll 1
         for (int c = 0; c < BN; c += 64) {
           const int col = n0 + c;
