@@ -319,6 +319,28 @@ fd_status fd_train_step(fd_trainer tr, const float* latents, const float* target
 fd_status fd_train_status(fd_trainer tr, void* stream);
 fd_status fd_train_destroy(fd_trainer tr);
 
+/* Kernel kinds of the training step, for its per-kernel profile. */
+enum fd_train_kind {
+  FD_TK_LINEAR = 0,     /* forward products of the linears (embedding, blocks, upsampling, head) */
+  FD_TK_DGRAD = 1,      /* their input gradients, dX = dY W */
+  FD_TK_WGRAD = 2,      /* their weight gradients, dW = dY^T X */
+  FD_TK_ATTN_GEMM = 3,  /* the attention's products: S = Q K^T (forward and recomputed), P V,
+                           dP = dO V^T, dQ = dS K, dK = dS^T Q, dV = P^T dO */
+  FD_TK_SOFTMAX = 4,    /* band softmax, row dot delta = rowsum(dO o O), softmax backward */
+  FD_TK_TRANSPOSE = 5,  /* operand transposes for the products */
+  FD_TK_NORM = 6,       /* RMSNorm forward / backward, KV-norm (QK-norm) + 3D-RoPE fwd / bwd */
+  FD_TK_POINTWISE = 7,  /* bf16 casts, GELU forward / backward, copies, column sums, the
+                           PixelUnshuffle, upsampling permutes and the L1 loss */
+  FD_TK_COUNT = 8
+};
+/* Per-kernel profile of the training step: while enabled, every launch of fd_train_step is
+ * bracketed by CUDA events on its stream. fd_train_profile_collect synchronises the device,
+ * adds each kind's launch count and device milliseconds into launches[FD_TK_COUNT] /
+ * ms[FD_TK_COUNT] (the caller zeroes them) and releases the recorded events.
+ * Errors: FD_ERR_INVALID_ARG (null arguments), FD_ERR_CUDA. */
+fd_status fd_train_profile_enable(fd_trainer tr, int enable);
+fd_status fd_train_profile_collect(fd_trainer tr, int64_t* launches, double* ms);
+
 /* Copy layer `layer` of the backbone (which = 0) or refinement (which = 1) ring into host
  * memory: K as [G][W * rows][64] bf16 bits, then V as [G][W * rows][64] fp16 bits (rows =
  * L backbone, r_t L refinement; row slot*rows + r holds token r of the chunk in ring slot

@@ -64,3 +64,18 @@ def training_step_flops(cfg, chunks: int) -> dict[str, int]:
     fwd = stream_flops(cfg, chunks)
     emb = sum(chunk_flops(cfg, t)["embed"] for t in range(chunks))
     return {"forward": fwd, "backward": 2 * fwd - emb}
+
+
+def training_kind_flops(cfg, chunks: int) -> dict[str, int]:
+    """training_step_flops split by the kernel kinds of the GPU step (enum fd_train_kind): the
+    linears' forward products, their input gradients (none for the patch-embedding), their weight
+    gradients, and the attention's products (S and P V forward, dP, dQ, dK, dV backward: three
+    times the forward's; the step's recomputation of S is not counted)."""
+    lin = emb = att = 0
+    for t in range(chunks):
+        f = chunk_flops(cfg, t)
+        a = f["attn_backbone"] + f["attn_refine"]
+        att += a
+        lin += sum(f.values()) - a
+        emb += f["embed"]
+    return {"linear": lin, "dgrad": lin - emb, "wgrad": lin, "attn_gemm": 3 * att}

@@ -134,6 +134,28 @@ __global__ void colsum_kernel(const float* __restrict__ x, long long rows, int c
   out[c] = s;
 }
 
+// The same sums in two stages, for many rows: part[k][c] = the sum of rows k R .. k R + R - 1
+// (in order), then out[c] = the sum of the parts in order. A fixed order, so repeatable bits.
+constexpr int kColsumRows = 256;
+__global__ void colsum_part_kernel(const float* __restrict__ x, long long rows, int cols, int ld,
+                                   float* __restrict__ part) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= cols) return;
+  const long long r0 = static_cast<long long>(blockIdx.y) * kColsumRows;
+  const long long r1 = r0 + kColsumRows < rows ? r0 + kColsumRows : rows;
+  float s = 0.f;
+  for (long long r = r0; r < r1; ++r) s += x[r * ld + c];
+  part[static_cast<size_t>(blockIdx.y) * cols + c] = s;
+}
+__global__ void colsum_finish_kernel(const float* __restrict__ part, int parts, int cols,
+                                     float* __restrict__ out) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= cols) return;
+  float s = 0.f;
+  for (int k = 0; k < parts; ++k) s += part[static_cast<size_t>(k) * cols + c];
+  out[c] = s;
+}
+
 // RoPE tables (host-computed in double): temporal (cos, sin) [frames][kBandT], row and column
 // [grid][kBandS]
 struct Rope {
@@ -159,9 +181,10 @@ __device__ __forceinline__ void head_rms(float (&v)[kDh], const float* g, float 
 
 // QKV forward of every row: slot < N query heads, then G key groups, then G value groups.
 // q2 = RoPE(q0) (RMS with g2 first when qk_norm), k2 = RoPE(RMS(k0; gk)), v1 = RMS(v0; g2)
-// (v0 when qk_norm). Outputs: q2 bf16 [M][N 64], k2 / v1 bf16 [G][M][64].
-__global__ void qkv_fwd_kernel(const float* __restrict__ qkv, int M, int Lp, int L, int gw, int N,
-                               int G, int qk_norm, const float* __restrict__ gk,
+// (v0 when qk_norm). Outputs: q2 bf16 head-major per chunk of Pc rows, [M / Pc][N][Pc][64]
+// (the rows of one chunk's heads of a KV group are then contiguous), k2 / v1 bf16 [G][M][64].
+__global__ void qkv_fwd_kernel(const float* __restrict__ qkv, int M, int Pc, int Lp, int L,
+                               int gw, int N, int G, int qk_norm, const float* __restrict__ gk,
                                const float* __restrict__ g2, float eps, Rope rp,
                                bf16* __restrict__ q2, bf16* __restrict__ k2,
                                bf16* __restrict__ v1) {
@@ -179,7 +202,7 @@ __global__ void qkv_fwd_kernel(const float* __restrict__ qkv, int M, int Lp, int
   if (is_k) head_rms(v, gk, eps);
   else if (is_q ? qk_norm != 0 : qk_norm == 0) head_rms(v, g2, eps);
   bf16* dst;
-  if (is_q) dst = q2 + static_cast<size_t>(row) * N * kDh + slot * kDh;
+  if (is_q) dst = q2 + (static_cast<size_t>(row / Pc * N + slot) * Pc + row % Pc) * kDh;
   else if (is_k) dst = k2 + (static_cast<size_t>(slot - N) * M + row) * kDh;
   else dst = v1 + (static_cast<size_t>(slot - N - G) * M + row) * kDh;
   if (is_q || is_k) {
@@ -214,12 +237,13 @@ __device__ __forceinline__ void head_rms_bwd(const float (&x)[kDh], float (&dy)[
   }
 }
 
-// QKV backward of every row: dq2 fp32 [M][N 64], dk2 / dv1 fp32 [G][M][64] -> dqkv fp32
+// QKV backward of every row: dq2 fp32 [M / Pc][N][Pc][64] (the layout of q2), dk2 / dv1 fp32
+// [G][M][64] -> dqkv fp32
 // [M][(N + 2G) 64] (inverse RoPE: the rotation by the negated angle; then the per-head RMS
 // backward where the forward normalised); gain terms tq [M N][64] (qk_norm), tk / tv [M G][64]
 __global__ void qkv_bwd_kernel(const float* __restrict__ qkv, const float* __restrict__ dq2,
                                const float* __restrict__ dk2, const float* __restrict__ dv1,
-                               int M, int Lp, int L, int gw, int N, int G, int qk_norm,
+                               int M, int Pc, int Lp, int L, int gw, int N, int G, int qk_norm,
                                const float* __restrict__ gk, const float* __restrict__ g2,
                                float eps, Rope rp, float* __restrict__ dqkv,
                                float* __restrict__ tq, float* __restrict__ tk,
@@ -233,7 +257,7 @@ __global__ void qkv_bwd_kernel(const float* __restrict__ qkv, const float* __res
   const bool is_q = slot < N, is_k = !is_q && slot < N + G;
   float d[kDh], x[kDh];
   const float* src;
-  if (is_q) src = dq2 + static_cast<size_t>(row) * N * kDh + slot * kDh;
+  if (is_q) src = dq2 + (static_cast<size_t>(row / Pc * N + slot) * Pc + row % Pc) * kDh;
   else if (is_k) src = dk2 + (static_cast<size_t>(slot - N) * M + row) * kDh;
   else src = dv1 + (static_cast<size_t>(slot - N - G) * M + row) * kDh;
 #pragma unroll
@@ -262,54 +286,105 @@ __global__ void qkv_bwd_kernel(const float* __restrict__ qkv, const float* __res
   for (int j = 0; j < kDh; ++j) dst[j] = d[j];
 }
 
-// Band softmax of one (query chunk, head): S fp32 [rows][n] (row pitch n); column c is a key
-// of a token (c mod Lp < L); P = softmax(S scale) over the valid columns, 0 elsewhere, as fp32
-// and bf16. One warp per row.
-__global__ void softmax_band_kernel(const float* __restrict__ S, int rows, int n, float scale,
-                                    int Lp, int L, float* __restrict__ P32,
-                                    bf16* __restrict__ P16) {
+// Band softmax of one (query chunk, KV group): S fp32 [rows][n] (row pitch n), rows = the
+// group's heads x the chunk's rows; column c is a key of a token (c mod Lp < L). P = softmax(S
+// scale) over the valid columns (0 elsewhere) as bf16, and lse = log sum exp(S scale) of each
+// row (natural log) for the backward. One warp per row: an online max / sum pass, then the
+// write pass.
+__global__ void softmax_lse_kernel(const float* __restrict__ S, int rows, int n, float scale,
+                                   int Lp, int L, bf16* __restrict__ P16,
+                                   float* __restrict__ lse) {
   const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
   const float* s = S + static_cast<size_t>(row) * n;
-  float m = -INFINITY;
-  for (int c = lane; c < n; c += 32)
-    if (c % Lp < L) m = fmaxf(m, s[c] * scale);
-  m = warp_max(m);
-  float sum = 0.f;
-  for (int c = lane; c < n; c += 32)
-    if (c % Lp < L) sum += expf(s[c] * scale - m);
-  sum = warp_sum(sum);
-  const float inv = 1.0f / sum;
+  float m = -INFINITY, sum = 0.f;
   for (int c = lane; c < n; c += 32) {
-    const float p = c % Lp < L ? expf(s[c] * scale - m) * inv : 0.f;
-    P32[static_cast<size_t>(row) * n + c] = p;
+    if (c % Lp >= L) continue;
+    const float v = s[c] * scale;
+    if (v > m) {
+      sum = sum * expf(m - v) + 1.0f;
+      m = v;
+    } else {
+      sum += expf(v - m);
+    }
+  }
+  const float mw = warp_max(m);
+  sum = warp_sum(m == -INFINITY ? 0.f : sum * expf(m - mw));
+  const float l = mw + logf(sum);
+  for (int c = lane; c < n; c += 32) {
+    const float p = c % Lp < L ? expf(s[c] * scale - l) : 0.f;
     P16[static_cast<size_t>(row) * n + c] = __float2bfloat16_rn(p);
+  }
+  if (lane == 0) lse[row] = l;
+}
+
+// delta[(c N + h) Pc + l] = sum_j dO[c Pc + l][h 64 + j] O[((c N + h) Pc + l) 64 + j]: dO fp32
+// rows [M][N 64], O fp32 head-major [M / Pc][N][Pc][64]; one warp per (chunk, head, row)
+__global__ void delta_kernel(const float* __restrict__ dO, const float* __restrict__ O, int M,
+                             int Pc, int N, float* __restrict__ delta) {
+  const long long w = (blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (w >= static_cast<long long>(M) * N) return;
+  const int c = static_cast<int>(w / (static_cast<long long>(N) * Pc));
+  const int h = static_cast<int>(w / Pc % N), l = static_cast<int>(w % Pc);
+  const float* a = dO + (static_cast<size_t>(c) * Pc + l) * N * kDh + h * kDh;
+  const float* b = O + static_cast<size_t>(w) * kDh;
+  float v = a[lane] * b[lane] + a[lane + 32] * b[lane + 32];
+  v = warp_sum(v);
+  if (lane == 0) delta[w] = v;
+}
+
+// Softmax backward of one (query chunk, KV group), one 32 x 32 tile per block: with P = exp(S
+// scale - lse) on the valid columns, dS = P (dP - delta) scale (the scale of the scores folded
+// in: dQ = dS K, dK = dS^T Q). Writes dS [rows][n] and, through the tile, dS^T and P^T
+// [n][rows] (bf16) for the key-side products.
+__global__ void attn_grad_kernel(const float* __restrict__ S, const float* __restrict__ dP,
+                                 const float* __restrict__ lse, const float* __restrict__ delta,
+                                 int rows, int n, float scale, int Lp, int L,
+                                 bf16* __restrict__ dS, bf16* __restrict__ dST,
+                                 bf16* __restrict__ PT) {
+  __shared__ bf16 tp[32][34], td[32][34];
+  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  const int c = c0 + threadIdx.x;
+  const bool valid = c < n && c % Lp < L;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = r0 + i;
+    bf16 p16 = __float2bfloat16_rn(0.f), d16 = p16;
+    if (r < rows && c < n) {
+      const size_t e = static_cast<size_t>(r) * n + c;
+      const float p = valid ? expf(S[e] * scale - lse[r]) : 0.f;
+      d16 = __float2bfloat16_rn(p * (dP[e] - delta[r]) * scale);
+      p16 = __float2bfloat16_rn(p);
+      dS[e] = d16;
+    }
+    tp[i][threadIdx.x] = p16;
+    td[i][threadIdx.x] = d16;
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int cc = c0 + i, r = r0 + threadIdx.x;
+    if (cc < n && r < rows) {
+      const size_t e = static_cast<size_t>(cc) * rows + r;
+      PT[e] = tp[threadIdx.x][i];
+      dST[e] = td[threadIdx.x][i];
+    }
   }
 }
 
-// delta[r] = sum_j dO[r][j] O[r][j] over the 64 values of one head (pitches in elements)
-__global__ void rowdot_kernel(const float* __restrict__ a, int lda, const float* __restrict__ b,
-                              int ldb, int rows, float* __restrict__ out) {
-  const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (row >= rows) return;
-  float s = a[static_cast<size_t>(row) * lda + lane] * b[static_cast<size_t>(row) * ldb + lane] +
-            a[static_cast<size_t>(row) * lda + lane + 32] *
-                b[static_cast<size_t>(row) * ldb + lane + 32];
-  s = warp_sum(s);
-  if (lane == 0) out[row] = s;
-}
-
-// dS = P (dP - delta) scale (the scale of the scores folded in: dQ = dS K, dK = dS^T Q)
-__global__ void dsoftmax_kernel(const float* __restrict__ P, const float* __restrict__ dP,
-                                const float* __restrict__ delta, int rows, int n, float scale,
-                                bf16* __restrict__ dS) {
-  const long long total = static_cast<long long>(rows) * n;
+// head-major [M / Pc][N][Pc][64] fp32 <-> rows [M][N 64]: to_rows = 1 reads head-major x and
+// writes bf16 rows; to_rows = 0 reads fp32 rows and writes bf16 head-major
+__global__ void head_permute_kernel(const float* __restrict__ x, int M, int Pc, int N,
+                                    int to_rows, bf16* __restrict__ y) {
+  const long long total = static_cast<long long>(M) * N * kDh;
   for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<long long>(gridDim.x) * blockDim.x) {
-    const int r = static_cast<int>(i / n);
-    dS[i] = __float2bfloat16_rn(P[i] * (dP[i] - delta[r]) * scale);
+    // i indexes the rows layout: row m, head h, element j
+    const long long m = i / (static_cast<long long>(N) * kDh);
+    const int h = static_cast<int>(i / kDh % N), j = static_cast<int>(i % kDh);
+    const long long hm = ((m / Pc * N + h) * Pc + m % Pc) * kDh + j;
+    if (to_rows) y[i] = __float2bfloat16_rn(x[hm]);
+    else y[hm] = __float2bfloat16_rn(x[i]);
   }
 }
 
@@ -417,14 +492,36 @@ struct fd_trainer_s {
     int M, Pc;  // rows, rows per chunk
     std::vector<float*> h;  // block inputs (h[nblocks] = stack output), fp32 [M][D]
     std::vector<bf16*> u, q2, k2, v1, o, u2, a;
-    std::vector<float*> qkv, o32, hm, z;
+    std::vector<float*> qkv, o32, hm, z, lse;  // o32 head-major, lse [M / Pc][N][Pc]
   } sB, sR;
   // scratch
   bf16 *x0, *y16, *yh16, *a1, *vT, *kT, *do16, *dS, *P16, *dST, *PT, *QT, *dOT, *dy16, *dyT,
       *xT, *dqkv16;
-  float *e, *z1, *F, *dF, *loss_part, *S, *P32, *dP, *delta, *dq2, *dk2, *dv1, *dqkv, *tq, *tk,
+  float *e, *z1, *F, *dF, *loss_part, *S, *dP, *delta, *dq2, *dk2, *dv1, *dqkv, *tq, *tk,
       *tv, *gA, *gB, *gC, *tbuf, *gtmp;
   int loss_blocks = 0;
+  int hs = 1;  // heads of one KV group per attention product (a divisor of N / G)
+  float* colsum_part = nullptr;  // partial column sums
+  size_t colsum_elems = 0;
+  // per-kernel profile (fd_train_profile_enable): events around each launch, by kernel kind
+  struct Rec {
+    int kind;
+    cudaEvent_t a, b;
+  };
+  bool prof = false;
+  std::vector<cudaEvent_t> ev_free, ev_all;
+  std::vector<Rec> rec;
+  cudaEvent_t event() {
+    if (!ev_free.empty()) {
+      cudaEvent_t e = ev_free.back();
+      ev_free.pop_back();
+      return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    ev_all.push_back(e);
+    return e;
+  }
 };
 
 namespace {
@@ -461,44 +558,93 @@ struct Run {
   fd_trainer_s* tr;
   cudaStream_t s;
   bool ok = true;
+  cudaEvent_t t0 = nullptr;  // start event of the launch being profiled
+  int t_kind = 0;
 
   void check(cudaError_t e) {
     if (e != cudaSuccess) ok = false;
   }
-  void gemm(int epi, int M, int N, int K, const bf16* A, int lda, const bf16* Wm, int ldw,
-            const float* bias, float* out, int ldo) {
-    if (!ok) return;
+  // bracket the next launch with profile events (when the profile is enabled)
+  bool begin(int kind) {
+    if (!ok) return false;
+    if (tr->prof) {
+      t0 = tr->event();
+      t_kind = kind;
+      if (t0 != nullptr) check(cudaEventRecord(t0, s));
+    }
+    return ok;
+  }
+  void end() {
+    if (t0 == nullptr) return;
+    cudaEvent_t t1 = tr->event();
+    if (t1 != nullptr) {
+      check(cudaEventRecord(t1, s));
+      tr->rec.push_back({t_kind, t0, t1});
+    } else {
+      tr->ev_free.push_back(t0);
+    }
+    t0 = nullptr;
+  }
+  void gemm(int kind, int epi, int M, int N, int K, const bf16* A, int lda, const bf16* Wm,
+            int ldw, const float* bias, float* out, int ldo) {
+    if (!begin(kind)) return;
     check(fd::gemm_view(epi, M, N, K, A, lda, Wm, ldw, bias ? bias : tr->zero_bias, out, ldo,
                         tr->err, s));
+    end();
   }
   void bf(const float* x, long long n, bf16* y) {
-    if (!ok) return;
+    if (!begin(FD_TK_POINTWISE)) return;
     fd::train::to_bf16_kernel<<<blocks_for(n, 256), 256, 0, s>>>(x, n, y);
     check(cudaGetLastError());
+    end();
   }
   template <typename T>
   void transpose(const T* x, int rows, int cols, int ldx, T* y, int ldy) {
-    if (!ok) return;
+    if (!begin(FD_TK_TRANSPOSE)) return;
     dim3 grid((cols + 31) / 32, (rows + 31) / 32);
     fd::train::transpose_kernel<T><<<grid, dim3(32, 8), 0, s>>>(x, rows, cols, ldx, y, ldy);
     check(cudaGetLastError());
+    end();
   }
   void colsum(const float* x, long long rows, int cols, int ld, float* out) {
-    if (!ok) return;
-    fd::train::colsum_kernel<<<(cols + 127) / 128, 128, 0, s>>>(x, rows, cols, ld, out);
+    const int parts = static_cast<int>((rows + fd::train::kColsumRows - 1) /
+                                       fd::train::kColsumRows);
+    if (static_cast<size_t>(parts) * cols > tr->colsum_elems) {
+      ok = false;
+      return;
+    }
+    if (!begin(FD_TK_POINTWISE)) return;
+    fd::train::colsum_part_kernel<<<dim3((cols + 127) / 128, parts), 128, 0, s>>>(
+        x, rows, cols, ld, tr->colsum_part);
     check(cudaGetLastError());
+    fd::train::colsum_finish_kernel<<<(cols + 127) / 128, 128, 0, s>>>(tr->colsum_part, parts,
+                                                                      cols, out);
+    check(cudaGetLastError());
+    end();
+  }
+  void copy(float* dst, const float* src, size_t n) {
+    if (!begin(FD_TK_POINTWISE)) return;
+    check(cudaMemcpyAsync(dst, src, sizeof(float) * n, cudaMemcpyDeviceToDevice, s));
+    end();
+  }
+  void zero(float* dst, size_t n) {
+    if (!begin(FD_TK_POINTWISE)) return;
+    check(cudaMemsetAsync(dst, 0, sizeof(float) * n, s));
+    end();
   }
   void rmsnorm(const float* x, const float* g, int M, bf16* u) {
-    if (!ok) return;
+    if (!begin(FD_TK_NORM)) return;
     check(fd::launch_rmsnorm(x, g, M, tr->D, tr->eps, u, s));
+    end();
   }
   // dx = RMSNorm backward (+ add), the gain's gradient into grad
   void rmsnorm_bwd(const float* x, const float* g, const float* dy, const float* add, int M,
                    float* dx, float* grad) {
-    if (!ok) return;
+    if (!begin(FD_TK_NORM)) return;
     fd::train::rmsnorm_bwd_kernel<<<(M + 7) / 8, 256, 0, s>>>(x, g, dy, add, M, tr->D, tr->eps,
                                                              dx, tr->tbuf);
     check(cudaGetLastError());
+    end();
     colsum(tr->tbuf, M, tr->D, tr->D, grad);
   }
   // weight gradient of a linear out = X W^T: dW [n_out][n_in] = dY^T X with dY16 [M][n_out]
@@ -509,9 +655,9 @@ struct Run {
     transpose(dY16, M, n_out, n_out, dyT, M);
     transpose(X16, M, n_in, n_in, xT, M);
     if (n_in % 32 == 0) {
-      gemm(fd::EPI_F32, n_out, n_in, M, dyT, M, xT, M, nullptr, dW, n_in);
+      gemm(FD_TK_WGRAD, fd::EPI_F32, n_out, n_in, M, dyT, M, xT, M, nullptr, dW, n_in);
     } else {  // the product in the other orientation (its N = n_out), then transposed
-      gemm(fd::EPI_F32, n_in, n_out, M, xT, M, dyT, M, nullptr, tr->gtmp, n_out);
+      gemm(FD_TK_WGRAD, fd::EPI_F32, n_in, n_out, M, xT, M, dyT, M, nullptr, tr->gtmp, n_out);
       transpose(tr->gtmp, n_in, n_out, n_out, dW, n_in);
     }
   }
@@ -524,10 +670,14 @@ struct Run {
 // (vnorm|qnorm).g, out.w, out.b, norm2.g, mlp1.w, mlp1.b, mlp2.w, mlp2.b
 enum { kN1 = 0, kQW, kQB, kKG, kG2, kOW, kOB, kN2, kM1W, kM1B, kM2W, kM2B, kBlockEntries };
 
-// attention forward of every (query chunk, head) of one block: S, band softmax, O = P V
+// attention forward of one block (Sec. 3.3, Eq. attention over the chunk window), per (query
+// chunk i, KV group g): the rows of the group's heads form one product with the window's keys
+// (chunks max(0, i - W + 1) .. i, contiguous in k2 / v1): S = Q K^T, band softmax (P bf16 and
+// each row's log-sum-exp), O = P V, O head-major fp32 in st.o32. A group's heads go tr->hs at a
+// time (all of them unless S would pass its size bound).
 void attn_fwd(Run& r, fd_trainer_s::Stack& st, int b) {
   fd_trainer_s* tr = r.tr;
-  const int M = st.M, Pc = st.Pc, hpg = tr->N / tr->G;
+  const int M = st.M, Pc = st.Pc, N = tr->N, hpg = N / tr->G, rows = tr->hs * Pc;
   // V^T [G][64][M] for the P V products
   for (int g = 0; g < tr->G; ++g)
     r.transpose(st.v1[b] + static_cast<size_t>(g) * M * 64, M, 64, 64,
@@ -535,69 +685,79 @@ void attn_fwd(Run& r, fd_trainer_s::Stack& st, int b) {
   for (int i = 0; i < tr->T; ++i) {
     const int j0 = i - tr->Wn + 1 > 0 ? i - tr->Wn + 1 : 0;
     const int k0 = j0 * Pc, nk = (i + 1) * Pc - k0;
-    for (int h = 0; h < tr->N; ++h) {
-      const int g = h / hpg;
-      r.gemm(fd::EPI_F32, Pc, nk, 64, st.q2[b] + static_cast<size_t>(i) * Pc * tr->NQ + h * 64,
-             tr->NQ, st.k2[b] + (static_cast<size_t>(g) * M + k0) * 64, 64, nullptr, tr->S, nk);
-      if (r.ok) {
-        fd::train::softmax_band_kernel<<<(Pc + 7) / 8, 256, 0, r.s>>>(
-            tr->S, Pc, nk, 0.125f, tr->Lp, tr->L, tr->P32, tr->P16);
+    for (int h0 = 0; h0 < N; h0 += tr->hs) {  // tr->hs heads of group h0 / hpg at a time
+      const int g = h0 / hpg;
+      const size_t q0 = (static_cast<size_t>(i) * N + h0) * Pc;  // first row, head-major
+      r.gemm(FD_TK_ATTN_GEMM, fd::EPI_F32, rows, nk, 64, st.q2[b] + q0 * 64, 64,
+             st.k2[b] + (static_cast<size_t>(g) * M + k0) * 64, 64, nullptr, tr->S, nk);
+      if (r.begin(FD_TK_SOFTMAX)) {
+        fd::train::softmax_lse_kernel<<<(rows + 7) / 8, 256, 0, r.s>>>(
+            tr->S, rows, nk, 0.125f, tr->Lp, tr->L, tr->P16, st.lse[b] + q0);
         r.check(cudaGetLastError());
+        r.end();
       }
-      r.gemm(fd::EPI_F32, Pc, 64, nk, tr->P16, nk, tr->vT + static_cast<size_t>(g) * 64 * M + k0,
-             M, nullptr, st.o32[b] + static_cast<size_t>(i) * Pc * tr->NQ + h * 64, tr->NQ);
+      r.gemm(FD_TK_ATTN_GEMM, fd::EPI_F32, rows, 64, nk, tr->P16, nk,
+             tr->vT + static_cast<size_t>(g) * 64 * M + k0, M, nullptr, st.o32[b] + q0 * 64, 64);
     }
   }
 }
 
-// attention backward: dq2 (fp32 [M][N 64]), dk2, dv1 (fp32 [G][M][64], accumulated over the
-// heads and query chunks that read each key) from do32 / do16
+// attention backward of one block: dq2 (fp32, the head-major layout of q2), dk2, dv1 (fp32
+// [G][M][64], accumulated over the query chunks whose windows hold each key; the group's heads
+// sum inside each product) from dO (tr->gA, fp32 rows [M][N 64])
 void attn_bwd(Run& r, fd_trainer_s::Stack& st, int b) {
   fd_trainer_s* tr = r.tr;
-  const int M = st.M, Pc = st.Pc, hpg = tr->N / tr->G;
-  if (r.ok) r.check(cudaMemsetAsync(tr->dk2, 0, sizeof(float) * tr->G * M * 64, r.s));
-  if (r.ok) r.check(cudaMemsetAsync(tr->dv1, 0, sizeof(float) * tr->G * M * 64, r.s));
+  const int M = st.M, Pc = st.Pc, N = tr->N, hpg = N / tr->G, rows = tr->hs * Pc;
+  r.zero(tr->dk2, static_cast<size_t>(tr->G) * M * 64);
+  r.zero(tr->dv1, static_cast<size_t>(tr->G) * M * 64);
   for (int g = 0; g < tr->G; ++g)
     r.transpose(st.k2[b] + static_cast<size_t>(g) * M * 64, M, 64, 64,
                 tr->kT + static_cast<size_t>(g) * 64 * M, M);
+  // dO head-major (bf16) and delta = rowsum(dO o O) of every (chunk, head, row)
+  if (r.begin(FD_TK_POINTWISE)) {
+    const long long n = static_cast<long long>(M) * tr->NQ;
+    fd::train::head_permute_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(tr->gA, M, Pc, N, 0,
+                                                                         tr->do16);
+    r.check(cudaGetLastError());
+    r.end();
+  }
+  if (r.begin(FD_TK_SOFTMAX)) {
+    const long long n = static_cast<long long>(M) * N * 32;
+    fd::train::delta_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(tr->gA, st.o32[b], M, Pc, N,
+                                                                  tr->delta);
+    r.check(cudaGetLastError());
+    r.end();
+  }
   for (int i = 0; i < tr->T; ++i) {
     const int j0 = i - tr->Wn + 1 > 0 ? i - tr->Wn + 1 : 0;
     const int k0 = j0 * Pc, nk = (i + 1) * Pc - k0;
-    for (int h = 0; h < tr->N; ++h) {
-      const int g = h / hpg;
-      const size_t qoff = static_cast<size_t>(i) * Pc * tr->NQ + h * 64;
+    for (int h0 = 0; h0 < N; h0 += tr->hs) {
+      const int g = h0 / hpg;
+      const size_t q0 = (static_cast<size_t>(i) * N + h0) * Pc;
       const bf16* Kw = st.k2[b] + (static_cast<size_t>(g) * M + k0) * 64;
       const bf16* Vw = st.v1[b] + (static_cast<size_t>(g) * M + k0) * 64;
-      // P recomputed
-      r.gemm(fd::EPI_F32, Pc, nk, 64, st.q2[b] + qoff, tr->NQ, Kw, 64, nullptr, tr->S, nk);
-      if (r.ok) {
-        fd::train::softmax_band_kernel<<<(Pc + 7) / 8, 256, 0, r.s>>>(
-            tr->S, Pc, nk, 0.125f, tr->Lp, tr->L, tr->P32, tr->P16);
+      // S recomputed, dP = dO V^T
+      r.gemm(FD_TK_ATTN_GEMM, fd::EPI_F32, rows, nk, 64, st.q2[b] + q0 * 64, 64, Kw, 64,
+             nullptr, tr->S, nk);
+      r.gemm(FD_TK_ATTN_GEMM, fd::EPI_F32, rows, nk, 64, tr->do16 + q0 * 64, 64, Vw, 64,
+             nullptr, tr->dP, nk);
+      if (r.begin(FD_TK_SOFTMAX)) {
+        const dim3 grid((nk + 31) / 32, (rows + 31) / 32);
+        fd::train::attn_grad_kernel<<<grid, dim3(32, 8), 0, r.s>>>(
+            tr->S, tr->dP, st.lse[b] + q0, tr->delta + q0, rows, nk, 0.125f, tr->Lp, tr->L,
+            tr->dS, tr->dST, tr->PT);
         r.check(cudaGetLastError());
-      }
-      // dP = dO V^T
-      r.gemm(fd::EPI_F32, Pc, nk, 64, tr->do16 + qoff, tr->NQ, Vw, 64, nullptr, tr->dP, nk);
-      if (r.ok) {
-        fd::train::rowdot_kernel<<<(Pc + 7) / 8, 256, 0, r.s>>>(
-            tr->gA + qoff, tr->NQ, st.o32[b] + qoff, tr->NQ, Pc, tr->delta);
-        r.check(cudaGetLastError());
-        const long long n = static_cast<long long>(Pc) * nk;
-        fd::train::dsoftmax_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(
-            tr->P32, tr->dP, tr->delta, Pc, nk, 0.125f, tr->dS);
-        r.check(cudaGetLastError());
+        r.end();
       }
       // dQ = dS K
-      r.gemm(fd::EPI_F32, Pc, 64, nk, tr->dS, nk, tr->kT + static_cast<size_t>(g) * 64 * M + k0,
-             M, nullptr, tr->dq2 + qoff, tr->NQ);
-      // dK += dS^T Q
-      r.transpose(tr->dS, Pc, nk, nk, tr->dST, Pc);
-      r.transpose(st.q2[b] + qoff, Pc, 64, tr->NQ, tr->QT, Pc);
-      r.gemm(fd::EPI_RESID, nk, 64, Pc, tr->dST, Pc, tr->QT, Pc, nullptr,
+      r.gemm(FD_TK_ATTN_GEMM, fd::EPI_F32, rows, 64, nk, tr->dS, nk,
+             tr->kT + static_cast<size_t>(g) * 64 * M + k0, M, nullptr, tr->dq2 + q0 * 64, 64);
+      // dK += dS^T Q, dV += P^T dO (K of both products: the group's rows)
+      r.transpose(st.q2[b] + q0 * 64, rows, 64, 64, tr->QT, rows);
+      r.gemm(FD_TK_ATTN_GEMM, fd::EPI_RESID, nk, 64, rows, tr->dST, rows, tr->QT, rows, nullptr,
              tr->dk2 + (static_cast<size_t>(g) * M + k0) * 64, 64);
-      // dV += P^T dO
-      r.transpose(tr->P16, Pc, nk, nk, tr->PT, Pc);
-      r.transpose(tr->do16 + qoff, Pc, 64, tr->NQ, tr->dOT, Pc);
-      r.gemm(fd::EPI_RESID, nk, 64, Pc, tr->PT, Pc, tr->dOT, Pc, nullptr,
+      r.transpose(tr->do16 + q0 * 64, rows, 64, 64, tr->dOT, rows);
+      r.gemm(FD_TK_ATTN_GEMM, fd::EPI_RESID, nk, 64, rows, tr->PT, rows, tr->dOT, rows, nullptr,
              tr->dv1 + (static_cast<size_t>(g) * M + k0) * 64, 64);
     }
   }
@@ -608,35 +768,39 @@ void block_fwd(Run& r, fd_trainer_s::Stack& st, int b, size_t e0) {
   fd_trainer_s* tr = r.tr;
   const int M = st.M;
   r.rmsnorm(st.h[b], r.wf(e0 + kN1), M, st.u[b]);
-  r.gemm(fd::EPI_F32, M, tr->QO, tr->D, st.u[b], tr->D, r.wb(e0 + kQW), tr->D, r.wf(e0 + kQB),
+  r.gemm(FD_TK_LINEAR, fd::EPI_F32, M, tr->QO, tr->D, st.u[b], tr->D, r.wb(e0 + kQW), tr->D, r.wf(e0 + kQB),
          st.qkv[b], tr->QO);
-  if (r.ok) {
+  if (r.begin(FD_TK_NORM)) {
     const fd::train::Rope rp{tr->rope_t, tr->rope_y, tr->rope_x};
     const long long n = static_cast<long long>(M) * (tr->N + 2 * tr->G);
     fd::train::qkv_fwd_kernel<<<blocks_for(n, 128), 128, 0, r.s>>>(
-        st.qkv[b], M, tr->Lp, tr->L, tr->gw, tr->N, tr->G, tr->cfg.qk_norm, r.wf(e0 + kKG),
+        st.qkv[b], M, st.Pc, tr->Lp, tr->L, tr->gw, tr->N, tr->G, tr->cfg.qk_norm, r.wf(e0 + kKG),
         r.wf(e0 + kG2), tr->eps, rp, st.q2[b], st.k2[b], st.v1[b]);
     r.check(cudaGetLastError());
+    r.end();
   }
   attn_fwd(r, st, b);
-  r.bf(st.o32[b], static_cast<long long>(M) * tr->NQ, st.o[b]);
-  if (r.ok)
-    r.check(cudaMemcpyAsync(st.hm[b], st.h[b], sizeof(float) * M * tr->D,
-                            cudaMemcpyDeviceToDevice, r.s));
-  r.gemm(fd::EPI_RESID, M, tr->D, tr->NQ, st.o[b], tr->NQ, r.wb(e0 + kOW), tr->NQ,
+  if (r.begin(FD_TK_POINTWISE)) {  // O rows (bf16) for the output projection
+    const long long n = static_cast<long long>(M) * tr->NQ;
+    fd::train::head_permute_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.o32[b], M, st.Pc,
+                                                                         tr->N, 1, st.o[b]);
+    r.check(cudaGetLastError());
+    r.end();
+  }
+  r.copy(st.hm[b], st.h[b], static_cast<size_t>(M) * tr->D);
+  r.gemm(FD_TK_LINEAR, fd::EPI_RESID, M, tr->D, tr->NQ, st.o[b], tr->NQ, r.wb(e0 + kOW), tr->NQ,
          r.wf(e0 + kOB), st.hm[b], tr->D);
   r.rmsnorm(st.hm[b], r.wf(e0 + kN2), M, st.u2[b]);
-  r.gemm(fd::EPI_F32, M, tr->Dm, tr->D, st.u2[b], tr->D, r.wb(e0 + kM1W), tr->D,
+  r.gemm(FD_TK_LINEAR, fd::EPI_F32, M, tr->Dm, tr->D, st.u2[b], tr->D, r.wb(e0 + kM1W), tr->D,
          r.wf(e0 + kM1B), st.z[b], tr->Dm);
-  if (r.ok) {
+  if (r.begin(FD_TK_POINTWISE)) {
     const long long n = static_cast<long long>(M) * tr->Dm;
     fd::train::gelu_fwd_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.z[b], n, st.a[b]);
     r.check(cudaGetLastError());
+    r.end();
   }
-  if (r.ok)
-    r.check(cudaMemcpyAsync(st.h[b + 1], st.hm[b], sizeof(float) * M * tr->D,
-                            cudaMemcpyDeviceToDevice, r.s));
-  r.gemm(fd::EPI_RESID, M, tr->D, tr->Dm, st.a[b], tr->Dm, r.wb(e0 + kM2W), tr->Dm,
+  r.copy(st.h[b + 1], st.hm[b], static_cast<size_t>(M) * tr->D);
+  r.gemm(FD_TK_LINEAR, fd::EPI_RESID, M, tr->D, tr->Dm, st.a[b], tr->Dm, r.wb(e0 + kM2W), tr->Dm,
          r.wf(e0 + kM2B), st.h[b + 1], tr->D);
 }
 
@@ -648,18 +812,19 @@ void block_bwd(Run& r, fd_trainer_s::Stack& st, int b, size_t e0,
   float* dho = tr->gB;
   r.bf(dho, static_cast<long long>(M) * D, tr->dy16);
   // MLP layer 2
-  r.gemm(fd::EPI_F32, M, Dm, D, tr->dy16, D, lt.mlp2, D, nullptr, tr->gC, Dm);  // da
+  r.gemm(FD_TK_DGRAD, fd::EPI_F32, M, Dm, D, tr->dy16, D, lt.mlp2, D, nullptr, tr->gC, Dm);  // da
   r.wgrad(tr->dy16, D, st.a[b], Dm, M, r.grad(g, e0 + kM2W));
   r.colsum(dho, M, D, D, r.grad(g, e0 + kM2B));
   // GELU'
-  if (r.ok) {
+  if (r.begin(FD_TK_POINTWISE)) {
     const long long n = static_cast<long long>(M) * Dm;
     fd::train::gelu_bwd_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.z[b], tr->gC, n,
                                                                       tr->gC, tr->dqkv16);
     r.check(cudaGetLastError());
+    r.end();
   }
   // MLP layer 1
-  r.gemm(fd::EPI_F32, M, D, Dm, tr->dqkv16, Dm, lt.mlp1, Dm, nullptr, tr->gA, D);  // du2
+  r.gemm(FD_TK_DGRAD, fd::EPI_F32, M, D, Dm, tr->dqkv16, Dm, lt.mlp1, Dm, nullptr, tr->gA, D);  // du2
   r.wgrad(tr->dqkv16, Dm, st.u2[b], D, M, r.grad(g, e0 + kM1W));
   r.colsum(tr->gC, M, Dm, Dm, r.grad(g, e0 + kM1B));
   // RMSNorm 2, plus the residual
@@ -667,21 +832,21 @@ void block_bwd(Run& r, fd_trainer_s::Stack& st, int b, size_t e0,
   float* dhm = tr->gC;
   r.bf(dhm, static_cast<long long>(M) * D, tr->dy16);
   // output projection
-  r.gemm(fd::EPI_F32, M, NQ, D, tr->dy16, D, lt.out, D, nullptr, tr->gA, NQ);  // dO (fp32)
+  r.gemm(FD_TK_DGRAD, fd::EPI_F32, M, NQ, D, tr->dy16, D, lt.out, D, nullptr, tr->gA, NQ);  // dO (fp32)
   r.wgrad(tr->dy16, D, st.o[b], NQ, M, r.grad(g, e0 + kOW));
   r.colsum(dhm, M, D, D, r.grad(g, e0 + kOB));
-  r.bf(tr->gA, static_cast<long long>(M) * NQ, tr->do16);
-  // attention (reads dO from gA / do16)
+  // attention (reads dO from gA)
   attn_bwd(r, st, b);
   // KV-norm / QK-norm and RoPE backward
-  if (r.ok) {
+  if (r.begin(FD_TK_NORM)) {
     const fd::train::Rope rp{tr->rope_t, tr->rope_y, tr->rope_x};
     const long long n = static_cast<long long>(M) * (tr->N + 2 * tr->G);
     fd::train::qkv_bwd_kernel<<<blocks_for(n, 128), 128, 0, r.s>>>(
-        st.qkv[b], tr->dq2, tr->dk2, tr->dv1, M, tr->Lp, tr->L, tr->gw, tr->N, tr->G,
+        st.qkv[b], tr->dq2, tr->dk2, tr->dv1, M, st.Pc, tr->Lp, tr->L, tr->gw, tr->N, tr->G,
         tr->cfg.qk_norm, r.wf(e0 + kKG), r.wf(e0 + kG2), tr->eps, rp, tr->dqkv, tr->tq, tr->tk,
         tr->tv);
     r.check(cudaGetLastError());
+    r.end();
   }
   r.colsum(tr->tk, static_cast<long long>(M) * tr->G, 64, 64, r.grad(g, e0 + kKG));
   if (tr->cfg.qk_norm)
@@ -690,7 +855,7 @@ void block_bwd(Run& r, fd_trainer_s::Stack& st, int b, size_t e0,
     r.colsum(tr->tv, static_cast<long long>(M) * tr->G, 64, 64, r.grad(g, e0 + kG2));
   r.bf(tr->dqkv, static_cast<long long>(M) * QO, tr->dqkv16);
   // QKV projection
-  r.gemm(fd::EPI_F32, M, D, QO, tr->dqkv16, QO, lt.qkv, QO, nullptr, tr->gA, D);  // du
+  r.gemm(FD_TK_DGRAD, fd::EPI_F32, M, D, QO, tr->dqkv16, QO, lt.qkv, QO, nullptr, tr->gA, D);  // du
   r.wgrad(tr->dqkv16, QO, st.u[b], D, M, r.grad(g, e0 + kQW));
   r.colsum(tr->dqkv, M, QO, QO, r.grad(g, e0 + kQB));
   // RMSNorm 1, plus the residual: dh_in
@@ -760,7 +925,19 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
             MR = tr->MR;
   const int Mmax = MB > MR ? MB : MR;
   const int Pmax = tr->rt > 1 ? tr->rt * tr->Lp : tr->Lp;
-  const int Kmax = tr->Wn * Pmax;
+  const int Kmax = std::min(tr->T, tr->Wn) * Pmax;  // keys of one query chunk's window
+  // heads per attention product: all of a KV group's, unless S (fp32 [heads Pmax][Kmax]) would
+  // pass 512 M elements; then the largest divisor of the group size that stays within it
+  {
+    const int hpg = tr->N / tr->G;
+    tr->hs = 1;
+    for (int d = hpg; d >= 1; --d)
+      if (hpg % d == 0 && static_cast<size_t>(d) * Pmax * Kmax <= (static_cast<size_t>(1) << 29)) {
+        tr->hs = d;
+        break;
+      }
+  }
+  const size_t RK = static_cast<size_t>(tr->hs) * Pmax * Kmax;  // one product's scores
   tr->err = dalloc<int>(tr, 4, ok);
   tr->zero_bias = dalloc<float>(tr, std::max({Kmax, Dm, QO, NQ, tr->rt * D, tr->Cr, D}), ok);
   // RoPE tables, fp64 on the host (frames 0 .. T r_t - 1; rows; columns)
@@ -810,6 +987,7 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
       st.k2.push_back(dalloc<bf16>(tr, static_cast<size_t>(G) * M * 64, ok));
       st.v1.push_back(dalloc<bf16>(tr, static_cast<size_t>(G) * M * 64, ok));
       st.o32.push_back(dalloc<float>(tr, static_cast<size_t>(M) * NQ, ok));
+      st.lse.push_back(dalloc<float>(tr, static_cast<size_t>(M) * tr->N, ok));
       st.o.push_back(dalloc<bf16>(tr, static_cast<size_t>(M) * NQ, ok));
       st.hm.push_back(dalloc<float>(tr, static_cast<size_t>(M) * D, ok));
       st.u2.push_back(dalloc<bf16>(tr, static_cast<size_t>(M) * D, ok));
@@ -828,12 +1006,12 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   tr->vT = dalloc<bf16>(tr, static_cast<size_t>(G) * 64 * Mmax, ok);
   tr->kT = dalloc<bf16>(tr, static_cast<size_t>(G) * 64 * Mmax, ok);
   tr->do16 = dalloc<bf16>(tr, static_cast<size_t>(Mmax) * NQ, ok);
-  tr->dS = dalloc<bf16>(tr, static_cast<size_t>(Pmax) * Kmax, ok);
-  tr->P16 = dalloc<bf16>(tr, static_cast<size_t>(Pmax) * Kmax, ok);
-  tr->dST = dalloc<bf16>(tr, static_cast<size_t>(Pmax) * Kmax, ok);
-  tr->PT = dalloc<bf16>(tr, static_cast<size_t>(Pmax) * Kmax, ok);
-  tr->QT = dalloc<bf16>(tr, static_cast<size_t>(64) * Pmax, ok);
-  tr->dOT = dalloc<bf16>(tr, static_cast<size_t>(64) * Pmax, ok);
+  tr->dS = dalloc<bf16>(tr, RK, ok);
+  tr->P16 = dalloc<bf16>(tr, RK, ok);
+  tr->dST = dalloc<bf16>(tr, RK, ok);
+  tr->PT = dalloc<bf16>(tr, RK, ok);
+  tr->QT = dalloc<bf16>(tr, static_cast<size_t>(64) * tr->hs * Pmax, ok);
+  tr->dOT = dalloc<bf16>(tr, static_cast<size_t>(64) * tr->hs * Pmax, ok);
   tr->dy16 = dalloc<bf16>(tr, wide, ok);
   tr->dyT = dalloc<bf16>(tr, wide, ok);
   tr->xT = dalloc<bf16>(tr, wide, ok);
@@ -844,10 +1022,16 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   tr->dF = dalloc<float>(tr, static_cast<size_t>(MR) * tr->Cr, ok);
   tr->loss_blocks = static_cast<int>((static_cast<long long>(MR) * tr->Cr + 255) / 256);
   tr->loss_part = dalloc<float>(tr, tr->loss_blocks, ok);
-  tr->S = dalloc<float>(tr, static_cast<size_t>(Pmax) * Kmax, ok);
-  tr->P32 = dalloc<float>(tr, static_cast<size_t>(Pmax) * Kmax, ok);
-  tr->dP = dalloc<float>(tr, static_cast<size_t>(Pmax) * Kmax, ok);
-  tr->delta = dalloc<float>(tr, Pmax, ok);
+  tr->S = dalloc<float>(tr, RK, ok);
+  tr->dP = dalloc<float>(tr, RK, ok);
+  tr->delta = dalloc<float>(tr, static_cast<size_t>(Mmax) * tr->N, ok);
+  {
+    const size_t R = fd::train::kColsumRows;
+    const size_t widest = std::max({D, Dm, QO, NQ, tr->rt * D, tr->Cr});
+    tr->colsum_elems = std::max((static_cast<size_t>(Mmax) * tr->N + R - 1) / R * 64,
+                                (static_cast<size_t>(Mmax) + R - 1) / R * widest);
+    tr->colsum_part = dalloc<float>(tr, tr->colsum_elems, ok);
+  }
   tr->dq2 = dalloc<float>(tr, static_cast<size_t>(Mmax) * NQ, ok);
   tr->dk2 = dalloc<float>(tr, static_cast<size_t>(G) * Mmax * 64, ok);
   tr->dv1 = dalloc<float>(tr, static_cast<size_t>(G) * Mmax * 64, ok);
@@ -908,66 +1092,78 @@ fd_status fd_train_step(fd_trainer tr, const float* latents, const float* target
   const int D = tr->D, MB = tr->MB, MR = tr->MR, rt = tr->rt;
   const size_t eB = 2, eF = eB + static_cast<size_t>(tr->nb) * kBlockEntries;
   const size_t eR = eF + 3, eH = eR + static_cast<size_t>(tr->nr) * kBlockEntries;
-  if (r.ok) r.check(cudaMemsetAsync(tr->err, 0, sizeof(int), r.s));
+  if (r.begin(FD_TK_POINTWISE)) {
+    r.check(cudaMemsetAsync(tr->err, 0, sizeof(int), r.s));
+    r.end();
+  }
   // ---- forward
   // patch-embedding (Eq. projection) of every chunk: PixelUnshuffle rows, then the linear
   const size_t chw = static_cast<size_t>(tr->C) * tr->H * tr->W;
-  for (int c = 0; c < tr->T && r.ok; ++c)
+  for (int c = 0; c < tr->T && r.begin(FD_TK_POINTWISE); ++c) {
     r.check(fd::launch_unshuffle(latents + c * chw, tr->C, tr->H, tr->W, tr->p,
                                  tr->x0 + static_cast<size_t>(c) * tr->Lp * tr->cin, r.s));
-  r.gemm(fd::EPI_F32, MB, D, tr->cin, tr->x0, tr->cin, r.wb(0), tr->cin, r.wf(1), tr->sB.h[0], D);
+    r.end();
+  }
+  r.gemm(FD_TK_LINEAR, fd::EPI_F32, MB, D, tr->cin, tr->x0, tr->cin, r.wb(0), tr->cin, r.wf(1), tr->sB.h[0], D);
   for (int b = 0; b < tr->nb; ++b)
     block_fwd(r, tr->sB, b, eB + static_cast<size_t>(b) * kBlockEntries);
   // final norm and temporal upsampling (Eq. temporal_upsample): channel block tau -> frame tau
   const float* hBo = tr->sB.h[tr->nb];
   r.rmsnorm(hBo, r.wf(eF), MB, tr->y16);
-  r.gemm(fd::EPI_F32, MB, rt * D, D, tr->y16, D, r.wb(eF + 1), D, r.wf(eF + 2), tr->e, rt * D);
-  if (r.ok) {
+  r.gemm(FD_TK_LINEAR, fd::EPI_F32, MB, rt * D, D, tr->y16, D, r.wb(eF + 1), D, r.wf(eF + 2), tr->e, rt * D);
+  if (r.begin(FD_TK_POINTWISE)) {
     const long long n = static_cast<long long>(MB) * rt * D;
     fd::train::tup_permute_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(
         tr->e, tr->T, rt, tr->Lp, D, 0, tr->sR.h[0], nullptr);
     r.check(cudaGetLastError());
+    r.end();
   }
   for (int b = 0; b < tr->nr; ++b)
     block_fwd(r, tr->sR, b, eR + static_cast<size_t>(b) * kBlockEntries);
   // head (Sec. 3.4 Step 3): RMSNorm, Linear + GELU, Linear to C r_s^2 per refined token
   const float* hRo = tr->sR.h[tr->nr];
   r.rmsnorm(hRo, r.wf(eH), MR, tr->yh16);
-  r.gemm(fd::EPI_F32, MR, D, D, tr->yh16, D, r.wb(eH + 1), D, r.wf(eH + 2), tr->z1, D);
-  if (r.ok) {
+  r.gemm(FD_TK_LINEAR, fd::EPI_F32, MR, D, D, tr->yh16, D, r.wb(eH + 1), D, r.wf(eH + 2), tr->z1, D);
+  if (r.begin(FD_TK_POINTWISE)) {
     const long long n = static_cast<long long>(MR) * D;
     fd::train::gelu_fwd_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(tr->z1, n, tr->a1);
     r.check(cudaGetLastError());
+    r.end();
   }
-  r.gemm(fd::EPI_F32, MR, tr->Cr, D, tr->a1, D, r.wb(eH + 3), D, r.wf(eH + 4), tr->F, tr->Cr);
+  r.gemm(FD_TK_LINEAR, fd::EPI_F32, MR, tr->Cr, D, tr->a1, D, r.wb(eH + 3), D, r.wf(eH + 4), tr->F, tr->Cr);
   // ---- loss (L1 over every pixel of the clip) and its gradient through the pixel shuffle
   const double total = static_cast<double>(tr->T) * rt * tr->Cout * tr->gh * tr->rs * tr->gw *
                        tr->rs;
   const float inv_total = static_cast<float>(1.0 / total);
-  if (r.ok) {
+  if (r.begin(FD_TK_POINTWISE)) {
     fd::train::l1_head_kernel<<<tr->loss_blocks, 256, 0, r.s>>>(
         tr->F, targets, tr->T, rt, tr->Lp, tr->L, tr->gh, tr->gw, tr->Cout, tr->rs, inv_total,
         tr->dF, tr->loss_part);
     r.check(cudaGetLastError());
+    r.end();
+  }
+  if (r.begin(FD_TK_POINTWISE)) {
     fd::train::finish_loss_kernel<<<1, 32, 0, r.s>>>(tr->loss_part, tr->loss_blocks, inv_total,
                                                      loss);
     r.check(cudaGetLastError());
+    r.end();
   }
   // ---- backward
   float* g = grads;
   // head layer 2
   r.bf(tr->dF, static_cast<long long>(MR) * tr->Cr, tr->dy16);
-  r.gemm(fd::EPI_F32, MR, D, tr->Cr, tr->dy16, tr->Cr, tr->t_head2, tr->Cr, nullptr, tr->gC, D);
+  r.gemm(FD_TK_DGRAD, fd::EPI_F32, MR, D, tr->Cr, tr->dy16, tr->Cr, tr->t_head2, tr->Cr, nullptr, tr->gC, D);
   r.wgrad(tr->dy16, tr->Cr, tr->a1, D, MR, r.grad(g, eH + 3));
   r.colsum(tr->dF, MR, tr->Cr, tr->Cr, r.grad(g, eH + 4));
   // head layer 1 (GELU')
-  if (r.ok) {
+  if (r.begin(FD_TK_POINTWISE)) {
     const long long n = static_cast<long long>(MR) * D;
     fd::train::gelu_bwd_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(tr->z1, tr->gC, n, tr->gC,
                                                                       tr->dqkv16);
     r.check(cudaGetLastError());
+    r.end();
   }
-  r.gemm(fd::EPI_F32, MR, D, D, tr->dqkv16, D, tr->t_head1, D, nullptr, tr->gA, D);
+  r.gemm(FD_TK_DGRAD, fd::EPI_F32, MR, D, D, tr->dqkv16, D, tr->t_head1, D, nullptr, tr->gA, D);
   r.wgrad(tr->dqkv16, D, tr->yh16, D, MR, r.grad(g, eH + 1));
   r.colsum(tr->gC, MR, D, D, r.grad(g, eH + 2));
   // the head's RMSNorm
@@ -975,13 +1171,14 @@ fd_status fd_train_step(fd_trainer tr, const float* latents, const float* target
   for (int b = tr->nr - 1; b >= 0; --b)
     block_bwd(r, tr->sR, b, eR + static_cast<size_t>(b) * kBlockEntries, tr->tR[b], g);
   // temporal upsampling: refined frame tau back to channel block tau
-  if (r.ok) {
+  if (r.begin(FD_TK_POINTWISE)) {
     const long long n = static_cast<long long>(MB) * rt * D;
     fd::train::tup_permute_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(
         tr->gB, tr->T, rt, tr->Lp, D, 1, tr->gC, tr->dqkv16);
     r.check(cudaGetLastError());
+    r.end();
   }
-  r.gemm(fd::EPI_F32, MB, D, rt * D, tr->dqkv16, rt * D, tr->t_tup, rt * D, nullptr, tr->gA, D);
+  r.gemm(FD_TK_DGRAD, fd::EPI_F32, MB, D, rt * D, tr->dqkv16, rt * D, tr->t_tup, rt * D, nullptr, tr->gA, D);
   r.wgrad(tr->dqkv16, rt * D, tr->y16, D, MB, r.grad(g, eF + 1));
   r.colsum(tr->gC, MB, rt * D, rt * D, r.grad(g, eF + 2));
   r.rmsnorm_bwd(hBo, r.wf(eF), tr->gA, nullptr, MB, tr->gB, r.grad(g, eF));
@@ -1043,9 +1240,34 @@ fd_status fd_train_status(fd_trainer tr, void* stream) {
   return e ? FD_ERR_DEVICE_TIMEOUT : FD_OK;
 }
 
+fd_status fd_train_profile_enable(fd_trainer tr, int enable) {
+  if (tr == nullptr) return FD_ERR_INVALID_ARG;
+  tr->prof = enable != 0;
+  return FD_OK;
+}
+
+fd_status fd_train_profile_collect(fd_trainer tr, int64_t* launches, double* ms) {
+  if (tr == nullptr || launches == nullptr || ms == nullptr) return FD_ERR_INVALID_ARG;
+  if (cudaDeviceSynchronize() != cudaSuccess) return FD_ERR_CUDA;
+  fd_status st = FD_OK;
+  for (const fd_trainer_s::Rec& e : tr->rec) {
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, e.a, e.b) != cudaSuccess) st = FD_ERR_CUDA;
+    if (e.kind >= 0 && e.kind < FD_TK_COUNT) {
+      launches[e.kind] += 1;
+      ms[e.kind] += t;
+    }
+    tr->ev_free.push_back(e.a);
+    tr->ev_free.push_back(e.b);
+  }
+  tr->rec.clear();
+  return st;
+}
+
 fd_status fd_train_destroy(fd_trainer tr) {
   if (tr == nullptr) return FD_ERR_INVALID_ARG;
   cudaDeviceSynchronize();
+  for (cudaEvent_t e : tr->ev_all) cudaEventDestroy(e);
   for (void* ptr : tr->allocs) cudaFree(ptr);
   fd::weights_add_user(tr->w, -1);
   delete tr;

@@ -27,6 +27,9 @@ EPI_F32, EPI_RESID, EPI_GELU, EPI_TUP, EPI_SWIGLU = 0, 1, 2, 3, 4
 # fd_kernel_kind order
 KERNEL_KINDS = ["unshuffle", "embed", "rmsnorm", "qkv", "attn_backbone", "attn_refine", "out",
                 "mlp1", "mlp2", "tup", "head1", "head2", "pixel", "advance", "rope"]
+# kernel kinds of the training step (enum fd_train_kind)
+TRAIN_KINDS = ["linear", "dgrad", "wgrad", "attn_gemm", "softmax", "transpose", "norm",
+               "pointwise"]
 
 
 class FdError(RuntimeError):
@@ -84,6 +87,9 @@ _SIGS = {
     "fd_train_create": (_I, [ctypes.POINTER(fd_config), _P, _I, ctypes.POINTER(_P)]),
     "fd_train_step": (_I, [_P, _P, _P, _P, _P, _P]),
     "fd_train_status": (_I, [_P, _P]),
+    "fd_train_profile_enable": (_I, [_P, _I]),
+    "fd_train_profile_collect": (_I, [_P, ctypes.POINTER(ctypes.c_int64),
+                                      ctypes.POINTER(ctypes.c_double)]),
     "fd_train_destroy": (_I, [_P]),
     "fd_state_bytes": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
     "fd_save_state": (_I, [_P, _P, ctypes.c_size_t, _P]),
@@ -380,6 +386,19 @@ class Trainer:
 
     def status(self, stream=None) -> int:
         return lib().fd_train_status(self.handle, _stream_ptr(stream))
+
+    def profile(self, enable: bool) -> None:
+        _check(lib().fd_train_profile_enable(self.handle, 1 if enable else 0),
+               "fd_train_profile_enable")
+
+    def profile_collect(self) -> dict:
+        """{kind name: (launches, device ms)} of the steps since the last collect."""
+        n = len(TRAIN_KINDS)
+        launches = (ctypes.c_int64 * n)()
+        ms = (ctypes.c_double * n)()
+        _check(lib().fd_train_profile_collect(self.handle, launches, ms),
+               "fd_train_profile_collect")
+        return {k: (int(launches[i]), float(ms[i])) for i, k in enumerate(TRAIN_KINDS)}
 
     def close(self) -> None:
         if getattr(self, "handle", None):

@@ -157,3 +157,31 @@ def test_l1_pixel_backward_kernel():
     want_dF = pixel_shuffle_bwd(l1_bwd(pix, x, total), frames, gh, gw, C, rs)
     assert abs(float(loss.item()) - want_loss) <= 1e-6 * want_loss
     assert float((dF.cpu().double() - want_dF).abs().max()) <= 1e-7 / total
+
+
+def test_training_profile_counts_every_kind():
+    """fd_train_profile_*: one profiled step brackets launches of every kernel kind; a second
+    collect returns nothing (the events were released); the profiled step's gradients equal an
+    unprofiled step's bits."""
+    cfg = synth.PRESETS["tiny_rt"]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    x = synth.make_target_pixels(cfg, min_abs=0.3)
+    W = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    tr = fdp.Trainer(cfg, W, len(z))
+    lat = torch.from_numpy(np.ascontiguousarray(np.stack(z))).cuda()
+    tgt = torch.from_numpy(np.ascontiguousarray(np.stack(x))).cuda()
+    loss = torch.zeros(1, device="cuda")
+    plain = torch.zeros(tr.grad_elems, device="cuda")
+    tr.step(lat, tgt, loss, plain)
+    grads = torch.zeros(tr.grad_elems, device="cuda")
+    tr.profile(True)
+    tr.step(lat, tgt, loss, grads)
+    prof = tr.profile_collect()
+    tr.profile(False)
+    assert set(prof) == set(fdp.TRAIN_KINDS)
+    for k, (n, ms) in prof.items():
+        assert n > 0 and ms > 0, (k, n, ms)
+    assert all(v == (0, 0.0) for v in tr.profile_collect().values())
+    assert torch.equal(grads, plain)
+    tr.close()
+    W.close()
