@@ -41,6 +41,7 @@ def parse():
                          "forked CUDA stream per decoder (fd_decode_chunks)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-secondary", action="store_true", help="skip the 720p line")
+    ap.add_argument("--no-training", action="store_true", help="skip the training-step line")
     return ap.parse_args()
 
 
@@ -388,6 +389,8 @@ def run_ours(args, rank: int, world: int):
     }
     if rank == 0 and world == 1 and not args.no_secondary and cfg.name == "480p":
         line["secondary"] = secondary_720p(args, stream, blob)
+    if rank == 0 and world == 1 and not args.no_training and cfg.name == "480p":
+        line["training"] = training_line(args, stream, blob)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(cfg, w)
     if batch is not None:
@@ -471,6 +474,77 @@ def secondary_720p(args, stream, blob):
                          "gemm_frac": round(kp["gemm_frac"], 3),
                          "measured_over": "1 profiled stream (CUDA events around each launch)"},
             "kernels": kp["kernels"], "device_ok": ok}
+
+
+TRAIN_CHUNKS = 2
+
+
+def training_line(args, stream, blob):
+    """Streaming training step of the 480p model (fd_train_step) over a clip of TRAIN_CHUNKS
+    latent chunks: forward with every activation kept, L1 loss against the target pixels, every
+    parameter's gradient. Synthetic latents and targets, the bench's random-init weights; inputs
+    resident in HBM. Steps timed with CUDA events on the launching stream; then one profiled
+    step (events around every launch) for the per-kind times and the dominant kind's roofline."""
+    import numpy as np
+    import torch
+
+    import synth
+    from paper_2607_14898_gb300 import costs
+    from paper_2607_14898_gb300 import flashdec as fdp
+
+    cfg = synth.PRESETS["480p"]
+    T = TRAIN_CHUNKS
+    weights = fdp.Weights(cfg, blob)
+    tr = fdp.Trainer(cfg, weights, T)
+    lat = torch.from_numpy(synth.make_latents(cfg, chunks=T)).cuda()
+    tgt = torch.from_numpy(np.ascontiguousarray(
+        np.stack(synth.make_target_pixels(cfg, chunks=T, min_abs=0.3)))).cuda()
+    loss = torch.zeros(1, device="cuda")
+    grads = torch.zeros(tr.grad_elems, device="cuda")
+    for _ in range(max(3, args.warmup)):
+        tr.step(lat, tgt, loss, grads, stream)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    steps = max(1, args.steps)
+    a.record(stream)
+    for _ in range(steps):
+        tr.step(lat, tgt, loss, grads, stream)
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / steps
+    ok = tr.status(stream) == fdp.FD_OK
+    tr.profile(True)
+    tr.step(lat, tgt, loss, grads, stream)
+    prof = tr.profile_collect()
+    tr.profile(False)
+    tr.close()
+    weights.close()
+    _, sustained, hbm, peak_src = peaks()
+    fl = costs.training_kind_flops(cfg, T)
+    total = sum(fl.values())
+    kinds = {}
+    for k, (n, kms) in prof.items():
+        e = {"launches": n, "ms": round(kms, 3)}
+        if k in fl and kms > 0:
+            e["tflops"] = round(fl[k] / (kms * 1e-3) / 1e12, 1)
+        kinds[k] = e
+    top = max(prof, key=lambda k: prof[k][1])
+    dom = {"kernel": f"{top} (the kind with the most device time in the profiled step)"}
+    if top in fl:
+        ach = fl[top] / (prof[top][1] * 1e-3) / 1e12
+        dom.update({"bound": "tensor", "achieved": round(ach, 1), "peak": sustained,
+                    "unit": "TFLOP/s", "frac": round(ach / sustained, 3),
+                    "peak_source": f"bf16_tflops_sustained ({peak_src})",
+                    "work": "algorithmic FLOPs of the kind (costs.training_kind_flops)"})
+    return {"workload": f"480p model (24 + 2 blocks, D 1024), streaming training step over a "
+                        f"clip of {T} latent chunks ({T * cfg.r_t} frames): forward with the "
+                        "activations kept, L1 loss, every parameter's gradient",
+            "ms_per_step": round(ms, 3), "steps": steps,
+            "frames_per_s": round(T * cfg.r_t / (ms * 1e-3), 2),
+            "tflops": round(total / (ms * 1e-3) / 1e12, 1),
+            "tensor_frac_step": round(total / (ms * 1e-3) / 1e12 / sustained, 3),
+            "roofline": dom, "kinds": kinds,
+            "profiled_ms": round(sum(v[1] for v in prof.values()), 3), "device_ok": ok}
 
 
 def cpu_model() -> str:

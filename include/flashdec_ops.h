@@ -159,6 +159,19 @@ fd_status fd_op_unshuffle(const float* z, int C, int H, int W, int p, void* x0, 
 fd_status fd_op_pixel_head(const float* F, int frames, int grid_h, int grid_w, int channels,
                            int rs, int out_dtype, void* pixels, void* stream);
 
+/* Head layer 2 with the pixel shuffle folded into the product's epilogue (Sec. 3.4 Step 3;
+ * the decoder's last product, run this way by fd_decode_chunk): in one launch, the pixels that
+ * fd_op_pixel_head gives from fd_op_linear's F = A W^T + b, bit for bit, without storing F.
+ * A bf16 [M][K], the rows of frame tau's tokens at tau L .. tau L + L - 1 (L = grid_h grid_w);
+ * W bf16 [channels rs^2][K]; bias fp32 [channels rs^2]. The first `frames` frames (frames L <=
+ * M) are written: pixels [channels][frames][grid_h rs][grid_w rs], fp32 clamped to [-1, 1]
+ * (out_dtype FD_DTYPE_F32) or uint8 codes (FD_DTYPE_U8). 128 x 256 tiles on single CTAs. rs % 4 == 0, 32 % rs == 0,
+ * K % 8 == 0, (channels rs^2) % 32 == 0; 16-byte aligned A / W / bias / pixels.
+ * Errors: FD_ERR_INVALID_ARG, FD_ERR_CUDA; err_dev as for fd_op_linear. */
+fd_status fd_op_linear_pixel(int M, int K, const void* A, const void* W, const float* bias,
+                             int frames, int grid_h, int grid_w, int channels, int rs,
+                             int out_dtype, void* pixels, int* err_dev, void* stream);
+
 /* ---- single kernels of the training step (fd_train_step), for per-kernel checks ---- */
 
 /* RMSNorm backward (the derivative of y = x r g, r = (mean(x^2) + eps)^(-1/2), Sec. 3.2):

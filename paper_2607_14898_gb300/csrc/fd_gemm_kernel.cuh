@@ -602,6 +602,45 @@ __global__ void __launch_bounds__(192, 1)
             bulk_commit();
           }
         }
+      } else if (BN == 256 && !PAIR && p.epi == EPI_PIXEL) {
+        // head layer 2 with the pixel shuffle (Sec. 3.4 Step 3): each 32-column chunk of the
+        // token's row is 32 / rs pixel rows of rs pixels, written as groups of 4 pixels
+        const PixelEpi& px = p.pix;
+        const int tau = row / px.tokens, l = row - tau * px.tokens;
+        const bool out_row = row_ok && tau < px.frames;
+        const int gy = l / px.gw, gx = l - gy * px.gw;
+        const int rs = px.rs, rs2 = rs * rs, Wo = px.gw * rs, Ho = px.gh * rs;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          const int col = n0 + c;
+          if (col >= p.N) break;
+          uint32_t r[32];
+          __syncwarp();
+          tmem_ld_32x32b_x32(tbase + c, r);
+          tmem_ld_wait();
+          float bb[32];
+          load32(p.bias + col, bb);
+          if (!out_row) continue;
+          const int ch = col / rs2, rem = col - ch * rs2;
+#pragma unroll
+          for (int j = 0; j < 32; j += 4) {
+            const int y = gy * rs + (rem + j) / rs, x = gx * rs + (rem + j) % rs;
+            const size_t o = ((static_cast<size_t>(ch) * px.frames + tau) * Ho + y) * Wo + x;
+            const float v0 = __uint_as_float(r[j]) + bb[j];
+            const float v1 = __uint_as_float(r[j + 1]) + bb[j + 1];
+            const float v2 = __uint_as_float(r[j + 2]) + bb[j + 2];
+            const float v3 = __uint_as_float(r[j + 3]) + bb[j + 3];
+            if (px.u8) {
+              *reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(px.out) + o) =
+                  quant_u8(v0) | (quant_u8(v1) << 8) | (quant_u8(v2) << 16) |
+                  (quant_u8(v3) << 24);
+            } else {
+              *reinterpret_cast<float4*>(static_cast<float*>(px.out) + o) =
+                  make_float4(fminf(fmaxf(v0, -1.f), 1.f), fminf(fmaxf(v1, -1.f), 1.f),
+                              fminf(fmaxf(v2, -1.f), 1.f), fminf(fmaxf(v3, -1.f), 1.f));
+            }
+          }
+        }
       } else {  // EPI_F32, EPI_RESID, EPI_TUP: fp32 slabs of 32 columns
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {

@@ -45,6 +45,18 @@ enum EpiKind : int {
   EPI_GELU_F8 = 6,  // out_f8[r][c] = e4m3(GELU(acc * col_scale + bias) * out_scale)
   EPI_SWIGLU_F8 = 7,  // gated: out_f8[r][32j + i] = e4m3(SiLU(g) u out_scale) with g, u the
                       // (acc * col_scale + bias) of the interleaved gate / up columns
+  EPI_PIXEL = 8,  // head layer 2 with the pixel shuffle: row tau L + l, column c rs^2 + dy rs + dx
+                  // -> pixel [c][tau][gy rs + dy][gx rs + dx] (l = gy gw + gx), clamped to
+                  // [-1, 1] as fp32 or as its uint8 code; frames past pix.frames are not written
+};
+
+// Output of EPI_PIXEL (the pixel head folded into the last product of the decoder).
+struct PixelEpi {
+  void* out;        // [C][frames][gh rs][gw rs], fp32 or uint8
+  int u8;
+  int frames;       // frames written (rows tau L + l with tau >= frames are dropped)
+  int tokens;       // L: rows per frame
+  int gh, gw, rs;   // token grid and the spatial upscale (rs % 4 == 0, 32 % rs == 0)
 };
 
 // One stream of a batched QKV launch: its cache ring, chunk counter and temporal RoPE table.
@@ -113,7 +125,12 @@ struct GemmParams {
   // W is never written by a kernel of the stream (the decoder's weights): its first stages may
   // load before the dependency on the previous kernel is resolved
   int w_static;
+  PixelEpi pix;  // EPI_PIXEL
 };
+// EPI_PIXEL is compiled into the single-CTA 256-wide instance only
+inline bool gemm_pixel_epilogue_ok(int bn, bool pair, int rs) {
+  return bn == 256 && !pair && rs % 4 == 0 && 32 % rs == 0;
+}
 
 // one stream of a batched attention launch (grid y = stream): its ring's K and V^T maps, its
 // chunk counter and error word

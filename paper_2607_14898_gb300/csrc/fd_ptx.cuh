@@ -456,6 +456,13 @@ __device__ __forceinline__ float f16x2_sum(uint32_t a) {
   return __low2float(h) + __high2float(h);
 }
 
+// uint8 pixel code of a decoder output: NaN -> -1 through fmaxf, then the clamp to [-1, 1];
+// code = rint_even(fl(fl(x + 1) * 127.5))
+__device__ __forceinline__ uint32_t quant_u8(float x) {
+  x = fminf(fmaxf(x, -1.0f), 1.0f);
+  return static_cast<uint32_t>(__float2int_rn(__fmul_rn(__fadd_rn(x, 1.0f), 127.5f)));
+}
+
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));

@@ -106,11 +106,6 @@ __global__ void rmsnorm_kernel(const float* __restrict__ h, const float* __restr
   }
 }
 
-__device__ __forceinline__ uint32_t quant_u8(float x) {
-  // NaN -> -1 through fmaxf, then the clamp; code = rint_even(fl(fl(x + 1) * 127.5))
-  x = fminf(fmaxf(x, -1.0f), 1.0f);
-  return static_cast<uint32_t>(__float2int_rn(__fmul_rn(__fadd_rn(x, 1.0f), 127.5f)));
-}
 
 // pix[c][tau][y][x] = clamp(F[tau*L + (y/rs)*gw + x/rs][c*rs*rs + (y%rs)*rs + x%rs]); rs % 4 == 0
 // frame tau's tokens are rows tau * frame_rows .. + gh gw - 1 of F (frame_rows >= gh gw)

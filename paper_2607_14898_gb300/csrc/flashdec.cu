@@ -674,14 +674,22 @@ fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_
   ph.out_bf16 = h->hid;
   ph.ld_out = d.D;
   if ((st = run_linear(h, FD_K_HEAD1, h->tm_uR, w->head1, R, ph, h->so_hidH, s))) return st;
+  // the causal frame count (Fig. 2): chunk 0 emits refined frame 0 only (rows 0 .. L-1 of F)
+  const int frames = d.f1 && h->t_host == 0 ? 1 : d.rt;
   fd::GemmParams pf{};
+  if (fd::gemm_pixel_epilogue_ok(w->head2.bn, w->head2.pair, d.rs)) {
+    // the pixel shuffle, clamp (and uint8 code) in the product's epilogue: F is never stored
+    pf.epi = fd::EPI_PIXEL;
+    pf.pix = {pixels, d.u8 ? 1 : 0, frames, d.L, d.gh, d.gw, d.rs};
+    if ((st = run_linear(h, FD_K_HEAD2, h->tm_hidH, w->head2, R, pf, h->so_F, s))) return st;
+    int* state = h->state;
+    return traced(h, FD_K_ADVANCE, s, [&] { return fd::launch_advance(state, s); });
+  }
   pf.epi = fd::EPI_F32;
   pf.out_f32 = h->F;
   pf.ld_out = d.head_out;
   if ((st = run_linear(h, FD_K_HEAD2, h->tm_hidH, w->head2, R, pf, h->so_F, s))) return st;
   const float* F = h->F;
-  // the causal frame count (Fig. 2): chunk 0 emits refined frame 0 only (rows 0 .. L-1 of F)
-  const int frames = d.f1 && h->t_host == 0 ? 1 : d.rt;
   if ((st = traced(h, FD_K_PIXEL, s, [&] {
          return fd::launch_pixel_head(F, frames, d.gh, d.gw, d.Cout, d.rs, d.u8 ? 1 : 0, pixels,
                                       s);
@@ -1925,6 +1933,34 @@ fd_status fd_op_linear_tiled(int epilogue, int M, int N, int K, const void* A, c
   p.tup_tokens = M;
   p.tup_hidden = tup_hidden;
   return launch_ok(fd::launch_gemm(ta, tb, to, to, to, p, bn, pair == 2, num_sms(),
+                                   static_cast<cudaStream_t>(stream)));
+}
+
+fd_status fd_op_linear_pixel(int M, int K, const void* A, const void* W, const float* bias,
+                             int frames, int grid_h, int grid_w, int channels, int rs,
+                             int out_dtype, void* pixels, int* err_dev, void* stream) {
+  if (A == nullptr || W == nullptr || bias == nullptr || pixels == nullptr ||
+      err_dev == nullptr || M < 1 || K < 1 || grid_h < 1 || grid_w < 1 || channels < 1 ||
+      frames < 1 || (out_dtype != FD_DTYPE_F32 && out_dtype != FD_DTYPE_U8))
+    return FD_ERR_INVALID_ARG;
+  if (!fd::gemm_pixel_epilogue_ok(256, false, rs) || K % 8) return FD_ERR_INVALID_ARG;
+  const long long L = static_cast<long long>(grid_h) * grid_w;
+  const long long N = static_cast<long long>(channels) * rs * rs;
+  if (N % 32 || N > (1 << 20) || L * frames > M || L > (1 << 24)) return FD_ERR_INVALID_ARG;
+  if (!aligned16(A) || !aligned16(W) || !aligned16(bias) || !aligned16(pixels))
+    return FD_ERR_INVALID_ARG;
+  fd_status st = check_device();
+  if (st) return st;
+  CUtensorMap ta, tb;
+  if (!tmap_bf16(&ta, A, K, M, static_cast<uint64_t>(K) * 2, 64, 128) ||
+      !tmap_bf16(&tb, W, K, static_cast<int>(N), static_cast<uint64_t>(K) * 2, 64, 256))
+    return FD_ERR_CUDA;
+  fd::GemmParams p{};
+  p.M = M; p.N = static_cast<int>(N); p.K = K; p.epi = fd::EPI_PIXEL; p.bias = bias;
+  p.err = err_dev;
+  p.pix = {pixels, out_dtype == FD_DTYPE_U8 ? 1 : 0, frames, static_cast<int>(L), grid_h, grid_w,
+           rs};
+  return launch_ok(fd::launch_gemm(ta, tb, ta, ta, ta, p, 256, false, num_sms(),
                                    static_cast<cudaStream_t>(stream)));
 }
 

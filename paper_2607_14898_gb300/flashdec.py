@@ -81,6 +81,7 @@ _SIGS = {
     "fd_debug_read_ring": (_I, [_P, _I, _I, _P, ctypes.c_size_t]),
     "fd_debug_wait_timeout": (_I, [_P, ctypes.c_uint, _P]),
     "fd_train_grad_elems": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
+    "fd_op_linear_pixel": (_I, [_I, _I, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P]),
     "fd_op_rmsnorm_bwd": (_I, [_P, _P, _P, _I, _I, _F, _P, _P, _P, _P]),
     "fd_op_gelu_bwd": (_I, [_P, _P, ctypes.c_int64, _P, _P, _P]),
     "fd_op_l1_pixel_bwd": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P]),
@@ -553,6 +554,15 @@ def op_unshuffle(z, p, x0, stream=None) -> None:
 def op_pixel_head(F, frames, grid_h, grid_w, channels, rs, out_dtype, pixels, stream=None) -> None:
     _check(lib().fd_op_pixel_head(_ptr(F), frames, grid_h, grid_w, channels, rs, out_dtype,
                                   _ptr(pixels), _stream_ptr(stream)), "fd_op_pixel_head")
+
+
+def op_linear_pixel(A, W, bias, frames, grid_h, grid_w, channels, rs, out_dtype, pixels,
+                    err=None, stream=None) -> None:
+    """Head layer 2 with the pixel shuffle in its epilogue (fd_op_linear_pixel)."""
+    M, K = A.shape
+    _check(lib().fd_op_linear_pixel(M, K, _ptr(A), _ptr(W), _ptr(bias), frames, grid_h, grid_w,
+                                    channels, rs, out_dtype, _ptr(pixels), _ptr(err),
+                                    _stream_ptr(stream)), "fd_op_linear_pixel")
 
 
 def op_rmsnorm_bwd(x, g, dy, eps, dx, dg, stream=None) -> None:

@@ -98,6 +98,35 @@ def test_linear_cta_pairs(M, N, K, bn):
         assert torch.equal(g1, g2)
 
 
+@pytest.mark.parametrize("frames_in,frames,gh,gw,C,rs,u8", [
+    (4, 4, 30, 52, 3, 16, False),  # 480p refinement rows -> 4 fp32 frames
+    (4, 4, 45, 80, 3, 16, True),   # 720p, uint8 codes
+    (4, 1, 6, 7, 3, 16, False),    # first chunk of a one-frame-first stream: frame 0 only
+    (2, 2, 9, 11, 3, 8, True),     # rs 8 (four pixel rows per 32 columns), ragged tiles
+])
+def test_linear_pixel_equals_linear_then_pixel_head(frames_in, frames, gh, gw, C, rs, u8):
+    """The pixel shuffle folded into head layer 2's epilogue gives the bits of the two-launch
+    path (fd_op_linear's F, then fd_op_pixel_head), fp32 and uint8, including outputs past the
+    clamp (the inputs are scaled so that some pre-activations leave [-1, 1])."""
+    L = gh * gw
+    M, K, N = frames_in * L, 256, C * rs * rs
+    A, W, b = linear_case(M, N, K, seed=M + N)
+    Ad, Wd, bd = dev(A, torch.bfloat16), dev(W * 3.0, torch.bfloat16), dev(b)
+    err = err_word()
+    F = torch.zeros(M, N, device="cuda")
+    fdp.op_linear(fdp.EPI_F32, Ad, Wd, bd, F, err=err, bn=256)
+    shape = (C, frames, gh * rs, gw * rs)
+    dtype = torch.uint8 if u8 else torch.float32
+    want = torch.zeros(shape, dtype=dtype, device="cuda")
+    code = 2 if u8 else 0  # FD_DTYPE_U8 / FD_DTYPE_F32
+    fdp.op_pixel_head(F, frames, gh, gw, C, rs, code, want)
+    got = torch.full(shape, 7, dtype=dtype, device="cuda")
+    fdp.op_linear_pixel(Ad, Wd, bd, frames, gh, gw, C, rs, code, got, err=err)
+    check_err(err)
+    assert float((F.abs() > 1).float().mean()) > 0.01  # the clamp is exercised
+    assert torch.equal(got, want)
+
+
 def test_gelu_epilogue_is_the_exact_erf_gelu_at_bf16():
     """The GELU epilogue evaluates erf with Abramowitz & Stegun 7.1.26 (error <= 1.5e-7): on a
     grid of pre-activations from -8 to 8 (A holds x in one column, W picks it, the bias shifts
