@@ -132,7 +132,9 @@ struct Cursor {
 
 // kBatched: grid y = stream of p.streams (K / V maps, counter and error word from there; Q,
 // output and workspace offset by the stream)
-template <bool kBatched>
+// kLse (batched only): also write each row's log-sum-exp of the scaled scores (natural log) to
+// p.lse[(stream * heads + head) * p.lse_pitch + row], for a backward that recomputes P
+template <bool kBatched, bool kLse = false>
 __global__ void __launch_bounds__(attn::kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQ8,
                 const __grid_constant__ CUtensorMap tmK,
@@ -546,6 +548,9 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
       const int c_hi = wr.cta_of(cur.pair * nblk + nblk - 1);
       if (c_lo == c_hi) {  // the whole pair was done here
         if (valid_row) {
+          if constexpr (kLse)
+            p.lse[(static_cast<size_t>(blockIdx.y) * p.heads + g * hpg + hl) * p.lse_pitch + r] =
+                (m_used + __log2f(l_run)) * 0.69314718055994531f;
           const float inv = 1.0f / l_run;
           uint4* dst = reinterpret_cast<uint4*>(out_row);
 #pragma unroll
@@ -614,6 +619,9 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
           }
         }
         const float inv = 1.0f / l;
+        if constexpr (kLse)
+          p.lse[(static_cast<size_t>(blockIdx.y) * p.heads + g * hpg + hl) * p.lse_pitch + r] =
+              (M + __log2f(l)) * 0.69314718055994531f;
         uint4* dst = reinterpret_cast<uint4*>(OUT_ROWS + static_cast<size_t>(r) * p.ld_out +
                                               (g * hpg + hl) * kHeadDim);
 #pragma unroll
@@ -658,9 +666,15 @@ cudaError_t launch_attention(const CUtensorMap& tmQ, const CUtensorMap& tmQ8,
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(attn_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                attn::kSmem);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(attn_kernel<true, true>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, attn::kSmem);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
+  if (p.streams != nullptr && p.lse != nullptr)
+    return launch_pdl(attn_kernel<true, true>, dim3(p.parts, p.n_streams), dim3(attn::kThreads),
+                      attn::kSmem, s, tmQ, tmQ8, tmK, tmVt, p);
   if (p.streams != nullptr)
     return launch_pdl(attn_kernel<true>, dim3(p.parts, p.n_streams), dim3(attn::kThreads),
                       attn::kSmem, s, tmQ, tmQ8, tmK, tmVt, p);

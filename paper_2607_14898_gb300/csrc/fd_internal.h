@@ -165,6 +165,10 @@ struct AttnParams {
   int n_streams;
   int q_rows_stream;
   size_t ws_stride;
+  // batched only, optional: each row's natural-log log-sum-exp of the scaled scores, at
+  // lse[(stream * heads + head) * lse_pitch + row] (the training step's backward)
+  float* lse;
+  int lse_pitch;
 };
 
 // launch wrappers; return cudaGetLastError() of the launch
@@ -245,6 +249,18 @@ void weights_add_user(fd_weights w, int delta);
 cudaError_t gemm_view(int epi, int M, int N, int K, const __nv_bfloat16* A, int lda,
                       const __nv_bfloat16* W, int ldw, const float* bias, float* out, int ldo,
                       int* err, cudaStream_t s);
+// Band attention of the training step on the batched attention kernel, one "stream" per query
+// chunk i: its keys are chunks max(0, i - W + 1) .. i of unpadded K bf16 [G][pitch][64] and
+// V^T fp16 [G][64][pitch] (rows_per_chunk keys per chunk), so stream i's maps start at key
+// max(0, i - W + 1) * rows_per_chunk and its key count is min(i + 1, W) rows_per_chunk with
+// steps_dev[i] = i. Fills host[0 .. T-1]; false if a map cannot be made (the V^T start must
+// be 16-byte aligned: rows_per_chunk % 8 == 0 unless T == 1).
+bool band_attention_maps(AttnStream* host, int T, int W, int rows_per_chunk, int G, int pitch,
+                         const __nv_bfloat16* k, const __half* vt, const int* steps_dev,
+                         int* err);
+// Q maps of the attention kernel over q bf16 [rows][heads 64]: boxes of 128 and of 8 rows
+bool attention_q_maps(CUtensorMap* q, CUtensorMap* q8, const __nv_bfloat16* base, int rows,
+                      int heads);
 
 // GEMM tile widths compiled in
 inline bool gemm_bn_supported(int bn) {

@@ -183,11 +183,15 @@ __device__ __forceinline__ void head_rms(float (&v)[kDh], const float* g, float 
 // q2 = RoPE(q0) (RMS with g2 first when qk_norm), k2 = RoPE(RMS(k0; gk)), v1 = RMS(v0; g2)
 // (v0 when qk_norm). Outputs: q2 bf16 head-major per chunk of Pc rows, [M / Pc][N][Pc][64]
 // (the rows of one chunk's heads of a KV group are then contiguous), k2 / v1 bf16 [G][M][64].
+// With qr non-null, also: q rows bf16 [M][N 64] (the attention kernel's layout), and the
+// real tokens' K bf16 [G][pitch][64] and V^T fp16 [G][64][pitch] without the padding rows
+// (chunk c's Lu = Pc / Lp * L keys at c Lu ...), the keys of the fused band attention.
 __global__ void qkv_fwd_kernel(const float* __restrict__ qkv, int M, int Pc, int Lp, int L,
                                int gw, int N, int G, int qk_norm, const float* __restrict__ gk,
                                const float* __restrict__ g2, float eps, Rope rp,
                                bf16* __restrict__ q2, bf16* __restrict__ k2,
-                               bf16* __restrict__ v1) {
+                               bf16* __restrict__ v1, bf16* __restrict__ qr,
+                               bf16* __restrict__ ku, __half* __restrict__ vtu, int pitch) {
   const int slots = N + 2 * G;
   const long long idx = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;
   if (idx >= static_cast<long long>(M) * slots) return;
@@ -216,6 +220,24 @@ __global__ void qkv_fwd_kernel(const float* __restrict__ qkv, int M, int Pc, int
   }
 #pragma unroll
   for (int j = 0; j < kDh; ++j) dst[j] = __float2bfloat16_rn(v[j]);
+  if (qr == nullptr) return;
+  if (is_q) {
+    bf16* d = qr + static_cast<size_t>(row) * N * kDh + slot * kDh;
+#pragma unroll
+    for (int j = 0; j < kDh; ++j) d[j] = __float2bfloat16_rn(v[j]);
+    return;
+  }
+  if (row % Lp >= L) return;  // padding rows are no keys
+  const int key = row / Pc * (Pc / Lp * L) + row % Pc / Lp * L + row % Lp;
+  if (is_k) {
+    bf16* d = ku + (static_cast<size_t>(slot - N) * pitch + key) * kDh;
+#pragma unroll
+    for (int j = 0; j < kDh; ++j) d[j] = __float2bfloat16_rn(v[j]);
+  } else {
+    __half* d = vtu + static_cast<size_t>(slot - N - G) * kDh * pitch + key;
+#pragma unroll
+    for (int j = 0; j < kDh; ++j) d[static_cast<size_t>(j) * pitch] = __float2half_rn(v[j]);
+  }
 }
 
 // RMS over one head, backward: x the pre-norm values, dy the gradient of the normed output
@@ -319,18 +341,19 @@ __global__ void softmax_lse_kernel(const float* __restrict__ S, int rows, int n,
   if (lane == 0) lse[row] = l;
 }
 
-// delta[(c N + h) Pc + l] = sum_j dO[c Pc + l][h 64 + j] O[((c N + h) Pc + l) 64 + j]: dO fp32
-// rows [M][N 64], O fp32 head-major [M / Pc][N][Pc][64]; one warp per (chunk, head, row)
-__global__ void delta_kernel(const float* __restrict__ dO, const float* __restrict__ O, int M,
+// delta[(c N + h) Pc + l] = sum_j dO[c Pc + l][h 64 + j] O[c Pc + l][h 64 + j]: dO fp32 and
+// O bf16, both rows [M][N 64]; one warp per (chunk, head, row)
+__global__ void delta_kernel(const float* __restrict__ dO, const bf16* __restrict__ O, int M,
                              int Pc, int N, float* __restrict__ delta) {
   const long long w = (blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (w >= static_cast<long long>(M) * N) return;
   const int c = static_cast<int>(w / (static_cast<long long>(N) * Pc));
   const int h = static_cast<int>(w / Pc % N), l = static_cast<int>(w % Pc);
-  const float* a = dO + (static_cast<size_t>(c) * Pc + l) * N * kDh + h * kDh;
-  const float* b = O + static_cast<size_t>(w) * kDh;
-  float v = a[lane] * b[lane] + a[lane + 32] * b[lane + 32];
+  const size_t e = (static_cast<size_t>(c) * Pc + l) * N * kDh + h * kDh;
+  const float* a = dO + e;
+  const bf16* b = O + e;
+  float v = a[lane] * __bfloat162float(b[lane]) + a[lane + 32] * __bfloat162float(b[lane + 32]);
   v = warp_sum(v);
   if (lane == 0) delta[w] = v;
 }
@@ -341,7 +364,7 @@ __global__ void delta_kernel(const float* __restrict__ dO, const float* __restri
 // [n][rows] (bf16) for the key-side products.
 __global__ void attn_grad_kernel(const float* __restrict__ S, const float* __restrict__ dP,
                                  const float* __restrict__ lse, const float* __restrict__ delta,
-                                 int rows, int n, float scale, int Lp, int L,
+                                 int rows, int n, float scale, int Pc, int Lp, int L,
                                  bf16* __restrict__ dS, bf16* __restrict__ dST,
                                  bf16* __restrict__ PT) {
   __shared__ bf16 tp[32][34], td[32][34];
@@ -353,7 +376,8 @@ __global__ void attn_grad_kernel(const float* __restrict__ S, const float* __res
     bf16 p16 = __float2bfloat16_rn(0.f), d16 = p16;
     if (r < rows && c < n) {
       const size_t e = static_cast<size_t>(r) * n + c;
-      const float p = valid ? expf(S[e] * scale - lse[r]) : 0.f;
+      // padding query rows (their dO is zero) take P = 0 as well
+      const float p = valid && r % Pc % Lp < L ? expf(S[e] * scale - lse[r]) : 0.f;
       d16 = __float2bfloat16_rn(p * (dP[e] - delta[r]) * scale);
       p16 = __float2bfloat16_rn(p);
       dS[e] = d16;
@@ -492,7 +516,22 @@ struct fd_trainer_s {
     int M, Pc;  // rows, rows per chunk
     std::vector<float*> h;  // block inputs (h[nblocks] = stack output), fp32 [M][D]
     std::vector<bf16*> u, q2, k2, v1, o, u2, a;
-    std::vector<float*> qkv, o32, hm, z, lse;  // o32 head-major, lse [M / Pc][N][Pc]
+    std::vector<float*> qkv, hm, z, lse;  // lse [M / Pc][N][Pc]
+    float* o32 = nullptr;  // head-major O of the materialised forward (scratch)
+    // the fused band attention of the forward (the decode's batched attention kernel, one
+    // stream per query chunk); off when its maps cannot be made
+    struct {
+      bool on = false;
+      bf16* qr = nullptr;      // q rows [M][N 64]
+      bf16* k = nullptr;       // K [G][pitch][64] of the real tokens
+      __half* vt = nullptr;    // V^T [G][64][pitch]
+      int pitch = 0, Lu = 0, parts = 1, pairs = 0;
+      fd::AttnStream* streams = nullptr;  // device [T]
+      int* steps = nullptr;               // device [T] = 0 .. T-1
+      float* ws = nullptr;                // [T][ws_stride] partial results and counters
+      size_t ws_stride = 0;
+      CUtensorMap tmQ, tmQ8;
+    } band;
   } sB, sR;
   // scratch
   bf16 *x0, *y16, *yh16, *a1, *vT, *kT, *do16, *dS, *P16, *dST, *PT, *QT, *dOT, *dy16, *dyT,
@@ -678,6 +717,29 @@ enum { kN1 = 0, kQW, kQB, kKG, kG2, kOW, kOB, kN2, kM1W, kM1B, kM2W, kM2B, kBloc
 void attn_fwd(Run& r, fd_trainer_s::Stack& st, int b) {
   fd_trainer_s* tr = r.tr;
   const int M = st.M, Pc = st.Pc, N = tr->N, hpg = N / tr->G, rows = tr->hs * Pc;
+  if (st.band.on) {
+    // the decode's batched attention kernel, one stream per query chunk: stream i's queries are
+    // its Pc rows (padding rows computed, not used), its keys the window's real tokens; O as
+    // bf16 rows into st.o, each row's log-sum-exp into st.lse
+    auto& bd = st.band;
+    fd::AttnParams a{};
+    a.Lq = Pc; a.heads = N; a.groups = tr->G; a.ring_pitch = bd.pitch;
+    a.rows_per_chunk = bd.Lu; a.window = tr->Wn; a.step_dev = bd.steps; a.n_keys_host = 0;
+    a.out = st.o[b]; a.ld_out = tr->NQ;
+    a.scale_log2 = static_cast<float>(1.4426950408889634 / 8.0);
+    a.err = tr->err;
+    a.lq_pad = fd::attention_lq_pad(Pc);
+    a.parts = bd.parts;
+    fd::attention_workspace_split(bd.ws, bd.parts, bd.pairs, a);
+    a.streams = bd.streams; a.n_streams = tr->T; a.q_rows_stream = Pc;
+    a.ws_stride = bd.ws_stride;
+    a.lse = st.lse[b]; a.lse_pitch = Pc;
+    if (r.begin(FD_TK_ATTN_GEMM)) {
+      r.check(fd::launch_attention(bd.tmQ, bd.tmQ8, bd.tmQ, bd.tmQ, a, r.s));
+      r.end();
+    }
+    return;
+  }
   // V^T [G][64][M] for the P V products
   for (int g = 0; g < tr->G; ++g)
     r.transpose(st.v1[b] + static_cast<size_t>(g) * M * 64, M, 64, 64,
@@ -697,8 +759,15 @@ void attn_fwd(Run& r, fd_trainer_s::Stack& st, int b) {
         r.end();
       }
       r.gemm(FD_TK_ATTN_GEMM, fd::EPI_F32, rows, 64, nk, tr->P16, nk,
-             tr->vT + static_cast<size_t>(g) * 64 * M + k0, M, nullptr, st.o32[b] + q0 * 64, 64);
+             tr->vT + static_cast<size_t>(g) * 64 * M + k0, M, nullptr, st.o32 + q0 * 64, 64);
     }
+  }
+  if (r.begin(FD_TK_POINTWISE)) {  // O rows (bf16) for the output projection
+    const long long n = static_cast<long long>(M) * tr->NQ;
+    fd::train::head_permute_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.o32, M, Pc, N, 1,
+                                                                         st.o[b]);
+    r.check(cudaGetLastError());
+    r.end();
   }
 }
 
@@ -723,7 +792,7 @@ void attn_bwd(Run& r, fd_trainer_s::Stack& st, int b) {
   }
   if (r.begin(FD_TK_SOFTMAX)) {
     const long long n = static_cast<long long>(M) * N * 32;
-    fd::train::delta_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(tr->gA, st.o32[b], M, Pc, N,
+    fd::train::delta_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(tr->gA, st.o[b], M, Pc, N,
                                                                   tr->delta);
     r.check(cudaGetLastError());
     r.end();
@@ -744,7 +813,7 @@ void attn_bwd(Run& r, fd_trainer_s::Stack& st, int b) {
       if (r.begin(FD_TK_SOFTMAX)) {
         const dim3 grid((nk + 31) / 32, (rows + 31) / 32);
         fd::train::attn_grad_kernel<<<grid, dim3(32, 8), 0, r.s>>>(
-            tr->S, tr->dP, st.lse[b] + q0, tr->delta + q0, rows, nk, 0.125f, tr->Lp, tr->L,
+            tr->S, tr->dP, st.lse[b] + q0, tr->delta + q0, rows, nk, 0.125f, Pc, tr->Lp, tr->L,
             tr->dS, tr->dST, tr->PT);
         r.check(cudaGetLastError());
         r.end();
@@ -775,18 +844,12 @@ void block_fwd(Run& r, fd_trainer_s::Stack& st, int b, size_t e0) {
     const long long n = static_cast<long long>(M) * (tr->N + 2 * tr->G);
     fd::train::qkv_fwd_kernel<<<blocks_for(n, 128), 128, 0, r.s>>>(
         st.qkv[b], M, st.Pc, tr->Lp, tr->L, tr->gw, tr->N, tr->G, tr->cfg.qk_norm, r.wf(e0 + kKG),
-        r.wf(e0 + kG2), tr->eps, rp, st.q2[b], st.k2[b], st.v1[b]);
+        r.wf(e0 + kG2), tr->eps, rp, st.q2[b], st.k2[b], st.v1[b], st.band.on ? st.band.qr : nullptr,
+        st.band.k, st.band.vt, st.band.pitch);
     r.check(cudaGetLastError());
     r.end();
   }
   attn_fwd(r, st, b);
-  if (r.begin(FD_TK_POINTWISE)) {  // O rows (bf16) for the output projection
-    const long long n = static_cast<long long>(M) * tr->NQ;
-    fd::train::head_permute_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.o32[b], M, st.Pc,
-                                                                         tr->N, 1, st.o[b]);
-    r.check(cudaGetLastError());
-    r.end();
-  }
   r.copy(st.hm[b], st.h[b], static_cast<size_t>(M) * tr->D);
   r.gemm(FD_TK_LINEAR, fd::EPI_RESID, M, tr->D, tr->NQ, st.o[b], tr->NQ, r.wb(e0 + kOW), tr->NQ,
          r.wf(e0 + kOB), st.hm[b], tr->D);
@@ -986,7 +1049,6 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
       st.q2.push_back(dalloc<bf16>(tr, static_cast<size_t>(M) * NQ, ok));
       st.k2.push_back(dalloc<bf16>(tr, static_cast<size_t>(G) * M * 64, ok));
       st.v1.push_back(dalloc<bf16>(tr, static_cast<size_t>(G) * M * 64, ok));
-      st.o32.push_back(dalloc<float>(tr, static_cast<size_t>(M) * NQ, ok));
       st.lse.push_back(dalloc<float>(tr, static_cast<size_t>(M) * tr->N, ok));
       st.o.push_back(dalloc<bf16>(tr, static_cast<size_t>(M) * NQ, ok));
       st.hm.push_back(dalloc<float>(tr, static_cast<size_t>(M) * D, ok));
@@ -997,6 +1059,48 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   };
   alloc_stack(tr->sB, MB, tr->Lp, tr->nb);
   alloc_stack(tr->sR, MR, tr->rt * tr->Lp, tr->nr);
+  // the forward's band attention: per stack, the query rows, unpadded K / V^T (allocated
+  // zeroed: keys past the clip read zeros), the kernel's per-chunk stream table and its
+  // workspace (counters zero); else the materialised forward with its head-major O scratch
+  int sms = 0, dev = 0;
+  if (ok) ok = cudaGetDevice(&dev) == cudaSuccess &&
+               cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess;
+  auto setup_band = [&](fd_trainer_s::Stack& st, int Lu) {
+    auto& bd = st.band;
+    const int T = tr->T, M = st.M;
+    bd.Lu = Lu;
+    bd.pitch = (T * Lu + 127) / 128 * 128;
+    bd.on = ok && (Lu % 8 == 0 || T == 1);
+    if (bd.on) {
+      bd.qr = dalloc<bf16>(tr, static_cast<size_t>(M) * NQ, ok);
+      bd.k = dalloc<bf16>(tr, static_cast<size_t>(G) * bd.pitch * 64, ok);
+      bd.vt = dalloc<__half>(tr, static_cast<size_t>(G) * 64 * bd.pitch, ok);
+      bd.steps = dalloc<int>(tr, T, ok);
+      bd.streams = dalloc<fd::AttnStream>(tr, T, ok);
+      const int keys = std::min(T, tr->Wn) * Lu;
+      bd.pairs = fd::attention_units(st.Pc, tr->N, G);
+      const long long units = static_cast<long long>(bd.pairs) * ((keys + 127) / 128);
+      bd.parts = static_cast<int>(std::max(1LL, std::min<long long>(std::max(1, sms / T), units)));
+      bd.ws_stride = (fd::attention_workspace_floats(bd.parts, bd.pairs) + 63) / 64 * 64;
+      bd.ws = dalloc<float>(tr, bd.ws_stride * T, ok);
+    }
+    if (bd.on && ok) {
+      std::vector<fd::AttnStream> host(T);
+      std::vector<int> steps(T);
+      for (int i = 0; i < T; ++i) steps[i] = i;
+      bd.on = fd::band_attention_maps(host.data(), T, tr->Wn, Lu, G, bd.pitch, bd.k, bd.vt,
+                                      bd.steps, tr->err) &&
+              fd::attention_q_maps(&bd.tmQ, &bd.tmQ8, bd.qr, M, tr->N);
+      if (bd.on)
+        ok = cudaMemcpy(bd.streams, host.data(), T * sizeof(fd::AttnStream),
+                        cudaMemcpyHostToDevice) == cudaSuccess &&
+             cudaMemcpy(bd.steps, steps.data(), T * sizeof(int), cudaMemcpyHostToDevice) ==
+                 cudaSuccess;
+    }
+    if (!bd.on) st.o32 = dalloc<float>(tr, static_cast<size_t>(M) * NQ, ok);
+  };
+  setup_band(tr->sB, tr->L);
+  setup_band(tr->sR, tr->rt * tr->L);
   const size_t wide = static_cast<size_t>(Mmax) *
                       std::max({D, Dm, QO, NQ, tr->rt * D, tr->Cr});
   tr->x0 = dalloc<bf16>(tr, static_cast<size_t>(MB) * tr->cin, ok);

@@ -1251,6 +1251,34 @@ void weights_add_user(fd_weights w, int delta) {
   if (w) w->live_handles += delta;
 }
 
+bool band_attention_maps(AttnStream* host, int T, int W, int rows_per_chunk, int G, int pitch,
+                         const __nv_bfloat16* k, const __half* vt, const int* steps_dev,
+                         int* err) {
+  for (int i = 0; i < T; ++i) {
+    const int j0 = i - W + 1 > 0 ? i - W + 1 : 0;
+    const uint64_t key0 = static_cast<uint64_t>(j0) * rows_per_chunk;
+    if ((key0 * 2) % 16 != 0 || key0 >= static_cast<uint64_t>(pitch)) return false;
+    // K rows g pitch + key of the window, from its first key on
+    if (!tmap_bf16(&host[i].k, k + key0 * kHeadDim, kHeadDim,
+                   static_cast<uint64_t>(G) * pitch - key0, kHeadDim * 2, 64, 128))
+      return false;
+    // V^T [G 64][pitch] from column key0 on (the row pitch stays pitch)
+    if (!tmap_f16(&host[i].vt, vt + key0, pitch - key0, static_cast<uint64_t>(G) * kHeadDim,
+                  static_cast<uint64_t>(pitch) * 2, 64, 64))
+      return false;
+    host[i].step_dev = steps_dev + i;
+    host[i].err = err;
+  }
+  return true;
+}
+
+bool attention_q_maps(CUtensorMap* q, CUtensorMap* q8, const __nv_bfloat16* base, int rows,
+                      int heads) {
+  const uint64_t NQ = static_cast<uint64_t>(heads) * kHeadDim;
+  return tmap_bf16(q, base, NQ, rows, NQ * 2, 64, 128) &&
+         tmap_bf16(q8, base, NQ, rows, NQ * 2, 64, 8);
+}
+
 cudaError_t gemm_view(int epi, int M, int N, int K, const __nv_bfloat16* A, int lda,
                       const __nv_bfloat16* W, int ldw, const float* bias, float* out, int ldo,
                       int* err, cudaStream_t s) {
