@@ -11,4 +11,11 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CU
   return launch_gemm_t<0>(tmA, tmB, tmO, tmK, tmV, p, bn, pair, num_sms, s);
 }
 
+// the scores-backward instance: tmA / tmB = Q / K, tmdO / tmV the second product's operands
+cudaError_t launch_gemm_scores_bwd(const CUtensorMap& tmA, const CUtensorMap& tmB,
+                                   const CUtensorMap& tmdO, const CUtensorMap& tmV,
+                                   const GemmParams& p, int num_sms, cudaStream_t s) {
+  return launch_bn<128, false, 0, true>(tmA, tmB, tmA, tmdO, tmV, p, num_sms, s);
+}
+
 }  // namespace fd

@@ -131,13 +131,22 @@ __device__ __forceinline__ void rope_table(const QkvEpi& q, const float2* rope_t
 }
 
 // QKV: 0 for every epilogue but EPI_QKV (no QKV code), 1 for EPI_QKV on one stream, 2 for
-// EPI_QKV on stacked streams (q.streams > 0)
-template <int BN, bool PAIR, int QKV>
+// EPI_QKV on stacked streams (q.streams > 0).
+// DS (single CTAs, K = 64): the attention's scores backward. Each tile holds two products, S =
+// Q K^T (tmA, tmB) and dP = dO V^T (tmK, tmV: A and B of the second product), one K block each,
+// in two TMEM accumulators; the epilogue turns them into dS = P (dP - delta) scale with P =
+// exp(S scale - lse) (p.ds), written as dS rows and dS^T, P^T columns (bf16). S and dP are never
+// stored.
+template <int BN, bool PAIR, int QKV, bool DS = false>
 __global__ void __launch_bounds__(192, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ GemmParams p) {
   using C = GemmCfg<BN, PAIR>;
+  // accumulator columns of one tile (DS: S and dP side by side), two tiles in flight
+  constexpr uint32_t kAccCols = DS ? 2 * BN : BN;
+  constexpr int kTmemCols = DS ? 4 * BN : C::kTmemCols;
+  static_assert(!DS || (!PAIR && QKV == 0 && 4 * BN <= 512), "scores backward: single CTAs");
   extern __shared__ __align__(1024) uint8_t smem[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -163,7 +172,7 @@ __global__ void __launch_bounds__(192, 1)
   const int cta0 = PAIR ? static_cast<int>(blockIdx.x) / 2 : static_cast<int>(blockIdx.x);
   const int ctas = PAIR ? static_cast<int>(gridDim.x) / 2 : static_cast<int>(gridDim.x);
   const int kel = p.fp8 ? 2 * kBK : kBK;  // K elements per 128-byte stage row
-  const int nk = (p.K + kel - 1) / kel;
+  const int nk = DS ? 2 : (p.K + kel - 1) / kel;  // DS: the two products' K blocks
   const uint32_t full_tx = PAIR ? 2 * C::kStageBytes : C::kStageBytes;  // on rank 0's barrier
   const uint32_t bar_full0 = PAIR ? mapa_rank(bar_full, 0) : bar_full;
   auto load = [&](uint32_t dst, const CUtensorMap* m, int s, int x, int y) {
@@ -203,10 +212,10 @@ __global__ void __launch_bounds__(192, 1)
   grid_dep_wait();  // inputs written by the previous kernel; TMEM freed by its CTAs
   if (warp == 1) {
     if (PAIR) {
-      tmem_alloc_pair(smem_u32(tmem_slot), C::kTmemCols);
+      tmem_alloc_pair(smem_u32(tmem_slot), kTmemCols);
       tmem_relinquish_pair();
     } else {
-      tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
+      tmem_alloc(smem_u32(tmem_slot), kTmemCols);
       tmem_relinquish();
     }
   }
@@ -231,6 +240,11 @@ __global__ void __launch_bounds__(192, 1)
         }
         if (!mbar_wait(bar_empty + 8 * s, ph ^ 1, p.err, ERR_WAIT_MMA)) { ok = false; break; }
         if (rank == 0) mbar_expect_tx(bar_full + 8 * s, full_tx);
+        if (DS) {  // block 0: Q and K; block 1: dO and V (K = 64, one block each)
+          load(sA + s * C::kABytes, kb == 0 ? &tmA : &tmK, s, 0, m0);
+          load(sB + s * C::kBBytes, kb == 0 ? &tmB : &tmV, s, 0, nb0);
+          continue;
+        }
         load(sA + s * C::kABytes, &tmA, s, kb * kel, m0);
         load(sB + s * C::kBBytes, &tmB, s, kb * kel, nb0);
       }
@@ -253,8 +267,11 @@ __global__ void __launch_bounds__(192, 1)
       const int acc = tc & 1;
       if (!mbar_wait(bar_tempty + 8 * acc, ((tc >> 1) & 1) ^ 1, p.err, ERR_WAIT_EPI)) break;
       tc_fence_after();
-      const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * BN);
+      const uint32_t d_acc = tmem + static_cast<uint32_t>(acc) * kAccCols;
       for (int kb = 0; kb < nk; ++kb, ++it) {
+        // DS: each K block is its own product, in its own accumulator
+        const uint32_t d_tmem = DS ? d_acc + static_cast<uint32_t>(kb) * BN : d_acc;
+        const int kacc = DS ? 0 : kb;  // accumulate over K blocks (DS: within the block only)
         const int s = it % C::kStages;
         if (!mbar_wait(bar_full + 8 * s, (it / C::kStages) & 1, p.err, ERR_WAIT_TMA)) {
           ok = false;
@@ -274,8 +291,8 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
             const uint64_t da = sdesc_k_sw128(a0 + 32 * k), db = sdesc_k_sw128(b0 + 32 * k);
-            if (PAIR) mma_bf16_ss_pair(d_tmem, da, db, idesc, (kb | k) != 0);
-            else mma_bf16_ss(d_tmem, da, db, idesc, (kb | k) != 0);
+            if (PAIR) mma_bf16_ss_pair(d_tmem, da, db, idesc, (kacc | k) != 0);
+            else mma_bf16_ss(d_tmem, da, db, idesc, (kacc | k) != 0);
           }
         }
         // stage s free (in both CTAs of a pair) once these MMAs have read it
@@ -327,10 +344,10 @@ __global__ void __launch_bounds__(192, 1)
       const int row = m0 + rloc;
       const bool row_ok = row < p.M;
       const uint32_t tbase =
-          tmem + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(acc * BN);
+          tmem + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(acc) * kAccCols;
       // The tile's bias (and column-scale) lines go into L1 while its MMAs still run, so the
       // per-chunk loads below do not each wait a round trip to L2 after the accumulator is ready.
-      if (lane < BN / 32 && n0 + 32 * lane < p.N) {
+      if (!DS && lane < BN / 32 && n0 + 32 * lane < p.N) {
         prefetch_l1(p.bias + n0 + 32 * lane);
         if (p.col_scale != nullptr) prefetch_l1(p.col_scale + n0 + 32 * lane);
       }
@@ -462,6 +479,48 @@ __global__ void __launch_bounds__(192, 1)
             for (int j = 0; j < 64; ++j)
               dst[static_cast<size_t>(j) * q.ring_pitch] = __float2half_rn(v[j]);
           }
+        }
+      } else if (DS) {
+        // scores backward of the tile: P = exp(S scale - lse) (0 on padding rows and keys),
+        // dS = P (dP - delta) scale; dS rows (4 x 16 B per thread and chunk), dS^T and P^T
+        // columns (one bf16 per lane and column: the warp's 32 rows are contiguous there)
+        const DsEpi& q = p.ds;
+        const bool live = row_ok && row % q.Pc % q.Lp < q.L;
+        const float lse = row_ok ? __ldg(q.lse + row) : 0.f;
+        const float dlt = row_ok ? __ldg(q.delta + row) : 0.f;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          const int col = n0 + c;
+          if (col >= p.N) break;  // N % 32 == 0
+          uint32_t rs[32], rp[32];
+          __syncwarp();
+          tmem_ld_32x32b_x32(tbase + c, rs);
+          tmem_ld_32x32b_x32(tbase + BN + c, rp);
+          tmem_ld_wait();
+          if (!row_ok) continue;
+          uint32_t dsw[16];
+#pragma unroll
+          for (int j = 0; j < 32; j += 2) {
+            float pj[2], dj[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const bool key = (col + j + e) % q.Lp < q.L;
+              pj[e] = live && key ? expf(__uint_as_float(rs[j + e]) * q.scale - lse) : 0.f;
+              dj[e] = pj[e] * (__uint_as_float(rp[j + e]) - dlt) * q.scale;
+            }
+            dsw[j / 2] = pack_bf16x2(dj[0], dj[1]);
+            const __nv_bfloat162 pb = __floats2bfloat162_rn(pj[0], pj[1]);
+            const __nv_bfloat162 db = __floats2bfloat162_rn(dj[0], dj[1]);
+            const size_t t0 = static_cast<size_t>(col + j) * p.M + row;
+            q.PT[t0] = pb.x;
+            q.PT[t0 + p.M] = pb.y;
+            q.dST[t0] = db.x;
+            q.dST[t0 + p.M] = db.y;
+          }
+          uint4* d = reinterpret_cast<uint4*>(q.dS + static_cast<size_t>(row) * p.N + col);
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            d[k] = make_uint4(dsw[4 * k], dsw[4 * k + 1], dsw[4 * k + 2], dsw[4 * k + 3]);
         }
       } else if (p.epi == EPI_GELU) {
 #pragma unroll 1
@@ -699,19 +758,19 @@ __global__ void __launch_bounds__(192, 1)
   else __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    if (PAIR) tmem_dealloc_pair(tmem, C::kTmemCols);
-    else tmem_dealloc(tmem, C::kTmemCols);
+    if (PAIR) tmem_dealloc_pair(tmem, kTmemCols);
+    else tmem_dealloc(tmem, kTmemCols);
   }
 }
 
-template <int BN, bool PAIR, int QKV>
+template <int BN, bool PAIR, int QKV, bool DS = false>
 static cudaError_t launch_bn(const CUtensorMap& tmA, const CUtensorMap& tmB,
                              const CUtensorMap& tmO, const CUtensorMap& tmK,
                              const CUtensorMap& tmV, const GemmParams& p, int num_sms,
                              cudaStream_t s) {
   using C = GemmCfg<BN, PAIR>;
   static const cudaError_t attr = cudaFuncSetAttribute(
-      gemm_kernel<BN, PAIR, QKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+      gemm_kernel<BN, PAIR, QKV, DS>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
   if (attr != cudaSuccess) return attr;
   const int rows = PAIR ? 2 * kBM : kBM;
   const int tiles = ((p.M + rows - 1) / rows) * ((p.N + BN - 1) / BN);
@@ -744,7 +803,7 @@ static cudaError_t launch_bn(const CUtensorMap& tmA, const CUtensorMap& tmB,
   }
   const int units = tiles < slots ? tiles : slots;
   cfg.gridDim = dim3(PAIR ? 2 * units : units);
-  return cudaLaunchKernelEx(&cfg, gemm_kernel<BN, PAIR, QKV>, tmA, tmB, tmO, tmK, tmV, p);
+  return cudaLaunchKernelEx(&cfg, gemm_kernel<BN, PAIR, QKV, DS>, tmA, tmB, tmO, tmK, tmV, p);
 }
 
 template <int QKV>

@@ -50,6 +50,17 @@ enum EpiKind : int {
                   // [-1, 1] as fp32 or as its uint8 code; frames past pix.frames are not written
 };
 
+// The scores-backward GEMM (attention training): rows r of S / dP are (head, query) rows of
+// one query chunk, Pc rows per head (padding rows r % Pc % Lp >= L), columns keys (padding keys
+// c % Lp >= L); dS bf16 [M][N]; dS^T, P^T bf16 [N][M].
+struct DsEpi {
+  const float* lse;    // [M] log-sum-exp of the row's scaled scores (natural log)
+  const float* delta;  // [M] rowsum(dO o O)
+  float scale;         // 1 / sqrt(D_h)
+  int Pc, Lp, L;
+  __nv_bfloat16 *dS, *dST, *PT;
+};
+
 // Output of EPI_PIXEL (the pixel head folded into the last product of the decoder).
 struct PixelEpi {
   void* out;        // [C][frames][gh rs][gw rs], fp32 or uint8
@@ -126,6 +137,7 @@ struct GemmParams {
   // load before the dependency on the previous kernel is resolved
   int w_static;
   PixelEpi pix;  // EPI_PIXEL
+  DsEpi ds;      // the scores-backward instance
 };
 // EPI_PIXEL is compiled into the single-CTA 256-wide instance only
 inline bool gemm_pixel_epilogue_ok(int bn, bool pair, int rs) {
@@ -177,6 +189,10 @@ struct AttnParams {
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmO,
                         const CUtensorMap& tmK, const CUtensorMap& tmV, const GemmParams& p,
                         int bn, bool pair, int num_sms, cudaStream_t s);
+// the scores-backward instance (DS): S = Q K^T (tmA, tmB) and dP = dO V^T (tmdO, tmV), K = 64
+cudaError_t launch_gemm_scores_bwd(const CUtensorMap& tmA, const CUtensorMap& tmB,
+                                   const CUtensorMap& tmdO, const CUtensorMap& tmV,
+                                   const GemmParams& p, int num_sms, cudaStream_t s);
 // the EPI_QKV instances (launch_gemm forwards to it for that epilogue)
 cudaError_t launch_gemm_qkv(const CUtensorMap& tmA, const CUtensorMap& tmB,
                             const CUtensorMap& tmO, const CUtensorMap& tmK,
@@ -249,6 +265,12 @@ void weights_add_user(fd_weights w, int delta);
 cudaError_t gemm_view(int epi, int M, int N, int K, const __nv_bfloat16* A, int lda,
                       const __nv_bfloat16* W, int ldw, const float* bias, float* out, int ldo,
                       int* err, cudaStream_t s);
+// The attention's scores backward in one launch (the DS GEMM instance, 128 x 128 tiles):
+// S = Q K^T and dP = dO V^T (Q, dO bf16 [M][64] with row pitch ldq; K, V bf16 [N][64] with row
+// pitch ldk), then dS, dS^T, P^T as DsEpi describes. N % 32 == 0.
+cudaError_t scores_bwd(int M, int N, const __nv_bfloat16* Q, const __nv_bfloat16* dO, int ldq,
+                       const __nv_bfloat16* K, const __nv_bfloat16* V, int ldk, const DsEpi& ds,
+                       int* err, cudaStream_t s);
 // Band attention of the training step on the batched attention kernel, one "stream" per query
 // chunk i: its keys are chunks max(0, i - W + 1) .. i of unpadded K bf16 [G][pitch][64] and
 // V^T fp16 [G][64][pitch] (rows_per_chunk keys per chunk), so stream i's maps start at key

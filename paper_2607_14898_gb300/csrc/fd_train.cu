@@ -358,44 +358,6 @@ __global__ void delta_kernel(const float* __restrict__ dO, const bf16* __restric
   if (lane == 0) delta[w] = v;
 }
 
-// Softmax backward of one (query chunk, KV group), one 32 x 32 tile per block: with P = exp(S
-// scale - lse) on the valid columns, dS = P (dP - delta) scale (the scale of the scores folded
-// in: dQ = dS K, dK = dS^T Q). Writes dS [rows][n] and, through the tile, dS^T and P^T
-// [n][rows] (bf16) for the key-side products.
-__global__ void attn_grad_kernel(const float* __restrict__ S, const float* __restrict__ dP,
-                                 const float* __restrict__ lse, const float* __restrict__ delta,
-                                 int rows, int n, float scale, int Pc, int Lp, int L,
-                                 bf16* __restrict__ dS, bf16* __restrict__ dST,
-                                 bf16* __restrict__ PT) {
-  __shared__ bf16 tp[32][34], td[32][34];
-  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
-  const int c = c0 + threadIdx.x;
-  const bool valid = c < n && c % Lp < L;
-  for (int i = threadIdx.y; i < 32; i += 8) {
-    const int r = r0 + i;
-    bf16 p16 = __float2bfloat16_rn(0.f), d16 = p16;
-    if (r < rows && c < n) {
-      const size_t e = static_cast<size_t>(r) * n + c;
-      // padding query rows (their dO is zero) take P = 0 as well
-      const float p = valid && r % Pc % Lp < L ? expf(S[e] * scale - lse[r]) : 0.f;
-      d16 = __float2bfloat16_rn(p * (dP[e] - delta[r]) * scale);
-      p16 = __float2bfloat16_rn(p);
-      dS[e] = d16;
-    }
-    tp[i][threadIdx.x] = p16;
-    td[i][threadIdx.x] = d16;
-  }
-  __syncthreads();
-  for (int i = threadIdx.y; i < 32; i += 8) {
-    const int cc = c0 + i, r = r0 + threadIdx.x;
-    if (cc < n && r < rows) {
-      const size_t e = static_cast<size_t>(cc) * rows + r;
-      PT[e] = tp[threadIdx.x][i];
-      dST[e] = td[threadIdx.x][i];
-    }
-  }
-}
-
 // head-major [M / Pc][N][Pc][64] fp32 <-> rows [M][N 64]: to_rows = 1 reads head-major x and
 // writes bf16 rows; to_rows = 0 reads fp32 rows and writes bf16 head-major
 __global__ void head_permute_kernel(const float* __restrict__ x, int M, int Pc, int N,
@@ -454,12 +416,21 @@ __global__ void l1_head_kernel(const float* __restrict__ F, const float* __restr
   if (threadIdx.x == 0) part[blockIdx.x] = red[0];
 }
 
+// one block of kLossThreads: thread t sums parts t, t + kLossThreads, ... in fp64, then a
+// fixed-order tree over the threads (the same bits every step)
+constexpr int kLossThreads = 1024;
 __global__ void finish_loss_kernel(const float* __restrict__ part, int n, float inv_total,
                                    float* __restrict__ loss) {
-  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+  __shared__ double acc[kLossThreads];
   double s = 0.0;
-  for (int i = 0; i < n; ++i) s += part[i];
-  *loss = static_cast<float>(s * inv_total);
+  for (int i = threadIdx.x; i < n; i += kLossThreads) s += part[i];
+  acc[threadIdx.x] = s;
+  __syncthreads();
+  for (int w = kLossThreads / 2; w > 0; w >>= 1) {
+    if (static_cast<int>(threadIdx.x) < w) acc[threadIdx.x] += acc[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *loss = static_cast<float>(acc[0] * inv_total);
 }
 
 // temporal upsampling layout (Eq. temporal_upsample, reading R6): channel block tau of token
@@ -536,7 +507,7 @@ struct fd_trainer_s {
   // scratch
   bf16 *x0, *y16, *yh16, *a1, *vT, *kT, *do16, *dS, *P16, *dST, *PT, *QT, *dOT, *dy16, *dyT,
       *xT, *dqkv16;
-  float *e, *z1, *F, *dF, *loss_part, *S, *dP, *delta, *dq2, *dk2, *dv1, *dqkv, *tq, *tk,
+  float *e, *z1, *F, *dF, *loss_part, *S, *delta, *dq2, *dk2, *dv1, *dqkv, *tq, *tk,
       *tv, *gA, *gB, *gC, *tbuf, *gtmp;
   int loss_blocks = 0;
   int hs = 1;  // heads of one KV group per attention product (a divisor of N / G)
@@ -805,17 +776,14 @@ void attn_bwd(Run& r, fd_trainer_s::Stack& st, int b) {
       const size_t q0 = (static_cast<size_t>(i) * N + h0) * Pc;
       const bf16* Kw = st.k2[b] + (static_cast<size_t>(g) * M + k0) * 64;
       const bf16* Vw = st.v1[b] + (static_cast<size_t>(g) * M + k0) * 64;
-      // S recomputed, dP = dO V^T
-      r.gemm(FD_TK_ATTN_GEMM, fd::EPI_F32, rows, nk, 64, st.q2[b] + q0 * 64, 64, Kw, 64,
-             nullptr, tr->S, nk);
-      r.gemm(FD_TK_ATTN_GEMM, fd::EPI_F32, rows, nk, 64, tr->do16 + q0 * 64, 64, Vw, 64,
-             nullptr, tr->dP, nk);
-      if (r.begin(FD_TK_SOFTMAX)) {
-        const dim3 grid((nk + 31) / 32, (rows + 31) / 32);
-        fd::train::attn_grad_kernel<<<grid, dim3(32, 8), 0, r.s>>>(
-            tr->S, tr->dP, st.lse[b] + q0, tr->delta + q0, rows, nk, 0.125f, Pc, tr->Lp, tr->L,
-            tr->dS, tr->dST, tr->PT);
-        r.check(cudaGetLastError());
+      // S = Q K^T (recomputed) and dP = dO V^T in one launch, the softmax backward in its
+      // epilogue: dS = P (dP - delta) / sqrt(D_h) with P = exp(S / sqrt(D_h) - lse), written as
+      // dS, dS^T and P^T; S and dP are never stored
+      if (r.begin(FD_TK_ATTN_GEMM)) {
+        const fd::DsEpi ds{st.lse[b] + q0, tr->delta + q0, 0.125f, Pc, tr->Lp, tr->L,
+                           tr->dS, tr->dST, tr->PT};
+        r.check(fd::scores_bwd(rows, nk, st.q2[b] + q0 * 64, tr->do16 + q0 * 64, 64, Kw, Vw, 64,
+                               ds, tr->err, r.s));
         r.end();
       }
       // dQ = dS K
@@ -1111,7 +1079,9 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   tr->kT = dalloc<bf16>(tr, static_cast<size_t>(G) * 64 * Mmax, ok);
   tr->do16 = dalloc<bf16>(tr, static_cast<size_t>(Mmax) * NQ, ok);
   tr->dS = dalloc<bf16>(tr, RK, ok);
-  tr->P16 = dalloc<bf16>(tr, RK, ok);
+  // S and P of the materialised forward (a stack whose band attention is off)
+  const bool materialised = !tr->sB.band.on || !tr->sR.band.on;
+  if (materialised) tr->P16 = dalloc<bf16>(tr, RK, ok);
   tr->dST = dalloc<bf16>(tr, RK, ok);
   tr->PT = dalloc<bf16>(tr, RK, ok);
   tr->QT = dalloc<bf16>(tr, static_cast<size_t>(64) * tr->hs * Pmax, ok);
@@ -1126,8 +1096,7 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   tr->dF = dalloc<float>(tr, static_cast<size_t>(MR) * tr->Cr, ok);
   tr->loss_blocks = static_cast<int>((static_cast<long long>(MR) * tr->Cr + 255) / 256);
   tr->loss_part = dalloc<float>(tr, tr->loss_blocks, ok);
-  tr->S = dalloc<float>(tr, RK, ok);
-  tr->dP = dalloc<float>(tr, RK, ok);
+  if (materialised) tr->S = dalloc<float>(tr, RK, ok);
   tr->delta = dalloc<float>(tr, static_cast<size_t>(Mmax) * tr->N, ok);
   {
     const size_t R = fd::train::kColsumRows;
@@ -1247,7 +1216,8 @@ fd_status fd_train_step(fd_trainer tr, const float* latents, const float* target
     r.end();
   }
   if (r.begin(FD_TK_POINTWISE)) {
-    fd::train::finish_loss_kernel<<<1, 32, 0, r.s>>>(tr->loss_part, tr->loss_blocks, inv_total,
+    fd::train::finish_loss_kernel<<<1, fd::train::kLossThreads, 0, r.s>>>(tr->loss_part,
+                                                                         tr->loss_blocks, inv_total,
                                                      loss);
     r.check(cudaGetLastError());
     r.end();
@@ -1331,7 +1301,8 @@ fd_status fd_op_l1_pixel_bwd(const float* F, const float* target, int frames, in
   fd::train::l1_head_kernel<<<blocks, 256, 0, s>>>(F, target, 1, frames, L, L, grid_h, grid_w,
                                                    channels, rs, inv_total, dF, work);
   if (cudaGetLastError() != cudaSuccess) return FD_ERR_CUDA;
-  fd::train::finish_loss_kernel<<<1, 32, 0, s>>>(work, blocks, inv_total, loss);
+  fd::train::finish_loss_kernel<<<1, fd::train::kLossThreads, 0, s>>>(work, blocks, inv_total,
+                                                                       loss);
   return cudaGetLastError() == cudaSuccess ? FD_OK : FD_ERR_CUDA;
 }
 

@@ -307,8 +307,9 @@ int pick_bn_step(int M, int N, int step, bool narrow_on_ties = false) {
   const int sms = num_sms();
   int best = 128;
   long long best_cost = -1;
-  for (int bn : {96, 128, 192, 256}) {
+  for (int bn : {64, 96, 128, 192, 256}) {
     if (bn % step) continue;
+    if (bn == 64 && N > 64) continue;  // 64-wide tiles only for products that narrow
     const long long tiles = static_cast<long long>((M + 127) / 128) * ((N + bn - 1) / bn);
     const long long rounds = (tiles + sms - 1) / sms;
     const long long cost = rounds * (128 + bn);
@@ -1249,6 +1250,22 @@ size_t weights_entries(fd_weights w, const void** ptrs, size_t n) {
 
 void weights_add_user(fd_weights w, int delta) {
   if (w) w->live_handles += delta;
+}
+
+cudaError_t scores_bwd(int M, int N, const __nv_bfloat16* Q, const __nv_bfloat16* dO, int ldq,
+                       const __nv_bfloat16* K, const __nv_bfloat16* V, int ldk, const DsEpi& ds,
+                       int* err, cudaStream_t s) {
+  if (M < 1 || N < 32 || N % 32 || ldq % 8 || ldk % 8) return cudaErrorInvalidValue;
+  CUtensorMap tq, tdo, tk, tv;
+  if (!tmap_bf16(&tq, Q, kHeadDim, M, static_cast<uint64_t>(ldq) * 2, 64, 128) ||
+      !tmap_bf16(&tdo, dO, kHeadDim, M, static_cast<uint64_t>(ldq) * 2, 64, 128) ||
+      !tmap_bf16(&tk, K, kHeadDim, N, static_cast<uint64_t>(ldk) * 2, 64, 128) ||
+      !tmap_bf16(&tv, V, kHeadDim, N, static_cast<uint64_t>(ldk) * 2, 64, 128))
+    return cudaErrorInvalidValue;
+  GemmParams p{};
+  p.M = M; p.N = N; p.K = kHeadDim; p.epi = EPI_F32; p.err = err;
+  p.ds = ds;
+  return launch_gemm_scores_bwd(tq, tk, tdo, tv, p, num_sms(), s);
 }
 
 bool band_attention_maps(AttnStream* host, int T, int W, int rows_per_chunk, int G, int pitch,
