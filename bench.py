@@ -42,6 +42,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-secondary", action="store_true", help="skip the 720p line")
     ap.add_argument("--no-training", action="store_true", help="skip the training-step line")
+    ap.add_argument("--training-only", action="store_true",
+                    help="run only the training-step line (one GPU; for profiling it alone)")
     return ap.parse_args()
 
 
@@ -667,6 +669,18 @@ def main():
         if rank != 0:
             return
         print(json.dumps(run_reference(args)), flush=True)
+        return
+    if args.training_only:
+        import torch
+
+        import synth
+        from paper_2607_14898_gb300 import flashdec as fdp
+        cfg = synth.PRESETS["480p"]
+        torch.cuda.set_device(0)
+        stream = torch.cuda.Stream()
+        line = {"training": training_line(args, stream,
+                                          fdp.pack_blob(cfg, synth.make_weights(cfg)))}
+        print(json.dumps(line), flush=True)
         return
     line = run_ours(args, rank, world)
     if rank == 0:

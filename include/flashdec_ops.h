@@ -174,6 +174,17 @@ fd_status fd_op_linear_pixel(int M, int K, const void* A, const void* W, const f
 
 /* ---- single kernels of the training step (fd_train_step), for per-kernel checks ---- */
 
+/* The attention's scores backward in one launch (the training step's, Sec. 3.3 attention with
+ * its softmax derivative): S = Q K^T and dP = dO V^T on the tensor cores (never stored), then
+ *   P = exp(S / sqrt(64) - lse[r]), dS = P (dP - delta[r]) / sqrt(64)
+ * with P = 0 on padding query rows (r mod Pc mod Lp >= L) and padding keys (c mod Lp >= L),
+ * written as dS bf16 [M][N], dS^T and P^T bf16 [N][M]. Q, dO bf16 [M][64]; K, V bf16 [N][64];
+ * lse, delta fp32 [M]. N % 32 == 0, Pc % Lp == 0, 0 < L <= Lp; 16-byte aligned.
+ * Errors: FD_ERR_INVALID_ARG, FD_ERR_CUDA; err_dev as for fd_op_linear. */
+fd_status fd_op_scores_bwd(int M, int N, const void* Q, const void* dO, const void* K,
+                           const void* V, const float* lse, const float* delta, int Pc, int Lp,
+                           int L, void* dS, void* dST, void* PT, int* err_dev, void* stream);
+
 /* RMSNorm backward (the derivative of y = x r g, r = (mean(x^2) + eps)^(-1/2), Sec. 3.2):
  * dx = r (dy g) - x r^3 sum_j(dy_j g_j x_j) / D and dg = sum over rows of dy x r.
  * x, dy, dx fp32 [M][D]; g, dg fp32 [D]; work: fp32 [M][D] scratch of the caller. */

@@ -1266,6 +1266,24 @@ fd_status fd_train_step(fd_trainer tr, const float* latents, const float* target
 }
 
 // ---- single kernels of the step, for per-kernel checks (include/flashdec_ops.h)
+fd_status fd_op_scores_bwd(int M, int N, const void* Q, const void* dO, const void* K,
+                           const void* V, const float* lse, const float* delta, int Pc, int Lp,
+                           int L, void* dS, void* dST, void* PT, int* err_dev, void* stream) {
+  if (!Q || !dO || !K || !V || !lse || !delta || !dS || !dST || !PT || !err_dev || M < 1 ||
+      N < 32 || N % 32 || Lp < 1 || Pc < Lp || Pc % Lp || L < 1 || L > Lp)
+    return FD_ERR_INVALID_ARG;
+  const void* const ptrs[7] = {Q, dO, K, V, dS, dST, PT};
+  for (const void* ptr : ptrs)
+    if (reinterpret_cast<uintptr_t>(ptr) & 15u) return FD_ERR_INVALID_ARG;
+  const fd::DsEpi ds{lse, delta, 0.125f, Pc, Lp, L, static_cast<bf16*>(dS),
+                     static_cast<bf16*>(dST), static_cast<bf16*>(PT)};
+  const cudaError_t e = fd::scores_bwd(M, N, static_cast<const bf16*>(Q),
+                                       static_cast<const bf16*>(dO), 64,
+                                       static_cast<const bf16*>(K), static_cast<const bf16*>(V),
+                                       64, ds, err_dev, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FD_OK : FD_ERR_CUDA;
+}
+
 fd_status fd_op_rmsnorm_bwd(const float* x, const float* g, const float* dy, int M, int D,
                             float eps, float* dx, float* dg, float* work, void* stream) {
   if (!x || !g || !dy || !dx || !dg || !work || M < 1 || D < 1 || D > 65536)

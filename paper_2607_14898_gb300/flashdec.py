@@ -83,6 +83,7 @@ _SIGS = {
     "fd_train_grad_elems": (ctypes.c_size_t, [ctypes.POINTER(fd_config)]),
     "fd_op_linear_pixel": (_I, [_I, _I, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P]),
     "fd_op_rmsnorm_bwd": (_I, [_P, _P, _P, _I, _I, _F, _P, _P, _P, _P]),
+    "fd_op_scores_bwd": (_I, [_I, _I, _P, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P]),
     "fd_op_gelu_bwd": (_I, [_P, _P, ctypes.c_int64, _P, _P, _P]),
     "fd_op_l1_pixel_bwd": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P]),
     "fd_train_create": (_I, [ctypes.POINTER(fd_config), _P, _I, ctypes.POINTER(_P)]),
@@ -563,6 +564,15 @@ def op_linear_pixel(A, W, bias, frames, grid_h, grid_w, channels, rs, out_dtype,
     _check(lib().fd_op_linear_pixel(M, K, _ptr(A), _ptr(W), _ptr(bias), frames, grid_h, grid_w,
                                     channels, rs, out_dtype, _ptr(pixels), _ptr(err),
                                     _stream_ptr(stream)), "fd_op_linear_pixel")
+
+
+def op_scores_bwd(Q, dO, K, V, lse, delta, Pc, Lp, L, dS, dST, PT, err=None,
+                  stream=None) -> None:
+    """The attention's scores backward in one launch (fd_op_scores_bwd)."""
+    M, N = Q.shape[0], K.shape[0]
+    _check(lib().fd_op_scores_bwd(M, N, _ptr(Q), _ptr(dO), _ptr(K), _ptr(V), _ptr(lse),
+                                  _ptr(delta), Pc, Lp, L, _ptr(dS), _ptr(dST), _ptr(PT), _ptr(err),
+                                  _stream_ptr(stream)), "fd_op_scores_bwd")
 
 
 def op_rmsnorm_bwd(x, g, dy, eps, dx, dg, stream=None) -> None:

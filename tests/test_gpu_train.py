@@ -10,6 +10,7 @@ import torch
 import oracle
 import synth
 from oracle.backward import training_step_explicit
+import oracle.backward as oracle_bwd
 
 pytestmark = pytest.mark.gpu
 
@@ -157,6 +158,59 @@ def test_l1_pixel_backward_kernel():
     want_dF = pixel_shuffle_bwd(l1_bwd(pix, x, total), frames, gh, gw, C, rs)
     assert abs(float(loss.item()) - want_loss) <= 1e-6 * want_loss
     assert float((dF.cpu().double() - want_dF).abs().max()) <= 1e-7 / total
+
+
+@pytest.mark.parametrize("heads,Pc,Lp,L,N", [
+    (2, 256, 128, 100, 384),   # padding query rows and padding keys, ragged 128-row tiles
+    (4, 128, 128, 128, 256),   # no padding (the 480p backbone's heads of one group, shrunk)
+    (1, 384, 384, 360, 1152),  # one head, three chunks of keys
+])
+def test_scores_backward_kernel(heads, Pc, Lp, L, N):
+    """fd_op_scores_bwd (S and dP on the tensor cores, the softmax derivative in the epilogue)
+    against oracle.attention_bwd: its dS, dS^T and P^T chained through fp64 products (dQ = dS K,
+    dK = dS^T Q, dV = P^T dO) give the oracle's gradients of one KV group, with the log-sum-exp
+    and delta of an fp64 forward. Padding query rows carry dO = 0, as in the step."""
+    from helpers import bf16_values, randn
+    M = heads * Pc
+    rows = torch.arange(M)
+    live = (rows % Pc % Lp) < L
+    keys = (torch.arange(N) % Lp) < L
+    q = torch.from_numpy(bf16_values(randn((M, 64), M + N, 1.0))).double()
+    k = torch.from_numpy(bf16_values(randn((N, 64), M + N + 1, 1.0))).double()
+    v = torch.from_numpy(bf16_values(randn((N, 64), M + N + 2, 1.0))).double()
+    do = torch.from_numpy(bf16_values(randn((M, 64), M + N + 3, 1.0))).double()
+    do[~live] = 0.0
+    # the forward's log-sum-exp and delta = rowsum(dO o O), from their definitions in fp64
+    s = (q @ k.T) / 8.0
+    s[:, ~keys] = float("-inf")
+    lse = torch.logsumexp(s, dim=1)
+    o = torch.softmax(s, dim=1) @ v
+    delta = (do * o).sum(dim=1)
+    cu = lambda t: t.to(torch.bfloat16).cuda()
+    dS = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    dST = torch.empty(N, M, dtype=torch.bfloat16, device="cuda")
+    PT = torch.empty(N, M, dtype=torch.bfloat16, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    fdp.op_scores_bwd(cu(q), cu(do), cu(k), cu(v), lse.float().cuda(), delta.float().cuda(), Pc,
+                      Lp, L, dS, dST, PT, err=err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    assert torch.equal(dST.cpu(), dS.cpu().T.contiguous())
+    dS, PT = dS.cpu().double(), PT.cpu().double()
+    assert float(dS[~live].abs().sum()) == 0.0 and float(PT[:, ~live].abs().sum()) == 0.0
+    assert float(PT[~keys].abs().sum()) == 0.0  # padding rows and keys: P = dS = 0
+    # the oracle's gradients of the group (its heads as query heads over one KV group)
+    allowed = keys[None, :].expand(Pc, N)
+    dq, dk, dv = oracle_bwd.attention_bwd(q.reshape(heads, Pc, 64), k[None], v[None],
+                                          do.reshape(heads, Pc, 64), allowed)
+    got = {"dq": (dS @ k).reshape(heads, Pc, 64), "dk": dS.T @ q, "dv": PT @ do}
+    want = {"dq": dq, "dk": dk[0], "dv": dv[0]}
+    for name in got:
+        w = want[name].clone()
+        if name == "dq":
+            w[~live.reshape(heads, Pc)] = 0.0
+        rel = float((got[name] - w).norm() / w.norm())
+        assert rel < 1e-2, (name, rel)
 
 
 def test_training_profile_counts_every_kind():
