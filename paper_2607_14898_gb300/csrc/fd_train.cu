@@ -5,15 +5,21 @@
 // Training through the rolling cache has the gradient of one pass over the whole clip under
 // the block sliding-window mask (query chunk i sees key chunks i-W < j <= i), so the GPU runs
 // all T chunks at once: the forward of every block with its activations kept, the L1 term of
-// the pixels, then the backward block by block in reverse. Every product is the library's
-// tcgen05 GEMM (gemm_view) on bf16 operands with fp32 accumulation: the linear layers, their
-// input gradients dX = dY W (with the transposed weights) and weight gradients dW = dY^T X
-// (with transposed activations), and the attention of each (query chunk, head) over its band
-// of key chunks: S = Q K^T, O = P V, and in the backward dP = dO V^T, dQ = dS K, dK += dS^T Q,
-// dV += P^T dO, with P recomputed. Row-wise and element-wise steps (RMSNorm and its backward,
-// KV-norm / QK-norm with 3D-RoPE and their backward, GELU and GELU', the band softmax and
-// dS = P (dP - rowsum(dO O)), the L1 term through the pixel shuffle, bias and gain sums) are
-// the kernels below.
+// the pixels, then the backward block by block in reverse. Every product runs on the tensor
+// cores with bf16 operands and fp32 accumulation:
+//   - the linear layers, their input gradients dX = dY W (with the transposed weights) and
+//     weight gradients dW = dY^T X (with transposed activations): the library's GEMM
+//     (gemm_view);
+//   - the attention forward: the decode's batched attention kernel with one stream per query
+//     chunk over the window of its key chunks, writing each row's log-sum-exp (attn_fwd);
+//   - the attention backward per (query chunk, KV group): one launch for S = Q K^T and
+//     dP = dO V^T with the softmax derivative dS = P (dP - rowsum(dO O)) in its epilogue
+//     (scores_bwd: S and dP stay in tensor memory), then dQ = dS K, dK += dS^T Q, dV += P^T dO
+//     on the GEMM (attn_bwd).
+// Row-wise and element-wise steps (RMSNorm and its backward, KV-norm / QK-norm with 3D-RoPE and
+// their backward, GELU and GELU', rowsum(dO O), the L1 term through the pixel shuffle, bias and
+// gain sums) are the kernels below. Where a stack's keys per chunk are not a multiple of 8, its
+// attention forward is materialised instead (S, the band softmax, O = P V).
 //
 // Rows: chunk c's L tokens sit at rows c Lp .. c Lp + L - 1 with Lp = 128 ceil(L / 128), the
 // refined frame (c, tau) at rows (c r_t + tau) Lp ...; padding rows carry finite values
@@ -680,11 +686,13 @@ struct Run {
 // (vnorm|qnorm).g, out.w, out.b, norm2.g, mlp1.w, mlp1.b, mlp2.w, mlp2.b
 enum { kN1 = 0, kQW, kQB, kKG, kG2, kOW, kOB, kN2, kM1W, kM1B, kM2W, kM2B, kBlockEntries };
 
-// attention forward of one block (Sec. 3.3, Eq. attention over the chunk window), per (query
-// chunk i, KV group g): the rows of the group's heads form one product with the window's keys
-// (chunks max(0, i - W + 1) .. i, contiguous in k2 / v1): S = Q K^T, band softmax (P bf16 and
-// each row's log-sum-exp), O = P V, O head-major fp32 in st.o32. A group's heads go tr->hs at a
-// time (all of them unless S would pass its size bound).
+// attention forward of one block (Sec. 3.3, Eq. attention over the chunk window): O rows (bf16)
+// into st.o and each row's log-sum-exp into st.lse. On the batched attention kernel when the
+// stack's band maps exist; else materialised per (query chunk i, KV group g): the rows of the
+// group's heads form one product with the window's keys (chunks max(0, i - W + 1) .. i,
+// contiguous in k2 / v1): S = Q K^T, band softmax (P bf16 and the log-sum-exp), O = P V (head-
+// major fp32 in st.o32, then permuted into st.o). A group's heads go tr->hs at a time (all of
+// them unless S would pass its size bound).
 void attn_fwd(Run& r, fd_trainer_s::Stack& st, int b) {
   fd_trainer_s* tr = r.tr;
   const int M = st.M, Pc = st.Pc, N = tr->N, hpg = N / tr->G, rows = tr->hs * Pc;
