@@ -145,6 +145,12 @@ PRESETS: dict[str, FDConfig] = {
     "720p_wide_d3": FDConfig(latent_h=90, latent_w=160, patch=2, hidden=1536, heads=24,
                              kv_groups=3, n_blocks=2, n_refine=1, window=8, r_t=4, out_u8=True,
                              name="720p_wide_d3", chunks=2, latent_mode="ar1"),
+    # the 480p token grid (60x104 latents, 1560 tokens: 1664 padded rows, 3120 refined rows per
+    # chunk) at reduced width and depth, for the training step's parity at the product's token
+    # count (the fp64 oracle's backward stays within seconds)
+    "train_480p_grid": FDConfig(latent_h=60, latent_w=104, patch=2, hidden=256, heads=4,
+                                kv_groups=2, n_blocks=2, n_refine=1, window=2, r_t=2,
+                                name="train_480p_grid", chunks=3),
     # degenerate window W=1: every chunk attends to itself only (no temporal context)
     "tiny_w1": FDConfig(window=1, n_refine=1, r_t=2, name="tiny_w1", chunks=3),
     # refinement exercised at tiny size: r_t=2, one refinement block, 3 chunks

@@ -58,11 +58,13 @@ def split(cfg, flat):
     return out
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "tiny_qk", "small"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "tiny_qk", "small", "train_480p_grid"])
 def test_training_step_matches_the_oracle(name):
     """Loss and every parameter's gradient of one step over the preset's clip. The targets keep
     0.3 away from zero, so that no pixel sits near the kink of |x_hat - x| (the outputs of the
-    seeded decoder stay well inside [-0.3, 0.3])."""
+    seeded decoder stay well inside [-0.3, 0.3]). train_480p_grid has the 480p token grid (1560
+    tokens per frame, padded to 1664 rows; 3120 refined rows per chunk) at reduced width and
+    depth: the padding, the fused forward's key maps and the band at the product's token count."""
     cfg = synth.PRESETS[name]
     w, z = synth.make_weights(cfg), synth.make_latents(cfg)
     x = synth.make_target_pixels(cfg, min_abs=0.3)
