@@ -300,11 +300,13 @@ fd_status fd_debug_wait_timeout(fd_handle h, unsigned int limit_us, void* stream
  * Readings: the loss takes the head's output before the clamp (T1); the mean of |x_hat - x|
  * over every pixel of the clip (T3); the gradient flows through the cache (T2).
  *   fd_train_create: a trainer for clips of `chunks` (1 .. 256) latent frames of cfg (equal to
- *     the weights' cfg; the GELU MLP in bf16 with r_t frames from every chunk: mlp_gated,
- *     mlp_fp8 and first_chunk_frames give FD_ERR_CONFIG). Allocates the saved activations and
- *     scratch, transposes the weights; synchronous. The trainer is a user of w.
+ *     the weights' cfg; the bf16-valued decoder with either MLP form and either first-chunk
+ *     rule: mlp_fp8 gives FD_ERR_CONFIG). Allocates the saved activations and scratch,
+ *     transposes the weights; synchronous. The trainer is a user of w.
  *   fd_train_step: latents device fp32 [T][C'][H'][W']; targets device fp32
- *     [T][C][r_t][H' 8][W' 8] (the pixels of each chunk, fd_pixels_bytes apart); loss: one
+ *     [T][C][r_t][H' 8][W' 8] (the pixels of each chunk, fd_pixels_bytes apart; with
+ *     first_chunk_frames = 1, chunk 0's frames 1 .. r_t-1 are not read and the mean runs over
+ *     the (T - 1) r_t + 1 frames the clip decodes to); loss: one
  *     device fp32; grads: device fp32 of fd_train_grad_elems(cfg) elements, written in the
  *     weight-blob order (each tensor's gradient where its weights sit in the blob). 16-byte
  *     aligned buffers. Enqueued on `stream`; a trainer runs one step at a time.

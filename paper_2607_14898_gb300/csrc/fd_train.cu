@@ -131,6 +131,57 @@ __global__ void rmsnorm_bwd_kernel(const float* __restrict__ x, const float* __r
 }
 
 // out[c] = sum over rows of x[r][c], rows in order (deterministic)
+// Gated MLP (the XL layout, reading R7): layer 1's output z [M][2 Dm] holds, on the device,
+// the gate and up columns of 32 hidden units side by side in blocks of 64 (gate unit 32 j + i
+// at column 64 j + i, its up column at 64 j + 32 + i); a = SiLU(gate) up, in unit order.
+__device__ __forceinline__ float logistic(float x) { return 1.0f / (1.0f + expf(-x)); }
+__global__ void swiglu_fwd_kernel(const float* __restrict__ z, long long M, int Dm,
+                                  bf16* __restrict__ a) {
+  const long long n = M * Dm;
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const long long m = i / Dm;
+    const int u = static_cast<int>(i % Dm);
+    const float* zr = z + m * 2 * Dm + (u / 32) * 64 + u % 32;
+    const float g = zr[0], up = zr[32];
+    a[i] = __float2bfloat16_rn(g * logistic(g) * up);
+  }
+}
+// its backward: d gate = da up SiLU'(gate) with SiLU'(x) = s(x) (1 + x (1 - s(x))), d up =
+// da SiLU(gate); dz in the interleaved layout, fp32 and a bf16 copy
+__global__ void swiglu_bwd_kernel(const float* __restrict__ z, const float* __restrict__ da,
+                                  long long M, int Dm, float* __restrict__ dz,
+                                  bf16* __restrict__ dz16) {
+  const long long n = M * Dm;
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const long long m = i / Dm;
+    const int u = static_cast<int>(i % Dm);
+    const long long c = m * 2 * Dm + (u / 32) * 64 + u % 32;
+    const float g = z[c], up = z[c + 32], d = da[i];
+    const float sg = logistic(g);
+    const float dg = d * up * sg * (1.0f + g * (1.0f - sg)), du = d * g * sg;
+    dz[c] = dg;
+    dz[c + 32] = du;
+    dz16[c] = __float2bfloat16_rn(dg);
+    dz16[c + 32] = __float2bfloat16_rn(du);
+  }
+}
+// rows of a gated layer 1's gradient from the device's interleaved order back to the blob's
+// (gate rows, then up rows): dst row r = src row of blob row r
+__global__ void gated_rows_kernel(const float* __restrict__ src, int rows, int len,
+                                  float* __restrict__ dst) {
+  const long long n = static_cast<long long>(rows) * len;
+  const int gate = rows / 2;
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int r = static_cast<int>(i / len), k = static_cast<int>(i % len);
+    const int u = r < gate ? r : r - gate;
+    const int dr = (u / 32) * 64 + (r < gate ? 0 : 32) + u % 32;
+    dst[i] = src[static_cast<size_t>(dr) * len + k];
+  }
+}
+
 __global__ void colsum_kernel(const float* __restrict__ x, long long rows, int cols, int ld,
                               float* __restrict__ out) {
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
@@ -382,11 +433,12 @@ __global__ void head_permute_kernel(const float* __restrict__ x, int M, int Pc, 
 
 // L1 term of the pixels (reading T3: the mean of |x_hat - x| over the clip, unclamped output,
 // reading T1) through the pixel shuffle: F [R][C rs^2] with refined row (c r_t + tau) Lp + l,
-// target [T][C][r_t][H][W]; dF = sign(F - x) / total (0 on padding rows); per-block partial
-// sums of |F - x| into part[blockIdx.x] (fixed-order tree)
+// target [T][C][r_t][H][W]; dF = sign(F - x) / total (0 on padding rows, and on chunk 0's
+// frames tau >= first, which a one-frame first chunk does not emit); per-block partial sums of
+// |F - x| into part[blockIdx.x] (fixed-order tree)
 __global__ void l1_head_kernel(const float* __restrict__ F, const float* __restrict__ target,
-                               int T, int rt, int Lp, int L, int gh, int gw, int C, int rs,
-                               float inv_total, float* __restrict__ dF,
+                               int T, int rt, int first, int Lp, int L, int gh, int gw, int C,
+                               int rs, float inv_total, float* __restrict__ dF,
                                float* __restrict__ part) {
   __shared__ float red[256];
   const int cols = C * rs * rs;
@@ -399,8 +451,8 @@ __global__ void l1_head_kernel(const float* __restrict__ F, const float* __restr
     const int l = static_cast<int>(row % Lp);
     const long long ft = row / Lp;  // c r_t + tau
     float g = 0.f;
-    if (l < L) {
-      const int c = static_cast<int>(ft / rt), tau = static_cast<int>(ft % rt);
+    const int c = static_cast<int>(ft / rt), tau = static_cast<int>(ft % rt);
+    if (l < L && (c > 0 || tau < first)) {
       const int ch = col / (rs * rs), ij = col % (rs * rs);
       const int ii = ij / rs, jj = ij % rs;
       const int h = l / gw, w = l % gw;
@@ -475,6 +527,10 @@ struct fd_trainer_s {
   int T = 0;
   // shapes
   int C, H, W, p, D, N, G, NQ, QO, Dm, nb, nr, Wn, rt, rs, Cout, Cr, cin, gh, gw, L, Lp, MB, MR;
+  int Dz = 0;          // MLP layer 1's outputs: Dm, or 2 Dm for the gated MLP (interleaved)
+  bool gated = false;  // gated-SiLU MLP (the XL layout)
+  bool f1 = false;     // chunk 0 emits one frame (first_chunk_frames = 1)
+  float *dz32 = nullptr, *dwz = nullptr;  // gated: dz [M][2 Dm], layer 1's gradients (device order)
   float eps;
   std::vector<const void*> wt;   // device tensors of the weights, blob order
   std::vector<size_t> goff;      // element offset of each tensor in the gradient blob
@@ -830,11 +886,15 @@ void block_fwd(Run& r, fd_trainer_s::Stack& st, int b, size_t e0) {
   r.gemm(FD_TK_LINEAR, fd::EPI_RESID, M, tr->D, tr->NQ, st.o[b], tr->NQ, r.wb(e0 + kOW), tr->NQ,
          r.wf(e0 + kOB), st.hm[b], tr->D);
   r.rmsnorm(st.hm[b], r.wf(e0 + kN2), M, st.u2[b]);
-  r.gemm(FD_TK_LINEAR, fd::EPI_F32, M, tr->Dm, tr->D, st.u2[b], tr->D, r.wb(e0 + kM1W), tr->D,
-         r.wf(e0 + kM1B), st.z[b], tr->Dm);
+  r.gemm(FD_TK_LINEAR, fd::EPI_F32, M, tr->Dz, tr->D, st.u2[b], tr->D, r.wb(e0 + kM1W), tr->D,
+         r.wf(e0 + kM1B), st.z[b], tr->Dz);
   if (r.begin(FD_TK_POINTWISE)) {
     const long long n = static_cast<long long>(M) * tr->Dm;
-    fd::train::gelu_fwd_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.z[b], n, st.a[b]);
+    if (tr->gated)
+      fd::train::swiglu_fwd_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.z[b], M, tr->Dm,
+                                                                         st.a[b]);
+    else
+      fd::train::gelu_fwd_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.z[b], n, st.a[b]);
     r.check(cudaGetLastError());
     r.end();
   }
@@ -854,18 +914,41 @@ void block_bwd(Run& r, fd_trainer_s::Stack& st, int b, size_t e0,
   r.gemm(FD_TK_DGRAD, fd::EPI_F32, M, Dm, D, tr->dy16, D, lt.mlp2, D, nullptr, tr->gC, Dm);  // da
   r.wgrad(tr->dy16, D, st.a[b], Dm, M, r.grad(g, e0 + kM2W));
   r.colsum(dho, M, D, D, r.grad(g, e0 + kM2B));
-  // GELU'
+  // GELU' (or the gated SiLU's derivative into the interleaved dz)
+  const int Dz = tr->Dz;
+  float* dz = tr->gated ? tr->dz32 : tr->gC;
   if (r.begin(FD_TK_POINTWISE)) {
     const long long n = static_cast<long long>(M) * Dm;
-    fd::train::gelu_bwd_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.z[b], tr->gC, n,
-                                                                      tr->gC, tr->dqkv16);
+    if (tr->gated)
+      fd::train::swiglu_bwd_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.z[b], tr->gC, M, Dm,
+                                                                          dz, tr->dqkv16);
+    else
+      fd::train::gelu_bwd_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(st.z[b], tr->gC, n,
+                                                                        tr->gC, tr->dqkv16);
     r.check(cudaGetLastError());
     r.end();
   }
   // MLP layer 1
-  r.gemm(FD_TK_DGRAD, fd::EPI_F32, M, D, Dm, tr->dqkv16, Dm, lt.mlp1, Dm, nullptr, tr->gA, D);  // du2
-  r.wgrad(tr->dqkv16, Dm, st.u2[b], D, M, r.grad(g, e0 + kM1W));
-  r.colsum(tr->gC, M, Dm, Dm, r.grad(g, e0 + kM1B));
+  r.gemm(FD_TK_DGRAD, fd::EPI_F32, M, D, Dz, tr->dqkv16, Dz, lt.mlp1, Dz, nullptr, tr->gA, D);  // du2
+  if (tr->gated) {  // gradients in the device's interleaved rows, then into the blob's order
+    float* dwz = tr->dwz;
+    float* dbz = tr->dwz + static_cast<size_t>(Dz) * D;
+    r.wgrad(tr->dqkv16, Dz, st.u2[b], D, M, dwz);
+    r.colsum(dz, M, Dz, Dz, dbz);
+    if (r.begin(FD_TK_POINTWISE)) {
+      const long long n = static_cast<long long>(Dz) * D;
+      fd::train::gated_rows_kernel<<<blocks_for(n, 256), 256, 0, r.s>>>(
+          dwz, Dz, D, r.grad(g, e0 + kM1W));
+      r.check(cudaGetLastError());
+      fd::train::gated_rows_kernel<<<blocks_for(Dz, 256), 256, 0, r.s>>>(
+          dbz, Dz, 1, r.grad(g, e0 + kM1B));
+      r.check(cudaGetLastError());
+      r.end();
+    }
+  } else {
+    r.wgrad(tr->dqkv16, Dz, st.u2[b], D, M, r.grad(g, e0 + kM1W));
+    r.colsum(dz, M, Dz, Dz, r.grad(g, e0 + kM1B));
+  }
   // RMSNorm 2, plus the residual
   r.rmsnorm_bwd(st.hm[b], r.wf(e0 + kN2), tr->gA, dho, M, tr->gC, r.grad(g, e0 + kN2));
   float* dhm = tr->gC;
@@ -913,8 +996,8 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   const fd_config* wc = fd::weights_config(w);
   if (fd_weights_blob_elems(cfg) == 0 || std::memcmp(cfg, wc, sizeof(fd_config)) != 0)
     return FD_ERR_CONFIG;
-  // the decoder as the configs define it: the GELU MLP in bf16, r_t frames from every chunk
-  if (cfg->mlp_gated || cfg->mlp_fp8 || cfg->first_chunk_frames) return FD_ERR_CONFIG;
+  // the bf16-valued decoder: GELU or gated-SiLU MLPs, r_t frames per chunk or one from chunk 0
+  if (cfg->mlp_fp8) return FD_ERR_CONFIG;
   if (chunks < 1 || chunks > 256) return FD_ERR_INVALID_ARG;
   fd_trainer tr = new (std::nothrow) fd_trainer_s;
   if (tr == nullptr) return FD_ERR_OOM;
@@ -924,6 +1007,9 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   tr->C = cfg->latent_channels; tr->H = cfg->latent_h; tr->W = cfg->latent_w; tr->p = cfg->patch;
   tr->D = cfg->hidden; tr->N = cfg->heads; tr->G = cfg->kv_groups; tr->NQ = tr->N * 64;
   tr->QO = (tr->N + 2 * tr->G) * 64; tr->Dm = cfg->mlp_ratio * tr->D; tr->nb = cfg->n_blocks;
+  tr->gated = cfg->mlp_gated != 0;
+  tr->Dz = tr->gated ? 2 * tr->Dm : tr->Dm;
+  tr->f1 = cfg->first_chunk_frames == 1;
   tr->nr = cfg->n_refine; tr->Wn = cfg->window; tr->rt = cfg->r_t;
   tr->rs = cfg->vae_spatial * cfg->patch; tr->Cout = cfg->out_channels;
   tr->Cr = tr->Cout * tr->rs * tr->rs; tr->cin = tr->C * tr->p * tr->p;
@@ -939,7 +1025,7 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   {
     const size_t D = tr->D, blk[kBlockEntries] = {
         D, static_cast<size_t>(tr->QO) * D, static_cast<size_t>(tr->QO), 64, 64,
-        D * tr->NQ, D, D, static_cast<size_t>(tr->Dm) * D, static_cast<size_t>(tr->Dm),
+        D * tr->NQ, D, D, static_cast<size_t>(tr->Dz) * D, static_cast<size_t>(tr->Dz),
         D * tr->Dm, D};
     std::vector<size_t> elems = {D * tr->cin, D};
     for (int b = 0; b < tr->nb; ++b) elems.insert(elems.end(), blk, blk + kBlockEntries);
@@ -1029,7 +1115,7 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
       st.o.push_back(dalloc<bf16>(tr, static_cast<size_t>(M) * NQ, ok));
       st.hm.push_back(dalloc<float>(tr, static_cast<size_t>(M) * D, ok));
       st.u2.push_back(dalloc<bf16>(tr, static_cast<size_t>(M) * D, ok));
-      st.z.push_back(dalloc<float>(tr, static_cast<size_t>(M) * Dm, ok));
+      st.z.push_back(dalloc<float>(tr, static_cast<size_t>(M) * tr->Dz, ok));
       st.a.push_back(dalloc<bf16>(tr, static_cast<size_t>(M) * Dm, ok));
     }
   };
@@ -1078,7 +1164,7 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   setup_band(tr->sB, tr->L);
   setup_band(tr->sR, tr->rt * tr->L);
   const size_t wide = static_cast<size_t>(Mmax) *
-                      std::max({D, Dm, QO, NQ, tr->rt * D, tr->Cr});
+                      std::max({D, tr->Dz, QO, NQ, tr->rt * D, tr->Cr});
   tr->x0 = dalloc<bf16>(tr, static_cast<size_t>(MB) * tr->cin, ok);
   tr->y16 = dalloc<bf16>(tr, static_cast<size_t>(MB) * D, ok);
   tr->yh16 = dalloc<bf16>(tr, static_cast<size_t>(MR) * D, ok);
@@ -1108,7 +1194,7 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   tr->delta = dalloc<float>(tr, static_cast<size_t>(Mmax) * tr->N, ok);
   {
     const size_t R = fd::train::kColsumRows;
-    const size_t widest = std::max({D, Dm, QO, NQ, tr->rt * D, tr->Cr});
+    const size_t widest = std::max({D, tr->Dz, QO, NQ, tr->rt * D, tr->Cr});
     tr->colsum_elems = std::max((static_cast<size_t>(Mmax) * tr->N + R - 1) / R * 64,
                                 (static_cast<size_t>(Mmax) + R - 1) / R * widest);
     tr->colsum_part = dalloc<float>(tr, tr->colsum_elems, ok);
@@ -1124,7 +1210,12 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   tr->gB = dalloc<float>(tr, wide, ok);
   tr->gC = dalloc<float>(tr, wide, ok);
   tr->tbuf = dalloc<float>(tr, static_cast<size_t>(Mmax) * D, ok);
-  tr->gtmp = dalloc<float>(tr, static_cast<size_t>(D) * std::max({D, Dm, QO, tr->Cr, tr->cin}), ok);
+  tr->gtmp = dalloc<float>(tr, static_cast<size_t>(D) * std::max({D, tr->Dz, QO, tr->Cr, tr->cin}),
+                           ok);
+  if (tr->gated) {
+    tr->dz32 = dalloc<float>(tr, static_cast<size_t>(Mmax) * tr->Dz, ok);
+    tr->dwz = dalloc<float>(tr, static_cast<size_t>(tr->Dz) * (D + 1), ok);
+  }
   // transposed weights [in][out] for the input gradients dX = dY W
   auto wT = [&](size_t entry, int n_out, int n_in) -> bf16* {
     bf16* t = dalloc<bf16>(tr, static_cast<size_t>(n_out) * n_in, ok);
@@ -1139,7 +1230,7 @@ fd_status fd_train_create(const fd_config* cfg, fd_weights w, int chunks, fd_tra
   auto stackT = [&](std::vector<fd_trainer_s::LinT>& v, size_t e0, int nblocks) {
     for (int b = 0; b < nblocks; ++b) {
       const size_t e = e0 + static_cast<size_t>(b) * kBlockEntries;
-      v.push_back({wT(e + kQW, QO, D), wT(e + kOW, D, NQ), wT(e + kM1W, Dm, D),
+      v.push_back({wT(e + kQW, QO, D), wT(e + kOW, D, NQ), wT(e + kM1W, tr->Dz, D),
                    wT(e + kM2W, D, Dm)});
     }
   };
@@ -1213,13 +1304,14 @@ fd_status fd_train_step(fd_trainer tr, const float* latents, const float* target
   }
   r.gemm(FD_TK_LINEAR, fd::EPI_F32, MR, tr->Cr, D, tr->a1, D, r.wb(eH + 3), D, r.wf(eH + 4), tr->F, tr->Cr);
   // ---- loss (L1 over every pixel of the clip) and its gradient through the pixel shuffle
-  const double total = static_cast<double>(tr->T) * rt * tr->Cout * tr->gh * tr->rs * tr->gw *
-                       tr->rs;
+  const int first = tr->f1 ? 1 : rt;  // frames chunk 0 emits (reading R16)
+  const double total = (static_cast<double>(tr->T - 1) * rt + first) * tr->Cout * tr->gh *
+                       tr->rs * tr->gw * tr->rs;
   const float inv_total = static_cast<float>(1.0 / total);
   if (r.begin(FD_TK_POINTWISE)) {
     fd::train::l1_head_kernel<<<tr->loss_blocks, 256, 0, r.s>>>(
-        tr->F, targets, tr->T, rt, tr->Lp, tr->L, tr->gh, tr->gw, tr->Cout, tr->rs, inv_total,
-        tr->dF, tr->loss_part);
+        tr->F, targets, tr->T, rt, first, tr->Lp, tr->L, tr->gh, tr->gw, tr->Cout, tr->rs,
+        inv_total, tr->dF, tr->loss_part);
     r.check(cudaGetLastError());
     r.end();
   }
@@ -1324,8 +1416,8 @@ fd_status fd_op_l1_pixel_bwd(const float* F, const float* target, int frames, in
   const int blocks = static_cast<int>((n + 255) / 256);
   const float inv_total = static_cast<float>(1.0 / static_cast<double>(n));
   // one chunk of `frames` refined frames, rows unpadded (Lp = L)
-  fd::train::l1_head_kernel<<<blocks, 256, 0, s>>>(F, target, 1, frames, L, L, grid_h, grid_w,
-                                                   channels, rs, inv_total, dF, work);
+  fd::train::l1_head_kernel<<<blocks, 256, 0, s>>>(F, target, 1, frames, frames, L, L, grid_h,
+                                                   grid_w, channels, rs, inv_total, dF, work);
   if (cudaGetLastError() != cudaSuccess) return FD_ERR_CUDA;
   fd::train::finish_loss_kernel<<<1, fd::train::kLossThreads, 0, s>>>(work, blocks, inv_total,
                                                                        loss);

@@ -182,6 +182,11 @@ PRESETS: dict[str, FDConfig] = {
     # XL layout at tiny size: 48-channel 16x latent, patch 1, gated-SiLU MLP, refinement
     "tiny_gated": FDConfig(latent_channels=48, latent_h=10, latent_w=13, vae_spatial=16,
                            mlp_gated=True, n_refine=1, r_t=2, name="tiny_gated", chunks=3),
+    # the XL layout at tiny size with the rest of XL's stream rules: W=2, r_t=4 and the
+    # one-frame first chunk (training-step parity of the gated MLP under the causal frame count)
+    "tiny_xl": FDConfig(latent_channels=48, latent_h=10, latent_w=13, vae_spatial=16,
+                        mlp_gated=True, n_refine=1, window=2, r_t=4, first_chunk_frames=1,
+                        name="tiny_xl", chunks=3),
     # FlashDecoder-XL as the paper's configuration table gives it: Wan2.2 latents (48
     # channels, 16x spatial), patch 1, D=1536, 24 heads / 3 KV groups, 20 + 2 blocks, W=2,
     # r_t=4, gated-SiLU MLP 4x; 480p (30x52 latent), 720p (45x80), 1080p (68x120)

@@ -37,6 +37,11 @@ def gpu_step(cfg, w, z, x):
     W = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
     tr = fdp.Trainer(cfg, W, len(z))
     lat = torch.from_numpy(np.ascontiguousarray(np.stack(z))).cuda()
+    # the step's target layout has r_t frames per chunk; a one-frame chunk 0 is padded with
+    # NaN, which the step must not read
+    rt = cfg.r_t
+    x = [np.concatenate([c, np.full(c.shape[:1] + (rt - c.shape[1],) + c.shape[2:], np.nan,
+                                    np.float32)], axis=1) if c.shape[1] < rt else c for c in x]
     tgt = torch.from_numpy(np.ascontiguousarray(np.stack(x))).cuda()
     loss = torch.zeros(1, device="cuda")
     grads = torch.full((tr.grad_elems,), float("nan"), device="cuda")
@@ -58,13 +63,16 @@ def split(cfg, flat):
     return out
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "tiny_qk", "small", "train_480p_grid"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_rt", "tiny_qk", "small", "train_480p_grid",
+                                  "tiny_gated", "small_f1", "tiny_xl"])
 def test_training_step_matches_the_oracle(name):
     """Loss and every parameter's gradient of one step over the preset's clip. The targets keep
     0.3 away from zero, so that no pixel sits near the kink of |x_hat - x| (the outputs of the
     seeded decoder stay well inside [-0.3, 0.3]). train_480p_grid has the 480p token grid (1560
     tokens per frame, padded to 1664 rows; 3120 refined rows per chunk) at reduced width and
-    depth: the padding, the fused forward's key maps and the band at the product's token count."""
+    depth: the padding, the fused forward's key maps and the band at the product's token count.
+    tiny_gated, small_f1 and tiny_xl carry the XL layout's gated-SiLU MLP and the one-frame
+    first chunk (whose loss covers the (T - 1) r_t + 1 frames the clip decodes to)."""
     cfg = synth.PRESETS[name]
     w, z = synth.make_weights(cfg), synth.make_latents(cfg)
     x = synth.make_target_pixels(cfg, min_abs=0.3)
@@ -85,16 +93,15 @@ def test_training_step_matches_the_oracle(name):
 
 
 def test_training_step_is_deterministic_and_refuses_other_layouts():
-    """Two steps on the same inputs give the same bits (no order-dependent sums); the gated
-    MLP, FP8 MLPs and the one-frame first chunk are refused at creation."""
+    """Two steps on the same inputs give the same bits (no order-dependent sums); FP8 MLPs
+    (the inference-only lossy setting) are refused at creation."""
     cfg = synth.PRESETS["tiny_rt"]
     w, z = synth.make_weights(cfg), synth.make_latents(cfg)
     x = synth.make_target_pixels(cfg, min_abs=0.3)
     a = gpu_step(cfg, w, z, x)
     b = gpu_step(cfg, w, z, x)
     assert a[0] == b[0] and torch.equal(a[1], b[1])
-    for other in (synth.PRESETS["tiny_gated"], synth.PRESETS["small_fp8"],
-                  synth.PRESETS["small_f1"]):
+    for other in (synth.PRESETS["small_fp8"], synth.PRESETS["tiny_gated_fp8"]):
         W = fdp.Weights(other, fdp.pack_blob(other, synth.make_weights(other)))
         with pytest.raises(fdp.FdError) as e:
             fdp.Trainer(other, W, 2)

@@ -122,7 +122,7 @@ def test_l1_bwd_is_the_sign_over_the_count():
 
 
 @pytest.mark.parametrize("name", ["tiny", "tiny_rt", "small", "tiny_gated", "tiny_qk",
-                                  "small_f1"])
+                                  "small_f1", "tiny_xl"])
 def test_explicit_step_equals_autograd_step(name):
     """The hand-written backward over the whole clip (masked one-pass form) gives the
     streaming step's loss and every gradient, to rounding."""
