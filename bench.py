@@ -40,7 +40,8 @@ def parse():
                     help="several streams per GPU: stacked GEMMs (fd_decode_batch) or one "
                          "forked CUDA stream per decoder (fd_decode_chunks)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-secondary", action="store_true", help="skip the 720p line")
+    ap.add_argument("--no-secondary", action="store_true",
+                    help="skip the other configurations (720p, 480p x 8, 720p wide, XL 480p)")
     ap.add_argument("--no-training", action="store_true", help="skip the training-step line")
     ap.add_argument("--training-only", action="store_true",
                     help="run only the training-step line (one GPU; for profiling it alone)")
@@ -390,7 +391,7 @@ def run_ours(args, rank: int, world: int):
         "kernels": kernels,
     }
     if rank == 0 and world == 1 and not args.no_secondary and cfg.name == "480p":
-        line["secondary"] = secondary_720p(args, stream, blob)
+        line["secondary"] = {n: secondary_line(args, stream, n, blob) for n in SECONDARY}
     if rank == 0 and world == 1 and not args.no_training and cfg.name == "480p":
         line["training"] = training_line(args, stream, blob)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -405,10 +406,16 @@ def run_ours(args, rank: int, world: int):
     return line
 
 
-def secondary_720p(args, stream, blob):
-    """720p stream (config 3: 32 chunks, uint8 pixels): frames/s and per-chunk latency, same
-    procedure as the headline, plus its own per-kernel profile and roofline. The model (and so
-    the weight blob) is the 480p one; only the latent grid differs."""
+# further configurations of the benchmark, each timed like the headline in the same run
+SECONDARY = ("720p", "480p_x8", "720p_wide", "xl_480p")
+
+
+def secondary_line(args, stream, name, blob480):
+    """One more configuration: warm-up streams, then one timed stream (CUDA events around each
+    chunk on the launching stream), then its own per-kernel profile (stream 0 decoded alone,
+    events around every launch) with the attention's roofline. Configurations with the 480p
+    model's weight layout (720p, 480p x 8) reuse its blob; the others draw their own weights.
+    Several streams per GPU (480p x 8) decode through fd_decode_batch, as the headline does."""
     import statistics as st
 
     import torch
@@ -417,26 +424,43 @@ def secondary_720p(args, stream, blob):
     from paper_2607_14898_gb300 import costs
     from paper_2607_14898_gb300 import flashdec as fdp
 
-    cfg = synth.PRESETS["720p"]
-    chunks = cfg.chunks
+    cfg = synth.PRESETS[name]
+    chunks, S = cfg.chunks, cfg.streams
+    base = synth.PRESETS["480p"]
+    same = (synth.weight_layout(cfg) == synth.weight_layout(base)
+            and cfg.mlp_gated == base.mlp_gated and cfg.mlp_fp8 == base.mlp_fp8)
+    blob = blob480 if same else fdp.pack_blob(cfg, synth.make_weights(cfg))
     weights = fdp.Weights(cfg, blob)
-    dec = fdp.Decoder(cfg, weights)
-    z = torch.from_numpy(synth.make_latents(cfg, chunks=chunks)).cuda()
-    pix = [torch.empty(3, cfg.r_t, cfg.out_h, cfg.out_w, dtype=torch.uint8, device="cuda")
-           for _ in range(chunks)]
+    decs = [fdp.Decoder(cfg, weights) for _ in range(S)]
+    batch = fdp.Batch(cfg, weights, S) if S > 1 else None
+    zs = [torch.from_numpy(synth.make_latents(cfg, chunks=chunks, seed=sd)).cuda()
+          for sd in range(cfg.latent_seed, cfg.latent_seed + S)]
+    dt = torch.uint8 if cfg.out_u8 else torch.float32
+    pixs = [[torch.empty(cfg.out_channels, cfg.r_t, cfg.out_h, cfg.out_w, dtype=dt,
+                         device="cuda") for _ in range(chunks)] for _ in range(S)]
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(chunks)]
 
     def step(record):
-        dec.reset()
+        for d in decs:
+            d.reset()
         for t in range(chunks):
             if record:
                 ev[t][0].record(stream)
-            dec.decode_chunk(z[t], pix[t], stream)
+            if batch is None:
+                decs[0].decode_chunk(zs[0][t], pixs[0][t], stream)
+            else:
+                batch.decode(decs, [z[t] for z in zs], [p[t] for p in pixs], stream)
             if record:
                 ev[t][1].record(stream)
 
+    def step_single():
+        decs[0].reset()
+        for t in range(chunks):
+            decs[0].decode_chunk(zs[0][t], pixs[0][t], stream)
+
+    warm = 1 if chunks * cfg.tokens > 16 * 3600 else max(1, args.warmup)
     with torch.cuda.stream(stream):
-        for _ in range(max(1, args.warmup)):
+        for _ in range(warm):
             step(False)
         torch.cuda.synchronize()
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -447,25 +471,37 @@ def secondary_720p(args, stream, blob):
     ms = a.elapsed_time(b)
     lat = [ev[t][0].elapsed_time(ev[t][1]) for t in range(chunks)]
     steady = lat[cfg.window - 1:]
-    ok = dec.sync_status() == fdp.FD_OK
-    # per-kernel profile: one more stream with CUDA events around every launch
-    dec.profile(True)
+    ok = all(d.sync_status() == fdp.FD_OK for d in decs)
+    decs[0].profile(True)
     with torch.cuda.stream(stream):
-        step(False)
+        step_single()
     torch.cuda.synchronize()
-    prof = dec.profile_collect()
-    dec.profile(False)
+    prof = decs[0].profile_collect()
+    decs[0].profile(False)
     _, sustained, _, peak_src = peaks()
     kp = kernel_profile(cfg, prof, chunks, 1, sustained)
-    dec.close()
+    if batch is not None:
+        batch.close()
+    for d in decs:
+        d.close()
     weights.close()
-    flops = costs.stream_flops(cfg, chunks)
-    return {"workload": f"720p single stream (config 3), {chunks} chunks, uint8 pixels",
-            "frames_per_s": round(chunks * cfg.r_t / (ms * 1e-3), 2),
+    flops = S * costs.stream_flops(cfg, chunks)
+    fp8 = bool(cfg.mlp_fp8)
+    return {"workload": f"{name}: {S} stream{'s' if S > 1 else ''} of {chunks} chunks, latent "
+                        f"{cfg.latent_channels}x{cfg.latent_h}x{cfg.latent_w}, patch {cfg.patch} "
+                        f"({cfg.tokens} tokens/chunk), {cfg.n_blocks}+{cfg.n_refine} blocks, "
+                        f"D={cfg.hidden}, {cfg.heads} heads / {cfg.kv_groups} KV groups, "
+                        f"{'gated-SiLU' if cfg.mlp_gated else 'GELU'} MLP, W={cfg.window}, "
+                        f"{'uint8' if cfg.out_u8 else 'fp32'} pixels, "
+                        f"{'AR(1)' if cfg.latent_mode == 'ar1' else 'N(0,1)'} latents"
+                        + (", fd_decode_batch (stacked GEMMs)" if S > 1 else ""),
+            "frames_per_s": round(S * chunks * cfg.r_t / (ms * 1e-3), 2),
+            "warmup_streams": warm,
             "p50_ms": round(st.median(lat), 3), "steady_p50_ms": round(st.median(steady), 3),
             "p99_ms": round(sorted(lat)[max(0, int(0.99 * len(lat)) - 1)], 3),
             "tensor_frac_step": round(flops / (ms * 1e-3) / 1e12 / sustained, 3),
-            "roofline": {"kernel": "attention (attn_kernel, backbone + refinement launches)",
+            "roofline": {"kernel": "attention (attn_kernel, backbone + refinement launches)"
+                                   + (", stream 0 alone" if S > 1 else ""),
                          "bound": "tensor", "achieved": round(kp["att_tflops"], 1),
                          "peak": sustained, "unit": "TFLOP/s",
                          "frac": round(kp["att_tflops"] / sustained, 3),
@@ -474,6 +510,8 @@ def secondary_720p(args, stream, blob):
                          "us_per_launch": round(1e3 * kp["att_ms"] / kp["att_n"], 2),
                          "gemm_tflops": round(kp["gemm_tflops"], 1),
                          "gemm_frac": round(kp["gemm_frac"], 3),
+                         "gemm_peak": ("bf16 sustained; the FP8 MLP products against 2x that"
+                                       if fp8 else "bf16 sustained"),
                          "measured_over": "1 profiled stream (CUDA events around each launch)"},
             "kernels": kp["kernels"], "device_ok": ok}
 
