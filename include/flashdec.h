@@ -222,9 +222,10 @@ fd_status fd_decode_chunk_host(fd_handle h, const float* latent_host, void* pixe
 /* Restart the stream: Algorithm 1's initialisation again for a new latent sequence, t = 0 and
  * the caches logically empty (their memory is not cleared; stale entries are never read
  * because attention at chunk t reads only chunks <= t). Clears the error state.
- * Stream-ordered: enqueued on the stream of the handle's last decode call, so the next decode
- * on that stream starts from chunk 0 without a host wait. A decode on ANOTHER stream must
- * first wait for that one (e.g. an event), or call fd_sync_status first.
+ * Stream-ordered: enqueued on the stream of the handle's last call, with no host wait. The
+ * handle's next call that touches its device state (a decode, fd_load_state,
+ * fd_debug_wait_timeout) is ordered after the reset whatever stream it is given: on another
+ * stream it first waits for an event the reset recorded.
  * Errors: FD_ERR_INVALID_ARG (null handle), FD_ERR_CUDA. */
 fd_status fd_reset(fd_handle h);
 

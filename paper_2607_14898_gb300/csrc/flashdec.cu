@@ -394,6 +394,10 @@ struct fd_handle_s {
   uint64_t serial = 0;
   bool error = false;
   cudaStream_t last_stream = nullptr;
+  // fd_reset's clears, recorded on its stream; the next call that touches the handle's device
+  // state on another stream waits for them (after_reset)
+  cudaEvent_t ev_reset = nullptr;
+  bool reset_pending = false;
   // fd_decode_chunks: a library-owned stream on which this handle's chunk runs beside the
   // other handles', forked from and joined back to the caller's stream (created on first use)
   cudaStream_t side = nullptr;
@@ -625,6 +629,16 @@ fd_status run_block(fd_handle h, const LayerW& lw, Ring& r, float* hbuf, int row
   p1.ld_out = d.Mr * d.D;
   if ((st = run_linear(h, FD_K_MLP1, tm_u, lw.mlp1, rows, p1, so_hid, s))) return st;
   return run_linear(h, FD_K_MLP2, tm_hid, lw.mlp2, rows, po, so_h, s);
+}
+
+// Order a call on stream s after a pending fd_reset, whose clears ran on the stream of the
+// handle's previous call: a wait on the reset's event when s is another stream.
+fd_status after_reset(fd_handle h, cudaStream_t s) {
+  if (!h->reset_pending) return FD_OK;
+  if (s != h->last_stream && cudaStreamWaitEvent(s, h->ev_reset, 0) != cudaSuccess)
+    return FD_ERR_CUDA;
+  h->reset_pending = false;
+  return FD_OK;
 }
 
 fd_status decode_one(fd_handle h, const float* latent, void* pixels, cudaStream_t s) {
@@ -1441,6 +1455,7 @@ fd_status fd_decode_chunk(fd_handle h, const float* latent_dev, void* pixels_dev
   if (h->error) return FD_ERR_STATE;
   if (h->t_host >= (1LL << 30)) return FD_ERR_STATE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (after_reset(h, s) != FD_OK) return FD_ERR_CUDA;
   h->last_stream = s;
   fd_status st = decode_one(h, latent_dev, pixels_dev, s);
   if (st != FD_OK) {
@@ -1478,6 +1493,7 @@ fd_status fd_decode_chunks(fd_handle* hs, int n, const float* const* latents_dev
   for (int i = 0; i < n; ++i) {
     fd_handle h = hs[i];
     if (cudaStreamWaitEvent(h->side, hs[0]->ev_fork, 0) != cudaSuccess) return FD_ERR_CUDA;
+    if (after_reset(h, h->side) != FD_OK) return FD_ERR_CUDA;
     fd_status st = decode_one(h, latents_dev[i], pixels_dev[i], h->side);
     if (st == FD_OK && cudaEventRecord(h->ev_join, h->side) != cudaSuccess) st = FD_ERR_CUDA;
     if (st != FD_OK) {
@@ -1666,6 +1682,8 @@ fd_status fd_decode_batch(fd_batch b, fd_handle* hs, int n, const float* const* 
     b->table_for.resize(n);
     for (int i = 0; i < n; ++i) b->table_for[i] = hs[i]->serial;
   }
+  for (int i = 0; i < n; ++i)
+    if (after_reset(hs[i], s) != FD_OK) return FD_ERR_CUDA;
   const fd_status st = decode_batch(b, hs, n, latents_dev, pixels_dev, s);
   for (int i = 0; i < n; ++i) {
     if (st != FD_OK) {
@@ -1711,6 +1729,9 @@ fd_status fd_decode_chunk_host(fd_handle h, const float* latent_host, void* pixe
 
 fd_status fd_reset(fd_handle h) {
   if (h == nullptr) return FD_ERR_INVALID_ARG;
+  if (h->ev_reset == nullptr &&
+      cudaEventCreateWithFlags(&h->ev_reset, cudaEventDisableTiming) != cudaSuccess)
+    return FD_ERR_CUDA;
   if (cudaMemsetAsync(h->state, 0, 2 * sizeof(int), h->last_stream) != cudaSuccess)
     return FD_ERR_CUDA;
   // a launch stopped by an error may leave attention counters non-zero
@@ -1718,6 +1739,8 @@ fd_status fd_reset(fd_handle h) {
       cudaMemsetAsync(h->attn_ws, 0, sizeof(int) * attn_pairs(h->d), h->last_stream) !=
           cudaSuccess)
     return FD_ERR_CUDA;
+  if (cudaEventRecord(h->ev_reset, h->last_stream) != cudaSuccess) return FD_ERR_CUDA;
+  h->reset_pending = true;
   h->t_host = 0;
   h->error = false;
   return FD_OK;
@@ -1731,6 +1754,7 @@ fd_status fd_destroy(fd_handle h) {
     cudaStreamDestroy(h->side);
   }
   if (h->ev_fork != nullptr) cudaEventDestroy(h->ev_fork);
+  if (h->ev_reset != nullptr) cudaEventDestroy(h->ev_reset);
   if (h->ev_join != nullptr) cudaEventDestroy(h->ev_join);
   for (size_t i = 0; i < h->ev_start.size(); ++i) {
     cudaEventDestroy(h->ev_start[i]);
@@ -1838,6 +1862,7 @@ fd_status fd_load_state(fd_handle h, const void* host_buf, size_t bytes, void* s
       !same_cfg(&hd.cfg, &h->cfg) || hd.t < 0 || hd.t >= (1LL << 30))
     return FD_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (after_reset(h, s) != FD_OK) return FD_ERR_CUDA;
   const uint8_t* src = static_cast<const uint8_t*>(host_buf) + sizeof(hd);
   auto copy_in = [&](std::vector<Ring>& rings, int pitch) -> bool {
     const size_t n = ring_bytes(h->d, pitch);
@@ -1885,6 +1910,7 @@ fd_status fd_sync_status(fd_handle h) {
 fd_status fd_debug_wait_timeout(fd_handle h, unsigned int limit_us, void* stream) {
   if (h == nullptr || limit_us < 1 || limit_us > 100000) return FD_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (after_reset(h, s) != FD_OK) return FD_ERR_CUDA;
   if (fd::launch_wait_check(h->state + 1, 1000ull * limit_us, s) != cudaSuccess)
     return FD_ERR_CUDA;
   h->last_stream = s;

@@ -85,6 +85,38 @@ def test_decode_deterministic_after_reset():
         assert torch.equal(x, y)
 
 
+def test_reset_orders_a_decode_on_another_stream():
+    """fd_reset enqueues its clears on the stream of the handle's last call (A). Stream A is
+    held busy by a sleep kernel when the reset is enqueued, and the next chunk is decoded on
+    stream B at once: it must still be chunk 0 of a new stream (the decode waits for the reset's
+    event), bit for bit the chunk 0 of a fresh decode, and the chunk after it chunk 1."""
+    cfg = synth.PRESETS["tiny_rt"]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    fresh = gpu_stream(cfg, w, z, chunks=2)
+    W = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    dec = fdp.Decoder(cfg, W)
+    shape = (cfg.out_channels, cfg.r_t, cfg.out_h, cfg.out_w)
+    a, b = torch.cuda.Stream(), torch.cuda.Stream()
+    for t in range(2):
+        dec.decode_chunk(dev(z[t]), torch.empty(shape, device="cuda"), a)
+    torch.cuda.synchronize()
+    lat = [dev(z[t]) for t in range(2)]
+    got = [torch.empty(shape, device="cuda") for _ in range(2)]
+    torch.cuda.synchronize()
+    with torch.cuda.stream(a):
+        torch.cuda._sleep(200_000_000)      # about 0.1 s of stream A
+    dec.reset()                             # clears enqueued on A, behind the sleep
+    for t in range(2):
+        dec.decode_chunk(lat[t], got[t], b)
+    torch.cuda.synchronize()
+    assert dec.sync_status() == fdp.FD_OK
+    assert dec.chunk_index == 2
+    for t in range(2):
+        assert torch.equal(got[t].cpu(), fresh[t]), t
+    dec.close()
+    W.close()
+
+
 def test_decode_chunks_concurrent_streams_match_single_stream_decodes():
     """fd_decode_chunks runs independent streams (one weights object, three handles, seeds s)
     concurrently on forked streams; each stream's pixels are bit-identical to decoding it alone
