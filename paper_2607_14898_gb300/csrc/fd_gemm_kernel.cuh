@@ -257,15 +257,17 @@ __global__ void __launch_bounds__(192, 1)
       else
         mbar_wait(bar_full + 8 * (j % C::kStages), (j / C::kStages) & 1, p.err, ERR_WAIT_TMA);
     }
-  } else if (aligned && warp == 1 && lane == 0 && rank == 0) {
+  } else if (aligned && warp == 1 && rank == 0) {
     // ------------------------------------------------------------ MMA issuer
+    // (the whole warp runs the loop; one elected lane issues)
     const uint32_t idesc =
         p.fp8 ? idesc_e4m3_f32(tile_rows, BN) : idesc_bf16_f32(tile_rows, BN);
     int it = 0, tc = 0;
     bool ok = true;
     for (int tile = cta0; tile < tiles && ok; tile += ctas, ++tc) {
       const int acc = tc & 1;
-      if (!mbar_wait(bar_tempty + 8 * acc, ((tc >> 1) & 1) ^ 1, p.err, ERR_WAIT_EPI)) break;
+      if (!mbar_wait_warp(bar_tempty + 8 * acc, ((tc >> 1) & 1) ^ 1, p.err, ERR_WAIT_EPI))
+        break;
       tc_fence_after();
       const uint32_t d_acc = tmem + static_cast<uint32_t>(acc) * kAccCols;
       for (int kb = 0; kb < nk; ++kb, ++it) {
@@ -273,7 +275,7 @@ __global__ void __launch_bounds__(192, 1)
         const uint32_t d_tmem = DS ? d_acc + static_cast<uint32_t>(kb) * BN : d_acc;
         const int kacc = DS ? 0 : kb;  // accumulate over K blocks (DS: within the block only)
         const int s = it % C::kStages;
-        if (!mbar_wait(bar_full + 8 * s, (it / C::kStages) & 1, p.err, ERR_WAIT_TMA)) {
+        if (!mbar_wait_warp(bar_full + 8 * s, (it / C::kStages) & 1, p.err, ERR_WAIT_TMA)) {
           ok = false;
           break;
         }
@@ -284,29 +286,29 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
           for (int k = 0; k < 4; ++k) {  // 4 x 32 e4m3 = one 128-byte row
             const uint64_t da = sdesc_k_sw128(a0 + 32 * k), db = sdesc_k_sw128(b0 + 32 * k);
-            if (PAIR) mma_e4m3_ss_pair(d_tmem, da, db, idesc, (kb | k) != 0);
-            else mma_e4m3_ss(d_tmem, da, db, idesc, (kb | k) != 0);
+            if (PAIR) mma_e4m3_ss_pair_w(d_tmem, da, db, idesc, (kb | k) != 0);
+            else mma_e4m3_ss_w(d_tmem, da, db, idesc, (kb | k) != 0);
           }
         } else {
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
             const uint64_t da = sdesc_k_sw128(a0 + 32 * k), db = sdesc_k_sw128(b0 + 32 * k);
-            if (PAIR) mma_bf16_ss_pair(d_tmem, da, db, idesc, (kacc | k) != 0);
-            else mma_bf16_ss(d_tmem, da, db, idesc, (kacc | k) != 0);
+            if (PAIR) mma_bf16_ss_pair_w(d_tmem, da, db, idesc, (kacc | k) != 0);
+            else mma_bf16_ss_w(d_tmem, da, db, idesc, (kacc | k) != 0);
           }
         }
         // stage s free (in both CTAs of a pair) once these MMAs have read it
-        if (PAIR) mma_commit_pair(bar_empty + 8 * s, 3);
-        else mma_commit(bar_empty + 8 * s);
+        if (PAIR) mma_commit_pair_w(bar_empty + 8 * s, 3);
+        else mma_commit_w(bar_empty + 8 * s);
       }
       if (ok) {
-        if (PAIR) mma_commit_pair(bar_tfull + 8 * acc, 3);
-        else mma_commit(bar_tfull + 8 * acc);
+        if (PAIR) mma_commit_pair_w(bar_tfull + 8 * acc, 3);
+        else mma_commit_w(bar_tfull + 8 * acc);
       }
     }
-    if (PAIR) mma_commit_pair(bar_done, 1);
-    else mma_commit(bar_done);
-    mbar_wait(bar_done, 0, p.err, ERR_WAIT_MMA);
+    if (PAIR) mma_commit_pair_w(bar_done, 1);
+    else mma_commit_w(bar_done);
+    mbar_wait_warp(bar_done, 0, p.err, ERR_WAIT_MMA);
   } else if (aligned && warp >= 2) {
     // ------------------------------------------------------------ epilogue
     const int quarter = warp & 3;  // TMEM lanes this warp may read
