@@ -282,20 +282,15 @@ __global__ void __launch_bounds__(192, 1)
         tc_fence_after();
         const uint32_t a0 = sA + s * C::kABytes;
         const uint32_t b0 = sB + s * C::kBBytes;
+        // one 128-byte row of the stage: 4 MMAs of K = 16 bf16 (or 32 e4m3) elements
+        static_assert(kBK == 64, "a K block is one 128-byte swizzle row of bf16");
+        const uint64_t da = sdesc_k_sw128(a0), db = sdesc_k_sw128(b0);
         if (p.fp8) {
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {  // 4 x 32 e4m3 = one 128-byte row
-            const uint64_t da = sdesc_k_sw128(a0 + 32 * k), db = sdesc_k_sw128(b0 + 32 * k);
-            if (PAIR) mma_e4m3_ss_pair_w(d_tmem, da, db, idesc, (kb | k) != 0);
-            else mma_e4m3_ss_w(d_tmem, da, db, idesc, (kb | k) != 0);
-          }
+          if (PAIR) mma4_e4m3_ss_pair_w(d_tmem, da, db, idesc, kb != 0);
+          else mma4_e4m3_ss_w(d_tmem, da, db, idesc, kb != 0);
         } else {
-#pragma unroll
-          for (int k = 0; k < kBK / 16; ++k) {
-            const uint64_t da = sdesc_k_sw128(a0 + 32 * k), db = sdesc_k_sw128(b0 + 32 * k);
-            if (PAIR) mma_bf16_ss_pair_w(d_tmem, da, db, idesc, (kacc | k) != 0);
-            else mma_bf16_ss_w(d_tmem, da, db, idesc, (kacc | k) != 0);
-          }
+          if (PAIR) mma4_bf16_ss_pair_w(d_tmem, da, db, idesc, kacc != 0);
+          else mma4_bf16_ss_w(d_tmem, da, db, idesc, kacc != 0);
         }
         // stage s free (in both CTAs of a pair) once these MMAs have read it
         if (PAIR) mma_commit_pair_w(bar_empty + 8 * s, 3);
