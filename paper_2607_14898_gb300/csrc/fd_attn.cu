@@ -351,8 +351,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         tc_fence_after();
         const uint64_t dq = dq0 + static_cast<uint64_t>((2 * qb * kQBytes) >> 4);
         const uint64_t dk = dk0 + static_cast<uint64_t>(((J % kStages) * kKBytes) >> 4);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) mma_bf16_ss(s_tmem, dq + 2 * k, dk + 2 * k, idesc_s, k != 0);
+        mma4_bf16_ss(s_tmem, dq, dk, idesc_s, 0u);
         mma_commit(bar(kBarS + x));
         if (c.last) mma_commit(bar(kBarQFree + qb));
         return true;
@@ -377,11 +376,9 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
         tc_fence_after();
         if (!ok) break;
         const uint64_t dv = dv0 + static_cast<uint64_t>((st * kVBytes) >> 4);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          mma_bf16_ts(o_tmem, p_tmem + 8u * kk,
-                      dv + static_cast<uint64_t>((((kk >> 2) * kVSub) >> 4) + 2 * (kk & 3)),
-                      idesc_o, (!here.first || kk != 0) ? 1u : 0u);
+        // keys 0-63 of the block (P columns 0-31, V^T sub-block 0), then keys 64-127
+        mma4_bf16_ts(o_tmem, p_tmem, dv, idesc_o, here.first ? 0u : 1u);
+        mma4_bf16_ts(o_tmem, p_tmem + 32u, dv + static_cast<uint64_t>(kVSub >> 4), idesc_o, 1u);
         mma_commit(bar(kBarPv + x));
         mma_commit(bar(kBarKvEmpty + st));  // one of the two arrivals that free the stage
       }
