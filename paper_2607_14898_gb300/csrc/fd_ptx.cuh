@@ -171,35 +171,6 @@ __device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols
   asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
                : "memory");
 }
-// D (+)= A B^T on the CTA pair, issued by the even CTA: M = 256 (A rows 0..127 from this CTA's
-// shared memory, 128..255 from the peer's at the same offset), B's N rows split in halves the
-// same way; each CTA's TMEM receives its 128 rows of D
-__device__ __forceinline__ void mma_bf16_ss_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                                 uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-__device__ __forceinline__ void mma_e4m3_ss_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                                 uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// arrive once on the mbarrier at this offset in every CTA of cta_mask when the pair MMAs
-// issued so far by this thread have completed
-__device__ __forceinline__ void mma_commit_pair(uint32_t bar, uint16_t cta_mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-      " [%0], %1;" ::"r"(bar), "h"(cta_mask)
-      : "memory");
-}
 
 // Bulk tensor stores from shared memory (async proxy); each call is one bulk group after
 // bulk_commit(). The source tile must be made visible first (fence_proxy_async_smem + sync).
@@ -265,43 +236,12 @@ __device__ __forceinline__ void tc_fence_before() {
 __device__ __forceinline__ void tc_fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
-// D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulate, cta_group::1.
-__device__ __forceinline__ void mma_bf16_ss(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                            uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// D[tmem] (+)= A[smem] * B[smem]^T, e4m3 inputs (K = 32 per instruction), fp32 accumulate.
-__device__ __forceinline__ void mma_e4m3_ss(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                            uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
 // four floats as e4m3 bytes (round to nearest even, saturating at 448), f0 in the low byte
 __device__ __forceinline__ uint32_t pack_e4m3x4(float f0, float f1, float f2, float f3) {
   uint16_t lo, hi;
   asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(lo) : "f"(f1), "f"(f0));
   asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(hi) : "f"(f3), "f"(f2));
   return static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
-}
-// D[tmem] (+)= A[tmem] * B[smem]^T: A (M=128 rows = TMEM lanes, K packed two bf16 per 32-bit
-// column) read from tensor memory, B from shared memory.
-__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
-                                            uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
 }
 // ---- MMAs and commits issued by one lane of a converged warp: the whole warp runs the issue
 // loop and elect.sync picks the lane (always the same one, so its commits track its own
@@ -315,6 +255,8 @@ __device__ __forceinline__ void mma_commit_w(uint32_t bar) {
       "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}"
       ::"r"(bar) : "memory");
 }
+// arrive once on the mbarrier at this offset in every CTA of cta_mask when the pair MMAs
+// issued so far by the elected lane have completed
 __device__ __forceinline__ void mma_commit_pair_w(uint32_t bar, uint16_t cta_mask) {
   asm volatile(
       "{\n\t.reg .pred e;\n\t.reg .b32 r;\n\t"
@@ -323,9 +265,14 @@ __device__ __forceinline__ void mma_commit_pair_w(uint32_t bar, uint16_t cta_mas
       ".b64 [%0], %1;\n\t}" ::"r"(bar), "h"(cta_mask)
       : "memory");
 }
-// One K block of 64 bf16 (or 128 e4m3) elements: four MMAs at K offsets of 32 bytes inside the
-// 128-byte swizzle atom (2 in the encoded descriptor address), issued back to back from one
-// asm block by one elected lane; the first accumulates if `accumulate`, the others always.
+// D[tmem] (+)= A[smem] B[smem]^T with fp32 accumulation, bf16 (kind::f16, K = 16 per MMA) or
+// e4m3 (kind::f8f6f4, K = 32) inputs, over one K block of 64 bf16 (or 128 e4m3) elements: four
+// MMAs at K offsets of 32 bytes inside the 128-byte swizzle atom (2 in the encoded descriptor
+// address), issued back to back from one asm block by one elected lane; the first accumulates
+// if `accumulate`, the others always. The _pair forms run on the CTA pair (cta_group::2),
+// issued by the even CTA: M = 256 (A rows 0..127 from this CTA's shared memory, 128..255 from
+// the peer's at the same offset), B's N rows split in halves the same way; each CTA's TMEM
+// receives its 128 rows of D.
 // Measured on the GB300 at 104-124 cycles per MMA against 125-126 for separate elected MMAs.
 #define FD_MMA4_BODY(KIND, GROUP)                                                          \
   "{\n\t.reg .pred p, q, e;\n\t.reg .b32 r;\n\t.reg .b64 a1, a2, a3, b1, b2, b3;\n\t"     \
@@ -380,8 +327,9 @@ __device__ __forceinline__ void mma4_bf16_ss(uint32_t d_tmem, uint64_t adesc, ui
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
-// Four MMAs with A from TMEM: A columns a, a + 8, a + 16, a + 24 (16 fp16 K elements each) and
-// B descriptors at 32-byte K steps; the first accumulates if `accumulate`, the others always.
+// Four MMAs with A from TMEM (M = 128 rows = TMEM lanes, K packed two 16-bit values per 32-bit
+// column): A columns a, a + 8, a + 16, a + 24 (16 K elements each) and B descriptors at 32-byte
+// K steps in shared memory; the first accumulates if `accumulate`, the others always.
 __device__ __forceinline__ void mma4_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
                                              uint32_t idesc, uint32_t accumulate) {
   asm volatile(
