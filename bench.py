@@ -122,12 +122,12 @@ def source_hash(*names: str) -> str:
 
 def ncu_traffic(kernel_file: str, workload: str, launch: str):
     """DRAM bytes of one launch of a kernel (launch = which of its launches was captured) from
-    the committed ncu summary, if the kernel source has not changed since the counters were
-    taken (else None)."""
+    the committed ncu summary, if the kernel source (its file and the PTX primitives it
+    includes) has not changed since the counters were taken (else None)."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
-    cur = source_hash(kernel_file)
+    cur = source_hash(kernel_file, "fd_ptx.cuh")
     with open(path) as fh:
         for line in fh:
             f = line.split()
