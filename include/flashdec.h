@@ -219,6 +219,20 @@ fd_status fd_batch_destroy(fd_batch b);
 fd_status fd_decode_chunk_host(fd_handle h, const float* latent_host, void* pixels_host,
                                void* stream);
 
+/* n consecutive chunks of the stream (Algorithm 1's loop, n times) from / to HOST memory, with
+ * the copies overlapped with the decoding: while chunk t decodes on `stream`, chunk t+1's
+ * latent is copied in and chunk t-1's pixels copied out on a library-owned copy stream (two
+ * device buffers of each, used alternately). latents_host[t]: fp32 [C'][H'][W']
+ * (fd_latent_bytes); pixels_host[t]: fd_pixels_bytes (a one-frame first chunk writes its first
+ * 1/r_t). Pinned host memory for asynchronous copies. Stream-ordered: `stream` continues after
+ * the last chunk's pixels are in host memory; the host buffers must stay valid until then. The
+ * pixels are those of n fd_decode_chunk calls, bit for bit. The copy stream, events and the
+ * second buffers are created on first use (2 * (latent + pixel) bytes of device memory at most).
+ * Errors: FD_ERR_INVALID_ARG (null handle or pointer, n < 0), FD_ERR_STATE (handle in error,
+ * or the chunk counter would pass 2^30), FD_ERR_OOM, FD_ERR_CUDA (the handle is then in error). */
+fd_status fd_decode_sequence_host(fd_handle h, int n, const float* const* latents_host,
+                                  void* const* pixels_host, void* stream);
+
 /* Restart the stream: Algorithm 1's initialisation again for a new latent sequence, t = 0 and
  * the caches logically empty (their memory is not cleared; stale entries are never read
  * because attention at chunk t reads only chunks <= t). Clears the error state.

@@ -423,6 +423,12 @@ struct fd_handle_s {
   // host-buffer decode: library-owned device copies of the latent and the pixels
   float* latent_buf = nullptr;
   void* pixel_buf = nullptr;
+  // fd_decode_sequence_host (created on first use): a copy stream, the second latent / pixel
+  // buffers, and per buffer the events latent in, chunk decoded, pixels out
+  cudaStream_t copy = nullptr;
+  float* latent_buf2 = nullptr;
+  void* pixel_buf2 = nullptr;
+  cudaEvent_t ev_cfork = nullptr, ev_in[2] = {}, ev_done[2] = {}, ev_out[2] = {};
   // tracing: launch count and, while profiling, one event pair per launch
   int64_t launches = 0;
   bool profiling = false;
@@ -1727,6 +1733,80 @@ fd_status fd_decode_chunk_host(fd_handle h, const float* latent_host, void* pixe
   return FD_OK;
 }
 
+// The copy stream, events and second buffers of fd_decode_sequence_host
+static fd_status sequence_setup(fd_handle h) {
+  if (h->copy != nullptr) return FD_OK;
+  if (cudaMalloc(&h->latent_buf2, fd_latent_bytes(&h->cfg)) != cudaSuccess ||
+      cudaMalloc(&h->pixel_buf2, fd_pixels_bytes(&h->cfg)) != cudaSuccess)
+    return FD_ERR_OOM;
+  cudaEvent_t* evs[7] = {&h->ev_cfork, &h->ev_in[0], &h->ev_in[1], &h->ev_done[0],
+                         &h->ev_done[1], &h->ev_out[0], &h->ev_out[1]};
+  for (cudaEvent_t* e : evs)
+    if (cudaEventCreateWithFlags(e, cudaEventDisableTiming) != cudaSuccess) return FD_ERR_CUDA;
+  if (cudaStreamCreateWithFlags(&h->copy, cudaStreamNonBlocking) != cudaSuccess)
+    return FD_ERR_CUDA;
+  return FD_OK;
+}
+
+fd_status fd_decode_sequence_host(fd_handle h, int n, const float* const* latents_host,
+                                  void* const* pixels_host, void* stream) {
+  if (h == nullptr || n < 0 || (n > 0 && (latents_host == nullptr || pixels_host == nullptr)))
+    return FD_ERR_INVALID_ARG;
+  for (int t = 0; t < n; ++t)
+    if (latents_host[t] == nullptr || pixels_host[t] == nullptr) return FD_ERR_INVALID_ARG;
+  if (h->error) return FD_ERR_STATE;
+  if (h->t_host + n >= (1LL << 30)) return FD_ERR_STATE;
+  if (n == 0) return FD_OK;
+  fd_status st = sequence_setup(h);
+  if (st != FD_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaStream_t c = h->copy;
+  if (after_reset(h, s) != FD_OK) return FD_ERR_CUDA;
+  h->last_stream = s;
+  float* lat[2] = {h->latent_buf, h->latent_buf2};
+  void* pix[2] = {h->pixel_buf, h->pixel_buf2};
+  const size_t lb = fd_latent_bytes(&h->cfg);
+  auto fail = [&](fd_status e) {
+    h->error = true;
+    return e;
+  };
+  auto ok = [](cudaError_t e) { return e == cudaSuccess; };
+  // the copies start after the work already on the caller's stream (earlier users of the
+  // buffers); chunk 0's latent goes in first
+  if (!ok(cudaEventRecord(h->ev_cfork, s)) || !ok(cudaStreamWaitEvent(c, h->ev_cfork, 0)) ||
+      !ok(cudaMemcpyAsync(lat[0], latents_host[0], lb, cudaMemcpyHostToDevice, c)) ||
+      !ok(cudaEventRecord(h->ev_in[0], c)))
+    return fail(FD_ERR_CUDA);
+  for (int t = 0; t < n; ++t) {
+    const int b = t & 1, nb = (t + 1) & 1;
+    // the next latent, into the buffer chunk t-1 read, while chunk t decodes; it goes ahead of
+    // chunk t's pixels on the copy stream
+    if (t + 1 < n) {
+      if ((t >= 1 && !ok(cudaStreamWaitEvent(c, h->ev_done[nb], 0))) ||
+          !ok(cudaMemcpyAsync(lat[nb], latents_host[t + 1], lb, cudaMemcpyHostToDevice, c)) ||
+          !ok(cudaEventRecord(h->ev_in[nb], c)))
+        return fail(FD_ERR_CUDA);
+    }
+    // chunk t: its latent is in, and chunk t-2's pixels have left the buffer it writes
+    if (!ok(cudaStreamWaitEvent(s, h->ev_in[b], 0)) ||
+        (t >= 2 && !ok(cudaStreamWaitEvent(s, h->ev_out[b], 0))))
+      return fail(FD_ERR_CUDA);
+    const size_t pb = fd_pixels_bytes(&h->cfg) / (h->d.f1 && h->t_host == 0 ? h->d.rt : 1);
+    if ((st = decode_one(h, lat[b], pix[b], s)) != FD_OK) return fail(st);
+    h->t_host++;
+    // its pixels out on the copy stream once it is decoded
+    if (!ok(cudaEventRecord(h->ev_done[b], s)) || !ok(cudaStreamWaitEvent(c, h->ev_done[b], 0)) ||
+        !ok(cudaMemcpyAsync(pixels_host[t], pix[b], pb, cudaMemcpyDeviceToHost, c)) ||
+        !ok(cudaEventRecord(h->ev_out[b], c)))
+      return fail(FD_ERR_CUDA);
+  }
+  // the caller's stream continues once every chunk's pixels are out
+  if (!ok(cudaStreamWaitEvent(s, h->ev_out[(n - 1) & 1], 0)) ||
+      (n >= 2 && !ok(cudaStreamWaitEvent(s, h->ev_out[n & 1], 0))))
+    return fail(FD_ERR_CUDA);
+  return FD_OK;
+}
+
 fd_status fd_reset(fd_handle h) {
   if (h == nullptr) return FD_ERR_INVALID_ARG;
   if (h->ev_reset == nullptr &&
@@ -1755,6 +1835,15 @@ fd_status fd_destroy(fd_handle h) {
   }
   if (h->ev_fork != nullptr) cudaEventDestroy(h->ev_fork);
   if (h->ev_reset != nullptr) cudaEventDestroy(h->ev_reset);
+  if (h->copy != nullptr) {
+    cudaStreamSynchronize(h->copy);
+    cudaStreamDestroy(h->copy);
+  }
+  for (cudaEvent_t e : {h->ev_cfork, h->ev_in[0], h->ev_in[1], h->ev_done[0], h->ev_done[1],
+                        h->ev_out[0], h->ev_out[1]})
+    if (e != nullptr) cudaEventDestroy(e);
+  cudaFree(h->latent_buf2);
+  cudaFree(h->pixel_buf2);
   if (h->ev_join != nullptr) cudaEventDestroy(h->ev_join);
   for (size_t i = 0; i < h->ev_start.size(); ++i) {
     cudaEventDestroy(h->ev_start[i]);

@@ -66,6 +66,7 @@ _SIGS = {
     "fd_decode_chunks": (_I, [ctypes.POINTER(_P), _I, ctypes.POINTER(_P), ctypes.POINTER(_P),
                               _P]),
     "fd_decode_chunk_host": (_I, [_P, _P, _P, _P]),
+    "fd_decode_sequence_host": (_I, [_P, _I, _P, _P, _P]),
     "fd_batch_create": (_I, [ctypes.POINTER(fd_config), _P, _I, ctypes.POINTER(_P)]),
     "fd_decode_batch": (_I, [_P, ctypes.POINTER(_P), _I, ctypes.POINTER(_P),
                              ctypes.POINTER(_P), _P]),
@@ -290,6 +291,29 @@ class Decoder:
         pp = pixels_host.ctypes.data if isinstance(pixels_host, np.ndarray) else _ptr(pixels_host)
         _check(lib().fd_decode_chunk_host(self.handle, lp, pp, _stream_ptr(stream)),
                "fd_decode_chunk_host")
+
+    def decode_sequence_host(self, latents_host, pixels_host, stream=None) -> None:
+        """Decode len(latents_host) consecutive chunks from / to host buffers (pinned torch
+        tensors or numpy arrays), the copies overlapped with the decoding
+        (fd_decode_sequence_host)."""
+        n = len(latents_host)
+        if len(pixels_host) != n:
+            raise ValueError("one pixel buffer per latent")
+        t0 = self.chunk_index
+        dt = "uint8" if self.cfg.out_dtype == DTYPE_U8 else "float32"
+        lps, pps = [], []
+        for i, (z, p) in enumerate(zip(latents_host, pixels_host)):
+            pix = self._pixels_bytes
+            if self.cfg.first_chunk_frames == 1 and t0 + i == 0:
+                pix //= self.cfg.r_t
+            check_buffer(z, "latent", self._latent_bytes, "float32", False, None)
+            check_buffer(p, "pixels", pix, dt, False, None)
+            lps.append(z.ctypes.data if isinstance(z, np.ndarray) else _ptr(z))
+            pps.append(p.ctypes.data if isinstance(p, np.ndarray) else _ptr(p))
+        ls = (_P * max(n, 1))(*lps)
+        ps = (_P * max(n, 1))(*pps)
+        _check(lib().fd_decode_sequence_host(self.handle, n, ls, ps, _stream_ptr(stream)),
+               "fd_decode_sequence_host")
 
     def reset(self) -> None:
         _check(lib().fd_reset(self.handle), "fd_reset")

@@ -314,6 +314,49 @@ def test_decode_chunk_host_matches_oracle(name):
         assert torch.equal(got[t], dev_out[t]), t
 
 
+@pytest.mark.parametrize("name", ["small", "small_f1", "small_u8"])
+def test_decode_sequence_host_equals_device_decodes(name):
+    """fd_decode_sequence_host (the overlapped host-buffer call the end-to-end benchmark times:
+    chunk t decodes while chunk t+1's latent goes in and chunk t-1's pixels come out on the
+    library's copy stream, two device buffers of each) gives the pixels of fd_decode_chunk bit
+    for bit. The stream goes in two calls (chunks 0..2, then the rest: the second call continues
+    the first's chunk counter and reuses its buffers), then again after fd_reset in one call.
+    The pixel buffers start filled with 7s, so a copy that was missed or came from the wrong
+    buffer shows."""
+    cfg = synth.PRESETS[name]
+    w, z = synth.make_weights(cfg), synth.make_latents(cfg)
+    dev_out = gpu_stream(cfg, w, z)
+    Wt = fdp.Weights(cfg, fdp.pack_blob(cfg, w))
+    dec = fdp.Decoder(cfg, Wt)
+    stream = torch.cuda.Stream()
+    dt = torch.uint8 if cfg.out_u8 else torch.float32
+    lat = [torch.from_numpy(np.ascontiguousarray(z[t])).pin_memory() for t in range(cfg.chunks)]
+
+    def pixels():
+        out = []
+        for t in range(cfg.chunks):
+            frames = 1 if (t == 0 and getattr(cfg, "first_chunk_frames", 0) == 1) else cfg.r_t
+            out.append(torch.full((cfg.out_channels, frames, cfg.out_h, cfg.out_w), 7,
+                                  dtype=dt).pin_memory())
+        return out
+
+    first = pixels()
+    dec.decode_sequence_host(lat[:3], first[:3], stream)
+    dec.decode_sequence_host(lat[3:], first[3:], stream)
+    stream.synchronize()
+    assert dec.sync_status() == fdp.FD_OK and dec.chunk_index == cfg.chunks
+    dec.reset()
+    again = pixels()
+    dec.decode_sequence_host(lat, again, stream)
+    stream.synchronize()
+    assert dec.sync_status() == fdp.FD_OK
+    dec.close()
+    Wt.close()
+    for t in range(cfg.chunks):
+        assert torch.equal(first[t], dev_out[t]), t
+        assert torch.equal(again[t], dev_out[t]), t
+
+
 def test_window_relative_rope_mode():
     """rope_mode = window (the temporal RoPE index counted from the window's first frame, Sec.
     4.3) against the oracle's window-relative decode, which keeps un-rotated keys and re-rotates
