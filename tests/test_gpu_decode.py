@@ -286,8 +286,9 @@ def test_decode_full_token_count_reduced_depth(name):
 
 @pytest.mark.parametrize("name", ["small", "small_f1", "small_u8"])
 def test_decode_chunk_host_matches_oracle(name):
-    """fd_decode_chunk_host (the call the end-to-end benchmark times: pinned host latents in,
-    pinned host pixels out, copies on the stream) against the oracle, chunk by chunk, and bit
+    """fd_decode_chunk_host (pinned host latents in, pinned host pixels out, copies on the
+    stream; the end-to-end benchmark's call for several streams per GPU) against the oracle,
+    chunk by chunk, and bit
     for bit equal to the device-buffer call. small_f1 checks the one-frame first chunk of the
     causal frame count (its copy-back is one frame)."""
     cfg = synth.PRESETS[name]
