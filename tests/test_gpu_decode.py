@@ -288,9 +288,8 @@ def test_decode_full_token_count_reduced_depth(name):
 def test_decode_chunk_host_matches_oracle(name):
     """fd_decode_chunk_host (pinned host latents in, pinned host pixels out, copies on the
     stream; the end-to-end benchmark's call for several streams per GPU) against the oracle,
-    chunk by chunk, and bit
-    for bit equal to the device-buffer call. small_f1 checks the one-frame first chunk of the
-    causal frame count (its copy-back is one frame)."""
+    chunk by chunk, and bit for bit equal to the device-buffer call. small_f1 checks the
+    one-frame first chunk of the causal frame count (its copy-back is one frame)."""
     cfg = synth.PRESETS[name]
     w, z = synth.make_weights(cfg), synth.make_latents(cfg)
     want = oracle.decode_stream(cfg, w, z)
