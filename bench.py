@@ -663,7 +663,7 @@ def cpu_baseline(cfg, w):
 # ---------------------------------------------------------------------------- reference arm
 def run_reference(args):
     """The oracle (there is no reference implementation: the reference is a paper), on the
-    host cores. A steady-state chunk of the 480p stream takes about 21 s there (16 cores), so
+    host cores. A steady-state chunk of the 480p stream takes about 43 s there (16 cores), so
     that W + K steps end within a few minutes each step is a smaller sample of the same
     stream: chunk 0 after a reset (the cache holds that one chunk). The steady-state rate is
     the cpu_baseline of the GPU arm's line."""
