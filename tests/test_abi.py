@@ -119,6 +119,7 @@ def test_status_strings_and_null_arguments():
         assert L.fd_status_str(code)
     assert L.fd_weights_blob_elems(None) == 0
     assert L.fd_decode_chunk(None, None, None, None) == 1
+    assert L.fd_decode_sequence_host(None, 1, None, None, None) == 1
     assert L.fd_reset(None) == 1 and L.fd_destroy(None) == 1
     out = ctypes.c_void_p()
     c = fdp.make_config(synth.PRESETS["tiny"])
