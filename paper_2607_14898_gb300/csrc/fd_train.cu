@@ -130,7 +130,6 @@ __global__ void rmsnorm_bwd_kernel(const float* __restrict__ x, const float* __r
   }
 }
 
-// out[c] = sum over rows of x[r][c], rows in order (deterministic)
 // Gated MLP (the XL layout, reading R7): layer 1's output z [M][2 Dm] holds, on the device,
 // the gate and up columns of 32 hidden units side by side in blocks of 64 (gate unit 32 j + i
 // at column 64 j + i, its up column at 64 j + 32 + i); a = SiLU(gate) up, in unit order.
@@ -182,6 +181,7 @@ __global__ void gated_rows_kernel(const float* __restrict__ src, int rows, int l
   }
 }
 
+// out[c] = sum over rows of x[r][c], rows in order (deterministic)
 __global__ void colsum_kernel(const float* __restrict__ x, long long rows, int cols, int ld,
                               float* __restrict__ out) {
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
